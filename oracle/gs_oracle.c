@@ -1,0 +1,333 @@
+/*
+ * gs_oracle.c -- plain, slow, single-threaded CPU oracle for gradient
+ * sparsification (Wangni, Wang, Liu, Zhang, "Gradient Sparsification for
+ * Communication-Efficient Distributed Optimization", arXiv:1710.09854).
+ *
+ * TEST INFRASTRUCTURE ONLY.  Nothing on the product path may link, load or
+ * call this file: only tests/, __graft_entry__.smoke() and bench.py's
+ * cpu_baseline / reference leg use it.  It shares no code, header, table or
+ * constant with the CUDA library; the two are compared, never combined.
+ *
+ * Everything is fp64 (the paper fixes no precision), evaluated in the order
+ * the paper states it, with no blocking, fusion or reordering:
+ *
+ *   Section 3      Q(g)_i = Z_i g_i / p_i with Z_i ~ Bernoulli(p_i).
+ *   Proposition 1  p_i = min(lambda |g_i|, 1).
+ *   Algorithm 3    greedy rescaling of the active set {i : p_i != 1} until
+ *                  the scaling factor c drops to <= 1 (or `iters` rescalings
+ *                  have been made).
+ *   Algorithm 1    step 6: the M sparse vectors are summed (the 1/M of the
+ *                  average is left to the caller).
+ *
+ * Readings where the paper is silent (each is listed in the design doc):
+ *   - `iters` is the maximum number of rescalings (Algorithm 3, steps 4-10);
+ *     iters = 0 returns p^0.  Section 5 runs two.
+ *   - A coordinate is active iff fl64(lambda |g_i|) < 1 (step 5 "p_i != 1").
+ *   - g_i = 0 gives p_i = 0; such coordinates are never kept.
+ *   - If the active mass sum_{i in I} p_i is 0 the loop stops.
+ *   - If sum |g_i| = 0, lambda = 0 and nothing is kept.
+ *   - The Bernoulli draw uses Philox4x32-10 (Salmon et al., SC'11), key =
+ *     (seed lo, seed hi), counter = (q lo, q hi, worker, step) with q = i/4,
+ *     word i mod 4; u_i = word * 2^-32 and Z_i = [u_i < p_i].
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define GSO_OK 0
+#define GSO_INVALID 1
+#define GSO_NONFINITE 4
+#define GSO_INTERNAL 6
+
+#if defined(__GNUC__)
+#define GSO_EXPORT __attribute__((visibility("default")))
+#else
+#define GSO_EXPORT
+#endif
+
+/* ------------------------------------------------------------------------
+ * Philox4x32-10 (Salmon, Moraes, Dror, Shaw, "Parallel Random Numbers: As
+ * Easy as 1, 2, 3", SC'11).  One round maps the counter (X0, X1, X2, X3)
+ * under key (K0, K1) to
+ *     (hi(M1*X2) ^ X1 ^ K0,  lo(M1*X2),  hi(M0*X0) ^ X3 ^ K1,  lo(M0*X0))
+ * with the published multipliers M0 = 0xD2511F53, M1 = 0xCD9E8D57; between
+ * rounds the key is bumped by the Weyl constants (0x9E3779B9, 0xBB67AE85).
+ * Ten rounds.
+ * ---------------------------------------------------------------------- */
+GSO_EXPORT void gso_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t out[4])
+{
+    uint32_t x0 = ctr[0], x1 = ctr[1], x2 = ctr[2], x3 = ctr[3];
+    uint32_t k0 = key[0], k1 = key[1];
+    int r;
+    for (r = 0; r < 10; r++) {
+        uint64_t prod0 = (uint64_t)0xD2511F53u * (uint64_t)x0;
+        uint64_t prod1 = (uint64_t)0xCD9E8D57u * (uint64_t)x2;
+        uint32_t hi0 = (uint32_t)(prod0 >> 32), lo0 = (uint32_t)prod0;
+        uint32_t hi1 = (uint32_t)(prod1 >> 32), lo1 = (uint32_t)prod1;
+        uint32_t y0 = hi1 ^ x1 ^ k0;
+        uint32_t y1 = lo1;
+        uint32_t y2 = hi0 ^ x3 ^ k1;
+        uint32_t y3 = lo0;
+        x0 = y0; x1 = y1; x2 = y2; x3 = y3;
+        k0 += 0x9E3779B9u;
+        k1 += 0xBB67AE85u;
+    }
+    out[0] = x0; out[1] = x1; out[2] = x2; out[3] = x3;
+}
+
+/* The 32-bit random word that decides coordinate i of worker `worker` at
+ * training step `step`. */
+GSO_EXPORT uint32_t gso_word(uint64_t seed, uint32_t step, uint32_t worker, int64_t i)
+{
+    uint64_t q = (uint64_t)i / 4u;
+    uint32_t ctr[4], key[2], out[4];
+    ctr[0] = (uint32_t)(q & 0xFFFFFFFFu);
+    ctr[1] = (uint32_t)(q >> 32);
+    ctr[2] = worker;
+    ctr[3] = step;
+    key[0] = (uint32_t)(seed & 0xFFFFFFFFu);
+    key[1] = (uint32_t)(seed >> 32);
+    gso_philox4x32_10(ctr, key, out);
+    return out[(uint64_t)i % 4u];
+}
+
+/* u_i in [0, 1): the word scaled by 2^-32 (exact in fp64). */
+GSO_EXPORT double gso_uniform(uint64_t seed, uint32_t step, uint32_t worker, int64_t i)
+{
+    return (double)gso_word(seed, step, worker, i) * 0x1p-32;
+}
+
+/* Fill u[0..n) with the uniforms of coordinates i0 .. i0+n-1. */
+GSO_EXPORT void gso_uniforms(uint64_t seed, uint32_t step, uint32_t worker, int64_t i0, int64_t n, double* u)
+{
+    int64_t k;
+    for (k = 0; k < n; k++) u[k] = gso_uniform(seed, step, worker, i0 + k);
+}
+
+/* Result of the greedy solve. */
+typedef struct {
+    double lambda;     /* final lambda */
+    int64_t capped;    /* #{i : p_i = 1} at the final lambda */
+    int32_t iters_run; /* rescalings performed */
+    int32_t pad;
+    double sum_p;      /* sum_i p_i at the final lambda */
+    double l1;         /* sum_i |g_i| */
+} gso_info;
+
+static int check_args(int64_t d, double kappa, int iters)
+{
+    if (d < 1) return GSO_INVALID;
+    if (!(kappa > 0.0) || kappa > 1.0) return GSO_INVALID;
+    if (iters < 0) return GSO_INVALID;
+    return GSO_OK;
+}
+
+/* ------------------------------------------------------------------------
+ * Algorithm 3 in the lambda form of Proposition 1.
+ *
+ * Step 3 sets p^0_i = min(rho d |g_i| / sum|g|, 1), i.e. lambda_0 = rho d / S.
+ * At iteration j the active set is I = {i : lambda_j |g_i| < 1}; with
+ * K = d - |I| capped coordinates and A = sum_{i in I} p_i^j the scaling
+ * variable of step 6 is c = (rho d - d + |I|) / A = (rho d - K) / A.  Step 7
+ * stops when c <= 1; otherwise step 8 rescales the active p by c, which is
+ * lambda_{j+1} = c lambda_j (capped entries stay at 1 because c > 1).
+ * ---------------------------------------------------------------------- */
+GSO_EXPORT int gso_greedy_lambda(const float* g, int64_t d, double kappa, int iters, gso_info* info)
+{
+    int rc = check_args(d, kappa, iters);
+    double S = 0.0, budget, lambda, A;
+    int64_t i, K;
+    int32_t j;
+    if (rc != GSO_OK) return rc;
+
+    for (i = 0; i < d; i++) S += fabs((double)g[i]);
+    if (!isfinite(S)) return GSO_NONFINITE;
+
+    memset(info, 0, sizeof(*info));
+    info->l1 = S;
+    if (S == 0.0) return GSO_OK; /* nothing to keep: lambda = 0 */
+
+    budget = kappa * (double)d;
+    lambda = budget / S; /* step 3 */
+    j = 0;
+    while (j < iters) {  /* steps 4-10 */
+        K = 0;
+        A = 0.0;
+        for (i = 0; i < d; i++) {
+            double x = lambda * fabs((double)g[i]);
+            if (x >= 1.0) K++;     /* p_i = 1: outside the active set */
+            else A += x;           /* p_i^j for i in I */
+        }
+        if (A == 0.0) break;       /* no active mass left */
+        {
+            double c = (budget - (double)K) / A; /* step 6 */
+            if (c <= 1.0) break;                 /* step 7 */
+            lambda = c * lambda;                 /* step 8 */
+        }
+        j++;                                     /* step 9 */
+    }
+
+    K = 0;
+    A = 0.0;
+    for (i = 0; i < d; i++) {
+        double x = lambda * fabs((double)g[i]);
+        if (x >= 1.0) K++;
+        else A += x;
+    }
+    info->lambda = lambda;
+    info->capped = K;
+    info->iters_run = j;
+    info->sum_p = (double)K + A;
+    return GSO_OK;
+}
+
+/* ------------------------------------------------------------------------
+ * Algorithm 3 exactly as printed: it carries the probability vector itself.
+ * Step 3 computes p^0_i = min(rho d |g_i| / sum|g|, 1); each pass forms the
+ * active set, the scaling variable c, stops on c <= 1, and replaces the
+ * active entries by min(c p_i, 1).  Used to check the lambda form above.
+ * ---------------------------------------------------------------------- */
+GSO_EXPORT int gso_greedy_pvector(const float* g, int64_t d, double kappa, int iters, double* p, int32_t* iters_run)
+{
+    int rc = check_args(d, kappa, iters);
+    double S = 0.0, rd;
+    int64_t i;
+    int32_t j = 0;
+    if (rc != GSO_OK) return rc;
+
+    for (i = 0; i < d; i++) S += fabs((double)g[i]);
+    if (!isfinite(S)) return GSO_NONFINITE;
+    if (S == 0.0) {
+        for (i = 0; i < d; i++) p[i] = 0.0;
+        *iters_run = 0;
+        return GSO_OK;
+    }
+    rd = kappa * (double)d;
+    for (i = 0; i < d; i++) {
+        double t = rd * fabs((double)g[i]) / S;
+        p[i] = t < 1.0 ? t : 1.0;
+    }
+    while (j < iters) {
+        int64_t nI = 0;
+        double sumI = 0.0, c;
+        for (i = 0; i < d; i++) {
+            if (p[i] != 1.0) { nI++; sumI += p[i]; }
+        }
+        if (sumI == 0.0) break;
+        c = (rd - (double)d + (double)nI) / sumI;
+        if (c <= 1.0) break;
+        for (i = 0; i < d; i++) {
+            if (p[i] != 1.0) {
+                double t = c * p[i];
+                p[i] = t < 1.0 ? t : 1.0;
+            }
+        }
+        j++;
+    }
+    *iters_run = j;
+    return GSO_OK;
+}
+
+/* p_i = min(lambda |g_i|, 1) (Proposition 1) with lambda from Algorithm 3. */
+GSO_EXPORT int gso_probabilities(const float* g, int64_t d, double kappa, int iters, double* p, gso_info* info)
+{
+    int64_t i;
+    int rc = gso_greedy_lambda(g, d, kappa, iters, info);
+    if (rc != GSO_OK) return rc;
+    for (i = 0; i < d; i++) {
+        double x = info->lambda * fabs((double)g[i]);
+        p[i] = x < 1.0 ? x : 1.0;
+    }
+    return GSO_OK;
+}
+
+/* ------------------------------------------------------------------------
+ * Section 3: draw Z_i ~ Bernoulli(p_i), amplify kept entries to g_i / p_i,
+ * and write them as (index, value) pairs in ascending index order (the plain
+ * coding of the non-zero coordinates of Q(g), section 3.3).
+ *
+ * `i0` offsets both the Philox counter and the written index: coordinate k
+ * of this vector is coordinate i0 + k of the worker's full vector (used for
+ * layer-wise sparsification, where each layer is solved on its own but the
+ * random stream follows the worker's flat index).
+ * idx / val must hold d entries.
+ * ---------------------------------------------------------------------- */
+GSO_EXPORT int gso_sparsify(const float* g, int64_t d, double kappa, int iters, uint64_t seed, uint32_t step,
+                            uint32_t worker, int64_t i0, int32_t* idx, float* val, int64_t* nnz, gso_info* info)
+{
+    int64_t i, n = 0;
+    int rc = gso_greedy_lambda(g, d, kappa, iters, info);
+    *nnz = 0;
+    if (rc != GSO_OK) return rc;
+    for (i = 0; i < d; i++) {
+        double gi = (double)g[i];
+        double x = info->lambda * fabs(gi);
+        double p = x < 1.0 ? x : 1.0;
+        double u;
+        if (p == 0.0) continue; /* g_i = 0 is never kept */
+        u = gso_uniform(seed, step, worker, i0 + i);
+        if (u < p) {
+            idx[n] = (int32_t)(i0 + i);
+            val[n] = (float)(gi / p);
+            n++;
+        }
+    }
+    *nnz = n;
+    return GSO_OK;
+}
+
+/* Layer-wise sparsification (section 5.2): each segment [off[l], off[l+1])
+ * of the worker's vector gets its own Algorithm 3 with budget kappa * d_l.
+ * The per-segment results are concatenated in index order; lambdas[l] (if
+ * not NULL) receives each segment's lambda. */
+GSO_EXPORT int gso_segmented_sparsify(const float* g, const int64_t* off, int L, double kappa, int iters, uint64_t seed,
+                                      uint32_t step, uint32_t worker, int32_t* idx, float* val, int64_t* nnz,
+                                      double* lambdas)
+{
+    int l;
+    int64_t total = 0;
+    *nnz = 0;
+    if (L < 1 || off[0] != 0) return GSO_INVALID;
+    for (l = 0; l < L; l++) {
+        int64_t n = 0;
+        gso_info info;
+        int rc;
+        if (off[l + 1] <= off[l]) return GSO_INVALID;
+        rc = gso_sparsify(g + off[l], off[l + 1] - off[l], kappa, iters, seed, step, worker, off[l], idx + total,
+                          val + total, &n, &info);
+        if (rc != GSO_OK) return rc;
+        if (lambdas) lambdas[l] = info.lambda;
+        total += n;
+    }
+    *nnz = total;
+    return GSO_OK;
+}
+
+/* ------------------------------------------------------------------------
+ * Algorithm 1, step 6, as a sum: out_i = sum_{m=0}^{M-1} Q(g^m)_i, added in
+ * fp32 in worker order m = 0, 1, ... .  Each worker's sparse vector is first
+ * written out densely, then added to the running fp32 sum.
+ * ---------------------------------------------------------------------- */
+GSO_EXPORT int gso_aggregate(const int32_t* const* idx, const float* const* val, const int64_t* nnz, int M, int64_t d,
+                             float* out)
+{
+    int m;
+    int64_t i, e;
+    float* dense;
+    if (M < 1 || d < 1) return GSO_INVALID;
+    dense = (float*)malloc((size_t)d * sizeof(float));
+    if (!dense) return GSO_INTERNAL;
+    for (i = 0; i < d; i++) out[i] = 0.0f;
+    for (m = 0; m < M; m++) {
+        for (i = 0; i < d; i++) dense[i] = 0.0f;
+        for (e = 0; e < nnz[m]; e++) {
+            int64_t k = idx[m][e];
+            if (k < 0 || k >= d) { free(dense); return GSO_INVALID; }
+            dense[k] = val[m][e];
+        }
+        for (i = 0; i < d; i++) out[i] = out[i] + dense[i];
+    }
+    free(dense);
+    return GSO_OK;
+}
