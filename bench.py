@@ -1,0 +1,472 @@
+"""Benchmark of the GB300 gradient-sparsification path.
+
+One step = gs_batched_sparsify over M worker gradients + gs_sparse_aggregate
+of the M sparse vectors (steps (1)-(6) of the path), on inputs resident in
+HBM.  Default workload: M = 16 workers, d = 2^24 fp32, Student-t(3)
+gradients with 1% zeros, kappa = 0.01, 3 greedy iterations.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gs|reference]
+                  [--workload c1..c5] [--kappa K] [--dtype f32|bf16]
+
+Under torchrun (N > 1) every rank runs its own replica of the workload on
+its own GPU (weak scaling; the path has no cross-replica exchange) and rank 0
+prints one JSON line with the whole-job throughput.  `--impl reference`
+times the CPU oracle (the single-threaded C restatement of the paper) on a
+bounded sample of the same workload, on the host cores.
+"""
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import workloads  # noqa: E402
+
+METRIC = "sparsified coords/s and achieved HBM GB/s vs peak (d=2^24, M=16 workers)"
+UNIT = "coords/s"
+L2_BYTES = 129 * 1024 * 1024
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, "fallback"
+
+
+# ---------------------------------------------------------------------------
+# Distributed plumbing (one process per GPU; replicas only)
+# ---------------------------------------------------------------------------
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def init_dist(backend):
+    import torch.distributed as dist
+    ws, rank, _ = dist_env()
+    if ws > 1 and not dist.is_initialized():
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group(backend=backend, rank=rank, world_size=ws)
+    return ws, rank
+
+
+def barrier():
+    import torch.distributed as dist
+    if dist.is_available() and dist.is_initialized():
+        dist.barrier()
+
+
+def max_over_ranks(x, device=None):
+    """Largest value of x over all ranks (x itself without a process group)."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()):
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(x, device=None):
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()):
+        return float(x)
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+def job_throughput(units_per_rank, ms_max, n_ranks):
+    """Whole-job units/s: all ranks' units over the slowest rank's time."""
+    return units_per_rank * n_ranks / (ms_max / 1e3)
+
+
+# ---------------------------------------------------------------------------
+# Workload construction
+# ---------------------------------------------------------------------------
+def make_workload(name, kappa=None, dtype=None, rank=0):
+    import torch
+    w = {"c1": workloads.C1, "c2": workloads.C2, "c3": workloads.C3, "c4": workloads.C4, "c5": workloads.C5}[name]
+    kappa = w.kappa if kappa is None else kappa
+    dtype = dtype or w.dtype
+    off = None
+    if name == "c1":
+        g = workloads.device_c1(w.d, seed=w.data_seed + 1000 * rank)
+    elif name == "c2":
+        g = workloads.device_logreg(w.M, w.d, seed0=w.data_seed + 1000 * rank)
+    elif name == "c3":
+        g = workloads.device_student_t(w.M, w.d, seed0=w.data_seed + 1000 * rank)
+    elif name == "c4":
+        g, off = workloads.device_layerwise(w.M, seed0=w.data_seed + 1000 * rank)
+    else:
+        g = workloads.device_lognormal(w.M, w.d, seed0=w.data_seed + 1000 * rank)
+    if dtype == "bf16":
+        g = g.to(torch.bfloat16)
+    torch.cuda.synchronize()
+    return w, g, off, kappa, dtype
+
+
+def algorithmic_bytes(M, d, esz, nnz_total):
+    """Bytes the path must move at least (one read of g, the (idx, val) codes
+    written and read back, the dense sum written)."""
+    sparsify = M * d * esz + nnz_total * 8
+    aggregate = nnz_total * 8 + d * 4
+    return sparsify, aggregate
+
+
+# ---------------------------------------------------------------------------
+# Clock sampling during the timed region
+# ---------------------------------------------------------------------------
+class Clocks:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            os.makedirs(os.path.join(ROOT, "gpurun_out"), exist_ok=True)
+            self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{self.gpu}.csv")
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.fh, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.15)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.fh.close()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower() == "active":
+                        reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# ---------------------------------------------------------------------------
+# The GPU arm
+# ---------------------------------------------------------------------------
+def run_gpu(args):
+    import torch
+    ws, rank = init_dist("nccl")
+    _, _, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    import paper_1710_09854_gb300 as gs
+    gs.lib()
+
+    w, g, off, kappa, dtype = make_workload(args.workload, args.kappa, args.dtype, rank)
+    M, d = g.shape
+    esz = g.element_size()
+    cap = d
+    idx = torch.empty((M, cap), dtype=torch.int32, device=dev)
+    val = torch.empty((M, cap), dtype=torch.float32, device=dev)
+    nnz = torch.empty(M, dtype=torch.int32, device=dev)
+    out = torch.empty(d, dtype=torch.float32, device=dev)
+    idx_rows = [idx[m] for m in range(M)]
+    val_rows = [val[m] for m in range(M)]
+    stream = torch.cuda.current_stream(dev)
+
+    def step(t):
+        if off is None:
+            gs.gs_batched_sparsify(g, kappa, w.iters, w.seed, t, 0, idx, val, nnz, stream=stream)
+        else:
+            gs.gs_segmented_sparsify(g, off, kappa, w.iters, w.seed, t, 0, idx, val, nnz, stream=stream)
+        gs.gs_sparse_aggregate(idx_rows, val_rows, nnz, d, out, stream=stream)
+
+    for t in range(args.warmup):
+        step(t)
+    torch.cuda.synchronize()
+    rc = gs.gs_sync_status(stream)
+    if rc != gs.GS_OK:
+        raise RuntimeError(f"device status after warm-up: {gs.status_string(rc)}")
+    nnz_total = int(nnz.sum().item())
+
+    # ---- timed region: exactly K steps, barrier + synchronize on both sides
+    gs.gs_set_option(gs.GS_OPT_KERNEL_TIMING, 1)
+    gs.gs_kernel_times()  # reset counters
+    clocks = Clocks(local)
+    clocks.start()
+    barrier()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for t in range(args.steps):
+        step(args.warmup + t)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    clk = clocks.stop()
+    ktimes = gs.gs_kernel_times()
+    gs.gs_set_option(gs.GS_OPT_KERNEL_TIMING, 0)
+    ms_local = e0.elapsed_time(e1) / args.steps
+    ms = max_over_ranks(ms_local, dev)
+    rc = gs.gs_sync_status(stream)
+    if rc != gs.GS_OK:
+        raise RuntimeError(f"device status after timing: {gs.status_string(rc)}")
+
+    coords = M * d
+    value = job_throughput(coords, ms, ws)
+    b_sp, b_ag = algorithmic_bytes(M, d, esz, nnz_total)
+    hbm, peak_kind = peaks()
+    launches = int(sum(n for _, n in ktimes.values()))
+    dom = max(ktimes.items(), key=lambda kv: kv[1][0])
+    dom_name, (dom_ms, dom_n) = dom
+    per_launch_ms = dom_ms / max(dom_n, 1)
+    # Algorithmic bytes of the dominant kernel per launch.
+    kernel_bytes = {
+        "k_stream": M * d * esz,                 # one read of g
+        "k_write": nnz_total * 8,                # the (idx, val) codes written
+        "k_tiles": nnz_total * 8 + d * 4,        # codes read, dense sum written
+        "k_count": 0,
+    }
+    kb = kernel_bytes.get(dom_name, 0)
+    achieved = kb / (per_launch_ms / 1e3) / 1e9 if kb else 0.0
+    traffic = load_traffic(dom_name, args.workload, dtype, kappa)
+    roofline = {"kernel": dom_name, "bound": "hbm", "achieved": round(achieved, 1), "peak": hbm,
+                "peak_kind": peak_kind, "unit": "GB/s", "frac": round(achieved / hbm, 4),
+                "traffic": traffic, "algorithmic_bytes_per_launch": kb,
+                "ms_per_launch": round(per_launch_ms, 4)}
+    pipe_gbs = (b_sp + b_ag) / (ms / 1e3) / 1e9
+    kernels = {k: {"ms_per_step": round(v[0] / args.steps, 4), "launches": v[1]} for k, v in ktimes.items() if v[1]}
+
+    # ---- end to end through the host-buffer entry point
+    e2e = None
+    if not args.no_e2e and off is None:
+        e2e = run_e2e(gs, g, kappa, w, args, dev, stream, ws)
+
+    result = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": dtype, "data": "synthetic",
+        "config": {"workload": w.name, "M": M, "d": d, "kappa": kappa, "iters": w.iters, "dtype": dtype,
+                   "parallelism": f"replicas{ws}", "l2": "inputs exceed L2 (%.2f GB of g per step)" % (M * d * esz / 1e9)},
+        "hbm_gbs_pipeline": round(pipe_gbs, 1),
+        "pipeline_roofline": {"bound": "hbm", "algorithmic_bytes": b_sp + b_ag, "achieved": round(pipe_gbs, 1),
+                              "peak": hbm, "frac": round(pipe_gbs / hbm, 4), "unit": "GB/s"},
+        "roofline": roofline,
+        "kernels": kernels,
+        "nnz_per_step": nnz_total,
+        "gpu_launches": launches,
+        "clocks": clk,
+        "e2e": e2e,
+    }
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_baseline_sample(g, off, kappa, w, budget_s=args.cpu_seconds)
+    return result, rank
+
+
+def run_e2e(gs, g, kappa, w, args, dev, stream, ws):
+    import torch
+    M, d = g.shape
+    gh = g.cpu().pin_memory()
+    g_dev = torch.empty_like(g)
+    idx = torch.empty((M, d), dtype=torch.int32, device=dev)
+    val = torch.empty((M, d), dtype=torch.float32, device=dev)
+    nnz = torch.empty(M, dtype=torch.int32, device=dev)
+    out = torch.empty(d, dtype=torch.float32, device=dev)
+    out_h = torch.empty(d, dtype=torch.float32).pin_memory()
+    nnz_h = torch.empty(M, dtype=torch.int32).pin_memory()
+    n = max(3, min(args.steps, args.e2e_steps))
+    for t in range(2):
+        gs.gs_pipeline_host(gh, kappa, w.iters, w.seed, t, 0, g_dev, idx, val, nnz, out, out_h, nnz_h, stream=stream)
+    torch.cuda.synchronize()
+    barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for t in range(n):
+        gs.gs_pipeline_host(gh, kappa, w.iters, w.seed, t, 0, g_dev, idx, val, nnz, out, out_h, nnz_h, stream=stream)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = max_over_ranks(e0.elapsed_time(e1) / n, dev)
+    rc = gs.gs_sync_status(stream)
+    if rc != gs.GS_OK:
+        raise RuntimeError(f"device status after e2e: {gs.status_string(rc)}")
+    return {"value": job_throughput(M * d, ms, ws), "unit": UNIT, "ms_per_step": ms,
+            "h2d_bytes_per_step": M * d * g.element_size(), "d2h_bytes_per_step": d * 4 + M * 4,
+            "api": "gs_pipeline_host", "host_memory": "pinned"}
+
+
+def load_traffic(kernel, workload, dtype, kappa):
+    """DRAM bytes per launch of `kernel` from the committed ncu summary, if it
+    was taken on the current kernel build (profiles/traffic.json)."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    try:
+        with open(path) as f:
+            t = json.load(f)
+    except (OSError, ValueError):
+        return None
+    key = f"{kernel}:{workload}:{dtype}:{kappa}"
+    ent = t.get(key)
+    if not ent:
+        return None
+    try:
+        src = os.path.join(ROOT, "paper_1710_09854_gb300", "csrc")
+        import hashlib
+        h = hashlib.sha256()
+        for fn in sorted(os.listdir(src)):
+            with open(os.path.join(src, fn), "rb") as f:
+                h.update(f.read())
+        if ent.get("csrc_sha256") != h.hexdigest():
+            return None
+    except OSError:
+        return None
+    return ent.get("bytes_per_launch")
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (reported baseline and the reference arm)
+# ---------------------------------------------------------------------------
+def oracle_step(g_rows, off, kappa, iters, seed, step):
+    import oracle
+    il, vl = [], []
+    for m, row in enumerate(g_rows):
+        if off is None:
+            i, v, _ = oracle.sparsify(row, kappa, iters, seed, step, m)
+        else:
+            i, v, _ = oracle.segmented_sparsify(row, off, kappa, iters, seed, step, m)
+        il.append(i)
+        vl.append(v)
+    oracle.aggregate(il, vl, g_rows[0].size)
+
+
+def cpu_baseline_sample(g, off, kappa, w, budget_s=15.0):
+    """The oracle as it stands, single-threaded, on whole workers of the same
+    workload until about `budget_s` seconds of CPU work have run."""
+    import oracle
+    oracle.lib()
+    M, d = g.shape
+    rows = []
+    t0 = time.perf_counter()
+    done = 0
+    for m in range(M):
+        row = g[m].float().cpu().numpy()
+        rows.append(row)
+        s = time.perf_counter()
+        oracle_step([row], off, kappa, w.iters, w.seed, 0)
+        done += d
+        if time.perf_counter() - t0 > budget_s:
+            break
+    el = time.perf_counter() - t0
+    return {"value": done / el, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{done // d} of {M} workers at full d={d} (sparsify + sparse sum), {el:.1f} s"}
+
+
+def run_reference(args):
+    """Reference arm: the CPU oracle, timed on the host cores, each step a
+    bounded slice of the workload sized so the whole run takes minutes."""
+    ws, rank, _ = dist_env()
+    if ws > 1:
+        import torch.distributed as dist
+        init_dist("gloo")
+        if rank != 0:
+            dist.barrier()
+            return None, rank
+    import oracle
+    oracle.lib()
+    w = {"c1": workloads.C1, "c2": workloads.C2, "c3": workloads.C3, "c4": workloads.C4, "c5": workloads.C5}[
+        args.workload]
+    kappa = w.kappa if args.kappa is None else args.kappa
+    # Host copy of the same distribution (numpy generator), one worker at a time.
+    if args.workload in ("c3",):
+        full = workloads.gen_student_t(1, min(w.d, 1 << 22), seed0=w.data_seed)[0]
+    elif args.workload == "c5":
+        full = workloads.gen_c5(1, min(w.d, 1 << 22))[0]
+    else:
+        full = workloads.gen_c1(min(w.d, 1 << 20))
+    # Calibrate: coordinates per step so that (K + W) steps take ~150 s.
+    probe = full[: 1 << 16]
+    t = time.perf_counter()
+    oracle_step([probe], None, kappa, w.iters, w.seed, 0)
+    rate = probe.size / (time.perf_counter() - t)
+    per_step_s = min(10.0, 150.0 / max(1, args.steps + args.warmup))
+    n = int(min(full.size, max(1024, rate * per_step_s)))
+    sl = full[:n]
+    for t in range(args.warmup):
+        oracle_step([sl], None, kappa, w.iters, w.seed, t)
+    t0 = time.perf_counter()
+    for t in range(args.steps):
+        oracle_step([sl], None, kappa, w.iters, w.seed, args.warmup + t)
+    el = time.perf_counter() - t0
+    ms = el / args.steps * 1e3
+    value = n / (ms / 1e3)
+    sample = f"one worker slice of {n} coordinates per step (sparsify + sparse sum), single thread"
+    res = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "config": {"workload": w.name, "M": w.M, "d": w.d, "kappa": kappa, "iters": w.iters},
+           "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+           "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    if ws > 1:
+        import torch.distributed as dist
+        dist.barrier()
+    return res, rank
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="gs", choices=["gs", "reference"])
+    ap.add_argument("--workload", default="c3", choices=["c1", "c2", "c3", "c4", "c5"])
+    ap.add_argument("--kappa", type=float, default=None)
+    ap.add_argument("--dtype", default=None, choices=[None, "f32", "bf16"])
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=20)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        res, rank = run_reference(args)
+    else:
+        res, rank = run_gpu(args)
+    if rank == 0 and res is not None:
+        print(json.dumps(res), flush=True)
+    import torch.distributed as dist
+    if dist.is_available() and dist.is_initialized():
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

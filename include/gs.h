@@ -1,0 +1,199 @@
+/*
+ * gs.h -- C ABI of the GB300 gradient-sparsification library (libgs.so).
+ *
+ * The library computes, on one GPU, the data-parallel hot path of the
+ * gradient sparsification of Wangni, Wang, Liu and Zhang (arXiv:1710.09854):
+ * for each of M simulated workers with a dense gradient g (length d)
+ *   (1) the l1 sums of g (section 3.2, Algorithm 3, step 3),
+ *   (2) keep probabilities p_i = min(lambda |g_i|, 1) (Proposition 1) with
+ *       lambda from the greedy rescaling of Algorithm 3,
+ *   (3) one Bernoulli(p_i) draw per coordinate (section 3),
+ *   (4) amplification of kept entries to g_i / p_i (section 3),
+ *   (5) compaction of the kept entries to (int32 index, fp32 value) pairs
+ *       (the plain coding of section 3.3),
+ * and (6) the sum of the M sparse vectors into a dense fp32 vector
+ * (Algorithm 1, step 6, as a sum: the caller applies the 1/M).
+ *
+ * Conventions shared by every entry point:
+ *  - Array arguments are DEVICE pointers unless a parameter says "host".
+ *    The caller owns all of them; the library never frees caller memory.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *    stream).  Every call is asynchronous with respect to the host and
+ *    ordered on `stream`.
+ *  - Argument errors found on the host are returned at once and nothing is
+ *    enqueued.  Errors that only the GPU can see (non-finite gradients,
+ *    output capacity, malformed sparse input, a bounded wait that ran out)
+ *    are recorded in a per-device status word; gs_sync_status() waits for
+ *    the stream and returns (and clears) them.
+ *  - Scratch memory is taken stream-ordered from a memory pool owned by the
+ *    library (cudaMallocAsync / cudaFreeAsync on `stream`).
+ *  - The random draw of coordinate i of worker w at step t is word i mod 4
+ *    of Philox4x32-10 (Salmon et al., SC'11) with key = (seed lo, seed hi)
+ *    and counter = (q lo, q hi, w, t), q = i / 4; u_i = word * 2^-32 and
+ *    coordinate i is kept iff u_i < p_i.  Results are therefore a pure
+ *    function of (g, kappa, iters, seed, step, worker) and bit-identical
+ *    across runs and launch configurations.
+ *  - kappa is the density budget (the paper's rho, Algorithm 3): the
+ *    expected number of kept coordinates is at most kappa * d.  It must lie
+ *    in (0, 1].  iters >= 0 is the maximum number of rescalings of
+ *    Algorithm 3 (the paper's experiments use 2, section 5).
+ */
+#ifndef GS_H
+#define GS_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    GS_OK = 0,
+    GS_ERR_INVALID_ARG = 1, /* bad argument (host) or malformed sparse input (device) */
+    GS_ERR_CUDA = 2,        /* a CUDA runtime call failed */
+    GS_ERR_CAPACITY = 3,    /* more kept entries than the output capacity */
+    GS_ERR_NONFINITE = 4,   /* a gradient contains NaN or Inf */
+    GS_ERR_TIMEOUT = 5,     /* a bounded device-side wait ran out */
+    GS_ERR_INTERNAL = 6     /* library invariant violated */
+} gs_status;
+
+typedef enum { GS_DTYPE_F32 = 0, GS_DTYPE_BF16 = 1 } gs_dtype;
+
+/* Per-worker (per-segment for layer-wise calls) record of the greedy solve,
+ * written to device memory by the calls that take a `gs_info*`. */
+typedef struct {
+    double lambda;      /* final lambda of Proposition 1 */
+    double sum_p;       /* sum_i p_i at the final lambda (<= kappa d, Algorithm 3) */
+    int64_t capped;     /* #{i : p_i = 1} at the final lambda */
+    int32_t iters_run;  /* rescalings performed (<= iters) */
+    int32_t flags;      /* bit 0: the exact fallback solve was used */
+} gs_info;
+
+/* Human-readable name of a status code.  Never NULL. */
+const char* gs_status_string(int status);
+
+/* Library version as 10000*major + 100*minor + patch. */
+int gs_version(void);
+
+/* Wait for `stream`, then return the first device-side error recorded since
+ * the last call to gs_sync_status (GS_OK if none) and clear the record. */
+gs_status gs_sync_status(void* stream);
+
+/*
+ * Keep probabilities of one gradient (Proposition 1 with lambda from
+ * Algorithm 3):  p[i] = min(lambda |g[i]|, 1), rounded to fp32.
+ *   g     device, d fp32 values (read only)
+ *   d     length, 1 <= d < 2^31
+ *   p     device, d fp32 values (written)
+ */
+gs_status gs_probabilities(const float* g, int64_t d, double kappa, int iters, float* p, void* stream);
+
+/* gs_probabilities plus the solve record: `info` is a device pointer to one
+ * gs_info (may be NULL). */
+gs_status gs_probabilities_ex(const float* g, int64_t d, double kappa, int iters, float* p, gs_info* info,
+                              void* stream);
+
+/*
+ * Sparsify one worker's gradient (section 3): kept coordinates in
+ * ascending index order as idx[0..nnz) / val[0..nnz), val = g_i / p_i.
+ *   g      device, d fp32 values
+ *   idx    device, capacity d int32 (written)
+ *   val    device, capacity d fp32 (written)
+ *   nnz    device, one int32 (written)
+ * Equals row `worker` of gs_batched_sparsify(..., worker0 = worker, M = 1).
+ */
+gs_status gs_sparsify(const float* g, int64_t d, double kappa, int iters, uint64_t seed, uint32_t step,
+                      uint32_t worker, int32_t* idx, float* val, int32_t* nnz, void* stream);
+
+/*
+ * Sparsify M workers' gradients in one call (Algorithm 1, steps 4-5 for
+ * every worker).
+ *   g      device, M x d row-major; fp32 or bf16 per `dtype` (row m is
+ *          worker worker0 + m)
+ *   idx    device, M x cap int32: row m holds worker m's kept indices
+ *   val    device, M x cap fp32: the matching values g_i / p_i
+ *   nnz    device, M int32: kept count of each worker.  If a count exceeds
+ *          cap, only the first cap entries are written, nnz holds the true
+ *          count and GS_ERR_CAPACITY is recorded.
+ *   cap    row capacity, 1 <= cap <= d (cap = d can never overflow)
+ *   info   device, M gs_info records, or NULL
+ */
+gs_status gs_batched_sparsify(const void* g, int dtype, int M, int64_t d, double kappa, int iters, uint64_t seed,
+                              uint32_t step, uint32_t worker0, int32_t* idx, float* val, int32_t* nnz, int64_t cap,
+                              gs_info* info, void* stream);
+
+/*
+ * Layer-wise sparsification (section 5.2: each layer is sparsified on its
+ * own).  Each worker's vector is cut into L segments by the HOST array
+ * seg_offsets[0..L] (0 = seg_offsets[0] < ... < seg_offsets[L] = d); every
+ * segment gets its own Algorithm 3 with budget kappa * (segment length).
+ * Random words follow the worker's flat index, so each worker's output is
+ * one ascending list over all its segments.  Outputs as in
+ * gs_batched_sparsify; `info` (or NULL) holds M * L records, worker-major.
+ */
+gs_status gs_segmented_sparsify(const void* g, int dtype, int M, int64_t d, const int64_t* seg_offsets, int L,
+                                double kappa, int iters, uint64_t seed, uint32_t step, uint32_t worker0, int32_t* idx,
+                                float* val, int32_t* nnz, int64_t cap, gs_info* info, void* stream);
+
+/*
+ * Sum M sparse vectors into a dense fp32 vector (Algorithm 1, step 6):
+ *   out[i] = sum_{m=0}^{M-1} Q_m[i], added in fp32 in worker order, so the
+ *   result is deterministic.  `out` (device, d fp32) is overwritten.
+ *   idx, val   HOST arrays of M device pointers; list m holds nnz[m]
+ *              strictly ascending indices in [0, d) and their values
+ *   nnz        device, M int32
+ *   1 <= M <= 512.  An unsorted, duplicate or out-of-range index records
+ *   GS_ERR_INVALID_ARG and leaves `out` unspecified.
+ */
+gs_status gs_sparse_aggregate(const int32_t* const* idx, const float* const* val, const int32_t* nnz, int M, int64_t d,
+                              float* out, void* stream);
+
+/*
+ * The whole path for M workers with HOST buffers: copies g_host (M x d,
+ * `dtype`) to the device, runs gs_batched_sparsify and gs_sparse_aggregate,
+ * and copies the dense sum back to out_host (d fp32) and the kept counts to
+ * nnz_host (M int32).  g_dev / idx / val / nnz / out are caller-owned device
+ * buffers of the sizes gs_batched_sparsify / gs_sparse_aggregate require
+ * (idx, val: M x cap).  Host buffers should be pinned for full copy speed.
+ * Returns after enqueueing; the host buffers are valid once `stream` has
+ * been synchronised.
+ */
+gs_status gs_pipeline_host(const void* g_host, int dtype, int M, int64_t d, double kappa, int iters, uint64_t seed,
+                           uint32_t step, uint32_t worker0, void* g_dev, int32_t* idx, float* val, int32_t* nnz,
+                           int64_t cap, float* out, float* out_host, int32_t* nnz_host, void* stream);
+
+/*
+ * The random words the sampler draws (section 3, Z_i ~ Bernoulli(p_i)):
+ * out[k] = the Philox4x32-10 word of coordinate i0 + k of worker `worker` at
+ * `step` (see the conventions above), for k in [0, n).  Coordinate i is kept
+ * iff out * 2^-32 < p_i.  `out` is device memory for n uint32; i0 >= 0.
+ */
+gs_status gs_random_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t i0, int64_t n, uint32_t* out,
+                          void* stream);
+
+/* Library options for tests and diagnostics.
+ *   GS_OPT_FORCE_EXACT_SOLVE  1: skip the sampled bound and use the exact
+ *                              fallback solve for every worker (slow).
+ *   GS_OPT_SAMPLE_SIZE        sampled coordinates per segment for the bound
+ *                              on lambda (default 16384, >= 256).
+ * Options are process-wide; returns GS_ERR_INVALID_ARG for an unknown
+ * option or value. */
+typedef enum { GS_OPT_FORCE_EXACT_SOLVE = 1, GS_OPT_SAMPLE_SIZE = 2, GS_OPT_KERNEL_TIMING = 3 } gs_option;
+gs_status gs_set_option(int option, int64_t value);
+
+/* Tracing.  The library counts every kernel it launches; with
+ * GS_OPT_KERNEL_TIMING = 1 it also brackets each launch with CUDA events
+ * recorded on the launching stream.  gs_kernel_times() waits for the
+ * recorded events, writes for each kernel k < n the accumulated device time
+ * ms[k] and launch count launches[k] since the previous read (either array
+ * may be NULL), and resets both.  Kernel k is named by gs_kernel_name(k);
+ * gs_kernel_count() kernels exist. */
+int gs_kernel_count(void);
+const char* gs_kernel_name(int k);
+gs_status gs_kernel_times(double* ms, int64_t* launches, int n);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* GS_H */

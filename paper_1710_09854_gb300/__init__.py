@@ -1,0 +1,250 @@
+"""Python binding of libgs.so, the GB300 gradient-sparsification library.
+
+The functions carry the C-ABI names of include/gs.h and only marshal
+arguments: tensors become device pointers, shapes become sizes, the current
+torch stream becomes the cudaStream_t.  Every step of the computation runs in
+the library's CUDA kernels; there is no CPU fallback.  If libgs.so has not
+been built the first call raises.
+
+Build it with ``python -c "import __graft_entry__ as g; g.build()"`` (or
+``python paper_1710_09854_gb300/build.py``).
+"""
+import ctypes
+import os
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "libgs.so")
+
+GS_OK, GS_ERR_INVALID_ARG, GS_ERR_CUDA, GS_ERR_CAPACITY, GS_ERR_NONFINITE, GS_ERR_TIMEOUT, GS_ERR_INTERNAL = range(7)
+GS_DTYPE_F32, GS_DTYPE_BF16 = 0, 1
+GS_OPT_FORCE_EXACT_SOLVE, GS_OPT_SAMPLE_SIZE, GS_OPT_KERNEL_TIMING = 1, 2, 3
+
+# Symbols include/gs.h declares (checked by the tests).
+EXPORTS = ("gs_status_string", "gs_version", "gs_sync_status", "gs_probabilities", "gs_probabilities_ex",
+           "gs_sparsify", "gs_batched_sparsify", "gs_segmented_sparsify", "gs_sparse_aggregate",
+           "gs_pipeline_host", "gs_random_words", "gs_set_option", "gs_kernel_count", "gs_kernel_name",
+           "gs_kernel_times")
+
+
+class GSError(RuntimeError):
+    def __init__(self, code, where):
+        self.code = code
+        super().__init__(f"{where}: {status_string(code)}")
+
+
+class Info(ctypes.Structure):
+    """Mirror of gs_info (32 bytes)."""
+    _fields_ = [("lambda_", ctypes.c_double), ("sum_p", ctypes.c_double), ("capped", ctypes.c_int64),
+                ("iters_run", ctypes.c_int32), ("flags", ctypes.c_int32)]
+
+
+INFO_BYTES = ctypes.sizeof(Info)
+_LIB = None
+
+
+def lib():
+    global _LIB
+    if _LIB is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"CUDA library not built: {LIB_PATH} is missing "
+                               "(run `python -c \"import __graft_entry__ as g; g.build()\"`)")
+        L = ctypes.CDLL(LIB_PATH)
+        vp, i64, u64, u32, i32, dbl = (ctypes.c_void_p, ctypes.c_int64, ctypes.c_uint64, ctypes.c_uint32,
+                                       ctypes.c_int, ctypes.c_double)
+        sig = {
+            "gs_status_string": ([i32], ctypes.c_char_p),
+            "gs_version": ([], i32),
+            "gs_sync_status": ([vp], i32),
+            "gs_probabilities": ([vp, i64, dbl, i32, vp, vp], i32),
+            "gs_probabilities_ex": ([vp, i64, dbl, i32, vp, vp, vp], i32),
+            "gs_sparsify": ([vp, i64, dbl, i32, u64, u32, u32, vp, vp, vp, vp], i32),
+            "gs_batched_sparsify": ([vp, i32, i32, i64, dbl, i32, u64, u32, u32, vp, vp, vp, i64, vp, vp], i32),
+            "gs_segmented_sparsify": ([vp, i32, i32, i64, vp, i32, dbl, i32, u64, u32, u32, vp, vp, vp, i64, vp, vp],
+                                      i32),
+            "gs_sparse_aggregate": ([vp, vp, vp, i32, i64, vp, vp], i32),
+            "gs_pipeline_host": ([vp, i32, i32, i64, dbl, i32, u64, u32, u32, vp, vp, vp, vp, i64, vp, vp, vp, vp],
+                                 i32),
+            "gs_random_words": ([u64, u32, u32, i64, i64, vp, vp], i32),
+            "gs_set_option": ([i32, i64], i32),
+            "gs_kernel_count": ([], i32),
+            "gs_kernel_name": ([i32], ctypes.c_char_p),
+            "gs_kernel_times": ([vp, vp, i32], i32),
+        }
+        for name, (args, res) in sig.items():
+            f = getattr(L, name)
+            f.argtypes = args
+            f.restype = res
+        _LIB = L
+    return _LIB
+
+
+def status_string(code):
+    return lib().gs_status_string(int(code)).decode()
+
+
+def _check(rc, where):
+    if rc != GS_OK:
+        raise GSError(rc, where)
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _ptr(t, name, dtypes=None):
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if dtypes is not None and t.dtype not in dtypes:
+        raise ValueError(f"{name} has dtype {t.dtype}, expected one of {dtypes}")
+    return t.data_ptr()
+
+
+def _g_dtype(g):
+    import torch
+    if g.dtype == torch.float32:
+        return GS_DTYPE_F32
+    if g.dtype == torch.bfloat16:
+        return GS_DTYPE_BF16
+    raise ValueError(f"g must be float32 or bfloat16, got {g.dtype}")
+
+
+def info_tensor(n, device="cuda"):
+    """Device buffer for n gs_info records."""
+    import torch
+    return torch.zeros(n * INFO_BYTES, dtype=torch.uint8, device=device)
+
+
+def decode_info(t):
+    """gs_info records of a (device or host) buffer as a list of dicts."""
+    raw = t.cpu().numpy().tobytes() if hasattr(t, "cpu") else bytes(t)
+    n = len(raw) // INFO_BYTES
+    out = []
+    for k in range(n):
+        r = Info.from_buffer_copy(raw[k * INFO_BYTES:(k + 1) * INFO_BYTES])
+        out.append({"lambda": r.lambda_, "sum_p": r.sum_p, "capped": r.capped, "iters_run": r.iters_run,
+                    "flags": r.flags})
+    return out
+
+
+def gs_version():
+    return lib().gs_version()
+
+
+def gs_sync_status(stream=None):
+    return lib().gs_sync_status(_stream(stream))
+
+
+def gs_set_option(option, value):
+    _check(lib().gs_set_option(int(option), int(value)), "gs_set_option")
+
+
+def gs_kernel_count():
+    return lib().gs_kernel_count()
+
+
+def gs_kernel_name(k):
+    return lib().gs_kernel_name(int(k)).decode()
+
+
+def gs_kernel_times():
+    """{kernel name: (accumulated ms, launches)} since the previous read; resets."""
+    n = gs_kernel_count()
+    ms = (ctypes.c_double * n)()
+    nl = (ctypes.c_int64 * n)()
+    _check(lib().gs_kernel_times(ms, nl, n), "gs_kernel_times")
+    return {gs_kernel_name(k): (ms[k], nl[k]) for k in range(n)}
+
+
+def gs_random_words(seed, step, worker, i0, out, stream=None):
+    """out: int32 CUDA tensor receiving the words (bit patterns) of coordinates i0 .. i0 + out.numel() - 1."""
+    import torch
+    _check(lib().gs_random_words(int(seed), int(step), int(worker), int(i0), out.numel(),
+                                 _ptr(out, "out", (torch.int32,)), _stream(stream)), "gs_random_words")
+
+
+def gs_probabilities(g, kappa, iters, p, stream=None):
+    import torch
+    _check(lib().gs_probabilities(_ptr(g, "g", (torch.float32,)), g.numel(), float(kappa), int(iters),
+                                  _ptr(p, "p", (torch.float32,)), _stream(stream)), "gs_probabilities")
+
+
+def gs_probabilities_ex(g, kappa, iters, p, info=None, stream=None):
+    import torch
+    _check(lib().gs_probabilities_ex(_ptr(g, "g", (torch.float32,)), g.numel(), float(kappa), int(iters),
+                                     _ptr(p, "p", (torch.float32,)), _ptr(info, "info"), _stream(stream)),
+           "gs_probabilities_ex")
+
+
+def gs_sparsify(g, kappa, iters, seed, step, worker, idx, val, nnz, stream=None):
+    import torch
+    if idx.numel() < g.numel() or val.numel() < g.numel():
+        raise ValueError("idx / val need capacity d")
+    _check(lib().gs_sparsify(_ptr(g, "g", (torch.float32,)), g.numel(), float(kappa), int(iters), int(seed),
+                             int(step), int(worker), _ptr(idx, "idx", (torch.int32,)),
+                             _ptr(val, "val", (torch.float32,)), _ptr(nnz, "nnz", (torch.int32,)), _stream(stream)),
+           "gs_sparsify")
+
+
+def gs_batched_sparsify(g, kappa, iters, seed, step, worker0, idx, val, nnz, info=None, stream=None):
+    """g: (M, d) fp32/bf16; idx/val: (M, cap); nnz: (M,)."""
+    import torch
+    M, d = g.shape
+    cap = idx.shape[1]
+    if idx.shape[0] != M or tuple(val.shape) != tuple(idx.shape) or nnz.numel() != M:
+        raise ValueError("idx / val must be (M, cap) and nnz (M,)")
+    _check(lib().gs_batched_sparsify(_ptr(g, "g"), _g_dtype(g), M, d, float(kappa), int(iters), int(seed),
+                                     int(step), int(worker0), _ptr(idx, "idx", (torch.int32,)),
+                                     _ptr(val, "val", (torch.float32,)), _ptr(nnz, "nnz", (torch.int32,)), cap,
+                                     _ptr(info, "info"), _stream(stream)), "gs_batched_sparsify")
+
+
+def gs_segmented_sparsify(g, seg_offsets, kappa, iters, seed, step, worker0, idx, val, nnz, info=None, stream=None):
+    """g: (M, d); seg_offsets: host sequence of L+1 offsets (0 .. d)."""
+    import torch
+    M, d = g.shape
+    cap = idx.shape[1]
+    off = np.ascontiguousarray(seg_offsets, dtype=np.int64)
+    if idx.shape[0] != M or tuple(val.shape) != tuple(idx.shape) or nnz.numel() != M:
+        raise ValueError("idx / val must be (M, cap) and nnz (M,)")
+    _check(lib().gs_segmented_sparsify(_ptr(g, "g"), _g_dtype(g), M, d, off.ctypes.data, off.size - 1,
+                                       float(kappa), int(iters), int(seed), int(step), int(worker0),
+                                       _ptr(idx, "idx", (torch.int32,)), _ptr(val, "val", (torch.float32,)),
+                                       _ptr(nnz, "nnz", (torch.int32,)), cap, _ptr(info, "info"), _stream(stream)),
+           "gs_segmented_sparsify")
+
+
+def gs_sparse_aggregate(idx_list, val_list, nnz, d, out, stream=None):
+    """idx_list / val_list: M device tensors (or rows of (M, cap) tensors)."""
+    import torch
+    M = len(idx_list)
+    ip = (ctypes.c_void_p * M)(*[_ptr(x, "idx", (torch.int32,)) for x in idx_list])
+    vp = (ctypes.c_void_p * M)(*[_ptr(x, "val", (torch.float32,)) for x in val_list])
+    _check(lib().gs_sparse_aggregate(ip, vp, _ptr(nnz, "nnz", (torch.int32,)), M, int(d),
+                                     _ptr(out, "out", (torch.float32,)), _stream(stream)), "gs_sparse_aggregate")
+
+
+def gs_pipeline_host(g_host, kappa, iters, seed, step, worker0, g_dev, idx, val, nnz, out, out_host, nnz_host,
+                     stream=None):
+    """g_host: (M, d) pinned CPU tensor; out_host (d,) / nnz_host (M,) pinned CPU tensors."""
+    import torch
+    M, d = g_host.shape
+    cap = idx.shape[1]
+    for t, n in ((g_host, "g_host"), (out_host, "out_host"), (nnz_host, "nnz_host")):
+        if t.is_cuda or not t.is_contiguous():
+            raise ValueError(f"{n} must be a contiguous host tensor")
+    _check(lib().gs_pipeline_host(g_host.data_ptr(), _g_dtype(g_host), M, d, float(kappa), int(iters), int(seed),
+                                  int(step), int(worker0), _ptr(g_dev, "g_dev"), _ptr(idx, "idx", (torch.int32,)),
+                                  _ptr(val, "val", (torch.float32,)), _ptr(nnz, "nnz", (torch.int32,)), cap,
+                                  _ptr(out, "out", (torch.float32,)), out_host.data_ptr(), nnz_host.data_ptr(),
+                                  _stream(stream)), "gs_pipeline_host")

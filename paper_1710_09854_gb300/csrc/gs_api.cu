@@ -1,0 +1,365 @@
+// gs_api.cu -- the C ABI of libgs.so (declared in include/gs.h): argument
+// validation, the library's stream-ordered memory pool, the per-device
+// status word, and the order of the kernel launches of each call.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <map>
+#include <mutex>
+#include <vector>
+
+#include "gs.h"
+#include "gs_launch.h"
+#include "gs_trace.h"
+
+using namespace gs;
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+constexpr int64_t kMaxD = (int64_t)1 << 31;
+
+struct SegMeta {
+    int64_t* off = nullptr;     // device [L+1]
+    int32_t* chunk0 = nullptr;  // device [L+1]
+    int cpw = 0;
+};
+
+struct DevState {
+    bool ready = false;
+    cudaMemPool_t pool = nullptr;
+    int* status = nullptr;  // device word, OR of kSt* bits
+    std::map<std::vector<int64_t>, SegMeta> segs;
+};
+
+std::mutex g_mu;
+DevState g_dev[kMaxDevices];
+int g_force_exact = 0;
+int g_sample = 16384;
+
+gs_status device_state(DevState** out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return GS_ERR_CUDA;
+    std::lock_guard<std::mutex> lk(g_mu);
+    DevState& s = g_dev[dev];
+    if (!s.ready) {
+        cudaMemPoolProps props;
+        std::memset(&props, 0, sizeof(props));
+        props.allocType = cudaMemAllocationTypePinned;
+        props.location.type = cudaMemLocationTypeDevice;
+        props.location.id = dev;
+        if (cudaMemPoolCreate(&s.pool, &props) != cudaSuccess) return GS_ERR_CUDA;
+        uint64_t keep = UINT64_MAX;  // keep freed blocks for the next call
+        cudaMemPoolSetAttribute(s.pool, cudaMemPoolAttrReleaseThreshold, &keep);
+        if (cudaMalloc(&s.status, sizeof(int)) != cudaSuccess) return GS_ERR_CUDA;
+        if (cudaMemset(s.status, 0, sizeof(int)) != cudaSuccess) return GS_ERR_CUDA;
+        if (cudaDeviceSynchronize() != cudaSuccess) return GS_ERR_CUDA;
+        s.ready = true;
+    }
+    *out = &s;
+    return GS_OK;
+}
+
+// Segment tables for layer-wise calls, uploaded once per distinct layout.
+gs_status segment_meta(DevState* s, const int64_t* off, int L, SegMeta* out) {
+    std::vector<int64_t> key(off, off + L + 1);
+    std::lock_guard<std::mutex> lk(g_mu);
+    auto it = s->segs.find(key);
+    if (it != s->segs.end()) {
+        *out = it->second;
+        return GS_OK;
+    }
+    std::vector<int32_t> c0(L + 1);
+    int64_t acc = 0;
+    for (int l = 0; l < L; ++l) {
+        c0[l] = (int32_t)acc;
+        acc += (off[l + 1] - off[l] + chunk_size() - 1) / chunk_size();
+    }
+    c0[L] = (int32_t)acc;
+    if (acc > INT32_MAX) return GS_ERR_INVALID_ARG;
+    SegMeta m;
+    m.cpw = (int)acc;
+    if (cudaMalloc(&m.off, sizeof(int64_t) * (L + 1)) != cudaSuccess) return GS_ERR_CUDA;
+    if (cudaMalloc(&m.chunk0, sizeof(int32_t) * (L + 1)) != cudaSuccess) return GS_ERR_CUDA;
+    if (cudaMemcpy(m.off, off, sizeof(int64_t) * (L + 1), cudaMemcpyHostToDevice) != cudaSuccess) return GS_ERR_CUDA;
+    if (cudaMemcpy(m.chunk0, c0.data(), sizeof(int32_t) * (L + 1), cudaMemcpyHostToDevice) != cudaSuccess)
+        return GS_ERR_CUDA;
+    if (s->segs.size() >= 32) s->segs.clear();  // bounded cache (device tables are tiny; kept until exit)
+    s->segs[key] = m;
+    *out = m;
+    return GS_OK;
+}
+
+// Bump allocator over one pool allocation; a null base only measures.
+struct Arena {
+    char* base = nullptr;
+    size_t off = 0;
+    template <typename T>
+    T* take(size_t n) {
+        off = (off + 255) & ~(size_t)255;
+        T* p = base ? reinterpret_cast<T*>(base + off) : nullptr;
+        off += n * sizeof(T);
+        return p;
+    }
+};
+
+bool bad_kappa(double kappa) { return !(kappa > 0.0) || kappa > 1.0 || !std::isfinite(kappa); }
+
+struct Workspace {
+    SegParam* sp;
+    Lists ls;
+};
+
+void carve(Arena& a, Workspace& w, int n_seg, int n_chunks, int64_t n, bool build_p) {
+    std::memset(&w, 0, sizeof(w));
+    w.sp = a.take<SegParam>(n_seg);
+    w.ls.c_val = a.take<float>(n);
+    w.ls.c_cnt = a.take<int32_t>(n_chunks);
+    w.ls.s_low = a.take<double>(n_chunks);
+    if (build_p) {
+        w.ls.p_idx = a.take<int32_t>(n);
+        w.ls.p_g = a.take<float>(n);
+        w.ls.p_x = a.take<uint32_t>(n);
+        w.ls.p_cnt = a.take<int32_t>(n_chunks);
+        w.ls.k_cnt = a.take<int32_t>(n_chunks);
+        w.ls.k_off = a.take<int32_t>(n_chunks);
+    }
+}
+
+// Shared driver of every sparsify / probabilities call.
+gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off, int L, double kappa, int iters,
+              uint64_t seed, uint32_t step, uint32_t worker0, int32_t* idx, float* val, int32_t* nnz, int64_t cap,
+              gs_info* info, float* p, cudaStream_t st) {
+    const bool prob = p != nullptr;
+    if (!g || M < 1 || d < 1 || d >= kMaxD || bad_kappa(kappa) || iters < 0) return GS_ERR_INVALID_ARG;
+    if (dtype != GS_DTYPE_F32 && dtype != GS_DTYPE_BF16) return GS_ERR_INVALID_ARG;
+    const size_t esz = dtype == GS_DTYPE_F32 ? 4 : 2;
+    if ((reinterpret_cast<uintptr_t>(g) % esz) != 0) return GS_ERR_INVALID_ARG;
+    if (!prob && (!idx || !val || !nnz || cap < 1)) return GS_ERR_INVALID_ARG;
+    if ((int64_t)M > ((int64_t)1 << 40) / d) return GS_ERR_INVALID_ARG;
+    if (L < 1) return GS_ERR_INVALID_ARG;
+    if (L > 1) {
+        if (!seg_off || seg_off[0] != 0 || seg_off[L] != d) return GS_ERR_INVALID_ARG;
+        for (int l = 0; l < L; ++l)
+            if (seg_off[l + 1] <= seg_off[l]) return GS_ERR_INVALID_ARG;
+    }
+
+    DevState* s = nullptr;
+    gs_status rc = device_state(&s);
+    if (rc != GS_OK) return rc;
+
+    Layout Lo;
+    std::memset(&Lo, 0, sizeof(Lo));
+    Lo.g = g;
+    Lo.dtype = dtype;
+    Lo.M = M;
+    Lo.L = L;
+    Lo.d = d;
+    Lo.seed = seed;
+    Lo.step = step;
+    Lo.worker0 = worker0;
+    if (L == 1) {
+        const int64_t cpw = (d + chunk_size() - 1) / chunk_size();
+        Lo.cpw = (int)cpw;
+    } else {
+        SegMeta meta;
+        rc = segment_meta(s, seg_off, L, &meta);
+        if (rc != GS_OK) return rc;
+        Lo.seg_off = meta.off;
+        Lo.seg_chunk0 = meta.chunk0;
+        Lo.cpw = meta.cpw;
+    }
+    const int64_t n_chunks64 = (int64_t)M * Lo.cpw;
+    const int64_t n_seg64 = (int64_t)M * L;
+    if (n_chunks64 > INT32_MAX || n_seg64 > INT32_MAX) return GS_ERR_INVALID_ARG;
+    const int n_chunks = (int)n_chunks64, n_seg = (int)n_seg64;
+
+    Arena a;
+    Workspace w;
+    carve(a, w, n_seg, n_chunks, (int64_t)M * d, !prob);
+    void* mem = nullptr;
+    if (cudaMallocFromPoolAsync(&mem, a.off, s->pool, st) != cudaSuccess) return GS_ERR_CUDA;
+    a.base = static_cast<char*>(mem);
+    a.off = 0;
+    carve(a, w, n_seg, n_chunks, (int64_t)M * d, !prob);
+
+    int force;
+    int ns;
+    {
+        std::lock_guard<std::mutex> lk(g_mu);
+        force = g_force_exact;
+        ns = g_sample;
+    }
+    cudaError_t e = launch_bound(Lo, w.sp, n_seg, kappa, ns, force, st);
+    if (e == cudaSuccess) e = launch_stream(Lo, w.sp, w.ls, n_chunks, !prob, st);
+    if (e == cudaSuccess) e = launch_solve(Lo, w.sp, w.ls, n_seg, kappa, iters, force, s->status, info, st);
+    if (e == cudaSuccess) {
+        if (prob) e = launch_prob(Lo, w.sp, p, st);
+        else e = launch_compact(Lo, w.sp, w.ls, n_chunks, idx, val, nnz, cap, s->status, st);
+    }
+    cudaError_t ef = cudaFreeAsync(mem, st);
+    if (e != cudaSuccess || ef != cudaSuccess) return GS_ERR_CUDA;
+    return GS_OK;
+}
+
+gs_status run_aggregate(const int32_t* const* idx, const float* const* val, const int32_t* nnz, int M, int64_t d,
+                        float* out, int64_t cap, cudaStream_t st) {
+    if (!idx || !val || !nnz || !out || M < 1 || M > kMaxAggM || d < 1 || d >= kMaxD) return GS_ERR_INVALID_ARG;
+    for (int m = 0; m < M; ++m)
+        if (!idx[m] || !val[m]) return GS_ERR_INVALID_ARG;
+    DevState* s = nullptr;
+    gs_status rc = device_state(&s);
+    if (rc != GS_OK) return rc;
+    AggArgs A;
+    std::memset(&A, 0, sizeof(A));
+    for (int m = 0; m < M; ++m) {
+        A.idx[m] = idx[m];
+        A.val[m] = val[m];
+    }
+    A.nnz = nnz;
+    A.M = M;
+    A.d = d;
+    A.cap = cap;
+    const int nt = agg_tiles(d);
+    void* mem = nullptr;
+    const size_t bytes = sizeof(int32_t) * (size_t)M * (size_t)(nt + 1);
+    if (cudaMallocFromPoolAsync(&mem, bytes, s->pool, st) != cudaSuccess) return GS_ERR_CUDA;
+    cudaError_t e = launch_aggregate(A, static_cast<int32_t*>(mem), out, s->status, st);
+    cudaError_t ef = cudaFreeAsync(mem, st);
+    return (e == cudaSuccess && ef == cudaSuccess) ? GS_OK : GS_ERR_CUDA;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* gs_status_string(int status) {
+    switch (status) {
+        case GS_OK: return "GS_OK";
+        case GS_ERR_INVALID_ARG: return "GS_ERR_INVALID_ARG";
+        case GS_ERR_CUDA: return "GS_ERR_CUDA";
+        case GS_ERR_CAPACITY: return "GS_ERR_CAPACITY";
+        case GS_ERR_NONFINITE: return "GS_ERR_NONFINITE";
+        case GS_ERR_TIMEOUT: return "GS_ERR_TIMEOUT";
+        case GS_ERR_INTERNAL: return "GS_ERR_INTERNAL";
+        default: return "GS_UNKNOWN_STATUS";
+    }
+}
+
+int gs_version(void) { return 100; }
+
+gs_status gs_sync_status(void* stream) {
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    DevState* s = nullptr;
+    gs_status rc = device_state(&s);
+    if (rc != GS_OK) return rc;
+    int h = 0;
+    if (cudaMemcpyAsync(&h, s->status, sizeof(int), cudaMemcpyDeviceToHost, st) != cudaSuccess) return GS_ERR_CUDA;
+    if (cudaMemsetAsync(s->status, 0, sizeof(int), st) != cudaSuccess) return GS_ERR_CUDA;
+    if (cudaStreamSynchronize(st) != cudaSuccess) return GS_ERR_CUDA;
+    if (h & kStNonfinite) return GS_ERR_NONFINITE;
+    if (h & kStCapacity) return GS_ERR_CAPACITY;
+    if (h & kStInvalid) return GS_ERR_INVALID_ARG;
+    if (h & kStTimeout) return GS_ERR_TIMEOUT;
+    if (h & kStInternal) return GS_ERR_INTERNAL;
+    return GS_OK;
+}
+
+gs_status gs_probabilities(const float* g, int64_t d, double kappa, int iters, float* p, void* stream) {
+    return gs_probabilities_ex(g, d, kappa, iters, p, nullptr, stream);
+}
+
+gs_status gs_probabilities_ex(const float* g, int64_t d, double kappa, int iters, float* p, gs_info* info,
+                              void* stream) {
+    if (!p) return GS_ERR_INVALID_ARG;
+    return run(g, GS_DTYPE_F32, 1, d, nullptr, 1, kappa, iters, 0, 0, 0, nullptr, nullptr, nullptr, 0, info, p,
+               static_cast<cudaStream_t>(stream));
+}
+
+gs_status gs_sparsify(const float* g, int64_t d, double kappa, int iters, uint64_t seed, uint32_t step,
+                      uint32_t worker, int32_t* idx, float* val, int32_t* nnz, void* stream) {
+    return run(g, GS_DTYPE_F32, 1, d, nullptr, 1, kappa, iters, seed, step, worker, idx, val, nnz, d, nullptr,
+               nullptr, static_cast<cudaStream_t>(stream));
+}
+
+gs_status gs_batched_sparsify(const void* g, int dtype, int M, int64_t d, double kappa, int iters, uint64_t seed,
+                              uint32_t step, uint32_t worker0, int32_t* idx, float* val, int32_t* nnz, int64_t cap,
+                              gs_info* info, void* stream) {
+    return run(g, dtype, M, d, nullptr, 1, kappa, iters, seed, step, worker0, idx, val, nnz, cap, info, nullptr,
+               static_cast<cudaStream_t>(stream));
+}
+
+gs_status gs_segmented_sparsify(const void* g, int dtype, int M, int64_t d, const int64_t* seg_offsets, int L,
+                                double kappa, int iters, uint64_t seed, uint32_t step, uint32_t worker0, int32_t* idx,
+                                float* val, int32_t* nnz, int64_t cap, gs_info* info, void* stream) {
+    if (L < 1 || !seg_offsets) return GS_ERR_INVALID_ARG;
+    if (L == 1 && (seg_offsets[0] != 0 || seg_offsets[1] != d)) return GS_ERR_INVALID_ARG;
+    return run(g, dtype, M, d, seg_offsets, L, kappa, iters, seed, step, worker0, idx, val, nnz, cap, info, nullptr,
+               static_cast<cudaStream_t>(stream));
+}
+
+gs_status gs_sparse_aggregate(const int32_t* const* idx, const float* const* val, const int32_t* nnz, int M, int64_t d,
+                              float* out, void* stream) {
+    return run_aggregate(idx, val, nnz, M, d, out, INT64_MAX, static_cast<cudaStream_t>(stream));
+}
+
+gs_status gs_pipeline_host(const void* g_host, int dtype, int M, int64_t d, double kappa, int iters, uint64_t seed,
+                           uint32_t step, uint32_t worker0, void* g_dev, int32_t* idx, float* val, int32_t* nnz,
+                           int64_t cap, float* out, float* out_host, int32_t* nnz_host, void* stream) {
+    if (!g_host || !g_dev || !out || !out_host || !nnz_host) return GS_ERR_INVALID_ARG;
+    if (M < 1 || M > kMaxAggM || d < 1 || d >= kMaxD || cap < 1) return GS_ERR_INVALID_ARG;
+    if (dtype != GS_DTYPE_F32 && dtype != GS_DTYPE_BF16) return GS_ERR_INVALID_ARG;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    const size_t esz = dtype == GS_DTYPE_F32 ? 4 : 2;
+    if (cudaMemcpyAsync(g_dev, g_host, esz * (size_t)M * (size_t)d, cudaMemcpyHostToDevice, st) != cudaSuccess)
+        return GS_ERR_CUDA;
+    gs_status rc = run(g_dev, dtype, M, d, nullptr, 1, kappa, iters, seed, step, worker0, idx, val, nnz, cap, nullptr,
+                       nullptr, st);
+    if (rc != GS_OK) return rc;
+    std::vector<const int32_t*> ip(M);
+    std::vector<const float*> vp(M);
+    for (int m = 0; m < M; ++m) {
+        ip[m] = idx + (size_t)m * (size_t)cap;
+        vp[m] = val + (size_t)m * (size_t)cap;
+    }
+    rc = run_aggregate(ip.data(), vp.data(), nnz, M, d, out, cap, st);
+    if (rc != GS_OK) return rc;
+    if (cudaMemcpyAsync(out_host, out, sizeof(float) * (size_t)d, cudaMemcpyDeviceToHost, st) != cudaSuccess)
+        return GS_ERR_CUDA;
+    if (cudaMemcpyAsync(nnz_host, nnz, sizeof(int32_t) * (size_t)M, cudaMemcpyDeviceToHost, st) != cudaSuccess)
+        return GS_ERR_CUDA;
+    return GS_OK;
+}
+
+gs_status gs_random_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t i0, int64_t n, uint32_t* out,
+                          void* stream) {
+    if (!out || i0 < 0 || n < 0 || i0 > INT64_MAX - n) return GS_ERR_INVALID_ARG;
+    if (n == 0) return GS_OK;
+    return launch_words(seed, step, worker, i0, n, out, static_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? GS_OK
+               : GS_ERR_CUDA;
+}
+
+gs_status gs_set_option(int option, int64_t value) {
+    std::lock_guard<std::mutex> lk(g_mu);
+    switch (option) {
+        case GS_OPT_FORCE_EXACT_SOLVE:
+            if (value != 0 && value != 1) return GS_ERR_INVALID_ARG;
+            g_force_exact = (int)value;
+            return GS_OK;
+        case GS_OPT_SAMPLE_SIZE:
+            if (value < 256 || value > 32768) return GS_ERR_INVALID_ARG;
+            g_sample = (int)value;
+            return GS_OK;
+        case GS_OPT_KERNEL_TIMING:
+            if (value != 0 && value != 1) return GS_ERR_INVALID_ARG;
+            trace_set_timing((int)value);
+            return GS_OK;
+        default:
+            return GS_ERR_INVALID_ARG;
+    }
+}
+
+}  // extern "C"

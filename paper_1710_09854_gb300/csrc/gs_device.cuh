@@ -1,0 +1,264 @@
+// gs_device.cuh -- device-side building blocks of the GB300 gradient
+// sparsifier: Philox4x32-10, the chunk layout of M worker gradients, the
+// per-segment solve record, and deterministic block reductions.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace gs {
+
+// Coordinates per chunk: the unit of work of the streaming pass and the
+// capacity of each chunk's candidate lists.  A multiple of 4 so that chunk
+// starts inside a worker row keep the 4-coordinate Philox groups aligned.
+constexpr int kChunk = 16384;
+// Coordinates per output tile of the sparse sum.
+constexpr int kAggTile = 8192;
+// Threads per CTA of the streaming / solve / decide kernels.
+constexpr int kThreads = 256;
+constexpr int kWarps = kThreads / 32;
+// 4-coordinate groups each thread handles per step of the streaming pass.
+constexpr int kGroupsPerThread = 4;
+
+// Device status bits (the host maps them to gs_status codes).
+enum : int {
+    kStInvalid = 1 << 1,
+    kStCapacity = 1 << 3,
+    kStNonfinite = 1 << 4,
+    kStTimeout = 1 << 5,
+    kStInternal = 1 << 6,
+};
+
+// Segment flags.
+enum : int {
+    kSegExact = 1,       // the exact fallback solve ran for this segment
+    kSegNonfinite = 2,   // the segment holds NaN / Inf
+    kSegTakeAll = 4,     // the bound pass kept every candidate (short segment)
+};
+
+// Where the M gradients live and how they are cut into segments / chunks.
+struct Layout {
+    const void* g;            // M x d, row-major
+    int dtype;                // 0 fp32, 1 bf16
+    int M;
+    int L;                    // segments per worker (1: whole row)
+    int cpw;                  // chunks per worker
+    int64_t d;
+    const int64_t* seg_off;   // [L+1] local offsets; NULL when L == 1
+    const int32_t* seg_chunk0;// [L+1] first chunk (within a worker) of each segment; NULL when L == 1
+    uint64_t seed;
+    uint32_t step;
+    uint32_t worker0;
+};
+
+// Per-segment state: the bound of the sampling pass and the final solve.
+struct SegParam {
+    double lam_up;     // upper bound used to build the candidate lists
+    double lam;        // final lambda (Algorithm 3)
+    double sum_p;      // sum p at the final lambda
+    double l1;         // sum |g|
+    long long capped;  // #{p = 1}
+    float lam_up32;    // fl32(lam_up), rounded up
+    float t_c;         // |g| >= t_c goes to the capped-candidate list C
+    float lam32;       // fl32(lam)
+    float a_cap;       // smallest fp32 a with fl64(lam * a) >= 1 (capped iff |g| >= a_cap)
+    float inv_lam32;   // fl32(1 / lam): the amplified value of uncapped entries
+    int iters_run;
+    int flags;
+    int pad;
+};
+
+// Candidate lists written by the streaming pass, one region per chunk at the
+// chunk's flat offset (capacity = chunk length).
+struct Lists {
+    int32_t* p_idx;     // worker-local index of each kept candidate
+    float* p_g;         // its gradient value
+    uint32_t* p_x;      // its Philox word
+    int32_t* p_cnt;     // [n_chunks]
+    float* c_val;       // |g| of each capped candidate
+    int32_t* c_cnt;     // [n_chunks]
+    double* s_low;      // [n_chunks] sum of |g| outside C
+    int32_t* k_cnt;     // [n_chunks] kept count
+    int32_t* k_off;     // [n_chunks] exclusive offset of the chunk in its worker's output
+};
+
+struct Chunk {
+    int m;         // worker row
+    int l;         // segment within the row
+    int seg;       // m * L + l
+    int64_t lo;    // worker-local coordinate range [lo, hi)
+    int64_t hi;
+};
+
+__device__ __forceinline__ Chunk decode_chunk(const Layout& Lo, int c) {
+    Chunk ch;
+    ch.m = c / Lo.cpw;
+    int k = c - ch.m * Lo.cpw;
+    if (Lo.L == 1) {
+        ch.l = 0;
+        ch.lo = (int64_t)k * kChunk;
+        ch.hi = min(Lo.d, ch.lo + kChunk);
+    } else {
+        // last segment whose first chunk is <= k
+        int a = 0, b = Lo.L - 1;
+        while (a < b) {
+            int mid = (a + b + 1) >> 1;
+            if (Lo.seg_chunk0[mid] <= k) a = mid; else b = mid - 1;
+        }
+        ch.l = a;
+        ch.lo = Lo.seg_off[a] + (int64_t)(k - Lo.seg_chunk0[a]) * kChunk;
+        ch.hi = min(Lo.seg_off[a + 1], ch.lo + kChunk);
+    }
+    ch.seg = ch.m * Lo.L + ch.l;
+    return ch;
+}
+
+__device__ __forceinline__ void seg_range(const Layout& Lo, int seg, int& m, int& l, int64_t& lo, int64_t& hi,
+                                          int& c0, int& c1) {
+    m = seg / Lo.L;
+    l = seg - m * Lo.L;
+    if (Lo.L == 1) {
+        lo = 0;
+        hi = Lo.d;
+        c0 = m * Lo.cpw;
+        c1 = c0 + Lo.cpw;
+    } else {
+        lo = Lo.seg_off[l];
+        hi = Lo.seg_off[l + 1];
+        c0 = m * Lo.cpw + Lo.seg_chunk0[l];
+        c1 = m * Lo.cpw + Lo.seg_chunk0[l + 1];
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Philox4x32-10 (Salmon, Moraes, Dror, Shaw, SC'11).  Each round multiplies
+// words 0 and 2 by the published constants, swaps the high halves into the
+// odd positions crossed with the key, and bumps the key by the Weyl
+// increments.  The 32x32->64 products map to one wide integer multiply each.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ uint4 philox4x32_10(uint32_t c0, uint32_t c1, uint32_t c2, uint32_t c3, uint32_t k0,
+                                               uint32_t k1) {
+#pragma unroll
+    for (int r = 0; r < 10; ++r) {
+        const uint64_t m0 = (uint64_t)0xD2511F53u * (uint64_t)c0;
+        const uint64_t m1 = (uint64_t)0xCD9E8D57u * (uint64_t)c2;
+        const uint32_t n0 = (uint32_t)(m1 >> 32) ^ c1 ^ k0;
+        const uint32_t n2 = (uint32_t)(m0 >> 32) ^ c3 ^ k1;
+        c1 = (uint32_t)m1;
+        c3 = (uint32_t)m0;
+        c0 = n0;
+        c2 = n2;
+        k0 += 0x9E3779B9u;
+        k1 += 0xBB67AE85u;
+    }
+    return make_uint4(c0, c1, c2, c3);
+}
+
+// The 4 words of the 4-coordinate group q of worker `worker` at `step`.
+__device__ __forceinline__ uint4 group_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t q) {
+    return philox4x32_10((uint32_t)((uint64_t)q & 0xFFFFFFFFu), (uint32_t)((uint64_t)q >> 32), worker, step,
+                         (uint32_t)(seed & 0xFFFFFFFFu), (uint32_t)(seed >> 32));
+}
+
+__device__ __forceinline__ uint32_t word_of(const uint4& w, int s) {
+    return s == 0 ? w.x : (s == 1 ? w.y : (s == 2 ? w.z : w.w));
+}
+
+// 1 + (x >> 9) * 2^-23: a float in [1, 2) that never exceeds 1 + x * 2^-32.
+__device__ __forceinline__ float unit_plus_one(uint32_t x) {
+    return __uint_as_float(0x3F800000u | (x >> 9));
+}
+
+// ---------------------------------------------------------------------------
+// Loads
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float bf16_bits_to_float(uint32_t b) { return __uint_as_float(b << 16); }
+
+// Load the coordinates 4q..4q+3 of worker row `m` that fall in [lo, hi).
+// Returns a 4-bit mask of the valid ones; invalid slots read as 0.
+__device__ __forceinline__ int load_group(const Layout& Lo, int m, int64_t q, int64_t lo, int64_t hi, float v[4]) {
+    const int64_t i0 = q * 4;
+    const int64_t flat = (int64_t)m * Lo.d + i0;
+    const bool full = (i0 >= lo) && (i0 + 4 <= hi);
+    if (Lo.dtype == 0) {
+        const float* g = static_cast<const float*>(Lo.g);
+        if (full && ((reinterpret_cast<uintptr_t>(g + flat) & 15u) == 0)) {
+            float4 t = __ldcs(reinterpret_cast<const float4*>(g + flat));
+            v[0] = t.x; v[1] = t.y; v[2] = t.z; v[3] = t.w;
+            return 0xF;
+        }
+        int mask = 0;
+#pragma unroll
+        for (int s = 0; s < 4; ++s) {
+            const int64_t i = i0 + s;
+            if (i >= lo && i < hi) { v[s] = __ldcs(g + flat + s); mask |= 1 << s; }
+            else v[s] = 0.0f;
+        }
+        return mask;
+    } else {
+        const uint16_t* g = static_cast<const uint16_t*>(Lo.g);
+        if (full && ((reinterpret_cast<uintptr_t>(g + flat) & 7u) == 0)) {
+            uint2 t = __ldcs(reinterpret_cast<const uint2*>(g + flat));
+            v[0] = bf16_bits_to_float(t.x & 0xFFFFu); v[1] = bf16_bits_to_float(t.x >> 16);
+            v[2] = bf16_bits_to_float(t.y & 0xFFFFu); v[3] = bf16_bits_to_float(t.y >> 16);
+            return 0xF;
+        }
+        int mask = 0;
+#pragma unroll
+        for (int s = 0; s < 4; ++s) {
+            const int64_t i = i0 + s;
+            if (i >= lo && i < hi) { v[s] = bf16_bits_to_float(g[flat + s]); mask |= 1 << s; }
+            else v[s] = 0.0f;
+        }
+        return mask;
+    }
+}
+
+__device__ __forceinline__ float load_one(const Layout& Lo, int m, int64_t i) {
+    const int64_t flat = (int64_t)m * Lo.d + i;
+    if (Lo.dtype == 0) return static_cast<const float*>(Lo.g)[flat];
+    return bf16_bits_to_float(static_cast<const uint16_t*>(Lo.g)[flat]);
+}
+
+// ---------------------------------------------------------------------------
+// Deterministic block reductions (fixed shuffle tree, fixed warp order).
+// ---------------------------------------------------------------------------
+template <typename T>
+__device__ __forceinline__ T warp_sum(T v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+    return v;
+}
+
+// Sum over the block; every thread receives the result.  `sh` holds >= 33 T.
+template <typename T>
+__device__ __forceinline__ T block_sum(T v, T* sh) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+    v = warp_sum(v);
+    __syncthreads();
+    if (lane == 0) sh[warp] = v;
+    __syncthreads();
+    if (warp == 0) {
+        T t = lane < nw ? sh[lane] : T(0);
+        t = warp_sum(t);
+        if (lane == 0) sh[32] = t;
+    }
+    __syncthreads();
+    return sh[32];
+}
+
+// Smallest positive fp32 a with fl64(lam * a) >= 1; +inf when no finite
+// float qualifies (lam = 0 or lam * FLT_MAX < 1).  fl64(lam * a) is
+// monotone in a, so "fl64(lam*|g|) >= 1" is exactly "|g| >= a_cap".
+__device__ __forceinline__ float cap_threshold(double lam) {
+    if (!(lam > 0.0)) return __int_as_float(0x7F800000);
+    if (lam * 3.4028234663852886e38 < 1.0) return __int_as_float(0x7F800000);
+    uint32_t lo = 0, hi = 0x7F7FFFFFu;   // search the bit patterns of finite positive floats
+    while (lo < hi) {
+        uint32_t mid = lo + ((hi - lo) >> 1);
+        if (lam * (double)__uint_as_float(mid) >= 1.0) hi = mid; else lo = mid + 1;
+    }
+    return __uint_as_float(lo);
+}
+
+}  // namespace gs

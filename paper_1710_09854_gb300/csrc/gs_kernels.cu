@@ -1,0 +1,765 @@
+// gs_kernels.cu -- CUDA kernels (sm_103a) of the gradient-sparsification
+// path, Wangni et al., arXiv:1710.09854.
+//
+// One call over M worker gradients runs:
+//   k_bound    per segment: a stratified sample of |g| and Algorithm 3 run to
+//              its fixed point on the sample give an upper bound lam_up on
+//              the final lambda (a search bound only; correctness never
+//              depends on it, see k_solve).
+//   k_stream   ONE pass over g (section 3.2, Algorithm 3 step 3 needs
+//              sum |g|): per chunk, the sum of |g| outside the capped-candidate
+//              set C = {|g| >= t_c}, the values in C, and the ordered list P of
+//              coordinates whose Philox word could fall below p_i for any
+//              lambda <= lam_up (index, value, word).
+//   k_solve    per segment: Algorithm 3 (steps 3-10) run exactly on
+//              (S_low, C): every coordinate that any lambda_j <= lam_up caps
+//              is in C, so K_j and the uncapped l1 mass are exact.  If the
+//              final lambda exceeds lam_up the segment falls back to an exact
+//              multi-pass solve over g and rebuilds its P lists.
+//   k_count / k_scan / k_write
+//              the Bernoulli draw Z_i = [u_i < p_i] (section 3) on the P
+//              lists, amplification to g_i / p_i, and compaction into
+//              ascending (idx, val) per worker.
+//   k_bucket / k_tiles
+//              the worker-order fp32 sum of the M sparse vectors (Algorithm 1,
+//              step 6).
+#include <cuda_runtime.h>
+
+#include <cfloat>
+#include <cmath>
+#include <algorithm>
+#include <cstdint>
+
+#include "gs_device.cuh"
+#include "gs_launch.h"
+#include "gs_trace.h"
+
+namespace gs {
+
+namespace {
+
+#define kInf __int_as_float(0x7F800000)
+
+__device__ __forceinline__ uint32_t mix32(uint32_t h) {
+    h ^= h >> 16;
+    h *= 0x85EBCA6Bu;
+    h ^= h >> 13;
+    h *= 0xC2B2AE35u;
+    h ^= h >> 16;
+    return h;
+}
+
+// ---------------------------------------------------------------------------
+// Block-ordered append helper: per-thread counts for the kGroupsPerThread
+// sub-steps of one step (byte j of `packed` = count of sub-step j), returns
+// the offset of each sub-step's first entry of this thread relative to
+// `run`, and advances `run` by the block's total.  Order: sub-step, thread.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void ordered_offsets(uint32_t packed, uint32_t (*sh)[kWarps], int& buf, int& run,
+                                                int off[kGroupsPerThread]) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    uint32_t inc = packed;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t t = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+        if (lane >= o) inc += t;
+    }
+    const uint32_t excl = inc - packed;
+    if (lane == 31) sh[buf][warp] = inc;
+    __syncthreads();
+    int total = 0;
+#pragma unroll
+    for (int j = 0; j < kGroupsPerThread; ++j) {
+        int before = 0, cta = 0;
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) {
+            const int b = (int)((sh[buf][w] >> (8 * j)) & 0xFFu);
+            cta += b;
+            before += (w < warp) ? b : 0;
+        }
+        off[j] = run + total + before + (int)((excl >> (8 * j)) & 0xFFu);
+        total += cta;
+    }
+    run += total;
+    buf ^= 1;
+}
+
+// ---------------------------------------------------------------------------
+// Candidate lists of one chunk, built by the whole CTA (kThreads threads).
+//   P: 1 + (x >> 9) 2^-23 < fl32(lam_up32 |g| + 1 + 2^-20).  Since
+//      (x >> 9) 2^-23 <= u = x 2^-32, every coordinate kept under a lambda
+//      <= lam_up (u < min(lambda |g|, 1)) passes; the 2^-20 slack covers the
+//      fp32 rounding of the right-hand side.
+//   C: !(|g| < t_c) (NaN and Inf land here, so the l1 sum flags them).
+//   s_low: sum of |g| outside C; fp32 pairwise over 16 values, fp64 above.
+// Lists are written in ascending coordinate order.
+// ---------------------------------------------------------------------------
+template <bool kWithC>
+__device__ void chunk_candidates(const Layout& Lo, int c, const Chunk& ch, float lam_up32, float t_c, const Lists& Ls,
+                                 bool build_p) {
+    __shared__ uint32_t shP[2][kWarps];
+    __shared__ uint32_t shC[2][kWarps];
+    __shared__ double shd[33];
+    const int tid = threadIdx.x;
+    const int64_t q0 = ch.lo >> 2, q1 = (ch.hi + 3) >> 2;
+    const int64_t region = (int64_t)ch.m * Lo.d + ch.lo;
+    const uint32_t worker = Lo.worker0 + (uint32_t)ch.m;
+    const float pbias = 1.0f + 0x1p-20f;
+    double acc = 0.0;
+    int runP = 0, runC = 0, bufP = 0, bufC = 0;
+
+    for (int64_t qb = q0; qb < q1; qb += (int64_t)kThreads * kGroupsPerThread) {
+        float v[kGroupsPerThread][4];
+        uint4 w[kGroupsPerThread];
+        uint32_t pm = 0, cm = 0;
+        float s4[kGroupsPerThread];
+#pragma unroll
+        for (int j = 0; j < kGroupsPerThread; ++j) {
+            const int64_t q = qb + (int64_t)j * kThreads + tid;
+            int valid = 0;
+            if (q < q1) {
+                valid = load_group(Lo, ch.m, q, ch.lo, ch.hi, v[j]);
+            } else {
+                v[j][0] = v[j][1] = v[j][2] = v[j][3] = 0.0f;
+            }
+            float m4[4];
+            bool need = false;
+#pragma unroll
+            for (int s = 0; s < 4; ++s) {
+                const float a = fabsf(v[j][s]);
+                const bool vs = (valid >> s) & 1;
+                const bool in_c = vs && !(a < t_c);
+                m4[s] = (vs && !in_c) ? a : 0.0f;
+                if (in_c) cm |= 1u << (4 * j + s);
+                need = need || (vs && a > 0.0f);
+            }
+            s4[j] = (m4[0] + m4[1]) + (m4[2] + m4[3]);
+            w[j] = make_uint4(0, 0, 0, 0);
+            if (build_p && need) {
+                w[j] = group_words(Lo.seed, Lo.step, worker, q);
+#pragma unroll
+                for (int s = 0; s < 4; ++s) {
+                    const float a = fabsf(v[j][s]);
+                    const bool vs = (valid >> s) & 1;
+                    if (vs && unit_plus_one(word_of(w[j], s)) < fmaf(lam_up32, a, pbias)) pm |= 1u << (4 * j + s);
+                }
+            }
+        }
+        acc += (double)((s4[0] + s4[1]) + (s4[2] + s4[3]));
+
+        if (build_p) {
+            uint32_t packed = 0;
+#pragma unroll
+            for (int j = 0; j < kGroupsPerThread; ++j) packed |= (uint32_t)__popc((pm >> (4 * j)) & 0xFu) << (8 * j);
+            int off[kGroupsPerThread];
+            ordered_offsets(packed, shP, bufP, runP, off);
+#pragma unroll
+            for (int j = 0; j < kGroupsPerThread; ++j) {
+                uint32_t bits = (pm >> (4 * j)) & 0xFu;
+                int k = 0;
+                const int64_t q = qb + (int64_t)j * kThreads + tid;
+                while (bits) {
+                    const int s = __ffs(bits) - 1;
+                    bits &= bits - 1;
+                    const int64_t e = region + off[j] + k;
+                    Ls.p_idx[e] = (int32_t)(q * 4 + s);
+                    Ls.p_g[e] = v[j][s];
+                    Ls.p_x[e] = word_of(w[j], s);
+                    ++k;
+                }
+            }
+        }
+        if (kWithC) {
+            uint32_t packed = 0;
+#pragma unroll
+            for (int j = 0; j < kGroupsPerThread; ++j) packed |= (uint32_t)__popc((cm >> (4 * j)) & 0xFu) << (8 * j);
+            int off[kGroupsPerThread];
+            ordered_offsets(packed, shC, bufC, runC, off);
+#pragma unroll
+            for (int j = 0; j < kGroupsPerThread; ++j) {
+                uint32_t bits = (cm >> (4 * j)) & 0xFu;
+                int k = 0;
+                while (bits) {
+                    const int s = __ffs(bits) - 1;
+                    bits &= bits - 1;
+                    Ls.c_val[region + off[j] + k] = fabsf(v[j][s]);
+                    ++k;
+                }
+            }
+        }
+    }
+    const double tot = block_sum(acc, shd);
+    if (tid == 0) {
+        if (build_p) Ls.p_cnt[c] = runP;
+        if (kWithC) {
+            Ls.c_cnt[c] = runC;
+            Ls.s_low[c] = tot;
+        }
+    }
+    __syncthreads();
+}
+
+// Sums over one segment of one worker row, by one CTA: K = #{|g| >= acap},
+// su = sum of the other |g| (NaN / Inf propagate into su when acap is NaN).
+__device__ void segment_stats(const Layout& Lo, int m, int64_t lo, int64_t hi, float acap, double& K, double& su,
+                              double* shd) {
+    const int64_t q0 = lo >> 2, q1 = (hi + 3) >> 2;
+    double acc = 0.0, cnt = 0.0;
+    for (int64_t qb = q0; qb < q1; qb += (int64_t)kThreads * kGroupsPerThread) {
+        float s4[kGroupsPerThread];
+        int k = 0;
+#pragma unroll
+        for (int j = 0; j < kGroupsPerThread; ++j) {
+            const int64_t q = qb + (int64_t)j * kThreads + threadIdx.x;
+            float v[4] = {0.f, 0.f, 0.f, 0.f};
+            int valid = 0;
+            if (q < q1) valid = load_group(Lo, m, q, lo, hi, v);
+            float m4[4];
+#pragma unroll
+            for (int s = 0; s < 4; ++s) {
+                const float a = fabsf(v[s]);
+                const bool vs = (valid >> s) & 1;
+                const bool capped = vs && (a >= acap);
+                k += capped ? 1 : 0;
+                m4[s] = (vs && !capped) ? a : 0.0f;
+            }
+            s4[j] = (m4[0] + m4[1]) + (m4[2] + m4[3]);
+        }
+        acc += (double)((s4[0] + s4[1]) + (s4[2] + s4[3]));
+        cnt += (double)k;
+    }
+    su = block_sum(acc, shd);
+    K = block_sum(cnt, shd);
+}
+
+// ---------------------------------------------------------------------------
+// k_bound: one CTA per segment.
+// ---------------------------------------------------------------------------
+constexpr int kBoundThreads = 512;
+constexpr double kBoundZ = 5.0;
+
+__global__ void __launch_bounds__(kBoundThreads) k_bound(Layout Lo, SegParam* sp, double kappa, int ns,
+                                                         int force_exact) {
+    extern __shared__ float sa[];
+    __shared__ double shd[33];
+    __shared__ float s_acap;
+    const int s = blockIdx.x, tid = threadIdx.x;
+    int m, l, c0, c1;
+    int64_t lo, hi;
+    seg_range(Lo, s, m, l, lo, hi, c0, c1);
+    const int64_t len = hi - lo;
+    SegParam& P = sp[s];
+    if (len <= ns || force_exact) {
+        // Short segment (or exact mode): every coordinate is a candidate.
+        if (tid == 0) {
+            P.lam_up = (double)kInf;
+            P.lam_up32 = kInf;
+            P.t_c = 0.0f;
+            P.flags = kSegTakeAll;
+        }
+        return;
+    }
+    for (int k = tid; k < ns; k += blockDim.x) {
+        const int64_t a = lo + (int64_t)k * len / ns;
+        const int64_t b = lo + (int64_t)(k + 1) * len / ns;
+        const uint32_t h = mix32((uint32_t)k * 0x9E3779B9u ^ mix32((uint32_t)s + 0x68E31DA4u));
+        const int64_t pos = a + (int64_t)(h % (uint32_t)(b - a));
+        float x = fabsf(load_one(Lo, m, pos));
+        if (!(x < kInf)) x = 0.0f;  // non-finite values are reported by the solve
+        sa[k] = x;
+    }
+    __syncthreads();
+    float ls = 0.0f;
+    for (int k = tid; k < ns; k += blockDim.x) ls += sa[k];
+    const double S = block_sum((double)ls, shd);
+    const double budget = kappa * (double)ns;
+    double lam = S > 0.0 ? budget / S : 0.0;
+    double K = 0.0, Su = S;
+    bool take_all = !(S > 0.0);
+    for (int it = 0; it < 64 && !take_all; ++it) {
+        if (tid == 0) s_acap = cap_threshold(lam);
+        __syncthreads();
+        const float acap = s_acap;
+        float su = 0.0f;
+        int kc = 0;
+        for (int k = tid; k < ns; k += blockDim.x) {
+            const float x = sa[k];
+            if (x >= acap) ++kc; else su += x;
+        }
+        K = block_sum((double)kc, shd);
+        Su = block_sum((double)su, shd);
+        if (!(Su > 0.0)) { take_all = true; break; }
+        const double c = (budget - K) / (lam * Su);
+        if (!(c > 1.0)) break;
+        lam *= c;
+    }
+    if (tid == 0) {
+        double e = take_all ? 0.0 : lam * Su / budget;  // uncapped share of the budget
+        if (take_all || K >= budget || !(lam > 0.0)) {
+            P.lam_up = (double)kInf;
+            P.lam_up32 = kInf;
+            P.t_c = 0.0f;
+            P.flags = kSegTakeAll;
+        } else {
+            double margin = 1.0 + kBoundZ / sqrt(kappa * (double)ns) / fmax(e, 1.0 / 16.0);
+            margin = fmin(margin, 64.0);
+            const double up = lam * margin;
+            P.lam_up = up;
+            P.lam_up32 = __double2float_ru(up);
+            const double t = (1.0 / up) * (1.0 - 0x1p-20);
+            P.t_c = t > 3.4028234663852886e38 ? 3.4028234663852886e38f : __double2float_rd(t);
+            P.flags = 0;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// k_stream: the single pass over g.
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads) k_stream(Layout Lo, const SegParam* __restrict__ sp, Lists Ls,
+                                                     int n_chunks, int build_p) {
+    for (int c = blockIdx.x; c < n_chunks; c += gridDim.x) {
+        const Chunk ch = decode_chunk(Lo, c);
+        chunk_candidates<true>(Lo, c, ch, sp[ch.seg].lam_up32, sp[ch.seg].t_c, Ls, build_p != 0);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// k_solve: one CTA per segment.  Algorithm 3 in the lambda form of
+// Proposition 1: lambda_0 = kappa d / S (step 3); K = #{fl64(lambda |g|) >= 1}
+// (capped, outside the active set of step 5); A = lambda * (uncapped l1 mass)
+// = sum_{i in I} p_i; c = (kappa d - K) / A (step 6); stop if c <= 1 (step 7);
+// lambda <- c lambda (step 8).
+// ---------------------------------------------------------------------------
+__device__ void c_stats(const Lists& Ls, int c0, int c1, const Layout& Lo, float acap, double& K, double& su,
+                        double* shd) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    double acc = 0.0, cnt = 0.0;
+    for (int c = c0 + warp; c < c1; c += kWarps) {
+        const Chunk ch = decode_chunk(Lo, c);
+        const int64_t region = (int64_t)ch.m * Lo.d + ch.lo;
+        const int n = Ls.c_cnt[c];
+        float part = 0.0f;
+        int k = 0, run = 0;
+        for (int e = lane; e < n; e += 32) {
+            const float a = Ls.c_val[region + e];
+            if (a >= acap) ++k; else part += a;
+            if (++run == 16) { acc += (double)part; part = 0.0f; run = 0; }
+        }
+        acc += (double)part;
+        cnt += (double)k;
+    }
+    su = block_sum(acc, shd);
+    K = block_sum(cnt, shd);
+}
+
+__global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lists Ls, double kappa, int iters,
+                                                    int force_exact, int* status, gs_info_dev* info) {
+    __shared__ double shd[33];
+    __shared__ float s_acap;
+    const int s = blockIdx.x, tid = threadIdx.x;
+    int m, l, c0, c1;
+    int64_t lo, hi;
+    seg_range(Lo, s, m, l, lo, hi, c0, c1);
+    const int64_t len = hi - lo;
+    const double budget = kappa * (double)len;
+    const double lam_up = sp[s].lam_up;
+    int flags = sp[s].flags & kSegTakeAll;
+
+    // l1 mass outside C (fixed order) and inside C.
+    double sl = 0.0;
+    for (int c = c0 + tid; c < c1; c += kThreads) sl += Ls.s_low[c];
+    const double S_low = block_sum(sl, shd);
+    double Kc, Sc;
+    c_stats(Ls, c0, c1, Lo, __int_as_float(0x7FC00000), Kc, Sc, shd);  // NaN threshold: all of C summed
+    double S = S_low + Sc;
+
+    double lam = 0.0, K = 0.0, Su = 0.0;
+    int j = 0;
+    bool exact = force_exact != 0;
+    if (!isfinite(S)) {
+        flags |= kSegNonfinite;
+        if (tid == 0) atomicOr(status, kStNonfinite);
+    } else if (!exact && S > 0.0) {
+        lam = budget / S;
+        while (j < iters) {
+            if (tid == 0) s_acap = cap_threshold(lam);
+            __syncthreads();
+            double suc;
+            c_stats(Ls, c0, c1, Lo, s_acap, K, suc, shd);
+            const double A = lam * (S_low + suc);
+            if (A == 0.0) break;
+            const double cc = (budget - K) / A;
+            if (!(cc > 1.0)) break;
+            lam = cc * lam;
+            ++j;
+        }
+        if (tid == 0) s_acap = cap_threshold(lam);
+        __syncthreads();
+        double suc;
+        c_stats(Ls, c0, c1, Lo, s_acap, K, suc, shd);
+        Su = S_low + suc;
+        // The lists are exact only while lambda stays within the bound.
+        if (lam > lam_up) exact = true;
+    }
+
+    if (exact && isfinite(S)) {
+        // Exact fallback: every sum straight from g, by this CTA.
+        flags |= kSegExact;
+        double k0;
+        segment_stats(Lo, m, lo, hi, __int_as_float(0x7FC00000), k0, S, shd);
+        lam = S > 0.0 ? budget / S : 0.0;
+        j = 0;
+        K = 0.0;
+        Su = S;
+        if (lam > 0.0) {
+            while (j < iters) {
+                if (tid == 0) s_acap = cap_threshold(lam);
+                __syncthreads();
+                segment_stats(Lo, m, lo, hi, s_acap, K, Su, shd);
+                const double A = lam * Su;
+                if (A == 0.0) break;
+                const double cc = (budget - K) / A;
+                if (!(cc > 1.0)) break;
+                lam = cc * lam;
+                ++j;
+            }
+            if (tid == 0) s_acap = cap_threshold(lam);
+            __syncthreads();
+            segment_stats(Lo, m, lo, hi, s_acap, K, Su, shd);
+        }
+        // Rebuild this segment's P lists for the final lambda (sparsify calls only).
+        const float up32 = lam > 0.0 ? __double2float_ru(lam) : 0.0f;
+        for (int c = c0; Ls.p_idx != nullptr && c < c1; ++c) {
+            const Chunk ch = decode_chunk(Lo, c);
+            chunk_candidates<false>(Lo, c, ch, up32, 0.0f, Ls, true);
+        }
+    }
+
+    if (tid == 0) {
+        SegParam& P = sp[s];
+        P.lam = lam;
+        P.lam32 = (float)lam;
+        P.a_cap = cap_threshold(lam);
+        P.inv_lam32 = lam > 0.0 ? (float)(1.0 / lam) : 0.0f;
+        P.l1 = S;
+        P.capped = (long long)K;
+        P.sum_p = lam > 0.0 ? K + lam * Su : 0.0;
+        P.iters_run = j;
+        P.flags = flags;
+        if (info) {
+            info[s].lambda = lam;
+            info[s].sum_p = P.sum_p;
+            info[s].capped = (int64_t)K;
+            info[s].iters_run = j;
+            info[s].flags = (flags & kSegExact) ? 1 : 0;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Decision for one candidate: Z_i = [u_i < p_i] with p_i = min(fl64(lam |g_i|), 1)
+// and u_i = x 2^-32 (section 3).  fp32 decides whenever u is more than 2^-20
+// (relative) away from p; closer calls are settled in fp64.  Kept values
+// are g_i / p_i: g_i itself when capped, else sign(g_i) / lambda (the
+// constant-value form of section 5.3).
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ bool decide(float gv, uint32_t x, const SegParam& P, float& val) {
+    const float a = fabsf(gv);
+    if (a >= P.a_cap) {
+        val = gv;
+        return true;
+    }
+    const float p32 = P.lam32 * a;
+    const float u32 = __uint2float_rn(x) * 0x1p-32f;
+    bool keep;
+    if (u32 < p32 * (1.0f - 0x1p-20f)) keep = true;
+    else if (u32 > p32 * (1.0f + 0x1p-20f)) keep = false;
+    else keep = (double)x * 0x1p-32 < P.lam * (double)a;
+    val = copysignf(P.inv_lam32, gv);
+    return keep;
+}
+
+__global__ void __launch_bounds__(kThreads) k_count(Layout Lo, const SegParam* __restrict__ sp, Lists Ls,
+                                                    int n_chunks) {
+    __shared__ double shd[33];
+    for (int c = blockIdx.x; c < n_chunks; c += gridDim.x) {
+        const Chunk ch = decode_chunk(Lo, c);
+        const SegParam P = sp[ch.seg];
+        const int64_t region = (int64_t)ch.m * Lo.d + ch.lo;
+        const int n = Ls.p_cnt[c];
+        int k = 0;
+        for (int e = threadIdx.x; e < n; e += kThreads) {
+            float v;
+            k += decide(Ls.p_g[region + e], Ls.p_x[region + e], P, v) ? 1 : 0;
+        }
+        const double tot = block_sum((double)k, shd);
+        if (threadIdx.x == 0) Ls.k_cnt[c] = (int32_t)tot;
+    }
+}
+
+// One CTA per worker: exclusive scan of the kept counts over its chunks.
+__global__ void __launch_bounds__(kThreads) k_scan(Layout Lo, Lists Ls, int32_t* nnz, int64_t cap, int* status) {
+    __shared__ int sh[kWarps];
+    const int m = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int c0 = m * Lo.cpw, c1 = c0 + Lo.cpw;
+    long long run = 0;
+    for (int b = c0; b < c1; b += kThreads) {
+        const int c = b + threadIdx.x;
+        const int v = c < c1 ? Ls.k_cnt[c] : 0;
+        int inc = v;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int t = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+            if (lane >= o) inc += t;
+        }
+        if (lane == 31) sh[warp] = inc;
+        __syncthreads();
+        int before = 0, tot = 0;
+        for (int w = 0; w < kWarps; ++w) {
+            before += w < warp ? sh[w] : 0;
+            tot += sh[w];
+        }
+        if (c < c1) Ls.k_off[c] = (int32_t)(run + before + inc - v);
+        run += tot;
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) {
+        nnz[m] = (int32_t)run;
+        if (run > cap) atomicOr(status, kStCapacity);
+    }
+}
+
+__global__ void __launch_bounds__(kThreads) k_write(Layout Lo, const SegParam* __restrict__ sp, Lists Ls,
+                                                    int n_chunks, int32_t* idx, float* val, int64_t cap) {
+    __shared__ int sh[2][kWarps];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    for (int c = blockIdx.x; c < n_chunks; c += gridDim.x) {
+        const Chunk ch = decode_chunk(Lo, c);
+        const SegParam P = sp[ch.seg];
+        const int64_t region = (int64_t)ch.m * Lo.d + ch.lo;
+        const int n = Ls.p_cnt[c];
+        const int64_t out0 = (int64_t)ch.m * cap;
+        long long run = Ls.k_off[c];
+        int buf = 0;
+        for (int b = 0; b < n; b += kThreads) {
+            const int e = b + threadIdx.x;
+            float v = 0.0f;
+            int32_t i = 0;
+            bool keep = false;
+            if (e < n) {
+                keep = decide(Ls.p_g[region + e], Ls.p_x[region + e], P, v);
+                i = Ls.p_idx[region + e];
+            }
+            const unsigned bal = __ballot_sync(0xFFFFFFFFu, keep);
+            if (lane == 0) sh[buf][warp] = __popc(bal);
+            __syncthreads();
+            int before = 0, tot = 0;
+            for (int w = 0; w < kWarps; ++w) {
+                before += w < warp ? sh[buf][w] : 0;
+                tot += sh[buf][w];
+            }
+            if (keep) {
+                const long long pos = run + before + __popc(bal & ((1u << lane) - 1u));
+                if (pos < cap) {
+                    idx[out0 + pos] = i;
+                    val[out0 + pos] = v;
+                }
+            }
+            run += tot;
+            buf ^= 1;
+        }
+        __syncthreads();
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Dense probabilities of one worker: p_i = min(lambda |g_i|, 1).
+// ---------------------------------------------------------------------------
+__global__ void k_prob(Layout Lo, const SegParam* __restrict__ sp, float* p) {
+    const SegParam P = sp[0];
+    const int64_t n = Lo.d;
+    for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
+        const float a = fabsf(load_one(Lo, 0, i));
+        p[i] = (a >= P.a_cap) ? 1.0f : P.lam32 * a;
+    }
+}
+
+// Random words of coordinates i0 .. i0 + n - 1 (one Philox call per thread per word).
+__global__ void k_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t i0, int64_t n, uint32_t* out) {
+    for (int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k < n; k += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t i = i0 + k;
+        out[k] = word_of(group_words(seed, step, worker, i >> 2), (int)(i & 3));
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Sparse sum.  k_bucket finds, for every worker list and output tile, the
+// first entry at or after the tile (validating order and range); k_tiles
+// accumulates each tile in shared memory worker by worker, in order.
+// ---------------------------------------------------------------------------
+__global__ void k_bucket(AggArgs A, int32_t* off, int nt, int* status) {
+    const int m = blockIdx.y;
+    const int32_t* __restrict__ idx = A.idx[m];
+    long long n = A.nnz[m];
+    if (n > A.cap) n = A.cap;
+    if (n < 0) n = 0;
+    int32_t* o = off + (int64_t)m * (nt + 1);
+    for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e <= n;
+         e += (long long)gridDim.x * blockDim.x) {
+        long long t_cur = nt;
+        if (e < n) {
+            const int32_t i = idx[e];
+            if (i < 0 || (int64_t)i >= A.d) {
+                atomicOr(status, kStInvalid);
+                continue;
+            }
+            t_cur = i / kAggTile;
+        }
+        long long t_prev = -1;
+        if (e > 0) {
+            const int32_t ip = idx[e - 1];
+            if (ip < 0 || (int64_t)ip >= A.d) continue;
+            if (e < n && ip >= idx[e]) {
+                atomicOr(status, kStInvalid);
+                continue;
+            }
+            t_prev = ip / kAggTile;
+        }
+        for (long long t = t_prev + 1; t <= t_cur; ++t) o[t] = (int32_t)e;
+    }
+}
+
+__global__ void __launch_bounds__(kThreads) k_tiles(AggArgs A, const int32_t* __restrict__ off, int nt, float* out) {
+    __shared__ float acc[kAggTile];
+    for (int t = blockIdx.x; t < nt; t += gridDim.x) {
+        const int64_t base = (int64_t)t * kAggTile;
+        const int len = (int)min((int64_t)kAggTile, A.d - base);
+        for (int k = threadIdx.x; k < kAggTile; k += kThreads) acc[k] = 0.0f;
+        __syncthreads();
+        for (int m = 0; m < A.M; ++m) {
+            long long n = A.nnz[m];
+            if (n > A.cap) n = A.cap;
+            if (n < 0) n = 0;
+            const int32_t* o = off + (int64_t)m * (nt + 1);
+            long long lo = o[t], hi = o[t + 1];
+            lo = lo < 0 ? 0 : (lo > n ? n : lo);
+            hi = hi < lo ? lo : (hi > n ? n : hi);
+            const int32_t* __restrict__ idx = A.idx[m];
+            const float* __restrict__ val = A.val[m];
+            for (long long e = lo + threadIdx.x; e < hi; e += kThreads) {
+                const int64_t i = (int64_t)idx[e] - base;
+                if (i >= 0 && i < len) acc[i] += val[e];
+            }
+            __syncthreads();
+        }
+        float* dst = out + base;
+        if (len == kAggTile && (reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
+            for (int k = threadIdx.x; k < kAggTile / 4; k += kThreads)
+                reinterpret_cast<float4*>(dst)[k] = make_float4(acc[4 * k], acc[4 * k + 1], acc[4 * k + 2], acc[4 * k + 3]);
+        } else {
+            for (int k = threadIdx.x; k < len; k += kThreads) dst[k] = acc[k];
+        }
+        __syncthreads();
+    }
+}
+
+int sm_count() {
+    static int n = 0;
+    if (n == 0) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+        if (n <= 0) n = 1;
+    }
+    return n;
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// Host launchers
+// ---------------------------------------------------------------------------
+cudaError_t launch_bound(const Layout& Lo, SegParam* sp, int n_seg, double kappa, int ns, int force_exact,
+                         cudaStream_t st) {
+    const size_t smem = (size_t)ns * sizeof(float);
+    if (smem > 48 * 1024) {
+        cudaError_t e = cudaFuncSetAttribute(k_bound, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+    }
+    TraceScope ts(kKBound, st);
+    k_bound<<<n_seg, kBoundThreads, smem, st>>>(Lo, sp, kappa, ns, force_exact);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_stream(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, bool build_p,
+                          cudaStream_t st) {
+    const int grid = min(n_chunks, sm_count() * 8);
+    TraceScope ts(kKStream, st);
+    k_stream<<<grid, kThreads, 0, st>>>(Lo, sp, Ls, n_chunks, build_p ? 1 : 0);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_solve(const Layout& Lo, SegParam* sp, const Lists& Ls, int n_seg, double kappa, int iters,
+                         int force_exact, int* status, gs_info_dev* info, cudaStream_t st) {
+    TraceScope ts(kKSolve, st);
+    k_solve<<<n_seg, kThreads, 0, st>>>(Lo, sp, Ls, kappa, iters, force_exact, status, info);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, int32_t* idx,
+                           float* val, int32_t* nnz, int64_t cap, int* status, cudaStream_t st) {
+    const int grid = min(n_chunks, sm_count() * 8);
+    {
+        TraceScope ts(kKCount, st);
+        k_count<<<grid, kThreads, 0, st>>>(Lo, sp, Ls, n_chunks);
+    }
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    {
+        TraceScope ts(kKScan, st);
+        k_scan<<<Lo.M, kThreads, 0, st>>>(Lo, Ls, nnz, cap, status);
+    }
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    TraceScope ts(kKWrite, st);
+    k_write<<<grid, kThreads, 0, st>>>(Lo, sp, Ls, n_chunks, idx, val, cap);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_prob(const Layout& Lo, const SegParam* sp, float* p, cudaStream_t st) {
+    const int64_t blocks = std::min<int64_t>((Lo.d + 255) / 256, (int64_t)sm_count() * 16);
+    TraceScope ts(kKProb, st);
+    k_prob<<<(int)blocks, 256, 0, st>>>(Lo, sp, p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_aggregate(const AggArgs& A, int32_t* off, float* out, int* status, cudaStream_t st) {
+    const int nt = (int)((A.d + kAggTile - 1) / kAggTile);
+    // Bucket: enough blocks per worker to cover a full row of entries.
+    const int bx = (int)std::min<int64_t>((A.d + 255) / 256 + 1, 1024);
+    dim3 grid(bx, A.M);
+    {
+        TraceScope ts(kKBucket, st);
+        k_bucket<<<grid, 256, 0, st>>>(A, off, nt, status);
+    }
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const int tg = min(nt, sm_count() * 6);
+    TraceScope ts(kKTiles, st);
+    k_tiles<<<tg, kThreads, 0, st>>>(A, off, nt, out);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t i0, int64_t n, uint32_t* out,
+                         cudaStream_t st) {
+    const int64_t blocks = std::max<int64_t>(1, std::min<int64_t>((n + 255) / 256, (int64_t)sm_count() * 8));
+    TraceScope ts(kKWords, st);
+    k_words<<<(int)blocks, 256, 0, st>>>(seed, step, worker, i0, n, out);
+    return cudaGetLastError();
+}
+
+int agg_tiles(int64_t d) { return (int)((d + kAggTile - 1) / kAggTile); }
+int chunk_size() { return kChunk; }
+
+}  // namespace gs

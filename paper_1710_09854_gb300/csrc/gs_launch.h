@@ -1,0 +1,44 @@
+// gs_launch.h -- host-side launchers shared by the C ABI (gs_api.cu) and the
+// kernels (gs_kernels.cu).  Internal to libgs.so.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "gs.h"
+#include "gs_device.cuh"
+
+namespace gs {
+
+typedef gs_info gs_info_dev;
+
+// Largest M the sparse sum takes (its pointer tables travel as kernel
+// parameters: 2 x 512 x 8 bytes).
+constexpr int kMaxAggM = 512;
+
+struct AggArgs {
+    const int32_t* idx[kMaxAggM];
+    const float* val[kMaxAggM];
+    const int32_t* nnz;   // device, M
+    int M;
+    int64_t d;
+    int64_t cap;          // entries beyond cap in a list are never read
+};
+
+cudaError_t launch_bound(const Layout& Lo, SegParam* sp, int n_seg, double kappa, int ns, int force_exact,
+                         cudaStream_t st);
+cudaError_t launch_stream(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, bool build_p,
+                          cudaStream_t st);
+cudaError_t launch_solve(const Layout& Lo, SegParam* sp, const Lists& Ls, int n_seg, double kappa, int iters,
+                         int force_exact, int* status, gs_info_dev* info, cudaStream_t st);
+cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, int32_t* idx,
+                           float* val, int32_t* nnz, int64_t cap, int* status, cudaStream_t st);
+cudaError_t launch_prob(const Layout& Lo, const SegParam* sp, float* p, cudaStream_t st);
+cudaError_t launch_aggregate(const AggArgs& A, int32_t* off, float* out, int* status, cudaStream_t st);
+cudaError_t launch_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t i0, int64_t n, uint32_t* out,
+                         cudaStream_t st);
+int agg_tiles(int64_t d);
+int chunk_size();
+
+}  // namespace gs

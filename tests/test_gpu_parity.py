@@ -1,0 +1,371 @@
+"""GPU parity: the CUDA path through the C ABI against the CPU oracle, on the
+same seeded inputs, element by element (tolerances in tests/parity.py)."""
+import numpy as np
+import pytest
+
+import oracle
+import workloads
+from parity import compare_probabilities, compare_sparse, compare_sum
+
+pytestmark = pytest.mark.gpu
+
+SIZES = [1, 2, 3, 4, 5, 7, 31, 64, 1023, 4096, 4097, 16383, 16384, 16385, 50003, 65536, 200001]
+
+
+@pytest.fixture(scope="module")
+def gs():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_1710_09854_gb300 as gs
+    gs.gs_set_option(gs.GS_OPT_FORCE_EXACT_SOLVE, 0)
+    gs.gs_set_option(gs.GS_OPT_SAMPLE_SIZE, 16384)
+    assert gs.gs_sync_status() == gs.GS_OK
+    return gs
+
+
+def _dev(x):
+    import torch
+    return torch.from_numpy(np.ascontiguousarray(x)).cuda()
+
+
+def _vector(kind, d, seed):
+    rng = np.random.default_rng(seed)
+    if kind == "t3":
+        g = rng.standard_t(3, d)
+        g[rng.random(d) < 0.01] = 0
+    elif kind == "lognormal":
+        g = rng.lognormal(0, 2, d) * np.where(rng.random(d) < 0.5, -1, 1)
+        g[rng.random(d) < 0.001] *= 100
+    elif kind == "normal":
+        g = rng.standard_normal(d)
+    elif kind == "ties":
+        g = rng.integers(-3, 4, d).astype(np.float64)
+    else:
+        raise ValueError(kind)
+    return g.astype(np.float32)
+
+
+def _sparsify_batched(gs, g_host, kappa, iters, seed, step, worker0=0, dtype="f32", cap=None, info=False):
+    import torch
+    M, d = g_host.shape
+    cap = d if cap is None else cap
+    g = _dev(g_host)
+    if dtype == "bf16":
+        g = _dev(workloads.f32_to_bf16_bits(g_host).reshape(M, d)).view(torch.bfloat16)
+    idx = torch.full((M, cap), -1, dtype=torch.int32, device="cuda")
+    val = torch.zeros((M, cap), dtype=torch.float32, device="cuda")
+    nnz = torch.zeros(M, dtype=torch.int32, device="cuda")
+    inf = gs.info_tensor(M) if info else None
+    gs.gs_batched_sparsify(g, kappa, iters, seed, step, worker0, idx, val, nnz, info=inf)
+    return idx, val, nnz, inf
+
+
+# ---------------------------------------------------------------------------
+def test_random_words_match_oracle(gs):
+    import torch
+    for seed, step, worker, i0, n in [(1, 0, 0, 0, 4099), (2**40 + 3, 9, 15, 2**33 + 1, 1001),
+                                      (0xFFFFFFFFFFFFFFFF, 2**32 - 1, 2**32 - 1, 5, 77)]:
+        out = torch.empty(n, dtype=torch.int32, device="cuda")
+        gs.gs_random_words(seed, step, worker, i0, out)
+        got = out.cpu().numpy().view(np.uint32)
+        ref = (oracle.uniforms(seed, step, worker, i0, n) * 2.0**32).astype(np.uint64).astype(np.uint32)
+        np.testing.assert_array_equal(got, ref)
+
+
+@pytest.mark.parametrize("d", SIZES)
+def test_probabilities_sizes(gs, d):
+    import torch
+    for kind, kappa, iters in [("t3", 0.01, 3), ("lognormal", 0.1, 2), ("normal", 0.5, 0), ("ties", 0.05, 10)]:
+        g_host = _vector(kind, d, d * 7 + iters)
+        p = torch.empty(d, dtype=torch.float32, device="cuda")
+        info = gs.info_tensor(1)
+        gs.gs_probabilities_ex(_dev(g_host), kappa, iters, p, info)
+        assert gs.gs_sync_status() == gs.GS_OK
+        ref_info, _ = compare_probabilities(p.cpu().numpy(), g_host, kappa, iters)
+        got = gs.decode_info(info)[0]
+        if ref_info["lambda"] > 0:
+            assert got["lambda"] == pytest.approx(ref_info["lambda"], rel=1e-6)
+            assert got["sum_p"] == pytest.approx(ref_info["sum_p"], rel=1e-6)
+
+
+@pytest.mark.parametrize("d", SIZES)
+def test_sparsify_sizes(gs, d):
+    import torch
+    for kind, kappa, iters, seed, step, worker in [("t3", 0.01, 3, 1, 0, 0), ("lognormal", 0.1, 2, 99, 5, 3),
+                                                   ("normal", 0.3, 1, 2**35 + 1, 2**31, 2**32 - 2),
+                                                   ("ties", 0.5, 4, 7, 1, 1)]:
+        g_host = _vector(kind, d, d + step)
+        idx = torch.empty(d, dtype=torch.int32, device="cuda")
+        val = torch.empty(d, dtype=torch.float32, device="cuda")
+        nnz = torch.empty(1, dtype=torch.int32, device="cuda")
+        gs.gs_sparsify(_dev(g_host), kappa, iters, seed, step, worker, idx, val, nnz)
+        assert gs.gs_sync_status() == gs.GS_OK
+        n = int(nnz.item())
+        flips = compare_sparse(idx[:n].cpu().numpy(), val[:n].cpu().numpy(), g_host, kappa, iters, seed, step, worker)
+        assert flips <= 1
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_batched_parity(gs, dtype):
+    M, d, kappa, iters, seed, step, w0 = 5, 100_003, 0.02, 3, 11, 7, 3
+    g_host = np.stack([_vector(k, d, 50 + m) for m, k in enumerate(["t3", "lognormal", "normal", "t3", "ties"])])
+    if dtype == "bf16":
+        g_host = workloads.bf16_bits_to_f32(workloads.f32_to_bf16_bits(g_host)).reshape(M, d)
+    idx, val, nnz, inf = _sparsify_batched(gs, g_host, kappa, iters, seed, step, w0, dtype, info=True)
+    assert gs.gs_sync_status() == gs.GS_OK
+    n = nnz.cpu().numpy()
+    ii, vv = idx.cpu().numpy(), val.cpu().numpy()
+    infos = gs.decode_info(inf)
+    flips = 0
+    for m in range(M):
+        flips += compare_sparse(ii[m, :n[m]], vv[m, :n[m]], g_host[m], kappa, iters, seed, step, w0 + m)
+        ref = oracle.greedy_lambda(g_host[m], kappa, iters)
+        assert infos[m]["lambda"] == pytest.approx(ref["lambda"], rel=1e-6)
+        assert infos[m]["capped"] == ref["capped"]
+    assert flips <= 1
+
+
+def test_single_equals_batched_row(gs):
+    import torch
+    M, d = 3, 70_001
+    g_host = np.stack([_vector("lognormal", d, 900 + m) for m in range(M)])
+    idx, val, nnz, _ = _sparsify_batched(gs, g_host, 0.05, 2, 5, 3, worker0=10)
+    for m in range(M):
+        i1 = torch.empty(d, dtype=torch.int32, device="cuda")
+        v1 = torch.empty(d, dtype=torch.float32, device="cuda")
+        n1 = torch.empty(1, dtype=torch.int32, device="cuda")
+        gs.gs_sparsify(_dev(g_host[m]), 0.05, 2, 5, 3, 10 + m, i1, v1, n1)
+        k = int(nnz[m].item())
+        assert int(n1.item()) == k
+        assert torch.equal(i1[:k], idx[m, :k]) and torch.equal(v1[:k], val[m, :k])
+
+
+def test_deterministic(gs):
+    import torch
+    M, d = 4, 300_001
+    g_host = np.stack([_vector("t3", d, 77 + m) for m in range(M)])
+    a = _sparsify_batched(gs, g_host, 0.01, 3, 1, 0)
+    b = _sparsify_batched(gs, g_host, 0.01, 3, 1, 0)
+    assert torch.equal(a[2], b[2])
+    for m in range(M):
+        k = int(a[2][m].item())
+        assert torch.equal(a[0][m, :k], b[0][m, :k]) and torch.equal(a[1][m, :k], b[1][m, :k])
+
+
+def test_forced_exact_and_small_sample(gs):
+    M, d, kappa, iters = 3, 120_007, 0.03, 3
+    g_host = np.stack([_vector(k, d, 31 + m) for m, k in enumerate(["lognormal", "t3", "ties"])])
+    for opt, val in [(gs.GS_OPT_FORCE_EXACT_SOLVE, 1), (gs.GS_OPT_SAMPLE_SIZE, 256)]:
+        gs.gs_set_option(opt, val)
+        try:
+            idx, v, nnz, inf = _sparsify_batched(gs, g_host, kappa, iters, 3, 2, info=True)
+            assert gs.gs_sync_status() == gs.GS_OK
+        finally:
+            gs.gs_set_option(gs.GS_OPT_FORCE_EXACT_SOLVE, 0)
+            gs.gs_set_option(gs.GS_OPT_SAMPLE_SIZE, 16384)
+        n = nnz.cpu().numpy()
+        for m in range(M):
+            compare_sparse(idx[m, :n[m]].cpu().numpy(), v[m, :n[m]].cpu().numpy(), g_host[m], kappa, iters, 3, 2, m)
+        if opt == gs.GS_OPT_FORCE_EXACT_SOLVE:
+            assert all(r["flags"] & 1 for r in gs.decode_info(inf))
+
+
+def test_segmented_parity(gs):
+    import torch
+    rng = np.random.default_rng(4)
+    lens = [64, 3, 1, 17000, 5, 40000, 64, 16384, 2]
+    off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+    M, d = 3, int(off[-1])
+    g_host = np.stack([(rng.standard_normal(d) * rng.choice([1e-3, 1, 50], d)).astype(np.float32) for _ in range(M)])
+    kappa, iters, seed, step = 0.05, 2, 8, 4
+    g = _dev(g_host)
+    idx = torch.empty((M, d), dtype=torch.int32, device="cuda")
+    val = torch.empty((M, d), dtype=torch.float32, device="cuda")
+    nnz = torch.empty(M, dtype=torch.int32, device="cuda")
+    inf = gs.info_tensor(M * (off.size - 1))
+    gs.gs_segmented_sparsify(g, off, kappa, iters, seed, step, 0, idx, val, nnz, info=inf)
+    assert gs.gs_sync_status() == gs.GS_OK
+    infos = gs.decode_info(inf)
+    n = nnz.cpu().numpy()
+    for m in range(M):
+        ri, rv, lams = oracle.segmented_sparsify(g_host[m], off, kappa, iters, seed, step, m)
+        got_i, got_v = idx[m, :n[m]].cpu().numpy(), val[m, :n[m]].cpu().numpy()
+        # per segment comparison against the oracle's per-layer result
+        for l in range(off.size - 1):
+            a, b = off[l], off[l + 1]
+            sel = (got_i >= a) & (got_i < b)
+            r = oracle.sparsify(g_host[m, a:b], kappa, iters, seed, step, m, i0=a)
+            compare_sparse(got_i[sel], got_v[sel], g_host[m, a:b], kappa, iters, seed, step, m, i0=a, ref=r)
+            assert infos[m * (off.size - 1) + l]["lambda"] == pytest.approx(lams[l], rel=1e-6)
+
+
+def test_aggregate_parity_and_validation(gs):
+    import torch
+    rng = np.random.default_rng(3)
+    for M, d in [(1, 1), (3, 8191), (16, 100_000), (7, 3 * 8192 + 5)]:
+        il, vl = [], []
+        for m in range(M):
+            k = int(rng.integers(0, min(d, 5000) + 1))
+            il.append(np.sort(rng.choice(d, size=k, replace=False)).astype(np.int32))
+            vl.append((rng.standard_normal(k) * 10 ** rng.uniform(-3, 3, k)).astype(np.float32))
+        nnz = torch.tensor([x.size for x in il], dtype=torch.int32, device="cuda")
+        it = [_dev(x) if x.size else torch.zeros(1, dtype=torch.int32, device="cuda") for x in il]
+        vt = [_dev(x) if x.size else torch.zeros(1, dtype=torch.float32, device="cuda") for x in vl]
+        out = torch.full((d,), float("nan"), dtype=torch.float32, device="cuda")
+        gs.gs_sparse_aggregate(it, vt, nnz, d, out)
+        assert gs.gs_sync_status() == gs.GS_OK
+        ref = compare_sum(out.cpu().numpy(), il, vl, d)
+        np.testing.assert_array_equal(out.cpu().numpy(), ref)   # same fp32 adds in the same order
+    # unsorted and out-of-range lists are reported
+    for bad in (np.array([5, 3, 9], np.int32), np.array([1, 1, 2], np.int32), np.array([0, 10], np.int32)):
+        out = torch.zeros(10, dtype=torch.float32, device="cuda")
+        gs.gs_sparse_aggregate([_dev(bad)], [_dev(np.ones(bad.size, np.float32))],
+                               torch.tensor([bad.size], dtype=torch.int32, device="cuda"), 10, out)
+        assert gs.gs_sync_status() == gs.GS_ERR_INVALID_ARG
+
+
+def test_edge_cases(gs):
+    import torch
+    d = 40_000
+    # all zero: nothing kept
+    z = np.zeros((2, d), np.float32)
+    idx, val, nnz, inf = _sparsify_batched(gs, z, 0.1, 2, 1, 0, info=True)
+    assert gs.gs_sync_status() == gs.GS_OK and nnz.cpu().tolist() == [0, 0]
+    # kappa = 1 with enough iterations: every non-zero coordinate capped and kept as is
+    g = _vector("lognormal", d, 5)
+    g[::3] = 0
+    idx, val, nnz, _ = _sparsify_batched(gs, g[None], 1.0, 40, 1, 0)
+    k = int(nnz.item())
+    np.testing.assert_array_equal(idx[0, :k].cpu().numpy(), np.nonzero(g)[0])
+    np.testing.assert_array_equal(val[0, :k].cpu().numpy(), g[g != 0])
+    # equal magnitudes: p = kappa everywhere (uniform sampling)
+    e = np.where(np.arange(d) % 2 == 0, 2.0, -2.0).astype(np.float32)
+    p = torch.empty(d, dtype=torch.float32, device="cuda")
+    gs.gs_probabilities(_dev(e), 0.25, 3, p)
+    np.testing.assert_allclose(p.cpu().numpy(), 0.25, rtol=1e-6)
+    # one-hot
+    oh = np.zeros(d, np.float32)
+    oh[12345] = -3.0
+    gs.gs_probabilities(_dev(oh), 0.001, 2, p)
+    want = np.zeros(d)
+    want[12345] = 1
+    np.testing.assert_array_equal(p.cpu().numpy(), want)
+    # non-finite gradients are reported
+    for bad in (np.nan, np.inf, -np.inf):
+        b = _vector("normal", d, 1)
+        b[777] = bad
+        _sparsify_batched(gs, b[None], 0.1, 2, 1, 0)
+        assert gs.gs_sync_status() == gs.GS_ERR_NONFINITE
+    # capacity overflow: true count reported, writes clipped
+    g = _vector("normal", d, 2)
+    idx, val, nnz, _ = _sparsify_batched(gs, g[None], 0.5, 2, 1, 0, cap=100)
+    assert gs.gs_sync_status() == gs.GS_ERR_CAPACITY
+    assert int(nnz.item()) > 100
+    ri, rv, _ = oracle.sparsify(g, 0.5, 2, 1, 0, 0)
+    assert int(nnz.item()) == ri.size
+    np.testing.assert_array_equal(idx[0].cpu().numpy(), ri[:100])
+
+
+def test_pipeline_host_matches_device_path(gs):
+    import torch
+    M, d, kappa, iters, seed, step = 4, 65_537, 0.05, 2, 3, 1
+    g_host = np.stack([_vector("t3", d, 10 + m) for m in range(M)])
+    gh = torch.from_numpy(g_host).pin_memory()
+    g_dev = torch.empty((M, d), dtype=torch.float32, device="cuda")
+    idx = torch.empty((M, d), dtype=torch.int32, device="cuda")
+    val = torch.empty((M, d), dtype=torch.float32, device="cuda")
+    nnz = torch.empty(M, dtype=torch.int32, device="cuda")
+    out = torch.empty(d, dtype=torch.float32, device="cuda")
+    out_h = torch.empty(d, dtype=torch.float32).pin_memory()
+    nnz_h = torch.empty(M, dtype=torch.int32).pin_memory()
+    gs.gs_pipeline_host(gh, kappa, iters, seed, step, 0, g_dev, idx, val, nnz, out, out_h, nnz_h)
+    torch.cuda.synchronize()
+    assert gs.gs_sync_status() == gs.GS_OK
+    il, vl = [], []
+    for m in range(M):
+        ri, rv, _ = oracle.sparsify(g_host[m], kappa, iters, seed, step, m)
+        il.append(ri)
+        vl.append(rv)
+        assert nnz_h[m].item() == ri.size
+    compare_sum(out_h.numpy(), il, vl, d)
+
+
+# ---------------------------------------------------------------------------
+# Full-size workloads in the launch configuration bench.py times.
+# ---------------------------------------------------------------------------
+def _full_check(gs, g_dev, kappa, iters, seed=1, step=0, workers=None, offsets=None, dtype="f32"):
+    import torch
+    M, d = g_dev.shape
+    idx = torch.empty((M, d), dtype=torch.int32, device="cuda")
+    val = torch.empty((M, d), dtype=torch.float32, device="cuda")
+    nnz = torch.empty(M, dtype=torch.int32, device="cuda")
+    out = torch.empty(d, dtype=torch.float32, device="cuda")
+    if offsets is None:
+        gs.gs_batched_sparsify(g_dev, kappa, iters, seed, step, 0, idx, val, nnz)
+    else:
+        gs.gs_segmented_sparsify(g_dev, offsets, kappa, iters, seed, step, 0, idx, val, nnz)
+    gs.gs_sparse_aggregate([idx[m] for m in range(M)], [val[m] for m in range(M)], nnz, d, out)
+    assert gs.gs_sync_status() == gs.GS_OK
+    g_host = g_dev.float().cpu().numpy() if dtype == "bf16" else g_dev.cpu().numpy()
+    n = nnz.cpu().numpy()
+    workers = range(M) if workers is None else workers
+    il, vl = [], []
+    flips = 0
+    for m in range(M):
+        if offsets is None:
+            ref = oracle.sparsify(g_host[m], kappa, iters, seed, step, m)
+        else:
+            ri, rv, _ = oracle.segmented_sparsify(g_host[m], offsets, kappa, iters, seed, step, m)
+            ref = (ri, rv, {"lambda": float("nan")})
+        il.append(ref[0])
+        vl.append(ref[1])
+        if m in workers:
+            gi = idx[m, :n[m]].cpu().numpy()
+            gv = val[m, :n[m]].cpu().numpy()
+            if offsets is None:
+                flips += compare_sparse(gi, gv, g_host[m], kappa, iters, seed, step, m, ref=ref)
+            else:
+                np.testing.assert_array_equal(gi, ref[0])
+                np.testing.assert_allclose(gv, ref[1], rtol=1e-5)
+    compare_sum(out.cpu().numpy(), il, vl, d)
+    return flips
+
+
+def test_full_student_t_d2p24_m16(gs):
+    """The headline workload (M=16, d=2^24, kappa=0.01, 3 iterations)."""
+    import torch
+    w = workloads.C3
+    g = workloads.device_student_t(w.M, w.d, seed0=w.data_seed)
+    flips = _full_check(gs, g, w.kappa, w.iters, w.seed, w.step)
+    assert flips <= 2
+    del g
+    torch.cuda.empty_cache()
+
+
+def test_full_resnet50_layerwise(gs):
+    import torch
+    g, off = workloads.device_layerwise(2)
+    _full_check(gs, g, workloads.C4.kappa, workloads.C4.iters, offsets=off)
+    del g
+    torch.cuda.empty_cache()
+
+
+def test_full_logreg_c2(gs):
+    import torch
+    g = workloads.device_logreg(8, 1 << 20)
+    _full_check(gs, g, workloads.C2.kappa, workloads.C2.iters, workers=[0, 7])
+    del g
+    torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("kappa", [0.001, 0.01, 0.1])
+def test_lognormal_outliers_bf16_and_f32(gs, kappa):
+    import torch
+    g = workloads.device_lognormal(2, 1 << 23, seed0=5)
+    _full_check(gs, g, kappa, 3, workers=[0, 1])
+    _full_check(gs, g.to(torch.bfloat16), kappa, 3, workers=[1], dtype="bf16")
+    del g
+    torch.cuda.empty_cache()
