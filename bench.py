@@ -254,7 +254,8 @@ def run_gpu(args):
     # Algorithmic bytes of the dominant kernel per launch.
     kernel_bytes = {
         "k_stream": M * d * esz,                 # one read of g
-        "k_write": nnz_total * 8,                # the (idx, val) codes written
+        "k_stream_tma": M * d * esz,             # one read of g
+        "k_emit": nnz_total * 8,                 # the (idx, val) codes written
         "k_tiles": nnz_total * 8 + d * 4,        # codes read, dense sum written
         "k_count": 0,
     }

@@ -175,10 +175,20 @@ gs_status gs_random_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t
  *   GS_OPT_FORCE_EXACT_SOLVE  1: skip the sampled bound and use the exact
  *                              fallback solve for every worker (slow).
  *   GS_OPT_SAMPLE_SIZE        sampled coordinates per segment for the bound
- *                              on lambda (default 16384, >= 256).
+ *                              on lambda (default 16384, 256 .. 32768).
+ *   GS_OPT_KERNEL_TIMING      1: time every kernel launch (gs_kernel_times).
+ *   GS_OPT_STREAM_PATH        streaming pass over g: 0 automatic (the TMA
+ *                              kernel whenever the layout allows it), 1 the
+ *                              generic-load kernel, 2 the TMA kernel where
+ *                              eligible.
  * Options are process-wide; returns GS_ERR_INVALID_ARG for an unknown
  * option or value. */
-typedef enum { GS_OPT_FORCE_EXACT_SOLVE = 1, GS_OPT_SAMPLE_SIZE = 2, GS_OPT_KERNEL_TIMING = 3 } gs_option;
+typedef enum {
+    GS_OPT_FORCE_EXACT_SOLVE = 1,
+    GS_OPT_SAMPLE_SIZE = 2,
+    GS_OPT_KERNEL_TIMING = 3,
+    GS_OPT_STREAM_PATH = 4
+} gs_option;
 gs_status gs_set_option(int option, int64_t value);
 
 /* Tracing.  The library counts every kernel it launches; with

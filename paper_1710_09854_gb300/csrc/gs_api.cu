@@ -38,6 +38,7 @@ std::mutex g_mu;
 DevState g_dev[kMaxDevices];
 int g_force_exact = 0;
 int g_sample = 16384;
+int g_stream_path = 0;  // 0 auto, 1 generic loads, 2 TMA (when eligible)
 
 gs_status device_state(DevState** out) {
     int dev = 0;
@@ -118,13 +119,15 @@ void carve(Arena& a, Workspace& w, int n_seg, int n_chunks, int64_t n, bool buil
     w.ls.c_val = a.take<float>(n);
     w.ls.c_cnt = a.take<int32_t>(n_chunks);
     w.ls.s_low = a.take<double>(n_chunks);
+    w.ls.c_pre = a.take<int32_t>((size_t)n_chunks + n_seg);
     if (build_p) {
         w.ls.p_idx = a.take<int32_t>(n);
         w.ls.p_g = a.take<float>(n);
         w.ls.p_x = a.take<uint32_t>(n);
         w.ls.p_cnt = a.take<int32_t>(n_chunks);
-        w.ls.k_cnt = a.take<int32_t>(n_chunks);
         w.ls.k_off = a.take<int32_t>(n_chunks);
+        w.ls.k_state = a.take<unsigned long long>(n_chunks);
+        w.ls.ticket = a.take<int32_t>(1);
     }
 }
 
@@ -185,15 +188,22 @@ gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off
     a.off = 0;
     carve(a, w, n_seg, n_chunks, (int64_t)M * d, !prob);
 
-    int force;
-    int ns;
+    int force, ns, path;
     {
         std::lock_guard<std::mutex> lk(g_mu);
         force = g_force_exact;
         ns = g_sample;
+        path = g_stream_path;
     }
+    bool tma_ok = path != 1 && stream_tma_eligible(Lo);
+    for (int l = 0; tma_ok && L > 1 && l <= L; ++l)
+        if (seg_off[l] % 4 != 0) tma_ok = false;
     cudaError_t e = launch_bound(Lo, w.sp, n_seg, kappa, ns, force, st);
-    if (e == cudaSuccess) e = launch_stream(Lo, w.sp, w.ls, n_chunks, !prob, st);
+    if (e == cudaSuccess) {
+        bool used = false;
+        if (tma_ok) e = launch_stream_tma(Lo, w.sp, w.ls, n_chunks, s->status, st, &used);
+        if (e == cudaSuccess && !used) e = launch_stream(Lo, w.sp, w.ls, n_chunks, !prob, st);
+    }
     if (e == cudaSuccess) e = launch_solve(Lo, w.sp, w.ls, n_seg, kappa, iters, force, s->status, info, st);
     if (e == cudaSuccess) {
         if (prob) e = launch_prob(Lo, w.sp, p, st);
@@ -352,6 +362,10 @@ gs_status gs_set_option(int option, int64_t value) {
         case GS_OPT_SAMPLE_SIZE:
             if (value < 256 || value > 32768) return GS_ERR_INVALID_ARG;
             g_sample = (int)value;
+            return GS_OK;
+        case GS_OPT_STREAM_PATH:
+            if (value < 0 || value > 2) return GS_ERR_INVALID_ARG;
+            g_stream_path = (int)value;
             return GS_OK;
         case GS_OPT_KERNEL_TIMING:
             if (value != 0 && value != 1) return GS_ERR_INVALID_ARG;

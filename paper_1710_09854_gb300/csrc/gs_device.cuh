@@ -78,8 +78,10 @@ struct Lists {
     float* c_val;       // |g| of each capped candidate
     int32_t* c_cnt;     // [n_chunks]
     double* s_low;      // [n_chunks] sum of |g| outside C
-    int32_t* k_cnt;     // [n_chunks] kept count
-    int32_t* k_off;     // [n_chunks] exclusive offset of the chunk in its worker's output
+    int32_t* k_off;     // [n_chunks] offset of the chunk's first kept entry in its worker's output
+    unsigned long long* k_state;  // [n_emit_tiles] decoupled look-back words (zeroed by the streaming pass)
+    int32_t* ticket;    // emit-tile ticket counter (zeroed by the solve)
+    int32_t* c_pre;     // [n_chunks + n_seg] prefix scratch for segments with many chunks
 };
 
 struct Chunk {
@@ -166,7 +168,7 @@ __device__ __forceinline__ uint32_t word_of(const uint4& w, int s) {
 
 // 1 + (x >> 9) * 2^-23: a float in [1, 2) that never exceeds 1 + x * 2^-32.
 __device__ __forceinline__ float unit_plus_one(uint32_t x) {
-    return __uint_as_float(0x3F800000u | (x >> 9));
+    return __uint_as_float(0x3F800000u + (x >> 9));
 }
 
 // ---------------------------------------------------------------------------

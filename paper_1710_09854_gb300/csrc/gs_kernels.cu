@@ -191,6 +191,7 @@ __device__ void chunk_candidates(const Layout& Lo, int c, const Chunk& ch, float
     const double tot = block_sum(acc, shd);
     if (tid == 0) {
         if (build_p) Ls.p_cnt[c] = runP;
+        if (kWithC && Ls.k_state) Ls.k_state[c] = 0ull;
         if (kWithC) {
             Ls.c_cnt[c] = runC;
             Ls.s_low[c] = tot;
@@ -233,6 +234,72 @@ __device__ void segment_stats(const Layout& Lo, int m, int64_t lo, int64_t hi, f
 }
 
 // ---------------------------------------------------------------------------
+// Block-wide helpers over kThreads threads.
+// ---------------------------------------------------------------------------
+// Sum of two doubles over the block (one reduction); every thread gets both.
+__device__ __forceinline__ double2 block_sum2(double a, double b, double2* sh) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+    a = warp_sum(a);
+    b = warp_sum(b);
+    __syncthreads();
+    if (lane == 0) sh[warp] = make_double2(a, b);
+    __syncthreads();
+    if (warp == 0) {
+        double2 t = lane < nw ? sh[lane] : make_double2(0.0, 0.0);
+        t.x = warp_sum(t.x);
+        t.y = warp_sum(t.y);
+        if (lane == 0) sh[32] = t;
+    }
+    __syncthreads();
+    return sh[32];
+}
+
+// Exclusive scan of cnt[0..n) into pre[0..n]; pre[n] = total.  `pre` may live
+// in shared or global memory (written and read back by this block only).
+__device__ void block_exclusive_scan(const int32_t* __restrict__ cnt, int n, int32_t* pre, int* sh) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+    int run = 0;
+    for (int b = 0; b < n; b += blockDim.x) {
+        const int i = b + threadIdx.x;
+        const int v = i < n ? cnt[i] : 0;
+        int inc = v;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int t = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+            if (lane >= o) inc += t;
+        }
+        if (lane == 31) sh[warp] = inc;
+        __syncthreads();
+        if (warp == 0) {
+            int t = lane < nw ? sh[lane] : 0;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int u = __shfl_up_sync(0xFFFFFFFFu, t, o);
+                if (lane >= o) t += u;
+            }
+            sh[lane] = t;
+        }
+        __syncthreads();
+        const int before = warp > 0 ? sh[warp - 1] : 0;
+        if (i < n) pre[i] = run + before + inc - v;
+        run += sh[nw - 1];
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) pre[n] = run;
+    __syncthreads();
+}
+
+// Largest k in [0, n) with pre[k] <= e (pre ascending, pre[0] = 0).
+__device__ __forceinline__ int upper_slot(const int32_t* pre, int n, int e) {
+    int a = 0, b = n - 1;
+    while (a < b) {
+        const int mid = (a + b + 1) >> 1;
+        if (pre[mid] <= e) a = mid; else b = mid - 1;
+    }
+    return a;
+}
+
+// ---------------------------------------------------------------------------
 // k_bound: one CTA per segment.
 // ---------------------------------------------------------------------------
 constexpr int kBoundThreads = 512;
@@ -241,7 +308,7 @@ constexpr double kBoundZ = 5.0;
 __global__ void __launch_bounds__(kBoundThreads) k_bound(Layout Lo, SegParam* sp, double kappa, int ns,
                                                          int force_exact) {
     extern __shared__ float sa[];
-    __shared__ double shd[33];
+    __shared__ double2 sh2[33];
     __shared__ float s_acap;
     const int s = blockIdx.x, tid = threadIdx.x;
     int m, l, c0, c1;
@@ -259,6 +326,7 @@ __global__ void __launch_bounds__(kBoundThreads) k_bound(Layout Lo, SegParam* sp
         }
         return;
     }
+    float ls = 0.0f;
     for (int k = tid; k < ns; k += blockDim.x) {
         const int64_t a = lo + (int64_t)k * len / ns;
         const int64_t b = lo + (int64_t)(k + 1) * len / ns;
@@ -267,16 +335,15 @@ __global__ void __launch_bounds__(kBoundThreads) k_bound(Layout Lo, SegParam* sp
         float x = fabsf(load_one(Lo, m, pos));
         if (!(x < kInf)) x = 0.0f;  // non-finite values are reported by the solve
         sa[k] = x;
+        ls += x;
     }
-    __syncthreads();
-    float ls = 0.0f;
-    for (int k = tid; k < ns; k += blockDim.x) ls += sa[k];
-    const double S = block_sum((double)ls, shd);
+    const double S = block_sum2((double)ls, 0.0, sh2).x;
     const double budget = kappa * (double)ns;
     double lam = S > 0.0 ? budget / S : 0.0;
     double K = 0.0, Su = S;
     bool take_all = !(S > 0.0);
-    for (int it = 0; it < 64 && !take_all; ++it) {
+    // Algorithm 3 on the sample, run to (near) its fixed point.
+    for (int it = 0; it < 48 && !take_all; ++it) {
         if (tid == 0) s_acap = cap_threshold(lam);
         __syncthreads();
         const float acap = s_acap;
@@ -286,15 +353,16 @@ __global__ void __launch_bounds__(kBoundThreads) k_bound(Layout Lo, SegParam* sp
             const float x = sa[k];
             if (x >= acap) ++kc; else su += x;
         }
-        K = block_sum((double)kc, shd);
-        Su = block_sum((double)su, shd);
+        const double2 r = block_sum2((double)kc, (double)su, sh2);
+        K = r.x;
+        Su = r.y;
         if (!(Su > 0.0)) { take_all = true; break; }
         const double c = (budget - K) / (lam * Su);
-        if (!(c > 1.0)) break;
+        if (!(c > 1.0 + 1e-7)) break;
         lam *= c;
     }
     if (tid == 0) {
-        double e = take_all ? 0.0 : lam * Su / budget;  // uncapped share of the budget
+        const double e = take_all ? 0.0 : lam * Su / budget;  // uncapped share of the budget
         if (take_all || K >= budget || !(lam > 0.0)) {
             P.lam_up = (double)kInf;
             P.lam_up32 = kInf;
@@ -314,7 +382,7 @@ __global__ void __launch_bounds__(kBoundThreads) k_bound(Layout Lo, SegParam* sp
 }
 
 // ---------------------------------------------------------------------------
-// k_stream: the single pass over g.
+// k_stream (generic loads; any alignment): the single pass over g.
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(kThreads) k_stream(Layout Lo, const SegParam* __restrict__ sp, Lists Ls,
                                                      int n_chunks, int build_p) {
@@ -329,35 +397,50 @@ __global__ void __launch_bounds__(kThreads) k_stream(Layout Lo, const SegParam* 
 // Proposition 1: lambda_0 = kappa d / S (step 3); K = #{fl64(lambda |g|) >= 1}
 // (capped, outside the active set of step 5); A = lambda * (uncapped l1 mass)
 // = sum_{i in I} p_i; c = (kappa d - K) / A (step 6); stop if c <= 1 (step 7);
-// lambda <- c lambda (step 8).
+// lambda <- c lambda (step 8).  K and the uncapped mass come from (S_low, C):
+// every coordinate any lambda_j <= lam_up caps is in C.
 // ---------------------------------------------------------------------------
-__device__ void c_stats(const Lists& Ls, int c0, int c1, const Layout& Lo, float acap, double& K, double& su,
-                        double* shd) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    double acc = 0.0, cnt = 0.0;
-    for (int c = c0 + warp; c < c1; c += kWarps) {
-        const Chunk ch = decode_chunk(Lo, c);
-        const int64_t region = (int64_t)ch.m * Lo.d + ch.lo;
-        const int n = Ls.c_cnt[c];
-        float part = 0.0f;
-        int k = 0, run = 0;
-        for (int e = lane; e < n; e += 32) {
-            const float a = Ls.c_val[region + e];
-            if (a >= acap) ++k; else part += a;
-            if (++run == 16) { acc += (double)part; part = 0.0f; run = 0; }
-        }
-        acc += (double)part;
-        cnt += (double)k;
+constexpr int kSolveSmemChunks = 8192;   // chunk-prefix entries kept in shared memory
+constexpr int kSolveSmemC = 12288;       // candidate values kept in shared memory
+
+struct CView {
+    const float* smem;       // compacted candidates (nC <= kSolveSmemC), else NULL
+    const float* gbase;      // c_val + region of the segment's first chunk
+    const int32_t* pre;      // chunk prefix over the segment's chunks
+    int nch;
+    int nC;
+    __device__ __forceinline__ float at(int e) const {
+        if (smem) return smem[e];
+        const int k = upper_slot(pre, nch + 1, e);
+        return gbase[(int64_t)k * kChunk + (e - pre[k])];
     }
-    su = block_sum(acc, shd);
-    K = block_sum(cnt, shd);
+};
+
+// (#{a >= acap}, sum of the other a) over C; NaN acap sums everything.
+__device__ double2 c_stats(const CView& C, float acap, double2* sh2) {
+    double acc = 0.0;
+    float part = 0.0f;
+    int k = 0, run = 0;
+    for (int e = threadIdx.x; e < C.nC; e += blockDim.x) {
+        const float a = C.at(e);
+        if (a >= acap) ++k; else part += a;
+        if (++run == 16) { acc += (double)part; part = 0.0f; run = 0; }
+    }
+    acc += (double)part;
+    return block_sum2((double)k, acc, sh2);
 }
 
 __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lists Ls, double kappa, int iters,
                                                     int force_exact, int* status, gs_info_dev* info) {
+    extern __shared__ unsigned char dsm[];
+    int32_t* spre = reinterpret_cast<int32_t*>(dsm);                       // kSolveSmemChunks + 1
+    float* sc = reinterpret_cast<float*>(dsm + sizeof(int32_t) * (kSolveSmemChunks + 4));  // kSolveSmemC
+    __shared__ double2 sh2[33];
     __shared__ double shd[33];
+    __shared__ int shi[33];
     __shared__ float s_acap;
     const int s = blockIdx.x, tid = threadIdx.x;
+    if (s == 0 && tid == 0 && Ls.ticket) *Ls.ticket = 0;
     int m, l, c0, c1;
     int64_t lo, hi;
     seg_range(Lo, s, m, l, lo, hi, c0, c1);
@@ -366,13 +449,27 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
     const double lam_up = sp[s].lam_up;
     int flags = sp[s].flags & kSegTakeAll;
 
-    // l1 mass outside C (fixed order) and inside C.
+    // Candidate view: chunk prefix (shared or global scratch), values gathered to shared memory when they fit.
+    const int nch = c1 - c0;
+    int32_t* pre = nch <= kSolveSmemChunks ? spre : Ls.c_pre + c0 + s;
+    block_exclusive_scan(Ls.c_cnt + c0, nch, pre, shi);
+    CView C;
+    C.pre = pre;
+    C.nch = nch;
+    C.nC = pre[nch];
+    C.gbase = Ls.c_val + (int64_t)m * Lo.d + lo;
+    C.smem = nullptr;
+    if (C.nC <= kSolveSmemC) {
+        for (int e = tid; e < C.nC; e += blockDim.x) sc[e] = C.at(e);
+        __syncthreads();
+        C.smem = sc;
+    }
+
     double sl = 0.0;
-    for (int c = c0 + tid; c < c1; c += kThreads) sl += Ls.s_low[c];
+    for (int c = c0 + tid; c < c1; c += blockDim.x) sl += Ls.s_low[c];
     const double S_low = block_sum(sl, shd);
-    double Kc, Sc;
-    c_stats(Ls, c0, c1, Lo, __int_as_float(0x7FC00000), Kc, Sc, shd);  // NaN threshold: all of C summed
-    double S = S_low + Sc;
+    const double2 all = c_stats(C, __int_as_float(0x7FC00000), sh2);
+    double S = S_low + all.y;
 
     double lam = 0.0, K = 0.0, Su = 0.0;
     int j = 0;
@@ -385,20 +482,19 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
         while (j < iters) {
             if (tid == 0) s_acap = cap_threshold(lam);
             __syncthreads();
-            double suc;
-            c_stats(Ls, c0, c1, Lo, s_acap, K, suc, shd);
-            const double A = lam * (S_low + suc);
+            const double2 r = c_stats(C, s_acap, sh2);
+            const double A = lam * (S_low + r.y);
             if (A == 0.0) break;
-            const double cc = (budget - K) / A;
+            const double cc = (budget - r.x) / A;
             if (!(cc > 1.0)) break;
             lam = cc * lam;
             ++j;
         }
         if (tid == 0) s_acap = cap_threshold(lam);
         __syncthreads();
-        double suc;
-        c_stats(Ls, c0, c1, Lo, s_acap, K, suc, shd);
-        Su = S_low + suc;
+        const double2 r = c_stats(C, s_acap, sh2);
+        K = r.x;
+        Su = S_low + r.y;
         // The lists are exact only while lambda stays within the bound.
         if (lam > lam_up) exact = true;
     }
@@ -464,112 +560,170 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
 // are g_i / p_i: g_i itself when capped, else sign(g_i) / lambda (the
 // constant-value form of section 5.3).
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ bool decide(float gv, uint32_t x, const SegParam& P, float& val) {
-    const float a = fabsf(gv);
-    if (a >= P.a_cap) {
-        val = gv;
-        return true;
+struct Decider {
+    double lam;
+    float lam32, a_cap, inv_lam32;
+    __device__ __forceinline__ bool operator()(float gv, uint32_t x, float& val) const {
+        const float a = fabsf(gv);
+        if (a >= a_cap) {
+            val = gv;
+            return true;
+        }
+        const float p32 = lam32 * a;
+        const float u32 = __uint2float_rn(x) * 0x1p-32f;
+        bool keep;
+        if (u32 < p32 * (1.0f - 0x1p-20f)) keep = true;
+        else if (u32 > p32 * (1.0f + 0x1p-20f)) keep = false;
+        else keep = (double)x * 0x1p-32 < lam * (double)a;
+        val = copysignf(inv_lam32, gv);
+        return keep;
     }
-    const float p32 = P.lam32 * a;
-    const float u32 = __uint2float_rn(x) * 0x1p-32f;
-    bool keep;
-    if (u32 < p32 * (1.0f - 0x1p-20f)) keep = true;
-    else if (u32 > p32 * (1.0f + 0x1p-20f)) keep = false;
-    else keep = (double)x * 0x1p-32 < P.lam * (double)a;
-    val = copysignf(P.inv_lam32, gv);
-    return keep;
+};
+
+// ---------------------------------------------------------------------------
+// k_emit: decide + amplify + compact.  One CTA per emit tile (kEmitChunks
+// consecutive chunks of one worker), taken in ticket order; the worker's
+// output offset of the tile comes from a decoupled look-back over the
+// preceding tiles (Merrill & Garland, "Single-pass Parallel Prefix Scan with
+// Decoupled Look-back", 2016).  Every wait is bounded.
+// ---------------------------------------------------------------------------
+constexpr int kEmitChunks = 8;
+constexpr unsigned long long kFlagAgg = 1ull << 62, kFlagInc = 2ull << 62, kValMask = (1ull << 62) - 1;
+constexpr long long kSpinLimit = 1ll << 22;
+
+__device__ __forceinline__ unsigned long long ld_acquire(const unsigned long long* p) {
+    unsigned long long v;
+    asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ void st_release(unsigned long long* p, unsigned long long v) {
+    asm volatile("st.release.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
 }
 
-__global__ void __launch_bounds__(kThreads) k_count(Layout Lo, const SegParam* __restrict__ sp, Lists Ls,
-                                                    int n_chunks) {
-    __shared__ double shd[33];
-    for (int c = blockIdx.x; c < n_chunks; c += gridDim.x) {
+__global__ void __launch_bounds__(kThreads) k_emit(Layout Lo, const SegParam* __restrict__ sp, Lists Ls, int tpw,
+                                                   int32_t* idx, float* val, int32_t* nnz, int64_t cap, int* status) {
+    __shared__ int s_tile;
+    __shared__ int s_pre[kEmitChunks + 1];     // entry prefix over the tile's chunks
+    __shared__ int s_kc[kEmitChunks];          // kept per chunk
+    __shared__ long long s_prefix;
+    __shared__ int sh[2][kWarps];
+    __shared__ Decider s_dec[kEmitChunks];
+    __shared__ long long s_region[kEmitChunks];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    if (tid == 0) s_tile = atomicAdd(Ls.ticket, 1);
+    __syncthreads();
+    const int t = s_tile;
+    const int m = t / tpw;
+    const int k0 = (t - m * tpw) * kEmitChunks;
+    const int nck = min(kEmitChunks, Lo.cpw - k0);
+    const int cbase = m * Lo.cpw + k0;
+    if (tid < nck) {
+        const int c = cbase + tid;
         const Chunk ch = decode_chunk(Lo, c);
         const SegParam P = sp[ch.seg];
-        const int64_t region = (int64_t)ch.m * Lo.d + ch.lo;
-        const int n = Ls.p_cnt[c];
-        int k = 0;
-        for (int e = threadIdx.x; e < n; e += kThreads) {
-            float v;
-            k += decide(Ls.p_g[region + e], Ls.p_x[region + e], P, v) ? 1 : 0;
-        }
-        const double tot = block_sum((double)k, shd);
-        if (threadIdx.x == 0) Ls.k_cnt[c] = (int32_t)tot;
+        Decider dd;
+        dd.lam = P.lam;
+        dd.lam32 = P.lam32;
+        dd.a_cap = P.a_cap;
+        dd.inv_lam32 = P.inv_lam32;
+        s_dec[tid] = dd;
+        s_region[tid] = (long long)ch.m * Lo.d + ch.lo;
+        s_pre[tid + 1] = Ls.p_cnt[c];
+        s_kc[tid] = 0;
     }
-}
+    if (tid == 0) s_pre[0] = 0;
+    __syncthreads();
+    if (tid == 0)
+        for (int k = 0; k < nck; ++k) s_pre[k + 1] += s_pre[k];
+    __syncthreads();
+    const int n = s_pre[nck];
 
-// One CTA per worker: exclusive scan of the kept counts over its chunks.
-__global__ void __launch_bounds__(kThreads) k_scan(Layout Lo, Lists Ls, int32_t* nnz, int64_t cap, int* status) {
-    __shared__ int sh[kWarps];
-    const int m = blockIdx.x, lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int c0 = m * Lo.cpw, c1 = c0 + Lo.cpw;
-    long long run = 0;
-    for (int b = c0; b < c1; b += kThreads) {
-        const int c = b + threadIdx.x;
-        const int v = c < c1 ? Ls.k_cnt[c] : 0;
-        int inc = v;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int t = __shfl_up_sync(0xFFFFFFFFu, inc, o);
-            if (lane >= o) inc += t;
+    // Count kept entries per chunk.
+    int kept = 0;
+    for (int e = tid; e < n; e += kThreads) {
+        int k = 0;
+        while (k + 1 < nck && s_pre[k + 1] <= e) ++k;
+        const long long r = s_region[k] + (e - s_pre[k]);
+        float v;
+        if (s_dec[k](Ls.p_g[r], Ls.p_x[r], v)) {
+            atomicAdd(&s_kc[k], 1);
+            ++kept;
         }
-        if (lane == 31) sh[warp] = inc;
+    }
+    (void)kept;
+    __syncthreads();
+    if (tid == 0) {
+        long long cnt = 0;
+        for (int k = 0; k < nck; ++k) cnt += s_kc[k];
+        unsigned long long* st = Ls.k_state;
+        long long prefix = 0;
+        const int tw = t - m * tpw;  // tile index within the worker
+        if (tw == 0) {
+            st_release(&st[t], kFlagInc | (unsigned long long)cnt);
+        } else {
+            st_release(&st[t], kFlagAgg | (unsigned long long)cnt);
+            int j = t - 1;
+            for (;;) {
+                unsigned long long w = 0;
+                long long spins = 0;
+                while (((w = ld_acquire(&st[j])) >> 62) == 0 && ++spins < kSpinLimit) __nanosleep(64);
+                if ((w >> 62) == 0) {
+                    atomicOr(status, kStTimeout);
+                    break;
+                }
+                prefix += (long long)(w & kValMask);
+                if ((w >> 62) == 2) break;
+                --j;
+            }
+            st_release(&st[t], kFlagInc | (unsigned long long)(prefix + cnt));
+        }
+        s_prefix = prefix;
+        long long run = prefix;
+        for (int k = 0; k < nck; ++k) {
+            Ls.k_off[cbase + k] = (int32_t)run;
+            run += s_kc[k];
+        }
+        if (k0 + nck == Lo.cpw) {
+            nnz[m] = (int32_t)run;
+            if (run > cap) atomicOr(status, kStCapacity);
+        }
+    }
+    __syncthreads();
+
+    // Ordered write.
+    const int64_t out0 = (int64_t)m * cap;
+    long long run = s_prefix;
+    int buf = 0;
+    for (int b = 0; b < n; b += kThreads) {
+        const int e = b + tid;
+        float v = 0.0f;
+        int32_t i = 0;
+        bool keep = false;
+        if (e < n) {
+            int k = 0;
+            while (k + 1 < nck && s_pre[k + 1] <= e) ++k;
+            const long long r = s_region[k] + (e - s_pre[k]);
+            keep = s_dec[k](Ls.p_g[r], Ls.p_x[r], v);
+            i = Ls.p_idx[r];
+        }
+        const unsigned bal = __ballot_sync(0xFFFFFFFFu, keep);
+        if (lane == 0) sh[buf][warp] = __popc(bal);
         __syncthreads();
         int before = 0, tot = 0;
+#pragma unroll
         for (int w = 0; w < kWarps; ++w) {
-            before += w < warp ? sh[w] : 0;
-            tot += sh[w];
+            before += w < warp ? sh[buf][w] : 0;
+            tot += sh[buf][w];
         }
-        if (c < c1) Ls.k_off[c] = (int32_t)(run + before + inc - v);
+        if (keep) {
+            const long long pos = run + before + __popc(bal & ((1u << lane) - 1u));
+            if (pos < cap) {
+                idx[out0 + pos] = i;
+                val[out0 + pos] = v;
+            }
+        }
         run += tot;
-        __syncthreads();
-    }
-    if (threadIdx.x == 0) {
-        nnz[m] = (int32_t)run;
-        if (run > cap) atomicOr(status, kStCapacity);
-    }
-}
-
-__global__ void __launch_bounds__(kThreads) k_write(Layout Lo, const SegParam* __restrict__ sp, Lists Ls,
-                                                    int n_chunks, int32_t* idx, float* val, int64_t cap) {
-    __shared__ int sh[2][kWarps];
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    for (int c = blockIdx.x; c < n_chunks; c += gridDim.x) {
-        const Chunk ch = decode_chunk(Lo, c);
-        const SegParam P = sp[ch.seg];
-        const int64_t region = (int64_t)ch.m * Lo.d + ch.lo;
-        const int n = Ls.p_cnt[c];
-        const int64_t out0 = (int64_t)ch.m * cap;
-        long long run = Ls.k_off[c];
-        int buf = 0;
-        for (int b = 0; b < n; b += kThreads) {
-            const int e = b + threadIdx.x;
-            float v = 0.0f;
-            int32_t i = 0;
-            bool keep = false;
-            if (e < n) {
-                keep = decide(Ls.p_g[region + e], Ls.p_x[region + e], P, v);
-                i = Ls.p_idx[region + e];
-            }
-            const unsigned bal = __ballot_sync(0xFFFFFFFFu, keep);
-            if (lane == 0) sh[buf][warp] = __popc(bal);
-            __syncthreads();
-            int before = 0, tot = 0;
-            for (int w = 0; w < kWarps; ++w) {
-                before += w < warp ? sh[buf][w] : 0;
-                tot += sh[buf][w];
-            }
-            if (keep) {
-                const long long pos = run + before + __popc(bal & ((1u << lane) - 1u));
-                if (pos < cap) {
-                    idx[out0 + pos] = i;
-                    val[out0 + pos] = v;
-                }
-            }
-            run += tot;
-            buf ^= 1;
-        }
-        __syncthreads();
+        buf ^= 1;
     }
 }
 
@@ -596,9 +750,11 @@ __global__ void k_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t i
 // ---------------------------------------------------------------------------
 // Sparse sum.  k_bucket finds, for every worker list and output tile, the
 // first entry at or after the tile (validating order and range); k_tiles
-// accumulates each tile in shared memory worker by worker, in order.
+// gathers each tile's entries of all workers at once and adds them into a
+// shared-memory tile worker by worker, in order.
 // ---------------------------------------------------------------------------
-__global__ void k_bucket(AggArgs A, int32_t* off, int nt, int* status) {
+__global__ void __launch_bounds__(256) k_bucket(const __grid_constant__ AggArgs A, int32_t* off, int nt,
+                                                int* status) {
     const int m = blockIdx.y;
     const int32_t* __restrict__ idx = A.idx[m];
     long long n = A.nnz[m];
@@ -630,14 +786,21 @@ __global__ void k_bucket(AggArgs A, int32_t* off, int nt, int* status) {
     }
 }
 
-__global__ void __launch_bounds__(kThreads) k_tiles(AggArgs A, const int32_t* __restrict__ off, int nt, float* out) {
+constexpr int kAggPer = 8;   // entries each thread holds per batch
+
+__global__ void __launch_bounds__(kThreads) k_tiles(const __grid_constant__ AggArgs A,
+                                                    const int32_t* __restrict__ off, int nt, float* out) {
     __shared__ float acc[kAggTile];
+    __shared__ int32_t s_pre[kMaxAggM + 1];
+    __shared__ long long s_lo[kMaxAggM];
+    __shared__ int shi[33];
+    __shared__ int32_t s_cnt[kMaxAggM];
+    const int M = A.M;
     for (int t = blockIdx.x; t < nt; t += gridDim.x) {
         const int64_t base = (int64_t)t * kAggTile;
         const int len = (int)min((int64_t)kAggTile, A.d - base);
         for (int k = threadIdx.x; k < kAggTile; k += kThreads) acc[k] = 0.0f;
-        __syncthreads();
-        for (int m = 0; m < A.M; ++m) {
+        for (int m = threadIdx.x; m < M; m += kThreads) {
             long long n = A.nnz[m];
             if (n > A.cap) n = A.cap;
             if (n < 0) n = 0;
@@ -645,18 +808,41 @@ __global__ void __launch_bounds__(kThreads) k_tiles(AggArgs A, const int32_t* __
             long long lo = o[t], hi = o[t + 1];
             lo = lo < 0 ? 0 : (lo > n ? n : lo);
             hi = hi < lo ? lo : (hi > n ? n : hi);
-            const int32_t* __restrict__ idx = A.idx[m];
-            const float* __restrict__ val = A.val[m];
-            for (long long e = lo + threadIdx.x; e < hi; e += kThreads) {
-                const int64_t i = (int64_t)idx[e] - base;
-                if (i >= 0 && i < len) acc[i] += val[e];
+            s_lo[m] = lo;
+            s_cnt[m] = (int32_t)(hi - lo);
+        }
+        __syncthreads();
+        block_exclusive_scan(s_cnt, M, s_pre, shi);
+        const int total = s_pre[M];
+        for (int b = 0; b < total; b += kThreads * kAggPer) {
+            int mm[kAggPer];
+            int ii[kAggPer];
+            float vv[kAggPer];
+#pragma unroll
+            for (int j = 0; j < kAggPer; ++j) {
+                const int e = b + j * kThreads + threadIdx.x;
+                mm[j] = -1;
+                if (e < total) {
+                    const int m = upper_slot(s_pre, M + 1, e);
+                    const long long pos = s_lo[m] + (e - s_pre[m]);
+                    ii[j] = (int)((int64_t)A.idx[m][pos] - base);
+                    vv[j] = A.val[m][pos];
+                    mm[j] = m;
+                }
             }
-            __syncthreads();
+            const int e_last = min(total, b + kThreads * kAggPer) - 1;
+            const int m_first = upper_slot(s_pre, M + 1, b), m_last = upper_slot(s_pre, M + 1, e_last);
+            for (int m = m_first; m <= m_last; ++m) {
+#pragma unroll
+                for (int j = 0; j < kAggPer; ++j)
+                    if (mm[j] == m && ii[j] >= 0 && ii[j] < len) acc[ii[j]] += vv[j];
+                __syncthreads();
+            }
         }
         float* dst = out + base;
         if (len == kAggTile && (reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
             for (int k = threadIdx.x; k < kAggTile / 4; k += kThreads)
-                reinterpret_cast<float4*>(dst)[k] = make_float4(acc[4 * k], acc[4 * k + 1], acc[4 * k + 2], acc[4 * k + 3]);
+                reinterpret_cast<float4*>(dst)[k] = reinterpret_cast<const float4*>(acc)[k];
         } else {
             for (int k = threadIdx.x; k < len; k += kThreads) dst[k] = acc[k];
         }
@@ -694,7 +880,7 @@ cudaError_t launch_bound(const Layout& Lo, SegParam* sp, int n_seg, double kappa
 
 cudaError_t launch_stream(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, bool build_p,
                           cudaStream_t st) {
-    const int grid = min(n_chunks, sm_count() * 8);
+    const int grid = std::min(n_chunks, sm_count() * 8);
     TraceScope ts(kKStream, st);
     k_stream<<<grid, kThreads, 0, st>>>(Lo, sp, Ls, n_chunks, build_p ? 1 : 0);
     return cudaGetLastError();
@@ -702,28 +888,22 @@ cudaError_t launch_stream(const Layout& Lo, const SegParam* sp, const Lists& Ls,
 
 cudaError_t launch_solve(const Layout& Lo, SegParam* sp, const Lists& Ls, int n_seg, double kappa, int iters,
                          int force_exact, int* status, gs_info_dev* info, cudaStream_t st) {
+    const size_t smem = sizeof(int32_t) * (kSolveSmemChunks + 4) + sizeof(float) * kSolveSmemC;
+    cudaError_t e = cudaFuncSetAttribute(k_solve, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
     TraceScope ts(kKSolve, st);
-    k_solve<<<n_seg, kThreads, 0, st>>>(Lo, sp, Ls, kappa, iters, force_exact, status, info);
+    k_solve<<<n_seg, kThreads, smem, st>>>(Lo, sp, Ls, kappa, iters, force_exact, status, info);
     return cudaGetLastError();
 }
 
+int emit_tiles(int M, int cpw) { return M * ((cpw + kEmitChunks - 1) / kEmitChunks); }
+
 cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, int32_t* idx,
                            float* val, int32_t* nnz, int64_t cap, int* status, cudaStream_t st) {
-    const int grid = min(n_chunks, sm_count() * 8);
-    {
-        TraceScope ts(kKCount, st);
-        k_count<<<grid, kThreads, 0, st>>>(Lo, sp, Ls, n_chunks);
-    }
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    {
-        TraceScope ts(kKScan, st);
-        k_scan<<<Lo.M, kThreads, 0, st>>>(Lo, Ls, nnz, cap, status);
-    }
-    e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    TraceScope ts(kKWrite, st);
-    k_write<<<grid, kThreads, 0, st>>>(Lo, sp, Ls, n_chunks, idx, val, cap);
+    (void)n_chunks;
+    const int tpw = (Lo.cpw + kEmitChunks - 1) / kEmitChunks;
+    TraceScope ts(kKEmit, st);
+    k_emit<<<Lo.M * tpw, kThreads, 0, st>>>(Lo, sp, Ls, tpw, idx, val, nnz, cap, status);
     return cudaGetLastError();
 }
 
@@ -734,10 +914,18 @@ cudaError_t launch_prob(const Layout& Lo, const SegParam* sp, float* p, cudaStre
     return cudaGetLastError();
 }
 
+cudaError_t launch_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t i0, int64_t n, uint32_t* out,
+                         cudaStream_t st) {
+    const int64_t blocks = std::max<int64_t>(1, std::min<int64_t>((n + 255) / 256, (int64_t)sm_count() * 8));
+    TraceScope ts(kKWords, st);
+    k_words<<<(int)blocks, 256, 0, st>>>(seed, step, worker, i0, n, out);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_aggregate(const AggArgs& A, int32_t* off, float* out, int* status, cudaStream_t st) {
     const int nt = (int)((A.d + kAggTile - 1) / kAggTile);
-    // Bucket: enough blocks per worker to cover a full row of entries.
-    const int bx = (int)std::min<int64_t>((A.d + 255) / 256 + 1, 1024);
+    // Bucket: a few blocks per worker, grid-stride over its entries.
+    const int bx = std::max(1, std::min((sm_count() * 4 + A.M - 1) / A.M, (int)((A.d + 255) / 256 + 1)));
     dim3 grid(bx, A.M);
     {
         TraceScope ts(kKBucket, st);
@@ -745,17 +933,9 @@ cudaError_t launch_aggregate(const AggArgs& A, int32_t* off, float* out, int* st
     }
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    const int tg = min(nt, sm_count() * 6);
+    const int tg = std::min(nt, sm_count() * 4);
     TraceScope ts(kKTiles, st);
     k_tiles<<<tg, kThreads, 0, st>>>(A, off, nt, out);
-    return cudaGetLastError();
-}
-
-cudaError_t launch_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t i0, int64_t n, uint32_t* out,
-                         cudaStream_t st) {
-    const int64_t blocks = std::max<int64_t>(1, std::min<int64_t>((n + 255) / 256, (int64_t)sm_count() * 8));
-    TraceScope ts(kKWords, st);
-    k_words<<<(int)blocks, 256, 0, st>>>(seed, step, worker, i0, n, out);
     return cudaGetLastError();
 }
 

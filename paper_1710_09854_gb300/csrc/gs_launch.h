@@ -38,7 +38,11 @@ cudaError_t launch_prob(const Layout& Lo, const SegParam* sp, float* p, cudaStre
 cudaError_t launch_aggregate(const AggArgs& A, int32_t* off, float* out, int* status, cudaStream_t st);
 cudaError_t launch_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t i0, int64_t n, uint32_t* out,
                          cudaStream_t st);
+bool stream_tma_eligible(const Layout& Lo);
+cudaError_t launch_stream_tma(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, int* status,
+                              cudaStream_t st, bool* used);
 int agg_tiles(int64_t d);
+int emit_tiles(int M, int cpw);
 int chunk_size();
 
 }  // namespace gs

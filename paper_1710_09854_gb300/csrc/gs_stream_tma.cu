@@ -1,0 +1,426 @@
+// gs_stream_tma.cu -- the single streaming pass over g (steps 1-3 of the
+// path: l1 sums of Algorithm 3, the capped candidates, the ordered keep
+// candidates with their Philox words) as a persistent, warp-specialised
+// sm_103a kernel fed by the Tensor Memory Accelerator.
+//
+// One CTA per SM.  Warp 0 is the producer: one elected lane walks the CTA's
+// chunks and issues cp.async.bulk.tensor loads of whole stages (8192
+// coordinates) into a ring of shared-memory buffers, each guarded by a
+// "full" and an "empty" mbarrier.  The other kCW warps consume: every lane
+// owns 16 consecutive coordinates of a stage, reads them from shared memory
+// (the 128-byte swizzle of the tensor map makes those reads bank-conflict
+// free), draws the 4 Philox words of each 4-coordinate group, and tests
+// every coordinate against the bound lam_up.  A warp scan plus one named
+// barrier per stage orders the candidates of the 16 consumer warps, so each
+// chunk's lists come out in ascending coordinate order, as k_stream writes
+// them.
+//
+// The global tensor is g viewed as rows of 128 bytes (32 fp32 or 64 bf16);
+// a full stage is one 256 x 128 B (fp32) or 128 x 128 B (bf16) box; a partial
+// stage is loaded as 8-row boxes (rows past the tensor read as zero and
+// rows outside the chunk are masked).  Every wait is bounded: on a timeout
+// the CTA records GS_ERR_TIMEOUT, stops issuing, drains its outstanding
+// copies (again bounded) and leaves.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstdint>
+
+#include "gs_device.cuh"
+#include "gs_launch.h"
+#include "gs_trace.h"
+
+namespace gs {
+namespace {
+
+constexpr int kCW = 16;                        // consumer warps
+constexpr int kTmaThreads = 32 * (kCW + 1);
+constexpr int kStageCoords = kCW * 32 * 16;    // 8192 coordinates per stage
+constexpr int kStages = 6;
+constexpr int kRowBytes = 128;
+constexpr int kSmallRows = 8;                  // rows per box of a partial stage (1 KiB)
+constexpr long long kWaitLimit = 1ll << 22;    // try_wait polls before giving up
+
+struct StreamArgs {
+    Layout Lo;
+    const SegParam* sp;
+    Lists Ls;
+    int n_chunks;
+    int* status;
+};
+
+__device__ __forceinline__ uint32_t smem_addr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init(uint64_t* b, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(b)), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_tx(uint64_t* b, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(b)), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* b) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(b)) : "memory");
+}
+__device__ __forceinline__ bool mbar_test(uint64_t* b, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_addr(b)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// Wait until the phase with the given parity has completed; false on timeout.
+__device__ __forceinline__ bool mbar_wait(uint64_t* b, uint32_t parity) {
+    for (long long i = 0; i < kWaitLimit; ++i)
+        if (mbar_test(b, parity)) return true;
+    return false;
+}
+__device__ __forceinline__ void tma_load_rows(void* dst, const CUtensorMap* map, int row, uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+            smem_addr(dst)),
+        "l"(map), "r"(0), "r"(row), "r"(smem_addr(bar))
+        : "memory");
+}
+__device__ __forceinline__ void consumer_bar() {
+    asm volatile("bar.sync 1, %0;" ::"n"(kCW * 32) : "memory");
+}
+
+// Rows of the chunk: [r_first, r_end) of the 128-byte-row view.
+struct ChunkRows {
+    Chunk ch;
+    int64_t flat_lo, flat_hi;
+    int64_t r_first, r_end;
+};
+
+template <int kInner>
+__device__ __forceinline__ ChunkRows chunk_rows(const Layout& Lo, int c) {
+    ChunkRows r;
+    r.ch = decode_chunk(Lo, c);
+    r.flat_lo = (int64_t)r.ch.m * Lo.d + r.ch.lo;
+    r.flat_hi = (int64_t)r.ch.m * Lo.d + r.ch.hi;
+    r.r_first = r.flat_lo / kInner;
+    r.r_end = (r.flat_hi + kInner - 1) / kInner;
+    return r;
+}
+
+// kDtype 0: fp32 rows of 32; 1: bf16 rows of 64.
+template <int kDtype>
+__global__ void __maxnreg__(120)
+    k_stream_tma(const __grid_constant__ CUtensorMap map_big, const __grid_constant__ CUtensorMap map_small,
+                 StreamArgs A) {
+    constexpr int kInner = kDtype == 0 ? 32 : 64;          // elements per 128-byte row
+    constexpr int kStageRows = kStageCoords / kInner;      // 256 or 128
+    constexpr int kStageBytes = kStageRows * kRowBytes;    // 32 KiB or 16 KiB
+    extern __shared__ unsigned char dsm_raw[];
+    unsigned char* base = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(dsm_raw) + 1023) & ~uintptr_t(1023));
+    uint64_t* full = reinterpret_cast<uint64_t*>(base + kStages * kStageBytes);
+    uint64_t* empty = full + kStages;
+    uint32_t* tot = reinterpret_cast<uint32_t*>(empty + kStages);  // [2][kCW] packed (P | C << 16)
+    double* sl = reinterpret_cast<double*>(tot + 2 * kCW);           // [kCW]
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(sl + kCW);
+
+    const Layout& Lo = A.Lo;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], kCW);
+        }
+        *abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncthreads();
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane != 0) return;
+        long long it = 0;
+        bool ok = true;
+        for (int c = blockIdx.x; c < A.n_chunks && ok; c += gridDim.x) {
+            const ChunkRows cr = chunk_rows<kInner>(Lo, c);
+            for (int64_t r0 = cr.r_first; r0 < cr.r_end && ok; r0 += kStageRows, ++it) {
+                const int s = (int)(it % kStages);
+                if (it >= kStages && !mbar_wait(&empty[s], (uint32_t)(((it / kStages) - 1) & 1))) {
+                    ok = false;
+                    break;
+                }
+                if (*abort_flag) {
+                    ok = false;
+                    break;
+                }
+                const int rows = (int)std::min<int64_t>(kStageRows, cr.r_end - r0);
+                unsigned char* dst = base + s * kStageBytes;
+                if (rows == kStageRows) {
+                    mbar_arrive_tx(&full[s], kStageBytes);
+                    tma_load_rows(dst, &map_big, (int)r0, &full[s]);
+                } else {
+                    const int nb = (rows + kSmallRows - 1) / kSmallRows;
+                    mbar_arrive_tx(&full[s], (uint32_t)(nb * kSmallRows * kRowBytes));
+                    for (int b = 0; b < nb; ++b)
+                        tma_load_rows(dst + b * kSmallRows * kRowBytes, &map_small, (int)(r0 + b * kSmallRows),
+                                      &full[s]);
+                }
+            }
+        }
+        if (!ok) {
+            *abort_flag = 1;
+            atomicOr(A.status, kStTimeout);
+        }
+        // Drain: every issued stage's copy must have landed before the CTA may exit.
+        for (long long k = it - 1; k >= 0 && k >= it - kStages; --k)
+            mbar_wait(&full[k % kStages], (uint32_t)((k / kStages) & 1));
+        return;
+    }
+
+    // ---------------------------------------------------------------- consumers
+    const int cw = warp - 1;
+    const float pbias = 1.0f + 0x1p-20f;
+    long long it = 0;
+    int par = 0;
+    for (int c = blockIdx.x; c < A.n_chunks; c += gridDim.x) {
+        const ChunkRows cr = chunk_rows<kInner>(Lo, c);
+        const Chunk& ch = cr.ch;
+        const SegParam& P = A.sp[ch.seg];
+        const float lam_up32 = P.lam_up32, t_c = P.t_c;
+        const int64_t row0 = (int64_t)ch.m * Lo.d;          // flat index of the worker row
+        const int64_t region = cr.flat_lo;                   // this chunk's list region
+        const uint32_t worker = Lo.worker0 + (uint32_t)ch.m;
+        double acc = 0.0;
+        int runP = 0, runC = 0;
+        for (int64_t r0 = cr.r_first; r0 < cr.r_end; r0 += kStageRows, ++it) {
+            const int s = (int)(it % kStages);
+            bool live = !*abort_flag;
+            if (live && !mbar_wait(&full[s], (uint32_t)((it / kStages) & 1))) {
+                *abort_flag = 1;
+                atomicOr(A.status, kStTimeout);
+                live = false;
+            }
+            // This lane's 16 coordinates: 4 groups of 4 (each group one 16-byte
+            // fp32 chunk, or half of a bf16 chunk).
+            const int h = cw * 32 + lane;
+            int row, first_chunk;
+            if (kDtype == 0) { row = h >> 1; first_chunk = (h & 1) * 4; }
+            else { row = h >> 2; first_chunk = (h & 3) * 2; }
+            const int64_t f0 = (r0 + row) * kInner + (kDtype == 0 ? (h & 1) * 16 : (h & 3) * 16);
+            const bool any_valid = live && (f0 < cr.flat_hi) && (f0 + 16 > cr.flat_lo);
+            float v[16];
+            if (any_valid) {
+                const unsigned char* rp = base + s * kStageBytes + row * kRowBytes;
+                const int sw = row & 7;
+                if (kDtype == 0) {
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const float4 t = *reinterpret_cast<const float4*>(rp + (((first_chunk + j) ^ sw) << 4));
+                        v[4 * j] = t.x; v[4 * j + 1] = t.y; v[4 * j + 2] = t.z; v[4 * j + 3] = t.w;
+                    }
+                } else {
+#pragma unroll
+                    for (int j = 0; j < 2; ++j) {
+                        const uint4 t = *reinterpret_cast<const uint4*>(rp + (((first_chunk + j) ^ sw) << 4));
+                        const uint32_t u[4] = {t.x, t.y, t.z, t.w};
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            v[8 * j + 2 * k] = __uint_as_float(u[k] << 16);
+                            v[8 * j + 2 * k + 1] = __uint_as_float(u[k] & 0xFFFF0000u);
+                        }
+                    }
+                }
+            } else {
+#pragma unroll
+                for (int k = 0; k < 16; ++k) v[k] = 0.0f;
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&empty[s]);   // data is in registers: release the buffer
+
+            uint32_t pm = 0, cm = 0;
+            uint4 w[4];
+            if (any_valid) {
+                const bool whole = (f0 >= cr.flat_lo) && (f0 + 16 <= cr.flat_hi);
+                const int64_t q0 = (f0 - row0) >> 2;  // worker-local group of the first coordinate
+                float s4[4];
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    w[j] = group_words(Lo.seed, Lo.step, worker, q0 + j);
+                    float m4[4];
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        const int e = 4 * j + k;
+                        const bool valid = whole || (f0 + e >= cr.flat_lo && f0 + e < cr.flat_hi);
+                        const float a = fabsf(v[e]);
+                        const bool in_c = valid && !(a < t_c);
+                        m4[k] = (valid && !in_c) ? a : 0.0f;
+                        if (in_c) cm |= 1u << e;
+                        if (valid && unit_plus_one(word_of(w[j], k)) < fmaf(lam_up32, a, pbias)) pm |= 1u << e;
+                    }
+                    s4[j] = (m4[0] + m4[1]) + (m4[2] + m4[3]);
+                }
+                acc += (double)((s4[0] + s4[1]) + (s4[2] + s4[3]));
+            }
+
+            // Order the stage's candidates: lane scan, then warps through shared memory.
+            const uint32_t packed = (uint32_t)__popc(pm) | ((uint32_t)__popc(cm) << 16);
+            uint32_t inc = packed;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const uint32_t t = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+                if (lane >= o) inc += t;
+            }
+            if (lane == 31) tot[par * kCW + cw] = inc;
+            consumer_bar();
+            int beforeP = 0, beforeC = 0, allP = 0, allC = 0;
+#pragma unroll
+            for (int k = 0; k < kCW; ++k) {
+                const uint32_t t = tot[par * kCW + k];
+                allP += (int)(t & 0xFFFFu);
+                allC += (int)(t >> 16);
+                if (k < cw) {
+                    beforeP += (int)(t & 0xFFFFu);
+                    beforeC += (int)(t >> 16);
+                }
+            }
+            const uint32_t excl = inc - packed;
+            if (pm) {
+                int64_t e = region + runP + beforeP + (int)(excl & 0xFFFFu);
+                const int64_t i0 = f0 - row0;
+#pragma unroll
+                for (int k = 0; k < 16; ++k) {
+                    if ((pm >> k) & 1u) {
+                        A.Ls.p_idx[e] = (int32_t)(i0 + k);
+                        A.Ls.p_g[e] = v[k];
+                        A.Ls.p_x[e] = word_of(w[k >> 2], k & 3);
+                        ++e;
+                    }
+                }
+            }
+            if (cm) {
+                int64_t e = region + runC + beforeC + (int)(excl >> 16);
+#pragma unroll
+                for (int k = 0; k < 16; ++k) {
+                    if ((cm >> k) & 1u) {
+                        A.Ls.c_val[e] = fabsf(v[k]);
+                        ++e;
+                    }
+                }
+            }
+            runP += allP;
+            runC += allC;
+            par ^= 1;
+        }
+        // Chunk totals: per-warp l1 partials summed in warp order.
+        const double wsum = warp_sum(acc);
+        if (lane == 0) sl[cw] = wsum;
+        consumer_bar();
+        if (cw == 0 && lane == 0) {
+            double t = 0.0;
+            for (int k = 0; k < kCW; ++k) t += sl[k];
+            A.Ls.s_low[c] = t;
+            A.Ls.c_cnt[c] = runC;
+            if (A.Ls.p_cnt) A.Ls.p_cnt[c] = runP;
+            if (A.Ls.k_state) A.Ls.k_state[c] = 0ull;
+        }
+    }
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static bool tried = false;
+    if (!tried) {
+        tried = true;
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    }
+    return fn;
+}
+
+bool make_map(CUtensorMap* map, const void* g, int dtype, int64_t rows, int box_rows) {
+    EncodeTiledFn fn = encode_fn();
+    if (!fn) return false;
+    const int inner = dtype == 0 ? 32 : 64;
+    cuuint64_t dims[2] = {(cuuint64_t)inner, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)kRowBytes};
+    cuuint32_t box[2] = {(cuuint32_t)inner, (cuuint32_t)box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    const CUresult r = fn(map, dtype == 0 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                          const_cast<void*>(g), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                          CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+template <int kDtype>
+size_t tma_smem_bytes() {
+    constexpr int kInner = kDtype == 0 ? 32 : 64;
+    constexpr int kStageBytes = (kStageCoords / kInner) * kRowBytes;
+    return 1024 + (size_t)kStages * kStageBytes + 2 * kStages * 8 + 2 * kCW * 4 + kCW * 8 + 16;
+}
+
+int sm_count_tma() {
+    static int n = 0;
+    if (n == 0) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+        if (n <= 0) n = 1;
+    }
+    return n;
+}
+
+}  // namespace
+
+bool stream_tma_eligible(const Layout& Lo) {
+    if ((reinterpret_cast<uintptr_t>(Lo.g) & 15u) != 0) return false;
+    if (Lo.d % 4 != 0) return false;
+    const int64_t inner = Lo.dtype == 0 ? 32 : 64;
+    const int64_t total = (int64_t)Lo.M * Lo.d;
+    if (total % inner != 0) return false;
+    if (total / inner >= ((int64_t)1 << 31)) return false;
+    return encode_fn() != nullptr;
+}
+
+// Segment offsets must be multiples of 4 for the group alignment (checked by the caller).
+cudaError_t launch_stream_tma(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, int* status,
+                              cudaStream_t st, bool* used) {
+    *used = false;
+    const int64_t inner = Lo.dtype == 0 ? 32 : 64;
+    const int64_t rows = (int64_t)Lo.M * Lo.d / inner;
+    CUtensorMap big, small;
+    const int big_rows = kStageCoords / (int)inner;
+    if (!make_map(&big, Lo.g, Lo.dtype, rows, big_rows) || !make_map(&small, Lo.g, Lo.dtype, rows, kSmallRows))
+        return cudaSuccess;  // caller falls back to the generic pass
+    StreamArgs A;
+    A.Lo = Lo;
+    A.sp = sp;
+    A.Ls = Ls;
+    A.n_chunks = n_chunks;
+    A.status = status;
+    const int grid = std::min(n_chunks, sm_count_tma());
+    cudaError_t e;
+    TraceScope ts(kKStreamTma, st);
+    if (Lo.dtype == 0) {
+        const size_t smem = tma_smem_bytes<0>();
+        e = cudaFuncSetAttribute(k_stream_tma<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        k_stream_tma<0><<<grid, kTmaThreads, smem, st>>>(big, small, A);
+    } else {
+        const size_t smem = tma_smem_bytes<1>();
+        e = cudaFuncSetAttribute(k_stream_tma<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (e != cudaSuccess) return e;
+        k_stream_tma<1><<<grid, kTmaThreads, smem, st>>>(big, small, A);
+    }
+    *used = true;
+    return cudaGetLastError();
+}
+
+}  // namespace gs

@@ -11,8 +11,9 @@
 namespace gs {
 namespace {
 
-const char* kNames[kNumKernels] = {"k_bound", "k_stream", "k_solve", "k_count", "k_scan",
-                                   "k_write", "k_prob",   "k_words", "k_bucket", "k_tiles"};
+const char* kNames[kNumKernels] = {"k_bound", "k_stream", "k_solve", "k_emit",
+                                   "k_prob",  "k_words",  "k_bucket", "k_tiles",
+                                   "k_stream_tma"};
 
 struct Pending {
     int k;

@@ -9,13 +9,12 @@ enum KernelId : int {
     kKBound = 0,
     kKStream,
     kKSolve,
-    kKCount,
-    kKScan,
-    kKWrite,
+    kKEmit,
     kKProb,
     kKWords,
     kKBucket,
     kKTiles,
+    kKStreamTma,
     kNumKernels
 };
 

@@ -369,3 +369,59 @@ def test_lognormal_outliers_bf16_and_f32(gs, kappa):
     _full_check(gs, g.to(torch.bfloat16), kappa, 3, workers=[1], dtype="bf16")
     del g
     torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("path", [1, 2])
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_stream_paths(gs, path, dtype):
+    """The generic-load and the TMA streaming kernels both match the oracle,
+    on full stages, partial stages and chunk starts inside a 128-byte row."""
+    import torch
+    gs.gs_set_option(gs.GS_OPT_STREAM_PATH, path)
+    try:
+        gs.gs_kernel_times()
+        M, d = 3, (1 << 20) + 64 * 3 + 64       # d % 64 == 0: whole rows for both dtypes
+        g_host = np.stack([_vector(k, d, 70 + m) for m, k in enumerate(["t3", "lognormal", "ties"])])
+        if dtype == "bf16":
+            g_host = workloads.bf16_bits_to_f32(workloads.f32_to_bf16_bits(g_host)).reshape(M, d)
+        idx, val, nnz, _ = _sparsify_batched(gs, g_host, 0.02, 3, 9, 4, 2, dtype)
+        assert gs.gs_sync_status() == gs.GS_OK
+        n = nnz.cpu().numpy()
+        for m in range(M):
+            compare_sparse(idx[m, :n[m]].cpu().numpy(), val[m, :n[m]].cpu().numpy(), g_host[m], 0.02, 3, 9, 4, 2 + m)
+        # layer-wise with offsets that are multiples of 4 but not of a row
+        lens = [64, 1000, 4, 17004, 36, 40000, 20, 16384 * 2 + 4, 8]
+        off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
+        d2 = int(off[-1])
+        M2 = 2 if dtype == "f32" else 4             # M * d2 a multiple of 32 (fp32) / 64 (bf16)
+        assert (M2 * d2) % (32 if dtype == "f32" else 64) == 0
+        rng = np.random.default_rng(5)
+        g2 = np.stack([(rng.standard_normal(d2) * rng.choice([1e-3, 1, 50], d2)).astype(np.float32)
+                       for _ in range(M2)])
+        if dtype == "bf16":
+            g2 = workloads.bf16_bits_to_f32(workloads.f32_to_bf16_bits(g2)).reshape(M2, d2)
+            gd = _dev(workloads.f32_to_bf16_bits(g2).reshape(M2, d2)).view(torch.bfloat16)
+        else:
+            gd = _dev(g2)
+        idx = torch.empty((M2, d2), dtype=torch.int32, device="cuda")
+        val = torch.empty((M2, d2), dtype=torch.float32, device="cuda")
+        nnz = torch.empty(M2, dtype=torch.int32, device="cuda")
+        gs.gs_segmented_sparsify(gd, off, 0.05, 2, 8, 4, 0, idx, val, nnz)
+        assert gs.gs_sync_status() == gs.GS_OK
+        n = nnz.cpu().numpy()
+        for m in range(M2):
+            ri, rv, _ = oracle.segmented_sparsify(g2[m], off, 0.05, 2, 8, 4, m)
+            got_i = idx[m, :n[m]].cpu().numpy()
+            got_v = val[m, :n[m]].cpu().numpy()
+            for l in range(off.size - 1):
+                a, b = off[l], off[l + 1]
+                sel = (got_i >= a) & (got_i < b)
+                r = oracle.sparsify(g2[m, a:b], 0.05, 2, 8, 4, m, i0=a)
+                compare_sparse(got_i[sel], got_v[sel], g2[m, a:b], 0.05, 2, 8, 4, m, i0=a, ref=r)
+        times = gs.gs_kernel_times()
+        if path == 2:
+            assert times["k_stream_tma"][1] == 2 and times["k_stream"][1] == 0
+        else:
+            assert times["k_stream"][1] == 2 and times["k_stream_tma"][1] == 0
+    finally:
+        gs.gs_set_option(gs.GS_OPT_STREAM_PATH, 0)
