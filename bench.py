@@ -98,9 +98,15 @@ def job_throughput(units_per_rank, ms_max, n_ranks):
 # ---------------------------------------------------------------------------
 # Workload construction
 # ---------------------------------------------------------------------------
-def make_workload(name, kappa=None, dtype=None, rank=0):
+def make_workload(name, kappa=None, dtype=None, rank=0, workers=None, dim=None):
+    import dataclasses
     import torch
     w = {"c1": workloads.C1, "c2": workloads.C2, "c3": workloads.C3, "c4": workloads.C4, "c5": workloads.C5}[name]
+    if workers or dim:
+        if name == "c4":
+            raise SystemExit("--workers / --dim do not apply to the layer-wise workload")
+        w = dataclasses.replace(w, M=workers or w.M, d=dim or w.d,
+                                name=f"{w.name}_reduced_M{workers or w.M}_d{dim or w.d}")
     kappa = w.kappa if kappa is None else kappa
     dtype = dtype or w.dtype
     off = None
@@ -193,7 +199,7 @@ def run_gpu(args):
     import paper_1710_09854_gb300 as gs
     gs.lib()
 
-    w, g, off, kappa, dtype = make_workload(args.workload, args.kappa, args.dtype, rank)
+    w, g, off, kappa, dtype = make_workload(args.workload, args.kappa, args.dtype, rank, args.workers, args.dim)
     M, d = g.shape
     esz = g.element_size()
     cap = d
@@ -451,6 +457,8 @@ def main(argv=None):
     ap.add_argument("--workload", default="c3", choices=["c1", "c2", "c3", "c4", "c5"])
     ap.add_argument("--kappa", type=float, default=None)
     ap.add_argument("--dtype", default=None, choices=[None, "f32", "bf16"])
+    ap.add_argument("--workers", type=int, default=None, help="override M (reduced case for profiling)")
+    ap.add_argument("--dim", type=int, default=None, help="override d (reduced case for profiling)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-cpu-baseline", action="store_true")

@@ -72,6 +72,10 @@ typedef struct {
 /* Human-readable name of a status code.  Never NULL. */
 const char* gs_status_string(int status);
 
+/* Text of the last CUDA failure seen by this thread inside the library (the
+ * call that failed and the CUDA error name), "" if none.  Never NULL. */
+const char* gs_last_error(void);
+
 /* Library version as 10000*major + 100*minor + patch. */
 int gs_version(void);
 

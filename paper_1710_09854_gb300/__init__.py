@@ -22,7 +22,7 @@ GS_DTYPE_F32, GS_DTYPE_BF16 = 0, 1
 GS_OPT_FORCE_EXACT_SOLVE, GS_OPT_SAMPLE_SIZE, GS_OPT_KERNEL_TIMING, GS_OPT_STREAM_PATH = 1, 2, 3, 4
 
 # Symbols include/gs.h declares (checked by the tests).
-EXPORTS = ("gs_status_string", "gs_version", "gs_sync_status", "gs_probabilities", "gs_probabilities_ex",
+EXPORTS = ("gs_status_string", "gs_last_error", "gs_version", "gs_sync_status", "gs_probabilities", "gs_probabilities_ex",
            "gs_sparsify", "gs_batched_sparsify", "gs_segmented_sparsify", "gs_sparse_aggregate",
            "gs_pipeline_host", "gs_random_words", "gs_set_option", "gs_kernel_count", "gs_kernel_name",
            "gs_kernel_times")
@@ -56,6 +56,7 @@ def lib():
         sig = {
             "gs_status_string": ([i32], ctypes.c_char_p),
             "gs_version": ([], i32),
+            "gs_last_error": ([], ctypes.c_char_p),
             "gs_sync_status": ([vp], i32),
             "gs_probabilities": ([vp, i64, dbl, i32, vp, vp], i32),
             "gs_probabilities_ex": ([vp, i64, dbl, i32, vp, vp, vp], i32),
@@ -86,6 +87,8 @@ def status_string(code):
 
 def _check(rc, where):
     if rc != GS_OK:
+        if rc == GS_ERR_CUDA:
+            where = f"{where} [{lib().gs_last_error().decode()}]"
         raise GSError(rc, where)
 
 

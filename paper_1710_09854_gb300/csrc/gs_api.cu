@@ -5,6 +5,7 @@
 
 #include <cmath>
 #include <cstdint>
+#include <cstdio>
 #include <cstring>
 #include <map>
 #include <mutex>
@@ -36,13 +37,27 @@ struct DevState {
 
 std::mutex g_mu;
 DevState g_dev[kMaxDevices];
+thread_local char g_last_error[256] = "";
+
+// Returns GS_ERR_CUDA and remembers which call failed and why.
+gs_status cuda_fail(const char* where, cudaError_t e) {
+    snprintf(g_last_error, sizeof(g_last_error), "%s: %s (%s)", where, cudaGetErrorName(e), cudaGetErrorString(e));
+    return GS_ERR_CUDA;
+}
+
+#define GS_TRY(expr)                                  \
+    do {                                              \
+        const cudaError_t e_ = (expr);                \
+        if (e_ != cudaSuccess) return cuda_fail(#expr, e_); \
+    } while (0)
 int g_force_exact = 0;
 int g_sample = 16384;
 int g_stream_path = 0;  // 0 auto, 1 generic loads, 2 TMA (when eligible)
 
 gs_status device_state(DevState** out) {
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return GS_ERR_CUDA;
+    GS_TRY(cudaGetDevice(&dev));
+    if (dev < 0 || dev >= kMaxDevices) return cuda_fail("device ordinal", cudaErrorInvalidDevice);
     std::lock_guard<std::mutex> lk(g_mu);
     DevState& s = g_dev[dev];
     if (!s.ready) {
@@ -51,12 +66,12 @@ gs_status device_state(DevState** out) {
         props.allocType = cudaMemAllocationTypePinned;
         props.location.type = cudaMemLocationTypeDevice;
         props.location.id = dev;
-        if (cudaMemPoolCreate(&s.pool, &props) != cudaSuccess) return GS_ERR_CUDA;
+        GS_TRY(cudaMemPoolCreate(&s.pool, &props));
         uint64_t keep = UINT64_MAX;  // keep freed blocks for the next call
         cudaMemPoolSetAttribute(s.pool, cudaMemPoolAttrReleaseThreshold, &keep);
-        if (cudaMalloc(&s.status, sizeof(int)) != cudaSuccess) return GS_ERR_CUDA;
-        if (cudaMemset(s.status, 0, sizeof(int)) != cudaSuccess) return GS_ERR_CUDA;
-        if (cudaDeviceSynchronize() != cudaSuccess) return GS_ERR_CUDA;
+        GS_TRY(cudaMalloc(&s.status, sizeof(int)));
+        GS_TRY(cudaMemset(s.status, 0, sizeof(int)));
+        GS_TRY(cudaDeviceSynchronize());
         s.ready = true;
     }
     *out = &s;
@@ -82,11 +97,10 @@ gs_status segment_meta(DevState* s, const int64_t* off, int L, SegMeta* out) {
     if (acc > INT32_MAX) return GS_ERR_INVALID_ARG;
     SegMeta m;
     m.cpw = (int)acc;
-    if (cudaMalloc(&m.off, sizeof(int64_t) * (L + 1)) != cudaSuccess) return GS_ERR_CUDA;
-    if (cudaMalloc(&m.chunk0, sizeof(int32_t) * (L + 1)) != cudaSuccess) return GS_ERR_CUDA;
-    if (cudaMemcpy(m.off, off, sizeof(int64_t) * (L + 1), cudaMemcpyHostToDevice) != cudaSuccess) return GS_ERR_CUDA;
-    if (cudaMemcpy(m.chunk0, c0.data(), sizeof(int32_t) * (L + 1), cudaMemcpyHostToDevice) != cudaSuccess)
-        return GS_ERR_CUDA;
+    GS_TRY(cudaMalloc(&m.off, sizeof(int64_t) * (L + 1)));
+    GS_TRY(cudaMalloc(&m.chunk0, sizeof(int32_t) * (L + 1)));
+    GS_TRY(cudaMemcpy(m.off, off, sizeof(int64_t) * (L + 1), cudaMemcpyHostToDevice));
+    GS_TRY(cudaMemcpy(m.chunk0, c0.data(), sizeof(int32_t) * (L + 1), cudaMemcpyHostToDevice));
     if (s->segs.size() >= 32) s->segs.clear();  // bounded cache (device tables are tiny; kept until exit)
     s->segs[key] = m;
     *out = m;
@@ -121,9 +135,7 @@ void carve(Arena& a, Workspace& w, int n_seg, int n_chunks, int64_t n, bool buil
     w.ls.s_low = a.take<double>(n_chunks);
     w.ls.c_pre = a.take<int32_t>((size_t)n_chunks + n_seg);
     if (build_p) {
-        w.ls.p_idx = a.take<int32_t>(n);
-        w.ls.p_g = a.take<float>(n);
-        w.ls.p_x = a.take<uint32_t>(n);
+        w.ls.p_ent = a.take<int2>(n);
         w.ls.p_cnt = a.take<int32_t>(n_chunks);
         w.ls.k_off = a.take<int32_t>(n_chunks);
         w.ls.k_state = a.take<unsigned long long>(n_chunks);
@@ -183,7 +195,10 @@ gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off
     Workspace w;
     carve(a, w, n_seg, n_chunks, (int64_t)M * d, !prob);
     void* mem = nullptr;
-    if (cudaMallocFromPoolAsync(&mem, a.off, s->pool, st) != cudaSuccess) return GS_ERR_CUDA;
+    {
+        const cudaError_t ea = cudaMallocFromPoolAsync(&mem, a.off, s->pool, st);
+        if (ea != cudaSuccess) return cuda_fail("cudaMallocFromPoolAsync", ea);
+    }
     a.base = static_cast<char*>(mem);
     a.off = 0;
     carve(a, w, n_seg, n_chunks, (int64_t)M * d, !prob);
@@ -210,7 +225,8 @@ gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off
         else e = launch_compact(Lo, w.sp, w.ls, n_chunks, idx, val, nnz, cap, s->status, st);
     }
     cudaError_t ef = cudaFreeAsync(mem, st);
-    if (e != cudaSuccess || ef != cudaSuccess) return GS_ERR_CUDA;
+    if (e != cudaSuccess) return cuda_fail(launch_error_site(), e);
+    if (ef != cudaSuccess) return cuda_fail("cudaFreeAsync", ef);
     return GS_OK;
 }
 
@@ -235,10 +251,12 @@ gs_status run_aggregate(const int32_t* const* idx, const float* const* val, cons
     const int nt = agg_tiles(d);
     void* mem = nullptr;
     const size_t bytes = sizeof(int32_t) * (size_t)M * (size_t)(nt + 1);
-    if (cudaMallocFromPoolAsync(&mem, bytes, s->pool, st) != cudaSuccess) return GS_ERR_CUDA;
+    GS_TRY(cudaMallocFromPoolAsync(&mem, bytes, s->pool, st));
     cudaError_t e = launch_aggregate(A, static_cast<int32_t*>(mem), out, s->status, st);
     cudaError_t ef = cudaFreeAsync(mem, st);
-    return (e == cudaSuccess && ef == cudaSuccess) ? GS_OK : GS_ERR_CUDA;
+    if (e != cudaSuccess) return cuda_fail(launch_error_site(), e);
+    if (ef != cudaSuccess) return cuda_fail("cudaFreeAsync", ef);
+    return GS_OK;
 }
 
 }  // namespace
@@ -260,15 +278,17 @@ const char* gs_status_string(int status) {
 
 int gs_version(void) { return 100; }
 
+const char* gs_last_error(void) { return g_last_error; }
+
 gs_status gs_sync_status(void* stream) {
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     DevState* s = nullptr;
     gs_status rc = device_state(&s);
     if (rc != GS_OK) return rc;
     int h = 0;
-    if (cudaMemcpyAsync(&h, s->status, sizeof(int), cudaMemcpyDeviceToHost, st) != cudaSuccess) return GS_ERR_CUDA;
-    if (cudaMemsetAsync(s->status, 0, sizeof(int), st) != cudaSuccess) return GS_ERR_CUDA;
-    if (cudaStreamSynchronize(st) != cudaSuccess) return GS_ERR_CUDA;
+    GS_TRY(cudaMemcpyAsync(&h, s->status, sizeof(int), cudaMemcpyDeviceToHost, st));
+    GS_TRY(cudaMemsetAsync(s->status, 0, sizeof(int), st));
+    GS_TRY(cudaStreamSynchronize(st));
     if (h & kStNonfinite) return GS_ERR_NONFINITE;
     if (h & kStCapacity) return GS_ERR_CAPACITY;
     if (h & kStInvalid) return GS_ERR_INVALID_ARG;
@@ -323,8 +343,7 @@ gs_status gs_pipeline_host(const void* g_host, int dtype, int M, int64_t d, doub
     if (dtype != GS_DTYPE_F32 && dtype != GS_DTYPE_BF16) return GS_ERR_INVALID_ARG;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     const size_t esz = dtype == GS_DTYPE_F32 ? 4 : 2;
-    if (cudaMemcpyAsync(g_dev, g_host, esz * (size_t)M * (size_t)d, cudaMemcpyHostToDevice, st) != cudaSuccess)
-        return GS_ERR_CUDA;
+    GS_TRY(cudaMemcpyAsync(g_dev, g_host, esz * (size_t)M * (size_t)d, cudaMemcpyHostToDevice, st));
     gs_status rc = run(g_dev, dtype, M, d, nullptr, 1, kappa, iters, seed, step, worker0, idx, val, nnz, cap, nullptr,
                        nullptr, st);
     if (rc != GS_OK) return rc;
@@ -336,10 +355,8 @@ gs_status gs_pipeline_host(const void* g_host, int dtype, int M, int64_t d, doub
     }
     rc = run_aggregate(ip.data(), vp.data(), nnz, M, d, out, cap, st);
     if (rc != GS_OK) return rc;
-    if (cudaMemcpyAsync(out_host, out, sizeof(float) * (size_t)d, cudaMemcpyDeviceToHost, st) != cudaSuccess)
-        return GS_ERR_CUDA;
-    if (cudaMemcpyAsync(nnz_host, nnz, sizeof(int32_t) * (size_t)M, cudaMemcpyDeviceToHost, st) != cudaSuccess)
-        return GS_ERR_CUDA;
+    GS_TRY(cudaMemcpyAsync(out_host, out, sizeof(float) * (size_t)d, cudaMemcpyDeviceToHost, st));
+    GS_TRY(cudaMemcpyAsync(nnz_host, nnz, sizeof(int32_t) * (size_t)M, cudaMemcpyDeviceToHost, st));
     return GS_OK;
 }
 
@@ -347,9 +364,8 @@ gs_status gs_random_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t
                           void* stream) {
     if (!out || i0 < 0 || n < 0 || i0 > INT64_MAX - n) return GS_ERR_INVALID_ARG;
     if (n == 0) return GS_OK;
-    return launch_words(seed, step, worker, i0, n, out, static_cast<cudaStream_t>(stream)) == cudaSuccess
-               ? GS_OK
-               : GS_ERR_CUDA;
+    GS_TRY(launch_words(seed, step, worker, i0, n, out, static_cast<cudaStream_t>(stream)));
+    return GS_OK;
 }
 
 gs_status gs_set_option(int option, int64_t value) {

@@ -71,9 +71,7 @@ struct SegParam {
 // Candidate lists written by the streaming pass, one region per chunk at the
 // chunk's flat offset (capacity = chunk length).
 struct Lists {
-    int32_t* p_idx;     // worker-local index of each kept candidate
-    float* p_g;         // its gradient value
-    uint32_t* p_x;      // its Philox word
+    int2* p_ent;        // keep candidates: (worker-local index, bits of g_i)
     int32_t* p_cnt;     // [n_chunks]
     float* c_val;       // |g| of each capped candidate
     int32_t* c_cnt;     // [n_chunks]
@@ -162,13 +160,59 @@ __device__ __forceinline__ uint4 group_words(uint64_t seed, uint32_t step, uint3
                          (uint32_t)(seed & 0xFFFFFFFFu), (uint32_t)(seed >> 32));
 }
 
+// Philox4x32-10 for the groups q < 2^32 of one (worker, step): the first
+// round's terms that do not depend on q are computed once per chunk.
+struct PhiloxStream {
+    uint32_t x0, x1;     // words 0 and 1 after round 1 (independent of q)
+    uint32_t c3k1;       // step ^ key1, the constant half of word 2 after round 1
+    uint32_t k0, k1;     // key of round 2
+    __device__ __forceinline__ PhiloxStream(uint64_t seed, uint32_t step, uint32_t worker) {
+        const uint32_t s0 = (uint32_t)(seed & 0xFFFFFFFFu), s1 = (uint32_t)(seed >> 32);
+        const uint64_t m1 = (uint64_t)0xCD9E8D57u * (uint64_t)worker;
+        x0 = (uint32_t)(m1 >> 32) ^ 0u ^ s0;   // counter word 1 (q >> 32) is 0
+        x1 = (uint32_t)m1;
+        c3k1 = step ^ s1;
+        k0 = s0 + 0x9E3779B9u;
+        k1 = s1 + 0xBB67AE85u;
+    }
+    __device__ __forceinline__ uint4 words(uint32_t q) const {
+        const uint64_t m0 = (uint64_t)0xD2511F53u * (uint64_t)q;
+        uint32_t c0 = x0, c1 = x1, c2 = (uint32_t)(m0 >> 32) ^ c3k1, c3 = (uint32_t)m0;
+        uint32_t a = k0, b = k1;
+#pragma unroll
+        for (int r = 1; r < 10; ++r) {
+            const uint64_t p0 = (uint64_t)0xD2511F53u * (uint64_t)c0;
+            const uint64_t p1 = (uint64_t)0xCD9E8D57u * (uint64_t)c2;
+            const uint32_t n0 = (uint32_t)(p1 >> 32) ^ c1 ^ a;
+            const uint32_t n2 = (uint32_t)(p0 >> 32) ^ c3 ^ b;
+            c1 = (uint32_t)p1;
+            c3 = (uint32_t)p0;
+            c0 = n0;
+            c2 = n2;
+            a += 0x9E3779B9u;
+            b += 0xBB67AE85u;
+        }
+        return make_uint4(c0, c1, c2, c3);
+    }
+};
+
 __device__ __forceinline__ uint32_t word_of(const uint4& w, int s) {
     return s == 0 ? w.x : (s == 1 ? w.y : (s == 2 ? w.z : w.w));
 }
 
 // 1 + (x >> 9) * 2^-23: a float in [1, 2) that never exceeds 1 + x * 2^-32.
+// hi(x * 2^23) = x >> 9, so one multiply-add forms it on the integer-multiply pipe.
 __device__ __forceinline__ float unit_plus_one(uint32_t x) {
-    return __uint_as_float(0x3F800000u + (x >> 9));
+    uint32_t r;
+    asm("mad.hi.u32 %0, %1, 8388608, 1065353216;" : "=r"(r) : "r"(x));
+    return __uint_as_float(r);
+}
+
+// All ones when a < b (floats), else 0: one compare, no predicate round trip.
+__device__ __forceinline__ uint32_t lt_mask(float a, float b) {
+    uint32_t r;
+    asm("set.lt.u32.f32 %0, %1, %2;" : "=r"(r) : "f"(a), "f"(b));
+    return r;
 }
 
 // ---------------------------------------------------------------------------

@@ -161,10 +161,7 @@ __device__ void chunk_candidates(const Layout& Lo, int c, const Chunk& ch, float
                 while (bits) {
                     const int s = __ffs(bits) - 1;
                     bits &= bits - 1;
-                    const int64_t e = region + off[j] + k;
-                    Ls.p_idx[e] = (int32_t)(q * 4 + s);
-                    Ls.p_g[e] = v[j][s];
-                    Ls.p_x[e] = word_of(w[j], s);
+                    Ls.p_ent[region + off[j] + k] = make_int2((int32_t)(q * 4 + s), __float_as_int(v[j][s]));
                     ++k;
                 }
             }
@@ -526,7 +523,7 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
         }
         // Rebuild this segment's P lists for the final lambda (sparsify calls only).
         const float up32 = lam > 0.0 ? __double2float_ru(lam) : 0.0f;
-        for (int c = c0; Ls.p_idx != nullptr && c < c1; ++c) {
+        for (int c = c0; Ls.p_ent != nullptr && c < c1; ++c) {
             const Chunk ch = decode_chunk(Lo, c);
             chunk_candidates<false>(Lo, c, ch, up32, 0.0f, Ls, true);
         }
@@ -582,12 +579,15 @@ struct Decider {
 
 // ---------------------------------------------------------------------------
 // k_emit: decide + amplify + compact.  One CTA per emit tile (kEmitChunks
-// consecutive chunks of one worker), taken in ticket order; the worker's
-// output offset of the tile comes from a decoupled look-back over the
-// preceding tiles (Merrill & Garland, "Single-pass Parallel Prefix Scan with
-// Decoupled Look-back", 2016).  Every wait is bounded.
+// consecutive chunks of one worker), taken in ticket order.  Pass 1 draws
+// each candidate's Philox word again and records its decision as one bit
+// (a warp ballot per 32 candidates); the worker's output offset of the tile
+// comes from a decoupled look-back over the preceding tiles (Merrill &
+// Garland, "Single-pass Parallel Prefix Scan with Decoupled Look-back",
+// 2016; every wait bounded); pass 2 writes the kept entries in order.
 // ---------------------------------------------------------------------------
 constexpr int kEmitChunks = 8;
+constexpr int kEmitWords = kEmitChunks * kChunk / 32;   // decision words of the largest tile
 constexpr unsigned long long kFlagAgg = 1ull << 62, kFlagInc = 2ull << 62, kValMask = (1ull << 62) - 1;
 constexpr long long kSpinLimit = 1ll << 22;
 
@@ -602,19 +602,21 @@ __device__ __forceinline__ void st_release(unsigned long long* p, unsigned long 
 
 __global__ void __launch_bounds__(kThreads) k_emit(Layout Lo, const SegParam* __restrict__ sp, Lists Ls, int tpw,
                                                    int32_t* idx, float* val, int32_t* nnz, int64_t cap, int* status) {
+    __shared__ uint32_t bits[kEmitWords];     // decision bit of every candidate of the tile
+    __shared__ int32_t wpre[kEmitWords];      // kept candidates before each word
     __shared__ int s_tile;
-    __shared__ int s_pre[kEmitChunks + 1];     // entry prefix over the tile's chunks
-    __shared__ int s_kc[kEmitChunks];          // kept per chunk
-    __shared__ long long s_prefix;
-    __shared__ int sh[2][kWarps];
-    __shared__ Decider s_dec[kEmitChunks];
+    __shared__ int s_pre[kEmitChunks + 1];    // candidate prefix over the tile's chunks
     __shared__ long long s_region[kEmitChunks];
+    __shared__ Decider s_dec[kEmitChunks];
+    __shared__ long long s_prefix;
+    __shared__ int shi[33];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     if (tid == 0) s_tile = atomicAdd(Ls.ticket, 1);
     __syncthreads();
     const int t = s_tile;
     const int m = t / tpw;
-    const int k0 = (t - m * tpw) * kEmitChunks;
+    const int tw = t - m * tpw;                 // tile index within the worker
+    const int k0 = tw * kEmitChunks;
     const int nck = min(kEmitChunks, Lo.cpw - k0);
     const int cbase = m * Lo.cpw + k0;
     if (tid < nck) {
@@ -629,7 +631,6 @@ __global__ void __launch_bounds__(kThreads) k_emit(Layout Lo, const SegParam* __
         s_dec[tid] = dd;
         s_region[tid] = (long long)ch.m * Lo.d + ch.lo;
         s_pre[tid + 1] = Ls.p_cnt[c];
-        s_kc[tid] = 0;
     }
     if (tid == 0) s_pre[0] = 0;
     __syncthreads();
@@ -637,27 +638,59 @@ __global__ void __launch_bounds__(kThreads) k_emit(Layout Lo, const SegParam* __
         for (int k = 0; k < nck; ++k) s_pre[k + 1] += s_pre[k];
     __syncthreads();
     const int n = s_pre[nck];
+    const int nw = (n + 31) >> 5;
+    const PhiloxStream ph(Lo.seed, Lo.step, Lo.worker0 + (uint32_t)m);
 
-    // Count kept entries per chunk.
-    int kept = 0;
-    for (int e = tid; e < n; e += kThreads) {
-        int k = 0;
-        while (k + 1 < nck && s_pre[k + 1] <= e) ++k;
-        const long long r = s_region[k] + (e - s_pre[k]);
-        float v;
-        if (s_dec[k](Ls.p_g[r], Ls.p_x[r], v)) {
-            atomicAdd(&s_kc[k], 1);
-            ++kept;
+    // Pass 1: decisions.  Warp w takes candidates [32 w', 32 w' + 32) for w' = w, w + kWarps, ...
+    for (int wd = warp; wd < nw; wd += kWarps) {
+        const int e = wd * 32 + lane;
+        bool keep = false;
+        if (e < n) {
+            int k = 0;
+            while (k + 1 < nck && s_pre[k + 1] <= e) ++k;
+            const int2 ent = Ls.p_ent[s_region[k] + (e - s_pre[k])];
+            const uint32_t x = word_of(ph.words((uint32_t)ent.x >> 2), ent.x & 3);
+            float v;
+            keep = s_dec[k](__int_as_float(ent.y), x, v);
+        }
+        const uint32_t bal = __ballot_sync(0xFFFFFFFFu, keep);
+        if (lane == 0) bits[wd] = bal;
+    }
+    __syncthreads();
+    // Kept-count prefix over the decision words (contiguous words per thread).
+    const int per = (nw + kThreads - 1) / kThreads;
+    int mine = 0;
+    for (int k = 0; k < per; ++k) {
+        const int wd = tid * per + k;
+        if (wd < nw) mine += __popc(bits[wd]);
+    }
+    int inc = mine;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int u = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+        if (lane >= o) inc += u;
+    }
+    if (lane == 31) shi[warp] = inc;
+    __syncthreads();
+    int before = 0;
+    for (int w = 0; w < warp; ++w) before += shi[w];
+    int run = before + inc - mine;
+    for (int k = 0; k < per; ++k) {
+        const int wd = tid * per + k;
+        if (wd < nw) {
+            wpre[wd] = run;
+            run += __popc(bits[wd]);
         }
     }
-    (void)kept;
     __syncthreads();
+    auto kept_before = [&](int e) -> int {   // kept candidates of the tile before candidate e
+        if (e >= n) return nw ? wpre[nw - 1] + __popc(bits[nw - 1]) : 0;
+        return wpre[e >> 5] + __popc(bits[e >> 5] & ((1u << (e & 31)) - 1u));
+    };
     if (tid == 0) {
-        long long cnt = 0;
-        for (int k = 0; k < nck; ++k) cnt += s_kc[k];
+        const long long cnt = kept_before(n);
         unsigned long long* st = Ls.k_state;
         long long prefix = 0;
-        const int tw = t - m * tpw;  // tile index within the worker
         if (tw == 0) {
             st_release(&st[t], kFlagInc | (unsigned long long)cnt);
         } else {
@@ -678,52 +711,33 @@ __global__ void __launch_bounds__(kThreads) k_emit(Layout Lo, const SegParam* __
             st_release(&st[t], kFlagInc | (unsigned long long)(prefix + cnt));
         }
         s_prefix = prefix;
-        long long run = prefix;
-        for (int k = 0; k < nck; ++k) {
-            Ls.k_off[cbase + k] = (int32_t)run;
-            run += s_kc[k];
-        }
+        for (int k = 0; k < nck; ++k) Ls.k_off[cbase + k] = (int32_t)(prefix + kept_before(s_pre[k]));
         if (k0 + nck == Lo.cpw) {
-            nnz[m] = (int32_t)run;
-            if (run > cap) atomicOr(status, kStCapacity);
+            const long long total = prefix + cnt;
+            nnz[m] = (int32_t)total;
+            if (total > cap) atomicOr(status, kStCapacity);
         }
     }
     __syncthreads();
 
-    // Ordered write.
+    // Pass 2: kept entries in candidate order (consecutive lanes write consecutive slots).
+    const long long prefix = s_prefix;
     const int64_t out0 = (int64_t)m * cap;
-    long long run = s_prefix;
-    int buf = 0;
-    for (int b = 0; b < n; b += kThreads) {
-        const int e = b + tid;
-        float v = 0.0f;
-        int32_t i = 0;
-        bool keep = false;
-        if (e < n) {
+    for (int wd = warp; wd < nw; wd += kWarps) {
+        const uint32_t word = bits[wd];
+        if ((word >> lane) & 1u) {
+            const int e = wd * 32 + lane;
             int k = 0;
             while (k + 1 < nck && s_pre[k + 1] <= e) ++k;
-            const long long r = s_region[k] + (e - s_pre[k]);
-            keep = s_dec[k](Ls.p_g[r], Ls.p_x[r], v);
-            i = Ls.p_idx[r];
-        }
-        const unsigned bal = __ballot_sync(0xFFFFFFFFu, keep);
-        if (lane == 0) sh[buf][warp] = __popc(bal);
-        __syncthreads();
-        int before = 0, tot = 0;
-#pragma unroll
-        for (int w = 0; w < kWarps; ++w) {
-            before += w < warp ? sh[buf][w] : 0;
-            tot += sh[buf][w];
-        }
-        if (keep) {
-            const long long pos = run + before + __popc(bal & ((1u << lane) - 1u));
+            const int2 ent = Ls.p_ent[s_region[k] + (e - s_pre[k])];
+            const float gv = __int_as_float(ent.y);
+            const float v = fabsf(gv) >= s_dec[k].a_cap ? gv : copysignf(s_dec[k].inv_lam32, gv);
+            const long long pos = prefix + wpre[wd] + __popc(word & ((1u << lane) - 1u));
             if (pos < cap) {
-                idx[out0 + pos] = i;
+                idx[out0 + pos] = ent.x;
                 val[out0 + pos] = v;
             }
         }
-        run += tot;
-        buf ^= 1;
     }
 }
 
@@ -868,6 +882,7 @@ int sm_count() {
 // ---------------------------------------------------------------------------
 cudaError_t launch_bound(const Layout& Lo, SegParam* sp, int n_seg, double kappa, int ns, int force_exact,
                          cudaStream_t st) {
+    set_launch_error_site("k_bound launch");
     const size_t smem = (size_t)ns * sizeof(float);
     if (smem > 48 * 1024) {
         cudaError_t e = cudaFuncSetAttribute(k_bound, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -880,6 +895,7 @@ cudaError_t launch_bound(const Layout& Lo, SegParam* sp, int n_seg, double kappa
 
 cudaError_t launch_stream(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, bool build_p,
                           cudaStream_t st) {
+    set_launch_error_site("k_stream launch");
     const int grid = std::min(n_chunks, sm_count() * 8);
     TraceScope ts(kKStream, st);
     k_stream<<<grid, kThreads, 0, st>>>(Lo, sp, Ls, n_chunks, build_p ? 1 : 0);
@@ -888,6 +904,7 @@ cudaError_t launch_stream(const Layout& Lo, const SegParam* sp, const Lists& Ls,
 
 cudaError_t launch_solve(const Layout& Lo, SegParam* sp, const Lists& Ls, int n_seg, double kappa, int iters,
                          int force_exact, int* status, gs_info_dev* info, cudaStream_t st) {
+    set_launch_error_site("k_solve launch");
     const size_t smem = sizeof(int32_t) * (kSolveSmemChunks + 4) + sizeof(float) * kSolveSmemC;
     cudaError_t e = cudaFuncSetAttribute(k_solve, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
@@ -900,6 +917,7 @@ int emit_tiles(int M, int cpw) { return M * ((cpw + kEmitChunks - 1) / kEmitChun
 
 cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, int32_t* idx,
                            float* val, int32_t* nnz, int64_t cap, int* status, cudaStream_t st) {
+    set_launch_error_site("k_emit launch");
     (void)n_chunks;
     const int tpw = (Lo.cpw + kEmitChunks - 1) / kEmitChunks;
     TraceScope ts(kKEmit, st);
@@ -908,6 +926,7 @@ cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls
 }
 
 cudaError_t launch_prob(const Layout& Lo, const SegParam* sp, float* p, cudaStream_t st) {
+    set_launch_error_site("k_prob launch");
     const int64_t blocks = std::min<int64_t>((Lo.d + 255) / 256, (int64_t)sm_count() * 16);
     TraceScope ts(kKProb, st);
     k_prob<<<(int)blocks, 256, 0, st>>>(Lo, sp, p);
@@ -916,6 +935,7 @@ cudaError_t launch_prob(const Layout& Lo, const SegParam* sp, float* p, cudaStre
 
 cudaError_t launch_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t i0, int64_t n, uint32_t* out,
                          cudaStream_t st) {
+    set_launch_error_site("k_words launch");
     const int64_t blocks = std::max<int64_t>(1, std::min<int64_t>((n + 255) / 256, (int64_t)sm_count() * 8));
     TraceScope ts(kKWords, st);
     k_words<<<(int)blocks, 256, 0, st>>>(seed, step, worker, i0, n, out);
@@ -923,6 +943,7 @@ cudaError_t launch_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t 
 }
 
 cudaError_t launch_aggregate(const AggArgs& A, int32_t* off, float* out, int* status, cudaStream_t st) {
+    set_launch_error_site("k_bucket/k_tiles launch");
     const int nt = (int)((A.d + kAggTile - 1) / kAggTile);
     // Bucket: a few blocks per worker, grid-stride over its entries.
     const int bx = std::max(1, std::min((sm_count() * 4 + A.M - 1) / A.M, (int)((A.d + 255) / 256 + 1)));

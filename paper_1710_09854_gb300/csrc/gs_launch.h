@@ -41,6 +41,9 @@ cudaError_t launch_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t 
 bool stream_tma_eligible(const Layout& Lo);
 cudaError_t launch_stream_tma(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, int* status,
                               cudaStream_t st, bool* used);
+// The launchers record which step failed; the C ABI reports it.
+void set_launch_error_site(const char* where);
+const char* launch_error_site();
 int agg_tiles(int64_t d);
 int emit_tiles(int M, int cpw);
 int chunk_size();

@@ -107,9 +107,23 @@ __device__ __forceinline__ ChunkRows chunk_rows(const Layout& Lo, int c) {
     return r;
 }
 
+// Coordinate k (0..15) of a lane's 16, read back from its row of the stage
+// buffer (first_chunk: the lane's first 16-byte chunk; sw: the row's swizzle).
+template <int kDtype>
+__device__ __forceinline__ float stage_value(const unsigned char* rp, int first_chunk, int sw, int k) {
+    if (kDtype == 0) {
+        const int chunk = (first_chunk + (k >> 2)) ^ sw;
+        return *reinterpret_cast<const float*>(rp + (chunk << 4) + ((k & 3) << 2));
+    } else {
+        const int chunk = (first_chunk + (k >> 3)) ^ sw;
+        const uint16_t b = *reinterpret_cast<const uint16_t*>(rp + (chunk << 4) + ((k & 7) << 1));
+        return __uint_as_float((uint32_t)b << 16);
+    }
+}
+
 // kDtype 0: fp32 rows of 32; 1: bf16 rows of 64.
 template <int kDtype>
-__global__ void __maxnreg__(120)
+__global__ void __launch_bounds__(kTmaThreads, 1)
     k_stream_tma(const __grid_constant__ CUtensorMap map_big, const __grid_constant__ CUtensorMap map_small,
                  StreamArgs A) {
     constexpr int kInner = kDtype == 0 ? 32 : 64;          // elements per 128-byte row
@@ -179,16 +193,17 @@ __global__ void __maxnreg__(120)
     // ---------------------------------------------------------------- consumers
     const int cw = warp - 1;
     const float pbias = 1.0f + 0x1p-20f;
+    // Probability-only calls keep no keep-candidate lists (their pointer is NULL).
+    const bool build_p = A.Ls.p_ent != nullptr;
     long long it = 0;
     int par = 0;
     for (int c = blockIdx.x; c < A.n_chunks; c += gridDim.x) {
         const ChunkRows cr = chunk_rows<kInner>(Lo, c);
         const Chunk& ch = cr.ch;
-        const SegParam& P = A.sp[ch.seg];
-        const float lam_up32 = P.lam_up32, t_c = P.t_c;
+        const float nlam = -A.sp[ch.seg].lam_up32, t_c = A.sp[ch.seg].t_c;
         const int64_t row0 = (int64_t)ch.m * Lo.d;          // flat index of the worker row
         const int64_t region = cr.flat_lo;                   // this chunk's list region
-        const uint32_t worker = Lo.worker0 + (uint32_t)ch.m;
+        const PhiloxStream ph(Lo.seed, Lo.step, Lo.worker0 + (uint32_t)ch.m);
         double acc = 0.0;
         int runP = 0, runC = 0;
         for (int64_t r0 = cr.r_first; r0 < cr.r_end; r0 += kStageRows, ++it) {
@@ -199,18 +214,18 @@ __global__ void __maxnreg__(120)
                 atomicOr(A.status, kStTimeout);
                 live = false;
             }
-            // This lane's 16 coordinates: 4 groups of 4 (each group one 16-byte
-            // fp32 chunk, or half of a bf16 chunk).
+            // This lane's 16 coordinates: 4 Philox groups of 4.
             const int h = cw * 32 + lane;
-            int row, first_chunk;
-            if (kDtype == 0) { row = h >> 1; first_chunk = (h & 1) * 4; }
-            else { row = h >> 2; first_chunk = (h & 3) * 2; }
+            const int row = kDtype == 0 ? (h >> 1) : (h >> 2);
+            const int first_chunk = kDtype == 0 ? (h & 1) * 4 : (h & 3) * 2;
             const int64_t f0 = (r0 + row) * kInner + (kDtype == 0 ? (h & 1) * 16 : (h & 3) * 16);
+            const unsigned char* rp = base + s * kStageBytes + row * kRowBytes;
+            const int sw = row & 7;
             const bool any_valid = live && (f0 < cr.flat_hi) && (f0 + 16 > cr.flat_lo);
-            float v[16];
+            uint32_t pm = 0, cm = 0;
+            float s16 = 0.0f;
             if (any_valid) {
-                const unsigned char* rp = base + s * kStageBytes + row * kRowBytes;
-                const int sw = row & 7;
+                float v[16];
                 if (kDtype == 0) {
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
@@ -229,39 +244,62 @@ __global__ void __maxnreg__(120)
                         }
                     }
                 }
-            } else {
+                const uint32_t q0 = (uint32_t)((f0 - row0) >> 2);  // worker-local group of coordinate 0
+                if (f0 >= cr.flat_lo && f0 + 16 <= cr.flat_hi) {
+                    // All 16 coordinates belong to the chunk.
+                    float s4[4];
 #pragma unroll
-                for (int k = 0; k < 16; ++k) v[k] = 0.0f;
-            }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&empty[s]);   // data is in registers: release the buffer
-
-            uint32_t pm = 0, cm = 0;
-            uint4 w[4];
-            if (any_valid) {
-                const bool whole = (f0 >= cr.flat_lo) && (f0 + 16 <= cr.flat_hi);
-                const int64_t q0 = (f0 - row0) >> 2;  // worker-local group of the first coordinate
-                float s4[4];
-#pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    w[j] = group_words(Lo.seed, Lo.step, worker, q0 + j);
-                    float m4[4];
-#pragma unroll
-                    for (int k = 0; k < 4; ++k) {
-                        const int e = 4 * j + k;
-                        const bool valid = whole || (f0 + e >= cr.flat_lo && f0 + e < cr.flat_hi);
-                        const float a = fabsf(v[e]);
-                        const bool in_c = valid && !(a < t_c);
-                        m4[k] = (valid && !in_c) ? a : 0.0f;
-                        if (in_c) cm |= 1u << e;
-                        if (valid && unit_plus_one(word_of(w[j], k)) < fmaf(lam_up32, a, pbias)) pm |= 1u << e;
+                    for (int j = 0; j < 4; ++j) {
+                        const float a0 = fabsf(v[4 * j]), a1 = fabsf(v[4 * j + 1]);
+                        const float a2 = fabsf(v[4 * j + 2]), a3 = fabsf(v[4 * j + 3]);
+                        s4[j] = (a0 + a1) + (a2 + a3);
+                        if (build_p) {
+                            // candidate iff (1 + u) - lam_up |g| < 1 + 2^-20
+                            const uint4 w = ph.words(q0 + j);
+                            pm |= lt_mask(fmaf(nlam, a0, unit_plus_one(w.x)), pbias) & (1u << (4 * j));
+                            pm |= lt_mask(fmaf(nlam, a1, unit_plus_one(w.y)), pbias) & (2u << (4 * j));
+                            pm |= lt_mask(fmaf(nlam, a2, unit_plus_one(w.z)), pbias) & (4u << (4 * j));
+                            pm |= lt_mask(fmaf(nlam, a3, unit_plus_one(w.w)), pbias) & (8u << (4 * j));
+                        }
                     }
-                    s4[j] = (m4[0] + m4[1]) + (m4[2] + m4[3]);
+                    s16 = (s4[0] + s4[1]) + (s4[2] + s4[3]);
+                    if (!(s16 < t_c)) {
+                        // Some |g| may reach t_c (or be non-finite): split exactly.
+                        float m[16];
+#pragma unroll
+                        for (int k = 0; k < 16; ++k) {
+                            const float a = fabsf(v[k]);
+                            const bool in_c = !(a < t_c);
+                            cm |= in_c ? (1u << k) : 0u;
+                            m[k] = in_c ? 0.0f : a;
+                        }
+                        s16 = (((m[0] + m[1]) + (m[2] + m[3])) + ((m[4] + m[5]) + (m[6] + m[7]))) +
+                              (((m[8] + m[9]) + (m[10] + m[11])) + ((m[12] + m[13]) + (m[14] + m[15])));
+                    }
+                } else {
+                    // The lane straddles an edge of the chunk: test each coordinate.
+                    float m[16];
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const uint4 w = build_p ? ph.words(q0 + j) : make_uint4(0, 0, 0, 0);
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            const int e = 4 * j + k;
+                            const bool valid = f0 + e >= cr.flat_lo && f0 + e < cr.flat_hi;
+                            const float a = fabsf(v[e]);
+                            const bool in_c = valid && !(a < t_c);
+                            m[e] = (valid && !in_c) ? a : 0.0f;
+                            cm |= in_c ? (1u << e) : 0u;
+                            if (build_p && valid && fmaf(nlam, a, unit_plus_one(word_of(w, k))) < pbias) pm |= 1u << e;
+                        }
+                    }
+                    s16 = (((m[0] + m[1]) + (m[2] + m[3])) + ((m[4] + m[5]) + (m[6] + m[7]))) +
+                          (((m[8] + m[9]) + (m[10] + m[11])) + ((m[12] + m[13]) + (m[14] + m[15])));
                 }
-                acc += (double)((s4[0] + s4[1]) + (s4[2] + s4[3]));
             }
+            acc += (double)s16;
 
-            // Order the stage's candidates: lane scan, then warps through shared memory.
+            // Order the stage's candidates: lane scan, then the warps' totals by shuffle.
             const uint32_t packed = (uint32_t)__popc(pm) | ((uint32_t)__popc(cm) << 16);
             uint32_t inc = packed;
 #pragma unroll
@@ -271,43 +309,37 @@ __global__ void __maxnreg__(120)
             }
             if (lane == 31) tot[par * kCW + cw] = inc;
             consumer_bar();
-            int beforeP = 0, beforeC = 0, allP = 0, allC = 0;
+            const uint32_t tv = lane < kCW ? tot[par * kCW + lane] : 0u;
+            uint32_t ti = tv;
 #pragma unroll
-            for (int k = 0; k < kCW; ++k) {
-                const uint32_t t = tot[par * kCW + k];
-                allP += (int)(t & 0xFFFFu);
-                allC += (int)(t >> 16);
-                if (k < cw) {
-                    beforeP += (int)(t & 0xFFFFu);
-                    beforeC += (int)(t >> 16);
-                }
+            for (int o = 1; o < kCW; o <<= 1) {
+                const uint32_t t = __shfl_up_sync(0xFFFFFFFFu, ti, o);
+                if (lane >= o) ti += t;
             }
-            const uint32_t excl = inc - packed;
+            const uint32_t wbefore = __shfl_sync(0xFFFFFFFFu, ti - tv, cw);
+            const uint32_t wall = __shfl_sync(0xFFFFFFFFu, ti, kCW - 1);
+            const uint32_t excl = inc - packed + wbefore;
             if (pm) {
-                int64_t e = region + runP + beforeP + (int)(excl & 0xFFFFu);
-                const int64_t i0 = f0 - row0;
-#pragma unroll
-                for (int k = 0; k < 16; ++k) {
-                    if ((pm >> k) & 1u) {
-                        A.Ls.p_idx[e] = (int32_t)(i0 + k);
-                        A.Ls.p_g[e] = v[k];
-                        A.Ls.p_x[e] = word_of(w[k >> 2], k & 3);
-                        ++e;
-                    }
+                int64_t e = region + runP + (int)(excl & 0xFFFFu);
+                const int32_t i0 = (int32_t)(f0 - row0);
+                while (pm) {
+                    const int k = __ffs(pm) - 1;
+                    pm &= pm - 1u;
+                    A.Ls.p_ent[e++] = make_int2(i0 + k, __float_as_int(stage_value<kDtype>(rp, first_chunk, sw, k)));
                 }
             }
             if (cm) {
-                int64_t e = region + runC + beforeC + (int)(excl >> 16);
-#pragma unroll
-                for (int k = 0; k < 16; ++k) {
-                    if ((cm >> k) & 1u) {
-                        A.Ls.c_val[e] = fabsf(v[k]);
-                        ++e;
-                    }
+                int64_t e = region + runC + (int)(excl >> 16);
+                while (cm) {
+                    const int k = __ffs(cm) - 1;
+                    cm &= cm - 1u;
+                    A.Ls.c_val[e++] = fabsf(stage_value<kDtype>(rp, first_chunk, sw, k));
                 }
             }
-            runP += allP;
-            runC += allC;
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&empty[s]);   // this warp is done with the buffer
+            runP += (int)(wall & 0xFFFFu);
+            runC += (int)(wall >> 16);
             par ^= 1;
         }
         // Chunk totals: per-warp l1 partials summed in warp order.
@@ -392,6 +424,7 @@ bool stream_tma_eligible(const Layout& Lo) {
 // Segment offsets must be multiples of 4 for the group alignment (checked by the caller).
 cudaError_t launch_stream_tma(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, int* status,
                               cudaStream_t st, bool* used) {
+    set_launch_error_site("k_stream_tma launch");
     *used = false;
     const int64_t inner = Lo.dtype == 0 ? 32 : 64;
     const int64_t rows = (int64_t)Lo.M * Lo.d / inner;
@@ -410,13 +443,17 @@ cudaError_t launch_stream_tma(const Layout& Lo, const SegParam* sp, const Lists&
     TraceScope ts(kKStreamTma, st);
     if (Lo.dtype == 0) {
         const size_t smem = tma_smem_bytes<0>();
+        set_launch_error_site("k_stream_tma<fp32> shared-memory attribute");
         e = cudaFuncSetAttribute(k_stream_tma<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
+        set_launch_error_site("k_stream_tma<fp32> launch");
         k_stream_tma<0><<<grid, kTmaThreads, smem, st>>>(big, small, A);
     } else {
         const size_t smem = tma_smem_bytes<1>();
+        set_launch_error_site("k_stream_tma<bf16> shared-memory attribute");
         e = cudaFuncSetAttribute(k_stream_tma<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
+        set_launch_error_site("k_stream_tma<bf16> launch");
         k_stream_tma<1><<<grid, kTmaThreads, smem, st>>>(big, small, A);
     }
     *used = true;

@@ -6,6 +6,7 @@
 #include <vector>
 
 #include "gs.h"
+#include "gs_launch.h"
 #include "gs_trace.h"
 
 namespace gs {
@@ -41,6 +42,12 @@ cudaEvent_t take_event() {
 }  // namespace
 
 void trace_set_timing(int on) { timing_on.store(on ? 1 : 0); }
+
+namespace {
+thread_local const char* g_site = "kernel launch";
+}
+void set_launch_error_site(const char* where) { g_site = where; }
+const char* launch_error_site() { return g_site; }
 
 TraceScope::TraceScope(int k, cudaStream_t st) : k_(k), st_(st), a_(nullptr) {
     launches[k].fetch_add(1);

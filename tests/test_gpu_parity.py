@@ -390,10 +390,10 @@ def test_stream_paths(gs, path, dtype):
         for m in range(M):
             compare_sparse(idx[m, :n[m]].cpu().numpy(), val[m, :n[m]].cpu().numpy(), g_host[m], 0.02, 3, 9, 4, 2 + m)
         # layer-wise with offsets that are multiples of 4 but not of a row
-        lens = [64, 1000, 4, 17004, 36, 40000, 20, 16384 * 2 + 4, 8]
+        lens = [64, 1000, 4, 17004, 36, 40000, 20, 16384 * 2 + 4, 12]
         off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
         d2 = int(off[-1])
-        M2 = 2 if dtype == "f32" else 4             # M * d2 a multiple of 32 (fp32) / 64 (bf16)
+        M2 = 2                                      # M * d2 a multiple of 32 (fp32) and 64 (bf16)
         assert (M2 * d2) % (32 if dtype == "f32" else 64) == 0
         rng = np.random.default_rng(5)
         g2 = np.stack([(rng.standard_normal(d2) * rng.choice([1e-3, 1, 50], d2)).astype(np.float32)
