@@ -175,6 +175,10 @@ gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off
     Lo.seed = seed;
     Lo.step = step;
     Lo.worker0 = worker0;
+    for (int r = 0; r < 10; ++r) {
+        Lo.rk0[r] = (uint32_t)(seed & 0xFFFFFFFFu) + (uint32_t)r * 0x9E3779B9u;
+        Lo.rk1[r] = (uint32_t)(seed >> 32) + (uint32_t)r * 0xBB67AE85u;
+    }
     if (L == 1) {
         const int64_t cpw = (d + chunk_size() - 1) / chunk_size();
         Lo.cpw = (int)cpw;
@@ -376,7 +380,7 @@ gs_status gs_set_option(int option, int64_t value) {
             g_force_exact = (int)value;
             return GS_OK;
         case GS_OPT_SAMPLE_SIZE:
-            if (value < 256 || value > 32768) return GS_ERR_INVALID_ARG;
+            if (value < 256 || value > 32768 || value % 8 != 0) return GS_ERR_INVALID_ARG;
             g_sample = (int)value;
             return GS_OK;
         case GS_OPT_STREAM_PATH:

@@ -49,6 +49,7 @@ struct Layout {
     uint64_t seed;
     uint32_t step;
     uint32_t worker0;
+    uint32_t rk0[10], rk1[10];  // Philox round keys: seed lo / hi plus r times the Weyl increments
 };
 
 // Per-segment state: the bound of the sampling pass and the final solve.
@@ -162,35 +163,32 @@ __device__ __forceinline__ uint4 group_words(uint64_t seed, uint32_t step, uint3
 
 // Philox4x32-10 for the groups q < 2^32 of one (worker, step): the first
 // round's terms that do not depend on q are computed once per chunk.
+// The round keys come from the kernel's parameter space (Layout::rk0/rk1),
+// so every key XOR reads its key straight from the constant bank.
 struct PhiloxStream {
+    const uint32_t* rk0;
+    const uint32_t* rk1;
     uint32_t x0, x1;     // words 0 and 1 after round 1 (independent of q)
     uint32_t c3k1;       // step ^ key1, the constant half of word 2 after round 1
-    uint32_t k0, k1;     // key of round 2
-    __device__ __forceinline__ PhiloxStream(uint64_t seed, uint32_t step, uint32_t worker) {
-        const uint32_t s0 = (uint32_t)(seed & 0xFFFFFFFFu), s1 = (uint32_t)(seed >> 32);
+    __device__ __forceinline__ PhiloxStream(const Layout& Lo, uint32_t worker) : rk0(Lo.rk0), rk1(Lo.rk1) {
         const uint64_t m1 = (uint64_t)0xCD9E8D57u * (uint64_t)worker;
-        x0 = (uint32_t)(m1 >> 32) ^ 0u ^ s0;   // counter word 1 (q >> 32) is 0
+        x0 = (uint32_t)(m1 >> 32) ^ 0u ^ rk0[0];   // counter word 1 (q >> 32) is 0
         x1 = (uint32_t)m1;
-        c3k1 = step ^ s1;
-        k0 = s0 + 0x9E3779B9u;
-        k1 = s1 + 0xBB67AE85u;
+        c3k1 = Lo.step ^ rk1[0];
     }
     __device__ __forceinline__ uint4 words(uint32_t q) const {
         const uint64_t m0 = (uint64_t)0xD2511F53u * (uint64_t)q;
         uint32_t c0 = x0, c1 = x1, c2 = (uint32_t)(m0 >> 32) ^ c3k1, c3 = (uint32_t)m0;
-        uint32_t a = k0, b = k1;
 #pragma unroll
         for (int r = 1; r < 10; ++r) {
             const uint64_t p0 = (uint64_t)0xD2511F53u * (uint64_t)c0;
             const uint64_t p1 = (uint64_t)0xCD9E8D57u * (uint64_t)c2;
-            const uint32_t n0 = (uint32_t)(p1 >> 32) ^ c1 ^ a;
-            const uint32_t n2 = (uint32_t)(p0 >> 32) ^ c3 ^ b;
+            const uint32_t n0 = (uint32_t)(p1 >> 32) ^ c1 ^ rk0[r];
+            const uint32_t n2 = (uint32_t)(p0 >> 32) ^ c3 ^ rk1[r];
             c1 = (uint32_t)p1;
             c3 = (uint32_t)p0;
             c0 = n0;
             c2 = n2;
-            a += 0x9E3779B9u;
-            b += 0xBB67AE85u;
         }
         return make_uint4(c0, c1, c2, c3);
     }
@@ -206,6 +204,13 @@ __device__ __forceinline__ float unit_plus_one(uint32_t x) {
     uint32_t r;
     asm("mad.hi.u32 %0, %1, 8388608, 1065353216;" : "=r"(r) : "r"(x));
     return __uint_as_float(r);
+}
+
+// m | (t & bit) in one three-input logic op.
+__device__ __forceinline__ uint32_t or_and(uint32_t m, uint32_t t, uint32_t bit) {
+    uint32_t r;
+    asm("lop3.b32 %0, %1, %2, %3, 0xF8;" : "=r"(r) : "r"(m), "r"(t), "r"(bit));
+    return r;
 }
 
 // All ones when a < b (floats), else 0: one compare, no predicate round trip.

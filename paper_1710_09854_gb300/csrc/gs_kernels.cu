@@ -23,6 +23,7 @@
 //   k_bucket / k_tiles
 //              the worker-order fp32 sum of the M sparse vectors (Algorithm 1,
 //              step 6).
+#include <cooperative_groups.h>
 #include <cuda_runtime.h>
 
 #include <cfloat>
@@ -299,15 +300,51 @@ __device__ __forceinline__ int upper_slot(const int32_t* pre, int n, int e) {
 // ---------------------------------------------------------------------------
 // k_bound: one CTA per segment.
 // ---------------------------------------------------------------------------
-constexpr int kBoundThreads = 512;
 constexpr double kBoundZ = 5.0;
 
-__global__ void __launch_bounds__(kBoundThreads) k_bound(Layout Lo, SegParam* sp, double kappa, int ns,
-                                                         int force_exact) {
-    extern __shared__ float sa[];
-    __shared__ double2 sh2[33];
-    __shared__ float s_acap;
-    const int s = blockIdx.x, tid = threadIdx.x;
+// Sum of two floats over the block; every thread gets both.
+__device__ __forceinline__ float2 block_sum2f(float a, float b, float2* sh) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        a += __shfl_xor_sync(0xFFFFFFFFu, a, o);
+        b += __shfl_xor_sync(0xFFFFFFFFu, b, o);
+    }
+    __syncthreads();
+    if (lane == 0) sh[warp] = make_float2(a, b);
+    __syncthreads();
+    if (warp == 0) {
+        float2 t = lane < nw ? sh[lane] : make_float2(0.0f, 0.0f);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            t.x += __shfl_xor_sync(0xFFFFFFFFu, t.x, o);
+            t.y += __shfl_xor_sync(0xFFFFFFFFu, t.y, o);
+        }
+        if (lane == 0) sh[32] = t;
+    }
+    __syncthreads();
+    return sh[32];
+}
+
+// The bound only steers how many candidates the streaming pass keeps, so it
+// is estimated in fp32: a stratified sample of |g| (one coordinate drawn by
+// hash from each of ns equal strata) and Algorithm 3 run on the sample until
+// its scaling factor is within 1e-5 of 1.  One thread-block cluster of
+// kBoundCTAs CTAs per segment: each CTA draws ns / kBoundCTAs strata, and
+// every iteration's sums are exchanged through distributed shared memory
+// and added in rank order, so all CTAs of the cluster follow the same path.
+constexpr int kBoundCTAs = 8;
+constexpr int kBoundCtaThreads = 256;
+
+__global__ void __cluster_dims__(kBoundCTAs, 1, 1) __launch_bounds__(kBoundCtaThreads)
+    k_bound(Layout Lo, SegParam* sp, double kappa, int ns, int force_exact) {
+    namespace cg = cooperative_groups;
+    cg::cluster_group cluster = cg::this_cluster();
+    extern __shared__ float sa[];               // this CTA's ns / kBoundCTAs samples
+    __shared__ float2 sh2[33];
+    __shared__ float2 xch[2];                   // this CTA's partial sums, double-buffered by iteration
+    const int rank = (int)cluster.block_rank();
+    const int s = blockIdx.x / kBoundCTAs, tid = threadIdx.x;
     int m, l, c0, c1;
     int64_t lo, hi;
     seg_range(Lo, s, m, l, lo, hi, c0, c1);
@@ -315,52 +352,69 @@ __global__ void __launch_bounds__(kBoundThreads) k_bound(Layout Lo, SegParam* sp
     SegParam& P = sp[s];
     if (len <= ns || force_exact) {
         // Short segment (or exact mode): every coordinate is a candidate.
-        if (tid == 0) {
+        if (rank == 0 && tid == 0) {
             P.lam_up = (double)kInf;
             P.lam_up32 = kInf;
             P.t_c = 0.0f;
             P.flags = kSegTakeAll;
         }
-        return;
+        return;   // uniform over the cluster: no CTA reaches a cluster barrier
     }
+    const int per = ns / kBoundCTAs;
+    const uint32_t q = (uint32_t)(len / ns);                        // stratum width (the last one takes the rest)
+    const uint32_t q_last = (uint32_t)(len - (int64_t)(ns - 1) * q);
+    const uint32_t hs = mix32((uint32_t)s + 0x68E31DA4u);
     float ls = 0.0f;
-    for (int k = tid; k < ns; k += blockDim.x) {
-        const int64_t a = lo + (int64_t)k * len / ns;
-        const int64_t b = lo + (int64_t)(k + 1) * len / ns;
-        const uint32_t h = mix32((uint32_t)k * 0x9E3779B9u ^ mix32((uint32_t)s + 0x68E31DA4u));
-        const int64_t pos = a + (int64_t)(h % (uint32_t)(b - a));
+#pragma unroll 8
+    for (int kk = tid; kk < per; kk += kBoundCtaThreads) {
+        const int k = rank * per + kk;
+        const uint32_t h = mix32((uint32_t)k * 0x9E3779B9u ^ hs);
+        const int64_t pos = lo + (int64_t)k * q + (int64_t)(h % (k == ns - 1 ? q_last : q));
         float x = fabsf(load_one(Lo, m, pos));
         if (!(x < kInf)) x = 0.0f;  // non-finite values are reported by the solve
-        sa[k] = x;
+        sa[kk] = x;
         ls += x;
     }
-    const double S = block_sum2((double)ls, 0.0, sh2).x;
-    const double budget = kappa * (double)ns;
-    double lam = S > 0.0 ? budget / S : 0.0;
-    double K = 0.0, Su = S;
-    bool take_all = !(S > 0.0);
-    // Algorithm 3 on the sample, run to (near) its fixed point.
-    for (int it = 0; it < 48 && !take_all; ++it) {
-        if (tid == 0) s_acap = cap_threshold(lam);
-        __syncthreads();
-        const float acap = s_acap;
-        float su = 0.0f;
-        int kc = 0;
-        for (int k = tid; k < ns; k += blockDim.x) {
-            const float x = sa[k];
-            if (x >= acap) ++kc; else su += x;
+    // Cluster-wide sums of (a, b): local block sum, then every CTA adds the
+    // kBoundCTAs partials in rank order.
+    int buf = 0;
+    auto cluster_sum2 = [&](float a, float b) -> float2 {
+        const float2 loc = block_sum2f(a, b, sh2);
+        if (tid == 0) xch[buf] = loc;
+        cluster.sync();
+        float2 r = make_float2(0.0f, 0.0f);
+        for (int k = 0; k < kBoundCTAs; ++k) {
+            const float2 v = *cluster.map_shared_rank(&xch[buf], k);
+            r.x += v.x;
+            r.y += v.y;
         }
-        const double2 r = block_sum2((double)kc, (double)su, sh2);
+        buf ^= 1;
+        return r;
+    };
+    const float S = cluster_sum2(ls, 0.0f).x;
+    const float budget = (float)(kappa * (double)ns);
+    float lam = S > 0.0f ? budget / S : 0.0f;
+    float K = 0.0f, Su = S;
+    bool take_all = !(S > 0.0f) || !(lam < kInf);
+    for (int it = 0; it < 32 && !take_all; ++it) {
+        const float acap = 1.0f / lam;
+        float su = 0.0f, kc = 0.0f;
+        for (int kk = tid; kk < per; kk += kBoundCtaThreads) {
+            const float x = sa[kk];
+            if (x >= acap) kc += 1.0f; else su += x;
+        }
+        const float2 r = cluster_sum2(kc, su);
         K = r.x;
         Su = r.y;
-        if (!(Su > 0.0)) { take_all = true; break; }
-        const double c = (budget - K) / (lam * Su);
-        if (!(c > 1.0 + 1e-7)) break;
+        if (!(Su > 0.0f)) { take_all = true; break; }
+        const float c = (budget - K) / (lam * Su);
+        if (!(c > 1.0f + 1e-5f)) break;
         lam *= c;
     }
-    if (tid == 0) {
-        const double e = take_all ? 0.0 : lam * Su / budget;  // uncapped share of the budget
-        if (take_all || K >= budget || !(lam > 0.0)) {
+    cluster.sync();   // no CTA may leave while a peer still reads its partials
+    if (rank == 0 && tid == 0) {
+        const double e = take_all ? 0.0 : (double)lam * Su / budget;  // uncapped share of the budget
+        if (take_all || K >= budget || !(lam > 0.0f)) {
             P.lam_up = (double)kInf;
             P.lam_up32 = kInf;
             P.t_c = 0.0f;
@@ -368,7 +422,7 @@ __global__ void __launch_bounds__(kBoundThreads) k_bound(Layout Lo, SegParam* sp
         } else {
             double margin = 1.0 + kBoundZ / sqrt(kappa * (double)ns) / fmax(e, 1.0 / 16.0);
             margin = fmin(margin, 64.0);
-            const double up = lam * margin;
+            const double up = (double)lam * margin;
             P.lam_up = up;
             P.lam_up32 = __double2float_ru(up);
             const double t = (1.0 / up) * (1.0 - 0x1p-20);
@@ -552,8 +606,8 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
 
 // ---------------------------------------------------------------------------
 // Decision for one candidate: Z_i = [u_i < p_i] with p_i = min(fl64(lam |g_i|), 1)
-// and u_i = x 2^-32 (section 3).  fp32 decides whenever u is more than 2^-20
-// (relative) away from p; closer calls are settled in fp64.  Kept values
+// and u_i = x 2^-32 (section 3).  fp32 decides whenever u is more than 2^-21
+// away from p; closer calls are settled in fp64.  Kept values
 // are g_i / p_i: g_i itself when capped, else sign(g_i) / lambda (the
 // constant-value form of section 5.3).
 // ---------------------------------------------------------------------------
@@ -566,11 +620,14 @@ struct Decider {
             val = gv;
             return true;
         }
-        const float p32 = lam32 * a;
-        const float u32 = __uint2float_rn(x) * 0x1p-32f;
+        // 1 + u lies in [uf, uf + 2^-23) with uf exact; 1 + p is within 2^-23 of
+        // pf.  Outside a 2^-21 band the fp32 comparison is certain; inside it
+        // (probability ~2^-20 per candidate) fp64 decides.
+        const float uf = unit_plus_one(x);
+        const float pf = fmaf(lam32, a, 1.0f);
         bool keep;
-        if (u32 < p32 * (1.0f - 0x1p-20f)) keep = true;
-        else if (u32 > p32 * (1.0f + 0x1p-20f)) keep = false;
+        if (uf + 0x1p-21f < pf) keep = true;
+        else if (uf - 0x1p-21f > pf) keep = false;
         else keep = (double)x * 0x1p-32 < lam * (double)a;
         val = copysignf(inv_lam32, gv);
         return keep;
@@ -600,7 +657,8 @@ __device__ __forceinline__ void st_release(unsigned long long* p, unsigned long 
     asm volatile("st.release.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
 }
 
-__global__ void __launch_bounds__(kThreads) k_emit(Layout Lo, const SegParam* __restrict__ sp, Lists Ls, int tpw,
+__global__ void __launch_bounds__(kThreads) k_emit(const __grid_constant__ Layout Lo, const SegParam* __restrict__ sp,
+                                                   const __grid_constant__ Lists Ls, int tpw,
                                                    int32_t* idx, float* val, int32_t* nnz, int64_t cap, int* status) {
     __shared__ uint32_t bits[kEmitWords];     // decision bit of every candidate of the tile
     __shared__ int32_t wpre[kEmitWords];      // kept candidates before each word
@@ -639,7 +697,7 @@ __global__ void __launch_bounds__(kThreads) k_emit(Layout Lo, const SegParam* __
     __syncthreads();
     const int n = s_pre[nck];
     const int nw = (n + 31) >> 5;
-    const PhiloxStream ph(Lo.seed, Lo.step, Lo.worker0 + (uint32_t)m);
+    const PhiloxStream ph(Lo, Lo.worker0 + (uint32_t)m);
 
     // Pass 1: decisions.  Warp w takes candidates [32 w', 32 w' + 32) for w' = w, w + kWarps, ...
     for (int wd = warp; wd < nw; wd += kWarps) {
@@ -687,35 +745,46 @@ __global__ void __launch_bounds__(kThreads) k_emit(Layout Lo, const SegParam* __
         if (e >= n) return nw ? wpre[nw - 1] + __popc(bits[nw - 1]) : 0;
         return wpre[e >> 5] + __popc(bits[e >> 5] & ((1u << (e & 31)) - 1u));
     };
-    if (tid == 0) {
+    if (warp == 0) {
+        // Decoupled look-back, one warp: lane l inspects tile t-1-l of the same
+        // worker; the nearest inclusive prefix ends the walk, aggregates before
+        // it are summed; otherwise the window moves back by 32 tiles.
         const long long cnt = kept_before(n);
         unsigned long long* st = Ls.k_state;
         long long prefix = 0;
-        if (tw == 0) {
-            st_release(&st[t], kFlagInc | (unsigned long long)cnt);
-        } else {
-            st_release(&st[t], kFlagAgg | (unsigned long long)cnt);
-            int j = t - 1;
-            for (;;) {
-                unsigned long long w = 0;
+        if (lane == 0) st_release(&st[t], (tw == 0 ? kFlagInc : kFlagAgg) | (unsigned long long)cnt);
+        int j = t - 1;                  // newest tile of the current window
+        const int first = t - tw;       // the worker's first tile (publishes an inclusive prefix at once)
+        bool done = tw == 0;
+        while (!done) {
+            const int mine = j - lane;
+            unsigned long long w = kFlagInc;   // lanes before the worker's first tile read as empty inclusives
+            if (mine >= first) {
                 long long spins = 0;
-                while (((w = ld_acquire(&st[j])) >> 62) == 0 && ++spins < kSpinLimit) __nanosleep(64);
+                while (((w = ld_acquire(&st[mine])) >> 62) == 0 && ++spins < kSpinLimit) __nanosleep(32);
                 if ((w >> 62) == 0) {
                     atomicOr(status, kStTimeout);
-                    break;
+                    w = kFlagInc;
                 }
-                prefix += (long long)(w & kValMask);
-                if ((w >> 62) == 2) break;
-                --j;
             }
-            st_release(&st[t], kFlagInc | (unsigned long long)(prefix + cnt));
+            const unsigned inc_mask = __ballot_sync(0xFFFFFFFFu, (w >> 62) == 2);
+            const int stop = inc_mask ? __ffs(inc_mask) - 1 : 32;   // nearest inclusive in the window
+            long long v = lane <= stop && lane < 32 ? (long long)(w & kValMask) : 0;
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
+            prefix += v;
+            if (inc_mask) done = true;
+            else j -= 32;
         }
-        s_prefix = prefix;
-        for (int k = 0; k < nck; ++k) Ls.k_off[cbase + k] = (int32_t)(prefix + kept_before(s_pre[k]));
-        if (k0 + nck == Lo.cpw) {
-            const long long total = prefix + cnt;
-            nnz[m] = (int32_t)total;
-            if (total > cap) atomicOr(status, kStCapacity);
+        if (lane == 0) {
+            if (tw != 0) st_release(&st[t], kFlagInc | (unsigned long long)(prefix + cnt));
+            s_prefix = prefix;
+            for (int k = 0; k < nck; ++k) Ls.k_off[cbase + k] = (int32_t)(prefix + kept_before(s_pre[k]));
+            if (k0 + nck == Lo.cpw) {
+                const long long total = prefix + cnt;
+                nnz[m] = (int32_t)total;
+                if (total > cap) atomicOr(status, kStCapacity);
+            }
         }
     }
     __syncthreads();
@@ -883,13 +952,13 @@ int sm_count() {
 cudaError_t launch_bound(const Layout& Lo, SegParam* sp, int n_seg, double kappa, int ns, int force_exact,
                          cudaStream_t st) {
     set_launch_error_site("k_bound launch");
-    const size_t smem = (size_t)ns * sizeof(float);
+    const size_t smem = (size_t)(ns / kBoundCTAs) * sizeof(float);
     if (smem > 48 * 1024) {
         cudaError_t e = cudaFuncSetAttribute(k_bound, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
     }
     TraceScope ts(kKBound, st);
-    k_bound<<<n_seg, kBoundThreads, smem, st>>>(Lo, sp, kappa, ns, force_exact);
+    k_bound<<<n_seg * kBoundCTAs, kBoundCtaThreads, smem, st>>>(Lo, sp, kappa, ns, force_exact);
     return cudaGetLastError();
 }
 

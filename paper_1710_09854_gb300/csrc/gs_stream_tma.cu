@@ -37,7 +37,7 @@ namespace {
 constexpr int kCW = 16;                        // consumer warps
 constexpr int kTmaThreads = 32 * (kCW + 1);
 constexpr int kStageCoords = kCW * 32 * 16;    // 8192 coordinates per stage
-constexpr int kStages = 6;
+constexpr int kStageBudget = 96 * 1024;          // shared memory for the ring of one CTA (2 CTAs per SM)
 constexpr int kRowBytes = 128;
 constexpr int kSmallRows = 8;                  // rows per box of a partial stage (1 KiB)
 constexpr long long kWaitLimit = 1ll << 22;    // try_wait polls before giving up
@@ -122,13 +122,23 @@ __device__ __forceinline__ float stage_value(const unsigned char* rp, int first_
 }
 
 // kDtype 0: fp32 rows of 32; 1: bf16 rows of 64.
+// Error-free fp32 accumulation (Knuth's TwoSum): hi + lo carries the exact
+// running sum to ~2^-48, so the per-lane sums never touch the fp64 pipe.
+__device__ __forceinline__ void two_sum_add(float& hi, float& lo, float x) {
+    const float s = hi + x;
+    const float bb = s - hi;
+    lo += (hi - (s - bb)) + (x - bb);
+    hi = s;
+}
+
 template <int kDtype>
-__global__ void __launch_bounds__(kTmaThreads, 1)
+__global__ void __launch_bounds__(kTmaThreads, 2)
     k_stream_tma(const __grid_constant__ CUtensorMap map_big, const __grid_constant__ CUtensorMap map_small,
-                 StreamArgs A) {
+                 const __grid_constant__ StreamArgs A) {
     constexpr int kInner = kDtype == 0 ? 32 : 64;          // elements per 128-byte row
     constexpr int kStageRows = kStageCoords / kInner;      // 256 or 128
     constexpr int kStageBytes = kStageRows * kRowBytes;    // 32 KiB or 16 KiB
+    constexpr int kStages = kStageBudget / kStageBytes;    // 3 or 6
     extern __shared__ unsigned char dsm_raw[];
     unsigned char* base = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(dsm_raw) + 1023) & ~uintptr_t(1023));
     uint64_t* full = reinterpret_cast<uint64_t*>(base + kStages * kStageBytes);
@@ -203,8 +213,8 @@ __global__ void __launch_bounds__(kTmaThreads, 1)
         const float nlam = -A.sp[ch.seg].lam_up32, t_c = A.sp[ch.seg].t_c;
         const int64_t row0 = (int64_t)ch.m * Lo.d;          // flat index of the worker row
         const int64_t region = cr.flat_lo;                   // this chunk's list region
-        const PhiloxStream ph(Lo.seed, Lo.step, Lo.worker0 + (uint32_t)ch.m);
-        double acc = 0.0;
+        const PhiloxStream ph(Lo, Lo.worker0 + (uint32_t)ch.m);
+        float acc_hi = 0.0f, acc_lo = 0.0f;
         int runP = 0, runC = 0;
         for (int64_t r0 = cr.r_first; r0 < cr.r_end; r0 += kStageRows, ++it) {
             const int s = (int)(it % kStages);
@@ -221,83 +231,80 @@ __global__ void __launch_bounds__(kTmaThreads, 1)
             const int64_t f0 = (r0 + row) * kInner + (kDtype == 0 ? (h & 1) * 16 : (h & 3) * 16);
             const unsigned char* rp = base + s * kStageBytes + row * kRowBytes;
             const int sw = row & 7;
-            const bool any_valid = live && (f0 < cr.flat_hi) && (f0 + 16 > cr.flat_lo);
+            // Whole stage inside the chunk: every lane's 16 coordinates are valid.
+            const bool stage_whole = r0 * kInner >= cr.flat_lo && (r0 + kStageRows) * kInner <= cr.flat_hi;
+            const bool any_valid = live && (stage_whole || ((f0 < cr.flat_hi) && (f0 + 16 > cr.flat_lo)));
             uint32_t pm = 0, cm = 0;
             float s16 = 0.0f;
             if (any_valid) {
-                float v[16];
-                if (kDtype == 0) {
-#pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        const float4 t = *reinterpret_cast<const float4*>(rp + (((first_chunk + j) ^ sw) << 4));
-                        v[4 * j] = t.x; v[4 * j + 1] = t.y; v[4 * j + 2] = t.z; v[4 * j + 3] = t.w;
-                    }
-                } else {
-#pragma unroll
-                    for (int j = 0; j < 2; ++j) {
-                        const uint4 t = *reinterpret_cast<const uint4*>(rp + (((first_chunk + j) ^ sw) << 4));
-                        const uint32_t u[4] = {t.x, t.y, t.z, t.w};
-#pragma unroll
-                        for (int k = 0; k < 4; ++k) {
-                            v[8 * j + 2 * k] = __uint_as_float(u[k] << 16);
-                            v[8 * j + 2 * k + 1] = __uint_as_float(u[k] & 0xFFFF0000u);
-                        }
-                    }
-                }
                 const uint32_t q0 = (uint32_t)((f0 - row0) >> 2);  // worker-local group of coordinate 0
-                if (f0 >= cr.flat_lo && f0 + 16 <= cr.flat_hi) {
-                    // All 16 coordinates belong to the chunk.
+                if (stage_whole || (f0 >= cr.flat_lo && f0 + 16 <= cr.flat_hi)) {
+                    // All 16 coordinates belong to the chunk: one group of 4 at a time.
                     float s4[4];
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
-                        const float a0 = fabsf(v[4 * j]), a1 = fabsf(v[4 * j + 1]);
-                        const float a2 = fabsf(v[4 * j + 2]), a3 = fabsf(v[4 * j + 3]);
+                        float a0, a1, a2, a3;
+                        if (kDtype == 0) {
+                            const float4 t = *reinterpret_cast<const float4*>(rp + (((first_chunk + j) ^ sw) << 4));
+                            a0 = fabsf(t.x); a1 = fabsf(t.y); a2 = fabsf(t.z); a3 = fabsf(t.w);
+                        } else {
+                            const uint2 t = *reinterpret_cast<const uint2*>(
+                                rp + (((first_chunk + (j >> 1)) ^ sw) << 4) + ((j & 1) << 3));
+                            a0 = fabsf(__uint_as_float(t.x << 16));
+                            a1 = fabsf(__uint_as_float(t.x & 0xFFFF0000u));
+                            a2 = fabsf(__uint_as_float(t.y << 16));
+                            a3 = fabsf(__uint_as_float(t.y & 0xFFFF0000u));
+                        }
                         s4[j] = (a0 + a1) + (a2 + a3);
                         if (build_p) {
                             // candidate iff (1 + u) - lam_up |g| < 1 + 2^-20
                             const uint4 w = ph.words(q0 + j);
-                            pm |= lt_mask(fmaf(nlam, a0, unit_plus_one(w.x)), pbias) & (1u << (4 * j));
-                            pm |= lt_mask(fmaf(nlam, a1, unit_plus_one(w.y)), pbias) & (2u << (4 * j));
-                            pm |= lt_mask(fmaf(nlam, a2, unit_plus_one(w.z)), pbias) & (4u << (4 * j));
-                            pm |= lt_mask(fmaf(nlam, a3, unit_plus_one(w.w)), pbias) & (8u << (4 * j));
+                            pm = or_and(pm, lt_mask(fmaf(nlam, a0, unit_plus_one(w.x)), pbias), 1u << (4 * j));
+                            pm = or_and(pm, lt_mask(fmaf(nlam, a1, unit_plus_one(w.y)), pbias), 2u << (4 * j));
+                            pm = or_and(pm, lt_mask(fmaf(nlam, a2, unit_plus_one(w.z)), pbias), 4u << (4 * j));
+                            pm = or_and(pm, lt_mask(fmaf(nlam, a3, unit_plus_one(w.w)), pbias), 8u << (4 * j));
                         }
                     }
                     s16 = (s4[0] + s4[1]) + (s4[2] + s4[3]);
                     if (!(s16 < t_c)) {
                         // Some |g| may reach t_c (or be non-finite): split exactly.
-                        float m[16];
 #pragma unroll
-                        for (int k = 0; k < 16; ++k) {
-                            const float a = fabsf(v[k]);
-                            const bool in_c = !(a < t_c);
-                            cm |= in_c ? (1u << k) : 0u;
-                            m[k] = in_c ? 0.0f : a;
+                        for (int j = 0; j < 4; ++j) {
+                            float m4[4];
+#pragma unroll
+                            for (int k = 0; k < 4; ++k) {
+                                const float a = fabsf(stage_value<kDtype>(rp, first_chunk, sw, 4 * j + k));
+                                const bool in_c = !(a < t_c);
+                                cm |= in_c ? (1u << (4 * j + k)) : 0u;
+                                m4[k] = in_c ? 0.0f : a;
+                            }
+                            s4[j] = (m4[0] + m4[1]) + (m4[2] + m4[3]);
                         }
-                        s16 = (((m[0] + m[1]) + (m[2] + m[3])) + ((m[4] + m[5]) + (m[6] + m[7]))) +
-                              (((m[8] + m[9]) + (m[10] + m[11])) + ((m[12] + m[13]) + (m[14] + m[15])));
+                        s16 = (s4[0] + s4[1]) + (s4[2] + s4[3]);
                     }
                 } else {
                     // The lane straddles an edge of the chunk: test each coordinate.
-                    float m[16];
+                    float s4[4];
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
                         const uint4 w = build_p ? ph.words(q0 + j) : make_uint4(0, 0, 0, 0);
+                        float m4[4];
 #pragma unroll
                         for (int k = 0; k < 4; ++k) {
                             const int e = 4 * j + k;
                             const bool valid = f0 + e >= cr.flat_lo && f0 + e < cr.flat_hi;
-                            const float a = fabsf(v[e]);
+                            const float a = valid ? fabsf(stage_value<kDtype>(rp, first_chunk, sw, e)) : 0.0f;
                             const bool in_c = valid && !(a < t_c);
-                            m[e] = (valid && !in_c) ? a : 0.0f;
+                            m4[k] = (valid && !in_c) ? a : 0.0f;
                             cm |= in_c ? (1u << e) : 0u;
                             if (build_p && valid && fmaf(nlam, a, unit_plus_one(word_of(w, k))) < pbias) pm |= 1u << e;
                         }
+                        s4[j] = (m4[0] + m4[1]) + (m4[2] + m4[3]);
                     }
-                    s16 = (((m[0] + m[1]) + (m[2] + m[3])) + ((m[4] + m[5]) + (m[6] + m[7]))) +
-                          (((m[8] + m[9]) + (m[10] + m[11])) + ((m[12] + m[13]) + (m[14] + m[15])));
+                    s16 = (s4[0] + s4[1]) + (s4[2] + s4[3]);
                 }
             }
-            acc += (double)s16;
+            two_sum_add(acc_hi, acc_lo, s16);
 
             // Order the stage's candidates: lane scan, then the warps' totals by shuffle.
             const uint32_t packed = (uint32_t)__popc(pm) | ((uint32_t)__popc(cm) << 16);
@@ -342,9 +349,16 @@ __global__ void __launch_bounds__(kTmaThreads, 1)
             runC += (int)(wall >> 16);
             par ^= 1;
         }
-        // Chunk totals: per-warp l1 partials summed in warp order.
-        const double wsum = warp_sum(acc);
-        if (lane == 0) sl[cw] = wsum;
+        // Chunk totals: the lanes' (hi, lo) pairs reduced error-free across the
+        // warp, then the warps' partials summed in warp order in fp64.
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const float oh = __shfl_xor_sync(0xFFFFFFFFu, acc_hi, o);
+            const float ol = __shfl_xor_sync(0xFFFFFFFFu, acc_lo, o);
+            two_sum_add(acc_hi, acc_lo, oh);
+            acc_lo += ol;
+        }
+        if (lane == 0) sl[cw] = (double)acc_hi + (double)acc_lo;
         consumer_bar();
         if (cw == 0 && lane == 0) {
             double t = 0.0;
@@ -395,6 +409,7 @@ template <int kDtype>
 size_t tma_smem_bytes() {
     constexpr int kInner = kDtype == 0 ? 32 : 64;
     constexpr int kStageBytes = (kStageCoords / kInner) * kRowBytes;
+    constexpr int kStages = kStageBudget / kStageBytes;
     return 1024 + (size_t)kStages * kStageBytes + 2 * kStages * 8 + 2 * kCW * 4 + kCW * 8 + 16;
 }
 
@@ -438,7 +453,7 @@ cudaError_t launch_stream_tma(const Layout& Lo, const SegParam* sp, const Lists&
     A.Ls = Ls;
     A.n_chunks = n_chunks;
     A.status = status;
-    const int grid = std::min(n_chunks, sm_count_tma());
+    const int grid = std::min(n_chunks, 2 * sm_count_tma());
     cudaError_t e;
     TraceScope ts(kKStreamTma, st);
     if (Lo.dtype == 0) {
