@@ -212,6 +212,9 @@ def run_gpu(args):
     stream = torch.cuda.current_stream(dev)
 
     def step(t):
+        if off is None and not args.separate:
+            gs.gs_sparsify_aggregate(g, kappa, w.iters, w.seed, t, 0, idx, val, nnz, out, stream=stream)
+            return
         if off is None:
             gs.gs_batched_sparsify(g, kappa, w.iters, w.seed, t, 0, idx, val, nnz, stream=stream)
         else:
@@ -285,6 +288,8 @@ def run_gpu(args):
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": dtype, "data": "synthetic",
         "config": {"workload": w.name, "M": M, "d": d, "kappa": kappa, "iters": w.iters, "dtype": dtype,
+                   "api": ("gs_segmented_sparsify + gs_sparse_aggregate" if off is not None else
+                           "gs_batched_sparsify + gs_sparse_aggregate" if args.separate else "gs_sparsify_aggregate"),
                    "parallelism": f"replicas{ws}", "l2": "inputs exceed L2 (%.2f GB of g per step)" % (M * d * esz / 1e9)},
         "hbm_gbs_pipeline": round(pipe_gbs, 1),
         "pipeline_roofline": {"bound": "hbm", "algorithmic_bytes": b_sp + b_ag, "achieved": round(pipe_gbs, 1),
@@ -459,6 +464,8 @@ def main(argv=None):
     ap.add_argument("--dtype", default=None, choices=[None, "f32", "bf16"])
     ap.add_argument("--workers", type=int, default=None, help="override M (reduced case for profiling)")
     ap.add_argument("--dim", type=int, default=None, help="override d (reduced case for profiling)")
+    ap.add_argument("--separate", action="store_true",
+                    help="time gs_batched_sparsify + gs_sparse_aggregate as two calls instead of gs_sparsify_aggregate")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-cpu-baseline", action="store_true")

@@ -153,8 +153,20 @@ gs_status gs_sparse_aggregate(const int32_t* const* idx, const float* const* val
                               float* out, void* stream);
 
 /*
+ * The whole path for M workers in one call (Algorithm 1, steps 4-6):
+ * gs_batched_sparsify, then the worker-order fp32 sum of the M sparse vectors
+ * into `out` (device, d fp32, overwritten), exactly as gs_sparse_aggregate
+ * would compute it.  The sum reuses the sparsify pass's per-chunk output
+ * offsets as its tile table, so it makes no extra pass over the codes.
+ * Arguments as in gs_batched_sparsify plus `out`; 1 <= M <= 512.
+ */
+gs_status gs_sparsify_aggregate(const void* g, int dtype, int M, int64_t d, double kappa, int iters, uint64_t seed,
+                                uint32_t step, uint32_t worker0, int32_t* idx, float* val, int32_t* nnz, int64_t cap,
+                                gs_info* info, float* out, void* stream);
+
+/*
  * The whole path for M workers with HOST buffers: copies g_host (M x d,
- * `dtype`) to the device, runs gs_batched_sparsify and gs_sparse_aggregate,
+ * `dtype`) to the device, runs gs_sparsify_aggregate,
  * and copies the dense sum back to out_host (d fp32) and the kept counts to
  * nnz_host (M int32).  g_dev / idx / val / nnz / out are caller-owned device
  * buffers of the sizes gs_batched_sparsify / gs_sparse_aggregate require

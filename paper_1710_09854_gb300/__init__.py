@@ -24,7 +24,7 @@ GS_OPT_FORCE_EXACT_SOLVE, GS_OPT_SAMPLE_SIZE, GS_OPT_KERNEL_TIMING, GS_OPT_STREA
 # Symbols include/gs.h declares (checked by the tests).
 EXPORTS = ("gs_status_string", "gs_last_error", "gs_version", "gs_sync_status", "gs_probabilities", "gs_probabilities_ex",
            "gs_sparsify", "gs_batched_sparsify", "gs_segmented_sparsify", "gs_sparse_aggregate",
-           "gs_pipeline_host", "gs_random_words", "gs_set_option", "gs_kernel_count", "gs_kernel_name",
+           "gs_sparsify_aggregate", "gs_pipeline_host", "gs_random_words", "gs_set_option", "gs_kernel_count", "gs_kernel_name",
            "gs_kernel_times")
 
 
@@ -65,6 +65,7 @@ def lib():
             "gs_segmented_sparsify": ([vp, i32, i32, i64, vp, i32, dbl, i32, u64, u32, u32, vp, vp, vp, i64, vp, vp],
                                       i32),
             "gs_sparse_aggregate": ([vp, vp, vp, i32, i64, vp, vp], i32),
+            "gs_sparsify_aggregate": ([vp, i32, i32, i64, dbl, i32, u64, u32, u32, vp, vp, vp, i64, vp, vp, vp], i32),
             "gs_pipeline_host": ([vp, i32, i32, i64, dbl, i32, u64, u32, u32, vp, vp, vp, vp, i64, vp, vp, vp, vp],
                                  i32),
             "gs_random_words": ([u64, u32, u32, i64, i64, vp, vp], i32),
@@ -235,6 +236,20 @@ def gs_sparse_aggregate(idx_list, val_list, nnz, d, out, stream=None):
     vp = (ctypes.c_void_p * M)(*[_ptr(x, "val", (torch.float32,)) for x in val_list])
     _check(lib().gs_sparse_aggregate(ip, vp, _ptr(nnz, "nnz", (torch.int32,)), M, int(d),
                                      _ptr(out, "out", (torch.float32,)), _stream(stream)), "gs_sparse_aggregate")
+
+
+def gs_sparsify_aggregate(g, kappa, iters, seed, step, worker0, idx, val, nnz, out, info=None, stream=None):
+    """gs_batched_sparsify of g (M, d) into idx / val / nnz plus the dense sum into out (d,)."""
+    import torch
+    M, d = g.shape
+    cap = idx.shape[1]
+    if idx.shape[0] != M or tuple(val.shape) != tuple(idx.shape) or nnz.numel() != M or out.numel() != d:
+        raise ValueError("idx / val must be (M, cap), nnz (M,), out (d,)")
+    _check(lib().gs_sparsify_aggregate(_ptr(g, "g"), _g_dtype(g), M, d, float(kappa), int(iters), int(seed),
+                                       int(step), int(worker0), _ptr(idx, "idx", (torch.int32,)),
+                                       _ptr(val, "val", (torch.float32,)), _ptr(nnz, "nnz", (torch.int32,)), cap,
+                                       _ptr(info, "info"), _ptr(out, "out", (torch.float32,)), _stream(stream)),
+           "gs_sparsify_aggregate")
 
 
 def gs_pipeline_host(g_host, kappa, iters, seed, step, worker0, g_dev, idx, val, nnz, out, out_host, nnz_host,

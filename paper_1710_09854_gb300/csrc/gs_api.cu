@@ -146,7 +146,7 @@ void carve(Arena& a, Workspace& w, int n_seg, int n_chunks, int64_t n, bool buil
 // Shared driver of every sparsify / probabilities call.
 gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off, int L, double kappa, int iters,
               uint64_t seed, uint32_t step, uint32_t worker0, int32_t* idx, float* val, int32_t* nnz, int64_t cap,
-              gs_info* info, float* p, cudaStream_t st) {
+              gs_info* info, float* p, cudaStream_t st, float* agg_out = nullptr) {
     const bool prob = p != nullptr;
     if (!g || M < 1 || d < 1 || d >= kMaxD || bad_kappa(kappa) || iters < 0) return GS_ERR_INVALID_ARG;
     if (dtype != GS_DTYPE_F32 && dtype != GS_DTYPE_BF16) return GS_ERR_INVALID_ARG;
@@ -227,6 +227,20 @@ gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off
     if (e == cudaSuccess) {
         if (prob) e = launch_prob(Lo, w.sp, p, st);
         else e = launch_compact(Lo, w.sp, w.ls, n_chunks, idx, val, nnz, cap, s->status, st);
+    }
+    if (e == cudaSuccess && agg_out) {
+        // The sum of the M rows just written, tiled by the chunks (L == 1).
+        AggArgs A;
+        std::memset(&A, 0, sizeof(A));
+        for (int m = 0; m < M; ++m) {
+            A.idx[m] = idx + (size_t)m * (size_t)cap;
+            A.val[m] = val + (size_t)m * (size_t)cap;
+        }
+        A.nnz = nnz;
+        A.M = M;
+        A.d = d;
+        A.cap = cap;
+        e = launch_aggregate_chunks(A, w.ls.k_off, Lo.cpw, agg_out, st);
     }
     cudaError_t ef = cudaFreeAsync(mem, st);
     if (e != cudaSuccess) return cuda_fail(launch_error_site(), e);
@@ -339,6 +353,14 @@ gs_status gs_sparse_aggregate(const int32_t* const* idx, const float* const* val
     return run_aggregate(idx, val, nnz, M, d, out, INT64_MAX, static_cast<cudaStream_t>(stream));
 }
 
+gs_status gs_sparsify_aggregate(const void* g, int dtype, int M, int64_t d, double kappa, int iters, uint64_t seed,
+                                uint32_t step, uint32_t worker0, int32_t* idx, float* val, int32_t* nnz, int64_t cap,
+                                gs_info* info, float* out, void* stream) {
+    if (!out || M < 1 || M > kMaxAggM) return GS_ERR_INVALID_ARG;
+    return run(g, dtype, M, d, nullptr, 1, kappa, iters, seed, step, worker0, idx, val, nnz, cap, info, nullptr,
+               static_cast<cudaStream_t>(stream), out);
+}
+
 gs_status gs_pipeline_host(const void* g_host, int dtype, int M, int64_t d, double kappa, int iters, uint64_t seed,
                            uint32_t step, uint32_t worker0, void* g_dev, int32_t* idx, float* val, int32_t* nnz,
                            int64_t cap, float* out, float* out_host, int32_t* nnz_host, void* stream) {
@@ -348,16 +370,8 @@ gs_status gs_pipeline_host(const void* g_host, int dtype, int M, int64_t d, doub
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     const size_t esz = dtype == GS_DTYPE_F32 ? 4 : 2;
     GS_TRY(cudaMemcpyAsync(g_dev, g_host, esz * (size_t)M * (size_t)d, cudaMemcpyHostToDevice, st));
-    gs_status rc = run(g_dev, dtype, M, d, nullptr, 1, kappa, iters, seed, step, worker0, idx, val, nnz, cap, nullptr,
-                       nullptr, st);
-    if (rc != GS_OK) return rc;
-    std::vector<const int32_t*> ip(M);
-    std::vector<const float*> vp(M);
-    for (int m = 0; m < M; ++m) {
-        ip[m] = idx + (size_t)m * (size_t)cap;
-        vp[m] = val + (size_t)m * (size_t)cap;
-    }
-    rc = run_aggregate(ip.data(), vp.data(), nnz, M, d, out, cap, st);
+    const gs_status rc = run(g_dev, dtype, M, d, nullptr, 1, kappa, iters, seed, step, worker0, idx, val, nnz, cap,
+                             nullptr, nullptr, st, out);
     if (rc != GS_OK) return rc;
     GS_TRY(cudaMemcpyAsync(out_host, out, sizeof(float) * (size_t)d, cudaMemcpyDeviceToHost, st));
     GS_TRY(cudaMemcpyAsync(nnz_host, nnz, sizeof(int32_t) * (size_t)M, cudaMemcpyDeviceToHost, st));

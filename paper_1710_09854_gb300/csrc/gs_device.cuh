@@ -298,12 +298,79 @@ __device__ __forceinline__ T block_sum(T v, T* sh) {
     return sh[32];
 }
 
+// Error-free fp32 accumulation (Knuth's TwoSum): hi + lo carries the exact
+// running sum to ~2^-48 without touching the fp64 pipe.
+__device__ __forceinline__ void two_sum_add(float& hi, float& lo, float x) {
+    const float s = hi + x;
+    const float bb = s - hi;
+    lo += (hi - (s - bb)) + (x - bb);
+    hi = s;
+}
+
+// (hi, lo) += (bh, bl) for two double-float values, renormalised.
+__device__ __forceinline__ void df_add(float& hi, float& lo, float bh, float bl) {
+    const float s = hi + bh;
+    const float bb = s - hi;
+    const float err = (hi - (s - bb)) + (bh - bb);
+    const float l = (lo + bl) + err;
+    const float t = s + l;
+    lo = l - (t - s);
+    hi = t;
+}
+
+// Sum of double-float values and of ints over the block (butterfly inside
+// warps, warps in order); every thread gets the result.
+__device__ __forceinline__ void block_sum_df(float& hi, float& lo, int& k, float4* sh) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float oh = __shfl_xor_sync(0xFFFFFFFFu, hi, o);
+        const float ol = __shfl_xor_sync(0xFFFFFFFFu, lo, o);
+        df_add(hi, lo, oh, ol);
+        k += __shfl_xor_sync(0xFFFFFFFFu, k, o);
+    }
+    __syncthreads();
+    if (lane == 0) sh[warp] = make_float4(hi, lo, __int_as_float(k), 0.0f);
+    __syncthreads();
+    if (warp == 0) {
+        float4 t = lane < nw ? sh[lane] : make_float4(0.0f, 0.0f, __int_as_float(0), 0.0f);
+        float h = t.x, l = t.y;
+        int kk = __float_as_int(t.z);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            const float oh = __shfl_xor_sync(0xFFFFFFFFu, h, o);
+            const float ol = __shfl_xor_sync(0xFFFFFFFFu, l, o);
+            df_add(h, l, oh, ol);
+            kk += __shfl_xor_sync(0xFFFFFFFFu, kk, o);
+        }
+        if (lane == 0) sh[32] = make_float4(h, l, __int_as_float(kk), 0.0f);
+    }
+    __syncthreads();
+    hi = sh[32].x;
+    lo = sh[32].y;
+    k = __float_as_int(sh[32].z);
+}
+
 // Smallest positive fp32 a with fl64(lam * a) >= 1; +inf when no finite
 // float qualifies (lam = 0 or lam * FLT_MAX < 1).  fl64(lam * a) is
 // monotone in a, so "fl64(lam*|g|) >= 1" is exactly "|g| >= a_cap".
 __device__ __forceinline__ float cap_threshold(double lam) {
     if (!(lam > 0.0)) return __int_as_float(0x7F800000);
     if (lam * 3.4028234663852886e38 < 1.0) return __int_as_float(0x7F800000);
+    // Start from an fp32 reciprocal and step one ulp at a time (a few fp64
+    // products); fall back to a bisection over the float bit patterns.
+    const float f = (float)lam;
+    if (f > 0.0f && f < 3.0e38f) {
+        uint32_t b = __float_as_uint(__frcp_rn(f));
+        if (b > 0u && b < 0x7F7FFFFFu) {
+            int guard = 0;
+            while (lam * (double)__uint_as_float(b) < 1.0 && b < 0x7F7FFFFFu && ++guard < 16) ++b;
+            while (b > 1u && lam * (double)__uint_as_float(b - 1u) >= 1.0 && ++guard < 32) --b;
+            if (lam * (double)__uint_as_float(b) >= 1.0 &&
+                (b == 1u || lam * (double)__uint_as_float(b - 1u) < 1.0))
+                return __uint_as_float(b);
+        }
+    }
     uint32_t lo = 0, hi = 0x7F7FFFFFu;   // search the bit patterns of finite positive floats
     while (lo < hi) {
         uint32_t mid = lo + ((hi - lo) >> 1);

@@ -467,18 +467,17 @@ struct CView {
     }
 };
 
-// (#{a >= acap}, sum of the other a) over C; NaN acap sums everything.
-__device__ double2 c_stats(const CView& C, float acap, double2* sh2) {
-    double acc = 0.0;
-    float part = 0.0f;
-    int k = 0, run = 0;
+// (#{a >= acap}, sum of the other a) over C; NaN acap sums everything.  The
+// sum is carried error-free in fp32 pairs, so no fp64 arithmetic per value.
+__device__ double2 c_stats(const CView& C, float acap, float4* sh4) {
+    float hi = 0.0f, lo = 0.0f;
+    int k = 0;
     for (int e = threadIdx.x; e < C.nC; e += blockDim.x) {
         const float a = C.at(e);
-        if (a >= acap) ++k; else part += a;
-        if (++run == 16) { acc += (double)part; part = 0.0f; run = 0; }
+        if (a >= acap) ++k; else two_sum_add(hi, lo, a);
     }
-    acc += (double)part;
-    return block_sum2((double)k, acc, sh2);
+    block_sum_df(hi, lo, k, sh4);
+    return make_double2((double)k, (double)hi + (double)lo);
 }
 
 __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lists Ls, double kappa, int iters,
@@ -486,7 +485,7 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
     extern __shared__ unsigned char dsm[];
     int32_t* spre = reinterpret_cast<int32_t*>(dsm);                       // kSolveSmemChunks + 1
     float* sc = reinterpret_cast<float*>(dsm + sizeof(int32_t) * (kSolveSmemChunks + 4));  // kSolveSmemC
-    __shared__ double2 sh2[33];
+    __shared__ float4 sh4[33];
     __shared__ double shd[33];
     __shared__ int shi[33];
     __shared__ float s_acap;
@@ -519,7 +518,7 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
     double sl = 0.0;
     for (int c = c0 + tid; c < c1; c += blockDim.x) sl += Ls.s_low[c];
     const double S_low = block_sum(sl, shd);
-    const double2 all = c_stats(C, __int_as_float(0x7FC00000), sh2);
+    const double2 all = c_stats(C, __int_as_float(0x7FC00000), sh4);
     double S = S_low + all.y;
 
     double lam = 0.0, K = 0.0, Su = 0.0;
@@ -533,7 +532,7 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
         while (j < iters) {
             if (tid == 0) s_acap = cap_threshold(lam);
             __syncthreads();
-            const double2 r = c_stats(C, s_acap, sh2);
+            const double2 r = c_stats(C, s_acap, sh4);
             const double A = lam * (S_low + r.y);
             if (A == 0.0) break;
             const double cc = (budget - r.x) / A;
@@ -543,7 +542,7 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
         }
         if (tid == 0) s_acap = cap_threshold(lam);
         __syncthreads();
-        const double2 r = c_stats(C, s_acap, sh2);
+        const double2 r = c_stats(C, s_acap, sh4);
         K = r.x;
         Su = S_low + r.y;
         // The lists are exact only while lambda stays within the bound.
@@ -644,6 +643,7 @@ struct Decider {
 // 2016; every wait bounded); pass 2 writes the kept entries in order.
 // ---------------------------------------------------------------------------
 constexpr int kEmitChunks = 8;
+constexpr int kEmitBatch = 8;                           // decision words per warp whose loads are in flight together
 constexpr int kEmitWords = kEmitChunks * kChunk / 32;   // decision words of the largest tile
 constexpr unsigned long long kFlagAgg = 1ull << 62, kFlagInc = 2ull << 62, kValMask = (1ull << 62) - 1;
 constexpr long long kSpinLimit = 1ll << 22;
@@ -699,20 +699,40 @@ __global__ void __launch_bounds__(kThreads) k_emit(const __grid_constant__ Layou
     const int nw = (n + 31) >> 5;
     const PhiloxStream ph(Lo, Lo.worker0 + (uint32_t)m);
 
-    // Pass 1: decisions.  Warp w takes candidates [32 w', 32 w' + 32) for w' = w, w + kWarps, ...
-    for (int wd = warp; wd < nw; wd += kWarps) {
-        const int e = wd * 32 + lane;
-        bool keep = false;
-        if (e < n) {
-            int k = 0;
-            while (k + 1 < nck && s_pre[k + 1] <= e) ++k;
-            const int2 ent = Ls.p_ent[s_region[k] + (e - s_pre[k])];
-            const uint32_t x = word_of(ph.words((uint32_t)ent.x >> 2), ent.x & 3);
-            float v;
-            keep = s_dec[k](__int_as_float(ent.y), x, v);
+    // Pass 1: decisions.  Warp w takes the 32-candidate words w, w + kWarps, ...
+    // in batches of kEmitBatch words whose loads are all issued first.  A tile
+    // that fits one batch keeps its candidates in registers for pass 2.
+    auto chunk_of = [&](int e) -> int {
+        int k = 0;
+#pragma unroll
+        for (int step = kEmitChunks / 2; step > 0; step >>= 1)
+            if (k + step < nck && s_pre[k + step] <= e) k += step;
+        return k;
+    };
+    int2 ent[kEmitBatch];
+    int kk[kEmitBatch];
+    for (int base = 0; base < nw; base += kEmitBatch * kWarps) {
+#pragma unroll
+        for (int b = 0; b < kEmitBatch; ++b) {
+            const int e = (base + b * kWarps + warp) * 32 + lane;
+            kk[b] = -1;
+            if (e < n) {
+                kk[b] = chunk_of(e);
+                ent[b] = Ls.p_ent[s_region[kk[b]] + (e - s_pre[kk[b]])];
+            }
         }
-        const uint32_t bal = __ballot_sync(0xFFFFFFFFu, keep);
-        if (lane == 0) bits[wd] = bal;
+#pragma unroll
+        for (int b = 0; b < kEmitBatch; ++b) {
+            const int wd = base + b * kWarps + warp;
+            bool keep = false;
+            if (kk[b] >= 0) {
+                const uint32_t x = word_of(ph.words((uint32_t)ent[b].x >> 2), ent[b].x & 3);
+                float v;
+                keep = s_dec[kk[b]](__int_as_float(ent[b].y), x, v);
+            }
+            const uint32_t bal = __ballot_sync(0xFFFFFFFFu, keep);
+            if (lane == 0 && wd < nw) bits[wd] = bal;
+        }
     }
     __syncthreads();
     // Kept-count prefix over the decision words (contiguous words per thread).
@@ -792,19 +812,31 @@ __global__ void __launch_bounds__(kThreads) k_emit(const __grid_constant__ Layou
     // Pass 2: kept entries in candidate order (consecutive lanes write consecutive slots).
     const long long prefix = s_prefix;
     const int64_t out0 = (int64_t)m * cap;
-    for (int wd = warp; wd < nw; wd += kWarps) {
-        const uint32_t word = bits[wd];
-        if ((word >> lane) & 1u) {
-            const int e = wd * 32 + lane;
-            int k = 0;
-            while (k + 1 < nck && s_pre[k + 1] <= e) ++k;
-            const int2 ent = Ls.p_ent[s_region[k] + (e - s_pre[k])];
-            const float gv = __int_as_float(ent.y);
-            const float v = fabsf(gv) >= s_dec[k].a_cap ? gv : copysignf(s_dec[k].inv_lam32, gv);
-            const long long pos = prefix + wpre[wd] + __popc(word & ((1u << lane) - 1u));
-            if (pos < cap) {
-                idx[out0 + pos] = ent.x;
-                val[out0 + pos] = v;
+    const bool in_regs = nw <= kEmitBatch * kWarps;
+    for (int base = 0; base < nw; base += kEmitBatch * kWarps) {
+#pragma unroll
+        for (int b = 0; b < kEmitBatch; ++b) {
+            const int wd = base + b * kWarps + warp;
+            if (wd >= nw) continue;
+            const uint32_t word = bits[wd];
+            if ((word >> lane) & 1u) {
+                const int e = wd * 32 + lane;
+                int k;
+                int2 en;
+                if (in_regs) {
+                    k = kk[b];
+                    en = ent[b];
+                } else {
+                    k = chunk_of(e);
+                    en = Ls.p_ent[s_region[k] + (e - s_pre[k])];
+                }
+                const float gv = __int_as_float(en.y);
+                const float v = fabsf(gv) >= s_dec[k].a_cap ? gv : copysignf(s_dec[k].inv_lam32, gv);
+                const long long pos = prefix + wpre[wd] + __popc(word & ((1u << lane) - 1u));
+                if (pos < cap) {
+                    idx[out0 + pos] = en.x;
+                    val[out0 + pos] = v;
+                }
             }
         }
     }
@@ -838,57 +870,73 @@ __global__ void k_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t i
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) k_bucket(const __grid_constant__ AggArgs A, int32_t* off, int nt,
                                                 int* status) {
+    constexpr int kUnroll = 8;   // entries per thread whose loads are in flight together
     const int m = blockIdx.y;
     const int32_t* __restrict__ idx = A.idx[m];
     long long n = A.nnz[m];
     if (n > A.cap) n = A.cap;
     if (n < 0) n = 0;
     int32_t* o = off + (int64_t)m * (nt + 1);
-    for (long long e = (long long)blockIdx.x * blockDim.x + threadIdx.x; e <= n;
-         e += (long long)gridDim.x * blockDim.x) {
-        long long t_cur = nt;
-        if (e < n) {
-            const int32_t i = idx[e];
-            if (i < 0 || (int64_t)i >= A.d) {
-                atomicOr(status, kStInvalid);
-                continue;
-            }
-            t_cur = i / kAggTile;
+    const long long stride = (long long)gridDim.x * blockDim.x;
+    for (long long e0 = (long long)blockIdx.x * blockDim.x + threadIdx.x; e0 <= n; e0 += stride * kUnroll) {
+        int32_t cur[kUnroll], prev[kUnroll];
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+            const long long e = e0 + u * stride;
+            cur[u] = e < n ? idx[e] : 0;
+            prev[u] = (e > 0 && e <= n) ? idx[e - 1] : 0;
         }
-        long long t_prev = -1;
-        if (e > 0) {
-            const int32_t ip = idx[e - 1];
-            if (ip < 0 || (int64_t)ip >= A.d) continue;
-            if (e < n && ip >= idx[e]) {
-                atomicOr(status, kStInvalid);
-                continue;
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+            const long long e = e0 + u * stride;
+            if (e > n) break;
+            long long t_cur = nt;
+            if (e < n) {
+                if (cur[u] < 0 || (int64_t)cur[u] >= A.d) {
+                    atomicOr(status, kStInvalid);
+                    continue;
+                }
+                t_cur = cur[u] / kAggTile;
             }
-            t_prev = ip / kAggTile;
+            long long t_prev = -1;
+            if (e > 0) {
+                if (prev[u] < 0 || (int64_t)prev[u] >= A.d) continue;
+                if (e < n && prev[u] >= cur[u]) {
+                    atomicOr(status, kStInvalid);
+                    continue;
+                }
+                t_prev = prev[u] / kAggTile;
+            }
+            for (long long t = t_prev + 1; t <= t_cur; ++t) o[t] = (int32_t)e;
         }
-        for (long long t = t_prev + 1; t <= t_cur; ++t) o[t] = (int32_t)e;
     }
 }
 
 constexpr int kAggPer = 8;   // entries each thread holds per batch
 
+// Tiles of kTile coordinates.  off[m * off_stride + t] is the first entry of
+// worker m at or after tile t; the end of the last tile is the list length.
+template <int kTile>
 __global__ void __launch_bounds__(kThreads) k_tiles(const __grid_constant__ AggArgs A,
-                                                    const int32_t* __restrict__ off, int nt, float* out) {
-    __shared__ float acc[kAggTile];
+                                                    const int32_t* __restrict__ off, int off_stride, int nt,
+                                                    float* out) {
+    extern __shared__ float acc[];   // kTile floats
     __shared__ int32_t s_pre[kMaxAggM + 1];
     __shared__ long long s_lo[kMaxAggM];
     __shared__ int shi[33];
     __shared__ int32_t s_cnt[kMaxAggM];
     const int M = A.M;
     for (int t = blockIdx.x; t < nt; t += gridDim.x) {
-        const int64_t base = (int64_t)t * kAggTile;
-        const int len = (int)min((int64_t)kAggTile, A.d - base);
-        for (int k = threadIdx.x; k < kAggTile; k += kThreads) acc[k] = 0.0f;
+        const int64_t base = (int64_t)t * kTile;
+        const int len = (int)min((int64_t)kTile, A.d - base);
+        for (int k = threadIdx.x; k < kTile / 4; k += kThreads)
+            reinterpret_cast<float4*>(acc)[k] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
         for (int m = threadIdx.x; m < M; m += kThreads) {
             long long n = A.nnz[m];
             if (n > A.cap) n = A.cap;
             if (n < 0) n = 0;
-            const int32_t* o = off + (int64_t)m * (nt + 1);
-            long long lo = o[t], hi = o[t + 1];
+            const int32_t* o = off + (int64_t)m * off_stride;
+            long long lo = o[t], hi = t + 1 < nt ? o[t + 1] : n;
             lo = lo < 0 ? 0 : (lo > n ? n : lo);
             hi = hi < lo ? lo : (hi > n ? n : hi);
             s_lo[m] = lo;
@@ -923,8 +971,8 @@ __global__ void __launch_bounds__(kThreads) k_tiles(const __grid_constant__ AggA
             }
         }
         float* dst = out + base;
-        if (len == kAggTile && (reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
-            for (int k = threadIdx.x; k < kAggTile / 4; k += kThreads)
+        if (len == kTile && (reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
+            for (int k = threadIdx.x; k < kTile / 4; k += kThreads)
                 reinterpret_cast<float4*>(dst)[k] = reinterpret_cast<const float4*>(acc)[k];
         } else {
             for (int k = threadIdx.x; k < len; k += kThreads) dst[k] = acc[k];
@@ -1012,7 +1060,7 @@ cudaError_t launch_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t 
 }
 
 cudaError_t launch_aggregate(const AggArgs& A, int32_t* off, float* out, int* status, cudaStream_t st) {
-    set_launch_error_site("k_bucket/k_tiles launch");
+    set_launch_error_site("k_bucket launch");
     const int nt = (int)((A.d + kAggTile - 1) / kAggTile);
     // Bucket: a few blocks per worker, grid-stride over its entries.
     const int bx = std::max(1, std::min((sm_count() * 4 + A.M - 1) / A.M, (int)((A.d + 255) / 256 + 1)));
@@ -1023,9 +1071,23 @@ cudaError_t launch_aggregate(const AggArgs& A, int32_t* off, float* out, int* st
     }
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
+    set_launch_error_site("k_tiles launch");
     const int tg = std::min(nt, sm_count() * 4);
     TraceScope ts(kKTiles, st);
-    k_tiles<<<tg, kThreads, 0, st>>>(A, off, nt, out);
+    k_tiles<kAggTile><<<tg, kThreads, kAggTile * sizeof(float), st>>>(A, off, nt + 1, nt, out);
+    return cudaGetLastError();
+}
+
+// The sparse sum straight after a batched sparsify of whole rows: the
+// chunk offsets of k_emit are the tile table (tile = chunk), so no bucket pass.
+cudaError_t launch_aggregate_chunks(const AggArgs& A, const int32_t* k_off, int cpw, float* out, cudaStream_t st) {
+    set_launch_error_site("k_tiles (chunk table) launch");
+    const size_t smem = kChunk * sizeof(float);
+    cudaError_t e = cudaFuncSetAttribute(k_tiles<kChunk>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    const int tg = std::min(cpw, sm_count() * 3);
+    TraceScope ts(kKTiles, st);
+    k_tiles<kChunk><<<tg, kThreads, smem, st>>>(A, k_off, cpw, cpw, out);
     return cudaGetLastError();
 }
 

@@ -36,6 +36,7 @@ cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls
                            float* val, int32_t* nnz, int64_t cap, int* status, cudaStream_t st);
 cudaError_t launch_prob(const Layout& Lo, const SegParam* sp, float* p, cudaStream_t st);
 cudaError_t launch_aggregate(const AggArgs& A, int32_t* off, float* out, int* status, cudaStream_t st);
+cudaError_t launch_aggregate_chunks(const AggArgs& A, const int32_t* k_off, int cpw, float* out, cudaStream_t st);
 cudaError_t launch_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t i0, int64_t n, uint32_t* out,
                          cudaStream_t st);
 bool stream_tma_eligible(const Layout& Lo);

@@ -122,15 +122,6 @@ __device__ __forceinline__ float stage_value(const unsigned char* rp, int first_
 }
 
 // kDtype 0: fp32 rows of 32; 1: bf16 rows of 64.
-// Error-free fp32 accumulation (Knuth's TwoSum): hi + lo carries the exact
-// running sum to ~2^-48, so the per-lane sums never touch the fp64 pipe.
-__device__ __forceinline__ void two_sum_add(float& hi, float& lo, float x) {
-    const float s = hi + x;
-    const float bb = s - hi;
-    lo += (hi - (s - bb)) + (x - bb);
-    hi = s;
-}
-
 template <int kDtype>
 __global__ void __launch_bounds__(kTmaThreads, 2)
     k_stream_tma(const __grid_constant__ CUtensorMap map_big, const __grid_constant__ CUtensorMap map_small,

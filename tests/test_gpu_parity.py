@@ -425,3 +425,44 @@ def test_stream_paths(gs, path, dtype):
             assert times["k_stream"][1] == 2 and times["k_stream_tma"][1] == 0
     finally:
         gs.gs_set_option(gs.GS_OPT_STREAM_PATH, 0)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_sparsify_aggregate_fused(gs, dtype):
+    """gs_sparsify_aggregate equals gs_batched_sparsify + gs_sparse_aggregate
+    bit for bit, and the oracle's worker-order sum."""
+    import torch
+    M, d, kappa, iters, seed, step = 6, 3 * 16384 + 1000, 0.03, 3, 21, 2
+    g_host = np.stack([_vector(k, d, 400 + m) for m, k in enumerate(["t3", "lognormal", "normal"] * 2)])
+    if dtype == "bf16":
+        g_host = workloads.bf16_bits_to_f32(workloads.f32_to_bf16_bits(g_host)).reshape(M, d)
+        g = _dev(workloads.f32_to_bf16_bits(g_host).reshape(M, d)).view(torch.bfloat16)
+    else:
+        g = _dev(g_host)
+    for cap in (d, 700):   # 700 < kept count for some workers: the sum uses only the written entries
+        idx = torch.empty((M, cap), dtype=torch.int32, device="cuda")
+        val = torch.empty((M, cap), dtype=torch.float32, device="cuda")
+        nnz = torch.empty(M, dtype=torch.int32, device="cuda")
+        out = torch.empty(d, dtype=torch.float32, device="cuda")
+        gs.gs_sparsify_aggregate(g, kappa, iters, seed, step, 0, idx, val, nnz, out)
+        rc = gs.gs_sync_status()
+        n = np.minimum(nnz.cpu().numpy(), cap)
+        if cap == d:
+            assert rc == gs.GS_OK
+            out2 = torch.empty(d, dtype=torch.float32, device="cuda")
+            gs.gs_sparse_aggregate([idx[m] for m in range(M)], [val[m] for m in range(M)], nnz, d, out2)
+            assert gs.gs_sync_status() == gs.GS_OK
+            assert torch.equal(out, out2)
+            il, vl = [], []
+            for m in range(M):
+                ri, rv, _ = oracle.sparsify(g_host[m], kappa, iters, seed, step, m)
+                compare_sparse(idx[m, :n[m]].cpu().numpy(), val[m, :n[m]].cpu().numpy(), g_host[m], kappa, iters,
+                               seed, step, m, ref=(ri, rv, oracle.greedy_lambda(g_host[m], kappa, iters)))
+                il.append(ri)
+                vl.append(rv)
+            compare_sum(out.cpu().numpy(), il, vl, d)
+        else:
+            assert rc == gs.GS_ERR_CAPACITY
+            il = [idx[m, :n[m]].cpu().numpy() for m in range(M)]
+            vl = [val[m, :n[m]].cpu().numpy() for m in range(M)]
+            np.testing.assert_array_equal(out.cpu().numpy(), oracle.aggregate(il, vl, d))
