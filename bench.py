@@ -444,7 +444,8 @@ def run_reference(args):
     res = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-           "config": {"workload": w.name, "M": w.M, "d": w.d, "kappa": kappa, "iters": w.iters},
+           "config": {"workload": w.name, "M": w.M, "d": w.d, "kappa": kappa, "iters": w.iters, "dtype": w.dtype,
+                      "api": "oracle (C, fp64)", "parallelism": f"replicas{ws}"},
            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     if ws > 1:
