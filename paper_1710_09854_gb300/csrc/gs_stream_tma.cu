@@ -34,10 +34,11 @@
 namespace gs {
 namespace {
 
-constexpr int kCW = 16;                        // consumer warps
+constexpr int kCW = 8;                         // consumer warps
 constexpr int kTmaThreads = 32 * (kCW + 1);
-constexpr int kStageCoords = kCW * 32 * 16;    // 8192 coordinates per stage
-constexpr int kStageBudget = 96 * 1024;          // shared memory for the ring of one CTA (2 CTAs per SM)
+constexpr int kLaneCoords = 32;                // coordinates per lane per stage
+constexpr int kStageCoords = kCW * 32 * kLaneCoords;   // 8192 coordinates per stage
+constexpr int kStageBudget = 96 * 1024;        // shared memory for the ring of one CTA (2 CTAs per SM)
 constexpr int kRowBytes = 128;
 constexpr int kSmallRows = 8;                  // rows per box of a partial stage (1 KiB)
 constexpr long long kWaitLimit = 1ll << 22;    // try_wait polls before giving up
@@ -89,25 +90,7 @@ __device__ __forceinline__ void consumer_bar() {
     asm volatile("bar.sync 1, %0;" ::"n"(kCW * 32) : "memory");
 }
 
-// Rows of the chunk: [r_first, r_end) of the 128-byte-row view.
-struct ChunkRows {
-    Chunk ch;
-    int64_t flat_lo, flat_hi;
-    int64_t r_first, r_end;
-};
-
-template <int kInner>
-__device__ __forceinline__ ChunkRows chunk_rows(const Layout& Lo, int c) {
-    ChunkRows r;
-    r.ch = decode_chunk(Lo, c);
-    r.flat_lo = (int64_t)r.ch.m * Lo.d + r.ch.lo;
-    r.flat_hi = (int64_t)r.ch.m * Lo.d + r.ch.hi;
-    r.r_first = r.flat_lo / kInner;
-    r.r_end = (r.flat_hi + kInner - 1) / kInner;
-    return r;
-}
-
-// Coordinate k (0..15) of a lane's 16, read back from its row of the stage
+// Coordinate k (0..31) of a lane's 32, read back from its row of the stage
 // buffer (first_chunk: the lane's first 16-byte chunk; sw: the row's swizzle).
 template <int kDtype>
 __device__ __forceinline__ float stage_value(const unsigned char* rp, int first_chunk, int sw, int k) {
@@ -120,6 +103,59 @@ __device__ __forceinline__ float stage_value(const unsigned char* rp, int first_
         return __uint_as_float((uint32_t)b << 16);
     }
 }
+
+// Group j (0..7, four coordinates) of a lane's 32 as |g| values.
+template <int kDtype>
+__device__ __forceinline__ float4 stage_group(const unsigned char* rp, int first_chunk, int sw, int j) {
+    if (kDtype == 0) {
+        const float4 t = *reinterpret_cast<const float4*>(rp + (((first_chunk + j) ^ sw) << 4));
+        return make_float4(fabsf(t.x), fabsf(t.y), fabsf(t.z), fabsf(t.w));
+    } else {
+        const uint2 t = *reinterpret_cast<const uint2*>(rp + (((first_chunk + (j >> 1)) ^ sw) << 4) + ((j & 1) << 3));
+        return make_float4(fabsf(__uint_as_float(t.x << 16)), fabsf(__uint_as_float(t.x & 0xFFFF0000u)),
+                           fabsf(__uint_as_float(t.y << 16)), fabsf(__uint_as_float(t.y & 0xFFFF0000u)));
+    }
+}
+
+// The chunks of one CTA (c = blockIdx.x, + gridDim.x, ...), with the
+// worker and chunk-within-worker advanced without divisions.
+struct ChunkWalk {
+    int c, m, k, dm, dk;
+    __device__ __forceinline__ explicit ChunkWalk(const Layout& Lo) {
+        c = blockIdx.x;
+        m = c / Lo.cpw;
+        k = c - m * Lo.cpw;
+        dm = gridDim.x / Lo.cpw;
+        dk = gridDim.x - dm * Lo.cpw;
+    }
+    __device__ __forceinline__ void next(const Layout& Lo) {
+        c += gridDim.x;
+        m += dm;
+        k += dk;
+        if (k >= Lo.cpw) {
+            k -= Lo.cpw;
+            ++m;
+        }
+    }
+    // The chunk's segment and worker-local range [lo, hi).
+    __device__ __forceinline__ void range(const Layout& Lo, int& seg, int64_t& lo, int64_t& hi) const {
+        int l = 0;
+        if (Lo.L == 1) {
+            lo = (int64_t)k * kChunk;
+            hi = min(Lo.d, lo + kChunk);
+        } else {
+            int a = 0, b = Lo.L - 1;
+            while (a < b) {
+                const int mid = (a + b + 1) >> 1;
+                if (Lo.seg_chunk0[mid] <= k) a = mid; else b = mid - 1;
+            }
+            l = a;
+            lo = Lo.seg_off[a] + (int64_t)(k - Lo.seg_chunk0[a]) * kChunk;
+            hi = min(Lo.seg_off[a + 1], lo + kChunk);
+        }
+        seg = m * Lo.L + l;
+    }
+};
 
 // kDtype 0: fp32 rows of 32; 1: bf16 rows of 64.
 template <int kDtype>
@@ -135,7 +171,7 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
     uint64_t* full = reinterpret_cast<uint64_t*>(base + kStages * kStageBytes);
     uint64_t* empty = full + kStages;
     uint32_t* tot = reinterpret_cast<uint32_t*>(empty + kStages);  // [2][kCW] packed (P | C << 16)
-    double* sl = reinterpret_cast<double*>(tot + 2 * kCW);           // [kCW]
+    float2* sl = reinterpret_cast<float2*>(tot + 2 * kCW);         // [kCW] double-float l1 partials
     volatile int* abort_flag = reinterpret_cast<volatile int*>(sl + kCW);
 
     const Layout& Lo = A.Lo;
@@ -153,13 +189,17 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
     if (warp == 0) {
         // ------------------------------------------------------------ producer
         if (lane != 0) return;
-        long long it = 0;
-        bool ok = true;
-        for (int c = blockIdx.x; c < A.n_chunks && ok; c += gridDim.x) {
-            const ChunkRows cr = chunk_rows<kInner>(Lo, c);
-            for (int64_t r0 = cr.r_first; r0 < cr.r_end && ok; r0 += kStageRows, ++it) {
-                const int s = (int)(it % kStages);
-                if (it >= kStages && !mbar_wait(&empty[s], (uint32_t)(((it / kStages) - 1) & 1))) {
+        int issued = 0, s = 0;
+        uint32_t empty_parity = 0;
+        bool wrapped = false, ok = true;
+        for (ChunkWalk cw(Lo); cw.c < A.n_chunks && ok; cw.next(Lo)) {
+            int seg;
+            int64_t lo, hi;
+            cw.range(Lo, seg, lo, hi);
+            const int64_t flat_lo = (int64_t)cw.m * Lo.d + lo, flat_hi = (int64_t)cw.m * Lo.d + hi;
+            const int64_t r_first = flat_lo / kInner, r_end = (flat_hi + kInner - 1) / kInner;
+            for (int64_t r0 = r_first; r0 < r_end; r0 += kStageRows) {
+                if (wrapped && !mbar_wait(&empty[s], empty_parity)) {
                     ok = false;
                     break;
                 }
@@ -167,7 +207,7 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
                     ok = false;
                     break;
                 }
-                const int rows = (int)std::min<int64_t>(kStageRows, cr.r_end - r0);
+                const int rows = (int)min((int64_t)kStageRows, r_end - r0);
                 unsigned char* dst = base + s * kStageBytes;
                 if (rows == kStageRows) {
                     mbar_arrive_tx(&full[s], kStageBytes);
@@ -179,6 +219,12 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
                         tma_load_rows(dst + b * kSmallRows * kRowBytes, &map_small, (int)(r0 + b * kSmallRows),
                                       &full[s]);
                 }
+                ++issued;
+                if (++s == kStages) {
+                    s = 0;
+                    if (wrapped) empty_parity ^= 1u;
+                    wrapped = true;
+                }
             }
         }
         if (!ok) {
@@ -186,81 +232,73 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
             atomicOr(A.status, kStTimeout);
         }
         // Drain: every issued stage's copy must have landed before the CTA may exit.
-        for (long long k = it - 1; k >= 0 && k >= it - kStages; --k)
+        for (int k = issued - 1; k >= 0 && k >= issued - kStages; --k)
             mbar_wait(&full[k % kStages], (uint32_t)((k / kStages) & 1));
         return;
     }
 
     // ---------------------------------------------------------------- consumers
-    const int cw = warp - 1;
+    const int cwp = warp - 1;
     const float pbias = 1.0f + 0x1p-20f;
     // Probability-only calls keep no keep-candidate lists (their pointer is NULL).
     const bool build_p = A.Ls.p_ent != nullptr;
-    long long it = 0;
-    int par = 0;
-    for (int c = blockIdx.x; c < A.n_chunks; c += gridDim.x) {
-        const ChunkRows cr = chunk_rows<kInner>(Lo, c);
-        const Chunk& ch = cr.ch;
-        const float nlam = -A.sp[ch.seg].lam_up32, t_c = A.sp[ch.seg].t_c;
-        const int64_t row0 = (int64_t)ch.m * Lo.d;          // flat index of the worker row
-        const int64_t region = cr.flat_lo;                   // this chunk's list region
-        const PhiloxStream ph(Lo, Lo.worker0 + (uint32_t)ch.m);
+    // This lane's 32 coordinates of every stage: one 128-byte row (fp32) or half of one (bf16).
+    const int h = cwp * 32 + lane;
+    const int row = kDtype == 0 ? h : (h >> 1);
+    const int first_chunk = kDtype == 0 ? 0 : (h & 1) * 4;
+    const int lane_off = row * kInner + (kDtype == 0 ? 0 : (h & 1) * 32);   // within the stage
+    const int sw = row & 7;
+    int s = 0, par = 0;
+    uint32_t full_parity = 0;
+    for (ChunkWalk cw(Lo); cw.c < A.n_chunks; cw.next(Lo)) {
+        int seg;
+        int64_t lo, hi;
+        cw.range(Lo, seg, lo, hi);
+        const int c = cw.c;
+        const float nlam = -A.sp[seg].lam_up32, t_c = A.sp[seg].t_c;
+        const int64_t flat_lo = (int64_t)cw.m * Lo.d + lo, flat_hi = (int64_t)cw.m * Lo.d + hi;
+        const int64_t r_first = flat_lo / kInner, r_end = (flat_hi + kInner - 1) / kInner;
+        const int len = (int)(hi - lo);
+        const int lead = (int)(flat_lo - r_first * kInner);   // coordinates of the first row before the chunk
+        const int span = (int)((r_end - r_first) * kInner);   // coordinates the chunk's stages cover
+        const PhiloxStream ph(Lo, Lo.worker0 + (uint32_t)cw.m);
         float acc_hi = 0.0f, acc_lo = 0.0f;
         int runP = 0, runC = 0;
-        for (int64_t r0 = cr.r_first; r0 < cr.r_end; r0 += kStageRows, ++it) {
-            const int s = (int)(it % kStages);
+        for (int stage_off = 0; stage_off < span; stage_off += kStageCoords) {
             bool live = !*abort_flag;
-            if (live && !mbar_wait(&full[s], (uint32_t)((it / kStages) & 1))) {
+            if (live && !mbar_wait(&full[s], full_parity)) {
                 *abort_flag = 1;
                 atomicOr(A.status, kStTimeout);
                 live = false;
             }
-            // This lane's 16 coordinates: 4 Philox groups of 4.
-            const int h = cw * 32 + lane;
-            const int row = kDtype == 0 ? (h >> 1) : (h >> 2);
-            const int first_chunk = kDtype == 0 ? (h & 1) * 4 : (h & 3) * 2;
-            const int64_t f0 = (r0 + row) * kInner + (kDtype == 0 ? (h & 1) * 16 : (h & 3) * 16);
             const unsigned char* rp = base + s * kStageBytes + row * kRowBytes;
-            const int sw = row & 7;
-            // Whole stage inside the chunk: every lane's 16 coordinates are valid.
-            const bool stage_whole = r0 * kInner >= cr.flat_lo && (r0 + kStageRows) * kInner <= cr.flat_hi;
-            const bool any_valid = live && (stage_whole || ((f0 < cr.flat_hi) && (f0 + 16 > cr.flat_lo)));
+            const int rel = stage_off + lane_off - lead;      // chunk-relative index of coordinate 0
+            const bool whole = (stage_off - lead >= 0) && (stage_off - lead + kStageCoords <= len);
             uint32_t pm = 0, cm = 0;
-            float s16 = 0.0f;
-            if (any_valid) {
-                const uint32_t q0 = (uint32_t)((f0 - row0) >> 2);  // worker-local group of coordinate 0
-                if (stage_whole || (f0 >= cr.flat_lo && f0 + 16 <= cr.flat_hi)) {
-                    // All 16 coordinates belong to the chunk: one group of 4 at a time.
-                    float s4[4];
+            float s32 = 0.0f;
+            if (live && (whole || (rel < len && rel + kLaneCoords > 0))) {
+                const uint32_t q0 = (uint32_t)((lo + rel) >> 2);   // worker-local group of coordinate 0
+                if (whole || (rel >= 0 && rel + kLaneCoords <= len)) {
+                    // All 32 coordinates belong to the chunk: one group of 4 at a time.
+                    float s4[8];
 #pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        float a0, a1, a2, a3;
-                        if (kDtype == 0) {
-                            const float4 t = *reinterpret_cast<const float4*>(rp + (((first_chunk + j) ^ sw) << 4));
-                            a0 = fabsf(t.x); a1 = fabsf(t.y); a2 = fabsf(t.z); a3 = fabsf(t.w);
-                        } else {
-                            const uint2 t = *reinterpret_cast<const uint2*>(
-                                rp + (((first_chunk + (j >> 1)) ^ sw) << 4) + ((j & 1) << 3));
-                            a0 = fabsf(__uint_as_float(t.x << 16));
-                            a1 = fabsf(__uint_as_float(t.x & 0xFFFF0000u));
-                            a2 = fabsf(__uint_as_float(t.y << 16));
-                            a3 = fabsf(__uint_as_float(t.y & 0xFFFF0000u));
-                        }
-                        s4[j] = (a0 + a1) + (a2 + a3);
+                    for (int j = 0; j < 8; ++j) {
+                        const float4 a = stage_group<kDtype>(rp, first_chunk, sw, j);
+                        s4[j] = (a.x + a.y) + (a.z + a.w);
                         if (build_p) {
                             // candidate iff (1 + u) - lam_up |g| < 1 + 2^-20
                             const uint4 w = ph.words(q0 + j);
-                            pm = or_and(pm, lt_mask(fmaf(nlam, a0, unit_plus_one(w.x)), pbias), 1u << (4 * j));
-                            pm = or_and(pm, lt_mask(fmaf(nlam, a1, unit_plus_one(w.y)), pbias), 2u << (4 * j));
-                            pm = or_and(pm, lt_mask(fmaf(nlam, a2, unit_plus_one(w.z)), pbias), 4u << (4 * j));
-                            pm = or_and(pm, lt_mask(fmaf(nlam, a3, unit_plus_one(w.w)), pbias), 8u << (4 * j));
+                            pm = or_and(pm, lt_mask(fmaf(nlam, a.x, unit_plus_one(w.x)), pbias), 1u << (4 * j));
+                            pm = or_and(pm, lt_mask(fmaf(nlam, a.y, unit_plus_one(w.y)), pbias), 2u << (4 * j));
+                            pm = or_and(pm, lt_mask(fmaf(nlam, a.z, unit_plus_one(w.z)), pbias), 4u << (4 * j));
+                            pm = or_and(pm, lt_mask(fmaf(nlam, a.w, unit_plus_one(w.w)), pbias), 8u << (4 * j));
                         }
                     }
-                    s16 = (s4[0] + s4[1]) + (s4[2] + s4[3]);
-                    if (!(s16 < t_c)) {
+                    s32 = ((s4[0] + s4[1]) + (s4[2] + s4[3])) + ((s4[4] + s4[5]) + (s4[6] + s4[7]));
+                    if (!(s32 < t_c)) {
                         // Some |g| may reach t_c (or be non-finite): split exactly.
 #pragma unroll
-                        for (int j = 0; j < 4; ++j) {
+                        for (int j = 0; j < 8; ++j) {
                             float m4[4];
 #pragma unroll
                             for (int k = 0; k < 4; ++k) {
@@ -271,19 +309,19 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
                             }
                             s4[j] = (m4[0] + m4[1]) + (m4[2] + m4[3]);
                         }
-                        s16 = (s4[0] + s4[1]) + (s4[2] + s4[3]);
+                        s32 = ((s4[0] + s4[1]) + (s4[2] + s4[3])) + ((s4[4] + s4[5]) + (s4[6] + s4[7]));
                     }
                 } else {
                     // The lane straddles an edge of the chunk: test each coordinate.
-                    float s4[4];
+                    float s4[8];
 #pragma unroll
-                    for (int j = 0; j < 4; ++j) {
+                    for (int j = 0; j < 8; ++j) {
                         const uint4 w = build_p ? ph.words(q0 + j) : make_uint4(0, 0, 0, 0);
                         float m4[4];
 #pragma unroll
                         for (int k = 0; k < 4; ++k) {
                             const int e = 4 * j + k;
-                            const bool valid = f0 + e >= cr.flat_lo && f0 + e < cr.flat_hi;
+                            const bool valid = rel + e >= 0 && rel + e < len;
                             const float a = valid ? fabsf(stage_value<kDtype>(rp, first_chunk, sw, e)) : 0.0f;
                             const bool in_c = valid && !(a < t_c);
                             m4[k] = (valid && !in_c) ? a : 0.0f;
@@ -292,10 +330,10 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
                         }
                         s4[j] = (m4[0] + m4[1]) + (m4[2] + m4[3]);
                     }
-                    s16 = (s4[0] + s4[1]) + (s4[2] + s4[3]);
+                    s32 = ((s4[0] + s4[1]) + (s4[2] + s4[3])) + ((s4[4] + s4[5]) + (s4[6] + s4[7]));
                 }
             }
-            two_sum_add(acc_hi, acc_lo, s16);
+            two_sum_add(acc_hi, acc_lo, s32);
 
             // Order the stage's candidates: lane scan, then the warps' totals by shuffle.
             const uint32_t packed = (uint32_t)__popc(pm) | ((uint32_t)__popc(cm) << 16);
@@ -305,7 +343,7 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
                 const uint32_t t = __shfl_up_sync(0xFFFFFFFFu, inc, o);
                 if (lane >= o) inc += t;
             }
-            if (lane == 31) tot[par * kCW + cw] = inc;
+            if (lane == 31) tot[par * kCW + cwp] = inc;
             consumer_bar();
             const uint32_t tv = lane < kCW ? tot[par * kCW + lane] : 0u;
             uint32_t ti = tv;
@@ -314,24 +352,24 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
                 const uint32_t t = __shfl_up_sync(0xFFFFFFFFu, ti, o);
                 if (lane >= o) ti += t;
             }
-            const uint32_t wbefore = __shfl_sync(0xFFFFFFFFu, ti - tv, cw);
+            const uint32_t wbefore = __shfl_sync(0xFFFFFFFFu, ti - tv, cwp);
             const uint32_t wall = __shfl_sync(0xFFFFFFFFu, ti, kCW - 1);
             const uint32_t excl = inc - packed + wbefore;
             if (pm) {
-                int64_t e = region + runP + (int)(excl & 0xFFFFu);
-                const int32_t i0 = (int32_t)(f0 - row0);
+                int2* e = A.Ls.p_ent + flat_lo + runP + (int)(excl & 0xFFFFu);
+                const int32_t i0 = (int32_t)(lo + rel);
                 while (pm) {
                     const int k = __ffs(pm) - 1;
                     pm &= pm - 1u;
-                    A.Ls.p_ent[e++] = make_int2(i0 + k, __float_as_int(stage_value<kDtype>(rp, first_chunk, sw, k)));
+                    *e++ = make_int2(i0 + k, __float_as_int(stage_value<kDtype>(rp, first_chunk, sw, k)));
                 }
             }
             if (cm) {
-                int64_t e = region + runC + (int)(excl >> 16);
+                float* e = A.Ls.c_val + flat_lo + runC + (int)(excl >> 16);
                 while (cm) {
                     const int k = __ffs(cm) - 1;
                     cm &= cm - 1u;
-                    A.Ls.c_val[e++] = fabsf(stage_value<kDtype>(rp, first_chunk, sw, k));
+                    *e++ = fabsf(stage_value<kDtype>(rp, first_chunk, sw, k));
                 }
             }
             __syncwarp();
@@ -339,22 +377,25 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
             runP += (int)(wall & 0xFFFFu);
             runC += (int)(wall >> 16);
             par ^= 1;
+            if (++s == kStages) {
+                s = 0;
+                full_parity ^= 1u;
+            }
         }
         // Chunk totals: the lanes' (hi, lo) pairs reduced error-free across the
-        // warp, then the warps' partials summed in warp order in fp64.
+        // warp, then the warps' partials in warp order.
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
             const float oh = __shfl_xor_sync(0xFFFFFFFFu, acc_hi, o);
             const float ol = __shfl_xor_sync(0xFFFFFFFFu, acc_lo, o);
-            two_sum_add(acc_hi, acc_lo, oh);
-            acc_lo += ol;
+            df_add(acc_hi, acc_lo, oh, ol);
         }
-        if (lane == 0) sl[cw] = (double)acc_hi + (double)acc_lo;
+        if (lane == 0) sl[cwp] = make_float2(acc_hi, acc_lo);
         consumer_bar();
-        if (cw == 0 && lane == 0) {
-            double t = 0.0;
-            for (int k = 0; k < kCW; ++k) t += sl[k];
-            A.Ls.s_low[c] = t;
+        if (cwp == 0 && lane == 0) {
+            float th = 0.0f, tl = 0.0f;
+            for (int k = 0; k < kCW; ++k) df_add(th, tl, sl[k].x, sl[k].y);
+            A.Ls.s_low[c] = (double)th + (double)tl;
             A.Ls.c_cnt[c] = runC;
             if (A.Ls.p_cnt) A.Ls.p_cnt[c] = runP;
             if (A.Ls.k_state) A.Ls.k_state[c] = 0ull;
