@@ -165,6 +165,38 @@ gs_status gs_sparsify_aggregate(const void* g, int dtype, int M, int64_t d, doub
                                 gs_info* info, float* out, void* stream);
 
 /*
+ * gs_sparsify without any allocation.  The paper has no counterpart: this is
+ * a library convenience for callers that cannot allocate device memory
+ * during a call -- a program that hands (nearly) all device memory to its
+ * own allocator at start-up, or a timed loop in which an allocation, which
+ * may block or grow the device's footprint, is not acceptable.  Everything
+ * else in this library takes scratch from its memory pool.
+ *
+ * Result and arguments as in gs_sparsify (same idx / val / nnz, bit for
+ * bit), plus:
+ *   d       1 <= d <= 4194304 (2^22); a larger d returns GS_ERR_INVALID_ARG
+ *           at once and gs_last_error() says why
+ *   info    device, one gs_info (may be NULL)
+ *   status  device, one int32 (may be NULL): receives, in stream order, the
+ *           gs_status of the device-side checks of this call (GS_OK,
+ *           GS_ERR_NONFINITE, GS_ERR_TIMEOUT, ...).  Such errors are not
+ *           recorded for gs_sync_status.
+ * Scratch is one static device array of about 48 MiB (sized for d = 2^22)
+ * and one static status word; every GPU that loads the library may hold
+ * them until the process exits.  The first call on a device looks up their
+ * addresses (a one-time set-up that may load the library's code onto the
+ * device): make that first call before any stream capture.  All calls on a
+ * device share the array, and each call leaves its contents behind: calls
+ * that may run at the same time (on different streams, or from host threads
+ * with no ordering between them) race and return wrong results, so order
+ * them, e.g. on one stream.  GS_OPT_* settings apply as for gs_sparsify;
+ * with GS_OPT_KERNEL_TIMING on, the library creates CUDA events.
+ */
+gs_status gs_sparsify_noalloc(const float* g, int64_t d, double kappa, int iters, uint64_t seed, uint32_t step,
+                              uint32_t worker, int32_t* idx, float* val, int32_t* nnz, gs_info* info, int32_t* status,
+                              void* stream);
+
+/*
  * The whole path for M workers with HOST buffers: copies g_host (M x d,
  * `dtype`) to the device, runs gs_sparsify_aggregate,
  * and copies the dense sum back to out_host (d fp32) and the kept counts to

@@ -24,7 +24,7 @@ GS_OPT_FORCE_EXACT_SOLVE, GS_OPT_SAMPLE_SIZE, GS_OPT_KERNEL_TIMING, GS_OPT_STREA
 # Symbols include/gs.h declares (checked by the tests).
 EXPORTS = ("gs_status_string", "gs_last_error", "gs_version", "gs_sync_status", "gs_probabilities", "gs_probabilities_ex",
            "gs_sparsify", "gs_batched_sparsify", "gs_segmented_sparsify", "gs_sparse_aggregate",
-           "gs_sparsify_aggregate", "gs_pipeline_host", "gs_random_words", "gs_set_option", "gs_kernel_count", "gs_kernel_name",
+           "gs_sparsify_aggregate", "gs_sparsify_noalloc", "gs_pipeline_host", "gs_random_words", "gs_set_option", "gs_kernel_count", "gs_kernel_name",
            "gs_kernel_times")
 
 
@@ -66,6 +66,7 @@ def lib():
                                       i32),
             "gs_sparse_aggregate": ([vp, vp, vp, i32, i64, vp, vp], i32),
             "gs_sparsify_aggregate": ([vp, i32, i32, i64, dbl, i32, u64, u32, u32, vp, vp, vp, i64, vp, vp, vp], i32),
+            "gs_sparsify_noalloc": ([vp, i64, dbl, i32, u64, u32, u32, vp, vp, vp, vp, vp, vp], i32),
             "gs_pipeline_host": ([vp, i32, i32, i64, dbl, i32, u64, u32, u32, vp, vp, vp, vp, i64, vp, vp, vp, vp],
                                  i32),
             "gs_random_words": ([u64, u32, u32, i64, i64, vp, vp], i32),
@@ -198,6 +199,23 @@ def gs_sparsify(g, kappa, iters, seed, step, worker, idx, val, nnz, stream=None)
                              int(step), int(worker), _ptr(idx, "idx", (torch.int32,)),
                              _ptr(val, "val", (torch.float32,)), _ptr(nnz, "nnz", (torch.int32,)), _stream(stream)),
            "gs_sparsify")
+
+
+def gs_sparsify_noalloc(g, kappa, iters, seed, step, worker, idx, val, nnz, info=None, status=None, stream=None):
+    """gs_sparsify on the library's static scratch (d <= 2^22): the call
+    itself allocates no device memory.  `status` (one int32 on the device,
+    optional) receives the call's device-side status code."""
+    import torch
+    if idx.numel() < g.numel() or val.numel() < g.numel():
+        raise ValueError("idx / val need capacity d")
+    L = lib()
+    rc = L.gs_sparsify_noalloc(_ptr(g, "g", (torch.float32,)), g.numel(), float(kappa), int(iters), int(seed),
+                               int(step), int(worker), _ptr(idx, "idx", (torch.int32,)),
+                               _ptr(val, "val", (torch.float32,)), _ptr(nnz, "nnz", (torch.int32,)),
+                               _ptr(info, "info"), _ptr(status, "status", (torch.int32,)), _stream(stream))
+    if rc == GS_ERR_INVALID_ARG and L.gs_last_error():
+        raise GSError(rc, f"gs_sparsify_noalloc [{L.gs_last_error().decode()}]")
+    _check(rc, "gs_sparsify_noalloc")
 
 
 def gs_batched_sparsify(g, kappa, iters, seed, step, worker0, idx, val, nnz, info=None, stream=None):

@@ -277,6 +277,139 @@ gs_status run_aggregate(const int32_t* const* idx, const float* const* val, cons
     return GS_OK;
 }
 
+// ---------------------------------------------------------------------------
+// Single-worker sparsify with no allocation (gs_sparsify_noalloc).  Its
+// scratch is one file-scope device array sized for d <= kNoAllocMaxD; a
+// device that loads this library holds the array until the process exits.
+
+constexpr int64_t kNoAllocMaxD = (int64_t)1 << 22;
+
+constexpr size_t up256(size_t b) { return (b + 255) & ~(size_t)255; }
+
+// Upper bound of what carve() takes for one worker and one segment.
+constexpr size_t noalloc_bytes(int64_t n) {
+    const size_t nc = (size_t)((n + kChunk - 1) / kChunk);
+    return up256(sizeof(SegParam)) + up256(sizeof(float) * n) + up256(sizeof(int32_t) * nc) +
+           up256(sizeof(double) * nc) + up256(sizeof(int32_t) * (nc + 1)) + up256(sizeof(int2) * n) +
+           up256(sizeof(int32_t) * nc) + up256(sizeof(int32_t) * nc) + up256(sizeof(unsigned long long) * nc) +
+           up256(sizeof(int32_t));
+}
+
+constexpr size_t kNoAllocBytes = noalloc_bytes(kNoAllocMaxD);
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocBytes];
+static __device__ int g_noalloc_status;  // OR of kSt* bits of the current call
+
+struct NoAllocDev {
+    bool ready = false;
+    char* scratch = nullptr;
+    int* status = nullptr;
+};
+NoAllocDev g_noalloc[kMaxDevices];
+
+// Device addresses of the array and the status word, looked up once per
+// device (the lookup may load this library's code onto the device).
+gs_status noalloc_device(NoAllocDev** out) {
+    int dev = 0;
+    GS_TRY(cudaGetDevice(&dev));
+    if (dev < 0 || dev >= kMaxDevices) return cuda_fail("device ordinal", cudaErrorInvalidDevice);
+    std::lock_guard<std::mutex> lk(g_mu);
+    NoAllocDev& s = g_noalloc[dev];
+    if (!s.ready) {
+        void* a = nullptr;
+        void* b = nullptr;
+        GS_TRY(cudaGetSymbolAddress(&a, g_noalloc_scratch));
+        GS_TRY(cudaGetSymbolAddress(&b, g_noalloc_status));
+        s.scratch = static_cast<char*>(a);
+        s.status = static_cast<int*>(b);
+        s.ready = true;
+    }
+    *out = &s;
+    return GS_OK;
+}
+
+// Turns the call's status bits into one gs_status code (same precedence as
+// gs_sync_status) for the caller's word.
+__global__ void k_noalloc_status(const int* bits, int32_t* code) {
+    const int h = *bits;
+    int32_t c = GS_OK;
+    if (h & kStNonfinite) c = GS_ERR_NONFINITE;
+    else if (h & kStCapacity) c = GS_ERR_CAPACITY;
+    else if (h & kStInvalid) c = GS_ERR_INVALID_ARG;
+    else if (h & kStTimeout) c = GS_ERR_TIMEOUT;
+    else if (h & kStInternal) c = GS_ERR_INTERNAL;
+    *code = c;
+}
+
+gs_status run_noalloc(const float* g, int64_t d, double kappa, int iters, uint64_t seed, uint32_t step,
+                      uint32_t worker, int32_t* idx, float* val, int32_t* nnz, gs_info* info, int32_t* status,
+                      cudaStream_t st) {
+    g_last_error[0] = '\0';
+    if (!g || !idx || !val || !nnz || d < 1 || bad_kappa(kappa) || iters < 0) return GS_ERR_INVALID_ARG;
+    if ((reinterpret_cast<uintptr_t>(g) % sizeof(float)) != 0) return GS_ERR_INVALID_ARG;
+    if (d > kNoAllocMaxD) {
+        snprintf(g_last_error, sizeof(g_last_error),
+                 "gs_sparsify_noalloc: d = %lld is above the limit %lld of its static scratch", (long long)d,
+                 (long long)kNoAllocMaxD);
+        return GS_ERR_INVALID_ARG;
+    }
+    NoAllocDev* s = nullptr;
+    gs_status rc = noalloc_device(&s);
+    if (rc != GS_OK) return rc;
+
+    Layout Lo;
+    std::memset(&Lo, 0, sizeof(Lo));
+    Lo.g = g;
+    Lo.dtype = GS_DTYPE_F32;
+    Lo.M = 1;
+    Lo.L = 1;
+    Lo.d = d;
+    Lo.seed = seed;
+    Lo.step = step;
+    Lo.worker0 = worker;
+    for (int r = 0; r < 10; ++r) {
+        Lo.rk0[r] = (uint32_t)(seed & 0xFFFFFFFFu) + (uint32_t)r * 0x9E3779B9u;
+        Lo.rk1[r] = (uint32_t)(seed >> 32) + (uint32_t)r * 0xBB67AE85u;
+    }
+    Lo.cpw = (int)((d + chunk_size() - 1) / chunk_size());
+    const int n_chunks = Lo.cpw;
+
+    Arena a;
+    Workspace w;
+    carve(a, w, 1, n_chunks, d, true);
+    if (a.off > kNoAllocBytes) return GS_ERR_INTERNAL;
+    a.base = s->scratch;
+    a.off = 0;
+    carve(a, w, 1, n_chunks, d, true);
+
+    int force, ns, path;
+    {
+        std::lock_guard<std::mutex> lk(g_mu);
+        force = g_force_exact;
+        ns = g_sample;
+        path = g_stream_path;
+    }
+    // The kernels zero the per-chunk states and the ticket themselves; the
+    // status word is the one thing left from the previous call.
+    GS_TRY(cudaMemsetAsync(s->status, 0, sizeof(int), st));
+    const bool tma_ok = path != 1 && stream_tma_eligible(Lo);
+    cudaError_t e = launch_bound(Lo, w.sp, 1, kappa, ns, force, st);
+    if (e == cudaSuccess) {
+        bool used = false;
+        if (tma_ok) e = launch_stream_tma(Lo, w.sp, w.ls, n_chunks, s->status, st, &used);
+        if (e == cudaSuccess && !used) e = launch_stream(Lo, w.sp, w.ls, n_chunks, true, st);
+    }
+    if (e == cudaSuccess) e = launch_solve(Lo, w.sp, w.ls, 1, kappa, iters, force, s->status, info, st);
+    if (e == cudaSuccess) e = launch_compact(Lo, w.sp, w.ls, n_chunks, idx, val, nnz, d, s->status, st);
+    if (e == cudaSuccess && status) {
+        k_noalloc_status<<<1, 1, 0, st>>>(s->status, status);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) set_launch_error_site("k_noalloc_status");
+    }
+    if (e != cudaSuccess) return cuda_fail(launch_error_site(), e);
+    return GS_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -359,6 +492,13 @@ gs_status gs_sparsify_aggregate(const void* g, int dtype, int M, int64_t d, doub
     if (!out || M < 1 || M > kMaxAggM) return GS_ERR_INVALID_ARG;
     return run(g, dtype, M, d, nullptr, 1, kappa, iters, seed, step, worker0, idx, val, nnz, cap, info, nullptr,
                static_cast<cudaStream_t>(stream), out);
+}
+
+gs_status gs_sparsify_noalloc(const float* g, int64_t d, double kappa, int iters, uint64_t seed, uint32_t step,
+                              uint32_t worker, int32_t* idx, float* val, int32_t* nnz, gs_info* info, int32_t* status,
+                              void* stream) {
+    return run_noalloc(g, d, kappa, iters, seed, step, worker, idx, val, nnz, info, status,
+                       static_cast<cudaStream_t>(stream));
 }
 
 gs_status gs_pipeline_host(const void* g_host, int dtype, int M, int64_t d, double kappa, int iters, uint64_t seed,
