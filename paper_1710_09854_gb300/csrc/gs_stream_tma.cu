@@ -1,26 +1,26 @@
 // gs_stream_tma.cu -- the single streaming pass over g (steps 1-3 of the
 // path: l1 sums of Algorithm 3, the capped candidates, the ordered keep
-// candidates with their Philox words) as a persistent, warp-specialised
-// sm_103a kernel fed by the Tensor Memory Accelerator.
+// candidates) as a persistent sm_103a kernel fed by the Tensor Memory
+// Accelerator.
 //
-// One CTA per SM.  Warp 0 is the producer: one elected lane walks the CTA's
-// chunks and issues cp.async.bulk.tensor loads of whole stages (8192
-// coordinates) into a ring of shared-memory buffers, each guarded by a
-// "full" and an "empty" mbarrier.  The other kCW warps consume: every lane
-// owns 16 consecutive coordinates of a stage, reads them from shared memory
-// (the 128-byte swizzle of the tensor map makes those reads bank-conflict
-// free), draws the 4 Philox words of each 4-coordinate group, and tests
-// every coordinate against the bound lam_up.  A warp scan plus one named
-// barrier per stage orders the candidates of the 16 consumer warps, so each
-// chunk's lists come out in ascending coordinate order, as k_stream writes
-// them.
+// Every warp owns whole chunks (chunk c goes to warp c mod (kCW * gridDim.x))
+// and a private ring of shared-memory buffers, each guarded by one "full"
+// mbarrier.  One lane of the warp keeps the ring kRing buffers ahead with
+// cp.async.bulk.tensor loads, refilling a buffer as soon as the warp is done
+// with it, so warps never wait for one another and a chunk's lists are
+// ordered by warp shuffles alone.  A warp takes its chunk 1024 coordinates
+// (one buffer) at a time: every lane owns 32 consecutive coordinates, reads
+// them from shared memory (the 128-byte swizzle of the tensor map makes those
+// reads bank-conflict free), draws the 4 Philox words of each 4-coordinate
+// group, and tests every coordinate against the bound lam_up.  Lists come out
+// in ascending coordinate order, exactly as k_stream writes them.
 //
 // The global tensor is g viewed as rows of 128 bytes (32 fp32 or 64 bf16);
-// a full stage is one 256 x 128 B (fp32) or 128 x 128 B (bf16) box; a partial
-// stage is loaded as 8-row boxes (rows past the tensor read as zero and
-// rows outside the chunk are masked).  Every wait is bounded: on a timeout
-// the CTA records GS_ERR_TIMEOUT, stops issuing, drains its outstanding
-// copies (again bounded) and leaves.
+// one buffer is one box of 32 x 128 B (fp32) or 16 x 128 B (bf16).  Rows
+// past the end of the tensor read as zero and coordinates outside the chunk
+// are masked.  Every wait is bounded: on a timeout the warp records
+// GS_ERR_TIMEOUT, stops issuing, waits (again bounded) for its outstanding
+// copies and leaves.
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -34,13 +34,12 @@
 namespace gs {
 namespace {
 
-constexpr int kCW = 8;                         // consumer warps
-constexpr int kTmaThreads = 32 * (kCW + 1);
-constexpr int kLaneCoords = 32;                // coordinates per lane per stage
-constexpr int kStageCoords = kCW * 32 * kLaneCoords;   // 8192 coordinates per stage
-constexpr int kStageBudget = 96 * 1024;        // shared memory for the ring of one CTA (2 CTAs per SM)
+constexpr int kCW = 8;                         // warps per CTA
+constexpr int kTmaThreads = 32 * kCW;
+constexpr int kLaneCoords = 32;                // coordinates per lane per buffer
+constexpr int kBufCoords = 32 * kLaneCoords;   // 1024 coordinates per buffer
+constexpr int kRingBudget = 96 * 1024;         // shared memory for the rings of one CTA (2 CTAs per SM)
 constexpr int kRowBytes = 128;
-constexpr int kSmallRows = 8;                  // rows per box of a partial stage (1 KiB)
 constexpr long long kWaitLimit = 1ll << 22;    // try_wait polls before giving up
 
 struct StreamArgs {
@@ -59,8 +58,10 @@ __device__ __forceinline__ void mbar_init(uint64_t* b, uint32_t count) {
 __device__ __forceinline__ void mbar_arrive_tx(uint64_t* b, uint32_t bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(b)), "r"(bytes) : "memory");
 }
-__device__ __forceinline__ void mbar_arrive(uint64_t* b) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(b)) : "memory");
+// Orders this thread's earlier shared-memory reads (generic proxy) before a
+// later TMA write (async proxy) to the same buffer.
+__device__ __forceinline__ void fence_proxy_async() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 __device__ __forceinline__ bool mbar_test(uint64_t* b, uint32_t parity) {
     uint32_t ok;
@@ -86,12 +87,16 @@ __device__ __forceinline__ void tma_load_rows(void* dst, const CUtensorMap* map,
         "l"(map), "r"(0), "r"(row), "r"(smem_addr(bar))
         : "memory");
 }
-__device__ __forceinline__ void consumer_bar() {
-    asm volatile("bar.sync 1, %0;" ::"n"(kCW * 32) : "memory");
+
+// (m << 1) | sign bit of r: appends one candidate flag to a mask in one funnel shift.
+__device__ __forceinline__ uint32_t shl_in(uint32_t m, float r) {
+    uint32_t o;
+    asm("shf.l.wrap.b32 %0, %1, %2, 1;" : "=r"(o) : "r"(__float_as_uint(r)), "r"(m));
+    return o;
 }
 
-// Coordinate k (0..31) of a lane's 32, read back from its row of the stage
-// buffer (first_chunk: the lane's first 16-byte chunk; sw: the row's swizzle).
+// Coordinate k (0..31) of a lane's 32, read back from its row of the buffer
+// (first_chunk: the lane's first 16-byte chunk; sw: the row's swizzle).
 template <int kDtype>
 __device__ __forceinline__ float stage_value(const unsigned char* rp, int first_chunk, int sw, int k) {
     if (kDtype == 0) {
@@ -117,19 +122,19 @@ __device__ __forceinline__ float4 stage_group(const unsigned char* rp, int first
     }
 }
 
-// The chunks of one CTA (c = blockIdx.x, + gridDim.x, ...), with the
-// worker and chunk-within-worker advanced without divisions.
+// The chunks c = first, first + step, ... with the worker and the chunk
+// within the worker advanced without divisions.
 struct ChunkWalk {
     int c, m, k, dm, dk;
-    __device__ __forceinline__ explicit ChunkWalk(const Layout& Lo) {
-        c = blockIdx.x;
+    __device__ __forceinline__ ChunkWalk(const Layout& Lo, int first, int step) {
+        c = first;
         m = c / Lo.cpw;
         k = c - m * Lo.cpw;
-        dm = gridDim.x / Lo.cpw;
-        dk = gridDim.x - dm * Lo.cpw;
+        dm = step / Lo.cpw;
+        dk = step - dm * Lo.cpw;
     }
-    __device__ __forceinline__ void next(const Layout& Lo) {
-        c += gridDim.x;
+    __device__ __forceinline__ void next(const Layout& Lo, int step) {
+        c += step;
         m += dm;
         k += dk;
         if (k >= Lo.cpw) {
@@ -155,130 +160,117 @@ struct ChunkWalk {
         }
         seg = m * Lo.L + l;
     }
+    // First row and end row (rows of kInner elements) of the chunk.
+    __device__ __forceinline__ void rows(const Layout& Lo, int inner, int64_t& flat_lo, int64_t& r_first,
+                                         int64_t& r_end, int& seg, int64_t& lo, int64_t& hi) const {
+        range(Lo, seg, lo, hi);
+        flat_lo = (int64_t)m * Lo.d + lo;
+        const int64_t flat_hi = (int64_t)m * Lo.d + hi;
+        r_first = flat_lo / inner;
+        r_end = (flat_hi + inner - 1) / inner;
+    }
 };
 
 // kDtype 0: fp32 rows of 32; 1: bf16 rows of 64.
 template <int kDtype>
 __global__ void __launch_bounds__(kTmaThreads, 2)
-    k_stream_tma(const __grid_constant__ CUtensorMap map_big, const __grid_constant__ CUtensorMap map_small,
-                 const __grid_constant__ StreamArgs A) {
+    k_stream_tma(const __grid_constant__ CUtensorMap map, const __grid_constant__ StreamArgs A) {
     constexpr int kInner = kDtype == 0 ? 32 : 64;          // elements per 128-byte row
-    constexpr int kStageRows = kStageCoords / kInner;      // 256 or 128
-    constexpr int kStageBytes = kStageRows * kRowBytes;    // 32 KiB or 16 KiB
-    constexpr int kStages = kStageBudget / kStageBytes;    // 3 or 6
+    constexpr int kBufRows = kBufCoords / kInner;          // 32 or 16
+    constexpr int kBufBytes = kBufRows * kRowBytes;        // 4 KiB or 2 KiB
+    constexpr int kRing = kRingBudget / (kCW * kBufBytes); // buffers per warp: 3 or 6
     extern __shared__ unsigned char dsm_raw[];
     unsigned char* base = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(dsm_raw) + 1023) & ~uintptr_t(1023));
-    uint64_t* full = reinterpret_cast<uint64_t*>(base + kStages * kStageBytes);
-    uint64_t* empty = full + kStages;
-    uint32_t* tot = reinterpret_cast<uint32_t*>(empty + kStages);  // [2][kCW] packed (P | C << 16)
-    float2* sl = reinterpret_cast<float2*>(tot + 2 * kCW);         // [kCW] double-float l1 partials
-    volatile int* abort_flag = reinterpret_cast<volatile int*>(sl + kCW);
+    uint64_t* full = reinterpret_cast<uint64_t*>(base + kCW * kRing * kBufBytes);   // [kCW][kRing]
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(full + kCW * kRing);
 
     const Layout& Lo = A.Lo;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int step = gridDim.x * kCW;                      // chunks between two of one warp
     if (threadIdx.x == 0) {
-        for (int s = 0; s < kStages; ++s) {
-            mbar_init(&full[s], 1);
-            mbar_init(&empty[s], kCW);
-        }
+        for (int i = 0; i < kCW * kRing; ++i) mbar_init(&full[i], 1);
         *abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     __syncthreads();
 
-    if (warp == 0) {
-        // ------------------------------------------------------------ producer
-        if (lane != 0) return;
-        int issued = 0, s = 0;
-        uint32_t empty_parity = 0;
-        bool wrapped = false, ok = true;
-        for (ChunkWalk cw(Lo); cw.c < A.n_chunks && ok; cw.next(Lo)) {
-            int seg;
-            int64_t lo, hi;
-            cw.range(Lo, seg, lo, hi);
-            const int64_t flat_lo = (int64_t)cw.m * Lo.d + lo, flat_hi = (int64_t)cw.m * Lo.d + hi;
-            const int64_t r_first = flat_lo / kInner, r_end = (flat_hi + kInner - 1) / kInner;
-            for (int64_t r0 = r_first; r0 < r_end; r0 += kStageRows) {
-                if (wrapped && !mbar_wait(&empty[s], empty_parity)) {
-                    ok = false;
-                    break;
-                }
-                if (*abort_flag) {
-                    ok = false;
-                    break;
-                }
-                const int rows = (int)min((int64_t)kStageRows, r_end - r0);
-                unsigned char* dst = base + s * kStageBytes;
-                if (rows == kStageRows) {
-                    mbar_arrive_tx(&full[s], kStageBytes);
-                    tma_load_rows(dst, &map_big, (int)r0, &full[s]);
-                } else {
-                    const int nb = (rows + kSmallRows - 1) / kSmallRows;
-                    mbar_arrive_tx(&full[s], (uint32_t)(nb * kSmallRows * kRowBytes));
-                    for (int b = 0; b < nb; ++b)
-                        tma_load_rows(dst + b * kSmallRows * kRowBytes, &map_small, (int)(r0 + b * kSmallRows),
-                                      &full[s]);
-                }
-                ++issued;
-                if (++s == kStages) {
-                    s = 0;
-                    if (wrapped) empty_parity ^= 1u;
-                    wrapped = true;
-                }
+    uint64_t* my_full = full + warp * kRing;
+    unsigned char* my_buf = base + warp * kRing * kBufBytes;
+    const int first = blockIdx.x * kCW + warp;
+
+    // Prefetch cursor: the next buffer's row and its chunk's end row.
+    ChunkWalk pc(Lo, first, step);
+    int64_t prow = 0, prow_end = 0;
+    if (pc.c < A.n_chunks) {
+        int64_t fl, lo, hi;
+        int seg;
+        pc.rows(Lo, kInner, fl, prow, prow_end, seg, lo, hi);
+    }
+    int issued = 0;
+    auto prefetch = [&]() {
+        if (pc.c >= A.n_chunks) return;
+        const int b = issued % kRing;
+        if (lane == 0) {
+            mbar_arrive_tx(&my_full[b], kBufBytes);
+            tma_load_rows(my_buf + b * kBufBytes, &map, (int)prow, &my_full[b]);
+        }
+        ++issued;
+        prow += kBufRows;
+        if (prow >= prow_end) {
+            pc.next(Lo, step);
+            if (pc.c < A.n_chunks) {
+                int64_t fl, lo, hi;
+                int seg;
+                pc.rows(Lo, kInner, fl, prow, prow_end, seg, lo, hi);
             }
         }
-        if (!ok) {
-            *abort_flag = 1;
-            atomicOr(A.status, kStTimeout);
-        }
-        // Drain: every issued stage's copy must have landed before the CTA may exit.
-        for (int k = issued - 1; k >= 0 && k >= issued - kStages; --k)
-            mbar_wait(&full[k % kStages], (uint32_t)((k / kStages) & 1));
-        return;
-    }
+    };
+#pragma unroll 1
+    for (int i = 0; i < kRing; ++i) prefetch();
 
-    // ---------------------------------------------------------------- consumers
-    const int cwp = warp - 1;
+    // candidate iff u' - 2^-20 - lam_up |g| < 0, u' = (x >> 9) 2^-23 <= u (the sign is exact)
     const float pbias = 1.0f + 0x1p-20f;
     // Probability-only calls keep no keep-candidate lists (their pointer is NULL).
     const bool build_p = A.Ls.p_ent != nullptr;
-    // This lane's 32 coordinates of every stage: one 128-byte row (fp32) or half of one (bf16).
-    const int h = cwp * 32 + lane;
-    const int row = kDtype == 0 ? h : (h >> 1);
-    const int first_chunk = kDtype == 0 ? 0 : (h & 1) * 4;
-    const int lane_off = row * kInner + (kDtype == 0 ? 0 : (h & 1) * 32);   // within the stage
-    const int sw = row & 7;
-    int s = 0, par = 0;
+    // This lane's 32 coordinates of every buffer: one 128-byte row (fp32) or half of one (bf16).
+    const int brow = kDtype == 0 ? lane : (lane >> 1);
+    const int first_chunk = kDtype == 0 ? 0 : (lane & 1) * 4;
+    const int lane_off = lane * kLaneCoords;                 // within the buffer
+    const int sw = brow & 7;
+    int slot = 0, consumed = 0;
     uint32_t full_parity = 0;
-    for (ChunkWalk cw(Lo); cw.c < A.n_chunks; cw.next(Lo)) {
+    bool live = true;
+    for (ChunkWalk cw(Lo, first, step); cw.c < A.n_chunks; cw.next(Lo, step)) {
         int seg;
-        int64_t lo, hi;
-        cw.range(Lo, seg, lo, hi);
+        int64_t lo, hi, flat_lo, r_first, r_end;
+        cw.rows(Lo, kInner, flat_lo, r_first, r_end, seg, lo, hi);
         const int c = cw.c;
         const float nlam = -A.sp[seg].lam_up32, t_c = A.sp[seg].t_c;
-        const int64_t flat_lo = (int64_t)cw.m * Lo.d + lo, flat_hi = (int64_t)cw.m * Lo.d + hi;
-        const int64_t r_first = flat_lo / kInner, r_end = (flat_hi + kInner - 1) / kInner;
         const int len = (int)(hi - lo);
         const int lead = (int)(flat_lo - r_first * kInner);   // coordinates of the first row before the chunk
-        const int span = (int)((r_end - r_first) * kInner);   // coordinates the chunk's stages cover
+        const int span = (int)((r_end - r_first) * kInner);   // coordinates the chunk's buffers cover
         const PhiloxStream ph(Lo, Lo.worker0 + (uint32_t)cw.m);
         float acc_hi = 0.0f, acc_lo = 0.0f;
         int runP = 0, runC = 0;
-        for (int stage_off = 0; stage_off < span; stage_off += kStageCoords) {
-            bool live = !*abort_flag;
-            if (live && !mbar_wait(&full[s], full_parity)) {
-                *abort_flag = 1;
-                atomicOr(A.status, kStTimeout);
-                live = false;
+        for (int buf_off = 0; buf_off < span; buf_off += kBufCoords) {
+            // live stays warp-uniform: the refill below is a warp-wide step.
+            live = __all_sync(0xFFFFFFFFu, live && !*abort_flag);
+            if (live) {
+                live = __all_sync(0xFFFFFFFFu, mbar_wait(&my_full[slot], full_parity));
+                if (live) {
+                    ++consumed;
+                } else if (lane == 0) {
+                    *abort_flag = 1;
+                    atomicOr(A.status, kStTimeout);
+                }
             }
-            const unsigned char* rp = base + s * kStageBytes + row * kRowBytes;
-            const int rel = stage_off + lane_off - lead;      // chunk-relative index of coordinate 0
-            const bool whole = (stage_off - lead >= 0) && (stage_off - lead + kStageCoords <= len);
+            const unsigned char* rp = my_buf + slot * kBufBytes + brow * kRowBytes;
+            const int rel = buf_off + lane_off - lead;      // chunk-relative index of coordinate 0
             uint32_t pm = 0, cm = 0;
             float s32 = 0.0f;
-            if (live && (whole || (rel < len && rel + kLaneCoords > 0))) {
+            if (live && rel < len && rel + kLaneCoords > 0) {
                 const uint32_t q0 = (uint32_t)((lo + rel) >> 2);   // worker-local group of coordinate 0
-                if (whole || (rel >= 0 && rel + kLaneCoords <= len)) {
+                if (rel >= 0 && rel + kLaneCoords <= len) {
                     // All 32 coordinates belong to the chunk: one group of 4 at a time.
                     float s4[8];
 #pragma unroll
@@ -286,14 +278,14 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
                         const float4 a = stage_group<kDtype>(rp, first_chunk, sw, j);
                         s4[j] = (a.x + a.y) + (a.z + a.w);
                         if (build_p) {
-                            // candidate iff (1 + u) - lam_up |g| < 1 + 2^-20
                             const uint4 w = ph.words(q0 + j);
-                            pm = or_and(pm, lt_mask(fmaf(nlam, a.x, unit_plus_one(w.x)), pbias), 1u << (4 * j));
-                            pm = or_and(pm, lt_mask(fmaf(nlam, a.y, unit_plus_one(w.y)), pbias), 2u << (4 * j));
-                            pm = or_and(pm, lt_mask(fmaf(nlam, a.z, unit_plus_one(w.z)), pbias), 4u << (4 * j));
-                            pm = or_and(pm, lt_mask(fmaf(nlam, a.w, unit_plus_one(w.w)), pbias), 8u << (4 * j));
+                            pm = shl_in(pm, fmaf(nlam, a.x, __fsub_rn(unit_plus_one(w.x), pbias)));
+                            pm = shl_in(pm, fmaf(nlam, a.y, __fsub_rn(unit_plus_one(w.y), pbias)));
+                            pm = shl_in(pm, fmaf(nlam, a.z, __fsub_rn(unit_plus_one(w.z), pbias)));
+                            pm = shl_in(pm, fmaf(nlam, a.w, __fsub_rn(unit_plus_one(w.w), pbias)));
                         }
                     }
+                    pm = __brev(pm);   // coordinate k at bit k
                     s32 = ((s4[0] + s4[1]) + (s4[2] + s4[3])) + ((s4[4] + s4[5]) + (s4[6] + s4[7]));
                     if (!(s32 < t_c)) {
                         // Some |g| may reach t_c (or be non-finite): split exactly.
@@ -326,7 +318,9 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
                             const bool in_c = valid && !(a < t_c);
                             m4[k] = (valid && !in_c) ? a : 0.0f;
                             cm |= in_c ? (1u << e) : 0u;
-                            if (build_p && valid && fmaf(nlam, a, unit_plus_one(word_of(w, k))) < pbias) pm |= 1u << e;
+                            if (build_p && valid &&
+                                shl_in(0u, fmaf(nlam, a, __fsub_rn(unit_plus_one(word_of(w, k)), pbias))) != 0u)
+                                pm |= 1u << e;
                         }
                         s4[j] = (m4[0] + m4[1]) + (m4[2] + m4[3]);
                     }
@@ -335,7 +329,7 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
             }
             two_sum_add(acc_hi, acc_lo, s32);
 
-            // Order the stage's candidates: lane scan, then the warps' totals by shuffle.
+            // Order the buffer's candidates by a lane scan.
             const uint32_t packed = (uint32_t)__popc(pm) | ((uint32_t)__popc(cm) << 16);
             uint32_t inc = packed;
 #pragma unroll
@@ -343,18 +337,8 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
                 const uint32_t t = __shfl_up_sync(0xFFFFFFFFu, inc, o);
                 if (lane >= o) inc += t;
             }
-            if (lane == 31) tot[par * kCW + cwp] = inc;
-            consumer_bar();
-            const uint32_t tv = lane < kCW ? tot[par * kCW + lane] : 0u;
-            uint32_t ti = tv;
-#pragma unroll
-            for (int o = 1; o < kCW; o <<= 1) {
-                const uint32_t t = __shfl_up_sync(0xFFFFFFFFu, ti, o);
-                if (lane >= o) ti += t;
-            }
-            const uint32_t wbefore = __shfl_sync(0xFFFFFFFFu, ti - tv, cwp);
-            const uint32_t wall = __shfl_sync(0xFFFFFFFFu, ti, kCW - 1);
-            const uint32_t excl = inc - packed + wbefore;
+            const uint32_t wall = __shfl_sync(0xFFFFFFFFu, inc, 31);
+            const uint32_t excl = inc - packed;
             if (pm) {
                 int2* e = A.Ls.p_ent + flat_lo + runP + (int)(excl & 0xFFFFu);
                 const int32_t i0 = (int32_t)(lo + rel);
@@ -372,35 +356,36 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
                     *e++ = fabsf(stage_value<kDtype>(rp, first_chunk, sw, k));
                 }
             }
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&empty[s]);   // this warp is done with the buffer
+            // The warp is done with the buffer: refill it with the buffer kRing ahead.
+            if (live) {
+                fence_proxy_async();
+                __syncwarp();
+                prefetch();
+            }
             runP += (int)(wall & 0xFFFFu);
             runC += (int)(wall >> 16);
-            par ^= 1;
-            if (++s == kStages) {
-                s = 0;
+            if (++slot == kRing) {
+                slot = 0;
                 full_parity ^= 1u;
             }
         }
-        // Chunk totals: the lanes' (hi, lo) pairs reduced error-free across the
-        // warp, then the warps' partials in warp order.
+        // Chunk total: the lanes' (hi, lo) pairs reduced error-free across the warp.
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
             const float oh = __shfl_xor_sync(0xFFFFFFFFu, acc_hi, o);
             const float ol = __shfl_xor_sync(0xFFFFFFFFu, acc_lo, o);
             df_add(acc_hi, acc_lo, oh, ol);
         }
-        if (lane == 0) sl[cwp] = make_float2(acc_hi, acc_lo);
-        consumer_bar();
-        if (cwp == 0 && lane == 0) {
-            float th = 0.0f, tl = 0.0f;
-            for (int k = 0; k < kCW; ++k) df_add(th, tl, sl[k].x, sl[k].y);
-            A.Ls.s_low[c] = (double)th + (double)tl;
+        if (lane == 0) {
+            A.Ls.s_low[c] = (double)acc_hi + (double)acc_lo;
             A.Ls.c_cnt[c] = runC;
             if (A.Ls.p_cnt) A.Ls.p_cnt[c] = runP;
             if (A.Ls.k_state) A.Ls.k_state[c] = 0ull;
         }
     }
+    // After a timeout, wait (bounded) for the copies still in flight into this
+    // warp's ring (consumed counts the buffers whose wait succeeded).
+    for (int n = consumed; n < issued; ++n) mbar_wait(&my_full[n % kRing], (uint32_t)((n / kRing) & 1));
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
@@ -440,9 +425,10 @@ bool make_map(CUtensorMap* map, const void* g, int dtype, int64_t rows, int box_
 template <int kDtype>
 size_t tma_smem_bytes() {
     constexpr int kInner = kDtype == 0 ? 32 : 64;
-    constexpr int kStageBytes = (kStageCoords / kInner) * kRowBytes;
-    constexpr int kStages = kStageBudget / kStageBytes;
-    return 1024 + (size_t)kStages * kStageBytes + 2 * kStages * 8 + 2 * kCW * 4 + kCW * 8 + 16;
+    constexpr int kBufBytes = (kBufCoords / kInner) * kRowBytes;
+    constexpr int kRing = kRingBudget / (kCW * kBufBytes);
+    // alignment slack + buffers + full barriers + abort flag
+    return 1024 + (size_t)kCW * kRing * kBufBytes + (size_t)kCW * kRing * 8 + 16;
 }
 
 int sm_count_tma() {
@@ -475,9 +461,8 @@ cudaError_t launch_stream_tma(const Layout& Lo, const SegParam* sp, const Lists&
     *used = false;
     const int64_t inner = Lo.dtype == 0 ? 32 : 64;
     const int64_t rows = (int64_t)Lo.M * Lo.d / inner;
-    CUtensorMap big, small;
-    const int big_rows = kStageCoords / (int)inner;
-    if (!make_map(&big, Lo.g, Lo.dtype, rows, big_rows) || !make_map(&small, Lo.g, Lo.dtype, rows, kSmallRows))
+    CUtensorMap map;
+    if (!make_map(&map, Lo.g, Lo.dtype, rows, kBufCoords / (int)inner))
         return cudaSuccess;  // caller falls back to the generic pass
     StreamArgs A;
     A.Lo = Lo;
@@ -485,7 +470,8 @@ cudaError_t launch_stream_tma(const Layout& Lo, const SegParam* sp, const Lists&
     A.Ls = Ls;
     A.n_chunks = n_chunks;
     A.status = status;
-    const int grid = std::min(n_chunks, 2 * sm_count_tma());
+    // One chunk per warp at a time; two CTAs per SM at most.
+    const int grid = std::min((n_chunks + kCW - 1) / kCW, 2 * sm_count_tma());
     cudaError_t e;
     TraceScope ts(kKStreamTma, st);
     if (Lo.dtype == 0) {
@@ -494,14 +480,14 @@ cudaError_t launch_stream_tma(const Layout& Lo, const SegParam* sp, const Lists&
         e = cudaFuncSetAttribute(k_stream_tma<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
         set_launch_error_site("k_stream_tma<fp32> launch");
-        k_stream_tma<0><<<grid, kTmaThreads, smem, st>>>(big, small, A);
+        k_stream_tma<0><<<grid, kTmaThreads, smem, st>>>(map, A);
     } else {
         const size_t smem = tma_smem_bytes<1>();
         set_launch_error_site("k_stream_tma<bf16> shared-memory attribute");
         e = cudaFuncSetAttribute(k_stream_tma<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
         set_launch_error_site("k_stream_tma<bf16> launch");
-        k_stream_tma<1><<<grid, kTmaThreads, smem, st>>>(big, small, A);
+        k_stream_tma<1><<<grid, kTmaThreads, smem, st>>>(map, A);
     }
     *used = true;
     return cudaGetLastError();
