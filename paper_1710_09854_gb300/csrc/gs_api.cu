@@ -138,8 +138,8 @@ void carve(Arena& a, Workspace& w, int n_seg, int n_chunks, int64_t n, bool buil
         w.ls.p_ent = a.take<int2>(n);
         w.ls.p_cnt = a.take<int32_t>(n_chunks);
         w.ls.k_off = a.take<int32_t>(n_chunks);
-        w.ls.k_state = a.take<unsigned long long>(n_chunks);
-        w.ls.ticket = a.take<int32_t>(1);
+        w.ls.e_bits = a.take<uint32_t>((size_t)n_chunks * (kChunk / 32));
+        w.ls.k_sub = a.take<int32_t>((size_t)n_chunks * kSubStride);
     }
 }
 
@@ -226,21 +226,7 @@ gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off
     if (e == cudaSuccess) e = launch_solve(Lo, w.sp, w.ls, n_seg, kappa, iters, force, s->status, info, st);
     if (e == cudaSuccess) {
         if (prob) e = launch_prob(Lo, w.sp, p, st);
-        else e = launch_compact(Lo, w.sp, w.ls, n_chunks, idx, val, nnz, cap, s->status, st);
-    }
-    if (e == cudaSuccess && agg_out) {
-        // The sum of the M rows just written, tiled by the chunks (L == 1).
-        AggArgs A;
-        std::memset(&A, 0, sizeof(A));
-        for (int m = 0; m < M; ++m) {
-            A.idx[m] = idx + (size_t)m * (size_t)cap;
-            A.val[m] = val + (size_t)m * (size_t)cap;
-        }
-        A.nnz = nnz;
-        A.M = M;
-        A.d = d;
-        A.cap = cap;
-        e = launch_aggregate_chunks(A, w.ls.k_off, Lo.cpw, agg_out, st);
+        else e = launch_compact(Lo, w.sp, w.ls, n_chunks, idx, val, nnz, cap, s->status, st, agg_out);
     }
     cudaError_t ef = cudaFreeAsync(mem, st);
     if (e != cudaSuccess) return cuda_fail(launch_error_site(), e);
@@ -291,8 +277,8 @@ constexpr size_t noalloc_bytes(int64_t n) {
     const size_t nc = (size_t)((n + kChunk - 1) / kChunk);
     return up256(sizeof(SegParam)) + up256(sizeof(float) * n) + up256(sizeof(int32_t) * nc) +
            up256(sizeof(double) * nc) + up256(sizeof(int32_t) * (nc + 1)) + up256(sizeof(int2) * n) +
-           up256(sizeof(int32_t) * nc) + up256(sizeof(int32_t) * nc) + up256(sizeof(unsigned long long) * nc) +
-           up256(sizeof(int32_t));
+           up256(sizeof(int32_t) * nc) + up256(sizeof(int32_t) * nc) + up256(sizeof(uint32_t) * nc * (kChunk / 32)) +
+           up256(sizeof(int32_t) * nc * kSubStride);
 }
 
 constexpr size_t kNoAllocBytes = noalloc_bytes(kNoAllocMaxD);
@@ -389,8 +375,8 @@ gs_status run_noalloc(const float* g, int64_t d, double kappa, int iters, uint64
         ns = g_sample;
         path = g_stream_path;
     }
-    // The kernels zero the per-chunk states and the ticket themselves; the
-    // status word is the one thing left from the previous call.
+    // Every scratch word a kernel reads was written earlier in the same call;
+    // the status word is the one thing left from the previous call.
     GS_TRY(cudaMemsetAsync(s->status, 0, sizeof(int), st));
     const bool tma_ok = path != 1 && stream_tma_eligible(Lo);
     cudaError_t e = launch_bound(Lo, w.sp, 1, kappa, ns, force, st);

@@ -12,6 +12,7 @@ namespace gs {
 // capacity of each chunk's candidate lists.  A multiple of 4 so that chunk
 // starts inside a worker row keep the 4-coordinate Philox groups aligned.
 constexpr int kChunk = 16384;
+constexpr int kSubStride = 17;   // k_sub entries per chunk (slice starts 0..16)
 // Coordinates per output tile of the sparse sum.
 constexpr int kAggTile = 8192;
 // Threads per CTA of the streaming / solve / decide kernels.
@@ -77,9 +78,10 @@ struct Lists {
     float* c_val;       // |g| of each capped candidate
     int32_t* c_cnt;     // [n_chunks]
     double* s_low;      // [n_chunks] sum of |g| outside C
-    int32_t* k_off;     // [n_chunks] offset of the chunk's first kept entry in its worker's output
-    unsigned long long* k_state;  // [n_emit_tiles] decoupled look-back words (zeroed by the streaming pass)
-    int32_t* ticket;    // emit-tile ticket counter (zeroed by the solve)
+    int32_t* k_off;     // [n_chunks] kept count of the chunk, then (after k_scan) the offset
+                        // of its first kept entry in its worker's output
+    uint32_t* e_bits;   // [n_chunks][kChunk / 32] decision bit of every keep candidate
+    int32_t* k_sub;     // [n_chunks][kSubStride] kept entries of the chunk before each 1024-coordinate slice
     int32_t* c_pre;     // [n_chunks + n_seg] prefix scratch for segments with many chunks
 };
 

@@ -189,7 +189,6 @@ __device__ void chunk_candidates(const Layout& Lo, int c, const Chunk& ch, float
     const double tot = block_sum(acc, shd);
     if (tid == 0) {
         if (build_p) Ls.p_cnt[c] = runP;
-        if (kWithC && Ls.k_state) Ls.k_state[c] = 0ull;
         if (kWithC) {
             Ls.c_cnt[c] = runC;
             Ls.s_low[c] = tot;
@@ -490,7 +489,6 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
     __shared__ int shi[33];
     __shared__ float s_acap;
     const int s = blockIdx.x, tid = threadIdx.x;
-    if (s == 0 && tid == 0 && Ls.ticket) *Ls.ticket = 0;
     int m, l, c0, c1;
     int64_t lo, hi;
     seg_range(Lo, s, m, l, lo, hi, c0, c1);
@@ -610,6 +608,12 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
 // are g_i / p_i: g_i itself when capped, else sign(g_i) / lambda (the
 // constant-value form of section 5.3).
 // ---------------------------------------------------------------------------
+// The exact fp64 comparison, kept out of line so that the compiler cannot
+// evaluate it (fp64 is slow on this part) for the common, certain calls.
+__device__ __noinline__ bool exact_keep(uint32_t x, double lam, float a) {
+    return (double)x * 0x1p-32 < lam * (double)a;
+}
+
 struct Decider {
     double lam;
     float lam32, a_cap, inv_lam32;
@@ -627,218 +631,267 @@ struct Decider {
         bool keep;
         if (uf + 0x1p-21f < pf) keep = true;
         else if (uf - 0x1p-21f > pf) keep = false;
-        else keep = (double)x * 0x1p-32 < lam * (double)a;
+        else keep = exact_keep(x, lam, a);
         val = copysignf(inv_lam32, gv);
         return keep;
     }
 };
 
 // ---------------------------------------------------------------------------
-// k_emit: decide + amplify + compact.  One CTA per emit tile (kEmitChunks
-// consecutive chunks of one worker), taken in ticket order.  Pass 1 draws
-// each candidate's Philox word again and records its decision as one bit
-// (a warp ballot per 32 candidates); the worker's output offset of the tile
-// comes from a decoupled look-back over the preceding tiles (Merrill &
-// Garland, "Single-pass Parallel Prefix Scan with Decoupled Look-back",
-// 2016; every wait bounded); pass 2 writes the kept entries in order.
+// Compaction in three steps with no waits between chunks:
+//   k_decide  one warp per chunk: draws each candidate's Philox word again,
+//             records its decision as one bit (a warp ballot per 32
+//             candidates) and the chunk's kept count;
+//   k_scan    one CTA per worker: exclusive prefix of the kept counts over
+//             the worker's chunks (the output offset of every chunk), nnz;
+//   k_emit    one warp per chunk: the kept entries in candidate order, with
+//             value g_i / p_i (consecutive lanes write consecutive slots).
 // ---------------------------------------------------------------------------
-constexpr int kEmitChunks = 8;
-constexpr int kEmitBatch = 8;                           // decision words per warp whose loads are in flight together
-constexpr int kEmitWords = kEmitChunks * kChunk / 32;   // decision words of the largest tile
-constexpr unsigned long long kFlagAgg = 1ull << 62, kFlagInc = 2ull << 62, kValMask = (1ull << 62) - 1;
-constexpr long long kSpinLimit = 1ll << 22;
+constexpr int kEmitWarps = 8;
+constexpr int kEmitBatch = 4;                            // candidate rounds whose loads are in flight together
+constexpr int kBitWords = kChunk / 32;                   // decision words per chunk
+constexpr int kSliceLog = 10;                            // sum slices of 1024 coordinates
+constexpr int kSlice = 1 << kSliceLog;
+constexpr int kSlices = kChunk / kSlice;                 // 16 slices per chunk
 
-__device__ __forceinline__ unsigned long long ld_acquire(const unsigned long long* p) {
-    unsigned long long v;
-    asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
-    return v;
+__device__ __forceinline__ Decider chunk_decider(const SegParam& P) {
+    Decider dd;
+    dd.lam = P.lam;
+    dd.lam32 = P.lam32;
+    dd.a_cap = P.a_cap;
+    dd.inv_lam32 = P.inv_lam32;
+    return dd;
 }
-__device__ __forceinline__ void st_release(unsigned long long* p, unsigned long long v) {
-    asm volatile("st.release.gpu.global.u64 [%0], %1;" ::"l"(p), "l"(v) : "memory");
-}
 
-__global__ void __launch_bounds__(kThreads) k_emit(const __grid_constant__ Layout Lo, const SegParam* __restrict__ sp,
-                                                   const __grid_constant__ Lists Ls, int tpw,
-                                                   int32_t* idx, float* val, int32_t* nnz, int64_t cap, int* status) {
-    __shared__ uint32_t bits[kEmitWords];     // decision bit of every candidate of the tile
-    __shared__ int32_t wpre[kEmitWords];      // kept candidates before each word
-    __shared__ int s_tile;
-    __shared__ int s_pre[kEmitChunks + 1];    // candidate prefix over the tile's chunks
-    __shared__ long long s_region[kEmitChunks];
-    __shared__ Decider s_dec[kEmitChunks];
-    __shared__ long long s_prefix;
-    __shared__ int shi[33];
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    if (tid == 0) s_tile = atomicAdd(Ls.ticket, 1);
-    __syncthreads();
-    const int t = s_tile;
-    const int m = t / tpw;
-    const int tw = t - m * tpw;                 // tile index within the worker
-    const int k0 = tw * kEmitChunks;
-    const int nck = min(kEmitChunks, Lo.cpw - k0);
-    const int cbase = m * Lo.cpw + k0;
-    if (tid < nck) {
-        const int c = cbase + tid;
-        const Chunk ch = decode_chunk(Lo, c);
-        const SegParam P = sp[ch.seg];
-        Decider dd;
-        dd.lam = P.lam;
-        dd.lam32 = P.lam32;
-        dd.a_cap = P.a_cap;
-        dd.inv_lam32 = P.inv_lam32;
-        s_dec[tid] = dd;
-        s_region[tid] = (long long)ch.m * Lo.d + ch.lo;
-        s_pre[tid + 1] = Ls.p_cnt[c];
-    }
-    if (tid == 0) s_pre[0] = 0;
-    __syncthreads();
-    if (tid == 0)
-        for (int k = 0; k < nck; ++k) s_pre[k + 1] += s_pre[k];
-    __syncthreads();
-    const int n = s_pre[nck];
-    const int nw = (n + 31) >> 5;
-    const PhiloxStream ph(Lo, Lo.worker0 + (uint32_t)m);
-
-    // Pass 1: decisions.  Warp w takes the 32-candidate words w, w + kWarps, ...
-    // in batches of kEmitBatch words whose loads are all issued first.  A tile
-    // that fits one batch keeps its candidates in registers for pass 2.
-    auto chunk_of = [&](int e) -> int {
-        int k = 0;
+__global__ void __launch_bounds__(kEmitWarps * 32) k_decide(const __grid_constant__ Layout Lo,
+                                                            const SegParam* __restrict__ sp,
+                                                            const __grid_constant__ Lists Ls, int n_chunks) {
+    const int lane = threadIdx.x & 31;
+    const int c = blockIdx.x * kEmitWarps + (threadIdx.x >> 5);
+    if (c >= n_chunks) return;
+    const Chunk ch = decode_chunk(Lo, c);
+    const Decider dd = chunk_decider(sp[ch.seg]);
+    const int n = Ls.p_cnt[c];
+    const int2* ent = Ls.p_ent + (int64_t)ch.m * Lo.d + ch.lo;
+    const PhiloxStream ph(Lo, Lo.worker0 + (uint32_t)ch.m);
+    uint32_t* wb = Ls.e_bits + (size_t)c * kBitWords;
+    int32_t* ks = Ls.k_sub + (size_t)c * kSubStride;
+    const int lo32 = (int)ch.lo;
+    int cnt = 0, last_sub = 0;   // kept so far; slice of the last candidate seen
+    for (int base = 0; base < n; base += 32 * kEmitBatch) {
+        int2 e[kEmitBatch];
 #pragma unroll
-        for (int step = kEmitChunks / 2; step > 0; step >>= 1)
-            if (k + step < nck && s_pre[k + step] <= e) k += step;
-        return k;
-    };
-    int2 ent[kEmitBatch];
-    int kk[kEmitBatch];
-    for (int base = 0; base < nw; base += kEmitBatch * kWarps) {
-#pragma unroll
-        for (int b = 0; b < kEmitBatch; ++b) {
-            const int e = (base + b * kWarps + warp) * 32 + lane;
-            kk[b] = -1;
-            if (e < n) {
-                kk[b] = chunk_of(e);
-                ent[b] = Ls.p_ent[s_region[kk[b]] + (e - s_pre[kk[b]])];
-            }
+        for (int r = 0; r < kEmitBatch; ++r) {
+            const int i = base + r * 32 + lane;
+            e[r] = i < n ? ent[i] : make_int2(0, 0);
         }
 #pragma unroll
-        for (int b = 0; b < kEmitBatch; ++b) {
-            const int wd = base + b * kWarps + warp;
+        for (int r = 0; r < kEmitBatch; ++r) {
+            const int i = base + r * 32 + lane;
             bool keep = false;
-            if (kk[b] >= 0) {
-                const uint32_t x = word_of(ph.words((uint32_t)ent[b].x >> 2), ent[b].x & 3);
+            if (i < n) {
+                const uint32_t x = word_of(ph.words((uint32_t)e[r].x >> 2), e[r].x & 3);
                 float v;
-                keep = s_dec[kk[b]](__int_as_float(ent[b].y), x, v);
+                keep = dd(__int_as_float(e[r].y), x, v);
             }
             const uint32_t bal = __ballot_sync(0xFFFFFFFFu, keep);
-            if (lane == 0 && wd < nw) bits[wd] = bal;
-        }
-    }
-    __syncthreads();
-    // Kept-count prefix over the decision words (contiguous words per thread).
-    const int per = (nw + kThreads - 1) / kThreads;
-    int mine = 0;
-    for (int k = 0; k < per; ++k) {
-        const int wd = tid * per + k;
-        if (wd < nw) mine += __popc(bits[wd]);
-    }
-    int inc = mine;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        const int u = __shfl_up_sync(0xFFFFFFFFu, inc, o);
-        if (lane >= o) inc += u;
-    }
-    if (lane == 31) shi[warp] = inc;
-    __syncthreads();
-    int before = 0;
-    for (int w = 0; w < warp; ++w) before += shi[w];
-    int run = before + inc - mine;
-    for (int k = 0; k < per; ++k) {
-        const int wd = tid * per + k;
-        if (wd < nw) {
-            wpre[wd] = run;
-            run += __popc(bits[wd]);
-        }
-    }
-    __syncthreads();
-    auto kept_before = [&](int e) -> int {   // kept candidates of the tile before candidate e
-        if (e >= n) return nw ? wpre[nw - 1] + __popc(bits[nw - 1]) : 0;
-        return wpre[e >> 5] + __popc(bits[e >> 5] & ((1u << (e & 31)) - 1u));
-    };
-    if (warp == 0) {
-        // Decoupled look-back, one warp: lane l inspects tile t-1-l of the same
-        // worker; the nearest inclusive prefix ends the walk, aggregates before
-        // it are summed; otherwise the window moves back by 32 tiles.
-        const long long cnt = kept_before(n);
-        unsigned long long* st = Ls.k_state;
-        long long prefix = 0;
-        if (lane == 0) st_release(&st[t], (tw == 0 ? kFlagInc : kFlagAgg) | (unsigned long long)cnt);
-        int j = t - 1;                  // newest tile of the current window
-        const int first = t - tw;       // the worker's first tile (publishes an inclusive prefix at once)
-        bool done = tw == 0;
-        while (!done) {
-            const int mine = j - lane;
-            unsigned long long w = kFlagInc;   // lanes before the worker's first tile read as empty inclusives
-            if (mine >= first) {
-                long long spins = 0;
-                while (((w = ld_acquire(&st[mine])) >> 62) == 0 && ++spins < kSpinLimit) __nanosleep(32);
-                if ((w >> 62) == 0) {
-                    atomicOr(status, kStTimeout);
-                    w = kFlagInc;
-                }
+            if (base + r * 32 < n) {
+                if (lane == 0) wb[(base >> 5) + r] = bal;
+                // Candidates are in ascending order: a candidate that opens slices
+                // (prev, sub] records the kept count before it for each of them.
+                const int sub = i < n ? (e[r].x - lo32) >> kSliceLog : kSlices;
+                int prev = __shfl_up_sync(0xFFFFFFFFu, sub, 1);
+                if (lane == 0) prev = last_sub;
+                const int before = cnt + __popc(bal & ((1u << lane) - 1u));
+                for (int t = prev + 1; t <= sub && t <= kSlices; ++t) ks[t] = before;
+                last_sub = __shfl_sync(0xFFFFFFFFu, sub, 31);
             }
-            const unsigned inc_mask = __ballot_sync(0xFFFFFFFFu, (w >> 62) == 2);
-            const int stop = inc_mask ? __ffs(inc_mask) - 1 : 32;   // nearest inclusive in the window
-            long long v = lane <= stop && lane < 32 ? (long long)(w & kValMask) : 0;
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xFFFFFFFFu, v, o);
-            prefix += v;
-            if (inc_mask) done = true;
-            else j -= 32;
-        }
-        if (lane == 0) {
-            if (tw != 0) st_release(&st[t], kFlagInc | (unsigned long long)(prefix + cnt));
-            s_prefix = prefix;
-            for (int k = 0; k < nck; ++k) Ls.k_off[cbase + k] = (int32_t)(prefix + kept_before(s_pre[k]));
-            if (k0 + nck == Lo.cpw) {
-                const long long total = prefix + cnt;
-                nnz[m] = (int32_t)total;
-                if (total > cap) atomicOr(status, kStCapacity);
-            }
+            cnt += __popc(bal);
         }
     }
-    __syncthreads();
+    // Slices after the last candidate (all of them if there is none).
+    if (n == 0) last_sub = 0;
+    if (lane <= kSlices && lane > last_sub) ks[lane] = cnt;
+    if (lane == 0) {
+        ks[0] = 0;
+        Ls.k_off[c] = cnt;
+    }
+}
 
-    // Pass 2: kept entries in candidate order (consecutive lanes write consecutive slots).
-    const long long prefix = s_prefix;
-    const int64_t out0 = (int64_t)m * cap;
-    const bool in_regs = nw <= kEmitBatch * kWarps;
-    for (int base = 0; base < nw; base += kEmitBatch * kWarps) {
+__global__ void __launch_bounds__(1024) k_scan(const __grid_constant__ Layout Lo, const __grid_constant__ Lists Ls,
+                                               int32_t* nnz, int64_t cap, int* status) {
+    __shared__ int s_w[32];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int m = blockIdx.x;
+    int32_t* a = Ls.k_off + (size_t)m * Lo.cpw;
+    long long carry = 0;
+    for (int base = 0; base < Lo.cpw; base += 1024) {
+        const int i = base + tid;
+        const int v = i < Lo.cpw ? a[i] : 0;
+        int inc = v;
 #pragma unroll
-        for (int b = 0; b < kEmitBatch; ++b) {
-            const int wd = base + b * kWarps + warp;
-            if (wd >= nw) continue;
-            const uint32_t word = bits[wd];
-            if ((word >> lane) & 1u) {
-                const int e = wd * 32 + lane;
-                int k;
-                int2 en;
-                if (in_regs) {
-                    k = kk[b];
-                    en = ent[b];
-                } else {
-                    k = chunk_of(e);
-                    en = Ls.p_ent[s_region[k] + (e - s_pre[k])];
-                }
-                const float gv = __int_as_float(en.y);
-                const float v = fabsf(gv) >= s_dec[k].a_cap ? gv : copysignf(s_dec[k].inv_lam32, gv);
-                const long long pos = prefix + wpre[wd] + __popc(word & ((1u << lane) - 1u));
-                if (pos < cap) {
-                    idx[out0 + pos] = en.x;
-                    val[out0 + pos] = v;
-                }
+        for (int o = 1; o < 32; o <<= 1) {
+            const int u = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+            if (lane >= o) inc += u;
+        }
+        if (lane == 31) s_w[warp] = inc;
+        __syncthreads();
+        if (warp == 0) {
+            int t = s_w[lane];
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int u = __shfl_up_sync(0xFFFFFFFFu, t, o);
+                if (lane >= o) t += u;
+            }
+            s_w[lane] = t;   // inclusive over warps
+        }
+        __syncthreads();
+        const int before = warp ? s_w[warp - 1] : 0;
+        if (i < Lo.cpw) a[i] = (int32_t)(carry + before + inc - v);
+        carry += s_w[31];
+        __syncthreads();
+    }
+    if (tid == 0) {
+        nnz[m] = (int32_t)carry;
+        if (carry > cap) atomicOr(status, kStCapacity);
+    }
+}
+
+__global__ void __launch_bounds__(kEmitWarps * 32) k_emit(const __grid_constant__ Layout Lo,
+                                                          const SegParam* __restrict__ sp,
+                                                          const __grid_constant__ Lists Ls, int n_chunks,
+                                                          int32_t* idx, float* val, int64_t cap) {
+    const int lane = threadIdx.x & 31;
+    const int c = blockIdx.x * kEmitWarps + (threadIdx.x >> 5);
+    if (c >= n_chunks) return;
+    const Chunk ch = decode_chunk(Lo, c);
+    const SegParam& P = sp[ch.seg];
+    const float a_cap = P.a_cap, inv_lam32 = P.inv_lam32;
+    const int n = Ls.p_cnt[c];
+    const int2* ent = Ls.p_ent + (int64_t)ch.m * Lo.d + ch.lo;
+    const uint32_t* wb = Ls.e_bits + (size_t)c * kBitWords;
+    const int64_t out0 = (int64_t)ch.m * cap;
+    long long pos0 = Ls.k_off[c];
+#pragma unroll 4
+    for (int base = 0; base < n; base += 32) {
+        const uint32_t word = wb[base >> 5];
+        if ((word >> lane) & 1u) {
+            const int2 en = ent[base + lane];
+            const float gv = __int_as_float(en.y);
+            const float v = fabsf(gv) >= a_cap ? gv : copysignf(inv_lam32, gv);
+            const long long pos = pos0 + __popc(word & ((1u << lane) - 1u));
+            if (pos < cap) {
+                idx[out0 + pos] = en.x;
+                val[out0 + pos] = v;
             }
         }
+        pos0 += __popc(word);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// k_sum: the sparse sum of Algorithm 1, step 6 over the compacted rows (L == 1),
+// one warp per 1024-coordinate slice.  The slice's entries of worker m are one
+// contiguous run of m's list (k_decide recorded where each slice starts), so
+// a warp gathers the runs of all workers, adds them into a private
+// shared-memory tile in worker order (a worker's entries have distinct
+// indices; __syncwarp separates workers) and writes the slice once.
+// ---------------------------------------------------------------------------
+constexpr int kSumWarps = 8;
+constexpr int kSumRounds = 4;                 // 32-entry rounds whose loads are in flight together
+
+__global__ void __launch_bounds__(kSumWarps * 32) k_sum(const __grid_constant__ Layout Lo,
+                                                        const __grid_constant__ Lists Ls,
+                                                        const int32_t* __restrict__ idx,
+                                                        const float* __restrict__ val, int64_t cap,
+                                                        int n_slices, float* out) {
+    __shared__ float tile[kSumWarps][kSlice];
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    const int gs = blockIdx.x * kSumWarps + w;
+    if (gs >= n_slices) return;
+    const int k = gs / kSlices, sl = gs - k * kSlices;
+    const int64_t t0 = (int64_t)k * kChunk + (int64_t)sl * kSlice;
+    if (t0 >= Lo.d) return;
+    const int tlen = (int)min((int64_t)kSlice, Lo.d - t0);
+    float* acc = tile[w];
+#pragma unroll
+    for (int i = 0; i < kSlice / 32; ++i) acc[i * 32 + lane] = 0.0f;
+    __syncwarp();
+    for (int mb = 0; mb < Lo.M; mb += 32) {
+        // Lane j describes worker mb + j: where its run starts and how long it is.
+        const int m = mb + lane;
+        long long a = 0;
+        int cnt = 0;
+        if (m < Lo.M) {
+            const int c = m * Lo.cpw + k;
+            const int32_t* ks = Ls.k_sub + (size_t)c * kSubStride;
+            const long long o = Ls.k_off[c];
+            long long lo_ = o + ks[sl], hi_ = o + ks[sl + 1];
+            lo_ = lo_ > cap ? cap : lo_;
+            hi_ = hi_ > cap ? cap : hi_;
+            a = (long long)m * cap + lo_;
+            cnt = hi_ > lo_ ? (int)(hi_ - lo_) : 0;
+        }
+        int pre = cnt;   // inclusive prefix over the lanes
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int u = __shfl_up_sync(0xFFFFFFFFu, pre, o);
+            if (lane >= o) pre += u;
+        }
+        const int total = __shfl_sync(0xFFFFFFFFu, pre, 31);
+        for (int base = 0; base < total; base += 32 * kSumRounds) {
+            int jj[kSumRounds], mm[kSumRounds];
+            float vv[kSumRounds];
+#pragma unroll
+            for (int r = 0; r < kSumRounds; ++r) {
+                const int e = base + r * 32 + lane;
+                // owner: the first lane whose inclusive prefix exceeds e
+                int q = 0;
+#pragma unroll
+                for (int step = 16; step > 0; step >>= 1) {
+                    const int pq = __shfl_sync(0xFFFFFFFFu, pre, q + step - 1);
+                    if (pq <= e) q += step;
+                }
+                const int pq0 = __shfl_sync(0xFFFFFFFFu, pre - cnt, q);
+                const long long aq = __shfl_sync(0xFFFFFFFFu, a, q);
+                mm[r] = e < total ? q : 32;
+                jj[r] = 0;
+                vv[r] = 0.0f;
+                if (e < total) {
+                    const long long pos = aq + (e - pq0);
+                    jj[r] = (int)((int64_t)idx[pos] - t0);
+                    vv[r] = val[pos];
+                    if ((unsigned)jj[r] >= (unsigned)tlen) mm[r] = 32;   // never for well-formed lists
+                }
+            }
+            // The workers present in this batch: m_first .. m_last (every lane shuffles).
+            int m_first = 32, m_last = -1;
+#pragma unroll
+            for (int r = 0; r < kSumRounds; ++r)
+                if (mm[r] < 32) {
+                    m_first = min(m_first, mm[r]);
+                    m_last = max(m_last, mm[r]);
+                }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                m_first = min(m_first, __shfl_xor_sync(0xFFFFFFFFu, m_first, o));
+                m_last = max(m_last, __shfl_xor_sync(0xFFFFFFFFu, m_last, o));
+            }
+            for (int q = m_first; q <= m_last; ++q) {
+#pragma unroll
+                for (int r = 0; r < kSumRounds; ++r)
+                    if (mm[r] == q) acc[jj[r]] += vv[r];
+                __syncwarp();
+            }
+        }
+    }
+    float* dst = out + t0;
+    if (tlen == kSlice && (reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
+#pragma unroll
+        for (int i = 0; i < kSlice / 128; ++i)
+            reinterpret_cast<float4*>(dst)[i * 32 + lane] = reinterpret_cast<const float4*>(acc)[i * 32 + lane];
+    } else {
+        for (int i = lane; i < tlen; i += 32) dst[i] = acc[i];
     }
 }
 
@@ -1030,15 +1083,37 @@ cudaError_t launch_solve(const Layout& Lo, SegParam* sp, const Lists& Ls, int n_
     return cudaGetLastError();
 }
 
-int emit_tiles(int M, int cpw) { return M * ((cpw + kEmitChunks - 1) / kEmitChunks); }
-
 cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, int32_t* idx,
-                           float* val, int32_t* nnz, int64_t cap, int* status, cudaStream_t st) {
-    set_launch_error_site("k_emit launch");
-    (void)n_chunks;
-    const int tpw = (Lo.cpw + kEmitChunks - 1) / kEmitChunks;
-    TraceScope ts(kKEmit, st);
-    k_emit<<<Lo.M * tpw, kThreads, 0, st>>>(Lo, sp, Ls, tpw, idx, val, nnz, cap, status);
+                           float* val, int32_t* nnz, int64_t cap, int* status, cudaStream_t st, float* sum_out) {
+    const int blocks = (n_chunks + kEmitWarps - 1) / kEmitWarps;
+    cudaError_t e;
+    {
+        set_launch_error_site("k_decide launch");
+        TraceScope ts(kKDecide, st);
+        k_decide<<<blocks, kEmitWarps * 32, 0, st>>>(Lo, sp, Ls, n_chunks);
+        e = cudaGetLastError();
+    }
+    if (e != cudaSuccess) return e;
+    {
+        set_launch_error_site("k_scan launch");
+        TraceScope ts(kKScan, st);
+        k_scan<<<Lo.M, 1024, 0, st>>>(Lo, Ls, nnz, cap, status);
+        e = cudaGetLastError();
+    }
+    if (e != cudaSuccess) return e;
+    {
+        set_launch_error_site("k_emit launch");
+        TraceScope ts(kKEmit, st);
+        k_emit<<<blocks, kEmitWarps * 32, 0, st>>>(Lo, sp, Ls, n_chunks, idx, val, cap);
+        e = cudaGetLastError();
+    }
+    if (e != cudaSuccess || !sum_out) return e;
+    // The sparse sum of the M compacted rows (L == 1), one warp per slice.
+    const int n_slices = Lo.cpw * kSlices;
+    set_launch_error_site("k_sum launch");
+    TraceScope ts(kKSum, st);
+    k_sum<<<(n_slices + kSumWarps - 1) / kSumWarps, kSumWarps * 32, 0, st>>>(Lo, Ls, idx, val, cap, n_slices,
+                                                                             sum_out);
     return cudaGetLastError();
 }
 
@@ -1075,19 +1150,6 @@ cudaError_t launch_aggregate(const AggArgs& A, int32_t* off, float* out, int* st
     const int tg = std::min(nt, sm_count() * 4);
     TraceScope ts(kKTiles, st);
     k_tiles<kAggTile><<<tg, kThreads, kAggTile * sizeof(float), st>>>(A, off, nt + 1, nt, out);
-    return cudaGetLastError();
-}
-
-// The sparse sum straight after a batched sparsify of whole rows: the
-// chunk offsets of k_emit are the tile table (tile = chunk), so no bucket pass.
-cudaError_t launch_aggregate_chunks(const AggArgs& A, const int32_t* k_off, int cpw, float* out, cudaStream_t st) {
-    set_launch_error_site("k_tiles (chunk table) launch");
-    const size_t smem = kChunk * sizeof(float);
-    cudaError_t e = cudaFuncSetAttribute(k_tiles<kChunk>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    const int tg = std::min(cpw, sm_count() * 3);
-    TraceScope ts(kKTiles, st);
-    k_tiles<kChunk><<<tg, kThreads, smem, st>>>(A, k_off, cpw, cpw, out);
     return cudaGetLastError();
 }
 

@@ -32,11 +32,13 @@ cudaError_t launch_stream(const Layout& Lo, const SegParam* sp, const Lists& Ls,
                           cudaStream_t st);
 cudaError_t launch_solve(const Layout& Lo, SegParam* sp, const Lists& Ls, int n_seg, double kappa, int iters,
                          int force_exact, int* status, gs_info_dev* info, cudaStream_t st);
+// Decide, scan and compact; with sum_out (L == 1 only) also the sparse sum of
+// the M compacted rows into sum_out (d fp32), fused with the compaction.
 cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, int32_t* idx,
-                           float* val, int32_t* nnz, int64_t cap, int* status, cudaStream_t st);
+                           float* val, int32_t* nnz, int64_t cap, int* status, cudaStream_t st,
+                           float* sum_out = nullptr);
 cudaError_t launch_prob(const Layout& Lo, const SegParam* sp, float* p, cudaStream_t st);
 cudaError_t launch_aggregate(const AggArgs& A, int32_t* off, float* out, int* status, cudaStream_t st);
-cudaError_t launch_aggregate_chunks(const AggArgs& A, const int32_t* k_off, int cpw, float* out, cudaStream_t st);
 cudaError_t launch_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t i0, int64_t n, uint32_t* out,
                          cudaStream_t st);
 bool stream_tma_eligible(const Layout& Lo);
@@ -46,7 +48,6 @@ cudaError_t launch_stream_tma(const Layout& Lo, const SegParam* sp, const Lists&
 void set_launch_error_site(const char* where);
 const char* launch_error_site();
 int agg_tiles(int64_t d);
-int emit_tiles(int M, int cpw);
 int chunk_size();
 
 }  // namespace gs

@@ -380,7 +380,6 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
             A.Ls.s_low[c] = (double)acc_hi + (double)acc_lo;
             A.Ls.c_cnt[c] = runC;
             if (A.Ls.p_cnt) A.Ls.p_cnt[c] = runP;
-            if (A.Ls.k_state) A.Ls.k_state[c] = 0ull;
         }
     }
     // After a timeout, wait (bounded) for the copies still in flight into this

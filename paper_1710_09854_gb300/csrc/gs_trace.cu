@@ -14,7 +14,7 @@ namespace {
 
 const char* kNames[kNumKernels] = {"k_bound", "k_stream", "k_solve", "k_emit",
                                    "k_prob",  "k_words",  "k_bucket", "k_tiles",
-                                   "k_stream_tma"};
+                                   "k_stream_tma", "k_decide", "k_scan", "k_sum"};
 
 struct Pending {
     int k;

@@ -15,6 +15,9 @@ enum KernelId : int {
     kKBucket,
     kKTiles,
     kKStreamTma,
+    kKDecide,
+    kKScan,
+    kKSum,
     kNumKernels
 };
 
