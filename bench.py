@@ -265,8 +265,8 @@ def run_gpu(args):
         "k_stream": M * d * esz,                 # one read of g
         "k_stream_tma": M * d * esz,             # one read of g
         "k_emit": nnz_total * 8,                 # the (idx, val) codes written
+        "k_sum": nnz_total * 8 + d * 4,          # codes read, dense sum written
         "k_tiles": nnz_total * 8 + d * 4,        # codes read, dense sum written
-        "k_count": 0,
     }
     kb = kernel_bytes.get(dom_name, 0)
     achieved = kb / (per_launch_ms / 1e3) / 1e9 if kb else 0.0
@@ -337,31 +337,38 @@ def run_e2e(gs, g, kappa, w, args, dev, stream, ws):
             "api": "gs_pipeline_host", "host_memory": "pinned"}
 
 
+KERNEL_SOURCES = {"k_stream_tma": ("gs_stream_tma.cu", "gs_device.cuh")}
+
+
+def source_digest(kernel):
+    """sha256 over the source files that define `kernel`."""
+    import hashlib
+    src = os.path.join(ROOT, "paper_1710_09854_gb300", "csrc")
+    h = hashlib.sha256()
+    for fn in KERNEL_SOURCES.get(kernel, ("gs_kernels.cu", "gs_device.cuh")):
+        with open(os.path.join(src, fn), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
 def load_traffic(kernel, workload, dtype, kappa):
-    """DRAM bytes per launch of `kernel` from the committed ncu summary, if it
-    was taken on the current kernel build (profiles/traffic.json)."""
-    path = os.path.join(ROOT, "profiles", "traffic.json")
+    """DRAM bytes per launch of `kernel` (ncu dram__bytes_read.sum +
+    dram__bytes_write.sum) from profiles/traffic.txt, if that figure was taken
+    on the kernel's current source (its sha256 matches); else None.
+    Line format: kernel workload dtype kappa bytes_per_launch sha256."""
+    path = os.path.join(ROOT, "profiles", "traffic.txt")
     try:
-        with open(path) as f:
-            t = json.load(f)
-    except (OSError, ValueError):
-        return None
-    key = f"{kernel}:{workload}:{dtype}:{kappa}"
-    ent = t.get(key)
-    if not ent:
-        return None
-    try:
-        src = os.path.join(ROOT, "paper_1710_09854_gb300", "csrc")
-        import hashlib
-        h = hashlib.sha256()
-        for fn in sorted(os.listdir(src)):
-            with open(os.path.join(src, fn), "rb") as f:
-                h.update(f.read())
-        if ent.get("csrc_sha256") != h.hexdigest():
-            return None
+        lines = open(path).read().splitlines()
+        digest = source_digest(kernel)
     except OSError:
         return None
-    return ent.get("bytes_per_launch")
+    for line in lines:
+        f = line.split()
+        if len(f) != 6 or line.startswith("#"):
+            continue
+        if f[0] == kernel and f[1] == workload and f[2] == dtype and float(f[3]) == float(kappa):
+            return int(f[4]) if f[5] == digest else None
+    return None
 
 
 # ---------------------------------------------------------------------------
