@@ -67,7 +67,8 @@ struct SegParam {
     float inv_lam32;   // fl32(1 / lam): the amplified value of uncapped entries
     int iters_run;
     int flags;
-    int pad;
+    int done;          // chunks of the segment whose streaming outputs are written (zeroed by k_bound)
+    int w_done;        // segment l == 0 only: chunks of the worker that k_decide has finished (zeroed by k_bound)
 };
 
 // Candidate lists written by the streaming pass, one region per chunk at the

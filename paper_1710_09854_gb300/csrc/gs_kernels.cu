@@ -234,22 +234,6 @@ __device__ void segment_stats(const Layout& Lo, int m, int64_t lo, int64_t hi, f
 // Block-wide helpers over kThreads threads.
 // ---------------------------------------------------------------------------
 // Sum of two doubles over the block (one reduction); every thread gets both.
-__device__ __forceinline__ double2 block_sum2(double a, double b, double2* sh) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
-    a = warp_sum(a);
-    b = warp_sum(b);
-    __syncthreads();
-    if (lane == 0) sh[warp] = make_double2(a, b);
-    __syncthreads();
-    if (warp == 0) {
-        double2 t = lane < nw ? sh[lane] : make_double2(0.0, 0.0);
-        t.x = warp_sum(t.x);
-        t.y = warp_sum(t.y);
-        if (lane == 0) sh[32] = t;
-    }
-    __syncthreads();
-    return sh[32];
-}
 
 // Exclusive scan of cnt[0..n) into pre[0..n]; pre[n] = total.  `pre` may live
 // in shared or global memory (written and read back by this block only).
@@ -333,15 +317,19 @@ __device__ __forceinline__ float2 block_sum2f(float a, float b, float2* sh) {
 // every iteration's sums are exchanged through distributed shared memory
 // and added in rank order, so all CTAs of the cluster follow the same path.
 constexpr int kBoundCTAs = 8;
-constexpr int kBoundCtaThreads = 256;
+constexpr int kBoundCtaThreads = 1024;
+constexpr int kBoundRun = 8;             // consecutive coordinates read per stratum
 
+// The 8 CTAs of a cluster share the segment's random sample loads (a run of
+// kBoundRun consecutive coordinates from each of ns / kBoundRun strata) and
+// store the |g| values straight into rank 0's shared memory; rank 0 then runs Algorithm 3
+// to its fixed point on the sample alone, with block-wide sums.
 __global__ void __cluster_dims__(kBoundCTAs, 1, 1) __launch_bounds__(kBoundCtaThreads)
     k_bound(Layout Lo, SegParam* sp, double kappa, int ns, int force_exact) {
     namespace cg = cooperative_groups;
     cg::cluster_group cluster = cg::this_cluster();
-    extern __shared__ float sa[];               // this CTA's ns / kBoundCTAs samples
+    extern __shared__ float sa[];               // rank 0: all ns samples
     __shared__ float2 sh2[33];
-    __shared__ float2 xch[2];                   // this CTA's partial sums, double-buffered by iteration
     const int rank = (int)cluster.block_rank();
     const int s = blockIdx.x / kBoundCTAs, tid = threadIdx.x;
     int m, l, c0, c1;
@@ -352,6 +340,8 @@ __global__ void __cluster_dims__(kBoundCTAs, 1, 1) __launch_bounds__(kBoundCtaTh
     if (len <= ns || force_exact) {
         // Short segment (or exact mode): every coordinate is a candidate.
         if (rank == 0 && tid == 0) {
+            P.done = 0;
+            P.w_done = 0;
             P.lam_up = (double)kInf;
             P.lam_up32 = kInf;
             P.t_c = 0.0f;
@@ -359,38 +349,35 @@ __global__ void __cluster_dims__(kBoundCTAs, 1, 1) __launch_bounds__(kBoundCtaTh
         }
         return;   // uniform over the cluster: no CTA reaches a cluster barrier
     }
-    const int per = ns / kBoundCTAs;
-    const uint32_t q = (uint32_t)(len / ns);                        // stratum width (the last one takes the rest)
-    const uint32_t q_last = (uint32_t)(len - (int64_t)(ns - 1) * q);
+    // ns / 8 strata; from each, 8 consecutive coordinates starting at a
+    // random multiple of 8 (one 32-byte sector of fp32 g).
+    const int per = ns / (kBoundRun * kBoundCTAs);                  // strata of this CTA
+    const int nst = per * kBoundCTAs;
+    ns = nst * kBoundRun;                                           // samples actually drawn
+    const int64_t q = len / nst;                                    // stratum width (the last one takes the rest)
+    const int64_t q_last = len - (int64_t)(nst - 1) * q;
     const uint32_t hs = mix32((uint32_t)s + 0x68E31DA4u);
-    float ls = 0.0f;
-#pragma unroll 8
-    for (int kk = tid; kk < per; kk += kBoundCtaThreads) {
-        const int k = rank * per + kk;
+    float* dst = cluster.map_shared_rank(sa, 0);
+    for (int e = tid; e < per * kBoundRun; e += kBoundCtaThreads) {
+        const int k = rank * per + e / kBoundRun;                   // stratum
+        const int r = e % kBoundRun;
         const uint32_t h = mix32((uint32_t)k * 0x9E3779B9u ^ hs);
-        const int64_t pos = lo + (int64_t)k * q + (int64_t)(h % (k == ns - 1 ? q_last : q));
+        const int64_t width = k == nst - 1 ? q_last : q;            // >= kBoundRun since len > ns
+        const int64_t runs = width / kBoundRun;
+        int64_t start = lo + (int64_t)k * q + (int64_t)(h % (uint32_t)runs) * kBoundRun;
+        start -= (start + (int64_t)m * Lo.d) % kBoundRun;           // align the run to the flat index
+        if (start < lo + (int64_t)k * q) start += kBoundRun;
+        const int64_t pos = min(start + r, hi - 1);
         float x = fabsf(load_one(Lo, m, pos));
         if (!(x < kInf)) x = 0.0f;  // non-finite values are reported by the solve
-        sa[kk] = x;
-        ls += x;
+        dst[k * kBoundRun + r] = x;
     }
-    // Cluster-wide sums of (a, b): local block sum, then every CTA adds the
-    // kBoundCTAs partials in rank order.
-    int buf = 0;
-    auto cluster_sum2 = [&](float a, float b) -> float2 {
-        const float2 loc = block_sum2f(a, b, sh2);
-        if (tid == 0) xch[buf] = loc;
-        cluster.sync();
-        float2 r = make_float2(0.0f, 0.0f);
-        for (int k = 0; k < kBoundCTAs; ++k) {
-            const float2 v = *cluster.map_shared_rank(&xch[buf], k);
-            r.x += v.x;
-            r.y += v.y;
-        }
-        buf ^= 1;
-        return r;
-    };
-    const float S = cluster_sum2(ls, 0.0f).x;
+    cluster.sync();   // the sample is complete in rank 0; nobody touches another CTA's memory after this
+    if (rank != 0) return;
+
+    float ls = 0.0f;
+    for (int k = tid; k < ns; k += kBoundCtaThreads) ls += sa[k];
+    const float S = block_sum2f(ls, 0.0f, sh2).x;
     const float budget = (float)(kappa * (double)ns);
     float lam = S > 0.0f ? budget / S : 0.0f;
     float K = 0.0f, Su = S;
@@ -398,11 +385,11 @@ __global__ void __cluster_dims__(kBoundCTAs, 1, 1) __launch_bounds__(kBoundCtaTh
     for (int it = 0; it < 32 && !take_all; ++it) {
         const float acap = 1.0f / lam;
         float su = 0.0f, kc = 0.0f;
-        for (int kk = tid; kk < per; kk += kBoundCtaThreads) {
-            const float x = sa[kk];
+        for (int k = tid; k < ns; k += kBoundCtaThreads) {
+            const float x = sa[k];
             if (x >= acap) kc += 1.0f; else su += x;
         }
-        const float2 r = cluster_sum2(kc, su);
+        const float2 r = block_sum2f(kc, su, sh2);
         K = r.x;
         Su = r.y;
         if (!(Su > 0.0f)) { take_all = true; break; }
@@ -410,8 +397,9 @@ __global__ void __cluster_dims__(kBoundCTAs, 1, 1) __launch_bounds__(kBoundCtaTh
         if (!(c > 1.0f + 1e-5f)) break;
         lam *= c;
     }
-    cluster.sync();   // no CTA may leave while a peer still reads its partials
-    if (rank == 0 && tid == 0) {
+    if (tid == 0) {
+        P.done = 0;
+        P.w_done = 0;
         const double e = take_all ? 0.0 : (double)lam * Su / budget;  // uncapped share of the budget
         if (take_all || K >= budget || !(lam > 0.0f)) {
             P.lam_up = (double)kInf;
@@ -452,6 +440,34 @@ __global__ void __launch_bounds__(kThreads) k_stream(Layout Lo, const SegParam* 
 // ---------------------------------------------------------------------------
 constexpr int kSolveSmemChunks = 8192;   // chunk-prefix entries kept in shared memory
 constexpr int kSolveSmemC = 12288;       // candidate values kept in shared memory
+constexpr int kSolvePer = 4;             // chunks per thread of the one-round start (segments <= 1024 chunks)
+
+// Exclusive prefix of v over the block (any blockDim <= 1024) and the total.
+__device__ __forceinline__ int block_scan_total(int v, int* sh, int& total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+    int inc = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int t = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+        if (lane >= o) inc += t;
+    }
+    if (lane == 31) sh[warp] = inc;
+    __syncthreads();
+    if (warp == 0) {
+        int t = lane < nw ? sh[lane] : 0;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int u = __shfl_up_sync(0xFFFFFFFFu, t, o);
+            if (lane >= o) t += u;
+        }
+        sh[lane] = t;
+    }
+    __syncthreads();
+    const int before = warp > 0 ? sh[warp - 1] : 0;
+    total = sh[nw - 1];
+    __syncthreads();
+    return before + inc - v;
+}
 
 struct CView {
     const float* smem;       // compacted candidates (nC <= kSolveSmemC), else NULL
@@ -466,17 +482,32 @@ struct CView {
     }
 };
 
-// (#{a >= acap}, sum of the other a) over C; NaN acap sums everything.  The
-// sum is carried error-free in fp32 pairs, so no fp64 arithmetic per value.
-__device__ double2 c_stats(const CView& C, float acap, float4* sh4) {
-    float hi = 0.0f, lo = 0.0f;
-    int k = 0;
+// c_stats as block-wide float totals: (hi, lo) error-free pair of the sum
+// and the count, in every thread; no fp64 arithmetic.
+__device__ __forceinline__ void c_stats_f(const CView& C, float acap, float4* sh4, float& hi, float& lo, int& k) {
+    hi = 0.0f;
+    lo = 0.0f;
+    k = 0;
     for (int e = threadIdx.x; e < C.nC; e += blockDim.x) {
         const float a = C.at(e);
         if (a >= acap) ++k; else two_sum_add(hi, lo, a);
     }
     block_sum_df(hi, lo, k, sh4);
-    return make_double2((double)k, (double)hi + (double)lo);
+}
+
+// Sum of one double per thread, added by warp 0 alone (fixed order); every
+// thread receives it.  `sh` holds blockDim.x + 1 doubles.
+__device__ __forceinline__ double warp0_sum_double(double v, double* sh) {
+    sh[threadIdx.x] = v;
+    __syncthreads();
+    if (threadIdx.x < 32) {
+        double t = 0.0;
+        for (int i = threadIdx.x; i < blockDim.x; i += 32) t += sh[i];
+        t = warp_sum(t);
+        if (threadIdx.x == 0) sh[blockDim.x] = t;
+    }
+    __syncthreads();
+    return sh[blockDim.x];
 }
 
 __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lists Ls, double kappa, int iters,
@@ -488,6 +519,9 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
     __shared__ double shd[33];
     __shared__ int shi[33];
     __shared__ float s_acap;
+    __shared__ double shdd[kThreads + 1];
+    __shared__ double s_S, s_lam;
+    __shared__ int s_go, s_fresh, s_j;
     const int s = blockIdx.x, tid = threadIdx.x;
     int m, l, c0, c1;
     int64_t lo, hi;
@@ -500,24 +534,73 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
     // Candidate view: chunk prefix (shared or global scratch), values gathered to shared memory when they fit.
     const int nch = c1 - c0;
     int32_t* pre = nch <= kSolveSmemChunks ? spre : Ls.c_pre + c0 + s;
-    block_exclusive_scan(Ls.c_cnt + c0, nch, pre, shi);
     CView C;
     C.pre = pre;
     C.nch = nch;
-    C.nC = pre[nch];
     C.gbase = Ls.c_val + (int64_t)m * Lo.d + lo;
     C.smem = nullptr;
-    if (C.nC <= kSolveSmemC) {
-        for (int e = tid; e < C.nC; e += blockDim.x) sc[e] = C.at(e);
-        __syncthreads();
-        C.smem = sc;
-    }
-
     double sl = 0.0;
-    for (int c = c0 + tid; c < c1; c += blockDim.x) sl += Ls.s_low[c];
-    const double S_low = block_sum(sl, shd);
-    const double2 all = c_stats(C, __int_as_float(0x7FC00000), sh4);
-    double S = S_low + all.y;
+    if (nch <= kSolvePer * kThreads) {
+        // Every chunk count and l1 partial in one round of loads (kSolvePer
+        // consecutive chunks per thread), one block scan, and each thread
+        // copies its own chunks' values of C.
+        int cnt[kSolvePer];
+        int tot = 0;
+#pragma unroll
+        for (int j = 0; j < kSolvePer; ++j) {
+            const int c = c0 + kSolvePer * tid + j;
+            cnt[j] = c < c1 ? Ls.c_cnt[c] : 0;
+            sl += c < c1 ? Ls.s_low[c] : 0.0;
+            tot += cnt[j];
+        }
+        int total;
+        int run = block_scan_total(tot, shi, total);
+#pragma unroll
+        for (int j = 0; j < kSolvePer; ++j) {
+            if (kSolvePer * tid + j < nch) pre[kSolvePer * tid + j] = run;
+            run += cnt[j];
+        }
+        if (tid == 0) pre[nch] = total;
+        C.nC = total;
+        if (total <= kSolveSmemC) {
+            int at = run - tot;
+#pragma unroll
+            for (int j = 0; j < kSolvePer; ++j) {
+                const int64_t base = (int64_t)(kSolvePer * tid + j) * kChunk;
+                for (int v = 0; v < cnt[j]; ++v) sc[at + v] = C.gbase[base + v];
+                at += cnt[j];
+            }
+            C.smem = sc;
+        }
+        __syncthreads();
+    } else {
+        block_exclusive_scan(Ls.c_cnt + c0, nch, pre, shi);
+        C.nC = pre[nch];
+        if (C.nC <= kSolveSmemC) {
+            for (int e = tid; e < C.nC; e += blockDim.x) sc[e] = C.at(e);
+            __syncthreads();
+            C.smem = sc;
+        }
+        for (int c = c0 + tid; c < c1; c += blockDim.x) sl += Ls.s_low[c];
+    }
+    // fp64 is slow on this part: fp64 sums run in warp 0 only, and the scalar
+    // recurrence of Algorithm 3 runs in thread 0 (broadcast through shared memory).
+    const double S_low = warp0_sum_double(sl, shdd);
+    float rh, rl;
+    int rk;
+    c_stats_f(C, __int_as_float(0x7FC00000), sh4, rh, rl, rk);
+    if (tid == 0) {
+        const double S0 = S_low + ((double)rh + (double)rl);
+        const bool run = isfinite(S0) && force_exact == 0 && S0 > 0.0;
+        s_S = S0;
+        s_lam = run ? budget / S0 : 0.0;
+        s_go = run && iters > 0 ? 1 : 0;
+        s_fresh = 0;
+        s_j = 0;
+        s_acap = cap_threshold(s_lam);
+    }
+    __syncthreads();
+    double S = s_S;
 
     double lam = 0.0, K = 0.0, Su = 0.0;
     int j = 0;
@@ -526,23 +609,35 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
         flags |= kSegNonfinite;
         if (tid == 0) atomicOr(status, kStNonfinite);
     } else if (!exact && S > 0.0) {
-        lam = budget / S;
-        while (j < iters) {
-            if (tid == 0) s_acap = cap_threshold(lam);
+        while (s_go) {
+            c_stats_f(C, s_acap, sh4, rh, rl, rk);
+            if (tid == 0) {
+                double lv = s_lam;
+                int go = 0, fresh = 1;      // fresh: (rh, rl, rk) are the stats at the final lambda
+                const double A = lv * (S_low + ((double)rh + (double)rl));
+                if (A != 0.0) {
+                    const double cc = (budget - (double)rk) / A;
+                    if (cc > 1.0) {
+                        lv = cc * lv;
+                        ++s_j;
+                        go = s_j < iters;
+                        fresh = 0;
+                        s_acap = cap_threshold(lv);
+                    }
+                }
+                s_lam = lv;
+                s_go = go;
+                s_fresh = fresh;
+            }
             __syncthreads();
-            const double2 r = c_stats(C, s_acap, sh4);
-            const double A = lam * (S_low + r.y);
-            if (A == 0.0) break;
-            const double cc = (budget - r.x) / A;
-            if (!(cc > 1.0)) break;
-            lam = cc * lam;
-            ++j;
         }
-        if (tid == 0) s_acap = cap_threshold(lam);
-        __syncthreads();
-        const double2 r = c_stats(C, s_acap, sh4);
-        K = r.x;
-        Su = S_low + r.y;
+        if (!s_fresh) c_stats_f(C, s_acap, sh4, rh, rl, rk);
+        lam = s_lam;
+        j = s_j;
+        if (tid == 0) {
+            K = (double)rk;
+            Su = S_low + ((double)rh + (double)rl);
+        }
         // The lists are exact only while lambda stays within the bound.
         if (lam > lam_up) exact = true;
     }
@@ -641,9 +736,9 @@ struct Decider {
 // Compaction in three steps with no waits between chunks:
 //   k_decide  one warp per chunk: draws each candidate's Philox word again,
 //             records its decision as one bit (a warp ballot per 32
-//             candidates) and the chunk's kept count;
-//   k_scan    one CTA per worker: exclusive prefix of the kept counts over
-//             the worker's chunks (the output offset of every chunk), nnz;
+//             candidates) and the chunk's kept count; the last warp to finish
+//             a worker's chunks turns its counts into output offsets
+//             (exclusive prefix) and writes nnz;
 //   k_emit    one warp per chunk: the kept entries in candidate order, with
 //             value g_i / p_i (consecutive lanes write consecutive slots).
 // ---------------------------------------------------------------------------
@@ -653,6 +748,7 @@ constexpr int kBitWords = kChunk / 32;                   // decision words per c
 constexpr int kSliceLog = 10;                            // sum slices of 1024 coordinates
 constexpr int kSlice = 1 << kSliceLog;
 constexpr int kSlices = kChunk / kSlice;                 // 16 slices per chunk
+constexpr int kScanPer = 8;                              // chunk counts per lane per step of the worker scan
 
 __device__ __forceinline__ Decider chunk_decider(const SegParam& P) {
     Decider dd;
@@ -663,9 +759,9 @@ __device__ __forceinline__ Decider chunk_decider(const SegParam& P) {
     return dd;
 }
 
-__global__ void __launch_bounds__(kEmitWarps * 32) k_decide(const __grid_constant__ Layout Lo,
-                                                            const SegParam* __restrict__ sp,
-                                                            const __grid_constant__ Lists Ls, int n_chunks) {
+__global__ void __launch_bounds__(kEmitWarps * 32) k_decide(const __grid_constant__ Layout Lo, SegParam* sp,
+                                                            const __grid_constant__ Lists Ls, int n_chunks,
+                                                            int32_t* nnz, int64_t cap, int* status) {
     const int lane = threadIdx.x & 31;
     const int c = blockIdx.x * kEmitWarps + (threadIdx.x >> 5);
     if (c >= n_chunks) return;
@@ -716,43 +812,42 @@ __global__ void __launch_bounds__(kEmitWarps * 32) k_decide(const __grid_constan
         ks[0] = 0;
         Ls.k_off[c] = cnt;
     }
-}
 
-__global__ void __launch_bounds__(1024) k_scan(const __grid_constant__ Layout Lo, const __grid_constant__ Lists Ls,
-                                               int32_t* nnz, int64_t cap, int* status) {
-    __shared__ int s_w[32];
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int m = blockIdx.x;
-    int32_t* a = Ls.k_off + (size_t)m * Lo.cpw;
+    // The last warp to finish one of the worker's chunks turns the worker's
+    // counts into output offsets (exclusive prefix) and writes nnz.
+    __threadfence();
+    int last = 0;
+    if (lane == 0) last = atomicAdd(&sp[ch.m * Lo.L].w_done, 1) == Lo.cpw - 1;
+    if (!__shfl_sync(0xFFFFFFFFu, last, 0)) return;
+    __threadfence();
+    int32_t* ko = Ls.k_off + (size_t)ch.m * Lo.cpw;
     long long carry = 0;
-    for (int base = 0; base < Lo.cpw; base += 1024) {
-        const int i = base + tid;
-        const int v = i < Lo.cpw ? a[i] : 0;
-        int inc = v;
+    for (int base = 0; base < Lo.cpw; base += 32 * kScanPer) {
+        int v[kScanPer];
+        int tot = 0;
+#pragma unroll
+        for (int j = 0; j < kScanPer; ++j) {
+            const int i = base + lane * kScanPer + j;
+            v[j] = i < Lo.cpw ? __ldcg(ko + i) : 0;
+            tot += v[j];
+        }
+        int inc = tot;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
             const int u = __shfl_up_sync(0xFFFFFFFFu, inc, o);
             if (lane >= o) inc += u;
         }
-        if (lane == 31) s_w[warp] = inc;
-        __syncthreads();
-        if (warp == 0) {
-            int t = s_w[lane];
+        long long run = carry + (inc - tot);
 #pragma unroll
-            for (int o = 1; o < 32; o <<= 1) {
-                const int u = __shfl_up_sync(0xFFFFFFFFu, t, o);
-                if (lane >= o) t += u;
-            }
-            s_w[lane] = t;   // inclusive over warps
+        for (int j = 0; j < kScanPer; ++j) {
+            const int i = base + lane * kScanPer + j;
+            if (i < Lo.cpw) ko[i] = (int32_t)run;
+            run += v[j];
         }
-        __syncthreads();
-        const int before = warp ? s_w[warp - 1] : 0;
-        if (i < Lo.cpw) a[i] = (int32_t)(carry + before + inc - v);
-        carry += s_w[31];
-        __syncthreads();
+        carry += __shfl_sync(0xFFFFFFFFu, inc, 31);
     }
-    if (tid == 0) {
-        nnz[m] = (int32_t)carry;
+    if (lane == 0) {
+        nnz[ch.m] = (int32_t)carry;
         if (carry > cap) atomicOr(status, kStCapacity);
     }
 }
@@ -1053,7 +1148,7 @@ int sm_count() {
 cudaError_t launch_bound(const Layout& Lo, SegParam* sp, int n_seg, double kappa, int ns, int force_exact,
                          cudaStream_t st) {
     set_launch_error_site("k_bound launch");
-    const size_t smem = (size_t)(ns / kBoundCTAs) * sizeof(float);
+    const size_t smem = (size_t)ns * sizeof(float);
     if (smem > 48 * 1024) {
         cudaError_t e = cudaFuncSetAttribute(k_bound, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
@@ -1090,14 +1185,7 @@ cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls
     {
         set_launch_error_site("k_decide launch");
         TraceScope ts(kKDecide, st);
-        k_decide<<<blocks, kEmitWarps * 32, 0, st>>>(Lo, sp, Ls, n_chunks);
-        e = cudaGetLastError();
-    }
-    if (e != cudaSuccess) return e;
-    {
-        set_launch_error_site("k_scan launch");
-        TraceScope ts(kKScan, st);
-        k_scan<<<Lo.M, 1024, 0, st>>>(Lo, Ls, nnz, cap, status);
+        k_decide<<<blocks, kEmitWarps * 32, 0, st>>>(Lo, const_cast<SegParam*>(sp), Ls, n_chunks, nnz, cap, status);
         e = cudaGetLastError();
     }
     if (e != cudaSuccess) return e;
