@@ -482,17 +482,22 @@ struct CView {
     }
 };
 
-// c_stats as block-wide float totals: (hi, lo) error-free pair of the sum
-// and the count, in every thread; no fp64 arithmetic.
-__device__ __forceinline__ void c_stats_f(const CView& C, float acap, float4* sh4, float& hi, float& lo, int& k) {
+// c_stats for one warp: every lane receives (hi, lo, count).
+__device__ __forceinline__ void warp_c_stats(const CView& C, float acap, float& hi, float& lo, int& k) {
     hi = 0.0f;
     lo = 0.0f;
     k = 0;
-    for (int e = threadIdx.x; e < C.nC; e += blockDim.x) {
+    for (int e = threadIdx.x & 31; e < C.nC; e += 32) {
         const float a = C.at(e);
         if (a >= acap) ++k; else two_sum_add(hi, lo, a);
     }
-    block_sum_df(hi, lo, k, sh4);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float oh = __shfl_xor_sync(0xFFFFFFFFu, hi, o);
+        const float ol = __shfl_xor_sync(0xFFFFFFFFu, lo, o);
+        df_add(hi, lo, oh, ol);
+        k += __shfl_xor_sync(0xFFFFFFFFu, k, o);
+    }
 }
 
 // Sum of one double per thread, added by warp 0 alone (fixed order); every
@@ -515,13 +520,12 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
     extern __shared__ unsigned char dsm[];
     int32_t* spre = reinterpret_cast<int32_t*>(dsm);                       // kSolveSmemChunks + 1
     float* sc = reinterpret_cast<float*>(dsm + sizeof(int32_t) * (kSolveSmemChunks + 4));  // kSolveSmemC
-    __shared__ float4 sh4[33];
     __shared__ double shd[33];
     __shared__ int shi[33];
     __shared__ float s_acap;
     __shared__ double shdd[kThreads + 1];
-    __shared__ double s_S, s_lam;
-    __shared__ int s_go, s_fresh, s_j;
+    __shared__ double s_S, s_lam, s_K, s_Su;
+    __shared__ int s_go, s_j;
     const int s = blockIdx.x, tid = threadIdx.x;
     int m, l, c0, c1;
     int64_t lo, hi;
@@ -583,63 +587,55 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
         }
         for (int c = c0 + tid; c < c1; c += blockDim.x) sl += Ls.s_low[c];
     }
-    // fp64 is slow on this part: fp64 sums run in warp 0 only, and the scalar
-    // recurrence of Algorithm 3 runs in thread 0 (broadcast through shared memory).
+    // fp64 is slow on this part and C is small: the l1 partials are summed and
+    // Algorithm 3 is iterated by warp 0 alone (warp shuffles only; every lane
+    // carries the same scalars), then the result is broadcast.
     const double S_low = warp0_sum_double(sl, shdd);
-    float rh, rl;
-    int rk;
-    c_stats_f(C, __int_as_float(0x7FC00000), sh4, rh, rl, rk);
-    if (tid == 0) {
+    if (tid < 32) {
+        float rh, rl;
+        int rk;
+        warp_c_stats(C, __int_as_float(0x7FC00000), rh, rl, rk);
         const double S0 = S_low + ((double)rh + (double)rl);
-        const bool run = isfinite(S0) && force_exact == 0 && S0 > 0.0;
-        s_S = S0;
-        s_lam = run ? budget / S0 : 0.0;
-        s_go = run && iters > 0 ? 1 : 0;
-        s_fresh = 0;
-        s_j = 0;
-        s_acap = cap_threshold(s_lam);
+        double lv = 0.0;
+        int jj = 0;
+        bool ex = force_exact != 0;
+        if (isfinite(S0) && !ex && S0 > 0.0) {
+            lv = budget / S0;
+            float acap = cap_threshold(lv);
+            bool fresh = false;   // (rh, rl, rk) are the stats at acap
+            while (jj < iters) {
+                warp_c_stats(C, acap, rh, rl, rk);
+                fresh = true;
+                const double A = lv * (S_low + ((double)rh + (double)rl));
+                if (A == 0.0) break;
+                const double cc = (budget - (double)rk) / A;
+                if (!(cc > 1.0)) break;
+                lv = cc * lv;
+                ++jj;
+                acap = cap_threshold(lv);
+                fresh = false;
+            }
+            if (!fresh) warp_c_stats(C, acap, rh, rl, rk);
+            // The lists are exact only while lambda stays within the bound.
+            if (lv > lam_up) ex = true;
+        }
+        if (tid == 0) {
+            s_S = S0;
+            s_lam = lv;
+            s_j = jj;
+            s_go = ex ? 1 : 0;
+            s_K = (double)rk;
+            s_Su = S_low + ((double)rh + (double)rl);
+        }
     }
     __syncthreads();
     double S = s_S;
-
-    double lam = 0.0, K = 0.0, Su = 0.0;
-    int j = 0;
-    bool exact = force_exact != 0;
+    double lam = s_lam, K = s_K, Su = s_Su;
+    int j = s_j;
+    bool exact = s_go != 0;
     if (!isfinite(S)) {
         flags |= kSegNonfinite;
         if (tid == 0) atomicOr(status, kStNonfinite);
-    } else if (!exact && S > 0.0) {
-        while (s_go) {
-            c_stats_f(C, s_acap, sh4, rh, rl, rk);
-            if (tid == 0) {
-                double lv = s_lam;
-                int go = 0, fresh = 1;      // fresh: (rh, rl, rk) are the stats at the final lambda
-                const double A = lv * (S_low + ((double)rh + (double)rl));
-                if (A != 0.0) {
-                    const double cc = (budget - (double)rk) / A;
-                    if (cc > 1.0) {
-                        lv = cc * lv;
-                        ++s_j;
-                        go = s_j < iters;
-                        fresh = 0;
-                        s_acap = cap_threshold(lv);
-                    }
-                }
-                s_lam = lv;
-                s_go = go;
-                s_fresh = fresh;
-            }
-            __syncthreads();
-        }
-        if (!s_fresh) c_stats_f(C, s_acap, sh4, rh, rl, rk);
-        lam = s_lam;
-        j = s_j;
-        if (tid == 0) {
-            K = (double)rk;
-            Su = S_low + ((double)rh + (double)rl);
-        }
-        // The lists are exact only while lambda stays within the bound.
-        if (lam > lam_up) exact = true;
     }
 
     if (exact && isfinite(S)) {
@@ -867,20 +863,29 @@ __global__ void __launch_bounds__(kEmitWarps * 32) k_emit(const __grid_constant_
     const uint32_t* wb = Ls.e_bits + (size_t)c * kBitWords;
     const int64_t out0 = (int64_t)ch.m * cap;
     long long pos0 = Ls.k_off[c];
-#pragma unroll 4
-    for (int base = 0; base < n; base += 32) {
-        const uint32_t word = wb[base >> 5];
-        if ((word >> lane) & 1u) {
-            const int2 en = ent[base + lane];
-            const float gv = __int_as_float(en.y);
-            const float v = fabsf(gv) >= a_cap ? gv : copysignf(inv_lam32, gv);
-            const long long pos = pos0 + __popc(word & ((1u << lane) - 1u));
-            if (pos < cap) {
-                idx[out0 + pos] = en.x;
-                val[out0 + pos] = v;
-            }
+    for (int base = 0; base < n; base += 32 * kEmitBatch) {
+        // All loads of kEmitBatch rounds first (candidates are ~all kept).
+        uint32_t wd[kEmitBatch];
+        int2 en[kEmitBatch];
+#pragma unroll
+        for (int r = 0; r < kEmitBatch; ++r) {
+            const int i = base + r * 32 + lane;
+            wd[r] = base + r * 32 < n ? wb[(base >> 5) + r] : 0u;
+            en[r] = i < n ? ent[i] : make_int2(0, 0);
         }
-        pos0 += __popc(word);
+#pragma unroll
+        for (int r = 0; r < kEmitBatch; ++r) {
+            if ((wd[r] >> lane) & 1u) {
+                const float gv = __int_as_float(en[r].y);
+                const float v = fabsf(gv) >= a_cap ? gv : copysignf(inv_lam32, gv);
+                const long long pos = pos0 + __popc(wd[r] & ((1u << lane) - 1u));
+                if (pos < cap) {
+                    idx[out0 + pos] = en[r].x;
+                    val[out0 + pos] = v;
+                }
+            }
+            pos0 += __popc(wd[r]);
+        }
     }
 }
 
@@ -888,19 +893,20 @@ __global__ void __launch_bounds__(kEmitWarps * 32) k_emit(const __grid_constant_
 // k_sum: the sparse sum of Algorithm 1, step 6 over the compacted rows (L == 1),
 // one warp per 1024-coordinate slice.  The slice's entries of worker m are one
 // contiguous run of m's list (k_decide recorded where each slice starts), so
-// a warp gathers the runs of all workers, adds them into a private
-// shared-memory tile in worker order (a worker's entries have distinct
-// indices; __syncwarp separates workers) and writes the slice once.
+// a warp gathers the runs of all workers (lane i takes entry i of a run),
+// adds them into a private shared-memory tile worker by worker (a worker's
+// entries have distinct indices; __syncwarp separates workers) and writes
+// the slice once.
 // ---------------------------------------------------------------------------
 constexpr int kSumWarps = 8;
-constexpr int kSumRounds = 4;                 // 32-entry rounds whose loads are in flight together
+constexpr int kSumGroup = 8;                  // workers whose entries are loaded together
 
 __global__ void __launch_bounds__(kSumWarps * 32) k_sum(const __grid_constant__ Layout Lo,
                                                         const __grid_constant__ Lists Ls,
                                                         const int32_t* __restrict__ idx,
                                                         const float* __restrict__ val, int64_t cap,
                                                         int n_slices, float* out) {
-    __shared__ float tile[kSumWarps][kSlice];
+    __shared__ __align__(16) float tile[kSumWarps][kSlice];
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
     const int gs = blockIdx.x * kSumWarps + w;
     if (gs >= n_slices) return;
@@ -910,72 +916,66 @@ __global__ void __launch_bounds__(kSumWarps * 32) k_sum(const __grid_constant__ 
     const int tlen = (int)min((int64_t)kSlice, Lo.d - t0);
     float* acc = tile[w];
 #pragma unroll
-    for (int i = 0; i < kSlice / 32; ++i) acc[i * 32 + lane] = 0.0f;
+    for (int i = 0; i < kSlice / 128; ++i)
+        reinterpret_cast<float4*>(acc)[i * 32 + lane] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
     __syncwarp();
     for (int mb = 0; mb < Lo.M; mb += 32) {
-        // Lane j describes worker mb + j: where its run starts and how long it is.
-        const int m = mb + lane;
+        // Lane q describes worker mb + q: where its run starts and how long it is.
+        const int nq = min(32, Lo.M - mb);
         long long a = 0;
         int cnt = 0;
-        if (m < Lo.M) {
-            const int c = m * Lo.cpw + k;
+        if (lane < nq) {
+            const int c = (mb + lane) * Lo.cpw + k;
             const int32_t* ks = Ls.k_sub + (size_t)c * kSubStride;
             const long long o = Ls.k_off[c];
             long long lo_ = o + ks[sl], hi_ = o + ks[sl + 1];
             lo_ = lo_ > cap ? cap : lo_;
             hi_ = hi_ > cap ? cap : hi_;
-            a = (long long)m * cap + lo_;
+            a = (long long)(mb + lane) * cap + lo_;
             cnt = hi_ > lo_ ? (int)(hi_ - lo_) : 0;
         }
-        int pre = cnt;   // inclusive prefix over the lanes
+        int maxc = cnt;
 #pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int u = __shfl_up_sync(0xFFFFFFFFu, pre, o);
-            if (lane >= o) pre += u;
-        }
-        const int total = __shfl_sync(0xFFFFFFFFu, pre, 31);
-        for (int base = 0; base < total; base += 32 * kSumRounds) {
-            int jj[kSumRounds], mm[kSumRounds];
-            float vv[kSumRounds];
+        for (int o = 16; o > 0; o >>= 1) maxc = max(maxc, __shfl_xor_sync(0xFFFFFFFFu, maxc, o));
+        if (maxc <= 32) {
+            // Every run fits one round: lane i takes entry i of each worker; the
+            // loads of kSumGroup workers are issued together, then the adds run
+            // worker by worker (a worker's entries have distinct indices).
+            for (int q0 = 0; q0 < nq; q0 += kSumGroup) {
+                int jj[kSumGroup];
+                float vv[kSumGroup];
 #pragma unroll
-            for (int r = 0; r < kSumRounds; ++r) {
-                const int e = base + r * 32 + lane;
-                // owner: the first lane whose inclusive prefix exceeds e
-                int q = 0;
-#pragma unroll
-                for (int step = 16; step > 0; step >>= 1) {
-                    const int pq = __shfl_sync(0xFFFFFFFFu, pre, q + step - 1);
-                    if (pq <= e) q += step;
+                for (int u = 0; u < kSumGroup; ++u) {
+                    const int q = q0 + u;
+                    const long long aq = __shfl_sync(0xFFFFFFFFu, a, q & 31);
+                    const int cq = __shfl_sync(0xFFFFFFFFu, cnt, q & 31);
+                    jj[u] = -1;
+                    vv[u] = 0.0f;
+                    if (q < nq && lane < cq) {
+                        const int j = (int)((int64_t)idx[aq + lane] - t0);
+                        vv[u] = val[aq + lane];
+                        if ((unsigned)j < (unsigned)tlen) jj[u] = j;   // always, for well-formed lists
+                    }
                 }
-                const int pq0 = __shfl_sync(0xFFFFFFFFu, pre - cnt, q);
+#pragma unroll
+                for (int u = 0; u < kSumGroup; ++u) {
+                    if (jj[u] >= 0) acc[jj[u]] += vv[u];
+                    __syncwarp();
+                }
+            }
+        } else {
+            // Long runs: worker by worker, 32 entries at a time.
+            for (int q = 0; q < nq; ++q) {
                 const long long aq = __shfl_sync(0xFFFFFFFFu, a, q);
-                mm[r] = e < total ? q : 32;
-                jj[r] = 0;
-                vv[r] = 0.0f;
-                if (e < total) {
-                    const long long pos = aq + (e - pq0);
-                    jj[r] = (int)((int64_t)idx[pos] - t0);
-                    vv[r] = val[pos];
-                    if ((unsigned)jj[r] >= (unsigned)tlen) mm[r] = 32;   // never for well-formed lists
+                const int cq = __shfl_sync(0xFFFFFFFFu, cnt, q);
+                for (int e0 = 0; e0 < cq; e0 += 32) {
+                    const int e = e0 + lane;
+                    if (e < cq) {
+                        const int j = (int)((int64_t)idx[aq + e] - t0);
+                        const float v = val[aq + e];
+                        if ((unsigned)j < (unsigned)tlen) acc[j] += v;
+                    }
                 }
-            }
-            // The workers present in this batch: m_first .. m_last (every lane shuffles).
-            int m_first = 32, m_last = -1;
-#pragma unroll
-            for (int r = 0; r < kSumRounds; ++r)
-                if (mm[r] < 32) {
-                    m_first = min(m_first, mm[r]);
-                    m_last = max(m_last, mm[r]);
-                }
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) {
-                m_first = min(m_first, __shfl_xor_sync(0xFFFFFFFFu, m_first, o));
-                m_last = max(m_last, __shfl_xor_sync(0xFFFFFFFFu, m_last, o));
-            }
-            for (int q = m_first; q <= m_last; ++q) {
-#pragma unroll
-                for (int r = 0; r < kSumRounds; ++r)
-                    if (mm[r] == q) acc[jj[r]] += vv[r];
                 __syncwarp();
             }
         }
