@@ -225,7 +225,11 @@ gs_status gs_random_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t
  *   GS_OPT_SAMPLE_SIZE        sampled coordinates per segment for the bound
  *                              on lambda (default 16384; a multiple of 8 in
  *                              256 .. 32768).
- *   GS_OPT_KERNEL_TIMING      1: time every kernel launch (gs_kernel_times).
+ *   GS_OPT_KERNEL_TIMING      1: time every kernel launch (gs_kernel_times);
+ *                              2: time the streaming pass only.  The events
+ *                              sit between launches, so a timed kernel does
+ *                              not overlap its neighbours' launch (mode 2
+ *                              leaves the rest of the chain overlapped).
  *   GS_OPT_STREAM_PATH        streaming pass over g: 0 automatic (the TMA
  *                              kernel whenever the layout allows it), 1 the
  *                              generic-load kernel, 2 the TMA kernel where

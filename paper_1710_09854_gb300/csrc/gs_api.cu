@@ -317,6 +317,7 @@ gs_status noalloc_device(NoAllocDev** out) {
 // Turns the call's status bits into one gs_status code (same precedence as
 // gs_sync_status) for the caller's word.
 __global__ void k_noalloc_status(const int* bits, int32_t* code) {
+    grid_dep_wait();
     const int h = *bits;
     int32_t c = GS_OK;
     if (h & kStNonfinite) c = GS_ERR_NONFINITE;
@@ -528,7 +529,7 @@ gs_status gs_set_option(int option, int64_t value) {
             g_stream_path = (int)value;
             return GS_OK;
         case GS_OPT_KERNEL_TIMING:
-            if (value != 0 && value != 1) return GS_ERR_INVALID_ARG;
+            if (value < 0 || value > 2) return GS_ERR_INVALID_ARG;
             trace_set_timing((int)value);
             return GS_OK;
         default:

@@ -201,6 +201,13 @@ __device__ __forceinline__ uint32_t word_of(const uint4& w, int s) {
     return s == 0 ? w.x : (s == 1 ? w.y : (s == 2 ? w.z : w.w));
 }
 
+// Programmatic dependent launch: a kernel launched with programmatic stream
+// serialization may start while its predecessor in the stream still runs;
+// this waits until the predecessor grid has completed and its writes are
+// visible.  Every kernel of the library calls it first, unconditionally (a
+// plain launch returns at once), so completion stays transitive down the stream.
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // 1 + (x >> 9) * 2^-23: a float in [1, 2) that never exceeds 1 + x * 2^-32.
 // hi(x * 2^23) = x >> 9, so one multiply-add forms it on the integer-multiply pipe.
 __device__ __forceinline__ float unit_plus_one(uint32_t x) {

@@ -326,6 +326,7 @@ constexpr int kBoundRun = 8;             // consecutive coordinates read per str
 // to its fixed point on the sample alone, with block-wide sums.
 __global__ void __cluster_dims__(kBoundCTAs, 1, 1) __launch_bounds__(kBoundCtaThreads)
     k_bound(Layout Lo, SegParam* sp, double kappa, int ns, int force_exact) {
+    grid_dep_wait();
     namespace cg = cooperative_groups;
     cg::cluster_group cluster = cg::this_cluster();
     extern __shared__ float sa[];               // rank 0: all ns samples
@@ -424,6 +425,7 @@ __global__ void __cluster_dims__(kBoundCTAs, 1, 1) __launch_bounds__(kBoundCtaTh
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(kThreads) k_stream(Layout Lo, const SegParam* __restrict__ sp, Lists Ls,
                                                      int n_chunks, int build_p) {
+    grid_dep_wait();
     for (int c = blockIdx.x; c < n_chunks; c += gridDim.x) {
         const Chunk ch = decode_chunk(Lo, c);
         chunk_candidates<true>(Lo, c, ch, sp[ch.seg].lam_up32, sp[ch.seg].t_c, Ls, build_p != 0);
@@ -517,6 +519,7 @@ __device__ __forceinline__ double warp0_sum_double(double v, double* sh) {
 
 __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lists Ls, double kappa, int iters,
                                                     int force_exact, int* status, gs_info_dev* info) {
+    grid_dep_wait();
     extern __shared__ unsigned char dsm[];
     int32_t* spre = reinterpret_cast<int32_t*>(dsm);                       // kSolveSmemChunks + 1
     float* sc = reinterpret_cast<float*>(dsm + sizeof(int32_t) * (kSolveSmemChunks + 4));  // kSolveSmemC
@@ -758,6 +761,7 @@ __device__ __forceinline__ Decider chunk_decider(const SegParam& P) {
 __global__ void __launch_bounds__(kEmitWarps * 32) k_decide(const __grid_constant__ Layout Lo, SegParam* sp,
                                                             const __grid_constant__ Lists Ls, int n_chunks,
                                                             int32_t* nnz, int64_t cap, int* status) {
+    grid_dep_wait();
     const int lane = threadIdx.x & 31;
     const int c = blockIdx.x * kEmitWarps + (threadIdx.x >> 5);
     if (c >= n_chunks) return;
@@ -852,6 +856,7 @@ __global__ void __launch_bounds__(kEmitWarps * 32) k_emit(const __grid_constant_
                                                           const SegParam* __restrict__ sp,
                                                           const __grid_constant__ Lists Ls, int n_chunks,
                                                           int32_t* idx, float* val, int64_t cap) {
+    grid_dep_wait();
     const int lane = threadIdx.x & 31;
     const int c = blockIdx.x * kEmitWarps + (threadIdx.x >> 5);
     if (c >= n_chunks) return;
@@ -906,6 +911,7 @@ __global__ void __launch_bounds__(kSumWarps * 32) k_sum(const __grid_constant__ 
                                                         const int32_t* __restrict__ idx,
                                                         const float* __restrict__ val, int64_t cap,
                                                         int n_slices, float* out) {
+    grid_dep_wait();
     __shared__ __align__(16) float tile[kSumWarps][kSlice];
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
     const int gs = blockIdx.x * kSumWarps + w;
@@ -994,6 +1000,7 @@ __global__ void __launch_bounds__(kSumWarps * 32) k_sum(const __grid_constant__ 
 // Dense probabilities of one worker: p_i = min(lambda |g_i|, 1).
 // ---------------------------------------------------------------------------
 __global__ void k_prob(Layout Lo, const SegParam* __restrict__ sp, float* p) {
+    grid_dep_wait();
     const SegParam P = sp[0];
     const int64_t n = Lo.d;
     for (int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (int64_t)gridDim.x * blockDim.x) {
@@ -1004,6 +1011,7 @@ __global__ void k_prob(Layout Lo, const SegParam* __restrict__ sp, float* p) {
 
 // Random words of coordinates i0 .. i0 + n - 1 (one Philox call per thread per word).
 __global__ void k_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t i0, int64_t n, uint32_t* out) {
+    grid_dep_wait();
     for (int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; k < n; k += (int64_t)gridDim.x * blockDim.x) {
         const int64_t i = i0 + k;
         out[k] = word_of(group_words(seed, step, worker, i >> 2), (int)(i & 3));
@@ -1018,6 +1026,7 @@ __global__ void k_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t i
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) k_bucket(const __grid_constant__ AggArgs A, int32_t* off, int nt,
                                                 int* status) {
+    grid_dep_wait();
     constexpr int kUnroll = 8;   // entries per thread whose loads are in flight together
     const int m = blockIdx.y;
     const int32_t* __restrict__ idx = A.idx[m];
@@ -1068,6 +1077,7 @@ template <int kTile>
 __global__ void __launch_bounds__(kThreads) k_tiles(const __grid_constant__ AggArgs A,
                                                     const int32_t* __restrict__ off, int off_stride, int nt,
                                                     float* out) {
+    grid_dep_wait();
     extern __shared__ float acc[];   // kTile floats
     __shared__ int32_t s_pre[kMaxAggM + 1];
     __shared__ long long s_lo[kMaxAggM];
@@ -1154,8 +1164,8 @@ cudaError_t launch_bound(const Layout& Lo, SegParam* sp, int n_seg, double kappa
         if (e != cudaSuccess) return e;
     }
     TraceScope ts(kKBound, st);
-    k_bound<<<n_seg * kBoundCTAs, kBoundCtaThreads, smem, st>>>(Lo, sp, kappa, ns, force_exact);
-    return cudaGetLastError();
+    return launch_dep(k_bound, dim3(n_seg * kBoundCTAs), dim3(kBoundCtaThreads), smem, st, Lo, sp, kappa, ns,
+                      force_exact);
 }
 
 cudaError_t launch_stream(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, bool build_p,
@@ -1163,8 +1173,7 @@ cudaError_t launch_stream(const Layout& Lo, const SegParam* sp, const Lists& Ls,
     set_launch_error_site("k_stream launch");
     const int grid = std::min(n_chunks, sm_count() * 8);
     TraceScope ts(kKStream, st);
-    k_stream<<<grid, kThreads, 0, st>>>(Lo, sp, Ls, n_chunks, build_p ? 1 : 0);
-    return cudaGetLastError();
+    return launch_dep(k_stream, dim3(grid), dim3(kThreads), 0, st, Lo, sp, Ls, n_chunks, build_p ? 1 : 0);
 }
 
 cudaError_t launch_solve(const Layout& Lo, SegParam* sp, const Lists& Ls, int n_seg, double kappa, int iters,
@@ -1174,8 +1183,8 @@ cudaError_t launch_solve(const Layout& Lo, SegParam* sp, const Lists& Ls, int n_
     cudaError_t e = cudaFuncSetAttribute(k_solve, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     TraceScope ts(kKSolve, st);
-    k_solve<<<n_seg, kThreads, smem, st>>>(Lo, sp, Ls, kappa, iters, force_exact, status, info);
-    return cudaGetLastError();
+    return launch_dep(k_solve, dim3(n_seg), dim3(kThreads), smem, st, Lo, sp, Ls, kappa, iters, force_exact, status,
+                      info);
 }
 
 cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, int32_t* idx,
@@ -1185,32 +1194,29 @@ cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls
     {
         set_launch_error_site("k_decide launch");
         TraceScope ts(kKDecide, st);
-        k_decide<<<blocks, kEmitWarps * 32, 0, st>>>(Lo, const_cast<SegParam*>(sp), Ls, n_chunks, nnz, cap, status);
-        e = cudaGetLastError();
+        e = launch_dep(k_decide, dim3(blocks), dim3(kEmitWarps * 32), 0, st, Lo, const_cast<SegParam*>(sp), Ls,
+                       n_chunks, nnz, cap, status);
     }
     if (e != cudaSuccess) return e;
     {
         set_launch_error_site("k_emit launch");
         TraceScope ts(kKEmit, st);
-        k_emit<<<blocks, kEmitWarps * 32, 0, st>>>(Lo, sp, Ls, n_chunks, idx, val, cap);
-        e = cudaGetLastError();
+        e = launch_dep(k_emit, dim3(blocks), dim3(kEmitWarps * 32), 0, st, Lo, sp, Ls, n_chunks, idx, val, cap);
     }
     if (e != cudaSuccess || !sum_out) return e;
     // The sparse sum of the M compacted rows (L == 1), one warp per slice.
     const int n_slices = Lo.cpw * kSlices;
     set_launch_error_site("k_sum launch");
     TraceScope ts(kKSum, st);
-    k_sum<<<(n_slices + kSumWarps - 1) / kSumWarps, kSumWarps * 32, 0, st>>>(Lo, Ls, idx, val, cap, n_slices,
-                                                                             sum_out);
-    return cudaGetLastError();
+    return launch_dep(k_sum, dim3((n_slices + kSumWarps - 1) / kSumWarps), dim3(kSumWarps * 32), 0, st, Lo, Ls,
+                      static_cast<const int32_t*>(idx), static_cast<const float*>(val), cap, n_slices, sum_out);
 }
 
 cudaError_t launch_prob(const Layout& Lo, const SegParam* sp, float* p, cudaStream_t st) {
     set_launch_error_site("k_prob launch");
     const int64_t blocks = std::min<int64_t>((Lo.d + 255) / 256, (int64_t)sm_count() * 16);
     TraceScope ts(kKProb, st);
-    k_prob<<<(int)blocks, 256, 0, st>>>(Lo, sp, p);
-    return cudaGetLastError();
+    return launch_dep(k_prob, dim3((int)blocks), dim3(256), 0, st, Lo, sp, p);
 }
 
 cudaError_t launch_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t i0, int64_t n, uint32_t* out,

@@ -175,6 +175,7 @@ struct ChunkWalk {
 template <int kDtype>
 __global__ void __launch_bounds__(kTmaThreads, 2)
     k_stream_tma(const __grid_constant__ CUtensorMap map, const __grid_constant__ StreamArgs A) {
+    grid_dep_wait();
     constexpr int kInner = kDtype == 0 ? 32 : 64;          // elements per 128-byte row
     constexpr int kBufRows = kBufCoords / kInner;          // 32 or 16
     constexpr int kBufBytes = kBufRows * kRowBytes;        // 4 KiB or 2 KiB
@@ -479,14 +480,16 @@ cudaError_t launch_stream_tma(const Layout& Lo, const SegParam* sp, const Lists&
         e = cudaFuncSetAttribute(k_stream_tma<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
         set_launch_error_site("k_stream_tma<fp32> launch");
-        k_stream_tma<0><<<grid, kTmaThreads, smem, st>>>(map, A);
+        e = launch_dep(k_stream_tma<0>, dim3(grid), dim3(kTmaThreads), smem, st, map, A);
+        if (e != cudaSuccess) return e;
     } else {
         const size_t smem = tma_smem_bytes<1>();
         set_launch_error_site("k_stream_tma<bf16> shared-memory attribute");
         e = cudaFuncSetAttribute(k_stream_tma<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
         set_launch_error_site("k_stream_tma<bf16> launch");
-        k_stream_tma<1><<<grid, kTmaThreads, smem, st>>>(map, A);
+        e = launch_dep(k_stream_tma<1>, dim3(grid), dim3(kTmaThreads), smem, st, map, A);
+        if (e != cudaSuccess) return e;
     }
     *used = true;
     return cudaGetLastError();

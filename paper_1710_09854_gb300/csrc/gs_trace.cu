@@ -41,7 +41,7 @@ cudaEvent_t take_event() {
 
 }  // namespace
 
-void trace_set_timing(int on) { timing_on.store(on ? 1 : 0); }
+void trace_set_timing(int mode) { timing_on.store(mode); }
 
 namespace {
 thread_local const char* g_site = "kernel launch";
@@ -51,7 +51,8 @@ const char* launch_error_site() { return g_site; }
 
 TraceScope::TraceScope(int k, cudaStream_t st) : k_(k), st_(st), a_(nullptr) {
     launches[k].fetch_add(1);
-    if (timing_on.load()) {
+    const int mode = timing_on.load();   // 1: every kernel; 2: the streaming pass only
+    if (mode == 1 || (mode == 2 && (k == kKStream || k == kKStreamTma))) {
         std::lock_guard<std::mutex> lk(mu);
         a_ = take_event();
         if (a_) cudaEventRecord(a_, st_);
