@@ -291,6 +291,27 @@ def run_gpu(args):
     gs.gs_set_option(gs.GS_OPT_KERNEL_TIMING, 0)
     kernels = {k: {"ms_per_step": round(v[0] / n_bd, 4), "launches": v[1]} for k, v in bd.items() if v[1]}
 
+    # Sparsify alone (steps 1-5, no sum) against B_sparsify, on the same inputs.
+    sp_only = None
+    if off is None:
+        for t in range(3):
+            gs.gs_batched_sparsify(g, kappa, w.iters, w.seed, t, 0, idx, val, nnz, stream=stream)
+        torch.cuda.synchronize()
+        s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s0.record(stream)
+        for t in range(n_bd):
+            gs.gs_batched_sparsify(g, kappa, w.iters, w.seed, args.warmup + t, 0, idx, val, nnz, stream=stream)
+        s1.record(stream)
+        torch.cuda.synchronize()
+        sp_ms = max_over_ranks(s0.elapsed_time(s1) / n_bd, dev)
+        sp_gbs = b_sp / (sp_ms / 1e3) / 1e9
+        sp_only = {"api": "gs_batched_sparsify", "steps": n_bd, "ms_per_step": round(sp_ms, 4),
+                   "algorithmic_bytes": b_sp, "achieved": round(sp_gbs, 1), "peak": hbm,
+                   "frac": round(sp_gbs / hbm, 4), "unit": "GB/s"}
+        rc = gs.gs_sync_status(stream)
+        if rc != gs.GS_OK:
+            raise RuntimeError(f"device status after the sparsify-only run: {gs.status_string(rc)}")
+
     # ---- end to end through the host-buffer entry point
     e2e = None
     if not args.no_e2e and off is None:
@@ -308,6 +329,7 @@ def run_gpu(args):
         "pipeline_roofline": {"bound": "hbm", "algorithmic_bytes": b_sp + b_ag, "achieved": round(pipe_gbs, 1),
                               "peak": hbm, "frac": round(pipe_gbs / hbm, 4), "unit": "GB/s"},
         "roofline": roofline,
+        "sparsify_roofline": sp_only,
         "kernels": kernels, "kernels_steps": n_bd,
         "nnz_per_step": nnz_total,
         "gpu_launches": launches,

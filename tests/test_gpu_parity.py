@@ -309,6 +309,20 @@ def _full_check(gs, g_dev, kappa, iters, seed=1, step=0, workers=None, offsets=N
         gs.gs_segmented_sparsify(g_dev, offsets, kappa, iters, seed, step, 0, idx, val, nnz)
     gs.gs_sparse_aggregate([idx[m] for m in range(M)], [val[m] for m in range(M)], nnz, d, out)
     assert gs.gs_sync_status() == gs.GS_OK
+    if offsets is None:
+        # The fused call (compaction + sum in one chain) equals the two calls bit for bit.
+        idx2 = torch.empty_like(idx)
+        val2 = torch.empty_like(val)
+        nnz2 = torch.empty_like(nnz)
+        out2 = torch.empty_like(out)
+        gs.gs_sparsify_aggregate(g_dev, kappa, iters, seed, step, 0, idx2, val2, nnz2, out2)
+        assert gs.gs_sync_status() == gs.GS_OK
+        assert torch.equal(nnz2, nnz)
+        assert torch.equal(out2, out)
+        for m in range(M):
+            k = int(nnz[m].item())
+            assert torch.equal(idx2[m, :k], idx[m, :k]) and torch.equal(val2[m, :k], val[m, :k])
+        del idx2, val2
     g_host = g_dev.float().cpu().numpy() if dtype == "bf16" else g_dev.cpu().numpy()
     n = nnz.cpu().numpy()
     workers = range(M) if workers is None else workers
@@ -466,3 +480,33 @@ def test_sparsify_aggregate_fused(gs, dtype):
             il = [idx[m, :n[m]].cpu().numpy() for m in range(M)]
             vl = [val[m, :n[m]].cpu().numpy() for m in range(M)]
             np.testing.assert_array_equal(out.cpu().numpy(), oracle.aggregate(il, vl, d))
+
+
+def test_sparsify_aggregate_fused_long_runs_many_workers(gs):
+    """The fused sum with more than 32 workers (several worker batches per
+    slice) and kappa large enough that runs exceed 32 entries per slice."""
+    import torch
+    M, d, kappa, iters, seed, step = 40, 2 * 16384 + 777, 0.2, 2, 5, 9
+    kinds = ["t3", "lognormal", "normal", "ties"]
+    g_host = np.stack([_vector(kinds[m % 4], d, 700 + m) for m in range(M)])
+    g = _dev(g_host)
+    idx = torch.empty((M, d), dtype=torch.int32, device="cuda")
+    val = torch.empty((M, d), dtype=torch.float32, device="cuda")
+    nnz = torch.empty(M, dtype=torch.int32, device="cuda")
+    out = torch.empty(d, dtype=torch.float32, device="cuda")
+    gs.gs_sparsify_aggregate(g, kappa, iters, seed, step, 0, idx, val, nnz, out)
+    assert gs.gs_sync_status() == gs.GS_OK
+    out2 = torch.empty(d, dtype=torch.float32, device="cuda")
+    gs.gs_sparse_aggregate([idx[m] for m in range(M)], [val[m] for m in range(M)], nnz, d, out2)
+    assert gs.gs_sync_status() == gs.GS_OK
+    assert torch.equal(out, out2)
+    n = nnz.cpu().numpy()
+    assert n.max() * 1024 / d > 32   # kept entries per 1024-coordinate slice well above 32
+    il, vl = [], []
+    for m in range(M):
+        ri, rv, _ = oracle.sparsify(g_host[m], kappa, iters, seed, step, m)
+        compare_sparse(idx[m, :n[m]].cpu().numpy(), val[m, :n[m]].cpu().numpy(), g_host[m], kappa, iters, seed,
+                       step, m, ref=(ri, rv, oracle.greedy_lambda(g_host[m], kappa, iters)))
+        il.append(ri)
+        vl.append(rv)
+    compare_sum(out.cpu().numpy(), il, vl, d)
