@@ -443,6 +443,7 @@ __global__ void __launch_bounds__(kThreads) k_stream(Layout Lo, const SegParam* 
 constexpr int kSolveSmemChunks = 8192;   // chunk-prefix entries kept in shared memory
 constexpr int kSolveSmemC = 12288;       // candidate values kept in shared memory
 constexpr int kSolvePer = 4;             // chunks per thread of the one-round start (segments <= 1024 chunks)
+constexpr int kSolveCTAs = 8;            // cluster size of k_solve for long segments
 
 // Exclusive prefix of v over the block (any blockDim <= 1024) and the total.
 __device__ __forceinline__ int block_scan_total(int v, int* sh, int& total) {
@@ -517,9 +518,16 @@ __device__ __forceinline__ double warp0_sum_double(double v, double* sh) {
     return sh[blockDim.x];
 }
 
+// Launched with clusters of 1 or kSolveCTAs CTAs per segment (block x / cluster
+// size = segment).  Small C: the cluster's rank 0 solves alone.  Large C: every
+// CTA of the cluster walks a share of the segment's chunks in each pass and the
+// CTA partials are combined through distributed shared memory in rank order.
 __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lists Ls, double kappa, int iters,
                                                     int force_exact, int* status, gs_info_dev* info) {
     grid_dep_wait();
+    namespace cg = cooperative_groups;
+    cg::cluster_group cluster = cg::this_cluster();
+    const int ncta = (int)cluster.num_blocks(), rank = (int)cluster.block_rank();
     extern __shared__ unsigned char dsm[];
     int32_t* spre = reinterpret_cast<int32_t*>(dsm);                       // kSolveSmemChunks + 1
     float* sc = reinterpret_cast<float*>(dsm + sizeof(int32_t) * (kSolveSmemChunks + 4));  // kSolveSmemC
@@ -528,8 +536,11 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
     __shared__ float s_acap;
     __shared__ double shdd[kThreads + 1];
     __shared__ double s_S, s_lam, s_K, s_Su;
-    __shared__ int s_go, s_j;
-    const int s = blockIdx.x, tid = threadIdx.x;
+    __shared__ int s_go, s_j, s_fresh;
+    __shared__ float4 sh4[33];
+    __shared__ float4 xch[2];           // this CTA's partial (hi, lo, count) of a pass, double-buffered
+    const int s = blockIdx.x / ncta, tid = threadIdx.x;
+    const int lane = tid & 31, warp = tid >> 5;
     int m, l, c0, c1;
     int64_t lo, hi;
     seg_range(Lo, s, m, l, lo, hi, c0, c1);
@@ -594,7 +605,90 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
     // Algorithm 3 is iterated by warp 0 alone (warp shuffles only; every lane
     // carries the same scalars), then the result is broadcast.
     const double S_low = warp0_sum_double(sl, shdd);
-    if (tid < 32) {
+    if (C.smem == nullptr) {
+        // Large C: passes over the segment's chunks shared by the cluster.
+        int buf = 0;
+        auto stats = [&](float acap, float& rh, float& rl, int& rk) {
+            float hi_ = 0.0f, lo_ = 0.0f;
+            int k_ = 0;
+            for (int q = rank * (kThreads / 32) + warp; q < nch; q += ncta * (kThreads / 32)) {
+                const int n = pre[q + 1] - pre[q];
+                const float* src = C.gbase + (int64_t)q * kChunk;
+                for (int e = lane; e < n; e += 32) {
+                    const float a = src[e];
+                    if (a >= acap) ++k_; else two_sum_add(hi_, lo_, a);
+                }
+            }
+            block_sum_df(hi_, lo_, k_, sh4);
+            if (tid == 0) xch[buf] = make_float4(hi_, lo_, __int_as_float(k_), 0.0f);
+            cluster.sync();
+            rh = 0.0f;
+            rl = 0.0f;
+            rk = 0;
+            for (int r = 0; r < ncta; ++r) {
+                const float4 v = *cluster.map_shared_rank(&xch[buf], r);
+                df_add(rh, rl, v.x, v.y);
+                rk += __float_as_int(v.z);
+            }
+            buf ^= 1;
+        };
+        float rh, rl;
+        int rk;
+        stats(__int_as_float(0x7FC00000), rh, rl, rk);
+        if (tid == 0) {
+            const double S0 = S_low + ((double)rh + (double)rl);
+            const bool run = isfinite(S0) && force_exact == 0 && S0 > 0.0;
+            s_S = S0;
+            s_lam = run ? budget / S0 : 0.0;
+            s_go = run && iters > 0 ? 1 : 0;
+            s_fresh = 1;
+            s_j = 0;
+            s_acap = cap_threshold(s_lam);
+            s_K = 0.0;
+            s_Su = S0;
+        }
+        __syncthreads();
+        const bool run = isfinite(s_S) && force_exact == 0 && s_S > 0.0;
+        if (run) {
+            s_fresh = 0;   // the first stats were taken with no threshold
+            __syncthreads();
+            while (s_go) {
+                stats(s_acap, rh, rl, rk);
+                if (tid == 0) {
+                    double lv = s_lam;
+                    int go = 0, fresh = 1;
+                    const double A = lv * (S_low + ((double)rh + (double)rl));
+                    if (A != 0.0) {
+                        const double cc = (budget - (double)rk) / A;
+                        if (cc > 1.0) {
+                            lv = cc * lv;
+                            ++s_j;
+                            go = s_j < iters;
+                            fresh = 0;
+                            s_acap = cap_threshold(lv);
+                        }
+                    }
+                    s_lam = lv;
+                    s_go = go;
+                    s_fresh = fresh;
+                }
+                __syncthreads();
+            }
+            if (!s_fresh) stats(s_acap, rh, rl, rk);
+            if (tid == 0) {
+                s_K = (double)rk;
+                s_Su = S_low + ((double)rh + (double)rl);
+                s_go = s_lam > lam_up ? 1 : 0;    // exact fallback needed
+            }
+        } else if (tid == 0) {
+            s_go = force_exact != 0 ? 1 : 0;
+        }
+        cluster.sync();   // no CTA may leave while a peer still reads its partials
+        if (rank != 0) return;
+        __syncthreads();
+    } else if (rank != 0) {
+        return;           // small C: rank 0 solves alone (uniform over the cluster)
+    } else if (tid < 32) {
         float rh, rl;
         int rk;
         warp_c_stats(C, __int_as_float(0x7FC00000), rh, rl, rk);
@@ -1183,8 +1277,11 @@ cudaError_t launch_solve(const Layout& Lo, SegParam* sp, const Lists& Ls, int n_
     cudaError_t e = cudaFuncSetAttribute(k_solve, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     TraceScope ts(kKSolve, st);
-    return launch_dep(k_solve, dim3(n_seg), dim3(kThreads), smem, st, Lo, sp, Ls, kappa, iters, force_exact, status,
-                      info);
+    // Long segments (where C can hold millions of values) get a cluster of
+    // kSolveCTAs CTAs each; layer-wise segments are short and take one.
+    const int ncta = (Lo.L == 1 && Lo.d >= ((int64_t)1 << 22)) ? kSolveCTAs : 1;
+    return launch_dep_cluster(k_solve, dim3(n_seg * ncta), dim3(kThreads), smem, ncta, st, Lo, sp, Ls, kappa, iters,
+                              force_exact, status, info);
 }
 
 cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, int32_t* idx,
