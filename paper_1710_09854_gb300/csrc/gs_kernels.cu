@@ -880,9 +880,14 @@ __global__ void __launch_bounds__(kEmitWarps * 32) k_decide(const __grid_constan
             const int i = base + r * 32 + lane;
             bool keep = false;
             if (i < n) {
-                const uint32_t x = word_of(ph.words((uint32_t)e[r].x >> 2), e[r].x & 3);
-                float v;
-                keep = dd(__int_as_float(e[r].y), x, v);
+                const float gv = __int_as_float(e[r].y);
+                if (fabsf(gv) >= dd.a_cap) {
+                    keep = true;   // capped: p = 1, kept whatever the draw
+                } else {
+                    const uint32_t x = word_of(ph.words((uint32_t)e[r].x >> 2), e[r].x & 3);
+                    float v;
+                    keep = dd(gv, x, v);
+                }
             }
             const uint32_t bal = __ballot_sync(0xFFFFFFFFu, keep);
             if (base + r * 32 < n) {
@@ -1064,17 +1069,28 @@ __global__ void __launch_bounds__(kSumWarps * 32) k_sum(const __grid_constant__ 
                 }
             }
         } else {
-            // Long runs: worker by worker, 32 entries at a time.
+            // Long runs: worker by worker, kSumGroup rounds of 32 entries loaded
+            // together (a worker's entries never share an index).
             for (int q = 0; q < nq; ++q) {
                 const long long aq = __shfl_sync(0xFFFFFFFFu, a, q);
                 const int cq = __shfl_sync(0xFFFFFFFFu, cnt, q);
-                for (int e0 = 0; e0 < cq; e0 += 32) {
-                    const int e = e0 + lane;
-                    if (e < cq) {
-                        const int j = (int)((int64_t)idx[aq + e] - t0);
-                        const float v = val[aq + e];
-                        if ((unsigned)j < (unsigned)tlen) acc[j] += v;
+                for (int e0 = 0; e0 < cq; e0 += 32 * kSumGroup) {
+                    int jj[kSumGroup];
+                    float vv[kSumGroup];
+#pragma unroll
+                    for (int u = 0; u < kSumGroup; ++u) {
+                        const int e = e0 + u * 32 + lane;
+                        jj[u] = -1;
+                        vv[u] = 0.0f;
+                        if (e < cq) {
+                            const int j = (int)((int64_t)idx[aq + e] - t0);
+                            vv[u] = val[aq + e];
+                            if ((unsigned)j < (unsigned)tlen) jj[u] = j;
+                        }
                     }
+#pragma unroll
+                    for (int u = 0; u < kSumGroup; ++u)
+                        if (jj[u] >= 0) acc[jj[u]] += vv[u];
                 }
                 __syncwarp();
             }
@@ -1277,9 +1293,13 @@ cudaError_t launch_solve(const Layout& Lo, SegParam* sp, const Lists& Ls, int n_
     cudaError_t e = cudaFuncSetAttribute(k_solve, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     TraceScope ts(kKSolve, st);
-    // Long segments (where C can hold millions of values) get a cluster of
-    // kSolveCTAs CTAs each; layer-wise segments are short and take one.
-    const int ncta = (Lo.L == 1 && Lo.d >= ((int64_t)1 << 22)) ? kSolveCTAs : 1;
+    // C holds about the capped coordinates, whose count the budget kappa d
+    // bounds at the fixed point: segments with a budget above 2^20 (where C can
+    // hold millions of values) get a cluster of kSolveCTAs CTAs, others one.
+    const int ncta = (Lo.L == 1 && kappa * (double)Lo.d > (double)(1 << 20)) ? kSolveCTAs : 1;
+    if (ncta == 1)
+        return launch_dep(k_solve, dim3(n_seg), dim3(kThreads), smem, st, Lo, sp, Ls, kappa, iters, force_exact,
+                          status, info);
     return launch_dep_cluster(k_solve, dim3(n_seg * ncta), dim3(kThreads), smem, ncta, st, Lo, sp, Ls, kappa, iters,
                               force_exact, status, info);
 }
