@@ -510,3 +510,22 @@ def test_sparsify_aggregate_fused_long_runs_many_workers(gs):
         il.append(ri)
         vl.append(rv)
     compare_sum(out.cpu().numpy(), il, vl, d)
+
+
+@pytest.mark.parametrize("force_exact", [0, 1])
+def test_cluster_solve_large_budget(gs, force_exact):
+    """Budgets above 2^20 run the solve on a cluster of CTAs per segment; with
+    heavy tails at a large kappa the capped-candidate set is far too large for
+    shared memory, so every pass walks the chunks (and the forced exact
+    fallback runs on the cluster's first CTA)."""
+    import torch
+    M, d, kappa, iters = 2, (1 << 23) + 4 * 777, 0.2, 3
+    g = workloads.device_lognormal(M, d, seed0=31)
+    gs.gs_set_option(gs.GS_OPT_FORCE_EXACT_SOLVE, force_exact)
+    try:
+        flips = _full_check(gs, g, kappa, iters, seed=4, step=6)
+    finally:
+        gs.gs_set_option(gs.GS_OPT_FORCE_EXACT_SOLVE, 0)
+    assert flips <= 2
+    del g
+    torch.cuda.empty_cache()
