@@ -284,6 +284,8 @@ __device__ __forceinline__ int upper_slot(const int32_t* pre, int n, int e) {
 // k_bound: one CTA per segment.
 // ---------------------------------------------------------------------------
 constexpr double kBoundZ = 5.0;
+constexpr double kBoundZs = 8.0;         // standard errors of the spread-based margin
+constexpr double kBoundFloor = 0.04;     // smallest relative margin
 
 // Sum of two floats over the block; every thread gets both.
 __device__ __forceinline__ float2 block_sum2f(float a, float b, float2* sh) {
@@ -302,6 +304,32 @@ __device__ __forceinline__ float2 block_sum2f(float a, float b, float2* sh) {
         for (int o = 16; o > 0; o >>= 1) {
             t.x += __shfl_xor_sync(0xFFFFFFFFu, t.x, o);
             t.y += __shfl_xor_sync(0xFFFFFFFFu, t.y, o);
+        }
+        if (lane == 0) sh[32] = t;
+    }
+    __syncthreads();
+    return sh[32];
+}
+
+// Three float sums over the block at once; every thread receives them (x, y, z).
+__device__ __forceinline__ float4 block_sum3f(float a, float b, float c, float4* sh) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = (blockDim.x + 31) >> 5;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        a += __shfl_xor_sync(0xFFFFFFFFu, a, o);
+        b += __shfl_xor_sync(0xFFFFFFFFu, b, o);
+        c += __shfl_xor_sync(0xFFFFFFFFu, c, o);
+    }
+    __syncthreads();
+    if (lane == 0) sh[warp] = make_float4(a, b, c, 0.0f);
+    __syncthreads();
+    if (warp == 0) {
+        float4 t = lane < nw ? sh[lane] : make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            t.x += __shfl_xor_sync(0xFFFFFFFFu, t.x, o);
+            t.y += __shfl_xor_sync(0xFFFFFFFFu, t.y, o);
+            t.z += __shfl_xor_sync(0xFFFFFFFFu, t.z, o);
         }
         if (lane == 0) sh[32] = t;
     }
@@ -331,6 +359,7 @@ __global__ void __cluster_dims__(kBoundCTAs, 1, 1) __launch_bounds__(kBoundCtaTh
     cg::cluster_group cluster = cg::this_cluster();
     extern __shared__ float sa[];               // rank 0: all ns samples
     __shared__ float2 sh2[33];
+    __shared__ float4 sh4[33];
     const int rank = (int)cluster.block_rank();
     const int s = blockIdx.x / kBoundCTAs, tid = threadIdx.x;
     int m, l, c0, c1;
@@ -383,16 +412,18 @@ __global__ void __cluster_dims__(kBoundCTAs, 1, 1) __launch_bounds__(kBoundCtaTh
     float lam = S > 0.0f ? budget / S : 0.0f;
     float K = 0.0f, Su = S;
     bool take_all = !(S > 0.0f) || !(lam < kInf);
+    float Sq = 0.0f;   // sum of squares of the uncapped sample values (for the margin)
     for (int it = 0; it < 32 && !take_all; ++it) {
         const float acap = 1.0f / lam;
-        float su = 0.0f, kc = 0.0f;
+        float su = 0.0f, kc = 0.0f, sq = 0.0f;
         for (int k = tid; k < ns; k += kBoundCtaThreads) {
             const float x = sa[k];
-            if (x >= acap) kc += 1.0f; else su += x;
+            if (x >= acap) kc += 1.0f; else { su += x; sq += x * x; }
         }
-        const float2 r = block_sum2f(kc, su, sh2);
+        const float4 r = block_sum3f(kc, su, sq, sh4);
         K = r.x;
         Su = r.y;
+        Sq = r.z;
         if (!(Su > 0.0f)) { take_all = true; break; }
         const float c = (budget - K) / (lam * Su);
         if (!(c > 1.0f + 1e-5f)) break;
@@ -401,20 +432,39 @@ __global__ void __cluster_dims__(kBoundCTAs, 1, 1) __launch_bounds__(kBoundCtaTh
     if (tid == 0) {
         P.done = 0;
         P.w_done = 0;
-        const double e = take_all ? 0.0 : (double)lam * Su / budget;  // uncapped share of the budget
+        const float e = take_all ? 0.0f : lam * Su / budget;  // uncapped share of the budget
         if (take_all || K >= budget || !(lam > 0.0f)) {
             P.lam_up = (double)kInf;
             P.lam_up32 = kInf;
             P.t_c = 0.0f;
             P.flags = kSegTakeAll;
         } else {
-            double margin = 1.0 + kBoundZ / sqrt(kappa * (double)ns) / fmax(e, 1.0 / 16.0);
-            margin = fmin(margin, 64.0);
-            const double up = (double)lam * margin;
-            P.lam_up = up;
-            P.lam_up32 = __double2float_ru(up);
-            const double t = (1.0 / up) * (1.0 - 0x1p-20);
-            P.t_c = t > 3.4028234663852886e38 ? 3.4028234663852886e38f : __double2float_rd(t);
+            // A count-based bound on the sample's error, tightened by the sample's
+            // own spread: lambda = (kappa d - K) / S_u at the fixed point, so its
+            // relative error is about that of S_u (std of a sum of the
+            // uncapped values) and of kappa d - K (binomial K).  A sample that
+            // caught large values also has a large spread, which keeps the bound
+            // safe for heavy tails; a violated bound only costs the exact fallback.
+            // (fp32 throughout: a heuristic, and fp64 is slow on this part)
+            const float kns = (float)kappa * (float)ns;
+            float margin = 1.0f + (float)kBoundZ * rsqrtf(kns) / fmaxf(e, 1.0f / 16.0f);
+            const float nu = (float)ns - K;
+            if (nu > 1.0f && Su > 0.0f && isfinite(Sq)) {
+                const float mean = Su / nu;
+                const float var = fmaxf(Sq / nu - mean * mean, 0.0f);
+                const float rel_s = sqrtf(var * nu) / Su;
+                const float room = kns - K;
+                const float rel_k = room > 0.0f ? sqrtf(K) / room : 1.0f;
+                margin = fminf(margin, 1.0f + fmaxf((float)kBoundFloor,
+                                                    (float)kBoundZs * sqrtf(rel_s * rel_s + rel_k * rel_k)));
+            }
+            margin = fminf(margin, 64.0f);
+            // lam_up32 rounded up and t_c rounded down keep both lists supersets;
+            // the fp64 bound is lam_up32 itself.
+            const float up32 = __fmul_ru(lam, margin);
+            P.lam_up32 = up32;
+            P.lam_up = (double)up32;
+            P.t_c = __fmul_rd(__frcp_rd(up32), 1.0f - 0x1p-20f);
             P.flags = 0;
         }
     }
