@@ -56,8 +56,18 @@ def lib():
                                              ctypes.c_void_p, ctypes.c_void_p, P(ctypes.c_int64), ctypes.c_void_p]
         L.gso_aggregate.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int, ctypes.c_int64,
                                     ctypes.c_void_p]
+        L.gso_hybrid_encode.argtypes = [ctypes.c_void_p, ctypes.c_int64, ctypes.c_double, ctypes.c_void_p,
+                                        ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p,
+                                        P(ctypes.c_int64), ctypes.c_void_p, P(ctypes.c_int64), P(ctypes.c_double)]
+        L.gso_hybrid_decode.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p,
+                                        ctypes.c_int64, ctypes.c_double, ctypes.c_void_p, ctypes.c_void_p,
+                                        P(ctypes.c_int64)]
+        L.gso_ternary_bits.argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64]
+        L.gso_ternary_bits.restype = ctypes.c_double
+        L.gso_comm_bits.argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_double, ctypes.c_int]
+        L.gso_comm_bits.restype = ctypes.c_double
         for f in ("gso_greedy_lambda", "gso_greedy_pvector", "gso_probabilities", "gso_sparsify",
-                  "gso_segmented_sparsify", "gso_aggregate"):
+                  "gso_segmented_sparsify", "gso_aggregate", "gso_hybrid_encode", "gso_hybrid_decode"):
             getattr(L, f).restype = ctypes.c_int
         _LIB = L
     return _LIB
@@ -148,3 +158,46 @@ def aggregate(idx_list, val_list, d):
     out = np.empty(d, dtype=np.float32)
     _check(lib().gso_aggregate(ip, vp, nn.ctypes.data, M, d, out.ctypes.data))
     return out
+
+
+def hybrid_encode(g, lam, idx, val):
+    """Section 3.3, eqs. (9)-(10): split the plain coding (idx, val) of Q(g)
+    into Q_A (capped: index, value) and Q_B (codes 2 * index + [g_i < 0]);
+    returns (qa_idx, qa_val, qb_code, 1 / lambda)."""
+    g, gp = _f32(g)
+    idx = np.ascontiguousarray(idx, dtype=np.int32)
+    val = np.ascontiguousarray(val, dtype=np.float32)
+    n = idx.size
+    qa_i = np.empty(max(n, 1), np.int32)
+    qa_v = np.empty(max(n, 1), np.float32)
+    qb = np.empty(max(n, 1), np.uint32)
+    na, nb, inv = ctypes.c_int64(), ctypes.c_int64(), ctypes.c_double()
+    _check(lib().gso_hybrid_encode(gp, g.size, float(lam), idx.ctypes.data, val.ctypes.data, n,
+                                   qa_i.ctypes.data, qa_v.ctypes.data, ctypes.byref(na), qb.ctypes.data,
+                                   ctypes.byref(nb), ctypes.byref(inv)))
+    return qa_i[:na.value].copy(), qa_v[:na.value].copy(), qb[:nb.value].copy(), inv.value
+
+
+def hybrid_decode(qa_idx, qa_val, qb_code, inv_lambda):
+    """Merge Q_A and Q_B back into the ascending (idx, val) lists."""
+    qa_idx = np.ascontiguousarray(qa_idx, dtype=np.int32)
+    qa_val = np.ascontiguousarray(qa_val, dtype=np.float32)
+    qb_code = np.ascontiguousarray(qb_code, dtype=np.uint32)
+    n = qa_idx.size + qb_code.size
+    idx = np.empty(max(n, 1), np.int32)
+    val = np.empty(max(n, 1), np.float32)
+    nn = ctypes.c_int64()
+    _check(lib().gso_hybrid_decode(qa_idx.ctypes.data, qa_val.ctypes.data, qa_idx.size, qb_code.ctypes.data,
+                                   qb_code.size, float(inv_lambda), idx.ctypes.data, val.ctypes.data,
+                                   ctypes.byref(nn)))
+    return idx[:nn.value].copy(), val[:nn.value].copy()
+
+
+def ternary_bits(d, n_neg, n_pos, n_cap):
+    """Entropy-coding length of the dense code in {0, -1, +1, 2}^d (section 3.3)."""
+    return lib().gso_ternary_bits(int(d), int(n_neg), int(n_pos), int(n_cap))
+
+
+def comm_bits(d, n_capped, sum_p_uncapped, b=32):
+    """One worker's summand of H(T, M) for one step (section 5)."""
+    return lib().gso_comm_bits(int(d), int(n_capped), float(sum_p_uncapped), int(b))

@@ -331,3 +331,100 @@ GSO_EXPORT int gso_aggregate(const int32_t* const* idx, const float* const* val,
     free(dense);
     return GSO_OK;
 }
+
+/* ------------------------------------------------------------------------
+ * Section 3.3, eqs. (9)-(10): the hybrid coding of Q(g).  The kept
+ * coordinates with p_i = 1 (the capped set S_k) go to Q_A as (index,
+ * g_i / p_i = g_i); every other kept coordinate has p_i = lambda |g_i|, so its
+ * value g_i / p_i is sign(g_i) / lambda and Q_B needs only its index and sign,
+ * plus the one shared scalar 1 / lambda.
+ *
+ * Input is the plain coding (idx, val, nnz) that gso_sparsify made from g
+ * with this lambda.  A Q_B entry is written as the code 2 * index + s with
+ * s = 1 for a negative g_i.  Both lists keep ascending index order.
+ * ---------------------------------------------------------------------- */
+GSO_EXPORT int gso_hybrid_encode(const float* g, int64_t d, double lambda, const int32_t* idx, const float* val,
+                                 int64_t nnz, int32_t* qa_idx, float* qa_val, int64_t* na, uint32_t* qb_code,
+                                 int64_t* nb, double* inv_lambda)
+{
+    int64_t e, a = 0, b = 0;
+    *na = 0;
+    *nb = 0;
+    if (d < 1 || nnz < 0 || nnz > d || !(lambda > 0.0)) return GSO_INVALID;
+    for (e = 0; e < nnz; e++) {
+        int64_t i = idx[e];
+        double gi, x;
+        if (i < 0 || i >= d) return GSO_INVALID;
+        gi = (double)g[i];
+        x = lambda * fabs(gi);
+        if (x >= 1.0) {                 /* p_i = min(x, 1) = 1: i is in S_k */
+            qa_idx[a] = (int32_t)i;
+            qa_val[a] = val[e];
+            a++;
+        } else {
+            qb_code[b] = (uint32_t)i * 2u + (gi < 0.0 ? 1u : 0u);
+            b++;
+        }
+    }
+    *na = a;
+    *nb = b;
+    *inv_lambda = 1.0 / lambda;
+    return GSO_OK;
+}
+
+/* The inverse: merge Q_A and Q_B back into one ascending list of (index,
+ * value), a Q_B entry taking the value +-fl32(1 / lambda). */
+GSO_EXPORT int gso_hybrid_decode(const int32_t* qa_idx, const float* qa_val, int64_t na, const uint32_t* qb_code,
+                                 int64_t nb, double inv_lambda, int32_t* idx, float* val, int64_t* nnz)
+{
+    int64_t a = 0, b = 0, n = 0;
+    const float mag = (float)inv_lambda;
+    while (a < na || b < nb) {
+        int64_t ib = b < nb ? (int64_t)(qb_code[b] >> 1) : -1;
+        if (b >= nb || (a < na && (int64_t)qa_idx[a] < ib)) {
+            idx[n] = qa_idx[a];
+            val[n] = qa_val[a];
+            a++;
+        } else {
+            if (a < na && (int64_t)qa_idx[a] == ib) return GSO_INVALID; /* one index in both lists */
+            idx[n] = (int32_t)ib;
+            val[n] = (qb_code[b] & 1u) ? -mag : mag;
+            b++;
+        }
+        n++;
+    }
+    *nnz = n;
+    return GSO_OK;
+}
+
+/* Section 3.3 (last paragraph): the dense code q in {0, -1, +1, 2}^d (0: not
+ * kept, -1/+1: the sign of a kept coordinate outside S_k, 2: a coordinate in
+ * S_k) under standard entropy coding takes sum_l d_l log2(d / d_l) bits over
+ * the symbols l with d_l > 0 -- at most 2d. */
+GSO_EXPORT double gso_ternary_bits(int64_t d, int64_t n_neg, int64_t n_pos, int64_t n_cap)
+{
+    int64_t counts[4];
+    double bits = 0.0;
+    int l;
+    counts[0] = d - n_neg - n_pos - n_cap;
+    counts[1] = n_neg;
+    counts[2] = n_pos;
+    counts[3] = n_cap;
+    for (l = 0; l < 4; l++) {
+        if (counts[l] < 0) return -1.0;
+        if (counts[l] > 0) bits += (double)counts[l] * log2((double)d / (double)counts[l]);
+    }
+    return bits;
+}
+
+/* Section 5: one worker's share of one step of the communication cost
+ * H(T, M) of gradient sparsification:
+ *   #{i : p_i = 1} (b + log2 d) + min(2d, log2 d * sum_{i : p_i < 1} p_i) + b
+ * for b-bit floating point numbers. */
+GSO_EXPORT double gso_comm_bits(int64_t d, int64_t n_capped, double sum_p_uncapped, int b)
+{
+    const double ld = log2((double)d);
+    double q = ld * sum_p_uncapped;
+    if (q > 2.0 * (double)d) q = 2.0 * (double)d;
+    return (double)n_capped * ((double)b + ld) + q + (double)b;
+}
