@@ -316,6 +316,7 @@ def run_gpu(args):
         rc = gs.gs_sync_status(stream)
         if rc != gs.GS_OK:
             raise RuntimeError(f"device status after the sparsify-only run: {gs.status_string(rc)}")
+    hybrid = run_hybrid(gs, g, kappa, w, args, dev, stream, n_bd, hbm) if off is None else None
 
     # ---- end to end through the host-buffer entry point
     e2e = None
@@ -335,6 +336,7 @@ def run_gpu(args):
                               "peak": hbm, "frac": round(pipe_gbs / hbm, 4), "unit": "GB/s"},
         "roofline": roofline,
         "sparsify_roofline": sp_only,
+        "hybrid_code": hybrid,
         "kernels": kernels, "kernels_steps": n_bd,
         "nnz_per_step": nnz_total,
         "gpu_launches": launches,
@@ -389,6 +391,67 @@ def source_digest(kernel):
         with open(os.path.join(src, fn), "rb") as f:
             h.update(f.read())
     return h.hexdigest()
+
+
+def run_hybrid(gs, g, kappa, w, args, dev, stream, n_steps, hbm):
+    """The hybrid code of section 3.3 (gs_batched_sparsify_hybrid) on the same
+    inputs: its time and bytes, and the coding lengths of one step -- plain
+    (index, value) pairs, this format (Q_A 64 bits, Q_B 32 bits, 32 bits of
+    1/lambda per worker), the paper's hybrid (b + log2 d and log2 d + 1 bits),
+    the entropy-coded dense {0, -1, +1, 2} code, and the section 5 summand of
+    H(T, M) (b = 32)."""
+    import math
+    import numpy as np
+    import torch
+    M, d = g.shape
+    qa_i = torch.empty((M, d), dtype=torch.int32, device=dev)
+    qa_v = torch.empty((M, d), dtype=torch.float32, device=dev)
+    qb = torch.empty((M, d), dtype=torch.int32, device=dev)
+    na = torch.empty(M, dtype=torch.int32, device=dev)
+    nb = torch.empty(M, dtype=torch.int32, device=dev)
+    il = torch.empty(M, dtype=torch.float32, device=dev)
+    info = torch.zeros(M * gs.INFO_BYTES, dtype=torch.uint8, device=dev)
+    for t in range(3):
+        gs.gs_batched_sparsify_hybrid(g, kappa, w.iters, w.seed, t, 0, qa_i, qa_v, qb, na, nb, il, info=info,
+                                      stream=stream)
+    torch.cuda.synchronize()
+    h0, h1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    h0.record(stream)
+    for t in range(n_steps):
+        gs.gs_batched_sparsify_hybrid(g, kappa, w.iters, w.seed, args.warmup + t, 0, qa_i, qa_v, qb, na, nb, il,
+                                      stream=stream)
+    h1.record(stream)
+    torch.cuda.synchronize()
+    ms = max_over_ranks(h0.elapsed_time(h1) / n_steps, dev)
+    # coding lengths of one step (step 0's outputs)
+    gs.gs_batched_sparsify_hybrid(g, kappa, w.iters, w.seed, 0, 0, qa_i, qa_v, qb, na, nb, il, info=info,
+                                  stream=stream)
+    torch.cuda.synchronize()
+    rc = gs.gs_sync_status(stream)
+    if rc != gs.GS_OK:
+        raise RuntimeError(f"device status after the hybrid-code run: {gs.status_string(rc)}")
+    rec = gs.decode_info(info)
+    a, b_ = na.cpu().numpy().astype(np.int64), nb.cpu().numpy().astype(np.int64)
+    ld = math.log2(d)
+    bits = {"plain": 0.0, "this_format": 0.0, "paper_hybrid": 0.0, "dense_entropy": 0.0, "H_summand": 0.0}
+    for m in range(M):
+        codes = qb[m, :int(b_[m])].cpu().numpy().view(np.uint32)
+        n_neg = int((codes & 1).sum())
+        bits["plain"] += 64.0 * (a[m] + b_[m])
+        bits["this_format"] += 64.0 * a[m] + 32.0 * b_[m] + 32.0
+        bits["paper_hybrid"] += a[m] * (32 + math.ceil(ld)) + b_[m] * (math.ceil(ld) + 1) + 32
+        counts = [d - a[m] - b_[m], n_neg, b_[m] - n_neg, a[m]]
+        bits["dense_entropy"] += sum(c * math.log2(d / c) for c in counts if c > 0)
+        sum_p_uncapped = rec[m]["sum_p"] - rec[m]["capped"]
+        bits["H_summand"] += rec[m]["capped"] * (32 + ld) + min(2 * d, ld * sum_p_uncapped) + 32
+    esz = g.element_size()
+    algo = M * d * esz + 8 * int(a.sum()) + 4 * int(b_.sum()) + 4 * M
+    gbs = algo / (ms / 1e3) / 1e9
+    return {"api": "gs_batched_sparsify_hybrid", "steps": n_steps, "ms_per_step": round(ms, 4),
+            "algorithmic_bytes": algo, "achieved": round(gbs, 1), "peak": hbm, "frac": round(gbs / hbm, 4),
+            "unit": "GB/s", "n_a": int(a.sum()), "n_b": int(b_.sum()),
+            "bits_per_step": {k: round(v) for k, v in bits.items()},
+            "bits_per_coordinate": {k: round(v / (M * d), 4) for k, v in bits.items()}}
 
 
 def load_traffic(kernel, workload, dtype, kappa):

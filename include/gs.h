@@ -127,6 +127,28 @@ gs_status gs_batched_sparsify(const void* g, int dtype, int M, int64_t d, double
                               gs_info* info, void* stream);
 
 /*
+ * gs_batched_sparsify with the hybrid code of section 3.3 (eqs. 9-10) in
+ * place of the plain (index, value) lists: the kept coordinates with p_i = 1
+ * (the capped set S_k) go to Q_A as (index, value g_i); every other kept
+ * coordinate has value sign(g_i) / lambda, so Q_B holds only its code
+ * 2 * index + (g_i < 0), and one fp32 1/lambda per worker gives the
+ * magnitude.  Both lists are in ascending index order; merged (a Q_B entry
+ * becoming +-inv_lam) they are exactly gs_batched_sparsify's idx / val.
+ *   qa_idx, qa_val  device, M x cap: row m holds worker m's Q_A
+ *   qb_code         device, M x cap uint32: row m holds worker m's Q_B
+ *   n_a, n_b        device, M int32: the lengths (a length above cap writes
+ *                   only cap entries and records GS_ERR_CAPACITY)
+ *   inv_lam         device, M fp32: fl32(1 / lambda) of each worker
+ *   cap             row capacity, >= 1 (cap = d can never overflow)
+ * Other arguments as in gs_batched_sparsify.  Q_A needs 8 bytes per entry,
+ * Q_B 4 (the index limit d < 2^31 leaves room for the sign bit).
+ */
+gs_status gs_batched_sparsify_hybrid(const void* g, int dtype, int M, int64_t d, double kappa, int iters,
+                                     uint64_t seed, uint32_t step, uint32_t worker0, int32_t* qa_idx, float* qa_val,
+                                     uint32_t* qb_code, int32_t* n_a, int32_t* n_b, float* inv_lam, int64_t cap,
+                                     gs_info* info, void* stream);
+
+/*
  * Layer-wise sparsification (section 5.2: each layer is sparsified on its
  * own).  Each worker's vector is cut into L segments by the HOST array
  * seg_offsets[0..L] (0 = seg_offsets[0] < ... < seg_offsets[L] = d); every

@@ -23,7 +23,7 @@ GS_OPT_FORCE_EXACT_SOLVE, GS_OPT_SAMPLE_SIZE, GS_OPT_KERNEL_TIMING, GS_OPT_STREA
 
 # Symbols include/gs.h declares (checked by the tests).
 EXPORTS = ("gs_status_string", "gs_last_error", "gs_version", "gs_sync_status", "gs_probabilities", "gs_probabilities_ex",
-           "gs_sparsify", "gs_batched_sparsify", "gs_segmented_sparsify", "gs_sparse_aggregate",
+           "gs_sparsify", "gs_batched_sparsify", "gs_batched_sparsify_hybrid", "gs_segmented_sparsify", "gs_sparse_aggregate",
            "gs_sparsify_aggregate", "gs_sparsify_noalloc", "gs_pipeline_host", "gs_random_words", "gs_set_option", "gs_kernel_count", "gs_kernel_name",
            "gs_kernel_times")
 
@@ -62,6 +62,8 @@ def lib():
             "gs_probabilities_ex": ([vp, i64, dbl, i32, vp, vp, vp], i32),
             "gs_sparsify": ([vp, i64, dbl, i32, u64, u32, u32, vp, vp, vp, vp], i32),
             "gs_batched_sparsify": ([vp, i32, i32, i64, dbl, i32, u64, u32, u32, vp, vp, vp, i64, vp, vp], i32),
+            "gs_batched_sparsify_hybrid": ([vp, i32, i32, i64, dbl, i32, u64, u32, u32, vp, vp, vp, vp, vp, vp, i64,
+                                            vp, vp], i32),
             "gs_segmented_sparsify": ([vp, i32, i32, i64, vp, i32, dbl, i32, u64, u32, u32, vp, vp, vp, i64, vp, vp],
                                       i32),
             "gs_sparse_aggregate": ([vp, vp, vp, i32, i64, vp, vp], i32),
@@ -229,6 +231,26 @@ def gs_batched_sparsify(g, kappa, iters, seed, step, worker0, idx, val, nnz, inf
                                      int(step), int(worker0), _ptr(idx, "idx", (torch.int32,)),
                                      _ptr(val, "val", (torch.float32,)), _ptr(nnz, "nnz", (torch.int32,)), cap,
                                      _ptr(info, "info"), _stream(stream)), "gs_batched_sparsify")
+
+
+def gs_batched_sparsify_hybrid(g, kappa, iters, seed, step, worker0, qa_idx, qa_val, qb_code, n_a, n_b, inv_lam,
+                               info=None, stream=None):
+    """g: (M, d) fp32/bf16; qa_idx/qa_val/qb_code: (M, cap) int32/fp32/uint32
+    (or int32 viewed as codes); n_a/n_b: (M,) int32; inv_lam: (M,) fp32."""
+    import torch
+    M, d = g.shape
+    cap = qa_idx.shape[1]
+    if tuple(qa_val.shape) != tuple(qa_idx.shape) or tuple(qb_code.shape) != tuple(qa_idx.shape):
+        raise ValueError("qa_idx, qa_val and qb_code must be (M, cap)")
+    if qa_idx.shape[0] != M or n_a.numel() != M or n_b.numel() != M or inv_lam.numel() != M:
+        raise ValueError("one row / count / 1-over-lambda per worker")
+    codes = (torch.int32, torch.uint32) if hasattr(torch, "uint32") else (torch.int32,)
+    _check(lib().gs_batched_sparsify_hybrid(_ptr(g, "g"), _g_dtype(g), M, d, float(kappa), int(iters), int(seed),
+                                            int(step), int(worker0), _ptr(qa_idx, "qa_idx", (torch.int32,)),
+                                            _ptr(qa_val, "qa_val", (torch.float32,)), _ptr(qb_code, "qb_code", codes),
+                                            _ptr(n_a, "n_a", (torch.int32,)), _ptr(n_b, "n_b", (torch.int32,)),
+                                            _ptr(inv_lam, "inv_lam", (torch.float32,)), cap, _ptr(info, "info"),
+                                            _stream(stream)), "gs_batched_sparsify_hybrid")
 
 
 def gs_segmented_sparsify(g, seg_offsets, kappa, iters, seed, step, worker0, idx, val, nnz, info=None, stream=None):

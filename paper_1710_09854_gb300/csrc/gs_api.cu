@@ -125,9 +125,11 @@ bool bad_kappa(double kappa) { return !(kappa > 0.0) || kappa > 1.0 || !std::isf
 struct Workspace {
     SegParam* sp;
     Lists ls;
+    int32_t* nnz;       // hybrid calls: the per-worker kept counts (plain calls write the caller's)
 };
 
-void carve(Arena& a, Workspace& w, int n_seg, int n_chunks, int64_t n, bool build_p) {
+void carve(Arena& a, Workspace& w, int n_seg, int n_chunks, int64_t n, bool build_p, bool hybrid = false,
+           int M = 0) {
     std::memset(&w, 0, sizeof(w));
     w.sp = a.take<SegParam>(n_seg);
     w.ls.c_val = a.take<float>(n);
@@ -140,19 +142,28 @@ void carve(Arena& a, Workspace& w, int n_seg, int n_chunks, int64_t n, bool buil
         w.ls.k_off = a.take<int32_t>(n_chunks);
         w.ls.e_bits = a.take<uint32_t>((size_t)n_chunks * (kChunk / 32));
         w.ls.k_sub = a.take<int32_t>((size_t)n_chunks * kSubStride);
+        if (hybrid) {
+            w.ls.k_offa = a.take<int32_t>(n_chunks);
+            w.nnz = a.take<int32_t>(M);
+        }
     }
 }
 
 // Shared driver of every sparsify / probabilities call.
 gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off, int L, double kappa, int iters,
               uint64_t seed, uint32_t step, uint32_t worker0, int32_t* idx, float* val, int32_t* nnz, int64_t cap,
-              gs_info* info, float* p, cudaStream_t st, float* agg_out = nullptr) {
+              gs_info* info, float* p, cudaStream_t st, float* agg_out = nullptr, const HybridOut* hy = nullptr) {
     const bool prob = p != nullptr;
     if (!g || M < 1 || d < 1 || d >= kMaxD || bad_kappa(kappa) || iters < 0) return GS_ERR_INVALID_ARG;
     if (dtype != GS_DTYPE_F32 && dtype != GS_DTYPE_BF16) return GS_ERR_INVALID_ARG;
     const size_t esz = dtype == GS_DTYPE_F32 ? 4 : 2;
     if ((reinterpret_cast<uintptr_t>(g) % esz) != 0) return GS_ERR_INVALID_ARG;
-    if (!prob && (!idx || !val || !nnz || cap < 1)) return GS_ERR_INVALID_ARG;
+    if (hy) {
+        if (!hy->qa_idx || !hy->qa_val || !hy->qb_code || !hy->n_a || !hy->n_b || !hy->inv_lam || cap < 1 || L != 1)
+            return GS_ERR_INVALID_ARG;
+    } else if (!prob && (!idx || !val || !nnz || cap < 1)) {
+        return GS_ERR_INVALID_ARG;
+    }
     if ((int64_t)M > ((int64_t)1 << 40) / d) return GS_ERR_INVALID_ARG;
     if (L < 1) return GS_ERR_INVALID_ARG;
     if (L > 1) {
@@ -197,7 +208,7 @@ gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off
 
     Arena a;
     Workspace w;
-    carve(a, w, n_seg, n_chunks, (int64_t)M * d, !prob);
+    carve(a, w, n_seg, n_chunks, (int64_t)M * d, !prob, hy != nullptr, M);
     void* mem = nullptr;
     {
         const cudaError_t ea = cudaMallocFromPoolAsync(&mem, a.off, s->pool, st);
@@ -205,7 +216,7 @@ gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off
     }
     a.base = static_cast<char*>(mem);
     a.off = 0;
-    carve(a, w, n_seg, n_chunks, (int64_t)M * d, !prob);
+    carve(a, w, n_seg, n_chunks, (int64_t)M * d, !prob, hy != nullptr, M);
 
     int force, ns, path;
     {
@@ -226,7 +237,8 @@ gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off
     if (e == cudaSuccess) e = launch_solve(Lo, w.sp, w.ls, n_seg, kappa, iters, force, s->status, info, st);
     if (e == cudaSuccess) {
         if (prob) e = launch_prob(Lo, w.sp, p, st);
-        else e = launch_compact(Lo, w.sp, w.ls, n_chunks, idx, val, nnz, cap, s->status, st, agg_out);
+        else e = launch_compact(Lo, w.sp, w.ls, n_chunks, idx, val, hy ? w.nnz : nnz, cap, s->status, st, agg_out,
+                                hy);
     }
     cudaError_t ef = cudaFreeAsync(mem, st);
     if (e != cudaSuccess) return cuda_fail(launch_error_site(), e);
@@ -479,6 +491,21 @@ gs_status gs_sparsify_aggregate(const void* g, int dtype, int M, int64_t d, doub
     if (!out || M < 1 || M > kMaxAggM) return GS_ERR_INVALID_ARG;
     return run(g, dtype, M, d, nullptr, 1, kappa, iters, seed, step, worker0, idx, val, nnz, cap, info, nullptr,
                static_cast<cudaStream_t>(stream), out);
+}
+
+gs_status gs_batched_sparsify_hybrid(const void* g, int dtype, int M, int64_t d, double kappa, int iters,
+                                     uint64_t seed, uint32_t step, uint32_t worker0, int32_t* qa_idx, float* qa_val,
+                                     uint32_t* qb_code, int32_t* n_a, int32_t* n_b, float* inv_lam, int64_t cap,
+                                     gs_info* info, void* stream) {
+    HybridOut h;
+    h.qa_idx = qa_idx;
+    h.qa_val = qa_val;
+    h.qb_code = qb_code;
+    h.n_a = n_a;
+    h.n_b = n_b;
+    h.inv_lam = inv_lam;
+    return run(g, dtype, M, d, nullptr, 1, kappa, iters, seed, step, worker0, nullptr, nullptr, nullptr, cap, info,
+               nullptr, static_cast<cudaStream_t>(stream), nullptr, &h);
 }
 
 gs_status gs_sparsify_noalloc(const float* g, int64_t d, double kappa, int iters, uint64_t seed, uint32_t step,

@@ -83,6 +83,7 @@ struct Lists {
                         // of its first kept entry in its worker's output
     uint32_t* e_bits;   // [n_chunks][kChunk / 32] decision bit of every keep candidate
     int32_t* k_sub;     // [n_chunks][kSubStride] kept entries of the chunk before each 1024-coordinate slice
+    int32_t* k_offa;    // [n_chunks] hybrid code only (else NULL): kept entries with p = 1, then their offsets
     int32_t* c_pre;     // [n_chunks + n_seg] prefix scratch for segments with many chunks
 };
 

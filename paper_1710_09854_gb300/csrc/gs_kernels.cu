@@ -893,6 +893,37 @@ constexpr int kSlice = 1 << kSliceLog;
 constexpr int kSlices = kChunk / kSlice;                 // 16 slices per chunk
 constexpr int kScanPer = 8;                              // chunk counts per lane per step of the worker scan
 
+// One warp turns n counts into their exclusive prefix in place (kScanPer
+// counts per lane per step, read past L1) and returns the total.
+__device__ __forceinline__ long long warp_scan_counts(int32_t* ko, int n, int lane) {
+    long long carry = 0;
+    for (int base = 0; base < n; base += 32 * kScanPer) {
+        int v[kScanPer];
+        int tot = 0;
+#pragma unroll
+        for (int j = 0; j < kScanPer; ++j) {
+            const int i = base + lane * kScanPer + j;
+            v[j] = i < n ? __ldcg(ko + i) : 0;
+            tot += v[j];
+        }
+        int inc = tot;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int u = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+            if (lane >= o) inc += u;
+        }
+        long long run = carry + (inc - tot);
+#pragma unroll
+        for (int j = 0; j < kScanPer; ++j) {
+            const int i = base + lane * kScanPer + j;
+            if (i < n) ko[i] = (int32_t)run;
+            run += v[j];
+        }
+        carry += __shfl_sync(0xFFFFFFFFu, inc, 31);
+    }
+    return carry;
+}
+
 __device__ __forceinline__ Decider chunk_decider(const SegParam& P) {
     Decider dd;
     dd.lam = P.lam;
@@ -904,7 +935,8 @@ __device__ __forceinline__ Decider chunk_decider(const SegParam& P) {
 
 __global__ void __launch_bounds__(kEmitWarps * 32) k_decide(const __grid_constant__ Layout Lo, SegParam* sp,
                                                             const __grid_constant__ Lists Ls, int n_chunks,
-                                                            int32_t* nnz, int64_t cap, int* status) {
+                                                            int32_t* nnz, int32_t* n_a, int32_t* n_b, int64_t cap,
+                                                            int* status) {
     grid_dep_wait();
     const int lane = threadIdx.x & 31;
     const int c = blockIdx.x * kEmitWarps + (threadIdx.x >> 5);
@@ -918,6 +950,7 @@ __global__ void __launch_bounds__(kEmitWarps * 32) k_decide(const __grid_constan
     int32_t* ks = Ls.k_sub + (size_t)c * kSubStride;
     const int lo32 = (int)ch.lo;
     int cnt = 0, last_sub = 0;   // kept so far; slice of the last candidate seen
+    int cnt_a = 0;               // kept with p = 1 (the hybrid code's Q_A)
     for (int base = 0; base < n; base += 32 * kEmitBatch) {
         int2 e[kEmitBatch];
 #pragma unroll
@@ -928,11 +961,12 @@ __global__ void __launch_bounds__(kEmitWarps * 32) k_decide(const __grid_constan
 #pragma unroll
         for (int r = 0; r < kEmitBatch; ++r) {
             const int i = base + r * 32 + lane;
-            bool keep = false;
+            bool keep = false, capped = false;
             if (i < n) {
                 const float gv = __int_as_float(e[r].y);
                 if (fabsf(gv) >= dd.a_cap) {
                     keep = true;   // capped: p = 1, kept whatever the draw
+                    capped = true;
                 } else {
                     const uint32_t x = word_of(ph.words((uint32_t)e[r].x >> 2), e[r].x & 3);
                     float v;
@@ -952,6 +986,7 @@ __global__ void __launch_bounds__(kEmitWarps * 32) k_decide(const __grid_constan
                 last_sub = __shfl_sync(0xFFFFFFFFu, sub, 31);
             }
             cnt += __popc(bal);
+            cnt_a += __popc(__ballot_sync(0xFFFFFFFFu, capped));
         }
     }
     // Slices after the last candidate (all of them if there is none).
@@ -960,6 +995,7 @@ __global__ void __launch_bounds__(kEmitWarps * 32) k_decide(const __grid_constan
     if (lane == 0) {
         ks[0] = 0;
         Ls.k_off[c] = cnt;
+        if (Ls.k_offa) Ls.k_offa[c] = cnt_a;
     }
 
     // The last warp to finish one of the worker's chunks turns the worker's
@@ -969,35 +1005,19 @@ __global__ void __launch_bounds__(kEmitWarps * 32) k_decide(const __grid_constan
     if (lane == 0) last = atomicAdd(&sp[ch.m * Lo.L].w_done, 1) == Lo.cpw - 1;
     if (!__shfl_sync(0xFFFFFFFFu, last, 0)) return;
     __threadfence();
-    int32_t* ko = Ls.k_off + (size_t)ch.m * Lo.cpw;
-    long long carry = 0;
-    for (int base = 0; base < Lo.cpw; base += 32 * kScanPer) {
-        int v[kScanPer];
-        int tot = 0;
-#pragma unroll
-        for (int j = 0; j < kScanPer; ++j) {
-            const int i = base + lane * kScanPer + j;
-            v[j] = i < Lo.cpw ? __ldcg(ko + i) : 0;
-            tot += v[j];
+    const long long total = warp_scan_counts(Ls.k_off + (size_t)ch.m * Lo.cpw, Lo.cpw, lane);
+    if (Ls.k_offa) {
+        // The hybrid code: Q_A offsets from the capped counts, Q_B's are the rest.
+        const long long ta = warp_scan_counts(Ls.k_offa + (size_t)ch.m * Lo.cpw, Lo.cpw, lane);
+        if (lane == 0) {
+            n_a[ch.m] = (int32_t)ta;
+            n_b[ch.m] = (int32_t)(total - ta);
+            if (ta > cap || total - ta > cap) atomicOr(status, kStCapacity);
         }
-        int inc = tot;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int u = __shfl_up_sync(0xFFFFFFFFu, inc, o);
-            if (lane >= o) inc += u;
-        }
-        long long run = carry + (inc - tot);
-#pragma unroll
-        for (int j = 0; j < kScanPer; ++j) {
-            const int i = base + lane * kScanPer + j;
-            if (i < Lo.cpw) ko[i] = (int32_t)run;
-            run += v[j];
-        }
-        carry += __shfl_sync(0xFFFFFFFFu, inc, 31);
     }
     if (lane == 0) {
-        nnz[ch.m] = (int32_t)carry;
-        if (carry > cap) atomicOr(status, kStCapacity);
+        nnz[ch.m] = (int32_t)total;
+        if (!Ls.k_offa && total > cap) atomicOr(status, kStCapacity);
     }
 }
 
@@ -1039,6 +1059,60 @@ __global__ void __launch_bounds__(kEmitWarps * 32) k_emit(const __grid_constant_
                 }
             }
             pos0 += __popc(wd[r]);
+        }
+    }
+}
+
+// The hybrid code of section 3.3 (eqs. 9-10) straight from the decisions: a
+// kept candidate with p = 1 goes to Q_A as (index, g_i); any other kept
+// candidate goes to Q_B as 2 * index + sign bit.  Offsets of both lists come
+// from k_decide's two scans; chunk 0's warp writes the worker's 1 / lambda.
+__global__ void __launch_bounds__(kEmitWarps * 32) k_emit_hybrid(const __grid_constant__ Layout Lo,
+                                                                 const SegParam* __restrict__ sp,
+                                                                 const __grid_constant__ Lists Ls, int n_chunks,
+                                                                 const __grid_constant__ HybridOut H, int64_t cap) {
+    grid_dep_wait();
+    const int lane = threadIdx.x & 31;
+    const int c = blockIdx.x * kEmitWarps + (threadIdx.x >> 5);
+    if (c >= n_chunks) return;
+    const Chunk ch = decode_chunk(Lo, c);
+    const SegParam& P = sp[ch.seg];
+    const float a_cap = P.a_cap;
+    if (c == ch.m * Lo.cpw && lane == 0) H.inv_lam[ch.m] = P.inv_lam32;
+    const int n = Ls.p_cnt[c];
+    const int2* ent = Ls.p_ent + (int64_t)ch.m * Lo.d + ch.lo;
+    const uint32_t* wb = Ls.e_bits + (size_t)c * kBitWords;
+    const int64_t out0 = (int64_t)ch.m * cap;
+    long long pa = Ls.k_offa[c], pb = (long long)Ls.k_off[c] - Ls.k_offa[c];
+    const uint32_t below = (1u << lane) - 1u;
+    for (int base = 0; base < n; base += 32 * kEmitBatch) {
+        uint32_t wd[kEmitBatch];
+        int2 en[kEmitBatch];
+#pragma unroll
+        for (int r = 0; r < kEmitBatch; ++r) {
+            const int i = base + r * 32 + lane;
+            wd[r] = base + r * 32 < n ? wb[(base >> 5) + r] : 0u;
+            en[r] = i < n ? ent[i] : make_int2(0, 0);
+        }
+#pragma unroll
+        for (int r = 0; r < kEmitBatch; ++r) {
+            const bool kept = (wd[r] >> lane) & 1u;
+            const float gv = __int_as_float(en[r].y);
+            const bool in_a = kept && fabsf(gv) >= a_cap;
+            const uint32_t ba = __ballot_sync(0xFFFFFFFFu, in_a);
+            const uint32_t bb = wd[r] & ~ba;
+            if (in_a) {
+                const long long q = pa + __popc(ba & below);
+                if (q < cap) {
+                    H.qa_idx[out0 + q] = en[r].x;
+                    H.qa_val[out0 + q] = gv;
+                }
+            } else if (kept) {
+                const long long q = pb + __popc(bb & below);
+                if (q < cap) H.qb_code[out0 + q] = (uint32_t)en[r].x * 2u + (gv < 0.0f ? 1u : 0u);
+            }
+            pa += __popc(ba);
+            pb += __popc(bb);
         }
     }
 }
@@ -1355,16 +1429,23 @@ cudaError_t launch_solve(const Layout& Lo, SegParam* sp, const Lists& Ls, int n_
 }
 
 cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, int32_t* idx,
-                           float* val, int32_t* nnz, int64_t cap, int* status, cudaStream_t st, float* sum_out) {
+                           float* val, int32_t* nnz, int64_t cap, int* status, cudaStream_t st, float* sum_out,
+                           const HybridOut* hybrid) {
     const int blocks = (n_chunks + kEmitWarps - 1) / kEmitWarps;
     cudaError_t e;
     {
         set_launch_error_site("k_decide launch");
         TraceScope ts(kKDecide, st);
         e = launch_dep(k_decide, dim3(blocks), dim3(kEmitWarps * 32), 0, st, Lo, const_cast<SegParam*>(sp), Ls,
-                       n_chunks, nnz, cap, status);
+                       n_chunks, nnz, hybrid ? hybrid->n_a : nullptr, hybrid ? hybrid->n_b : nullptr, cap, status);
     }
     if (e != cudaSuccess) return e;
+    if (hybrid) {
+        set_launch_error_site("k_emit_hybrid launch");
+        TraceScope ts(kKEmit, st);
+        return launch_dep(k_emit_hybrid, dim3(blocks), dim3(kEmitWarps * 32), 0, st, Lo, sp, Ls, n_chunks, *hybrid,
+                          cap);
+    }
     {
         set_launch_error_site("k_emit launch");
         TraceScope ts(kKEmit, st);

@@ -73,11 +73,23 @@ cudaError_t launch_stream(const Layout& Lo, const SegParam* sp, const Lists& Ls,
                           cudaStream_t st);
 cudaError_t launch_solve(const Layout& Lo, SegParam* sp, const Lists& Ls, int n_seg, double kappa, int iters,
                          int force_exact, int* status, gs_info_dev* info, cudaStream_t st);
+// Outputs of the hybrid coding (section 3.3): per worker m, rows of `cap`
+// entries at m * cap.
+struct HybridOut {
+    int32_t* qa_idx;    // Q_A: indices of the kept coordinates with p = 1
+    float* qa_val;      // Q_A: their values g_i
+    uint32_t* qb_code;  // Q_B: 2 * index + (g_i < 0) of the other kept coordinates
+    int32_t* n_a;       // [M] Q_A lengths
+    int32_t* n_b;       // [M] Q_B lengths
+    float* inv_lam;     // [M] fl32(1 / lambda), the magnitude of every Q_B value
+};
+
 // Decide, scan and compact; with sum_out (L == 1 only) also the sparse sum of
-// the M compacted rows into sum_out (d fp32), fused with the compaction.
+// the M compacted rows into sum_out (d fp32), fused with the compaction; with
+// hybrid (L == 1 only) the hybrid code instead of the plain lists.
 cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, int32_t* idx,
                            float* val, int32_t* nnz, int64_t cap, int* status, cudaStream_t st,
-                           float* sum_out = nullptr);
+                           float* sum_out = nullptr, const HybridOut* hybrid = nullptr);
 cudaError_t launch_prob(const Layout& Lo, const SegParam* sp, float* p, cudaStream_t st);
 cudaError_t launch_aggregate(const AggArgs& A, int32_t* off, float* out, int* status, cudaStream_t st);
 cudaError_t launch_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t i0, int64_t n, uint32_t* out,

@@ -529,3 +529,51 @@ def test_cluster_solve_large_budget(gs, force_exact):
     assert flips <= 2
     del g
     torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+@pytest.mark.parametrize("kind,kappa,d", [("t3", 0.02, 3 * 16384 + 1000), ("lognormal", 0.2, 2 * 16384 + 4),
+                                          ("normal", 0.05, 40_001)])
+def test_hybrid_code(gs, dtype, kind, kappa, d):
+    """gs_batched_sparsify_hybrid (section 3.3, eqs. 9-10): its Q_A / Q_B equal
+    the oracle's split of the plain lists bit for bit, decode to exactly the
+    plain output, and match the oracle's Q(g)."""
+    import torch
+    M, iters, seed, step = 4, 3, 13, 5
+    g_host = np.stack([_vector(kind, d, 900 + m) for m in range(M)])
+    if dtype == "bf16":
+        g_host = workloads.bf16_bits_to_f32(workloads.f32_to_bf16_bits(g_host)).reshape(M, d)
+        g = _dev(workloads.f32_to_bf16_bits(g_host).reshape(M, d)).view(torch.bfloat16)
+    else:
+        g = _dev(g_host)
+    idx, val, nnz, inf = _sparsify_batched(gs, g_host, kappa, iters, seed, step, 0, dtype, info=True)
+    assert gs.gs_sync_status() == gs.GS_OK
+    qa_i = torch.empty((M, d), dtype=torch.int32, device="cuda")
+    qa_v = torch.empty((M, d), dtype=torch.float32, device="cuda")
+    qb = torch.empty((M, d), dtype=torch.int32, device="cuda")
+    na = torch.empty(M, dtype=torch.int32, device="cuda")
+    nb = torch.empty(M, dtype=torch.int32, device="cuda")
+    il = torch.empty(M, dtype=torch.float32, device="cuda")
+    info = torch.zeros(M * gs.INFO_BYTES, dtype=torch.uint8, device="cuda")
+    gs.gs_batched_sparsify_hybrid(g, kappa, iters, seed, step, 0, qa_i, qa_v, qb, na, nb, il, info=info)
+    assert gs.gs_sync_status() == gs.GS_OK
+    rec = gs.decode_info(info)
+    n = nnz.cpu().numpy()
+    na_h, nb_h, il_h = na.cpu().numpy(), nb.cpu().numpy(), il.cpu().numpy()
+    for m in range(M):
+        lam = rec[m]["lambda"]
+        gi = idx[m, :n[m]].cpu().numpy()
+        gv = val[m, :n[m]].cpu().numpy()
+        ea, ev, eb, einv = oracle.hybrid_encode(g_host[m], lam, gi, gv)
+        got_a = qa_i[m, :na_h[m]].cpu().numpy()
+        got_v = qa_v[m, :na_h[m]].cpu().numpy()
+        got_b = qb[m, :nb_h[m]].cpu().numpy().view(np.uint32)
+        np.testing.assert_array_equal(got_a, ea)
+        np.testing.assert_array_equal(got_v, ev)
+        np.testing.assert_array_equal(got_b, eb)
+        assert il_h[m] == np.float32(einv)
+        assert na_h[m] == rec[m]["capped"]
+        di, dv = oracle.hybrid_decode(got_a, got_v, got_b, float(il_h[m]))
+        np.testing.assert_array_equal(di, gi)
+        np.testing.assert_array_equal(dv, gv)
+        compare_sparse(di, dv, g_host[m], kappa, iters, seed, step, m)
