@@ -66,7 +66,13 @@ def lib():
         L.gso_ternary_bits.restype = ctypes.c_double
         L.gso_comm_bits.argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_double, ctypes.c_int]
         L.gso_comm_bits.restype = ctypes.c_double
-        for f in ("gso_greedy_lambda", "gso_greedy_pvector", "gso_probabilities", "gso_sparsify",
+        L.gso_closed_form_lambda.argtypes = [ctypes.c_void_p, ctypes.c_int64, ctypes.c_double, P(Info)]
+        L.gso_probabilities_eps.argtypes = [ctypes.c_void_p, ctypes.c_int64, ctypes.c_double, ctypes.c_void_p,
+                                            P(Info)]
+        L.gso_sparsify_eps.argtypes = [ctypes.c_void_p, ctypes.c_int64, ctypes.c_double, ctypes.c_uint64,
+                                       ctypes.c_uint32, ctypes.c_uint32, ctypes.c_int64, ctypes.c_void_p,
+                                       ctypes.c_void_p, P(ctypes.c_int64), P(Info)]
+        for f in ("gso_closed_form_lambda", "gso_probabilities_eps", "gso_sparsify_eps", "gso_greedy_lambda", "gso_greedy_pvector", "gso_probabilities", "gso_sparsify",
                   "gso_segmented_sparsify", "gso_aggregate", "gso_hybrid_encode", "gso_hybrid_decode"):
             getattr(L, f).restype = ctypes.c_int
         _LIB = L
@@ -158,6 +164,36 @@ def aggregate(idx_list, val_list, d):
     out = np.empty(d, dtype=np.float32)
     _check(lib().gso_aggregate(ip, vp, nn.ctypes.data, M, d, out.ctypes.data))
     return out
+
+
+def closed_form_lambda(g, eps):
+    """Algorithm 2 (section 3.2): lambda of (7) for the smallest k of (6);
+    `capped` is that k."""
+    g, ptr = _f32(g)
+    info = Info()
+    _check(lib().gso_closed_form_lambda(ptr, g.size, float(eps), ctypes.byref(info)))
+    return info.as_dict()
+
+
+def probabilities_eps(g, eps):
+    """p of Algorithm 2: 1 on the k largest magnitudes, lambda |g_i| elsewhere."""
+    g, ptr = _f32(g)
+    p = np.empty(g.size, dtype=np.float64)
+    info = Info()
+    _check(lib().gso_probabilities_eps(ptr, g.size, float(eps), p.ctypes.data, ctypes.byref(info)))
+    return p, info.as_dict()
+
+
+def sparsify_eps(g, eps, seed, step, worker, i0=0):
+    """Q(g) with the p of Algorithm 2 and the same Philox draw as sparsify()."""
+    g, ptr = _f32(g)
+    idx = np.empty(g.size, dtype=np.int32)
+    val = np.empty(g.size, dtype=np.float32)
+    n = ctypes.c_int64()
+    info = Info()
+    _check(lib().gso_sparsify_eps(ptr, g.size, float(eps), seed, step, worker, i0, idx.ctypes.data,
+                                  val.ctypes.data, ctypes.byref(n), ctypes.byref(info)))
+    return idx[:n.value].copy(), val[:n.value].copy(), info.as_dict()
 
 
 def hybrid_encode(g, lam, idx, val):

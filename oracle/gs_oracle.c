@@ -18,6 +18,9 @@
  *                  have been made).
  *   Algorithm 1    step 6: the M sparse vectors are summed (the 1/M of the
  *                  average is left to the caller).
+ *   Algorithm 2    the closed-form solution of problem (4) for a variance
+ *                  budget epsilon: sort the magnitudes, take the smallest k
+ *                  satisfying (6), set p by (7).
  *
  * Readings where the paper is silent (each is listed in the design doc):
  *   - `iters` is the maximum number of rescalings (Algorithm 3, steps 4-10);
@@ -26,6 +29,11 @@
  *   - g_i = 0 gives p_i = 0; such coordinates are never kept.
  *   - If the active mass sum_{i in I} p_i is 0 the loop stops.
  *   - If sum |g_i| = 0, lambda = 0 and nothing is kept.
+ *   - Algorithm 2: the first display of section 3.2 squares g_(k) inside a
+ *     sum over i; it is read as g_(i)^2 (the only reading under which (6)
+ *     and (7) follow from it).  With g != 0 the smallest k of (6) is at most
+ *     (number of non-zero g_i) - 1, so the suffix in (7) holds a non-zero
+ *     entry and lambda is finite and positive; g = 0 gives lambda = 0.
  *   - The Bernoulli draw uses Philox4x32-10 (Salmon et al., SC'11), key =
  *     (seed lo, seed hi), counter = (q lo, q hi, worker, step) with q = i/4,
  *     word i mod 4; u_i = word * 2^-32 and Z_i = [u_i < p_i].
@@ -427,4 +435,112 @@ GSO_EXPORT double gso_comm_bits(int64_t d, int64_t n_capped, double sum_p_uncapp
     double q = ld * sum_p_uncapped;
     if (q > 2.0 * (double)d) q = 2.0 * (double)d;
     return (double)n_capped * ((double)b + ld) + q + (double)b;
+}
+
+/* ------------------------------------------------------------------------
+ * Section 3.2, Algorithm 2: the closed-form solution of problem (4),
+ *     min sum p_i  s.t.  sum g_i^2 / p_i <= (1 + eps) sum g_i^2,  0 < p_i <= 1.
+ * With the magnitudes sorted from the largest, a_1 >= a_2 >= ... >= a_d,
+ * step 1 takes the smallest k with
+ *     a_{k+1} sum_{i>k} a_i <= eps sum_i g_i^2 + sum_{i>k} a_i^2      (6)
+ * and step 2 sets p = 1 on the k largest and, on the rest,
+ *     p_i = |g_i| lambda,  lambda = sum_{i>k} a_i / (eps sum g^2 + sum_{i>k} a_i^2)   (7).
+ * The suffix sums are accumulated from the smallest magnitude up.
+ * `capped` receives k, `sum_p` = k + lambda sum_{i>k} a_i, `l1` = sum |g_i|,
+ * and *a_k the k-th largest magnitude (+inf when k = 0): p_i = 1 exactly
+ * for |g_i| >= a_k.
+ * ---------------------------------------------------------------------- */
+static int cmp_desc(const void* x, const void* y)
+{
+    const double a = *(const double*)x, b = *(const double*)y;
+    return (a < b) - (a > b);
+}
+
+static int closed_form(const float* g, int64_t d, double eps, gso_info* info, double* a_k)
+{
+    double *a, *A, *B, S = 0.0, l1 = 0.0;
+    int64_t i, k;
+    if (d < 1 || !(eps >= 0.0) || !isfinite(eps)) return GSO_INVALID;
+    memset(info, 0, sizeof(*info));
+    *a_k = INFINITY;
+    for (i = 0; i < d; i++) {
+        const double x = (double)g[i];
+        S += x * x;
+        l1 += fabs(x);
+    }
+    if (!isfinite(S) || !isfinite(l1)) return GSO_NONFINITE;
+    info->l1 = l1;
+    if (S == 0.0) return GSO_OK; /* g = 0: nothing to keep */
+
+    a = (double*)malloc((size_t)d * sizeof(double));
+    A = (double*)malloc((size_t)(d + 1) * sizeof(double));
+    B = (double*)malloc((size_t)(d + 1) * sizeof(double));
+    if (!a || !A || !B) { free(a); free(A); free(B); return GSO_INTERNAL; }
+    for (i = 0; i < d; i++) a[i] = fabs((double)g[i]);
+    qsort(a, (size_t)d, sizeof(double), cmp_desc);
+    /* A[j] = sum_{i >= j} a_i and B[j] = sum_{i >= j} a_i^2 over the sorted
+     * magnitudes (0-based j; A[d] = B[d] = 0). */
+    A[d] = 0.0;
+    B[d] = 0.0;
+    for (i = d - 1; i >= 0; i--) {
+        A[i] = A[i + 1] + a[i];
+        B[i] = B[i + 1] + a[i] * a[i];
+    }
+    /* (6) for k = 0, 1, ...: a_{k+1} is a[k] and the sums over i > k start at a[k]. */
+    for (k = 0; k < d; k++)
+        if (a[k] * A[k] <= eps * S + B[k]) break;
+    if (k == d) { free(a); free(A); free(B); return GSO_INTERNAL; } /* (6) holds at k = d - 1 when eps >= 0 */
+    info->lambda = A[k] / (eps * S + B[k]);
+    info->capped = k;
+    info->sum_p = (double)k + info->lambda * A[k];
+    if (k > 0) *a_k = a[k - 1];
+    free(a);
+    free(A);
+    free(B);
+    return GSO_OK;
+}
+
+GSO_EXPORT int gso_closed_form_lambda(const float* g, int64_t d, double eps, gso_info* info)
+{
+    double a_k;
+    return closed_form(g, d, eps, info, &a_k);
+}
+
+/* p from (7): 1 on the k largest magnitudes, lambda |g_i| elsewhere. */
+GSO_EXPORT int gso_probabilities_eps(const float* g, int64_t d, double eps, double* p, gso_info* info)
+{
+    double a_k;
+    int64_t i;
+    int rc = closed_form(g, d, eps, info, &a_k);
+    if (rc != GSO_OK) return rc;
+    for (i = 0; i < d; i++) {
+        const double x = fabs((double)g[i]);
+        p[i] = x >= a_k ? 1.0 : info->lambda * x;
+    }
+    return GSO_OK;
+}
+
+/* Section 3 with the p of Algorithm 2: the same Philox draw, amplification and
+ * ascending (index, value) output as gso_sparsify. */
+GSO_EXPORT int gso_sparsify_eps(const float* g, int64_t d, double eps, uint64_t seed, uint32_t step, uint32_t worker,
+                                int64_t i0, int32_t* idx, float* val, int64_t* nnz, gso_info* info)
+{
+    double a_k;
+    int64_t i, n = 0;
+    int rc = closed_form(g, d, eps, info, &a_k);
+    *nnz = 0;
+    if (rc != GSO_OK) return rc;
+    for (i = 0; i < d; i++) {
+        const double gi = (double)g[i];
+        const double x = fabs(gi);
+        const double p = x >= a_k ? 1.0 : info->lambda * x;
+        if (p == 0.0) continue;
+        if (gso_uniform(seed, step, worker, i0 + i) < p) {
+            idx[n] = (int32_t)(i0 + i);
+            val[n] = (float)(gi / p);
+            n++;
+        }
+    }
+    *nnz = n;
+    return GSO_OK;
 }
