@@ -149,6 +149,25 @@ gs_status gs_batched_sparsify_hybrid(const void* g, int dtype, int M, int64_t d,
                                      gs_info* info, void* stream);
 
 /*
+ * Algorithm 2 (section 3.2): the closed-form solution of problem (4) for a
+ * variance budget eps >= 0 instead of a density budget.  lambda is the one
+ * for which sum_i g_i^2 / p_i = (1 + eps) sum_i g_i^2 with
+ * p_i = min(lambda |g_i|, 1): (7) with the smallest k satisfying (6).  It is
+ * found without a sort (a histogram pass over g brackets 1 / lambda, then
+ * Newton steps over the values above the bracket's lower end), so each call
+ * reads g twice.  eps = 0 keeps every non-zero coordinate.  sum_i g_i^2 is
+ * accumulated in fp32 pairs: a |g_i| above ~1.8e19 (g_i^2 overflows fp32)
+ * is reported as GS_ERR_NONFINITE, as are NaN / Inf.  In the gs_info records
+ * `iters_run` counts the Newton steps and `capped` is k.
+ *   p      device, d fp32: p_i rounded to fp32 (gs_probabilities_eps)
+ * Other arguments as in gs_probabilities_ex / gs_batched_sparsify.
+ */
+gs_status gs_probabilities_eps(const float* g, int64_t d, double eps, float* p, gs_info* info, void* stream);
+gs_status gs_batched_sparsify_eps(const void* g, int dtype, int M, int64_t d, double eps, uint64_t seed, uint32_t step,
+                                  uint32_t worker0, int32_t* idx, float* val, int32_t* nnz, int64_t cap, gs_info* info,
+                                  void* stream);
+
+/*
  * Layer-wise sparsification (section 5.2: each layer is sparsified on its
  * own).  Each worker's vector is cut into L segments by the HOST array
  * seg_offsets[0..L] (0 = seg_offsets[0] < ... < seg_offsets[L] = d); every

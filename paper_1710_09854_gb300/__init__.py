@@ -23,7 +23,7 @@ GS_OPT_FORCE_EXACT_SOLVE, GS_OPT_SAMPLE_SIZE, GS_OPT_KERNEL_TIMING, GS_OPT_STREA
 
 # Symbols include/gs.h declares (checked by the tests).
 EXPORTS = ("gs_status_string", "gs_last_error", "gs_version", "gs_sync_status", "gs_probabilities", "gs_probabilities_ex",
-           "gs_sparsify", "gs_batched_sparsify", "gs_batched_sparsify_hybrid", "gs_segmented_sparsify", "gs_sparse_aggregate",
+           "gs_sparsify", "gs_batched_sparsify", "gs_batched_sparsify_hybrid", "gs_probabilities_eps", "gs_batched_sparsify_eps", "gs_segmented_sparsify", "gs_sparse_aggregate",
            "gs_sparsify_aggregate", "gs_sparsify_noalloc", "gs_pipeline_host", "gs_random_words", "gs_set_option", "gs_kernel_count", "gs_kernel_name",
            "gs_kernel_times")
 
@@ -64,6 +64,8 @@ def lib():
             "gs_batched_sparsify": ([vp, i32, i32, i64, dbl, i32, u64, u32, u32, vp, vp, vp, i64, vp, vp], i32),
             "gs_batched_sparsify_hybrid": ([vp, i32, i32, i64, dbl, i32, u64, u32, u32, vp, vp, vp, vp, vp, vp, i64,
                                             vp, vp], i32),
+            "gs_probabilities_eps": ([vp, i64, dbl, vp, vp, vp], i32),
+            "gs_batched_sparsify_eps": ([vp, i32, i32, i64, dbl, u64, u32, u32, vp, vp, vp, i64, vp, vp], i32),
             "gs_segmented_sparsify": ([vp, i32, i32, i64, vp, i32, dbl, i32, u64, u32, u32, vp, vp, vp, i64, vp, vp],
                                       i32),
             "gs_sparse_aggregate": ([vp, vp, vp, i32, i64, vp, vp], i32),
@@ -251,6 +253,27 @@ def gs_batched_sparsify_hybrid(g, kappa, iters, seed, step, worker0, qa_idx, qa_
                                             _ptr(n_a, "n_a", (torch.int32,)), _ptr(n_b, "n_b", (torch.int32,)),
                                             _ptr(inv_lam, "inv_lam", (torch.float32,)), cap, _ptr(info, "info"),
                                             _stream(stream)), "gs_batched_sparsify_hybrid")
+
+
+def gs_probabilities_eps(g, eps, p, info=None, stream=None):
+    """p of Algorithm 2 (variance budget eps) for one fp32 gradient."""
+    import torch
+    _check(lib().gs_probabilities_eps(_ptr(g, "g", (torch.float32,)), g.numel(), float(eps),
+                                      _ptr(p, "p", (torch.float32,)), _ptr(info, "info"), _stream(stream)),
+           "gs_probabilities_eps")
+
+
+def gs_batched_sparsify_eps(g, eps, seed, step, worker0, idx, val, nnz, info=None, stream=None):
+    """gs_batched_sparsify with lambda from Algorithm 2 (variance budget eps)."""
+    import torch
+    M, d = g.shape
+    cap = idx.shape[1]
+    if idx.shape[0] != M or tuple(val.shape) != tuple(idx.shape) or nnz.numel() != M:
+        raise ValueError("idx / val must be (M, cap) and nnz (M,)")
+    _check(lib().gs_batched_sparsify_eps(_ptr(g, "g"), _g_dtype(g), M, d, float(eps), int(seed), int(step),
+                                         int(worker0), _ptr(idx, "idx", (torch.int32,)),
+                                         _ptr(val, "val", (torch.float32,)), _ptr(nnz, "nnz", (torch.int32,)), cap,
+                                         _ptr(info, "info"), _stream(stream)), "gs_batched_sparsify_eps")
 
 
 def gs_segmented_sparsify(g, seg_offsets, kappa, iters, seed, step, worker0, idx, val, nnz, info=None, stream=None):

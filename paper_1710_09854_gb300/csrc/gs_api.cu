@@ -126,12 +126,18 @@ struct Workspace {
     SegParam* sp;
     Lists ls;
     int32_t* nnz;       // hybrid calls: the per-worker kept counts (plain calls write the caller's)
+    uint32_t* hist;     // Algorithm 2: per-segment magnitude histograms
+    double* u_sq;       // Algorithm 2: sum g^2 partials
 };
 
 void carve(Arena& a, Workspace& w, int n_seg, int n_chunks, int64_t n, bool build_p, bool hybrid = false,
-           int M = 0) {
+           int M = 0, bool alg2 = false) {
     std::memset(&w, 0, sizeof(w));
     w.sp = a.take<SegParam>(n_seg);
+    if (alg2) {
+        w.hist = a.take<uint32_t>(eps_hist_words(n_seg));
+        w.u_sq = a.take<double>(eps_units(n_chunks));
+    }
     w.ls.c_val = a.take<float>(n);
     w.ls.c_cnt = a.take<int32_t>(n_chunks);
     w.ls.s_low = a.take<double>(n_chunks);
@@ -149,12 +155,16 @@ void carve(Arena& a, Workspace& w, int n_seg, int n_chunks, int64_t n, bool buil
     }
 }
 
-// Shared driver of every sparsify / probabilities call.
+// Shared driver of every sparsify / probabilities call.  eps >= 0 selects
+// Algorithm 2 (variance budget eps; kappa and iters unused), else Algorithm 3.
 gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off, int L, double kappa, int iters,
               uint64_t seed, uint32_t step, uint32_t worker0, int32_t* idx, float* val, int32_t* nnz, int64_t cap,
-              gs_info* info, float* p, cudaStream_t st, float* agg_out = nullptr, const HybridOut* hy = nullptr) {
+              gs_info* info, float* p, cudaStream_t st, float* agg_out = nullptr, const HybridOut* hy = nullptr,
+              double eps = -1.0) {
     const bool prob = p != nullptr;
-    if (!g || M < 1 || d < 1 || d >= kMaxD || bad_kappa(kappa) || iters < 0) return GS_ERR_INVALID_ARG;
+    const bool alg2 = eps >= 0.0;
+    if (!g || M < 1 || d < 1 || d >= kMaxD) return GS_ERR_INVALID_ARG;
+    if (alg2 ? !std::isfinite(eps) : (bad_kappa(kappa) || iters < 0)) return GS_ERR_INVALID_ARG;
     if (dtype != GS_DTYPE_F32 && dtype != GS_DTYPE_BF16) return GS_ERR_INVALID_ARG;
     const size_t esz = dtype == GS_DTYPE_F32 ? 4 : 2;
     if ((reinterpret_cast<uintptr_t>(g) % esz) != 0) return GS_ERR_INVALID_ARG;
@@ -208,7 +218,7 @@ gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off
 
     Arena a;
     Workspace w;
-    carve(a, w, n_seg, n_chunks, (int64_t)M * d, !prob, hy != nullptr, M);
+    carve(a, w, n_seg, n_chunks, (int64_t)M * d, !prob, hy != nullptr, M, alg2);
     void* mem = nullptr;
     {
         const cudaError_t ea = cudaMallocFromPoolAsync(&mem, a.off, s->pool, st);
@@ -216,7 +226,7 @@ gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off
     }
     a.base = static_cast<char*>(mem);
     a.off = 0;
-    carve(a, w, n_seg, n_chunks, (int64_t)M * d, !prob, hy != nullptr, M);
+    carve(a, w, n_seg, n_chunks, (int64_t)M * d, !prob, hy != nullptr, M, alg2);
 
     int force, ns, path;
     {
@@ -228,13 +238,17 @@ gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off
     bool tma_ok = path != 1 && stream_tma_eligible(Lo);
     for (int l = 0; tma_ok && L > 1 && l <= L; ++l)
         if (seg_off[l] % 4 != 0) tma_ok = false;
-    cudaError_t e = launch_bound(Lo, w.sp, n_seg, kappa, ns, force, st);
+    cudaError_t e = alg2 ? launch_eps_bracket(Lo, w.sp, w.hist, w.u_sq, n_seg, n_chunks, eps, force, st)
+                         : launch_bound(Lo, w.sp, n_seg, kappa, ns, force, st);
     if (e == cudaSuccess) {
         bool used = false;
         if (tma_ok) e = launch_stream_tma(Lo, w.sp, w.ls, n_chunks, s->status, st, &used);
         if (e == cudaSuccess && !used) e = launch_stream(Lo, w.sp, w.ls, n_chunks, !prob, st);
     }
-    if (e == cudaSuccess) e = launch_solve(Lo, w.sp, w.ls, n_seg, kappa, iters, force, s->status, info, st);
+    if (e == cudaSuccess) {
+        e = alg2 ? launch_solve_eps(Lo, w.sp, w.ls, n_seg, eps, s->status, info, st)
+                 : launch_solve(Lo, w.sp, w.ls, n_seg, kappa, iters, force, s->status, info, st);
+    }
     if (e == cudaSuccess) {
         if (prob) e = launch_prob(Lo, w.sp, p, st);
         else e = launch_compact(Lo, w.sp, w.ls, n_chunks, idx, val, hy ? w.nnz : nnz, cap, s->status, st, agg_out,
@@ -506,6 +520,20 @@ gs_status gs_batched_sparsify_hybrid(const void* g, int dtype, int M, int64_t d,
     h.inv_lam = inv_lam;
     return run(g, dtype, M, d, nullptr, 1, kappa, iters, seed, step, worker0, nullptr, nullptr, nullptr, cap, info,
                nullptr, static_cast<cudaStream_t>(stream), nullptr, &h);
+}
+
+gs_status gs_probabilities_eps(const float* g, int64_t d, double eps, float* p, gs_info* info, void* stream) {
+    if (!p || !(eps >= 0.0) || !std::isfinite(eps)) return GS_ERR_INVALID_ARG;
+    return run(g, GS_DTYPE_F32, 1, d, nullptr, 1, 0.0, 0, 0, 0, 0, nullptr, nullptr, nullptr, 0, info, p,
+               static_cast<cudaStream_t>(stream), nullptr, nullptr, eps);
+}
+
+gs_status gs_batched_sparsify_eps(const void* g, int dtype, int M, int64_t d, double eps, uint64_t seed, uint32_t step,
+                                  uint32_t worker0, int32_t* idx, float* val, int32_t* nnz, int64_t cap, gs_info* info,
+                                  void* stream) {
+    if (!(eps >= 0.0) || !std::isfinite(eps)) return GS_ERR_INVALID_ARG;
+    return run(g, dtype, M, d, nullptr, 1, 0.0, 0, seed, step, worker0, idx, val, nnz, cap, info, nullptr,
+               static_cast<cudaStream_t>(stream), nullptr, nullptr, eps);
 }
 
 gs_status gs_sparsify_noalloc(const float* g, int64_t d, double kappa, int iters, uint64_t seed, uint32_t step,

@@ -97,6 +97,16 @@ cudaError_t launch_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t 
 bool stream_tma_eligible(const Layout& Lo);
 cudaError_t launch_stream_tma(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, int* status,
                               cudaStream_t st, bool* used);
+// Algorithm 2 (variance budget eps): the histogram pass and the bracket of
+// 1 / lambda (replaces launch_bound), and the Newton solve on C (replaces
+// launch_solve).  hist holds eps_hist_words(n_seg) words, u_sq
+// eps_units(n_chunks) doubles.
+size_t eps_hist_words(int n_seg);
+size_t eps_units(int n_chunks);
+cudaError_t launch_eps_bracket(const Layout& Lo, SegParam* sp, uint32_t* hist, double* u_sq, int n_seg, int n_chunks,
+                               double eps, int take_all, cudaStream_t st);
+cudaError_t launch_solve_eps(const Layout& Lo, SegParam* sp, const Lists& Ls, int n_seg, double eps, int* status,
+                             gs_info_dev* info, cudaStream_t st);
 // The launchers record which step failed; the C ABI reports it.
 void set_launch_error_site(const char* where);
 const char* launch_error_site();

@@ -18,6 +18,9 @@ enum KernelId : int {
     kKDecide,
     kKScan,
     kKSum,
+    kKEpsHist,
+    kKEpsBracket,
+    kKSolveEps,
     kNumKernels
 };
 

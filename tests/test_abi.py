@@ -74,3 +74,14 @@ def test_host_argument_checks(gs):
     assert L.gs_set_option(gs.GS_OPT_SAMPLE_SIZE, 100) == inv
     assert L.gs_set_option(gs.GS_OPT_FORCE_EXACT_SOLVE, 2) == inv
     assert L.gs_set_option(gs.GS_OPT_SAMPLE_SIZE, 16384) == 0
+
+
+def test_eps_entry_points_reject_bad_budgets():
+    # Host-side validation: these return before any CUDA call.
+    import paper_1710_09854_gb300 as gs
+    L = gs.lib()
+    fake = 256  # never dereferenced
+    for eps in (-0.5, float("nan"), float("inf")):
+        assert L.gs_probabilities_eps(fake, 10, eps, fake, None, None) == gs.GS_ERR_INVALID_ARG
+        assert L.gs_batched_sparsify_eps(fake, 0, 1, 10, eps, 1, 0, 0, fake, fake, fake, 10, None,
+                                         None) == gs.GS_ERR_INVALID_ARG
