@@ -317,6 +317,7 @@ def run_gpu(args):
         if rc != gs.GS_OK:
             raise RuntimeError(f"device status after the sparsify-only run: {gs.status_string(rc)}")
     hybrid = run_hybrid(gs, g, kappa, w, args, dev, stream, n_bd, hbm) if off is None else None
+    vbudget = run_variance_budget(gs, g, w, args, dev, stream, n_bd, hbm) if off is None else None
 
     # ---- end to end through the host-buffer entry point
     e2e = None
@@ -337,6 +338,7 @@ def run_gpu(args):
         "roofline": roofline,
         "sparsify_roofline": sp_only,
         "hybrid_code": hybrid,
+        "variance_budget": vbudget,
         "kernels": kernels, "kernels_steps": n_bd,
         "nnz_per_step": nnz_total,
         "gpu_launches": launches,
@@ -452,6 +454,63 @@ def run_hybrid(gs, g, kappa, w, args, dev, stream, n_steps, hbm):
             "unit": "GB/s", "n_a": int(a.sum()), "n_b": int(b_.sum()),
             "bits_per_step": {k: round(v) for k, v in bits.items()},
             "bits_per_coordinate": {k: round(v / (M * d), 4) for k, v in bits.items()}}
+
+
+VARIANCE_BUDGETS = (30.0, 1.0)   # about 1.2% and 21% density on the Student-t gradients
+
+
+def run_variance_budget(gs, g, w, args, dev, stream, n_steps, hbm):
+    """Algorithm 2 (gs_batched_sparsify_eps) on the same gradients for a few
+    variance budgets eps: time per step, density, Newton steps, the bytes of
+    the call (two reads of g, the kept (idx, val) pairs written) and the
+    histogram pass against its one read of g."""
+    import torch
+    M, d = g.shape
+    esz = g.element_size()
+    idx = torch.empty((M, d), dtype=torch.int32, device=dev)
+    val = torch.empty((M, d), dtype=torch.float32, device=dev)
+    nnz = torch.empty(M, dtype=torch.int32, device=dev)
+    info = torch.zeros(M * gs.INFO_BYTES, dtype=torch.uint8, device=dev)
+    out = []
+    for eps in VARIANCE_BUDGETS:
+        for t in range(3):
+            gs.gs_batched_sparsify_eps(g, eps, w.seed, t, 0, idx, val, nnz, info=info, stream=stream)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for t in range(n_steps):
+            gs.gs_batched_sparsify_eps(g, eps, w.seed, args.warmup + t, 0, idx, val, nnz, stream=stream)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms = max_over_ranks(e0.elapsed_time(e1) / n_steps, dev)
+        # per-kernel times with every launch bracketed (a few steps)
+        nb = min(n_steps, 20)
+        gs.gs_set_option(gs.GS_OPT_KERNEL_TIMING, 1)
+        gs.gs_kernel_times()
+        for t in range(nb):
+            gs.gs_batched_sparsify_eps(g, eps, w.seed, t, 0, idx, val, nnz, info=info, stream=stream)
+        torch.cuda.synchronize()
+        bd = gs.gs_kernel_times()
+        gs.gs_set_option(gs.GS_OPT_KERNEL_TIMING, 0)
+        rc = gs.gs_sync_status(stream)
+        if rc != gs.GS_OK:
+            raise RuntimeError(f"device status after the variance-budget run: {gs.status_string(rc)}")
+        rec = gs.decode_info(info)
+        kept = int(nnz.sum().item())
+        algo = 2 * M * d * esz + 8 * kept
+        gbs = algo / (ms / 1e3) / 1e9
+        hist_ms = bd.get("k_eps_hist", (0.0, 0))[0] / nb
+        hist_gbs = M * d * esz / (hist_ms / 1e3) / 1e9 if hist_ms > 0 else 0.0
+        out.append({"api": "gs_batched_sparsify_eps", "eps": eps, "steps": n_steps, "ms_per_step": round(ms, 4),
+                    "coords_per_s": M * d / (ms / 1e3), "density": round(kept / (M * d), 6),
+                    "newton_steps_max": max(r["iters_run"] for r in rec),
+                    "algorithmic_bytes": algo, "achieved": round(gbs, 1), "peak": hbm, "frac": round(gbs / hbm, 4),
+                    "unit": "GB/s",
+                    "hist_roofline": {"kernel": "k_eps_hist", "bound": "hbm", "algorithmic_bytes": M * d * esz,
+                                      "ms_per_launch": round(hist_ms, 4), "achieved": round(hist_gbs, 1),
+                                      "peak": hbm, "frac": round(hist_gbs / hbm, 4)},
+                    "kernels": {k: round(v[0] / nb, 4) for k, v in bd.items() if v[1]}})
+    return out
 
 
 def load_traffic(kernel, workload, dtype, kappa):

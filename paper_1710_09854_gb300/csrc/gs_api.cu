@@ -137,6 +137,7 @@ void carve(Arena& a, Workspace& w, int n_seg, int n_chunks, int64_t n, bool buil
     if (alg2) {
         w.hist = a.take<uint32_t>(eps_hist_words(n_seg));
         w.u_sq = a.take<double>(eps_units(n_chunks));
+        w.ls.b_low = a.take<double>(n_chunks);
     }
     w.ls.c_val = a.take<float>(n);
     w.ls.c_cnt = a.take<int32_t>(n_chunks);

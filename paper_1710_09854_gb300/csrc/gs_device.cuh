@@ -87,6 +87,7 @@ struct Lists {
     int32_t* k_sub;     // [n_chunks][kSubStride] kept entries of the chunk before each 1024-coordinate slice
     int32_t* k_offa;    // [n_chunks] hybrid code only (else NULL): kept entries with p = 1, then their offsets
     int32_t* c_pre;     // [n_chunks + n_seg] prefix scratch for segments with many chunks
+    double* b_low;      // [n_chunks] Algorithm 2 only (else NULL): sum of g^2 outside C
 };
 
 struct Chunk {

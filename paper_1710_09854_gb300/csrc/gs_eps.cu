@@ -28,7 +28,10 @@
 //                  pass over C (everything below t_c is summed in S_low).
 //                  From the right, Newton's steps on a convex piecewise-linear
 //                  function never pass the root, and a step that leaves the
-//                  set {|g| < t} unchanged has landed on it exactly.
+//                  set {|g| < t} unchanged has landed on it exactly.  Where
+//                  they crawl (eps = 0, where phi is flat at the root, or more
+//                  than 24 steps) a bisection over the fp32 bit patterns of t
+//                  finishes in at most 31 more passes.
 // Then the decide / emit (or probabilities) kernels of Algorithm 3 run as is.
 #include <cooperative_groups.h>
 #include <cuda_runtime.h>
@@ -51,11 +54,12 @@ constexpr int kUnitLog = 12;
 constexpr int kUnit = 1 << kUnitLog;                 // coordinates per S partial
 constexpr int kUnitsPerChunk = kChunk / kUnit;
 constexpr int kHistWarps = 8;
-constexpr int kHistBatch = 8;     // 4-coordinate groups per lane in flight
-constexpr int kHistCtasPerSm = 3; // 64 KB of warp histograms per CTA
+constexpr int kHistBatch = 8;     // 16-byte loads per lane in flight
+constexpr int kHistCtasPerSm = 5;   // 48 registers x 256 threads
 constexpr int kBrThreads = 256;
 constexpr int kBrPer = kHistBins / kBrThreads;
-constexpr int kEpsNewtonMax = 64;
+constexpr int kEpsNewtonMax = 24;
+constexpr int kEpsBisectMax = 32;   // a bisection over fp32 bit patterns ends within 31 passes
 constexpr int kEpsCTAs = 8;       // cluster size of k_solve_eps for long segments
 
 static_assert(kChunk % kUnit == 0, "units tile a chunk");
@@ -63,70 +67,105 @@ static_assert(kHistBins % kBrThreads == 0, "bins split evenly over the bracket C
 
 __device__ __forceinline__ float bin_lo(int b) { return __uint_as_float((uint32_t)b << kHistShift); }
 
-__device__ __forceinline__ void hist_flush(uint32_t* h, uint32_t* gh, int lane) {
-    __syncwarp();
-    for (int b = lane; b < kHistBins; b += 32) {
-        const uint32_t n = h[b];
-        if (n) {
-            atomicAdd(gh + b, n);
-            h[b] = 0u;
-        }
-    }
-    __syncwarp();
+__device__ __forceinline__ void hist_count(uint32_t* h, float x) {
+    atomicAdd(&h[(__float_as_uint(x) & 0x7FFFFFFFu) >> kHistShift], 1u);
 }
 
-// Each warp owns a contiguous run of 4096-coordinate units (so it meets a
-// new segment at most a few times) and its own histogram; it adds the
-// histogram into the segment's global one (integer atomics: the order does
-// not matter) whenever the segment changes.  S partials go to u_sq[unit],
-// each a fixed lane assignment and a fixed shuffle tree.
+// Counts and squares of 8 fp32 lanes' values (one 16-byte load each of 4).
+__device__ __forceinline__ float hist_batch_f32(uint32_t* h, const float4 (&v)[kHistBatch]) {
+    float s0 = 0.0f, s1 = 0.0f, s2 = 0.0f, s3 = 0.0f;
+#pragma unroll
+    for (int r = 0; r < kHistBatch; ++r) {
+        hist_count(h, v[r].x);
+        hist_count(h, v[r].y);
+        hist_count(h, v[r].z);
+        hist_count(h, v[r].w);
+        s0 = fmaf(v[r].x, v[r].x, s0);
+        s1 = fmaf(v[r].y, v[r].y, s1);
+        s2 = fmaf(v[r].z, v[r].z, s2);
+        s3 = fmaf(v[r].w, v[r].w, s3);
+    }
+    return (s0 + s1) + (s2 + s3);
+}
+
+// The same for bf16: each 16-byte load holds 8 values.
+__device__ __forceinline__ float hist_batch_bf16(uint32_t* h, const uint4 (&v)[kHistBatch]) {
+    float s[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll
+    for (int r = 0; r < kHistBatch; ++r) {
+        const uint32_t w[4] = {v[r].x, v[r].y, v[r].z, v[r].w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            const float a = bf16_bits_to_float(w[k] & 0xFFFFu), b = bf16_bits_to_float(w[k] >> 16);
+            hist_count(h, a);
+            hist_count(h, b);
+            s[k] = fmaf(a, a, s[k]);
+            s[k] = fmaf(b, b, s[k]);
+        }
+    }
+    return (s[0] + s[1]) + (s[2] + s[3]);
+}
+
+// gx CTAs per segment (block x: segment x / gx).  The CTAs of a segment share its 4096-coordinate units
+// (one warp per unit at a time) and one shared-memory histogram, added into
+// the segment's global histogram at the end (integer atomics: the order does
+// not matter).  Each unit's sum of squares is one fixed computation (lane
+// assignment, fma partials of 32 values, error-free running sum, fixed
+// shuffle tree), written to u_sq[unit].
 __global__ void __launch_bounds__(kHistWarps * 32) k_eps_hist(const __grid_constant__ Layout Lo, uint32_t* ghist,
-                                                              double* u_sq, int n_units, int per_warp) {
+                                                              double* u_sq, int gx) {
     grid_dep_wait();
-    extern __shared__ uint32_t hs[];   // [kHistWarps][kHistBins]
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    uint32_t* h = hs + warp * kHistBins;
-    for (int b = lane; b < kHistBins; b += 32) h[b] = 0u;
-    __syncwarp();
-    const int q = blockIdx.x * kHistWarps + warp;
-    const int u0 = q * per_warp;
-    const int u1 = min(n_units, u0 + per_warp);
-    int cur = -1;
-    for (int u = u0; u < u1; ++u) {
+    __shared__ uint32_t h[kHistBins];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    for (int b = tid; b < kHistBins; b += blockDim.x) h[b] = 0u;
+    __syncthreads();
+    const int s = blockIdx.x / gx, bx = blockIdx.x - s * gx;
+    int m, l, c0, c1;
+    int64_t slo, shi;
+    seg_range(Lo, s, m, l, slo, shi, c0, c1);
+    const int u_end = c1 * kUnitsPerChunk;
+    for (int u = c0 * kUnitsPerChunk + bx * kHistWarps + warp; u < u_end; u += gx * kHistWarps) {
         const int c = u / kUnitsPerChunk;
         const Chunk ch = decode_chunk(Lo, c);
-        if (ch.seg != cur) {
-            if (cur >= 0) hist_flush(h, ghist + (size_t)cur * kHistBins, lane);
-            cur = ch.seg;
-        }
         const int64_t lo = ch.lo + (int64_t)(u - c * kUnitsPerChunk) * kUnit;
         const int64_t hi = min(ch.hi, lo + kUnit);
         float sh = 0.0f, sl = 0.0f;
-        if (lo < hi) {
-            const int64_t q0 = lo >> 2, q1 = (hi - 1) >> 2;   // 4-coordinate groups touching [lo, hi)
-            for (int64_t base = q0; base <= q1; base += 32 * kHistBatch) {
-                float v[kHistBatch][4];
-                int mk[kHistBatch];
+        const int64_t flat = (int64_t)m * Lo.d + lo;
+        if (Lo.dtype == 0 && hi - lo == kUnit &&
+            (reinterpret_cast<uintptr_t>(static_cast<const float*>(Lo.g) + flat) & 15u) == 0) {
+            const float4* p4 = reinterpret_cast<const float4*>(static_cast<const float*>(Lo.g) + flat);
+#pragma unroll 1
+            for (int k0 = 0; k0 < kUnit / 128; k0 += kHistBatch) {   // 32 loads of 16 bytes per lane
+                float4 v[kHistBatch];
 #pragma unroll
-                for (int r = 0; r < kHistBatch; ++r) {
-                    const int64_t gq = base + r * 32 + lane;
-                    mk[r] = 0;
-                    v[r][0] = v[r][1] = v[r][2] = v[r][3] = 0.0f;
-                    if (gq <= q1) mk[r] = load_group(Lo, ch.m, gq, lo, hi, v[r]);
-                }
+                for (int r = 0; r < kHistBatch; ++r) v[r] = __ldcs(p4 + (k0 + r) * 32 + lane);
+                two_sum_add(sh, sl, hist_batch_f32(h, v));
+            }
+        } else if (Lo.dtype == 1 && hi - lo == kUnit &&
+                   (reinterpret_cast<uintptr_t>(static_cast<const uint16_t*>(Lo.g) + flat) & 15u) == 0) {
+            const uint4* p8 = reinterpret_cast<const uint4*>(static_cast<const uint16_t*>(Lo.g) + flat);
+#pragma unroll 1
+            for (int k0 = 0; k0 < kUnit / 256; k0 += kHistBatch) {   // 16 loads of 16 bytes per lane
+                uint4 v[kHistBatch];
 #pragma unroll
-                for (int r = 0; r < kHistBatch; ++r) {
+                for (int r = 0; r < kHistBatch; ++r) v[r] = __ldcs(p8 + (k0 + r) * 32 + lane);
+                two_sum_add(sh, sl, hist_batch_bf16(h, v));
+            }
+        } else if (lo < hi) {
+            // Ragged or unaligned unit: 4-coordinate groups with a validity mask.
+            const int64_t q0 = lo >> 2, q1 = (hi - 1) >> 2;
+            for (int64_t gq = q0 + lane; gq <= q1; gq += 32) {
+                float v[4];
+                const int mk = load_group(Lo, m, gq, lo, hi, v);
+                float s4 = 0.0f;
 #pragma unroll
-                    for (int k = 0; k < 4; ++k) {
-                        if ((mk[r] >> k) & 1) {
-                            const float a = fabsf(v[r][k]);
-                            atomicAdd(&h[__float_as_uint(a) >> kHistShift], 1u);
-                            const float p = a * a;
-                            two_sum_add(sh, sl, p);
-                            sl += fmaf(a, a, -p);   // the rounding error of a^2
-                        }
+                for (int k = 0; k < 4; ++k) {
+                    if ((mk >> k) & 1) {
+                        hist_count(h, v[k]);
+                        s4 = fmaf(v[k], v[k], s4);
                     }
                 }
+                two_sum_add(sh, sl, s4);
             }
         }
 #pragma unroll
@@ -137,7 +176,12 @@ __global__ void __launch_bounds__(kHistWarps * 32) k_eps_hist(const __grid_const
         }
         if (lane == 0) u_sq[u] = (double)sh + (double)sl;
     }
-    if (cur >= 0) hist_flush(h, ghist + (size_t)cur * kHistBins, lane);
+    __syncthreads();
+    uint32_t* gh = ghist + (size_t)s * kHistBins;
+    for (int b = tid; b < kHistBins; b += blockDim.x) {
+        const uint32_t n = h[b];
+        if (n) atomicAdd(gh + b, n);
+    }
 }
 
 // Exclusive prefix over the block of four doubles per thread (inclusive
@@ -229,10 +273,11 @@ __global__ void __launch_bounds__(kBrThreads) k_eps_bracket(const __grid_constan
     }
     __syncthreads();
 
-    // The targets carry a margin for the rounding of S and of the bounds
-    // (fp64 sums of up to 2^31 terms and one cancellation each).
+    // The targets carry a margin for the rounding of S (fp32 partials of 32
+    // squares, ~2^-20 relative at worst) and of the bounds (fp64 sums of up
+    // to 2^31 terms, one cancellation each).
     const double eS = eps * S;
-    const double slack = 0x1p-20 * eS + 0x1p-40 * S;
+    const double slack = 0x1p-16 * eS + 0x1p-40 * S;
     const double lo_target = eS - slack, hi_target = eS + slack;
     const double* P0 = pre;
     const double* P1 = pre + (kHistBins + 1);
@@ -290,7 +335,9 @@ __global__ void __launch_bounds__(kBrThreads) k_eps_bracket(const __grid_constan
 }
 
 struct EpsPart {
-    float uh, ul, qh, ql;   // sum |g| below the threshold, sum g^2 at or above it (double-float)
+    float uh, ul;           // sum |g| of C below the threshold (double-float)
+    float bh, bl;           // sum g^2 of C below it
+    float qh, ql;           // sum g^2 of C at or above it
     int below, above;       // counts of C below / at or above
 };
 
@@ -314,21 +361,26 @@ __global__ void __launch_bounds__(kThreads) k_solve_eps(const __grid_constant__ 
     int64_t lo, hi;
     seg_range(Lo, s, m, l, lo, hi, c0, c1);
     const int nch = c1 - c0;
-    const double S = sp[s].sq;
+    const double S_hist = sp[s].sq;   // the histogram pass's sum (non-finite check only)
     const float t_up = sp[s].t_up;
     const double lam_up = sp[s].lam_up;
     int flags = sp[s].flags & (kSegTakeAll | kSegNonfinite);
 
-    double sl = 0.0;
-    for (int c = c0 + tid; c < c1; c += blockDim.x) sl += Ls.s_low[c];
+    double sl = 0.0, bq = 0.0;
+    for (int c = c0 + tid; c < c1; c += blockDim.x) {
+        sl += Ls.s_low[c];
+        bq += Ls.b_low[c];
+    }
     const double S_low = block_sum(sl, shd);
+    const double B_low = block_sum(bq, shd);
     const float* cb = Ls.c_val + (int64_t)m * Lo.d + lo;
 
     int buf = 0;
-    // One pass over C at threshold tau: below = #{C : |g| < tau},
-    // U = S_low + their sum, Q = S - sum of g^2 over the rest.
-    auto pass = [&](float tau, int& below, int& above, double& U, double& Q) {
-        float uh = 0.0f, ul = 0.0f, qh = 0.0f, ql = 0.0f;
+    // One pass over C at threshold tau: below = #{C : |g| < tau}, U = S_low +
+    // their sum of |g|, Q = B_low + their sum of g^2, and Qa the sum of g^2
+    // over the rest of C.  Every sum is of positive terms (no cancellation).
+    auto pass = [&](float tau, int& below, int& above, double& U, double& Q, double& Qa) {
+        float uh = 0.0f, ul = 0.0f, bh = 0.0f, bl = 0.0f, qh = 0.0f, ql = 0.0f;
         int kb = 0, ka = 0;
         for (int q = rank * kWarps + warp; q < nch; q += ncta * kWarps) {
             const int n = Ls.c_cnt[c0 + q];
@@ -338,6 +390,9 @@ __global__ void __launch_bounds__(kThreads) k_solve_eps(const __grid_constant__ 
                 if (a < tau) {
                     ++kb;
                     two_sum_add(uh, ul, a);
+                    const float p = a * a;
+                    two_sum_add(bh, bl, p);
+                    bl += fmaf(a, a, -p);
                 } else {
                     ++ka;
                     const float p = a * a;
@@ -348,13 +403,16 @@ __global__ void __launch_bounds__(kThreads) k_solve_eps(const __grid_constant__ 
         }
         block_sum_df(uh, ul, kb, sh4);
         block_sum_df(qh, ql, ka, sh4);
-        if (tid == 0) xch[buf] = EpsPart{uh, ul, qh, ql, kb, ka};
+        int unused = 0;
+        block_sum_df(bh, bl, unused, sh4);
+        if (tid == 0) xch[buf] = EpsPart{uh, ul, bh, bl, qh, ql, kb, ka};
         cluster.sync();
-        float ruh = 0.0f, rul = 0.0f, rqh = 0.0f, rql = 0.0f;
+        float ruh = 0.0f, rul = 0.0f, rbh = 0.0f, rbl = 0.0f, rqh = 0.0f, rql = 0.0f;
         int rb = 0, ra = 0;
         for (int r = 0; r < ncta; ++r) {
             const EpsPart v = *cluster.map_shared_rank(&xch[buf], r);
             df_add(ruh, rul, v.uh, v.ul);
+            df_add(rbh, rbl, v.bh, v.bl);
             df_add(rqh, rql, v.qh, v.ql);
             rb += v.below;
             ra += v.above;
@@ -363,26 +421,33 @@ __global__ void __launch_bounds__(kThreads) k_solve_eps(const __grid_constant__ 
         below = rb;
         above = ra;
         U = S_low + ((double)ruh + (double)rul);
-        Q = S - ((double)rqh + (double)rql);
+        Q = B_low + ((double)rbh + (double)rbl);
+        Qa = (double)rqh + (double)rql;
     };
 
-    double lam = 0.0, U = 0.0, Q = 0.0;
+    double lam = 0.0, U = 0.0, Q = 0.0, Qa = 0.0;
     int below = 0, above = 0, it = 0;
     bool bad = false;
-    if ((flags & kSegNonfinite) || !isfinite(S)) {
+    float tau = t_up;
+    if (!(flags & kSegNonfinite) && isfinite(S_hist) && S_hist > 0.0) pass(tau, below, above, U, Q, Qa);
+    // S = sum g^2 from the sums of this pass (finer than the histogram's).
+    const double S = Q + Qa;
+    if ((flags & kSegNonfinite) || !isfinite(S_hist) || !isfinite(S) || !isfinite(U)) {
         flags |= kSegNonfinite;
         if (rank == 0 && tid == 0) atomicOr(status, kStNonfinite);
     } else if (S > 0.0) {
         const double eS = eps * S;
-        float tau = t_up;
-        pass(tau, below, above, U, Q);
-        if (!(U > 0.0)) {
-            // Nothing below t_up (only possible for eps = 0): start from the top.
+        if (!(U > 0.0) || !((double)tau * U - Q > eS)) {
+            // Nothing below t_up, or phi(t_up) not above eps S (only possible
+            // for eps = 0 or by rounding): start from the top.
             tau = __int_as_float(0x7F800000);
-            pass(tau, below, above, U, Q);
+            pass(tau, below, above, U, Q, Qa);
         }
         bool conv = false;
-        while (it < kEpsNewtonMax) {
+        // eps = 0 makes phi flat at the root, where Newton's steps are only
+        // weighted means: go straight to the bisection.
+        const int newton_max = eps > 0.0 ? kEpsNewtonMax : 0;
+        while (it < newton_max) {
             // The root of the piece of phi just left of tau.  a < tau1 holds
             // exactly when a < t1 for every float a (tau1 = t1 rounded up).
             const double t1 = (eS + Q) / U;
@@ -392,14 +457,13 @@ __global__ void __launch_bounds__(kThreads) k_solve_eps(const __grid_constant__ 
                 break;
             }
             int b1, a1;
-            double U1, Q1;
-            pass(tau1, b1, a1, U1, Q1);
+            double U1, Q1, Qa1;
+            pass(tau1, b1, a1, U1, Q1, Qa1);
             ++it;
             // No C value between tau and tau1: phi is linear there and t1 is the
             // root (a start left of the root, which only rounding of the bracket
             // could give, moves right and then converges from the right).
-            // Nothing left below tau1 (eps = 0): the previous piece gives it too.
-            if (b1 == below || !(U1 > 0.0)) {
+            if (b1 == below) {
                 conv = true;
                 break;
             }
@@ -408,6 +472,31 @@ __global__ void __launch_bounds__(kThreads) k_solve_eps(const __grid_constant__ 
             above = a1;
             U = U1;
             Q = Q1;
+        }
+        if (!conv) {
+            // Bisection over the fp32 bit patterns of the threshold, keeping
+            // phi(lo) <= eps S < phi(hi) (t_c, or 0, is a valid lo; tau a valid
+            // hi): it ends on the smallest float hi with phi(hi) > eps S, and
+            // the piece of phi left of hi holds the largest root.
+            uint32_t blo = __float_as_uint(sp[s].t_c), bhi = __float_as_uint(tau);
+            while (bhi - blo > 1u && it < kEpsNewtonMax + kEpsBisectMax) {
+                const uint32_t mid = blo + ((bhi - blo) >> 1);
+                const float tm = __uint_as_float(mid);
+                int b1, a1;
+                double U1, Q1, Qa1;
+                pass(tm, b1, a1, U1, Q1, Qa1);
+                ++it;
+                if ((double)tm * U1 - Q1 > eS) {
+                    bhi = mid;
+                    below = b1;
+                    above = a1;
+                    U = U1;
+                    Q = Q1;
+                } else {
+                    blo = mid;
+                }
+            }
+            conv = bhi - blo <= 1u;
         }
         lam = U / (eS + Q);
         // Not converged, or lambda beyond the bound the lists were built for:
@@ -459,19 +548,20 @@ cudaError_t launch_eps_bracket(const Layout& Lo, SegParam* sp, uint32_t* hist, d
     set_launch_error_site("k_eps_hist memset");
     cudaError_t e = cudaMemsetAsync(hist, 0, sizeof(uint32_t) * eps_hist_words(n_seg), st);
     if (e != cudaSuccess) return e;
-    const int n_units = (int)eps_units(n_chunks);
-    const int warps = std::max(1, std::min(n_units, sm_count_eps() * kHistCtasPerSm * kHistWarps));
-    const int per_warp = (n_units + warps - 1) / warps;
-    const int used = (n_units + per_warp - 1) / per_warp;
-    const int blocks = (used + kHistWarps - 1) / kHistWarps;
+    // Every segment gets the same number of CTAs, at most one warp per unit.
+    int max_units = 0;
+    if (Lo.L == 1) {
+        max_units = Lo.cpw * kUnitsPerChunk;
+    } else {
+        max_units = n_chunks * kUnitsPerChunk;   // a bound; CTAs without a unit exit at once
+    }
+    const int want = (sm_count_eps() * kHistCtasPerSm + n_seg - 1) / n_seg;
+    const int gx = std::max(1, std::min(want, (max_units + kHistWarps - 1) / kHistWarps));
     {
         set_launch_error_site("k_eps_hist launch");
-        const size_t smem = sizeof(uint32_t) * kHistWarps * kHistBins;
-        e = cudaFuncSetAttribute(k_eps_hist, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
         // A plain launch: its predecessor in the stream is the memset.
         TraceScope ts(kKEpsHist, st);
-        k_eps_hist<<<blocks, kHistWarps * 32, smem, st>>>(Lo, hist, u_sq, n_units, per_warp);
+        k_eps_hist<<<gx * n_seg, kHistWarps * 32, 0, st>>>(Lo, hist, u_sq, gx);
         e = cudaGetLastError();
     }
     if (e != cudaSuccess) return e;

@@ -93,6 +93,7 @@ __device__ __forceinline__ void ordered_offsets(uint32_t packed, uint32_t (*sh)[
 //      fp32 rounding of the right-hand side.
 //   C: !(|g| < t_c) (NaN and Inf land here, so the l1 sum flags them).
 //   s_low: sum of |g| outside C; fp32 pairwise over 16 values, fp64 above.
+//   b_low (Algorithm 2 only): the same for g^2.
 // Lists are written in ascending coordinate order.
 // ---------------------------------------------------------------------------
 template <bool kWithC>
@@ -106,14 +107,15 @@ __device__ void chunk_candidates(const Layout& Lo, int c, const Chunk& ch, float
     const int64_t region = (int64_t)ch.m * Lo.d + ch.lo;
     const uint32_t worker = Lo.worker0 + (uint32_t)ch.m;
     const float pbias = 1.0f + 0x1p-20f;
-    double acc = 0.0;
+    double acc = 0.0, acc2 = 0.0;
+    const bool sq = kWithC && Ls.b_low != nullptr;
     int runP = 0, runC = 0, bufP = 0, bufC = 0;
 
     for (int64_t qb = q0; qb < q1; qb += (int64_t)kThreads * kGroupsPerThread) {
         float v[kGroupsPerThread][4];
         uint4 w[kGroupsPerThread];
         uint32_t pm = 0, cm = 0;
-        float s4[kGroupsPerThread];
+        float s4[kGroupsPerThread], q4[kGroupsPerThread];
 #pragma unroll
         for (int j = 0; j < kGroupsPerThread; ++j) {
             const int64_t q = qb + (int64_t)j * kThreads + tid;
@@ -135,6 +137,7 @@ __device__ void chunk_candidates(const Layout& Lo, int c, const Chunk& ch, float
                 need = need || (vs && a > 0.0f);
             }
             s4[j] = (m4[0] + m4[1]) + (m4[2] + m4[3]);
+            q4[j] = (m4[0] * m4[0] + m4[1] * m4[1]) + (m4[2] * m4[2] + m4[3] * m4[3]);
             w[j] = make_uint4(0, 0, 0, 0);
             if (build_p && need) {
                 w[j] = group_words(Lo.seed, Lo.step, worker, q);
@@ -147,6 +150,7 @@ __device__ void chunk_candidates(const Layout& Lo, int c, const Chunk& ch, float
             }
         }
         acc += (double)((s4[0] + s4[1]) + (s4[2] + s4[3]));
+        if (sq) acc2 += (double)((q4[0] + q4[1]) + (q4[2] + q4[3]));
 
         if (build_p) {
             uint32_t packed = 0;
@@ -187,7 +191,9 @@ __device__ void chunk_candidates(const Layout& Lo, int c, const Chunk& ch, float
         }
     }
     const double tot = block_sum(acc, shd);
+    const double tot2 = sq ? block_sum(acc2, shd) : 0.0;
     if (tid == 0) {
+        if (sq) Ls.b_low[c] = tot2;
         if (build_p) Ls.p_cnt[c] = runP;
         if (kWithC) {
             Ls.c_cnt[c] = runC;

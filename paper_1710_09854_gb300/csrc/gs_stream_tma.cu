@@ -171,8 +171,9 @@ struct ChunkWalk {
     }
 };
 
-// kDtype 0: fp32 rows of 32; 1: bf16 rows of 64.
-template <int kDtype>
+// kDtype 0: fp32 rows of 32; 1: bf16 rows of 64.  kSq: also the sum of g^2
+// outside C (Algorithm 2's solve), the same way as s_low.
+template <int kDtype, bool kSq>
 __global__ void __launch_bounds__(kTmaThreads, 2)
     k_stream_tma(const __grid_constant__ CUtensorMap map, const __grid_constant__ StreamArgs A) {
     grid_dep_wait();
@@ -252,6 +253,7 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
         const int span = (int)((r_end - r_first) * kInner);   // coordinates the chunk's buffers cover
         const PhiloxStream ph(Lo, Lo.worker0 + (uint32_t)cw.m);
         float acc_hi = 0.0f, acc_lo = 0.0f;
+        float sq_hi = 0.0f, sq_lo = 0.0f;
         int runP = 0, runC = 0;
         for (int buf_off = 0; buf_off < span; buf_off += kBufCoords) {
             // live stays warp-uniform: the refill below is a warp-wide step.
@@ -268,16 +270,17 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
             const unsigned char* rp = my_buf + slot * kBufBytes + brow * kRowBytes;
             const int rel = buf_off + lane_off - lead;      // chunk-relative index of coordinate 0
             uint32_t pm = 0, cm = 0;
-            float s32 = 0.0f;
+            float s32 = 0.0f, q32 = 0.0f;
             if (live && rel < len && rel + kLaneCoords > 0) {
                 const uint32_t q0 = (uint32_t)((lo + rel) >> 2);   // worker-local group of coordinate 0
                 if (rel >= 0 && rel + kLaneCoords <= len) {
                     // All 32 coordinates belong to the chunk: one group of 4 at a time.
-                    float s4[8];
+                    float s4[8], q4[8];
 #pragma unroll
                     for (int j = 0; j < 8; ++j) {
                         const float4 a = stage_group<kDtype>(rp, first_chunk, sw, j);
                         s4[j] = (a.x + a.y) + (a.z + a.w);
+                        if (kSq) q4[j] = (a.x * a.x + a.y * a.y) + (a.z * a.z + a.w * a.w);
                         if (build_p) {
                             const uint4 w = ph.words(q0 + j);
                             pm = shl_in(pm, fmaf(nlam, a.x, __fsub_rn(unit_plus_one(w.x), pbias)));
@@ -288,6 +291,7 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
                     }
                     pm = __brev(pm);   // coordinate k at bit k
                     s32 = ((s4[0] + s4[1]) + (s4[2] + s4[3])) + ((s4[4] + s4[5]) + (s4[6] + s4[7]));
+                    if (kSq) q32 = ((q4[0] + q4[1]) + (q4[2] + q4[3])) + ((q4[4] + q4[5]) + (q4[6] + q4[7]));
                     if (!(s32 < t_c)) {
                         // Some |g| may reach t_c (or be non-finite): split exactly.
 #pragma unroll
@@ -301,12 +305,15 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
                                 m4[k] = in_c ? 0.0f : a;
                             }
                             s4[j] = (m4[0] + m4[1]) + (m4[2] + m4[3]);
+                            if (kSq) q4[j] = (m4[0] * m4[0] + m4[1] * m4[1]) + (m4[2] * m4[2] + m4[3] * m4[3]);
                         }
                         s32 = ((s4[0] + s4[1]) + (s4[2] + s4[3])) + ((s4[4] + s4[5]) + (s4[6] + s4[7]));
+                        if (kSq)
+                            q32 = ((q4[0] + q4[1]) + (q4[2] + q4[3])) + ((q4[4] + q4[5]) + (q4[6] + q4[7]));
                     }
                 } else {
                     // The lane straddles an edge of the chunk: test each coordinate.
-                    float s4[8];
+                    float s4[8], q4[8];
 #pragma unroll
                     for (int j = 0; j < 8; ++j) {
                         const uint4 w = build_p ? ph.words(q0 + j) : make_uint4(0, 0, 0, 0);
@@ -324,11 +331,14 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
                                 pm |= 1u << e;
                         }
                         s4[j] = (m4[0] + m4[1]) + (m4[2] + m4[3]);
+                        if (kSq) q4[j] = (m4[0] * m4[0] + m4[1] * m4[1]) + (m4[2] * m4[2] + m4[3] * m4[3]);
                     }
                     s32 = ((s4[0] + s4[1]) + (s4[2] + s4[3])) + ((s4[4] + s4[5]) + (s4[6] + s4[7]));
+                    if (kSq) q32 = ((q4[0] + q4[1]) + (q4[2] + q4[3])) + ((q4[4] + q4[5]) + (q4[6] + q4[7]));
                 }
             }
             two_sum_add(acc_hi, acc_lo, s32);
+            if (kSq) two_sum_add(sq_hi, sq_lo, q32);
 
             // Order the buffer's candidates by a lane scan.
             const uint32_t packed = (uint32_t)__popc(pm) | ((uint32_t)__popc(cm) << 16);
@@ -376,9 +386,15 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
             const float oh = __shfl_xor_sync(0xFFFFFFFFu, acc_hi, o);
             const float ol = __shfl_xor_sync(0xFFFFFFFFu, acc_lo, o);
             df_add(acc_hi, acc_lo, oh, ol);
+            if (kSq) {
+                const float qh = __shfl_xor_sync(0xFFFFFFFFu, sq_hi, o);
+                const float ql = __shfl_xor_sync(0xFFFFFFFFu, sq_lo, o);
+                df_add(sq_hi, sq_lo, qh, ql);
+            }
         }
         if (lane == 0) {
             A.Ls.s_low[c] = (double)acc_hi + (double)acc_lo;
+            if (kSq) A.Ls.b_low[c] = (double)sq_hi + (double)sq_lo;
             A.Ls.c_cnt[c] = runC;
             if (A.Ls.p_cnt) A.Ls.p_cnt[c] = runP;
         }
@@ -474,23 +490,21 @@ cudaError_t launch_stream_tma(const Layout& Lo, const SegParam* sp, const Lists&
     const int grid = std::min((n_chunks + kCW - 1) / kCW, 2 * sm_count_tma());
     cudaError_t e;
     TraceScope ts(kKStreamTma, st);
+    void (*kern)(const CUtensorMap, const StreamArgs);
+    size_t smem;
     if (Lo.dtype == 0) {
-        const size_t smem = tma_smem_bytes<0>();
-        set_launch_error_site("k_stream_tma<fp32> shared-memory attribute");
-        e = cudaFuncSetAttribute(k_stream_tma<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        set_launch_error_site("k_stream_tma<fp32> launch");
-        e = launch_dep(k_stream_tma<0>, dim3(grid), dim3(kTmaThreads), smem, st, map, A);
-        if (e != cudaSuccess) return e;
+        kern = Ls.b_low ? k_stream_tma<0, true> : k_stream_tma<0, false>;
+        smem = tma_smem_bytes<0>();
     } else {
-        const size_t smem = tma_smem_bytes<1>();
-        set_launch_error_site("k_stream_tma<bf16> shared-memory attribute");
-        e = cudaFuncSetAttribute(k_stream_tma<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-        if (e != cudaSuccess) return e;
-        set_launch_error_site("k_stream_tma<bf16> launch");
-        e = launch_dep(k_stream_tma<1>, dim3(grid), dim3(kTmaThreads), smem, st, map, A);
-        if (e != cudaSuccess) return e;
+        kern = Ls.b_low ? k_stream_tma<1, true> : k_stream_tma<1, false>;
+        smem = tma_smem_bytes<1>();
     }
+    set_launch_error_site("k_stream_tma shared-memory attribute");
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    set_launch_error_site(Lo.dtype == 0 ? "k_stream_tma<fp32> launch" : "k_stream_tma<bf16> launch");
+    e = launch_dep(kern, dim3(grid), dim3(kTmaThreads), smem, st, map, A);
+    if (e != cudaSuccess) return e;
     *used = true;
     return cudaGetLastError();
 }

@@ -142,9 +142,16 @@ def test_eps_degenerate_inputs(gs):
     assert n == nz.size
     np.testing.assert_array_equal(idx[0, :n].cpu().numpy(), nz)
     np.testing.assert_allclose(val[0, :n].cpu().numpy(), g[nz], rtol=1e-6)
+    # tiny budgets (every coordinate a candidate; the solve may finish by bisection)
+    p = torch.empty(d, dtype=torch.float32, device="cuda")
+    for e in (0.0, 1e-9, 2.0 ** -20, 2.0 ** -19):
+        info = gs.info_tensor(1)
+        gs.gs_probabilities_eps(_dev(g), e, p, info)
+        assert gs.gs_sync_status() == gs.GS_OK
+        ref = _check_p(p.cpu().numpy(), g, e)
+        assert gs.decode_info(info)[0]["lambda"] == pytest.approx(ref["lambda"], rel=1e-6)
     # equal magnitudes: p = 1 / (1 + eps) everywhere
     h = (0.5 * np.where(np.arange(d) % 3 == 0, -1.0, 1.0)).astype(np.float32)
-    p = torch.empty(d, dtype=torch.float32, device="cuda")
     gs.gs_probabilities_eps(_dev(h), 3.0, p)
     assert gs.gs_sync_status() == gs.GS_OK
     np.testing.assert_allclose(p.cpu().numpy(), 0.25, rtol=1e-6)
