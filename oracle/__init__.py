@@ -56,6 +56,8 @@ def lib():
                                              ctypes.c_void_p, ctypes.c_void_p, P(ctypes.c_int64), ctypes.c_void_p]
         L.gso_aggregate.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int, ctypes.c_int64,
                                     ctypes.c_void_p]
+        L.gso_average.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int, ctypes.c_int64,
+                                  ctypes.c_void_p]
         L.gso_hybrid_encode.argtypes = [ctypes.c_void_p, ctypes.c_int64, ctypes.c_double, ctypes.c_void_p,
                                         ctypes.c_void_p, ctypes.c_int64, ctypes.c_void_p, ctypes.c_void_p,
                                         P(ctypes.c_int64), ctypes.c_void_p, P(ctypes.c_int64), P(ctypes.c_double)]
@@ -73,7 +75,7 @@ def lib():
                                        ctypes.c_uint32, ctypes.c_uint32, ctypes.c_int64, ctypes.c_void_p,
                                        ctypes.c_void_p, P(ctypes.c_int64), P(Info)]
         for f in ("gso_closed_form_lambda", "gso_probabilities_eps", "gso_sparsify_eps", "gso_greedy_lambda", "gso_greedy_pvector", "gso_probabilities", "gso_sparsify",
-                  "gso_segmented_sparsify", "gso_aggregate", "gso_hybrid_encode", "gso_hybrid_decode"):
+                  "gso_segmented_sparsify", "gso_aggregate", "gso_average", "gso_hybrid_encode", "gso_hybrid_decode"):
             getattr(L, f).restype = ctypes.c_int
         _LIB = L
     return _LIB
@@ -163,6 +165,20 @@ def aggregate(idx_list, val_list, d):
     nn = np.array([x.size for x in idxs], dtype=np.int64)
     out = np.empty(d, dtype=np.float32)
     _check(lib().gso_aggregate(ip, vp, nn.ctypes.data, M, d, out.ctypes.data))
+    return out
+
+
+def average(idx_list, val_list, d):
+    """Algorithm 1 step 6: v = (1/M) sum_m Q(g^m) (fp32 sum in worker order,
+    then one fp32 division by M)."""
+    M = len(idx_list)
+    idxs = [np.ascontiguousarray(x, dtype=np.int32) for x in idx_list]
+    vals = [np.ascontiguousarray(x, dtype=np.float32) for x in val_list]
+    ip = (ctypes.c_void_p * M)(*[x.ctypes.data for x in idxs])
+    vp = (ctypes.c_void_p * M)(*[x.ctypes.data for x in vals])
+    nn = np.array([x.size for x in idxs], dtype=np.int64)
+    out = np.empty(d, dtype=np.float32)
+    _check(lib().gso_average(ip, vp, nn.ctypes.data, M, d, out.ctypes.data))
     return out
 
 

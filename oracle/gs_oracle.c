@@ -16,8 +16,9 @@
  *   Algorithm 3    greedy rescaling of the active set {i : p_i != 1} until
  *                  the scaling factor c drops to <= 1 (or `iters` rescalings
  *                  have been made).
- *   Algorithm 1    step 6: the M sparse vectors are summed (the 1/M of the
- *                  average is left to the caller).
+ *   Algorithm 1    step 6: the M sparse vectors are summed (gso_aggregate;
+ *                  gso_average also divides by M); step 7 sparsifies the
+ *                  average again (gso_sparsify on gso_average's output).
  *   Algorithm 2    the closed-form solution of problem (4) for a variance
  *                  budget epsilon: sort the magnitudes, take the smallest k
  *                  satisfying (6), set p by (7).
@@ -337,6 +338,24 @@ GSO_EXPORT int gso_aggregate(const int32_t* const* idx, const float* const* val,
         for (i = 0; i < d; i++) out[i] = out[i] + dense[i];
     }
     free(dense);
+    return GSO_OK;
+}
+
+/* ------------------------------------------------------------------------
+ * Algorithm 1, step 6 as printed: the average v = (1/M) sum_m Q(g^m).  The
+ * sum is gso_aggregate's (fp32, worker order); each coordinate is then divided
+ * by M in fp32 (one correctly rounded division).  Step 7 sparsifies v again,
+ * v = Q(v): that is gso_sparsify applied to this output, with a worker id of
+ * its own for the random stream.
+ * ---------------------------------------------------------------------- */
+GSO_EXPORT int gso_average(const int32_t* const* idx, const float* const* val, const int64_t* nnz, int M, int64_t d,
+                           float* out)
+{
+    int64_t i;
+    const float fm = (float)M;
+    int rc = gso_aggregate(idx, val, nnz, M, d, out);
+    if (rc != GSO_OK) return rc;
+    for (i = 0; i < d; i++) out[i] = out[i] / fm;
     return GSO_OK;
 }
 
