@@ -318,6 +318,7 @@ def run_gpu(args):
             raise RuntimeError(f"device status after the sparsify-only run: {gs.status_string(rc)}")
     hybrid = run_hybrid(gs, g, kappa, w, args, dev, stream, n_bd, hbm) if off is None else None
     vbudget = run_variance_budget(gs, g, w, args, dev, stream, n_bd, hbm) if off is None else None
+    resp = run_resparsify(gs, g, kappa, w, args, dev, stream, n_bd, hbm, ms) if off is None else None
 
     # ---- end to end through the host-buffer entry point
     e2e = None
@@ -339,6 +340,7 @@ def run_gpu(args):
         "sparsify_roofline": sp_only,
         "hybrid_code": hybrid,
         "variance_budget": vbudget,
+        "average_resparsify": resp,
         "kernels": kernels, "kernels_steps": n_bd,
         "nnz_per_step": nnz_total,
         "gpu_launches": launches,
@@ -454,6 +456,50 @@ def run_hybrid(gs, g, kappa, w, args, dev, stream, n_steps, hbm):
             "unit": "GB/s", "n_a": int(a.sum()), "n_b": int(b_.sum()),
             "bits_per_step": {k: round(v) for k, v in bits.items()},
             "bits_per_coordinate": {k: round(v / (M * d), 4) for k, v in bits.items()}}
+
+
+def run_resparsify(gs, g, kappa, w, args, dev, stream, n_steps, hbm, ms_fused):
+    """Algorithm 1 steps 4-7 (gs_sparsify_average_sparsify): the fused
+    sparsify + average, then step 7's Q(v) of the average (kappa_v = kappa,
+    the same iterations, a worker id of its own).  Step 7's own cost is the
+    difference to the fused call's time per step; its algorithmic bytes are one
+    read of v (4d) and the kept pairs of Q(v) written."""
+    import torch
+    M, d = g.shape
+    idx = torch.empty((M, d), dtype=torch.int32, device=dev)
+    val = torch.empty((M, d), dtype=torch.float32, device=dev)
+    nnz = torch.empty(M, dtype=torch.int32, device=dev)
+    v = torch.empty(d, dtype=torch.float32, device=dev)
+    idx_v = torch.empty(d, dtype=torch.int32, device=dev)
+    val_v = torch.empty(d, dtype=torch.float32, device=dev)
+    nnz_v = torch.empty(1, dtype=torch.int32, device=dev)
+    wv = 2 ** 32 - 1
+
+    def call(t):
+        gs.gs_sparsify_average_sparsify(g, kappa, w.iters, w.seed, t, 0, idx, val, nnz, v, kappa, w.iters, wv,
+                                        idx_v, val_v, nnz_v, stream=stream)
+    for t in range(3):
+        call(t)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for t in range(n_steps):
+        call(args.warmup + t)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = max_over_ranks(e0.elapsed_time(e1) / n_steps, dev)
+    rc = gs.gs_sync_status(stream)
+    if rc != gs.GS_OK:
+        raise RuntimeError(f"device status after the step-7 run: {gs.status_string(rc)}")
+    kv = int(nnz_v.item())
+    nz = int((v != 0).sum().item())
+    step7_ms = max(ms - ms_fused, 1e-6)
+    algo = 4 * d + 8 * kv
+    gbs = algo / (step7_ms / 1e3) / 1e9
+    return {"api": "gs_sparsify_average_sparsify", "steps": n_steps, "ms_per_step": round(ms, 4),
+            "step7_ms": round(step7_ms, 4), "kappa_v": kappa, "nnz_average": nz, "nnz_resparsified": kv,
+            "step7_algorithmic_bytes": algo, "step7_achieved": round(gbs, 1), "peak": hbm,
+            "step7_frac": round(gbs / hbm, 4), "unit": "GB/s"}
 
 
 VARIANCE_BUDGETS = (30.0, 1.0)   # about 1.2% and 21% density on the Student-t gradients

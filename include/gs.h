@@ -127,6 +127,26 @@ gs_status gs_batched_sparsify(const void* g, int dtype, int M, int64_t d, double
                               gs_info* info, void* stream);
 
 /*
+ * Algorithm 1, steps 4-7 in one call: every worker's Q(g^m) as in
+ * gs_sparsify_aggregate, their average v = (1/M) sum_m Q(g^m) (step 6: the
+ * fp32 sum in worker order, then one correctly rounded fp32 division by M per
+ * coordinate), and step 7's optional re-sparsification v <- Q(v) with its own
+ * density budget kappa_v and iters_v, drawn from the Philox stream of worker
+ * id worker_v (give it an id no worker uses, or the two stages share draws).
+ *   v                  device, d fp32: the average (written)
+ *   idx_v, val_v, nnz_v  device: Q(v) as ascending (index, value) pairs,
+ *                      capacity d, and its count
+ *   info               device, M + 1 gs_info records (the workers', then v's),
+ *                      or NULL
+ * Other arguments as in gs_sparsify_aggregate (1 <= M <= 512).
+ */
+gs_status gs_sparsify_average_sparsify(const void* g, int dtype, int M, int64_t d, double kappa, int iters,
+                                       uint64_t seed, uint32_t step, uint32_t worker0, int32_t* idx, float* val,
+                                       int32_t* nnz, int64_t cap, float* v, double kappa_v, int iters_v,
+                                       uint32_t worker_v, int32_t* idx_v, float* val_v, int32_t* nnz_v,
+                                       gs_info* info, void* stream);
+
+/*
  * gs_batched_sparsify with the hybrid code of section 3.3 (eqs. 9-10) in
  * place of the plain (index, value) lists: the kept coordinates with p_i = 1
  * (the capped set S_k) go to Q_A as (index, value g_i); every other kept

@@ -24,7 +24,7 @@ GS_OPT_FORCE_EXACT_SOLVE, GS_OPT_SAMPLE_SIZE, GS_OPT_KERNEL_TIMING, GS_OPT_STREA
 # Symbols include/gs.h declares (checked by the tests).
 EXPORTS = ("gs_status_string", "gs_last_error", "gs_version", "gs_sync_status", "gs_probabilities", "gs_probabilities_ex",
            "gs_sparsify", "gs_batched_sparsify", "gs_batched_sparsify_hybrid", "gs_probabilities_eps", "gs_batched_sparsify_eps", "gs_segmented_sparsify", "gs_sparse_aggregate",
-           "gs_sparsify_aggregate", "gs_sparsify_noalloc", "gs_pipeline_host", "gs_random_words", "gs_set_option", "gs_kernel_count", "gs_kernel_name",
+           "gs_sparsify_aggregate", "gs_sparsify_average_sparsify", "gs_sparsify_noalloc", "gs_pipeline_host", "gs_random_words", "gs_set_option", "gs_kernel_count", "gs_kernel_name",
            "gs_kernel_times")
 
 
@@ -70,6 +70,8 @@ def lib():
                                       i32),
             "gs_sparse_aggregate": ([vp, vp, vp, i32, i64, vp, vp], i32),
             "gs_sparsify_aggregate": ([vp, i32, i32, i64, dbl, i32, u64, u32, u32, vp, vp, vp, i64, vp, vp, vp], i32),
+            "gs_sparsify_average_sparsify": ([vp, i32, i32, i64, dbl, i32, u64, u32, u32, vp, vp, vp, i64, vp, dbl,
+                                              i32, u32, vp, vp, vp, vp, vp], i32),
             "gs_sparsify_noalloc": ([vp, i64, dbl, i32, u64, u32, u32, vp, vp, vp, vp, vp, vp], i32),
             "gs_pipeline_host": ([vp, i32, i32, i64, dbl, i32, u64, u32, u32, vp, vp, vp, vp, i64, vp, vp, vp, vp],
                                  i32),
@@ -313,6 +315,28 @@ def gs_sparsify_aggregate(g, kappa, iters, seed, step, worker0, idx, val, nnz, o
                                        _ptr(val, "val", (torch.float32,)), _ptr(nnz, "nnz", (torch.int32,)), cap,
                                        _ptr(info, "info"), _ptr(out, "out", (torch.float32,)), _stream(stream)),
            "gs_sparsify_aggregate")
+
+
+def gs_sparsify_average_sparsify(g, kappa, iters, seed, step, worker0, idx, val, nnz, v, kappa_v, iters_v,
+                                 worker_v, idx_v, val_v, nnz_v, info=None, stream=None):
+    """Algorithm 1 steps 4-7: Q(g^m) of g (M, d) into idx / val / nnz, their
+    average into v (d,), and Q(v) (density kappa_v, iters_v rescalings, worker
+    id worker_v) into idx_v / val_v (d,) and nnz_v (1,)."""
+    import torch
+    M, d = g.shape
+    cap = idx.shape[1]
+    if idx.shape[0] != M or tuple(val.shape) != tuple(idx.shape) or nnz.numel() != M or v.numel() != d:
+        raise ValueError("idx / val must be (M, cap), nnz (M,), v (d,)")
+    if idx_v.numel() < d or val_v.numel() < d or nnz_v.numel() != 1:
+        raise ValueError("idx_v / val_v need capacity d and nnz_v one entry")
+    _check(lib().gs_sparsify_average_sparsify(_ptr(g, "g"), _g_dtype(g), M, d, float(kappa), int(iters), int(seed),
+                                              int(step), int(worker0), _ptr(idx, "idx", (torch.int32,)),
+                                              _ptr(val, "val", (torch.float32,)), _ptr(nnz, "nnz", (torch.int32,)),
+                                              cap, _ptr(v, "v", (torch.float32,)), float(kappa_v), int(iters_v),
+                                              int(worker_v), _ptr(idx_v, "idx_v", (torch.int32,)),
+                                              _ptr(val_v, "val_v", (torch.float32,)),
+                                              _ptr(nnz_v, "nnz_v", (torch.int32,)), _ptr(info, "info"),
+                                              _stream(stream)), "gs_sparsify_average_sparsify")
 
 
 def gs_pipeline_host(g_host, kappa, iters, seed, step, worker0, g_dev, idx, val, nnz, out, out_host, nnz_host,

@@ -161,7 +161,7 @@ void carve(Arena& a, Workspace& w, int n_seg, int n_chunks, int64_t n, bool buil
 gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off, int L, double kappa, int iters,
               uint64_t seed, uint32_t step, uint32_t worker0, int32_t* idx, float* val, int32_t* nnz, int64_t cap,
               gs_info* info, float* p, cudaStream_t st, float* agg_out = nullptr, const HybridOut* hy = nullptr,
-              double eps = -1.0) {
+              double eps = -1.0, bool average = false) {
     const bool prob = p != nullptr;
     const bool alg2 = eps >= 0.0;
     if (!g || M < 1 || d < 1 || d >= kMaxD) return GS_ERR_INVALID_ARG;
@@ -253,7 +253,7 @@ gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off
     if (e == cudaSuccess) {
         if (prob) e = launch_prob(Lo, w.sp, p, st);
         else e = launch_compact(Lo, w.sp, w.ls, n_chunks, idx, val, hy ? w.nnz : nnz, cap, s->status, st, agg_out,
-                                hy);
+                                hy, average);
     }
     cudaError_t ef = cudaFreeAsync(mem, st);
     if (e != cudaSuccess) return cuda_fail(launch_error_site(), e);
@@ -506,6 +506,24 @@ gs_status gs_sparsify_aggregate(const void* g, int dtype, int M, int64_t d, doub
     if (!out || M < 1 || M > kMaxAggM) return GS_ERR_INVALID_ARG;
     return run(g, dtype, M, d, nullptr, 1, kappa, iters, seed, step, worker0, idx, val, nnz, cap, info, nullptr,
                static_cast<cudaStream_t>(stream), out);
+}
+
+gs_status gs_sparsify_average_sparsify(const void* g, int dtype, int M, int64_t d, double kappa, int iters,
+                                       uint64_t seed, uint32_t step, uint32_t worker0, int32_t* idx, float* val,
+                                       int32_t* nnz, int64_t cap, float* v, double kappa_v, int iters_v,
+                                       uint32_t worker_v, int32_t* idx_v, float* val_v, int32_t* nnz_v,
+                                       gs_info* info, void* stream) {
+    if (!v || !idx_v || !val_v || !nnz_v || M < 1 || M > kMaxAggM) return GS_ERR_INVALID_ARG;
+    if (bad_kappa(kappa_v) || iters_v < 0) return GS_ERR_INVALID_ARG;
+    if ((reinterpret_cast<uintptr_t>(v) % sizeof(float)) != 0) return GS_ERR_INVALID_ARG;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    // Steps 4-6: the workers' Q(g^m) and their average v.
+    gs_status rc = run(g, dtype, M, d, nullptr, 1, kappa, iters, seed, step, worker0, idx, val, nnz, cap, info,
+                       nullptr, st, v, nullptr, -1.0, true);
+    if (rc != GS_OK) return rc;
+    // Step 7: v = Q(v), drawn from the stream of worker id worker_v.
+    return run(v, GS_DTYPE_F32, 1, d, nullptr, 1, kappa_v, iters_v, seed, step, worker_v, idx_v, val_v, nnz_v, d,
+               info ? info + M : nullptr, nullptr, st);
 }
 
 gs_status gs_batched_sparsify_hybrid(const void* g, int dtype, int M, int64_t d, double kappa, int iters,

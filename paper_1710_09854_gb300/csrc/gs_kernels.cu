@@ -1139,7 +1139,7 @@ __global__ void __launch_bounds__(kSumWarps * 32) k_sum(const __grid_constant__ 
                                                         const __grid_constant__ Lists Ls,
                                                         const int32_t* __restrict__ idx,
                                                         const float* __restrict__ val, int64_t cap,
-                                                        int n_slices, float* out) {
+                                                        int n_slices, float div, float* out) {
     grid_dep_wait();
     __shared__ __align__(16) float tile[kSumWarps][kSlice];
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
@@ -1226,13 +1226,23 @@ __global__ void __launch_bounds__(kSumWarps * 32) k_sum(const __grid_constant__ 
             }
         }
     }
+    // div > 0: the average of Algorithm 1 step 6 (one correctly rounded
+    // division of the worker-order sum), else the sum itself.
     float* dst = out + t0;
     if (tlen == kSlice && (reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
 #pragma unroll
-        for (int i = 0; i < kSlice / 128; ++i)
-            reinterpret_cast<float4*>(dst)[i * 32 + lane] = reinterpret_cast<const float4*>(acc)[i * 32 + lane];
+        for (int i = 0; i < kSlice / 128; ++i) {
+            float4 t = reinterpret_cast<const float4*>(acc)[i * 32 + lane];
+            if (div > 0.0f) {
+                t.x = __fdiv_rn(t.x, div);
+                t.y = __fdiv_rn(t.y, div);
+                t.z = __fdiv_rn(t.z, div);
+                t.w = __fdiv_rn(t.w, div);
+            }
+            reinterpret_cast<float4*>(dst)[i * 32 + lane] = t;
+        }
     } else {
-        for (int i = lane; i < tlen; i += 32) dst[i] = acc[i];
+        for (int i = lane; i < tlen; i += 32) dst[i] = div > 0.0f ? __fdiv_rn(acc[i], div) : acc[i];
     }
 }
 
@@ -1436,7 +1446,7 @@ cudaError_t launch_solve(const Layout& Lo, SegParam* sp, const Lists& Ls, int n_
 
 cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, int32_t* idx,
                            float* val, int32_t* nnz, int64_t cap, int* status, cudaStream_t st, float* sum_out,
-                           const HybridOut* hybrid) {
+                           const HybridOut* hybrid, bool average) {
     const int blocks = (n_chunks + kEmitWarps - 1) / kEmitWarps;
     cudaError_t e;
     {
@@ -1463,7 +1473,8 @@ cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls
     set_launch_error_site("k_sum launch");
     TraceScope ts(kKSum, st);
     return launch_dep(k_sum, dim3((n_slices + kSumWarps - 1) / kSumWarps), dim3(kSumWarps * 32), 0, st, Lo, Ls,
-                      static_cast<const int32_t*>(idx), static_cast<const float*>(val), cap, n_slices, sum_out);
+                      static_cast<const int32_t*>(idx), static_cast<const float*>(val), cap, n_slices,
+                      average ? (float)Lo.M : 0.0f, sum_out);
 }
 
 cudaError_t launch_prob(const Layout& Lo, const SegParam* sp, float* p, cudaStream_t st) {

@@ -85,11 +85,12 @@ struct HybridOut {
 };
 
 // Decide, scan and compact; with sum_out (L == 1 only) also the sparse sum of
-// the M compacted rows into sum_out (d fp32), fused with the compaction; with
-// hybrid (L == 1 only) the hybrid code instead of the plain lists.
+// the M compacted rows into sum_out (d fp32), fused with the compaction (with
+// average, the sum divided by M); with hybrid (L == 1 only) the hybrid code
+// instead of the plain lists.
 cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, int32_t* idx,
                            float* val, int32_t* nnz, int64_t cap, int* status, cudaStream_t st,
-                           float* sum_out = nullptr, const HybridOut* hybrid = nullptr);
+                           float* sum_out = nullptr, const HybridOut* hybrid = nullptr, bool average = false);
 cudaError_t launch_prob(const Layout& Lo, const SegParam* sp, float* p, cudaStream_t st);
 cudaError_t launch_aggregate(const AggArgs& A, int32_t* off, float* out, int* status, cudaStream_t st);
 cudaError_t launch_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t i0, int64_t n, uint32_t* out,

@@ -85,3 +85,17 @@ def test_eps_entry_points_reject_bad_budgets():
         assert L.gs_probabilities_eps(fake, 10, eps, fake, None, None) == gs.GS_ERR_INVALID_ARG
         assert L.gs_batched_sparsify_eps(fake, 0, 1, 10, eps, 1, 0, 0, fake, fake, fake, 10, None,
                                          None) == gs.GS_ERR_INVALID_ARG
+
+
+def test_average_sparsify_rejects_bad_arguments():
+    # Host-side validation: these return before any CUDA call.
+    import paper_1710_09854_gb300 as gs
+    L = gs.lib()
+    fake = 256  # never dereferenced
+    args = lambda M, kv, iv, v: (fake, 0, M, 10, 0.1, 2, 1, 0, 0, fake, fake, fake, 10, v, kv, iv, 7, fake, fake,
+                                 fake, None, None)
+    assert L.gs_sparsify_average_sparsify(*args(0, 0.1, 2, fake)) == gs.GS_ERR_INVALID_ARG
+    assert L.gs_sparsify_average_sparsify(*args(513, 0.1, 2, fake)) == gs.GS_ERR_INVALID_ARG
+    assert L.gs_sparsify_average_sparsify(*args(4, 0.0, 2, fake)) == gs.GS_ERR_INVALID_ARG
+    assert L.gs_sparsify_average_sparsify(*args(4, 0.1, -1, fake)) == gs.GS_ERR_INVALID_ARG
+    assert L.gs_sparsify_average_sparsify(*args(4, 0.1, 2, None)) == gs.GS_ERR_INVALID_ARG
