@@ -319,6 +319,7 @@ def run_gpu(args):
     hybrid = run_hybrid(gs, g, kappa, w, args, dev, stream, n_bd, hbm) if off is None else None
     vbudget = run_variance_budget(gs, g, w, args, dev, stream, n_bd, hbm) if off is None else None
     resp = run_resparsify(gs, g, kappa, w, args, dev, stream, n_bd, hbm, ms) if off is None else None
+    lr = run_lr_sgd(dev, stream) if (off is None and not args.no_lr) else None
 
     # ---- end to end through the host-buffer entry point
     e2e = None
@@ -341,6 +342,7 @@ def run_gpu(args):
         "hybrid_code": hybrid,
         "variance_budget": vbudget,
         "average_resparsify": resp,
+        "lr_sgd": lr,
         "kernels": kernels, "kernels_steps": n_bd,
         "nnz_per_step": nnz_total,
         "gpu_launches": launches,
@@ -500,6 +502,48 @@ def run_resparsify(gs, g, kappa, w, args, dev, stream, n_steps, hbm, ms_fused):
             "step7_ms": round(step7_ms, 4), "kappa_v": kappa, "nnz_average": nz, "nnz_resparsified": kv,
             "step7_algorithmic_bytes": algo, "step7_achieved": round(gbs, 1), "peak": hbm,
             "step7_frac": round(gbs / hbm, 4), "unit": "GB/s"}
+
+
+def run_lr_sgd(dev, stream, passes=30, kappas=(0.1, 0.02)):
+    """The convex experiment of section 5.1 as a training workload around the
+    sparsifier (a reported check): l2-regularised logistic regression on the
+    section's synthetic data (N = 1024, d = 2048, C1 = 0.6, C2 = 4^-2,
+    lam2 = 1/(10 N)), M = 4 workers with minibatches of 8, step size
+    eta0 / ((1 + t/T0) var) with eta0 = M B / L (L: the largest sample loss's
+    smoothness) and T0 = five data passes.  The dense
+    baseline against the sparsified SGD at each density kappa (Algorithm 3,
+    two iterations): suboptimality f(w) - f* after 5, 10, 20 and all passes,
+    the run's var, the share of coordinates sent and the time per step."""
+    import time
+    import torch
+    import workloads
+    from paper_1710_09854_gb300 import logreg
+    N, d, M, B = 1024, 2048, 4, 8
+    lam2 = 1.0 / (10 * N)
+    Xh, yh = workloads.gen_sec51(N, d, 0.6, 1.0 / 16.0, seed=0)
+    f_star, _ = logreg.optimum(Xh, yh, lam2)
+    per_pass = N // (M * B)
+    steps = passes * per_pass
+    bh = workloads.minibatches(steps, M, B, N, seed=0)
+    X, y, batches = (torch.from_numpy(a).to(dev) for a in (Xh, yh, bh))
+    eta0, T0 = M * B / logreg.smoothness(Xh, lam2), 5.0 * per_pass
+    runs = {}
+    for kappa in (None,) + tuple(kappas):
+        name = "dense" if kappa is None else f"kappa_{kappa}"
+        res = logreg.train(X, y, batches, lam2, eta0, T0, kappa=kappa, iters=2, seed=1, log_every=per_pass,
+                           stream=stream)
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        logreg.train(X, y, batches, lam2, eta0, T0, kappa=kappa, iters=2, seed=1, log_every=None, stream=stream)
+        torch.cuda.synchronize()
+        ms = (time.perf_counter() - t0) * 1e3 / steps
+        curve = dict(res["curve"])
+        runs[name] = {"kappa": kappa, "var": round(res["var"], 4),
+                      "sent_fraction": round(res["kept_total"] / (steps * M * d), 5),
+                      "subopt": {str(p): curve[p * per_pass] - f_star for p in (5, 10, 20, passes)},
+                      "ms_per_step": round(ms, 4)}
+    return {"data": "section 5.1 synthetic, N=1024, d=2048, C1=0.6, C2=1/16, lam2=1/(10N)", "M": M, "B": B,
+            "passes": passes, "f_star": f_star, "f_0": float(dict(res["curve"])[0]), "runs": runs}
 
 
 VARIANCE_BUDGETS = (30.0, 1.0)   # about 1.2% and 21% density on the Student-t gradients
@@ -685,6 +729,7 @@ def main(argv=None):
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-lr", action="store_true", help="skip the section 5.1 training-loop report")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     args = ap.parse_args(argv)
     if args.warmup < 3:

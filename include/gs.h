@@ -188,6 +188,46 @@ gs_status gs_batched_sparsify_eps(const void* g, int dtype, int M, int64_t d, do
                                   void* stream);
 
 /*
+ * The training loop of the convex experiments of section 5.1 (l2-regularised
+ * logistic regression, eq. (14), by SGD over M simulated workers).  These are
+ * the loop's own kernels around the sparsifier, not part of it:
+ *
+ * gs_logreg_grad: worker m's minibatch gradient
+ *   G[m] = (1/B) sum_j grad_n_j + 2 lam2 w,
+ *   grad_n = -b_n a_n sigma(-b_n a_n^T w) / ln 2 (eq. (14) uses log2),
+ * over the rows n_j = batch[m * B + j] of X, and gsq[m] = ||G[m]||^2.
+ *   X      device, N x d fp32 row-major (rows a_n);  y  device, N fp32 labels in {-1, +1}
+ *   w      device, d fp32;  batch  device, M x B int32 row indices
+ *   G      device, M x d fp32 (written);  gsq  device, M fp32 (written)
+ *   1 <= B <= 64.  An index outside [0, N) is skipped and recorded as
+ *   GS_ERR_INVALID_ARG in the status word.
+ */
+gs_status gs_logreg_grad(const float* X, const float* y, int N, int d, const float* w, const int32_t* batch, int M,
+                         int B, float lam2, float* G, float* gsq, void* stream);
+
+/* margins[n] = b_n a_n^T w for all N rows (the objective of eq. (14) is
+ * mean(log2(1 + exp(-margins))) + lam2 ||w||^2).  margins: device, N fp32. */
+gs_status gs_logreg_margins(const float* X, const float* y, int N, int d, const float* w, float* margins,
+                            void* stream);
+
+/* out[m] = sum of val[m * cap + e]^2 over e < min(nnz[m], cap): ||Q(g^m)||^2
+ * from the plain lists.  All device pointers. */
+gs_status gs_row_sq_norms(const float* val, const int32_t* nnz, int M, int64_t cap, float* out, void* stream);
+
+/* v = sum of the M rows of G (M x d, device), in row order: the dense
+ * (unsparsified) aggregate. */
+gs_status gs_sum_rows(const float* G, int M, int64_t d, float* v, void* stream);
+
+/* One SGD step of section 5.1: w -= eta_t * scale * v with the step size
+ * divided by the variance factor, eta_t = eta0 / ((1 + t / T0) var_t),
+ * var_t = sum_m qsq[m] / sum_m gsq[m] (= ||Q(g)||^2 / ||g||^2 summed over
+ * workers; pass qsq = gsq for the unsparsified baseline).  log (device, 2
+ * floats, or NULL) receives (eta_t, var_t).  w, v, qsq, gsq are device
+ * pointers; T0 > 0, t >= 0. */
+gs_status gs_sgd_step(float* w, const float* v, int64_t d, float scale, float eta0, float T0, int t, const float* qsq,
+                      const float* gsq, int M, float* log, void* stream);
+
+/*
  * Layer-wise sparsification (section 5.2: each layer is sparsified on its
  * own).  Each worker's vector is cut into L segments by the HOST array
  * seg_offsets[0..L] (0 = seg_offsets[0] < ... < seg_offsets[L] = d); every

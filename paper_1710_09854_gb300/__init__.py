@@ -24,7 +24,8 @@ GS_OPT_FORCE_EXACT_SOLVE, GS_OPT_SAMPLE_SIZE, GS_OPT_KERNEL_TIMING, GS_OPT_STREA
 # Symbols include/gs.h declares (checked by the tests).
 EXPORTS = ("gs_status_string", "gs_last_error", "gs_version", "gs_sync_status", "gs_probabilities", "gs_probabilities_ex",
            "gs_sparsify", "gs_batched_sparsify", "gs_batched_sparsify_hybrid", "gs_probabilities_eps", "gs_batched_sparsify_eps", "gs_segmented_sparsify", "gs_sparse_aggregate",
-           "gs_sparsify_aggregate", "gs_sparsify_average_sparsify", "gs_sparsify_noalloc", "gs_pipeline_host", "gs_random_words", "gs_set_option", "gs_kernel_count", "gs_kernel_name",
+           "gs_sparsify_aggregate", "gs_sparsify_average_sparsify", "gs_sparsify_noalloc", "gs_pipeline_host", "gs_logreg_grad", "gs_logreg_margins", "gs_row_sq_norms", "gs_sum_rows", "gs_sgd_step",
+           "gs_random_words", "gs_set_option", "gs_kernel_count", "gs_kernel_name",
            "gs_kernel_times")
 
 
@@ -76,6 +77,12 @@ def lib():
             "gs_pipeline_host": ([vp, i32, i32, i64, dbl, i32, u64, u32, u32, vp, vp, vp, vp, i64, vp, vp, vp, vp],
                                  i32),
             "gs_random_words": ([u64, u32, u32, i64, i64, vp, vp], i32),
+            "gs_logreg_grad": ([vp, vp, i32, i32, vp, vp, i32, i32, ctypes.c_float, vp, vp, vp], i32),
+            "gs_logreg_margins": ([vp, vp, i32, i32, vp, vp, vp], i32),
+            "gs_row_sq_norms": ([vp, vp, i32, i64, vp, vp], i32),
+            "gs_sum_rows": ([vp, i32, i64, vp, vp], i32),
+            "gs_sgd_step": ([vp, vp, i64, ctypes.c_float, ctypes.c_float, ctypes.c_float, i32, vp, vp, i32, vp, vp],
+                            i32),
             "gs_set_option": ([i32, i64], i32),
             "gs_kernel_count": ([], i32),
             "gs_kernel_name": ([i32], ctypes.c_char_p),
@@ -175,6 +182,51 @@ def gs_kernel_times():
     nl = (ctypes.c_int64 * n)()
     _check(lib().gs_kernel_times(ms, nl, n), "gs_kernel_times")
     return {gs_kernel_name(k): (ms[k], nl[k]) for k in range(n)}
+
+
+def gs_logreg_grad(X, y, w, batch, lam2, G, gsq, stream=None):
+    """Minibatch gradients of eq. (14) for M workers: X (N, d), y (N,), w (d,),
+    batch (M, B) int32 row indices; G (M, d) and gsq (M,) are written."""
+    import torch
+    N, d = X.shape
+    M, B = batch.shape
+    if y.numel() != N or w.numel() != d or tuple(G.shape) != (M, d) or gsq.numel() != M:
+        raise ValueError("shapes: X (N, d), y (N,), w (d,), batch (M, B), G (M, d), gsq (M,)")
+    f32 = (torch.float32,)
+    _check(lib().gs_logreg_grad(_ptr(X, "X", f32), _ptr(y, "y", f32), N, d, _ptr(w, "w", f32),
+                                _ptr(batch, "batch", (torch.int32,)), M, B, float(lam2), _ptr(G, "G", f32),
+                                _ptr(gsq, "gsq", f32), _stream(stream)), "gs_logreg_grad")
+
+
+def gs_logreg_margins(X, y, w, margins, stream=None):
+    import torch
+    N, d = X.shape
+    f32 = (torch.float32,)
+    _check(lib().gs_logreg_margins(_ptr(X, "X", f32), _ptr(y, "y", f32), N, d, _ptr(w, "w", f32),
+                                   _ptr(margins, "margins", f32), _stream(stream)), "gs_logreg_margins")
+
+
+def gs_row_sq_norms(val, nnz, out, stream=None):
+    """val (M, cap) fp32, nnz (M,) int32 -> out (M,) = sum of the first nnz[m] values squared."""
+    import torch
+    M, cap = val.shape
+    _check(lib().gs_row_sq_norms(_ptr(val, "val", (torch.float32,)), _ptr(nnz, "nnz", (torch.int32,)), M, cap,
+                                 _ptr(out, "out", (torch.float32,)), _stream(stream)), "gs_row_sq_norms")
+
+
+def gs_sum_rows(G, v, stream=None):
+    import torch
+    M, d = G.shape
+    _check(lib().gs_sum_rows(_ptr(G, "G", (torch.float32,)), M, d, _ptr(v, "v", (torch.float32,)),
+                             _stream(stream)), "gs_sum_rows")
+
+
+def gs_sgd_step(w, v, scale, eta0, T0, t, qsq, gsq, log=None, stream=None):
+    import torch
+    f32 = (torch.float32,)
+    _check(lib().gs_sgd_step(_ptr(w, "w", f32), _ptr(v, "v", f32), w.numel(), float(scale), float(eta0), float(T0),
+                             int(t), _ptr(qsq, "qsq", f32), _ptr(gsq, "gsq", f32), gsq.numel(),
+                             _ptr(log, "log", f32), _stream(stream)), "gs_sgd_step")
 
 
 def gs_random_words(seed, step, worker, i0, out, stream=None):

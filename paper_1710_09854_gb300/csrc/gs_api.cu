@@ -562,6 +562,46 @@ gs_status gs_sparsify_noalloc(const float* g, int64_t d, double kappa, int iters
                        static_cast<cudaStream_t>(stream));
 }
 
+gs_status gs_logreg_grad(const float* X, const float* y, int N, int d, const float* w, const int32_t* batch, int M,
+                         int B, float lam2, float* G, float* gsq, void* stream) {
+    if (!X || !y || !w || !batch || !G || !gsq || N < 1 || d < 1 || M < 1 || B < 1 || B > kMaxLrBatch)
+        return GS_ERR_INVALID_ARG;
+    if (!std::isfinite(lam2) || lam2 < 0.0f) return GS_ERR_INVALID_ARG;
+    DevState* s = nullptr;
+    gs_status rc = device_state(&s);
+    if (rc != GS_OK) return rc;
+    GS_TRY(launch_lr_grad(X, y, N, d, w, batch, M, B, lam2, G, gsq, s->status, static_cast<cudaStream_t>(stream)));
+    return GS_OK;
+}
+
+gs_status gs_logreg_margins(const float* X, const float* y, int N, int d, const float* w, float* margins,
+                            void* stream) {
+    if (!X || !y || !w || !margins || N < 1 || d < 1) return GS_ERR_INVALID_ARG;
+    GS_TRY(launch_lr_margins(X, y, N, d, w, margins, static_cast<cudaStream_t>(stream)));
+    return GS_OK;
+}
+
+gs_status gs_row_sq_norms(const float* val, const int32_t* nnz, int M, int64_t cap, float* out, void* stream) {
+    if (!val || !nnz || !out || M < 1 || cap < 1) return GS_ERR_INVALID_ARG;
+    GS_TRY(launch_row_sq(val, nnz, M, cap, out, static_cast<cudaStream_t>(stream)));
+    return GS_OK;
+}
+
+gs_status gs_sum_rows(const float* G, int M, int64_t d, float* v, void* stream) {
+    if (!G || !v || M < 1 || d < 1) return GS_ERR_INVALID_ARG;
+    GS_TRY(launch_sum_rows(G, M, d, v, static_cast<cudaStream_t>(stream)));
+    return GS_OK;
+}
+
+gs_status gs_sgd_step(float* w, const float* v, int64_t d, float scale, float eta0, float T0, int t, const float* qsq,
+                      const float* gsq, int M, float* log, void* stream) {
+    if (!w || !v || !qsq || !gsq || d < 1 || M < 1 || t < 0 || !(T0 > 0.0f) || !std::isfinite(eta0) ||
+        !std::isfinite(scale))
+        return GS_ERR_INVALID_ARG;
+    GS_TRY(launch_sgd_step(w, v, d, scale, eta0, T0, t, qsq, gsq, M, log, static_cast<cudaStream_t>(stream)));
+    return GS_OK;
+}
+
 gs_status gs_pipeline_host(const void* g_host, int dtype, int M, int64_t d, double kappa, int iters, uint64_t seed,
                            uint32_t step, uint32_t worker0, void* g_dev, int32_t* idx, float* val, int32_t* nnz,
                            int64_t cap, float* out, float* out_host, int32_t* nnz_host, void* stream) {

@@ -108,6 +108,16 @@ cudaError_t launch_eps_bracket(const Layout& Lo, SegParam* sp, uint32_t* hist, d
                                double eps, int take_all, cudaStream_t st);
 cudaError_t launch_solve_eps(const Layout& Lo, SegParam* sp, const Lists& Ls, int n_seg, double eps, int* status,
                              gs_info_dev* info, cudaStream_t st);
+// The training loop of section 5.1 (gs_lr.cu).
+constexpr int kMaxLrBatch = 64;
+cudaError_t launch_lr_grad(const float* X, const float* y, int N, int d, const float* w, const int32_t* batch, int M,
+                           int B, float lam2, float* G, float* gsq, int* status, cudaStream_t st);
+cudaError_t launch_lr_margins(const float* X, const float* y, int N, int d, const float* w, float* out,
+                              cudaStream_t st);
+cudaError_t launch_row_sq(const float* val, const int32_t* nnz, int M, int64_t cap, float* out, cudaStream_t st);
+cudaError_t launch_sum_rows(const float* G, int M, int64_t d, float* v, cudaStream_t st);
+cudaError_t launch_sgd_step(float* w, const float* v, int64_t d, float scale, float eta0, float T0, int t,
+                            const float* qsq, const float* gsq, int M, float* log, cudaStream_t st);
 // The launchers record which step failed; the C ABI reports it.
 void set_launch_error_site(const char* where);
 const char* launch_error_site();

@@ -15,7 +15,8 @@ namespace {
 const char* kNames[kNumKernels] = {"k_bound", "k_stream", "k_solve", "k_emit",
                                    "k_prob",  "k_words",  "k_bucket", "k_tiles",
                                    "k_stream_tma", "k_decide", "k_scan", "k_sum",
-                                   "k_eps_hist", "k_eps_bracket", "k_solve_eps"};
+                                   "k_eps_hist", "k_eps_bracket", "k_solve_eps",
+                                   "k_lr_grad", "k_lr_margins", "k_row_sq", "k_sum_rows", "k_sgd_step"};
 
 struct Pending {
     int k;

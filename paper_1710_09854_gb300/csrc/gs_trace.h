@@ -21,6 +21,11 @@ enum KernelId : int {
     kKEpsHist,
     kKEpsBracket,
     kKSolveEps,
+    kKLrGrad,
+    kKLrMargins,
+    kKRowSq,
+    kKSumRows,
+    kKSgdStep,
     kNumKernels
 };
 

@@ -99,3 +99,19 @@ def test_average_sparsify_rejects_bad_arguments():
     assert L.gs_sparsify_average_sparsify(*args(4, 0.0, 2, fake)) == gs.GS_ERR_INVALID_ARG
     assert L.gs_sparsify_average_sparsify(*args(4, 0.1, -1, fake)) == gs.GS_ERR_INVALID_ARG
     assert L.gs_sparsify_average_sparsify(*args(4, 0.1, 2, None)) == gs.GS_ERR_INVALID_ARG
+
+
+def test_training_loop_entry_points_reject_bad_arguments():
+    # Host-side validation: these return before any CUDA call.
+    import paper_1710_09854_gb300 as gs
+    L = gs.lib()
+    fake = 256  # never dereferenced
+    bad = gs.GS_ERR_INVALID_ARG
+    assert L.gs_logreg_grad(fake, fake, 10, 10, fake, fake, 2, 65, 0.0, fake, fake, None) == bad   # B > 64
+    assert L.gs_logreg_grad(fake, fake, 10, 10, fake, fake, 2, 0, 0.0, fake, fake, None) == bad
+    assert L.gs_logreg_grad(fake, fake, 10, 10, fake, fake, 2, 8, -1.0, fake, fake, None) == bad
+    assert L.gs_logreg_margins(None, fake, 10, 10, fake, fake, None) == bad
+    assert L.gs_row_sq_norms(fake, fake, 0, 10, fake, None) == bad
+    assert L.gs_sum_rows(fake, 2, 0, fake, None) == bad
+    assert L.gs_sgd_step(fake, fake, 10, 1.0, 0.1, 0.0, 0, fake, fake, 2, None, None) == bad       # T0 = 0
+    assert L.gs_sgd_step(fake, fake, 10, 1.0, 0.1, 4.0, -1, fake, fake, 2, None, None) == bad      # t < 0

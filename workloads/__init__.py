@@ -24,6 +24,9 @@ GPU library is measured on:
       0.1% outliers scaled by 100; fp32 and bf16 (round-to-nearest-even from
       the same fp32 values); kappa in {0.001, 0.01, 0.1}, 3 iterations.
 
+Beside them, the training data of the section 5.1 experiment (gen_sec51)
+and the minibatch indices of its SGD runs (minibatches).
+
 Host (numpy) generators serve the CPU tests and reduced sizes; device
 (torch) generators make the full-size inputs quickly on the GPU.  The two use
 different random streams: a parity check always hands the same bytes to both
@@ -191,6 +194,29 @@ def gen_logreg(M, d, B=256, seed0=2, lam2=None):
         r = -b / (1.0 + np.exp(b * (X @ w))) / B
         g[m] = (X.T @ r + 2.0 * lam2 * w).astype(np.float32)
     return g
+
+
+def gen_sec51(N=1024, d=2048, C1=0.6, C2=1.0 / 16.0, seed=0):
+    """The synthetic data set of section 5.1: dense rows xbar_n ~ N(0, I), a
+    magnitude vector Bbar ~ U[0,1]^d whose entries at or below C2 are scaled by
+    C1, rows x_n = xbar_n * Bbar (element-wise), and labels
+    y_n = sign(xbar_n^T wbar) with wbar ~ N(0, I) (a zero sign counts as +1).
+    Returns fp32 X (N x d) and y (N)."""
+    rng = np.random.default_rng(seed)
+    xbar = rng.standard_normal((N, d))
+    Bbar = rng.uniform(0.0, 1.0, d)
+    Bbar = np.where(Bbar <= C2, C1 * Bbar, Bbar)
+    wbar = rng.standard_normal(d)
+    y = np.sign(xbar @ wbar)
+    y[y == 0] = 1.0
+    return (xbar * Bbar).astype(np.float32), y.astype(np.float32)
+
+
+def minibatches(T, M, B, N, seed=0):
+    """Row indices of T steps of M workers' minibatches of B, uniform with
+    replacement (int32, T x M x B)."""
+    rng = np.random.default_rng(seed + 7919)
+    return rng.integers(0, N, size=(T, M, B)).astype(np.int32)
 
 
 # ---------------------------------------------------------------------------
