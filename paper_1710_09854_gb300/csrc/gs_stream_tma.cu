@@ -95,6 +95,17 @@ __device__ __forceinline__ uint32_t shl_in(uint32_t m, float r) {
     return o;
 }
 
+// Keep-candidate test of one coordinate as a sign bit: negative iff
+// 1 + (x >> 9) 2^-23 < fl32(lam_up |g| + 1 + 2^-20), compared as the bit
+// patterns of two positive floats (integer subtraction, no fp32 rounding of
+// the difference).  (x >> 9) 2^-23 <= u = x 2^-32 and the rounding of the
+// right-hand side is below its 2^-20 slack, so every coordinate kept under a
+// lambda <= lam_up passes (NaN and Inf |g| pass too).
+__device__ __forceinline__ float cand_sign(uint32_t x, float lam_up, float a, float pbias) {
+    const uint32_t pf = __float_as_uint(fmaf(lam_up, a, pbias));
+    return __uint_as_float((x >> 9) + 0x3F800000u - pf);
+}
+
 // Coordinate k (0..31) of a lane's 32, read back from its row of the buffer
 // (first_chunk: the lane's first 16-byte chunk; sw: the row's swizzle).
 template <int kDtype>
@@ -230,7 +241,7 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
 #pragma unroll 1
     for (int i = 0; i < kRing; ++i) prefetch();
 
-    // candidate iff u' - 2^-20 - lam_up |g| < 0, u' = (x >> 9) 2^-23 <= u (the sign is exact)
+    // candidate iff 1 + (x >> 9) 2^-23 < fl32(lam_up |g| + 1 + 2^-20) (cand_sign)
     const float pbias = 1.0f + 0x1p-20f;
     // Probability-only calls keep no keep-candidate lists (their pointer is NULL).
     const bool build_p = A.Ls.p_ent != nullptr;
@@ -247,7 +258,7 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
         int64_t lo, hi, flat_lo, r_first, r_end;
         cw.rows(Lo, kInner, flat_lo, r_first, r_end, seg, lo, hi);
         const int c = cw.c;
-        const float nlam = -A.sp[seg].lam_up32, t_c = A.sp[seg].t_c;
+        const float lup = A.sp[seg].lam_up32, t_c = A.sp[seg].t_c;
         const int len = (int)(hi - lo);
         const int lead = (int)(flat_lo - r_first * kInner);   // coordinates of the first row before the chunk
         const int span = (int)((r_end - r_first) * kInner);   // coordinates the chunk's buffers cover
@@ -283,10 +294,10 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
                         if (kSq) q4[j] = (a.x * a.x + a.y * a.y) + (a.z * a.z + a.w * a.w);
                         if (build_p) {
                             const uint4 w = ph.words(q0 + j);
-                            pm = shl_in(pm, fmaf(nlam, a.x, __fsub_rn(unit_plus_one(w.x), pbias)));
-                            pm = shl_in(pm, fmaf(nlam, a.y, __fsub_rn(unit_plus_one(w.y), pbias)));
-                            pm = shl_in(pm, fmaf(nlam, a.z, __fsub_rn(unit_plus_one(w.z), pbias)));
-                            pm = shl_in(pm, fmaf(nlam, a.w, __fsub_rn(unit_plus_one(w.w), pbias)));
+                            pm = shl_in(pm, cand_sign(w.x, lup, a.x, pbias));
+                            pm = shl_in(pm, cand_sign(w.y, lup, a.y, pbias));
+                            pm = shl_in(pm, cand_sign(w.z, lup, a.z, pbias));
+                            pm = shl_in(pm, cand_sign(w.w, lup, a.w, pbias));
                         }
                     }
                     pm = __brev(pm);   // coordinate k at bit k
@@ -327,7 +338,7 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
                             m4[k] = (valid && !in_c) ? a : 0.0f;
                             cm |= in_c ? (1u << e) : 0u;
                             if (build_p && valid &&
-                                shl_in(0u, fmaf(nlam, a, __fsub_rn(unit_plus_one(word_of(w, k)), pbias))) != 0u)
+                                shl_in(0u, cand_sign(word_of(w, k), lup, a, pbias)) != 0u)
                                 pm |= 1u << e;
                         }
                         s4[j] = (m4[0] + m4[1]) + (m4[2] + m4[3]);
