@@ -13,17 +13,17 @@
 //
 //   k_eps_hist     one read of g.  Per segment, a count histogram of |g| over
 //                  2048 bins of its fp32 bit pattern (8 exponent and 3
-//                  mantissa bits: 1/8-octave bins; warp-private copies in
-//                  shared memory, integer atomics) and S in double-float
-//                  partials of 4096 coordinates.
+//                  mantissa bits: 1/8-octave bins; one shared-memory copy per
+//                  CTA, integer atomics) and S in partials of 4096
+//                  coordinates (fma partials of 32 squares, error-free sum).
 //   k_eps_bracket  one CTA per segment.  From the counts alone, bounds of phi
 //                  at every bin edge; the largest edge whose upper bound stays
 //                  below eps S is a certain lower bound t_c of t* (the
 //                  streaming pass's C threshold; lambda_up = 1 / t_c), the
 //                  smallest edge whose lower bound reaches eps S an upper
 //                  bound t_up.
-//   k_stream[_tma] unchanged: C = {|g| >= t_c}, S_low = sum of |g| below t_c,
-//                  and the keep candidates for lambda_up.
+//   k_stream[_tma] C = {|g| >= t_c}, S_low = sum of |g| below t_c, B_low =
+//                  sum of g^2 below t_c, and the keep candidates for lambda_up.
 //   k_solve_eps    Newton's method on phi(t) = eps S from t_up, each step one
 //                  pass over C (everything below t_c is summed in S_low).
 //                  From the right, Newton's steps on a convex piecewise-linear
@@ -106,8 +106,9 @@ __device__ __forceinline__ float hist_batch_bf16(uint32_t* h, const uint4 (&v)[k
     return (s[0] + s[1]) + (s[2] + s[3]);
 }
 
-// gx CTAs per segment (block x: segment x / gx).  The CTAs of a segment share its 4096-coordinate units
-// (one warp per unit at a time) and one shared-memory histogram, added into
+// gx CTAs per segment (block x: segment x / gx).  The CTAs of a segment share
+// its 4096-coordinate units (one warp per unit at a time); each CTA keeps one
+// shared-memory histogram, added into
 // the segment's global histogram at the end (integer atomics: the order does
 // not matter).  Each unit's sum of squares is one fixed computation (lane
 // assignment, fma partials of 32 values, error-free running sum, fixed

@@ -574,6 +574,49 @@ __device__ __forceinline__ double warp0_sum_double(double v, double* sh) {
     return sh[blockDim.x];
 }
 
+// cap_threshold kept out of line in the solve kernels: it is called from
+// several places, and inlining each copy (with its loops) bloats the code the
+// solve's single busy warp has to fetch.
+__device__ __noinline__ float cap_threshold_call(double lam) { return cap_threshold(lam); }
+
+// Exact fallback of k_solve for one segment, by the whole CTA: every sum of
+// Algorithm 3 straight from g, then the segment's P lists rebuilt for the
+// final lambda (sparsify calls only).  Out of line: it almost never runs, and
+// its code (the candidate builder included) would otherwise crowd the
+// instruction cache of the common path.
+__device__ __noinline__ void solve_exact(const Layout& Lo, const Lists& Ls, int m, int64_t lo, int64_t hi, int c0,
+                                         int c1, double budget, int iters, double* shd, double& S, double& lam,
+                                         double& K, double& Su, int& j) {
+    __shared__ float s_acap;
+    double k0;
+    segment_stats(Lo, m, lo, hi, __int_as_float(0x7FC00000), k0, S, shd);
+    lam = S > 0.0 ? budget / S : 0.0;
+    j = 0;
+    K = 0.0;
+    Su = S;
+    if (lam > 0.0) {
+        while (j < iters) {
+            if (threadIdx.x == 0) s_acap = cap_threshold_call(lam);
+            __syncthreads();
+            segment_stats(Lo, m, lo, hi, s_acap, K, Su, shd);
+            const double A = lam * Su;
+            if (A == 0.0) break;
+            const double cc = (budget - K) / A;
+            if (!(cc > 1.0)) break;
+            lam = cc * lam;
+            ++j;
+        }
+        if (threadIdx.x == 0) s_acap = cap_threshold_call(lam);
+        __syncthreads();
+        segment_stats(Lo, m, lo, hi, s_acap, K, Su, shd);
+    }
+    const float up32 = lam > 0.0 ? __double2float_ru(lam) : 0.0f;
+    for (int c = c0; Ls.p_ent != nullptr && c < c1; ++c) {
+        const Chunk ch = decode_chunk(Lo, c);
+        chunk_candidates<false>(Lo, c, ch, up32, 0.0f, Ls, true);
+    }
+}
+
 // Launched with clusters of 1 or kSolveCTAs CTAs per segment (block x / cluster
 // size = segment).  Small C: the cluster's rank 0 solves alone.  Large C: every
 // CTA of the cluster walks a share of the segment's chunks in each pass and the
@@ -699,7 +742,7 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
             s_go = run && iters > 0 ? 1 : 0;
             s_fresh = 1;
             s_j = 0;
-            s_acap = cap_threshold(s_lam);
+            s_acap = cap_threshold_call(s_lam);
             s_K = 0.0;
             s_Su = S0;
         }
@@ -721,7 +764,7 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
                             ++s_j;
                             go = s_j < iters;
                             fresh = 0;
-                            s_acap = cap_threshold(lv);
+                            s_acap = cap_threshold_call(lv);
                         }
                     }
                     s_lam = lv;
@@ -754,7 +797,7 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
         bool ex = force_exact != 0;
         if (isfinite(S0) && !ex && S0 > 0.0) {
             lv = budget / S0;
-            float acap = cap_threshold(lv);
+            float acap = cap_threshold_call(lv);
             bool fresh = false;   // (rh, rl, rk) are the stats at acap
             while (jj < iters) {
                 warp_c_stats(C, acap, rh, rl, rk);
@@ -765,7 +808,7 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
                 if (!(cc > 1.0)) break;
                 lv = cc * lv;
                 ++jj;
-                acap = cap_threshold(lv);
+                acap = cap_threshold_call(lv);
                 fresh = false;
             }
             if (!fresh) warp_c_stats(C, acap, rh, rl, rk);
@@ -792,43 +835,15 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
     }
 
     if (exact && isfinite(S)) {
-        // Exact fallback: every sum straight from g, by this CTA.
         flags |= kSegExact;
-        double k0;
-        segment_stats(Lo, m, lo, hi, __int_as_float(0x7FC00000), k0, S, shd);
-        lam = S > 0.0 ? budget / S : 0.0;
-        j = 0;
-        K = 0.0;
-        Su = S;
-        if (lam > 0.0) {
-            while (j < iters) {
-                if (tid == 0) s_acap = cap_threshold(lam);
-                __syncthreads();
-                segment_stats(Lo, m, lo, hi, s_acap, K, Su, shd);
-                const double A = lam * Su;
-                if (A == 0.0) break;
-                const double cc = (budget - K) / A;
-                if (!(cc > 1.0)) break;
-                lam = cc * lam;
-                ++j;
-            }
-            if (tid == 0) s_acap = cap_threshold(lam);
-            __syncthreads();
-            segment_stats(Lo, m, lo, hi, s_acap, K, Su, shd);
-        }
-        // Rebuild this segment's P lists for the final lambda (sparsify calls only).
-        const float up32 = lam > 0.0 ? __double2float_ru(lam) : 0.0f;
-        for (int c = c0; Ls.p_ent != nullptr && c < c1; ++c) {
-            const Chunk ch = decode_chunk(Lo, c);
-            chunk_candidates<false>(Lo, c, ch, up32, 0.0f, Ls, true);
-        }
+        solve_exact(Lo, Ls, m, lo, hi, c0, c1, budget, iters, shd, S, lam, K, Su, j);
     }
 
     if (tid == 0) {
         SegParam& P = sp[s];
         P.lam = lam;
         P.lam32 = (float)lam;
-        P.a_cap = cap_threshold(lam);
+        P.a_cap = cap_threshold_call(lam);
         P.inv_lam32 = lam > 0.0 ? (float)(1.0 / lam) : 0.0f;
         P.l1 = S;
         P.capped = (long long)K;
