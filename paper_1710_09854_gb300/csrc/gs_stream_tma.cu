@@ -285,24 +285,53 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
             if (live && rel < len && rel + kLaneCoords > 0) {
                 const uint32_t q0 = (uint32_t)((lo + rel) >> 2);   // worker-local group of coordinate 0
                 if (rel >= 0 && rel + kLaneCoords <= len) {
-                    // All 32 coordinates belong to the chunk: one group of 4 at a time.
+                    // All 32 coordinates belong to the chunk: groups of 4 in order.
+                    // Two groups per step (independent Philox chains) pays only in the
+                    // kSq instantiation (303 vs 320 us on 16 x 2^24); the plain one takes
+                    // one group per step (277 vs 287 us).
                     float s4[8], q4[8];
+                    if constexpr (!kSq) {
 #pragma unroll
-                    for (int j = 0; j < 8; ++j) {
+                        for (int j = 0; j < 8; ++j) {
+                            const float4 a = stage_group<kDtype>(rp, first_chunk, sw, j);
+                            s4[j] = (a.x + a.y) + (a.z + a.w);
+                            if (build_p) {
+                                const uint4 w = ph.words(q0 + j);
+                                pm = shl_in(pm, cand_sign(w.x, lup, a.x, pbias));
+                                pm = shl_in(pm, cand_sign(w.y, lup, a.y, pbias));
+                                pm = shl_in(pm, cand_sign(w.z, lup, a.z, pbias));
+                                pm = shl_in(pm, cand_sign(w.w, lup, a.w, pbias));
+                            }
+                        }
+                    } else {
+#pragma unroll
+                    for (int j = 0; j < 8; j += 2) {
                         const float4 a = stage_group<kDtype>(rp, first_chunk, sw, j);
+                        const float4 b = stage_group<kDtype>(rp, first_chunk, sw, j + 1);
                         s4[j] = (a.x + a.y) + (a.z + a.w);
-                        if (kSq) q4[j] = (a.x * a.x + a.y * a.y) + (a.z * a.z + a.w * a.w);
+                        s4[j + 1] = (b.x + b.y) + (b.z + b.w);
+                        if (kSq) {
+                            q4[j] = (a.x * a.x + a.y * a.y) + (a.z * a.z + a.w * a.w);
+                            q4[j + 1] = (b.x * b.x + b.y * b.y) + (b.z * b.z + b.w * b.w);
+                        }
                         if (build_p) {
                             const uint4 w = ph.words(q0 + j);
+                            const uint4 v = ph.words(q0 + j + 1);
                             pm = shl_in(pm, cand_sign(w.x, lup, a.x, pbias));
                             pm = shl_in(pm, cand_sign(w.y, lup, a.y, pbias));
                             pm = shl_in(pm, cand_sign(w.z, lup, a.z, pbias));
                             pm = shl_in(pm, cand_sign(w.w, lup, a.w, pbias));
+                            pm = shl_in(pm, cand_sign(v.x, lup, b.x, pbias));
+                            pm = shl_in(pm, cand_sign(v.y, lup, b.y, pbias));
+                            pm = shl_in(pm, cand_sign(v.z, lup, b.z, pbias));
+                            pm = shl_in(pm, cand_sign(v.w, lup, b.w, pbias));
                         }
+                    }
                     }
                     pm = __brev(pm);   // coordinate k at bit k
                     s32 = ((s4[0] + s4[1]) + (s4[2] + s4[3])) + ((s4[4] + s4[5]) + (s4[6] + s4[7]));
-                    if (kSq) q32 = ((q4[0] + q4[1]) + (q4[2] + q4[3])) + ((q4[4] + q4[5]) + (q4[6] + q4[7]));
+                    if constexpr (kSq)
+                        q32 = ((q4[0] + q4[1]) + (q4[2] + q4[3])) + ((q4[4] + q4[5]) + (q4[6] + q4[7]));
                     if (!(s32 < t_c)) {
                         // Some |g| may reach t_c (or be non-finite): split exactly.
 #pragma unroll
