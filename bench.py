@@ -19,6 +19,7 @@ import json
 import os
 import statistics
 import subprocess
+import tempfile
 import sys
 import time
 
@@ -151,9 +152,12 @@ class Clocks:
         self.path = None
 
     def start(self):
+        # The raw samples go to $GS_CLOCKS_DIR (kept for inspection) or a
+        # temporary directory; the summary goes into the JSON line.
         try:
-            os.makedirs(os.path.join(ROOT, "gpurun_out"), exist_ok=True)
-            self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{self.gpu}.csv")
+            out_dir = os.environ.get("GS_CLOCKS_DIR") or tempfile.mkdtemp(prefix="gs_clocks_")
+            os.makedirs(out_dir, exist_ok=True)
+            self.path = os.path.join(out_dir, f"clocks_rank{self.gpu}.csv")
             self.fh = open(self.path, "w")
             self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}",
                                           "--format=csv,noheader,nounits", "-lms", "100"],

@@ -23,7 +23,7 @@
  *                  budget epsilon: sort the magnitudes, take the smallest k
  *                  satisfying (6), set p by (7).
  *
- * Readings where the paper is silent (each is listed in the design doc):
+ * Readings where the paper is silent, ambiguous or garbled:
  *   - `iters` is the maximum number of rescalings (Algorithm 3, steps 4-10);
  *     iters = 0 returns p^0.  Section 5 runs two.
  *   - A coordinate is active iff fl64(lambda |g_i|) < 1 (step 5 "p_i != 1").
