@@ -61,6 +61,7 @@ constexpr int kBrPer = kHistBins / kBrThreads;
 constexpr int kEpsNewtonMax = 24;
 constexpr int kEpsBisectMax = 32;   // a bisection over fp32 bit patterns ends within 31 passes
 constexpr int kEpsCTAs = 8;       // cluster size of k_solve_eps for long segments
+constexpr int kPassUnroll = 8;    // loads per lane in flight in the passes over C
 
 static_assert(kChunk % kUnit == 0, "units tile a chunk");
 static_assert(kHistBins % kBrThreads == 0, "bins split evenly over the bracket CTA");
@@ -386,19 +387,29 @@ __global__ void __launch_bounds__(kThreads) k_solve_eps(const __grid_constant__ 
         for (int q = rank * kWarps + warp; q < nch; q += ncta * kWarps) {
             const int n = Ls.c_cnt[c0 + q];
             const float* src = cb + (int64_t)q * kChunk;
-            for (int e = lane; e < n; e += 32) {
-                const float a = src[e];
-                if (a < tau) {
-                    ++kb;
-                    two_sum_add(uh, ul, a);
+            // kPassUnroll loads per lane in flight, then the sums in index order.
+            for (int e0 = 0; e0 < n; e0 += 32 * kPassUnroll) {
+                float av[kPassUnroll];
+#pragma unroll
+                for (int u = 0; u < kPassUnroll; ++u) {
+                    const int e = e0 + u * 32 + lane;
+                    av[u] = e < n ? src[e] : 0.0f;
+                }
+#pragma unroll
+                for (int u = 0; u < kPassUnroll; ++u) {
+                    if (e0 + u * 32 + lane >= n) continue;
+                    const float a = av[u];
                     const float p = a * a;
-                    two_sum_add(bh, bl, p);
-                    bl += fmaf(a, a, -p);
-                } else {
-                    ++ka;
-                    const float p = a * a;
-                    two_sum_add(qh, ql, p);
-                    ql += fmaf(a, a, -p);
+                    if (a < tau) {
+                        ++kb;
+                        two_sum_add(uh, ul, a);
+                        two_sum_add(bh, bl, p);
+                        bl += fmaf(a, a, -p);
+                    } else {
+                        ++ka;
+                        two_sum_add(qh, ql, p);
+                        ql += fmaf(a, a, -p);
+                    }
                 }
             }
         }
