@@ -345,6 +345,18 @@ typedef enum {
 } gs_option;
 gs_status gs_set_option(int option, int64_t value);
 
+/*
+ * Self-test of the device-side timeouts (no counterpart in the paper).  Every
+ * spin wait in the library's kernels is bounded: on expiry the kernel records
+ * GS_ERR_TIMEOUT in the status word and returns.  This launches one warp that
+ * waits, with a short limit, on something that never completes -- kind 0: an
+ * mbarrier phase nothing arrives at (the primitive the streaming pass waits
+ * with), kind 1: a device flag nothing sets -- so the next gs_sync_status()
+ * returns GS_ERR_TIMEOUT and the context stays usable.  The call itself
+ * returns GS_OK (GS_ERR_INVALID_ARG for another kind).
+ */
+gs_status gs_selftest_timeout(int kind, void* stream);
+
 /* Tracing.  The library counts every kernel it launches; with
  * GS_OPT_KERNEL_TIMING = 1 it also brackets each launch with CUDA events
  * recorded on the launching stream.  gs_kernel_times() waits for the

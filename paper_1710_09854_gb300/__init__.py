@@ -25,7 +25,7 @@ GS_OPT_FORCE_EXACT_SOLVE, GS_OPT_SAMPLE_SIZE, GS_OPT_KERNEL_TIMING, GS_OPT_STREA
 EXPORTS = ("gs_status_string", "gs_last_error", "gs_version", "gs_sync_status", "gs_probabilities", "gs_probabilities_ex",
            "gs_sparsify", "gs_batched_sparsify", "gs_batched_sparsify_hybrid", "gs_probabilities_eps", "gs_batched_sparsify_eps", "gs_segmented_sparsify", "gs_sparse_aggregate",
            "gs_sparsify_aggregate", "gs_sparsify_average_sparsify", "gs_sparsify_noalloc", "gs_pipeline_host", "gs_logreg_grad", "gs_logreg_margins", "gs_row_sq_norms", "gs_sum_rows", "gs_sgd_step",
-           "gs_random_words", "gs_set_option", "gs_kernel_count", "gs_kernel_name",
+           "gs_random_words", "gs_selftest_timeout", "gs_set_option", "gs_kernel_count", "gs_kernel_name",
            "gs_kernel_times")
 
 
@@ -77,6 +77,7 @@ def lib():
             "gs_pipeline_host": ([vp, i32, i32, i64, dbl, i32, u64, u32, u32, vp, vp, vp, vp, i64, vp, vp, vp, vp],
                                  i32),
             "gs_random_words": ([u64, u32, u32, i64, i64, vp, vp], i32),
+            "gs_selftest_timeout": ([i32, vp], i32),
             "gs_logreg_grad": ([vp, vp, i32, i32, vp, vp, i32, i32, ctypes.c_float, vp, vp, vp], i32),
             "gs_logreg_margins": ([vp, vp, i32, i32, vp, vp, vp], i32),
             "gs_row_sq_norms": ([vp, vp, i32, i64, vp, vp], i32),
@@ -227,6 +228,12 @@ def gs_sgd_step(w, v, scale, eta0, T0, t, qsq, gsq, log=None, stream=None):
     _check(lib().gs_sgd_step(_ptr(w, "w", f32), _ptr(v, "v", f32), w.numel(), float(scale), float(eta0), float(T0),
                              int(t), _ptr(qsq, "qsq", f32), _ptr(gsq, "gsq", f32), gsq.numel(),
                              _ptr(log, "log", f32), _stream(stream)), "gs_sgd_step")
+
+
+def gs_selftest_timeout(kind, stream=None):
+    """Launch the bounded-wait self-test (kind 0: mbarrier, 1: flag); the next
+    gs_sync_status() returns GS_ERR_TIMEOUT."""
+    _check(lib().gs_selftest_timeout(int(kind), _stream(stream)), "gs_selftest_timeout")
 
 
 def gs_random_words(seed, step, worker, i0, out, stream=None):

@@ -619,6 +619,15 @@ gs_status gs_pipeline_host(const void* g_host, int dtype, int M, int64_t d, doub
     return GS_OK;
 }
 
+gs_status gs_selftest_timeout(int kind, void* stream) {
+    if (kind != 0 && kind != 1) return GS_ERR_INVALID_ARG;
+    DevState* s = nullptr;
+    gs_status rc = device_state(&s);
+    if (rc != GS_OK) return rc;
+    GS_TRY(launch_wait_selftest(kind, s->status, static_cast<cudaStream_t>(stream)));
+    return GS_OK;
+}
+
 gs_status gs_random_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t i0, int64_t n, uint32_t* out,
                           void* stream) {
     if (!out || i0 < 0 || n < 0 || i0 > INT64_MAX - n) return GS_ERR_INVALID_ARG;

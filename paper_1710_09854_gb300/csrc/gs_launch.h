@@ -96,6 +96,9 @@ cudaError_t launch_aggregate(const AggArgs& A, int32_t* off, float* out, int* st
 cudaError_t launch_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t i0, int64_t n, uint32_t* out,
                          cudaStream_t st);
 bool stream_tma_eligible(const Layout& Lo);
+// One warp's bounded wait on something that never completes (kind 0: an
+// mbarrier, kind 1: a device flag); records kStTimeout.
+cudaError_t launch_wait_selftest(int kind, int* status, cudaStream_t st);
 cudaError_t launch_stream_tma(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, int* status,
                               cudaStream_t st, bool* used);
 // Algorithm 2 (variance budget eps): the histogram pass and the bracket of

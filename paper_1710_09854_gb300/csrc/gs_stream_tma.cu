@@ -74,11 +74,38 @@ __device__ __forceinline__ bool mbar_test(uint64_t* b, uint32_t parity) {
         : "memory");
     return ok != 0;
 }
-// Wait until the phase with the given parity has completed; false on timeout.
-__device__ __forceinline__ bool mbar_wait(uint64_t* b, uint32_t parity) {
-    for (long long i = 0; i < kWaitLimit; ++i)
+// Wait until the phase with the given parity has completed; false after
+// `limit` polls (each try_wait returns by itself within a hardware time limit).
+__device__ __forceinline__ bool mbar_wait_n(uint64_t* b, uint32_t parity, long long limit) {
+    for (long long i = 0; i < limit; ++i)
         if (mbar_test(b, parity)) return true;
     return false;
+}
+__device__ __forceinline__ bool mbar_wait(uint64_t* b, uint32_t parity) { return mbar_wait_n(b, parity, kWaitLimit); }
+
+// A device word nothing ever writes (the self-test's flag).
+__device__ int g_never_set = 0;
+
+// Self-test of the bounded waits: one warp waits, with a short limit, on an
+// mbarrier that nothing arrives at (kind 0: the streaming kernel's primitive)
+// or on a flag that nothing sets (kind 1); on expiry it records kStTimeout in
+// the status word and returns, leaving the context usable.
+__global__ void k_wait_selftest(int kind, long long limit, int* status) {
+    grid_dep_wait();
+    __shared__ uint64_t bar;
+    if (threadIdx.x == 0) {
+        mbar_init(&bar, 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncwarp();
+    bool ok = false;
+    if (kind == 0) {
+        ok = mbar_wait_n(&bar, 0u, limit);   // phase 0 never completes
+    } else {
+        const volatile int* f = &g_never_set;
+        for (long long i = 0; i < limit && !ok; ++i) ok = *f != 0;
+    }
+    if (!__all_sync(0xFFFFFFFFu, ok) && threadIdx.x == 0) atomicOr(status, kStTimeout);
 }
 __device__ __forceinline__ void tma_load_rows(void* dst, const CUtensorMap* map, int row, uint64_t* bar) {
     asm volatile(
@@ -499,6 +526,14 @@ int sm_count_tma() {
 }
 
 }  // namespace
+
+cudaError_t launch_wait_selftest(int kind, int* status, cudaStream_t st) {
+    set_launch_error_site("k_wait_selftest launch");
+    // Short limits: the mbarrier wait gives up after 256 polls, the flag spin
+    // after 2^20 loads.
+    k_wait_selftest<<<1, 32, 0, st>>>(kind, kind == 0 ? 256 : (1ll << 20), status);
+    return cudaGetLastError();
+}
 
 bool stream_tma_eligible(const Layout& Lo) {
     if ((reinterpret_cast<uintptr_t>(Lo.g) & 15u) != 0) return false;

@@ -115,3 +115,8 @@ def test_training_loop_entry_points_reject_bad_arguments():
     assert L.gs_sum_rows(fake, 2, 0, fake, None) == bad
     assert L.gs_sgd_step(fake, fake, 10, 1.0, 0.1, 0.0, 0, fake, fake, 2, None, None) == bad       # T0 = 0
     assert L.gs_sgd_step(fake, fake, 10, 1.0, 0.1, 4.0, -1, fake, fake, 2, None, None) == bad      # t < 0
+
+
+def test_selftest_timeout_rejects_unknown_kind():
+    import paper_1710_09854_gb300 as gs
+    assert gs.lib().gs_selftest_timeout(2, None) == gs.GS_ERR_INVALID_ARG
