@@ -3,6 +3,7 @@
 // status word, and the order of the kernel launches of each call.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdint>
 #include <cstdio>
@@ -212,6 +213,11 @@ gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off
         Lo.seg_chunk0 = meta.chunk0;
         Lo.cpw = meta.cpw;
     }
+    int64_t max_seg_len = d;   // the longest segment (sizes the solve's shared memory)
+    if (L > 1) {
+        max_seg_len = 0;
+        for (int l = 0; l < L; ++l) max_seg_len = std::max<int64_t>(max_seg_len, seg_off[l + 1] - seg_off[l]);
+    }
     const int64_t n_chunks64 = (int64_t)M * Lo.cpw;
     const int64_t n_seg64 = (int64_t)M * L;
     if (n_chunks64 > INT32_MAX || n_seg64 > INT32_MAX) return GS_ERR_INVALID_ARG;
@@ -248,7 +254,7 @@ gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off
     }
     if (e == cudaSuccess) {
         e = alg2 ? launch_solve_eps(Lo, w.sp, w.ls, n_seg, eps, s->status, info, st)
-                 : launch_solve(Lo, w.sp, w.ls, n_seg, kappa, iters, force, s->status, info, st);
+                 : launch_solve(Lo, w.sp, w.ls, n_seg, kappa, iters, force, s->status, info, st, max_seg_len);
     }
     if (e == cudaSuccess) {
         if (prob) e = launch_prob(Lo, w.sp, p, st);
@@ -413,7 +419,7 @@ gs_status run_noalloc(const float* g, int64_t d, double kappa, int iters, uint64
         if (tma_ok) e = launch_stream_tma(Lo, w.sp, w.ls, n_chunks, s->status, st, &used);
         if (e == cudaSuccess && !used) e = launch_stream(Lo, w.sp, w.ls, n_chunks, true, st);
     }
-    if (e == cudaSuccess) e = launch_solve(Lo, w.sp, w.ls, 1, kappa, iters, force, s->status, info, st);
+    if (e == cudaSuccess) e = launch_solve(Lo, w.sp, w.ls, 1, kappa, iters, force, s->status, info, st, d);
     if (e == cudaSuccess) e = launch_compact(Lo, w.sp, w.ls, n_chunks, idx, val, nnz, d, s->status, st);
     if (e == cudaSuccess && status) {
         k_noalloc_status<<<1, 1, 0, st>>>(s->status, status);

@@ -529,7 +529,7 @@ __device__ __forceinline__ int block_scan_total(int v, int* sh, int& total) {
 }
 
 struct CView {
-    const float* smem;       // compacted candidates (nC <= kSolveSmemC), else NULL
+    const float* smem;       // compacted candidates (when they fit in shared memory), else NULL
     const float* gbase;      // c_val + region of the segment's first chunk
     const int32_t* pre;      // chunk prefix over the segment's chunks
     int nch;
@@ -622,14 +622,17 @@ __device__ __noinline__ void solve_exact(const Layout& Lo, const Lists& Ls, int 
 // CTA of the cluster walks a share of the segment's chunks in each pass and the
 // CTA partials are combined through distributed shared memory in rank order.
 __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lists Ls, double kappa, int iters,
-                                                    int force_exact, int* status, gs_info_dev* info) {
+                                                    int force_exact, int* status, gs_info_dev* info,
+                                                    int cap_chunks, int cap_c) {
     grid_dep_wait();
     namespace cg = cooperative_groups;
     cg::cluster_group cluster = cg::this_cluster();
     const int ncta = (int)cluster.num_blocks(), rank = (int)cluster.block_rank();
+    // Dynamic shared memory, sized by the launcher for the largest segment:
+    // cap_chunks chunk-prefix entries (+4), then cap_c candidate values.
     extern __shared__ unsigned char dsm[];
-    int32_t* spre = reinterpret_cast<int32_t*>(dsm);                       // kSolveSmemChunks + 1
-    float* sc = reinterpret_cast<float*>(dsm + sizeof(int32_t) * (kSolveSmemChunks + 4));  // kSolveSmemC
+    int32_t* spre = reinterpret_cast<int32_t*>(dsm);
+    float* sc = reinterpret_cast<float*>(dsm + sizeof(int32_t) * (cap_chunks + 4));
     __shared__ double shd[33];
     __shared__ int shi[33];
     __shared__ float s_acap;
@@ -650,7 +653,7 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
 
     // Candidate view: chunk prefix (shared or global scratch), values gathered to shared memory when they fit.
     const int nch = c1 - c0;
-    int32_t* pre = nch <= kSolveSmemChunks ? spre : Ls.c_pre + c0 + s;
+    int32_t* pre = nch <= cap_chunks ? spre : Ls.c_pre + c0 + s;
     CView C;
     C.pre = pre;
     C.nch = nch;
@@ -679,7 +682,7 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
         }
         if (tid == 0) pre[nch] = total;
         C.nC = total;
-        if (total <= kSolveSmemC) {
+        if (total <= cap_c) {
             int at = run - tot;
 #pragma unroll
             for (int j = 0; j < kSolvePer; ++j) {
@@ -693,7 +696,7 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
     } else {
         block_exclusive_scan(Ls.c_cnt + c0, nch, pre, shi);
         C.nC = pre[nch];
-        if (C.nC <= kSolveSmemC) {
+        if (C.nC <= cap_c) {
             for (int e = tid; e < C.nC; e += blockDim.x) sc[e] = C.at(e);
             __syncthreads();
             C.smem = sc;
@@ -1442,9 +1445,15 @@ cudaError_t launch_stream(const Layout& Lo, const SegParam* sp, const Lists& Ls,
 }
 
 cudaError_t launch_solve(const Layout& Lo, SegParam* sp, const Lists& Ls, int n_seg, double kappa, int iters,
-                         int force_exact, int* status, gs_info_dev* info, cudaStream_t st) {
+                         int force_exact, int* status, gs_info_dev* info, cudaStream_t st, int64_t max_seg_len) {
     set_launch_error_site("k_solve launch");
-    const size_t smem = sizeof(int32_t) * (kSolveSmemChunks + 4) + sizeof(float) * kSolveSmemC;
+    // Shared memory for the largest segment only: its chunk prefix and at most
+    // as many candidate values as it has coordinates (short layers then leave
+    // room for more resident CTAs).
+    const int64_t maxch = (max_seg_len + kChunk - 1) / kChunk + 1;
+    const int cap_chunks = (int)std::min<int64_t>(kSolveSmemChunks, maxch);
+    const int cap_c = (int)std::min<int64_t>(kSolveSmemC, max_seg_len);
+    const size_t smem = sizeof(int32_t) * (cap_chunks + 4) + sizeof(float) * cap_c;
     cudaError_t e = cudaFuncSetAttribute(k_solve, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     TraceScope ts(kKSolve, st);
@@ -1454,9 +1463,9 @@ cudaError_t launch_solve(const Layout& Lo, SegParam* sp, const Lists& Ls, int n_
     const int ncta = (Lo.L == 1 && kappa * (double)Lo.d > (double)(1 << 20)) ? kSolveCTAs : 1;
     if (ncta == 1)
         return launch_dep(k_solve, dim3(n_seg), dim3(kThreads), smem, st, Lo, sp, Ls, kappa, iters, force_exact,
-                          status, info);
+                          status, info, cap_chunks, cap_c);
     return launch_dep_cluster(k_solve, dim3(n_seg * ncta), dim3(kThreads), smem, ncta, st, Lo, sp, Ls, kappa, iters,
-                              force_exact, status, info);
+                              force_exact, status, info, cap_chunks, cap_c);
 }
 
 cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, int32_t* idx,

@@ -72,7 +72,7 @@ cudaError_t launch_bound(const Layout& Lo, SegParam* sp, int n_seg, double kappa
 cudaError_t launch_stream(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, bool build_p,
                           cudaStream_t st);
 cudaError_t launch_solve(const Layout& Lo, SegParam* sp, const Lists& Ls, int n_seg, double kappa, int iters,
-                         int force_exact, int* status, gs_info_dev* info, cudaStream_t st);
+                         int force_exact, int* status, gs_info_dev* info, cudaStream_t st, int64_t max_seg_len);
 // Outputs of the hybrid coding (section 3.3): per worker m, rows of `cap`
 // entries at m * cap.
 struct HybridOut {

@@ -577,3 +577,69 @@ def test_hybrid_code(gs, dtype, kind, kappa, d):
         np.testing.assert_array_equal(di, gi)
         np.testing.assert_array_equal(dv, gv)
         compare_sparse(di, dv, g_host[m], kappa, iters, seed, step, m)
+
+
+def test_outputs_stay_inside_their_buffers(gs):
+    """Guard bands: every output sits inside a larger sentinel-filled buffer;
+    after each call the band past the buffer and, within each row, the slots
+    past the written count still hold the sentinel."""
+    import torch
+    G = 4096
+    SI, SV = -123456789, -7.5e33
+    M, d = 5, 50003
+    g_host = np.stack([_vector(k, d, 90 + m) for m, k in enumerate(["t3", "lognormal", "normal", "t3", "ties"])])
+    g = _dev(g_host)
+
+    def bands(shape, dtype, fill):
+        n = int(np.prod(shape))
+        full = torch.full((n + G,), fill, dtype=dtype, device="cuda")
+        return full, full[:n].view(*shape)
+
+    def check_tail(full, n, fill):
+        assert bool((full[n:] == fill).all()), "write past the end of an output buffer"
+
+    def check_rows(view, counts, fill):
+        for m, k in enumerate(counts):
+            assert bool((view[m, min(int(k), view.shape[1]):] == fill).all()), "write past a row's count"
+
+    for cap in (d, 1000):
+        fi, idx = bands((M, cap), torch.int32, SI)
+        fv, val = bands((M, cap), torch.float32, SV)
+        fn, nnz = bands((M,), torch.int32, SI)
+        fo, out = bands((d,), torch.float32, SV)
+        gs.gs_sparsify_aggregate(g, 0.02, 3, 5, 1, 0, idx, val, nnz, out)
+        rc = gs.gs_sync_status()
+        assert rc == (gs.GS_OK if cap == d else gs.GS_ERR_CAPACITY)
+        counts = nnz.cpu().numpy()
+        check_tail(fi, M * cap, SI)
+        check_tail(fv, M * cap, SV)
+        check_tail(fn, M, SI)
+        check_tail(fo, d, SV)
+        check_rows(idx, counts, SI)
+        check_rows(val, counts, SV)
+    # the hybrid code
+    fa, qa_i = bands((M, d), torch.int32, SI)
+    fav, qa_v = bands((M, d), torch.float32, SV)
+    fb, qb = bands((M, d), torch.int32, SI)
+    fna, n_a = bands((M,), torch.int32, SI)
+    fnb, n_b = bands((M,), torch.int32, SI)
+    fl, il = bands((M,), torch.float32, SV)
+    gs.gs_batched_sparsify_hybrid(g, 0.05, 2, 5, 2, 0, qa_i, qa_v, qb, n_a, n_b, il)
+    assert gs.gs_sync_status() == gs.GS_OK
+    for full, n, fill in ((fa, M * d, SI), (fav, M * d, SV), (fb, M * d, SI), (fna, M, SI), (fnb, M, SI), (fl, M, SV)):
+        check_tail(full, n, fill)
+    check_rows(qa_i, n_a.cpu().numpy(), SI)
+    check_rows(qb, n_b.cpu().numpy(), SI)
+    # Algorithm 2 and the probabilities
+    fi, idx = bands((M, d), torch.int32, SI)
+    fv, val = bands((M, d), torch.float32, SV)
+    fn, nnz = bands((M,), torch.int32, SI)
+    gs.gs_batched_sparsify_eps(g, 0.5, 5, 3, 0, idx, val, nnz)
+    assert gs.gs_sync_status() == gs.GS_OK
+    check_tail(fi, M * d, SI)
+    check_tail(fv, M * d, SV)
+    check_rows(idx, nnz.cpu().numpy(), SI)
+    fp, p = bands((d,), torch.float32, SV)
+    gs.gs_probabilities(g[0].contiguous(), 0.02, 3, p)
+    assert gs.gs_sync_status() == gs.GS_OK
+    check_tail(fp, d, SV)
