@@ -683,12 +683,32 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
         if (tid == 0) pre[nch] = total;
         C.nC = total;
         if (total <= cap_c) {
-            int at = run - tot;
+            // The values of C copied to shared memory.  Many sparse chunks (at
+            // least two per thread, 32 values or fewer on average): each thread
+            // copies its own, their loads being independent.  Otherwise (few or
+            // dense chunks; a short segment takes every coordinate): a warp per
+            // chunk, or the whole CTA per chunk when there are few.
+            if (nch >= 2 * kThreads && total <= 32 * nch) {
+                int at = run - tot;
 #pragma unroll
-            for (int j = 0; j < kSolvePer; ++j) {
-                const int64_t base = (int64_t)(kSolvePer * tid + j) * kChunk;
-                for (int v = 0; v < cnt[j]; ++v) sc[at + v] = C.gbase[base + v];
-                at += cnt[j];
+                for (int j = 0; j < kSolvePer; ++j) {
+                    const int64_t base = (int64_t)(kSolvePer * tid + j) * kChunk;
+                    for (int v = 0; v < cnt[j]; ++v) sc[at + v] = C.gbase[base + v];
+                    at += cnt[j];
+                }
+            } else {
+                __syncthreads();   // pre[] complete
+                if (nch <= kWarps) {
+                    for (int q = 0; q < nch; ++q) {
+                        const int b = pre[q], n = pre[q + 1] - b;
+                        for (int v = tid; v < n; v += blockDim.x) sc[b + v] = C.gbase[(int64_t)q * kChunk + v];
+                    }
+                } else {
+                    for (int q = warp; q < nch; q += kWarps) {
+                        const int b = pre[q], n = pre[q + 1] - b;
+                        for (int v = lane; v < n; v += 32) sc[b + v] = C.gbase[(int64_t)q * kChunk + v];
+                    }
+                }
             }
             C.smem = sc;
         }
