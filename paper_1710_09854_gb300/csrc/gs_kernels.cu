@@ -358,7 +358,8 @@ constexpr int kBoundRun = 8;             // consecutive coordinates read per str
 // kBoundRun consecutive coordinates from each of ns / kBoundRun strata) and
 // store the |g| values straight into rank 0's shared memory; rank 0 then runs Algorithm 3
 // to its fixed point on the sample alone, with block-wide sums.
-__global__ void __cluster_dims__(kBoundCTAs, 1, 1) __launch_bounds__(kBoundCtaThreads)
+template <int kCTAs>
+__global__ void __cluster_dims__(kCTAs, 1, 1) __launch_bounds__(kBoundCtaThreads)
     k_bound(Layout Lo, SegParam* sp, double kappa, int ns, int force_exact) {
     grid_dep_wait();
     namespace cg = cooperative_groups;
@@ -367,14 +368,14 @@ __global__ void __cluster_dims__(kBoundCTAs, 1, 1) __launch_bounds__(kBoundCtaTh
     __shared__ float2 sh2[33];
     __shared__ float4 sh4[33];
     const int rank = (int)cluster.block_rank();
-    const int s = blockIdx.x / kBoundCTAs, tid = threadIdx.x;
+    const int s = blockIdx.x / kCTAs, tid = threadIdx.x;
     int m, l, c0, c1;
     int64_t lo, hi;
     seg_range(Lo, s, m, l, lo, hi, c0, c1);
     const int64_t len = hi - lo;
     SegParam& P = sp[s];
-    if (len <= ns || force_exact) {
-        // Short segment (or exact mode): every coordinate is a candidate.
+    if (force_exact) {
+        // Exact mode: every coordinate is a candidate.
         if (rank == 0 && tid == 0) {
             P.done = 0;
             P.w_done = 0;
@@ -385,15 +386,27 @@ __global__ void __cluster_dims__(kBoundCTAs, 1, 1) __launch_bounds__(kBoundCtaTh
         }
         return;   // uniform over the cluster: no CTA reaches a cluster barrier
     }
+    float* dst = cluster.map_shared_rank(sa, 0);
+    // A segment no longer than the sample is taken whole: the fixed point below
+    // is then Algorithm 3 itself (in fp32), whose iterates never pass the fixed
+    // point, so a 1% margin covers the fp32 rounding.
+    const bool whole = len <= ns;
+    if (whole) {
+        for (int e = rank * kBoundCtaThreads + tid; e < (int)len; e += kCTAs * kBoundCtaThreads) {
+            float x = fabsf(load_one(Lo, m, lo + e));
+            if (!(x < kInf)) x = 0.0f;  // non-finite values are reported by the solve
+            dst[e] = x;
+        }
+        ns = (int)len;
+    }
     // ns / 8 strata; from each, 8 consecutive coordinates starting at a
     // random multiple of 8 (one 32-byte sector of fp32 g).
-    const int per = ns / (kBoundRun * kBoundCTAs);                  // strata of this CTA
-    const int nst = per * kBoundCTAs;
-    ns = nst * kBoundRun;                                           // samples actually drawn
-    const int64_t q = len / nst;                                    // stratum width (the last one takes the rest)
-    const int64_t q_last = len - (int64_t)(nst - 1) * q;
+    const int per = whole ? 0 : ns / (kBoundRun * kCTAs);      // strata of this CTA
+    const int nst = per * kCTAs;
+    if (!whole) ns = nst * kBoundRun;                               // samples actually drawn
+    const int64_t q = whole ? 1 : len / nst;                        // stratum width (the last one takes the rest)
+    const int64_t q_last = whole ? 1 : len - (int64_t)(nst - 1) * q;
     const uint32_t hs = mix32((uint32_t)s + 0x68E31DA4u);
-    float* dst = cluster.map_shared_rank(sa, 0);
     for (int e = tid; e < per * kBoundRun; e += kBoundCtaThreads) {
         const int k = rank * per + e / kBoundRun;                   // stratum
         const int r = e % kBoundRun;
@@ -465,6 +478,7 @@ __global__ void __cluster_dims__(kBoundCTAs, 1, 1) __launch_bounds__(kBoundCtaTh
                                                     (float)kBoundZs * sqrtf(rel_s * rel_s + rel_k * rel_k)));
             }
             margin = fminf(margin, 64.0f);
+            if (whole) margin = 1.01f;
             // lam_up32 rounded up and t_c rounded down keep both lists supersets;
             // the fp64 bound is lam_up32 itself.
             const float up32 = __fmul_ru(lam, margin);
@@ -1446,14 +1460,20 @@ int sm_count() {
 cudaError_t launch_bound(const Layout& Lo, SegParam* sp, int n_seg, double kappa, int ns, int force_exact,
                          cudaStream_t st) {
     set_launch_error_site("k_bound launch");
+    // One worker row (or a few): clusters of kBoundCTAs CTAs share each
+    // segment's random sample loads.  Layer-wise calls have many short
+    // segments: one CTA each (every CTA of a cluster would hold the whole
+    // sample buffer, and clusters of 8 would take many waves).
     const size_t smem = (size_t)ns * sizeof(float);
+    const bool one = Lo.L > 1;
+    auto kern = one ? k_bound<1> : k_bound<kBoundCTAs>;
     if (smem > 48 * 1024) {
-        cudaError_t e = cudaFuncSetAttribute(k_bound, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
     }
     TraceScope ts(kKBound, st);
-    return launch_dep(k_bound, dim3(n_seg * kBoundCTAs), dim3(kBoundCtaThreads), smem, st, Lo, sp, kappa, ns,
-                      force_exact);
+    return launch_dep(kern, dim3(n_seg * (one ? 1 : kBoundCTAs)), dim3(kBoundCtaThreads), smem, st, Lo, sp, kappa,
+                      ns, force_exact);
 }
 
 cudaError_t launch_stream(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, bool build_p,
