@@ -224,6 +224,10 @@ def run_gpu(args):
             return
         if off is None:
             gs.gs_batched_sparsify(g, kappa, w.iters, w.seed, t, 0, idx, val, nnz, stream=stream)
+        elif not args.separate:
+            gs.gs_segmented_sparsify_aggregate(g, off, kappa, w.iters, w.seed, t, 0, idx, val, nnz, out,
+                                               stream=stream)
+            return
         else:
             gs.gs_segmented_sparsify(g, off, kappa, w.iters, w.seed, t, 0, idx, val, nnz, stream=stream)
         gs.gs_sparse_aggregate(idx_rows, val_rows, nnz, d, out, stream=stream)
@@ -335,7 +339,8 @@ def run_gpu(args):
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": dtype, "data": "synthetic",
         "config": {"workload": w.name, "M": M, "d": d, "kappa": kappa, "iters": w.iters, "dtype": dtype,
-                   "api": ("gs_segmented_sparsify + gs_sparse_aggregate" if off is not None else
+                   "api": (("gs_segmented_sparsify + gs_sparse_aggregate" if args.separate else
+                            "gs_segmented_sparsify_aggregate") if off is not None else
                            "gs_batched_sparsify + gs_sparse_aggregate" if args.separate else "gs_sparsify_aggregate"),
                    "parallelism": f"replicas{ws}", "l2": "inputs exceed L2 (%.2f GB of g per step)" % (M * d * esz / 1e9)},
         "hbm_gbs_pipeline": round(pipe_gbs, 1),

@@ -241,6 +241,17 @@ gs_status gs_segmented_sparsify(const void* g, int dtype, int M, int64_t d, cons
                                 float* val, int32_t* nnz, int64_t cap, gs_info* info, void* stream);
 
 /*
+ * gs_segmented_sparsify plus the sum of the M workers' sparse vectors into
+ * out (d fp32, overwritten), fused with the compaction exactly as in
+ * gs_sparsify_aggregate (the fp32 sum in worker order; entries beyond cap are
+ * neither written nor summed).  1 <= M <= 512.
+ */
+gs_status gs_segmented_sparsify_aggregate(const void* g, int dtype, int M, int64_t d, const int64_t* seg_offsets,
+                                          int L, double kappa, int iters, uint64_t seed, uint32_t step,
+                                          uint32_t worker0, int32_t* idx, float* val, int32_t* nnz, int64_t cap,
+                                          gs_info* info, float* out, void* stream);
+
+/*
  * Sum M sparse vectors into a dense fp32 vector (Algorithm 1, step 6):
  *   out[i] = sum_{m=0}^{M-1} Q_m[i], added in fp32 in worker order, so the
  *   result is deterministic.  `out` (device, d fp32) is overwritten.

@@ -23,7 +23,7 @@ GS_OPT_FORCE_EXACT_SOLVE, GS_OPT_SAMPLE_SIZE, GS_OPT_KERNEL_TIMING, GS_OPT_STREA
 
 # Symbols include/gs.h declares (checked by the tests).
 EXPORTS = ("gs_status_string", "gs_last_error", "gs_version", "gs_sync_status", "gs_probabilities", "gs_probabilities_ex",
-           "gs_sparsify", "gs_batched_sparsify", "gs_batched_sparsify_hybrid", "gs_probabilities_eps", "gs_batched_sparsify_eps", "gs_segmented_sparsify", "gs_sparse_aggregate",
+           "gs_sparsify", "gs_batched_sparsify", "gs_batched_sparsify_hybrid", "gs_probabilities_eps", "gs_batched_sparsify_eps", "gs_segmented_sparsify", "gs_segmented_sparsify_aggregate", "gs_sparse_aggregate",
            "gs_sparsify_aggregate", "gs_sparsify_average_sparsify", "gs_sparsify_noalloc", "gs_pipeline_host", "gs_logreg_grad", "gs_logreg_margins", "gs_row_sq_norms", "gs_sum_rows", "gs_sgd_step",
            "gs_random_words", "gs_selftest_timeout", "gs_set_option", "gs_kernel_count", "gs_kernel_name",
            "gs_kernel_times")
@@ -69,6 +69,8 @@ def lib():
             "gs_batched_sparsify_eps": ([vp, i32, i32, i64, dbl, u64, u32, u32, vp, vp, vp, i64, vp, vp], i32),
             "gs_segmented_sparsify": ([vp, i32, i32, i64, vp, i32, dbl, i32, u64, u32, u32, vp, vp, vp, i64, vp, vp],
                                       i32),
+            "gs_segmented_sparsify_aggregate": ([vp, i32, i32, i64, vp, i32, dbl, i32, u64, u32, u32, vp, vp, vp, i64,
+                                                 vp, vp, vp], i32),
             "gs_sparse_aggregate": ([vp, vp, vp, i32, i64, vp, vp], i32),
             "gs_sparsify_aggregate": ([vp, i32, i32, i64, dbl, i32, u64, u32, u32, vp, vp, vp, i64, vp, vp, vp], i32),
             "gs_sparsify_average_sparsify": ([vp, i32, i32, i64, dbl, i32, u64, u32, u32, vp, vp, vp, i64, vp, dbl,
@@ -350,6 +352,23 @@ def gs_segmented_sparsify(g, seg_offsets, kappa, iters, seed, step, worker0, idx
                                        _ptr(idx, "idx", (torch.int32,)), _ptr(val, "val", (torch.float32,)),
                                        _ptr(nnz, "nnz", (torch.int32,)), cap, _ptr(info, "info"), _stream(stream)),
            "gs_segmented_sparsify")
+
+
+def gs_segmented_sparsify_aggregate(g, seg_offsets, kappa, iters, seed, step, worker0, idx, val, nnz, out,
+                                    info=None, stream=None):
+    """gs_segmented_sparsify of g (M, d) plus the dense sum of the M rows into out (d,)."""
+    import torch
+    M, d = g.shape
+    cap = idx.shape[1]
+    off = np.ascontiguousarray(seg_offsets, dtype=np.int64)
+    if idx.shape[0] != M or tuple(val.shape) != tuple(idx.shape) or nnz.numel() != M or out.numel() != d:
+        raise ValueError("idx / val must be (M, cap), nnz (M,), out (d,)")
+    _check(lib().gs_segmented_sparsify_aggregate(_ptr(g, "g"), _g_dtype(g), M, d, off.ctypes.data, off.size - 1,
+                                                 float(kappa), int(iters), int(seed), int(step), int(worker0),
+                                                 _ptr(idx, "idx", (torch.int32,)), _ptr(val, "val", (torch.float32,)),
+                                                 _ptr(nnz, "nnz", (torch.int32,)), cap, _ptr(info, "info"),
+                                                 _ptr(out, "out", (torch.float32,)), _stream(stream)),
+           "gs_segmented_sparsify_aggregate")
 
 
 def gs_sparse_aggregate(idx_list, val_list, nnz, d, out, stream=None):

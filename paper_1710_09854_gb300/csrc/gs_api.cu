@@ -514,6 +514,16 @@ gs_status gs_sparsify_aggregate(const void* g, int dtype, int M, int64_t d, doub
                static_cast<cudaStream_t>(stream), out);
 }
 
+gs_status gs_segmented_sparsify_aggregate(const void* g, int dtype, int M, int64_t d, const int64_t* seg_offsets,
+                                          int L, double kappa, int iters, uint64_t seed, uint32_t step,
+                                          uint32_t worker0, int32_t* idx, float* val, int32_t* nnz, int64_t cap,
+                                          gs_info* info, float* out, void* stream) {
+    if (!out || M < 1 || M > kMaxAggM || L < 1 || !seg_offsets) return GS_ERR_INVALID_ARG;
+    if (L == 1 && (seg_offsets[0] != 0 || seg_offsets[1] != d)) return GS_ERR_INVALID_ARG;
+    return run(g, dtype, M, d, seg_offsets, L, kappa, iters, seed, step, worker0, idx, val, nnz, cap, info, nullptr,
+               static_cast<cudaStream_t>(stream), out);
+}
+
 gs_status gs_sparsify_average_sparsify(const void* g, int dtype, int M, int64_t d, double kappa, int iters,
                                        uint64_t seed, uint32_t step, uint32_t worker0, int32_t* idx, float* val,
                                        int32_t* nnz, int64_t cap, float* v, double kappa_v, int iters_v,

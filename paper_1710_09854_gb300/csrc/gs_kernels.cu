@@ -1198,9 +1198,12 @@ __global__ void __launch_bounds__(kSumWarps * 32) k_sum(const __grid_constant__ 
     const int gs = blockIdx.x * kSumWarps + w;
     if (gs >= n_slices) return;
     const int k = gs / kSlices, sl = gs - k * kSlices;
-    const int64_t t0 = (int64_t)k * kChunk + (int64_t)sl * kSlice;
-    if (t0 >= Lo.d) return;
-    const int tlen = (int)min((int64_t)kSlice, Lo.d - t0);
+    // Chunk k covers the same coordinates in every worker row (also for
+    // layer-wise layouts, whose chunks start at segment starts).
+    const Chunk ch = decode_chunk(Lo, k);
+    const int64_t t0 = ch.lo + (int64_t)sl * kSlice;
+    if (t0 >= ch.hi) return;
+    const int tlen = (int)min((int64_t)kSlice, ch.hi - t0);
     float* acc = tile[w];
 #pragma unroll
     for (int i = 0; i < kSlice / 128; ++i)
@@ -1532,7 +1535,7 @@ cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls
         e = launch_dep(k_emit, dim3(blocks), dim3(kEmitWarps * 32), 0, st, Lo, sp, Ls, n_chunks, idx, val, cap);
     }
     if (e != cudaSuccess || !sum_out) return e;
-    // The sparse sum of the M compacted rows (L == 1), one warp per slice.
+    // The sparse sum of the M compacted rows, one warp per slice.
     const int n_slices = Lo.cpw * kSlices;
     set_launch_error_site("k_sum launch");
     TraceScope ts(kKSum, st);

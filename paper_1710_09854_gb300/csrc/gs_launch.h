@@ -84,8 +84,8 @@ struct HybridOut {
     float* inv_lam;     // [M] fl32(1 / lambda), the magnitude of every Q_B value
 };
 
-// Decide, scan and compact; with sum_out (L == 1 only) also the sparse sum of
-// the M compacted rows into sum_out (d fp32), fused with the compaction (with
+// Decide, scan and compact; with sum_out also the sparse sum of the M
+// compacted rows into sum_out (d fp32), fused with the compaction (with
 // average, the sum divided by M); with hybrid (L == 1 only) the hybrid code
 // instead of the plain lists.
 cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, int32_t* idx,

@@ -200,6 +200,25 @@ def test_segmented_parity(gs):
             r = oracle.sparsify(g_host[m, a:b], kappa, iters, seed, step, m, i0=a)
             compare_sparse(got_i[sel], got_v[sel], g_host[m, a:b], kappa, iters, seed, step, m, i0=a, ref=r)
             assert infos[m * (off.size - 1) + l]["lambda"] == pytest.approx(lams[l], rel=1e-6)
+    _check_segmented_fused(gs, g, off, kappa, iters, seed, step, idx, val, nnz)
+
+
+def _check_segmented_fused(gs, g, off, kappa, iters, seed, step, idx, val, nnz):
+    """gs_segmented_sparsify_aggregate equals gs_segmented_sparsify followed by
+    gs_sparse_aggregate, bit for bit (lists, counts and the sum)."""
+    import torch
+    M, d = g.shape
+    out = torch.empty(d, dtype=torch.float32, device="cuda")
+    gs.gs_sparse_aggregate([idx[m] for m in range(M)], [val[m] for m in range(M)], nnz, d, out)
+    idx2, val2, nnz2 = torch.full_like(idx, -1), torch.zeros_like(val), torch.zeros_like(nnz)
+    out2 = torch.full_like(out, float("nan"))
+    gs.gs_segmented_sparsify_aggregate(g, off, kappa, iters, seed, step, 0, idx2, val2, nnz2, out2)
+    assert gs.gs_sync_status() == gs.GS_OK
+    assert torch.equal(nnz2, nnz)
+    assert torch.equal(out2, out)
+    for m in range(M):
+        k = int(nnz[m].item())
+        assert torch.equal(idx2[m, :k], idx[m, :k]) and torch.equal(val2[m, :k], val[m, :k])
 
 
 def test_aggregate_parity_and_validation(gs):
@@ -309,6 +328,8 @@ def _full_check(gs, g_dev, kappa, iters, seed=1, step=0, workers=None, offsets=N
         gs.gs_segmented_sparsify(g_dev, offsets, kappa, iters, seed, step, 0, idx, val, nnz)
     gs.gs_sparse_aggregate([idx[m] for m in range(M)], [val[m] for m in range(M)], nnz, d, out)
     assert gs.gs_sync_status() == gs.GS_OK
+    if offsets is not None:
+        _check_segmented_fused(gs, g_dev, offsets, kappa, iters, seed, step, idx, val, nnz)
     if offsets is None:
         # The fused call (compaction + sum in one chain) equals the two calls bit for bit.
         idx2 = torch.empty_like(idx)
