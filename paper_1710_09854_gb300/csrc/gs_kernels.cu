@@ -513,7 +513,7 @@ __global__ void __launch_bounds__(kThreads) k_stream(Layout Lo, const SegParam* 
 constexpr int kSolveSmemChunks = 8192;   // chunk-prefix entries kept in shared memory
 constexpr int kSolveSmemC = 12288;       // candidate values kept in shared memory
 constexpr int kSolvePer = 4;             // chunks per thread of the one-round start (segments <= 1024 chunks)
-constexpr int kSolveCTAs = 8;            // cluster size of k_solve for long segments
+constexpr int kSolveCTAs = 16;           // cluster size of k_solve for long segments (non-portable size)
 
 // Exclusive prefix of v over the block (any blockDim <= 1024) and the total.
 __device__ __forceinline__ int block_scan_total(int v, int* sh, int& total) {
@@ -1498,6 +1498,8 @@ cudaError_t launch_solve(const Layout& Lo, SegParam* sp, const Lists& Ls, int n_
     const int cap_c = (int)std::min<int64_t>(kSolveSmemC, max_seg_len);
     const size_t smem = sizeof(int32_t) * (cap_chunks + 4) + sizeof(float) * cap_c;
     cudaError_t e = cudaFuncSetAttribute(k_solve, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(k_solve, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
     if (e != cudaSuccess) return e;
     TraceScope ts(kKSolve, st);
     // C holds about the capped coordinates, whose count the budget kappa d
