@@ -69,6 +69,8 @@ struct SegParam {
     int flags;
     int done;          // chunks of the segment whose streaming outputs are written (zeroed by k_bound)
     int w_done;        // segment l == 0 only: chunks of the worker that k_decide has finished (zeroed by k_bound)
+    int next_chunk;    // segment 0 only: chunks the streaming pass has handed out past each warp's first
+                       // (zeroed by k_bound and k_eps_bracket)
     double sq;         // Algorithm 2 only: sum g_i^2 of the segment
     float t_up;        // Algorithm 2 only: an upper bound of 1 / lambda (+inf if none)
 };

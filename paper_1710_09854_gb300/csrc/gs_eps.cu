@@ -316,6 +316,7 @@ __global__ void __launch_bounds__(kBrThreads) k_eps_bracket(const __grid_constan
         SegParam& P = sp[s];
         P.done = 0;
         P.w_done = 0;
+        P.next_chunk = 0;
         P.sq = S;
         P.l1 = 0.0;
         int flags = 0;

@@ -344,20 +344,18 @@ __device__ __forceinline__ float4 block_sum3f(float a, float b, float c, float4*
 }
 
 // The bound only steers how many candidates the streaming pass keeps, so it
-// is estimated in fp32: a stratified sample of |g| (one coordinate drawn by
-// hash from each of ns equal strata) and Algorithm 3 run on the sample until
-// its scaling factor is within 1e-5 of 1.  One thread-block cluster of
-// kBoundCTAs CTAs per segment: each CTA draws ns / kBoundCTAs strata, and
-// every iteration's sums are exchanged through distributed shared memory
-// and added in rank order, so all CTAs of the cluster follow the same path.
+// is estimated in fp32: a stratified sample of |g| (a run of kBoundRun
+// consecutive coordinates, at a hashed position, from each of ns / kBoundRun
+// equal strata) and Algorithm 3 run on the sample until its scaling factor
+// is within 1e-5 of 1.
 constexpr int kBoundCTAs = 8;
 constexpr int kBoundCtaThreads = 1024;
 constexpr int kBoundRun = 8;             // consecutive coordinates read per stratum
 
-// The 8 CTAs of a cluster share the segment's random sample loads (a run of
-// kBoundRun consecutive coordinates from each of ns / kBoundRun strata) and
-// store the |g| values straight into rank 0's shared memory; rank 0 then runs Algorithm 3
-// to its fixed point on the sample alone, with block-wide sums.
+// One thread-block cluster of kCTAs CTAs per segment (kBoundCTAs, or one for
+// layer-wise calls): the CTAs share the sample's random loads and store the
+// |g| values straight into rank 0's shared memory (DSMEM); rank 0 then runs
+// Algorithm 3 to its fixed point on the sample alone, with block-wide sums.
 template <int kCTAs>
 __global__ void __cluster_dims__(kCTAs, 1, 1) __launch_bounds__(kBoundCtaThreads)
     k_bound(Layout Lo, SegParam* sp, double kappa, int ns, int force_exact) {
@@ -379,6 +377,7 @@ __global__ void __cluster_dims__(kCTAs, 1, 1) __launch_bounds__(kBoundCtaThreads
         if (rank == 0 && tid == 0) {
             P.done = 0;
             P.w_done = 0;
+            P.next_chunk = 0;
             P.lam_up = (double)kInf;
             P.lam_up32 = kInf;
             P.t_c = 0.0f;
@@ -451,6 +450,7 @@ __global__ void __cluster_dims__(kCTAs, 1, 1) __launch_bounds__(kBoundCtaThreads
     if (tid == 0) {
         P.done = 0;
         P.w_done = 0;
+        P.next_chunk = 0;
         const float e = take_all ? 0.0f : lam * Su / budget;  // uncapped share of the budget
         if (take_all || K >= budget || !(lam > 0.0f)) {
             P.lam_up = (double)kInf;

@@ -3,9 +3,13 @@
 // candidates) as a persistent sm_103a kernel fed by the Tensor Memory
 // Accelerator.
 //
-// Every warp owns whole chunks (chunk c goes to warp c mod (kCW * gridDim.x))
-// and a private ring of shared-memory buffers, each guarded by one "full"
-// mbarrier.  One lane of the warp keeps the ring kRing buffers ahead with
+// Every warp owns whole chunks and a private ring of shared-memory buffers,
+// each guarded by one "full" mbarrier.  A warp's first chunk is fixed by its
+// index; whenever its prefetcher passes the end of a chunk it takes the next
+// one from a counter shared by the grid (so the last round of chunks spreads
+// over the warps that are free, instead of a fixed 6 or 7 chunks per warp),
+// and a small per-warp queue hands the same sequence to the consumer.  One
+// lane of the warp keeps the ring kRing buffers ahead with
 // cp.async.bulk.tensor loads, refilling a buffer as soon as the warp is done
 // with it, so warps never wait for one another and a chunk's lists are
 // ordered by warp shuffles alone.  A warp takes its chunk 1024 coordinates
@@ -25,6 +29,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cstddef>
 #include <cstdint>
 
 #include "gs_device.cuh"
@@ -41,6 +46,7 @@ constexpr int kBufCoords = 32 * kLaneCoords;   // 1024 coordinates per buffer
 constexpr int kRingBudget = 96 * 1024;         // shared memory for the rings of one CTA (2 CTAs per SM)
 constexpr int kRowBytes = 128;
 constexpr long long kWaitLimit = 1ll << 22;    // try_wait polls before giving up
+constexpr int kQueue = 8;                      // per-warp queue of taken chunks (> kRing + 1)
 
 struct StreamArgs {
     Layout Lo;
@@ -48,6 +54,7 @@ struct StreamArgs {
     Lists Ls;
     int n_chunks;
     int* status;
+    int* next_chunk;   // chunks handed out past each warp's first (zero at launch)
 };
 
 __device__ __forceinline__ uint32_t smem_addr(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -160,25 +167,14 @@ __device__ __forceinline__ float4 stage_group(const unsigned char* rp, int first
     }
 }
 
-// The chunks c = first, first + step, ... with the worker and the chunk
-// within the worker advanced without divisions.
+// A chunk index with its worker and its chunk within the worker.
 struct ChunkWalk {
-    int c, m, k, dm, dk;
-    __device__ __forceinline__ ChunkWalk(const Layout& Lo, int first, int step) {
-        c = first;
-        m = c / Lo.cpw;
-        k = c - m * Lo.cpw;
-        dm = step / Lo.cpw;
-        dk = step - dm * Lo.cpw;
-    }
-    __device__ __forceinline__ void next(const Layout& Lo, int step) {
-        c += step;
-        m += dm;
-        k += dk;
-        if (k >= Lo.cpw) {
-            k -= Lo.cpw;
-            ++m;
-        }
+    int c, m, k;
+    __device__ __forceinline__ ChunkWalk(const Layout& Lo, int first) { jump(Lo, first); }
+    __device__ __forceinline__ void jump(const Layout& Lo, int cc) {
+        c = cc;
+        m = cc / Lo.cpw;
+        k = cc - m * Lo.cpw;
     }
     // The chunk's segment and worker-local range [lo, hi).
     __device__ __forceinline__ void range(const Layout& Lo, int& seg, int64_t& lo, int64_t& hi) const {
@@ -223,10 +219,14 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
     unsigned char* base = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(dsm_raw) + 1023) & ~uintptr_t(1023));
     uint64_t* full = reinterpret_cast<uint64_t*>(base + kCW * kRing * kBufBytes);   // [kCW][kRing]
     volatile int* abort_flag = reinterpret_cast<volatile int*>(full + kCW * kRing);
+    // Per-warp queue of the chunks the prefetcher took, in order, for the
+    // consumer (at most kRing + 1 <= 7 outstanding).
+    volatile int* my_q = reinterpret_cast<volatile int*>(full + kCW * kRing) + 4 + (threadIdx.x >> 5) * kQueue;
+    int qt = 0, qh = 0;   // queue tail (prefetcher) and head (consumer)
 
     const Layout& Lo = A.Lo;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int step = gridDim.x * kCW;                      // chunks between two of one warp
+    const int n_first = gridDim.x * kCW;                   // chunks 0 .. n_first - 1 are the warps' first
     if (threadIdx.x == 0) {
         for (int i = 0; i < kCW * kRing; ++i) mbar_init(&full[i], 1);
         *abort_flag = 0;
@@ -239,7 +239,7 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
     const int first = blockIdx.x * kCW + warp;
 
     // Prefetch cursor: the next buffer's row and its chunk's end row.
-    ChunkWalk pc(Lo, first, step);
+    ChunkWalk pc(Lo, first);
     int64_t prow = 0, prow_end = 0;
     if (pc.c < A.n_chunks) {
         int64_t fl, lo, hi;
@@ -257,7 +257,14 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
         ++issued;
         prow += kBufRows;
         if (prow >= prow_end) {
-            pc.next(Lo, step);
+            int nc = 0;
+            if (lane == 0) {
+                nc = n_first + atomicAdd(A.next_chunk, 1);
+                my_q[qt % kQueue] = nc;
+            }
+            nc = __shfl_sync(0xFFFFFFFFu, nc, 0);
+            ++qt;
+            pc.jump(Lo, nc);
             if (pc.c < A.n_chunks) {
                 int64_t fl, lo, hi;
                 int seg;
@@ -280,7 +287,22 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
     int slot = 0, consumed = 0;
     uint32_t full_parity = 0;
     bool live = true;
-    for (ChunkWalk cw(Lo, first, step); cw.c < A.n_chunks; cw.next(Lo, step)) {
+    // The consumer's next chunk: the one the prefetcher took after the
+    // current one; once the prefetcher has stopped (a timeout) the consumer
+    // takes chunks itself, so every chunk still gets its counts written.
+    auto take_next = [&](ChunkWalk& cw) {
+        __syncwarp();
+        int nc = 0;
+        if (qh != qt) {
+            nc = my_q[qh % kQueue];
+            ++qh;
+        } else {
+            if (lane == 0) nc = n_first + atomicAdd(A.next_chunk, 1);
+            nc = __shfl_sync(0xFFFFFFFFu, nc, 0);
+        }
+        cw.jump(Lo, nc);
+    };
+    for (ChunkWalk cw(Lo, first); cw.c < A.n_chunks; take_next(cw)) {
         int seg;
         int64_t lo, hi, flat_lo, r_first, r_end;
         cw.rows(Lo, kInner, flat_lo, r_first, r_end, seg, lo, hi);
@@ -510,8 +532,9 @@ size_t tma_smem_bytes() {
     constexpr int kInner = kDtype == 0 ? 32 : 64;
     constexpr int kBufBytes = (kBufCoords / kInner) * kRowBytes;
     constexpr int kRing = kRingBudget / (kCW * kBufBytes);
-    // alignment slack + buffers + full barriers + abort flag
-    return 1024 + (size_t)kCW * kRing * kBufBytes + (size_t)kCW * kRing * 8 + 16;
+    static_assert(kQueue > kRing + 1, "the chunk queue must hold every chunk the prefetcher can be ahead");
+    // alignment slack + buffers + full barriers + abort flag + chunk queues
+    return 1024 + (size_t)kCW * kRing * kBufBytes + (size_t)kCW * kRing * 8 + 16 + (size_t)kCW * kQueue * 4;
 }
 
 int sm_count_tma() {
@@ -561,6 +584,10 @@ cudaError_t launch_stream_tma(const Layout& Lo, const SegParam* sp, const Lists&
     A.Ls = Ls;
     A.n_chunks = n_chunks;
     A.status = status;
+    // The chunk counter lives in segment 0's parameters (zeroed by the kernel
+    // that wrote the bounds, which this launch waits for).
+    A.next_chunk = reinterpret_cast<int*>(reinterpret_cast<char*>(const_cast<SegParam*>(sp)) +
+                                          offsetof(SegParam, next_chunk));
     // One chunk per warp at a time; two CTAs per SM at most.
     const int grid = std::min((n_chunks + kCW - 1) / kCW, 2 * sm_count_tma());
     cudaError_t e;
