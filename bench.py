@@ -324,6 +324,7 @@ def run_gpu(args):
         rc = gs.gs_sync_status(stream)
         if rc != gs.GS_OK:
             raise RuntimeError(f"device status after the sparsify-only run: {gs.status_string(rc)}")
+    alg3 = run_alg3_state(gs, g, off, kappa, w, idx, val, nnz, stream)
     hybrid = run_hybrid(gs, g, kappa, w, args, dev, stream, n_bd, hbm) if off is None else None
     vbudget = run_variance_budget(gs, g, w, args, dev, stream, n_bd, hbm) if off is None else None
     resp = run_resparsify(gs, g, kappa, w, args, dev, stream, n_bd, hbm, ms) if off is None else None
@@ -348,6 +349,7 @@ def run_gpu(args):
                               "peak": hbm, "frac": round(pipe_gbs / hbm, 4), "unit": "GB/s"},
         "roofline": roofline,
         "sparsify_roofline": sp_only,
+        "algorithm3": alg3,
         "hybrid_code": hybrid,
         "variance_budget": vbudget,
         "average_resparsify": resp,
@@ -406,6 +408,46 @@ def source_digest(kernel):
         with open(os.path.join(src, fn), "rb") as f:
             h.update(f.read())
     return h.hexdigest()
+
+
+def alg3_summary(recs, kappa, seg_lens):
+    """Algorithm 3's state after one call, from its gs_info records (one per
+    worker and segment, `seg_lens` their lengths): lambda's range, how close
+    sum p came to the budget kappa * d_l (1 at the fixed point), the
+    rescalings taken (section 5 runs two) and the segments that needed the
+    exact fallback."""
+    fill = [r["sum_p"] / (kappa * n) for r, n in zip(recs, seg_lens)]
+    lam = [r["lambda"] for r in recs]
+    its = [r["iters_run"] for r in recs]
+    return {"records": len(recs), "lambda_min": min(lam), "lambda_max": max(lam),
+            "sum_p_over_budget_min": round(min(fill), 9), "sum_p_over_budget_max": round(max(fill), 9),
+            "iters_run": {str(k): its.count(k) for k in sorted(set(its))},
+            "capped_total": sum(r["capped"] for r in recs),
+            "exact_fallbacks": sum(1 for r in recs if r["flags"] & 1)}
+
+
+def run_alg3_state(gs, g, off, kappa, w, idx, val, nnz, stream):
+    """One more call, outside every timed region, that returns the gs_info
+    records, summarised by alg3_summary."""
+    import torch
+    M, d = g.shape
+    try:
+        if off is None:
+            info = gs.info_tensor(M)
+            gs.gs_batched_sparsify(g, kappa, w.iters, w.seed, 0, 0, idx, val, nnz, info=info, stream=stream)
+            lens = [d] * M
+        else:
+            L = len(off) - 1
+            info = gs.info_tensor(M * L)
+            gs.gs_segmented_sparsify(g, off, kappa, w.iters, w.seed, 0, 0, idx, val, nnz, info=info, stream=stream)
+            lens = [int(off[l + 1]) - int(off[l]) for _ in range(M) for l in range(L)]
+        torch.cuda.synchronize()
+        rc = gs.gs_sync_status(stream)
+        if rc != gs.GS_OK:
+            return {"error": gs.status_string(rc)}
+        return alg3_summary(gs.decode_info(info), kappa, lens)
+    except Exception as e:  # a report of its own: it never costs the bench line
+        return {"error": f"{type(e).__name__}: {e}"[:300]}
 
 
 def run_hybrid(gs, g, kappa, w, args, dev, stream, n_steps, hbm):
