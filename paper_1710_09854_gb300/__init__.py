@@ -124,6 +124,12 @@ def _ptr(t, name, dtypes=None):
         return None
     if not t.is_cuda:
         raise ValueError(f"{name} must be a CUDA tensor")
+    import torch
+    cur = torch.cuda.current_device()
+    if t.device.index is not None and t.device.index != cur:
+        # The library launches on the current device: memory of another
+        # device would be read through a pointer that is not valid there.
+        raise ValueError(f"{name} is on {t.device} but the current CUDA device is cuda:{cur}")
     if not t.is_contiguous():
         raise ValueError(f"{name} must be contiguous")
     if dtypes is not None and t.dtype not in dtypes:

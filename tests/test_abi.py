@@ -120,3 +120,20 @@ def test_training_loop_entry_points_reject_bad_arguments():
 def test_selftest_timeout_rejects_unknown_kind():
     import paper_1710_09854_gb300 as gs
     assert gs.lib().gs_selftest_timeout(2, None) == gs.GS_ERR_INVALID_ARG
+
+
+def test_tensors_must_live_on_the_current_device(monkeypatch):
+    """The binding refuses a tensor of another device before any call."""
+    import types
+    import torch
+    import paper_1710_09854_gb300 as gs
+    monkeypatch.setattr(torch.cuda, "current_device", lambda: 0)
+    t = types.SimpleNamespace(is_cuda=True, device=torch.device("cuda", 1), dtype=torch.float32,
+                              is_contiguous=lambda: True, data_ptr=lambda: 4096)
+    with pytest.raises(ValueError, match="current CUDA device"):
+        gs._ptr(t, "g")
+    t.device = torch.device("cuda", 0)
+    assert gs._ptr(t, "g") == 4096
+    cpu = types.SimpleNamespace(is_cuda=False)
+    with pytest.raises(ValueError, match="CUDA tensor"):
+        gs._ptr(cpu, "g")
