@@ -335,6 +335,13 @@ def run_gpu(args):
     if not args.no_e2e and off is None:
         e2e = run_e2e(gs, g, kappa, w, args, dev, stream, ws)
 
+    # ---- every configuration (GPU only), after the headline's own buffers are freed
+    configs = None
+    if not args.no_configs and args.workers is None and args.dim is None:
+        del idx, val, idx_rows, val_rows, out
+        torch.cuda.empty_cache()
+        configs = run_configs(gs, args, dev, stream, hbm, rank)
+
     result = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
@@ -359,10 +366,106 @@ def run_gpu(args):
         "gpu_launches": launches,
         "clocks": clk,
         "e2e": e2e,
+        "configs": configs,
     }
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_baseline_sample(g, off, kappa, w, budget_s=args.cpu_seconds)
     return result, rank
+
+
+# Every configuration of the path, each timed with the call bench.py times
+# for it: c1-c3 and c5 through gs_sparsify_aggregate, c4 through
+# gs_segmented_sparsify_aggregate.
+CONFIG_SWEEP = (("c1", None, None), ("c2", None, None), ("c3", None, None), ("c4", None, None),
+                ("c5", 0.001, "f32"), ("c5", 0.01, "f32"), ("c5", 0.1, "f32"),
+                ("c5", 0.001, "bf16"), ("c5", 0.01, "bf16"), ("c5", 0.1, "bf16"))
+
+
+def run_configs(gs, args, dev, stream, hbm, rank):
+    """One row per configuration: time per step of the fused call (steps
+    1-6), coordinates/s, the whole step against its algorithmic bytes (one
+    read of g, the kept pairs written and read back, the dense sum written)
+    and the streaming kernel against its one read of g, both as fractions of
+    the measured copy peak.  The step time comes from a loop with no events
+    between launches; the streaming kernel's time from a second loop in which
+    only that kernel carries events."""
+    import torch
+    rows = []
+    for name, kappa_o, dtype_o in CONFIG_SWEEP:
+        try:
+            w, g, off, kappa, dtype = make_workload(name, kappa_o, dtype_o, rank)
+            M, d = g.shape
+            esz = g.element_size()
+            idx = torch.empty((M, d), dtype=torch.int32, device=dev)
+            val = torch.empty((M, d), dtype=torch.float32, device=dev)
+            nnz = torch.empty(M, dtype=torch.int32, device=dev)
+            out = torch.empty(d, dtype=torch.float32, device=dev)
+
+            def step(t):
+                if off is None:
+                    gs.gs_sparsify_aggregate(g, kappa, w.iters, w.seed, t, 0, idx, val, nnz, out, stream=stream)
+                else:
+                    gs.gs_segmented_sparsify_aggregate(g, off, kappa, w.iters, w.seed, t, 0, idx, val, nnz, out,
+                                                       stream=stream)
+            n = 30 if name == "c5" else 200
+            for t in range(5):
+                step(t)
+            torch.cuda.synchronize()
+            if gs.gs_sync_status(stream) != gs.GS_OK:
+                raise RuntimeError("device status after warm-up")
+            kept = int(nnz.sum().item())
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for t in range(n):
+                step(5 + t)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            ms = max_over_ranks(e0.elapsed_time(e1) / n, dev)
+            gs.gs_set_option(gs.GS_OPT_KERNEL_TIMING, 2)
+            gs.gs_kernel_times()
+            for t in range(n):
+                step(5 + n + t)
+            torch.cuda.synchronize()
+            kt = gs.gs_kernel_times()
+            gs.gs_set_option(gs.GS_OPT_KERNEL_TIMING, 0)
+            if gs.gs_sync_status(stream) != gs.GS_OK:
+                raise RuntimeError("device status after timing")
+            sk = "k_stream_tma" if kt.get("k_stream_tma", (0, 0))[1] else "k_stream"
+            s_ms = kt[sk][0] / max(kt[sk][1], 1)
+            b_sp, b_ag = algorithmic_bytes(M, d, esz, kept)
+            step_gbs = (b_sp + b_ag) / (ms / 1e3) / 1e9
+            s_gbs = M * d * esz / (s_ms / 1e3) / 1e9
+            rows.append({"workload": w.name, "M": M, "d": d, "kappa": kappa, "dtype": dtype, "iters": w.iters,
+                         "api": "gs_segmented_sparsify_aggregate" if off is not None else "gs_sparsify_aggregate",
+                         "steps": n, "ms_per_step": round(ms, 5), "coords_per_s": M * d / (ms / 1e3),
+                         "nnz_per_step": kept, "algorithmic_bytes": b_sp + b_ag,
+                         "step_gbs": round(step_gbs, 1), "step_frac": round(step_gbs / hbm, 4),
+                         "stream_kernel": sk, "stream_ms": round(s_ms, 5), "stream_gbs": round(s_gbs, 1),
+                         "stream_frac": round(s_gbs / hbm, 4), "peak": hbm,
+                         "l2": ("fits in L2" if M * d * esz < L2_BYTES else "exceeds L2")})
+            del g, idx, val, nnz, out
+        except Exception as e:  # one failed row never costs the bench line
+            rows.append({"workload": name, "kappa": kappa_o, "dtype": dtype_o,
+                         "error": f"{type(e).__name__}: {e}"[:300]})
+        torch.cuda.empty_cache()
+    return rows
+
+
+def host_cpu():
+    """The host's logical CPU count and CPU model (lscpu's model name, else
+    the platform's machine name)."""
+    import platform
+    model = None
+    try:
+        outp = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in outp.splitlines():
+            if line.split(":")[0].strip() in ("Model name", "Model"):
+                model = line.split(":", 1)[1].strip()
+                if line.startswith("Model name"):
+                    break
+    except (OSError, subprocess.SubprocessError):
+        pass
+    return {"nproc": os.cpu_count(), "model": model or platform.machine()}
 
 
 def run_e2e(gs, g, kappa, w, args, dev, stream, ws):
@@ -711,7 +814,7 @@ def cpu_baseline_sample(g, off, kappa, w, budget_s=15.0):
         if time.perf_counter() - t0 > budget_s:
             break
     el = time.perf_counter() - t0
-    return {"value": done / el, "unit": UNIT, "cores": 1, "kind": "oracle",
+    return {"value": done / el, "unit": UNIT, "cores": 1, "kind": "oracle", "host": host_cpu(),
             "sample": f"{done // d} of {M} workers at full d={d} (sparsify + sparse sum), {el:.1f} s"}
 
 
@@ -759,7 +862,8 @@ def run_reference(args):
            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
            "config": {"workload": w.name, "M": w.M, "d": w.d, "kappa": kappa, "iters": w.iters, "dtype": w.dtype,
                       "api": "oracle (C, fp64)", "parallelism": f"replicas{ws}"},
-           "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+           "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample,
+                            "host": host_cpu()},
            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     if ws > 1:
         import torch.distributed as dist
@@ -785,6 +889,7 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-lr", action="store_true", help="skip the section 5.1 training-loop report")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--no-configs", action="store_true", help="skip the sweep over every configuration")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

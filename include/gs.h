@@ -54,7 +54,10 @@ typedef enum {
     GS_ERR_CAPACITY = 3,    /* more kept entries than the output capacity */
     GS_ERR_NONFINITE = 4,   /* a gradient contains NaN or Inf */
     GS_ERR_TIMEOUT = 5,     /* a bounded device-side wait ran out */
-    GS_ERR_INTERNAL = 6     /* library invariant violated */
+    GS_ERR_INTERNAL = 6,    /* library invariant violated */
+    GS_ERR_ABORTED = 7      /* a bounded wait ran out and a kernel then left with copies into its
+                               shared memory still in flight (the memory system stopped answering):
+                               every result since the previous status check is suspect */
 } gs_status;
 
 typedef enum { GS_DTYPE_F32 = 0, GS_DTYPE_BF16 = 1 } gs_dtype;
@@ -289,10 +292,12 @@ gs_status gs_sparsify_aggregate(const void* g, int dtype, int M, int64_t d, doub
  *   d       1 <= d <= 4194304 (2^22); a larger d returns GS_ERR_INVALID_ARG
  *           at once and gs_last_error() says why
  *   info    device, one gs_info (may be NULL)
- *   status  device, one int32 (may be NULL): receives, in stream order, the
- *           gs_status of the device-side checks of this call (GS_OK,
- *           GS_ERR_NONFINITE, GS_ERR_TIMEOUT, ...).  Such errors are not
- *           recorded for gs_sync_status.
+ *   status  device, one int32 (required; NULL returns GS_ERR_INVALID_ARG):
+ *           receives, in stream order, the gs_status of the device-side
+ *           checks of this call (GS_OK, GS_ERR_NONFINITE, GS_ERR_TIMEOUT,
+ *           ...).  It is the only place these errors are reported: they are
+ *           not recorded for gs_sync_status, whose status word this call
+ *           never touches (it lives in memory the library allocates).
  * Scratch is one static device array of about 48 MiB (sized for d = 2^22)
  * and one static status word; every GPU that loads the library may hold
  * them until the process exits.  The first call on a device looks up their

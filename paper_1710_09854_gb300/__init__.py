@@ -17,7 +17,8 @@ import numpy as np
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libgs.so")
 
-GS_OK, GS_ERR_INVALID_ARG, GS_ERR_CUDA, GS_ERR_CAPACITY, GS_ERR_NONFINITE, GS_ERR_TIMEOUT, GS_ERR_INTERNAL = range(7)
+(GS_OK, GS_ERR_INVALID_ARG, GS_ERR_CUDA, GS_ERR_CAPACITY, GS_ERR_NONFINITE, GS_ERR_TIMEOUT, GS_ERR_INTERNAL,
+ GS_ERR_ABORTED) = range(8)
 GS_DTYPE_F32, GS_DTYPE_BF16 = 0, 1
 GS_OPT_FORCE_EXACT_SOLVE, GS_OPT_SAMPLE_SIZE, GS_OPT_KERNEL_TIMING, GS_OPT_STREAM_PATH = 1, 2, 3, 4
 
@@ -274,10 +275,11 @@ def gs_sparsify(g, kappa, iters, seed, step, worker, idx, val, nnz, stream=None)
            "gs_sparsify")
 
 
-def gs_sparsify_noalloc(g, kappa, iters, seed, step, worker, idx, val, nnz, info=None, status=None, stream=None):
+def gs_sparsify_noalloc(g, kappa, iters, seed, step, worker, idx, val, nnz, status, info=None, stream=None):
     """gs_sparsify on the library's static scratch (d <= 2^22): the call
     itself allocates no device memory.  `status` (one int32 on the device,
-    optional) receives the call's device-side status code."""
+    required) receives the call's device-side status code: the only place
+    such errors are reported for this call."""
     import torch
     if idx.numel() < g.numel() or val.numel() < g.numel():
         raise ValueError("idx / val need capacity d")

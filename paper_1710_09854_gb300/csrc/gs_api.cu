@@ -353,7 +353,8 @@ __global__ void k_noalloc_status(const int* bits, int32_t* code) {
     grid_dep_wait();
     const int h = *bits;
     int32_t c = GS_OK;
-    if (h & kStNonfinite) c = GS_ERR_NONFINITE;
+    if (h & kStAborted) c = GS_ERR_ABORTED;
+    else if (h & kStNonfinite) c = GS_ERR_NONFINITE;
     else if (h & kStCapacity) c = GS_ERR_CAPACITY;
     else if (h & kStInvalid) c = GS_ERR_INVALID_ARG;
     else if (h & kStTimeout) c = GS_ERR_TIMEOUT;
@@ -366,6 +367,11 @@ gs_status run_noalloc(const float* g, int64_t d, double kappa, int iters, uint64
                       cudaStream_t st) {
     g_last_error[0] = '\0';
     if (!g || !idx || !val || !nnz || d < 1 || bad_kappa(kappa) || iters < 0) return GS_ERR_INVALID_ARG;
+    if (!status) {
+        // The caller's word is the one place this call's device-side errors go.
+        snprintf(g_last_error, sizeof(g_last_error), "gs_sparsify_noalloc: the status word is required");
+        return GS_ERR_INVALID_ARG;
+    }
     if ((reinterpret_cast<uintptr_t>(g) % sizeof(float)) != 0) return GS_ERR_INVALID_ARG;
     if (d > kNoAllocMaxD) {
         snprintf(g_last_error, sizeof(g_last_error),
@@ -421,7 +427,7 @@ gs_status run_noalloc(const float* g, int64_t d, double kappa, int iters, uint64
     }
     if (e == cudaSuccess) e = launch_solve(Lo, w.sp, w.ls, 1, kappa, iters, force, s->status, info, st, d);
     if (e == cudaSuccess) e = launch_compact(Lo, w.sp, w.ls, n_chunks, idx, val, nnz, d, s->status, st);
-    if (e == cudaSuccess && status) {
+    if (e == cudaSuccess) {
         k_noalloc_status<<<1, 1, 0, st>>>(s->status, status);
         e = cudaGetLastError();
         if (e != cudaSuccess) set_launch_error_site("k_noalloc_status");
@@ -443,6 +449,7 @@ const char* gs_status_string(int status) {
         case GS_ERR_NONFINITE: return "GS_ERR_NONFINITE";
         case GS_ERR_TIMEOUT: return "GS_ERR_TIMEOUT";
         case GS_ERR_INTERNAL: return "GS_ERR_INTERNAL";
+        case GS_ERR_ABORTED: return "GS_ERR_ABORTED";
         default: return "GS_UNKNOWN_STATUS";
     }
 }
@@ -460,6 +467,7 @@ gs_status gs_sync_status(void* stream) {
     GS_TRY(cudaMemcpyAsync(&h, s->status, sizeof(int), cudaMemcpyDeviceToHost, st));
     GS_TRY(cudaMemsetAsync(s->status, 0, sizeof(int), st));
     GS_TRY(cudaStreamSynchronize(st));
+    if (h & kStAborted) return GS_ERR_ABORTED;
     if (h & kStNonfinite) return GS_ERR_NONFINITE;
     if (h & kStCapacity) return GS_ERR_CAPACITY;
     if (h & kStInvalid) return GS_ERR_INVALID_ARG;

@@ -28,6 +28,7 @@ enum : int {
     kStNonfinite = 1 << 4,
     kStTimeout = 1 << 5,
     kStInternal = 1 << 6,
+    kStAborted = 1 << 7,   // a kernel left with copies into its shared memory still in flight
 };
 
 // Segment flags.

@@ -540,16 +540,7 @@ __global__ void __launch_bounds__(kThreads) k_solve_eps(const __grid_constant__ 
     }
 }
 
-int sm_count_eps() {
-    static int n = 0;
-    if (n == 0) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-        if (n <= 0) n = 1;
-    }
-    return n;
-}
+int sm_count_eps() { return device_sm_count(); }
 
 }  // namespace
 

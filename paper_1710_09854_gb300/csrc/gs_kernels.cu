@@ -29,6 +29,7 @@
 #include <cfloat>
 #include <cmath>
 #include <algorithm>
+#include <atomic>
 #include <cstdint>
 
 #include "gs_device.cuh"
@@ -1444,18 +1445,21 @@ __global__ void __launch_bounds__(kThreads) k_tiles(const __grid_constant__ AggA
     }
 }
 
-int sm_count() {
-    static int n = 0;
-    if (n == 0) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-        if (n <= 0) n = 1;
-    }
-    return n;
-}
+int sm_count() { return device_sm_count(); }
 
 }  // namespace
+
+int device_sm_count() {
+    constexpr int kMaxDev = 64;
+    static std::atomic<int> cache[kMaxDev];   // 0 = not looked up yet (static storage: zero-initialised)
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+    int n = (dev >= 0 && dev < kMaxDev) ? cache[dev].load(std::memory_order_relaxed) : 0;
+    if (n > 0) return n;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 1;
+    if (dev >= 0 && dev < kMaxDev) cache[dev].store(n, std::memory_order_relaxed);   // same value from any thread
+    return n;
+}
 
 // ---------------------------------------------------------------------------
 // Host launchers

@@ -126,5 +126,7 @@ void set_launch_error_site(const char* where);
 const char* launch_error_site();
 int agg_tiles(int64_t d);
 int chunk_size();
+// Multiprocessor count of the current device (looked up once per device ordinal).
+int device_sm_count();
 
 }  // namespace gs

@@ -31,6 +31,7 @@
 #include <algorithm>
 #include <cstddef>
 #include <cstdint>
+#include <mutex>
 
 #include "gs_device.cuh"
 #include "gs_launch.h"
@@ -489,26 +490,35 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
         }
     }
     // After a timeout, wait (bounded) for the copies still in flight into this
-    // warp's ring (consumed counts the buffers whose wait succeeded).
-    for (int n = consumed; n < issued; ++n) mbar_wait(&my_full[n % kRing], (uint32_t)((n / kRing) & 1));
+    // warp's ring (consumed counts the buffers whose wait succeeded).  The wait
+    // is bounded too: a copy that has not landed after another 2^22 polls
+    // means the memory system no longer answers, and waiting forever would
+    // hang the GPU for every later user of it.  Leaving instead records
+    // kStAborted, which the host reports as GS_ERR_ABORTED: a copy may still
+    // land in shared memory the CTA has given up, so every result since the
+    // last status check is suspect.
+    bool landed = true;
+    for (int n = consumed; n < issued; ++n) landed = mbar_wait(&my_full[n % kRing], (uint32_t)((n / kRing) & 1)) && landed;
+    if (!__all_sync(0xFFFFFFFFu, landed) && lane == 0) atomicOr(A.status, kStAborted);
 }
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
+// The driver's tensor-map encoder, looked up once per process (host threads
+// making their first call at the same time wait for one lookup).
 EncodeTiledFn encode_fn() {
     static EncodeTiledFn fn = nullptr;
-    static bool tried = false;
-    if (!tried) {
-        tried = true;
+    static std::once_flag once;
+    std::call_once(once, [] {
         void* p = nullptr;
         cudaDriverEntryPointQueryResult q;
         if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
                 cudaSuccess &&
             q == cudaDriverEntryPointSuccess)
             fn = reinterpret_cast<EncodeTiledFn>(p);
-    }
+    });
     return fn;
 }
 
@@ -537,16 +547,7 @@ size_t tma_smem_bytes() {
     return 1024 + (size_t)kCW * kRing * kBufBytes + (size_t)kCW * kRing * 8 + 16 + (size_t)kCW * kQueue * 4;
 }
 
-int sm_count_tma() {
-    static int n = 0;
-    if (n == 0) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
-        if (n <= 0) n = 1;
-    }
-    return n;
-}
+int sm_count_tma() { return device_sm_count(); }
 
 }  // namespace
 

@@ -9,6 +9,9 @@ Tolerances (applied by every GPU parity test):
   sparse sum   |gpu - oracle| <= 1e-5 * sum_m |Q_m[i]| (relative to the
                magnitude of the terms, since terms of both signs may cancel)
 """
+import concurrent.futures as cf
+import os
+
 import numpy as np
 
 import oracle
@@ -41,8 +44,13 @@ def compare_sparse(idx, val, g_row, kappa, iters, seed, step, worker, i0=0, ref=
     else:
         ri, rv, info = ref
     ri = ri.astype(np.int64)
-    common, ia, ib = np.intersect1d(idx, ri, assume_unique=True, return_indices=True)
-    only = np.setdiff1d(np.union1d(idx, ri), common)
+    if idx.size == ri.size and np.array_equal(idx, ri):
+        # the usual case: identical kept sets (no sort needed)
+        common, ia, ib = idx, np.arange(idx.size), np.arange(idx.size)
+        only = np.empty(0, dtype=np.int64)
+    else:
+        common, ia, ib = np.intersect1d(idx, ri, assume_unique=True, return_indices=True)
+        only = np.setdiff1d(np.union1d(idx, ri), common)
     lam = info["lambda"]
     for i in only:
         a = abs(float(g_row[i - i0]))
@@ -61,8 +69,22 @@ def compare_sum(out_gpu, idx_list, val_list, d):
     ref = oracle.aggregate(idx_list, val_list, d)
     mag = np.zeros(d, dtype=np.float64)
     for i, v in zip(idx_list, val_list):
-        np.add.at(mag, np.asarray(i, dtype=np.int64), np.abs(np.asarray(v, dtype=np.float64)))
+        i = np.asarray(i, dtype=np.int64)
+        assert i.size < 2 or np.all(np.diff(i) > 0), "oracle lists are strictly ascending"
+        mag[i] += np.abs(np.asarray(v, dtype=np.float64))   # distinct indices within one list
     err = np.abs(np.asarray(out_gpu, dtype=np.float64) - ref.astype(np.float64))
     bad = err > V_RTOL * mag
     assert not bad.any(), f"sparse sum differs at {int(bad.sum())} coordinates"
     return ref
+
+
+def oracle_rows(fn, rows, *args, threads=None, **kw):
+    """fn(rows[m], *args, worker=m, **kw) for every worker row, run on host
+    threads (the oracle is plain C called through ctypes, which releases the
+    interpreter lock, and keeps no state between calls).  Returns the results
+    in worker order."""
+    n = len(rows)
+    threads = threads or min(n, os.cpu_count() or 1)
+    with cf.ThreadPoolExecutor(max_workers=max(1, threads)) as ex:
+        futs = [ex.submit(fn, rows[m], *args, worker=m, **kw) for m in range(n)]
+        return [f.result() for f in futs]

@@ -5,7 +5,7 @@ import pytest
 
 import oracle
 import workloads
-from parity import compare_probabilities, compare_sparse, compare_sum
+from parity import compare_probabilities, compare_sparse, compare_sum, oracle_rows
 
 pytestmark = pytest.mark.gpu
 
@@ -316,6 +316,12 @@ def test_pipeline_host_matches_device_path(gs):
 # Full-size workloads in the launch configuration bench.py times.
 # ---------------------------------------------------------------------------
 def _full_check(gs, g_dev, kappa, iters, seed=1, step=0, workers=None, offsets=None, dtype="f32"):
+    """The fused call bench.py times (gs_sparsify_aggregate, or the layer-wise
+    gs_segmented_sparsify_aggregate) on a full-size input; the separate calls
+    (sparsify, then gs_sparse_aggregate) must equal it bit for bit.  Every
+    worker in `workers` (default: all) is compared with the oracle element by
+    element, and the fused sum with the oracle's worker-order sum of the
+    oracle's own lists over all M workers.  Returns the boundary flips."""
     import torch
     M, d = g_dev.shape
     idx = torch.empty((M, d), dtype=torch.int32, device="cuda")
@@ -323,49 +329,43 @@ def _full_check(gs, g_dev, kappa, iters, seed=1, step=0, workers=None, offsets=N
     nnz = torch.empty(M, dtype=torch.int32, device="cuda")
     out = torch.empty(d, dtype=torch.float32, device="cuda")
     if offsets is None:
-        gs.gs_batched_sparsify(g_dev, kappa, iters, seed, step, 0, idx, val, nnz)
+        gs.gs_sparsify_aggregate(g_dev, kappa, iters, seed, step, 0, idx, val, nnz, out)
     else:
-        gs.gs_segmented_sparsify(g_dev, offsets, kappa, iters, seed, step, 0, idx, val, nnz)
-    gs.gs_sparse_aggregate([idx[m] for m in range(M)], [val[m] for m in range(M)], nnz, d, out)
+        gs.gs_segmented_sparsify_aggregate(g_dev, offsets, kappa, iters, seed, step, 0, idx, val, nnz, out)
     assert gs.gs_sync_status() == gs.GS_OK
-    if offsets is not None:
-        _check_segmented_fused(gs, g_dev, offsets, kappa, iters, seed, step, idx, val, nnz)
+    # The separate calls equal the fused one bit for bit (lists, counts, sum).
+    idx2, val2 = torch.full_like(idx, -1), torch.zeros_like(val)
+    nnz2, out2 = torch.zeros_like(nnz), torch.full_like(out, float("nan"))
     if offsets is None:
-        # The fused call (compaction + sum in one chain) equals the two calls bit for bit.
-        idx2 = torch.empty_like(idx)
-        val2 = torch.empty_like(val)
-        nnz2 = torch.empty_like(nnz)
-        out2 = torch.empty_like(out)
-        gs.gs_sparsify_aggregate(g_dev, kappa, iters, seed, step, 0, idx2, val2, nnz2, out2)
-        assert gs.gs_sync_status() == gs.GS_OK
-        assert torch.equal(nnz2, nnz)
-        assert torch.equal(out2, out)
-        for m in range(M):
-            k = int(nnz[m].item())
-            assert torch.equal(idx2[m, :k], idx[m, :k]) and torch.equal(val2[m, :k], val[m, :k])
-        del idx2, val2
+        gs.gs_batched_sparsify(g_dev, kappa, iters, seed, step, 0, idx2, val2, nnz2)
+    else:
+        gs.gs_segmented_sparsify(g_dev, offsets, kappa, iters, seed, step, 0, idx2, val2, nnz2)
+    gs.gs_sparse_aggregate([idx2[m] for m in range(M)], [val2[m] for m in range(M)], nnz2, d, out2)
+    assert gs.gs_sync_status() == gs.GS_OK
+    assert torch.equal(nnz2, nnz)
+    assert torch.equal(out2, out)
+    for m in range(M):
+        k = int(nnz[m].item())
+        assert torch.equal(idx2[m, :k], idx[m, :k]) and torch.equal(val2[m, :k], val[m, :k])
+    del idx2, val2, out2
     g_host = g_dev.float().cpu().numpy() if dtype == "bf16" else g_dev.cpu().numpy()
+    rows = [g_host[m] for m in range(M)]
+    if offsets is None:
+        refs = oracle_rows(oracle.sparsify, rows, kappa, iters, seed, step)
+    else:
+        refs = oracle_rows(oracle.segmented_sparsify, rows, offsets, kappa, iters, seed, step)
     n = nnz.cpu().numpy()
     workers = range(M) if workers is None else workers
-    il, vl = [], []
     flips = 0
-    for m in range(M):
+    for m in workers:
+        gi = idx[m, :n[m]].cpu().numpy()
+        gv = val[m, :n[m]].cpu().numpy()
         if offsets is None:
-            ref = oracle.sparsify(g_host[m], kappa, iters, seed, step, m)
+            flips += compare_sparse(gi, gv, rows[m], kappa, iters, seed, step, m, ref=refs[m])
         else:
-            ri, rv, _ = oracle.segmented_sparsify(g_host[m], offsets, kappa, iters, seed, step, m)
-            ref = (ri, rv, {"lambda": float("nan")})
-        il.append(ref[0])
-        vl.append(ref[1])
-        if m in workers:
-            gi = idx[m, :n[m]].cpu().numpy()
-            gv = val[m, :n[m]].cpu().numpy()
-            if offsets is None:
-                flips += compare_sparse(gi, gv, g_host[m], kappa, iters, seed, step, m, ref=ref)
-            else:
-                np.testing.assert_array_equal(gi, ref[0])
-                np.testing.assert_allclose(gv, ref[1], rtol=1e-5)
-    compare_sum(out.cpu().numpy(), il, vl, d)
+            np.testing.assert_array_equal(gi, refs[m][0])
+            np.testing.assert_allclose(gv, refs[m][1], rtol=1e-5)
+    compare_sum(out.cpu().numpy(), [r[0] for r in refs], [r[1] for r in refs], d)
     return flips
 
 
@@ -380,28 +380,41 @@ def test_full_student_t_d2p24_m16(gs):
     torch.cuda.empty_cache()
 
 
-def test_full_resnet50_layerwise(gs):
+def test_full_resnet50_layerwise_m8(gs):
+    """The layer-wise workload at its configured size: 8 workers x 161
+    ResNet-50-shaped layers (25,557,032 coordinates), every worker and the sum."""
     import torch
-    g, off = workloads.device_layerwise(2)
-    _full_check(gs, g, workloads.C4.kappa, workloads.C4.iters, offsets=off)
+    w = workloads.C4
+    g, off = workloads.device_layerwise(w.M, seed0=w.data_seed)
+    _full_check(gs, g, w.kappa, w.iters, w.seed, w.step, offsets=off)
     del g
     torch.cuda.empty_cache()
 
 
 def test_full_logreg_c2(gs):
+    """The logistic-regression workload at its configured size, all 8 workers."""
     import torch
-    g = workloads.device_logreg(8, 1 << 20)
-    _full_check(gs, g, workloads.C2.kappa, workloads.C2.iters, workers=[0, 7])
+    w = workloads.C2
+    g = workloads.device_logreg(w.M, w.d, seed0=w.data_seed)
+    _full_check(gs, g, w.kappa, w.iters, w.seed, w.step)
     del g
     torch.cuda.empty_cache()
 
 
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
 @pytest.mark.parametrize("kappa", [0.001, 0.01, 0.1])
-def test_lognormal_outliers_bf16_and_f32(gs, kappa):
+def test_full_lognormal_outliers_c5(gs, kappa, dtype):
+    """The large workload at its configured size: 8 workers x 2^27 log-normal
+    magnitudes with 0.1% outliers, fp32 and bf16, each kappa of the sweep;
+    every worker compared with the oracle and the fused sum over all 8."""
     import torch
-    g = workloads.device_lognormal(2, 1 << 23, seed0=5)
-    _full_check(gs, g, kappa, 3, workers=[0, 1])
-    _full_check(gs, g.to(torch.bfloat16), kappa, 3, workers=[1], dtype="bf16")
+    w = workloads.C5
+    g = workloads.device_lognormal(w.M, w.d, seed0=w.data_seed)
+    if dtype == "bf16":
+        g = workloads.device_to_bf16(g)
+        torch.cuda.empty_cache()
+    flips = _full_check(gs, g, kappa, w.iters, w.seed, w.step, dtype=dtype)
+    assert flips <= 2
     del g
     torch.cuda.empty_cache()
 
