@@ -24,6 +24,12 @@ class Info(ctypes.Structure):
                 "sum_p": self.sum_p, "l1": self.l1}
 
 
+class DenseModel(ctypes.Structure):
+    """Quantized model of the dense code (frequencies over 2^15)."""
+    _fields_ = [("len_f", ctypes.c_uint32 * 31), ("len_c", ctypes.c_uint32 * 32), ("bit_f1", ctypes.c_uint32 * 30),
+                ("val_f", ctypes.c_uint32 * 3), ("val_c", ctypes.c_uint32 * 4)]
+
+
 class OracleError(RuntimeError):
     def __init__(self, code):
         super().__init__(f"oracle returned status {code}")
@@ -74,6 +80,13 @@ def lib():
         L.gso_sparsify_eps.argtypes = [ctypes.c_void_p, ctypes.c_int64, ctypes.c_double, ctypes.c_uint64,
                                        ctypes.c_uint32, ctypes.c_uint32, ctypes.c_int64, ctypes.c_void_p,
                                        ctypes.c_void_p, P(ctypes.c_int64), P(Info)]
+        L.gso_dense_model_build.argtypes = [ctypes.c_int64, ctypes.c_int64, ctypes.c_int64, ctypes.c_int64,
+                                            ctypes.POINTER(DenseModel)]
+        L.gso_dense_encode.argtypes = [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_void_p,
+                                       ctypes.c_int64, P(ctypes.c_int64)]
+        L.gso_dense_decode.argtypes = [ctypes.c_void_p, ctypes.c_int64, ctypes.c_int64, ctypes.c_void_p]
+        for f in ("gso_dense_model_build", "gso_dense_encode", "gso_dense_decode"):
+            getattr(L, f).restype = ctypes.c_int
         for f in ("gso_closed_form_lambda", "gso_probabilities_eps", "gso_sparsify_eps", "gso_greedy_lambda", "gso_greedy_pvector", "gso_probabilities", "gso_sparsify",
                   "gso_segmented_sparsify", "gso_aggregate", "gso_average", "gso_hybrid_encode", "gso_hybrid_decode"):
             getattr(L, f).restype = ctypes.c_int
@@ -253,3 +266,34 @@ def ternary_bits(d, n_neg, n_pos, n_cap):
 def comm_bits(d, n_capped, sum_p_uncapped, b=32):
     """One worker's summand of H(T, M) for one step (section 5)."""
     return lib().gso_comm_bits(int(d), int(n_capped), float(sum_p_uncapped), int(b))
+
+
+def dense_model(d, n_pos, n_neg, n_cap):
+    """Frequencies (over 2^15) of the dense code's models: bit lengths of the
+    zero runs, each bit below the leading one, and the non-zero values."""
+    m = DenseModel()
+    _check(lib().gso_dense_model_build(int(d), int(n_pos), int(n_neg), int(n_cap), ctypes.byref(m)))
+    return {"len_f": np.array(m.len_f, np.int64), "len_c": np.array(m.len_c, np.int64),
+            "bit_f1": np.array(m.bit_f1, np.int64), "val_f": np.array(m.val_f, np.int64),
+            "val_c": np.array(m.val_c, np.int64)}
+
+
+def dense_encode(qt, log2_k=9):
+    """Section 3.3: entropy code of q~ in {0, +1, -1, 2}^d (int8 values) as
+    16-bit words (header, chunk directory, one rANS stream per chunk of
+    2^log2_k non-zero symbols)."""
+    qt = np.ascontiguousarray(qt, dtype=np.int8)
+    n = ctypes.c_int64()
+    _check(lib().gso_dense_encode(qt.ctypes.data, qt.size, int(log2_k), None, 0, ctypes.byref(n)))
+    out = np.empty(n.value, dtype=np.uint16)
+    _check(lib().gso_dense_encode(qt.ctypes.data, qt.size, int(log2_k), out.ctypes.data, out.size,
+                                  ctypes.byref(n)))
+    return out
+
+
+def dense_decode(words, d):
+    """Inverse of dense_encode: q~ as int8 values."""
+    words = np.ascontiguousarray(words, dtype=np.uint16)
+    qt = np.empty(int(d), dtype=np.int8)
+    _check(lib().gso_dense_decode(words.ctypes.data, words.size, int(d), qt.ctypes.data))
+    return qt

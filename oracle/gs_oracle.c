@@ -563,3 +563,329 @@ GSO_EXPORT int gso_sparsify_eps(const float* g, int64_t d, double eps, uint64_t 
     *nnz = n;
     return GSO_OK;
 }
+
+/* ------------------------------------------------------------------------
+ * Section 3.3, last paragraph: the dense code q~ in {0, +1, -1, 2}^d of
+ * Q(g) -- q~_i = 0 where coordinate i is dropped, sign(g_i) where it is kept
+ * with p_i < 1, and 2 where p_i = 1 -- entropy coded under the static model
+ * the paper prices it with, P(s) = d_s / d (d_s = number of coordinates with
+ * symbol s), whose ideal length is sum_s d_s log2(d / d_s) <= 2d bits.
+ *
+ * The coder writes that model as one event per non-zero symbol: the run of
+ * zeros before it and its value.  Under the model the run length g is
+ * geometric, P(g) = (1 - p0) p0^g with p0 = d_0 / d, and the value given
+ * "non-zero" has P(t) = d_t / (d - d_0); the product P(g) P(t) is exactly
+ * the model's probability p0^g (d_t / d) of "g zeros, then t", so coding the
+ * events costs what coding the symbols one by one would.  The run is coded
+ * through v = g + 1: first its bit length l = floor(log2 v), with
+ * P(l) = p0^(2^l - 1) (1 - p0^(2^l)), then its l bits below the leading one,
+ * each on its own, bit k being 1 with probability p0^(2^k) / (1 + p0^(2^k))
+ * -- these are independent given l and multiply back to P(g) exactly.
+ *
+ * Layout of one vector's code (16-bit words, multi-word integers low word
+ * first):
+ *   header     d (2 words), d_{+1} (2), d_{-1} (2), d_2 (2), log2 K (1)
+ *   directory  per chunk of K consecutive non-zero symbols: the index of its
+ *              first non-zero (2 words) and its stream length in words (1)
+ *   streams    one rANS stream per chunk, in chunk order.
+ * A chunk's first non-zero is placed by the directory (its run is not
+ * coded); every later one codes its run from the previous non-zero; the
+ * zeros after the last non-zero are implied by d.
+ *
+ * rANS (Duda's asymmetric numeral systems, range variant): model
+ * probabilities are integer frequencies f_s over M = 2^15 with cumulative
+ * starts c_s; the state x lives in [2^15, 2^31); the encoder starts from
+ * x = 2^15, visits the chunk's coding steps in reverse order, and before
+ * each step emits the low 16 bits of x (x >>= 16) while x >= f_s 2^16, then
+ * sets x = floor(x / f_s) M + (x mod f_s) + c_s; at the end it flushes x as
+ * two words.  A chunk's stream is the flushed state (high word first)
+ * followed by the emitted words in reverse order of emission, so that the
+ * decoder reads it forward: slot = x mod M, s with c_s <= slot < c_s + f_s,
+ * x = f_s (x >> 15) + slot - c_s, and one word x = (x << 16) | w whenever x
+ * falls below 2^15; it must end at x = 2^15.
+ *
+ * Frequencies (fp64, correctly rounded, in the order written here):
+ *   p0 = d_0 / d;  s_0 = p0, s_{k+1} = s_k s_k  (k < 30)
+ *   bit k (k < 30): r = s_k / (1 + s_k), f_1 = (floor(r 2^16) + 1) >> 1
+ *                   clamped to [1, 2^15 - 1], f_0 = 2^15 - f_1
+ *   length l (l <= 30): P(l) = pi_l (1 - s_l), pi_0 = 1, pi_{l+1} = pi_l s_l
+ *   value t (+1, -1, 2): P(t) = d_t / (d - d_0)
+ *   multi-symbol models: f = max(1, floor(P 2^15)) for every symbol that can
+ *   occur (every l; the values with d_t > 0), then the largest f (first on
+ *   ties) absorbs 2^15 - sum f.
+ * ---------------------------------------------------------------------- */
+#define GSO_RANS_SCALE 15
+#define GSO_RANS_M (1u << GSO_RANS_SCALE)
+#define GSO_RANS_L (1u << 15)
+#define GSO_DENSE_LMAX 31   /* bit lengths 0 .. 30 (v = g + 1 < 2^31) */
+#define GSO_DENSE_BITS 30
+
+typedef struct {
+    uint32_t len_f[GSO_DENSE_LMAX], len_c[GSO_DENSE_LMAX + 1];
+    uint32_t bit_f1[GSO_DENSE_BITS];
+    uint32_t val_f[3], val_c[4];
+} gso_dense_model;
+
+static void gso_normalise(const double* P, const int* present, int n, uint32_t* f, uint32_t* c)
+{
+    int64_t sum = 0;
+    int s, best = -1;
+    for (s = 0; s < n; s++) {
+        if (present[s]) {
+            double q = floor(P[s] * (double)GSO_RANS_M);
+            f[s] = q < 1.0 ? 1u : (uint32_t)q;
+        } else {
+            f[s] = 0;
+        }
+        sum += f[s];
+        if (best < 0 || f[s] > f[best]) best = s;
+    }
+    f[best] = (uint32_t)((int64_t)f[best] + (int64_t)GSO_RANS_M - sum);
+    c[0] = 0;
+    for (s = 0; s < n; s++) c[s + 1] = c[s] + f[s];
+}
+
+/* The quantized model of one vector from its symbol counts. */
+GSO_EXPORT int gso_dense_model_build(int64_t d, int64_t n_pos, int64_t n_neg, int64_t n_cap, gso_dense_model* m)
+{
+    double sq[GSO_DENSE_LMAX], P[GSO_DENSE_LMAX], Pv[3], pi, p0;
+    int present[GSO_DENSE_LMAX], pv[3], k, l;
+    const int64_t nz = n_pos + n_neg + n_cap;
+    if (d < 1 || n_pos < 0 || n_neg < 0 || n_cap < 0 || nz > d) return GSO_INVALID;
+    p0 = (double)(d - nz) / (double)d;
+    sq[0] = p0;
+    for (k = 1; k < GSO_DENSE_LMAX; k++) sq[k] = sq[k - 1] * sq[k - 1];
+    for (k = 0; k < GSO_DENSE_BITS; k++) {
+        const double r = sq[k] / (1.0 + sq[k]);
+        uint32_t f1 = ((uint32_t)floor(r * 65536.0) + 1u) >> 1;
+        if (f1 < 1u) f1 = 1u;
+        if (f1 > GSO_RANS_M - 1u) f1 = GSO_RANS_M - 1u;
+        m->bit_f1[k] = f1;
+    }
+    pi = 1.0;
+    for (l = 0; l < GSO_DENSE_LMAX; l++) {
+        P[l] = pi * (1.0 - sq[l]);
+        pi = pi * sq[l];
+        present[l] = 1;
+    }
+    gso_normalise(P, present, GSO_DENSE_LMAX, m->len_f, m->len_c);
+    Pv[0] = nz > 0 ? (double)n_pos / (double)nz : 0.0;
+    Pv[1] = nz > 0 ? (double)n_neg / (double)nz : 0.0;
+    Pv[2] = nz > 0 ? (double)n_cap / (double)nz : 0.0;
+    pv[0] = n_pos > 0;
+    pv[1] = n_neg > 0;
+    pv[2] = n_cap > 0;
+    if (nz == 0) pv[0] = 1;   /* an unused model still sums to M */
+    gso_normalise(Pv, pv, 3, m->val_f, m->val_c);
+    return GSO_OK;
+}
+
+/* One coding step of a chunk: symbol s of a model given as (f, c). */
+typedef struct { uint32_t f, c; } gso_sym;
+
+/* Encoder of one chunk.  Steps are pushed in decode order into `st`, then
+ * coded in reverse; words are written in reverse emission order at out. */
+static int64_t gso_rans_chunk(const gso_sym* st, int64_t n_steps, uint16_t* out, int64_t cap)
+{
+    uint16_t* rev;
+    int64_t n = 0, i;
+    uint32_t x = GSO_RANS_L;
+    rev = (uint16_t*)malloc((size_t)(n_steps + 2) * sizeof(uint16_t));
+    if (!rev) return -1;
+    for (i = n_steps - 1; i >= 0; i--) {
+        const uint32_t f = st[i].f, c = st[i].c;
+        if ((uint64_t)x >= ((uint64_t)f << 16)) {
+            rev[n++] = (uint16_t)(x & 0xFFFFu);
+            x >>= 16;
+        }
+        x = (x / f) * GSO_RANS_M + (x % f) + c;
+    }
+    /* stored: the state's high word, its low word, then the emitted words last-first */
+    if (out && cap >= n + 2) {
+        out[0] = (uint16_t)(x >> 16);
+        out[1] = (uint16_t)(x & 0xFFFFu);
+        for (i = 0; i < n; i++) out[2 + i] = rev[n - 1 - i];
+    }
+    free(rev);
+    return n + 2;
+}
+
+static int gso_val_sym(int8_t q)
+{
+    return q == 1 ? 0 : (q == -1 ? 1 : 2);
+}
+
+static void put32(uint16_t* w, uint32_t v)
+{
+    w[0] = (uint16_t)(v & 0xFFFFu);
+    w[1] = (uint16_t)(v >> 16);
+}
+
+static uint32_t get32(const uint16_t* w)
+{
+    return (uint32_t)w[0] | ((uint32_t)w[1] << 16);
+}
+
+/* Encode the dense vector qt (values 0, +1, -1, 2) with chunks of
+ * K = 2^log2_k non-zero symbols.  Writes *n_words; out (capacity cap words)
+ * is filled only when the code fits. */
+GSO_EXPORT int gso_dense_encode(const int8_t* qt, int64_t d, int log2_k, uint16_t* out, int64_t cap,
+                                int64_t* n_words)
+{
+    int64_t n_pos = 0, n_neg = 0, n_cap = 0, nz, n_chunks, i, j, total, head;
+    int64_t* nzi;
+    gso_dense_model m;
+    gso_sym* st;
+    const int64_t K = (int64_t)1 << log2_k;
+    int rc;
+    if (d < 1 || d >= ((int64_t)1 << 31) || log2_k < 4 || log2_k > 10 || !n_words) return GSO_INVALID;
+    for (i = 0; i < d; i++) {
+        if (qt[i] == 1) n_pos++;
+        else if (qt[i] == -1) n_neg++;
+        else if (qt[i] == 2) n_cap++;
+        else if (qt[i] != 0) return GSO_INVALID;
+    }
+    rc = gso_dense_model_build(d, n_pos, n_neg, n_cap, &m);
+    if (rc != GSO_OK) return rc;
+    nz = n_pos + n_neg + n_cap;
+    n_chunks = (nz + K - 1) / K;
+    nzi = (int64_t*)malloc((size_t)(nz + 1) * sizeof(int64_t));
+    st = (gso_sym*)malloc((size_t)(K * (2 + GSO_DENSE_BITS)) * sizeof(gso_sym));
+    if (!nzi || !st) {
+        free(nzi);
+        free(st);
+        return GSO_INTERNAL;
+    }
+    for (i = 0, j = 0; i < d; i++)
+        if (qt[i] != 0) nzi[j++] = i;
+    head = 9 + 3 * n_chunks;
+    total = head;
+    if (out && cap >= 9) {
+        put32(out, (uint32_t)d);
+        put32(out + 2, (uint32_t)n_pos);
+        put32(out + 4, (uint32_t)n_neg);
+        put32(out + 6, (uint32_t)n_cap);
+        out[8] = (uint16_t)log2_k;
+    }
+    for (i = 0; i < n_chunks; i++) {
+        const int64_t a = i * K, b = (a + K < nz) ? a + K : nz;
+        int64_t n_steps = 0, len;
+        for (j = a; j < b; j++) {
+            if (j > a) {
+                const uint32_t v = (uint32_t)(nzi[j] - nzi[j - 1]);   /* run of zeros + 1 */
+                int l = 0, k;
+                while ((v >> (l + 1)) != 0u) l++;
+                st[n_steps].f = m.len_f[l];
+                st[n_steps].c = m.len_c[l];
+                n_steps++;
+                for (k = l - 1; k >= 0; k--) {
+                    const uint32_t bit = (v >> k) & 1u, f1 = m.bit_f1[k];
+                    st[n_steps].f = bit ? f1 : GSO_RANS_M - f1;
+                    st[n_steps].c = bit ? GSO_RANS_M - f1 : 0u;
+                    n_steps++;
+                }
+            }
+            {
+                const int s = gso_val_sym(qt[nzi[j]]);
+                st[n_steps].f = m.val_f[s];
+                st[n_steps].c = m.val_c[s];
+                n_steps++;
+            }
+        }
+        len = gso_rans_chunk(st, n_steps, (out && cap >= total) ? out + total : NULL,
+                             out ? cap - total : 0);
+        if (len < 0) {
+            free(nzi);
+            free(st);
+            return GSO_INTERNAL;
+        }
+        if (out && cap >= head) {
+            put32(out + 9 + 3 * i, (uint32_t)nzi[a]);
+            out[9 + 3 * i + 2] = (uint16_t)len;
+        }
+        total += len;
+    }
+    *n_words = total;
+    free(nzi);
+    free(st);
+    return GSO_OK;
+}
+
+/* rANS decoder state over one chunk's words. */
+typedef struct {
+    const uint16_t* w;
+    int64_t pos, n;
+    uint32_t x;
+    int bad;
+} gso_rans_dec;
+
+static uint32_t gso_rans_take(gso_rans_dec* r, const uint32_t* f, const uint32_t* c, int n_sym)
+{
+    const uint32_t slot = r->x & (GSO_RANS_M - 1u);
+    int s = 0;
+    while (s < n_sym - 1 && !(slot < c[s + 1])) s++;
+    r->x = f[s] * (r->x >> GSO_RANS_SCALE) + slot - c[s];
+    if (r->x < GSO_RANS_L) {
+        if (r->pos < r->n) r->x = (r->x << 16) | r->w[r->pos++];
+        else r->bad = 1;
+    }
+    return (uint32_t)s;
+}
+
+/* Decode a code written by gso_dense_encode into qt[0..d). */
+GSO_EXPORT int gso_dense_decode(const uint16_t* in, int64_t n_words, int64_t d, int8_t* qt)
+{
+    gso_dense_model m;
+    int64_t n_pos, n_neg, n_cap, nz, K, n_chunks, i, j, off;
+    int rc, log2_k;
+    if (n_words < 9 || d < 1 || (int64_t)get32(in) != d) return GSO_INVALID;
+    n_pos = get32(in + 2);
+    n_neg = get32(in + 4);
+    n_cap = get32(in + 6);
+    log2_k = in[8];
+    if (log2_k < 4 || log2_k > 10) return GSO_INVALID;
+    rc = gso_dense_model_build(d, n_pos, n_neg, n_cap, &m);
+    if (rc != GSO_OK) return rc;
+    nz = n_pos + n_neg + n_cap;
+    K = (int64_t)1 << log2_k;
+    n_chunks = (nz + K - 1) / K;
+    if (n_words < 9 + 3 * n_chunks) return GSO_INVALID;
+    memset(qt, 0, (size_t)d);
+    off = 9 + 3 * n_chunks;
+    for (i = 0; i < n_chunks; i++) {
+        const int64_t cnt = (i + 1) * K <= nz ? K : nz - i * K;
+        const int64_t len = in[9 + 3 * i + 2];
+        int64_t idx = get32(in + 9 + 3 * i);
+        uint32_t bitf[2], bitc[3];
+        gso_rans_dec r;
+        if (len < 2 || off + len > n_words) return GSO_INVALID;
+        r.w = in + off;
+        r.pos = 2;
+        r.n = len;
+        r.x = ((uint32_t)r.w[0] << 16) | r.w[1];
+        r.bad = 0;
+        for (j = 0; j < cnt; j++) {
+            uint32_t s;
+            if (j > 0) {
+                const int l = (int)gso_rans_take(&r, m.len_f, m.len_c, GSO_DENSE_LMAX);
+                uint32_t v = 1;
+                int k;
+                for (k = l - 1; k >= 0; k--) {
+                    bitf[1] = m.bit_f1[k];
+                    bitf[0] = GSO_RANS_M - bitf[1];
+                    bitc[0] = 0;
+                    bitc[1] = bitf[0];
+                    bitc[2] = GSO_RANS_M;
+                    v = 2u * v + gso_rans_take(&r, bitf, bitc, 2);
+                }
+                idx += v;
+            }
+            if (idx < 0 || idx >= d) return GSO_INVALID;
+            s = gso_rans_take(&r, m.val_f, m.val_c, 3);
+            qt[idx] = s == 0 ? 1 : (s == 1 ? -1 : 2);
+        }
+        if (r.bad || r.x != GSO_RANS_L || r.pos != r.n) return GSO_INVALID;
+        off += len;
+    }
+    return off == n_words ? GSO_OK : GSO_INVALID;
+}
