@@ -147,9 +147,9 @@ void carve(Arena& a, Workspace& w, int n_seg, int n_chunks, int64_t n, bool buil
     if (build_p) {
         w.ls.p_ent = a.take<int2>(n);
         w.ls.p_cnt = a.take<int32_t>(n_chunks);
+        w.ls.k_sub = a.take<int32_t>((size_t)n_chunks * kSubStride);
         w.ls.k_off = a.take<int32_t>(n_chunks);
         w.ls.e_bits = a.take<uint32_t>((size_t)n_chunks * (kChunk / 32));
-        w.ls.k_sub = a.take<int32_t>((size_t)n_chunks * kSubStride);
         if (hybrid) {
             w.ls.k_offa = a.take<int32_t>(n_chunks);
             w.nnz = a.take<int32_t>(M);
@@ -310,8 +310,7 @@ constexpr size_t noalloc_bytes(int64_t n) {
     const size_t nc = (size_t)((n + kChunk - 1) / kChunk);
     return up256(sizeof(SegParam)) + up256(sizeof(float) * n) + up256(sizeof(int32_t) * nc) +
            up256(sizeof(double) * nc) + up256(sizeof(int32_t) * (nc + 1)) + up256(sizeof(int2) * n) +
-           up256(sizeof(int32_t) * nc) + up256(sizeof(int32_t) * nc) + up256(sizeof(uint32_t) * nc * (kChunk / 32)) +
-           up256(sizeof(int32_t) * nc * kSubStride);
+           up256(sizeof(int32_t) * nc) + up256(sizeof(int32_t) * nc * kSubStride) + up256(sizeof(int32_t) * nc) + up256(sizeof(uint32_t) * nc * (kChunk / 32));
 }
 
 constexpr size_t kNoAllocBytes = noalloc_bytes(kNoAllocMaxD);

@@ -12,7 +12,11 @@ namespace gs {
 // capacity of each chunk's candidate lists.  A multiple of 4 so that chunk
 // starts inside a worker row keep the 4-coordinate Philox groups aligned.
 constexpr int kChunk = 16384;
-constexpr int kSubStride = 17;   // k_sub entries per chunk (slice starts 0..16)
+// Slices of 1024 coordinates per chunk: the unit of work of the sparse sum.
+constexpr int kSliceLog = 10;
+constexpr int kSlice = 1 << kSliceLog;
+constexpr int kSlices = kChunk / kSlice;
+constexpr int kSubStride = kSlices + 1;   // k_sub entries per chunk (slice starts 0..16)
 // Coordinates per output tile of the sparse sum.
 constexpr int kAggTile = 8192;
 // Threads per CTA of the streaming / solve / decide kernels.
@@ -81,13 +85,13 @@ struct SegParam {
 struct Lists {
     int2* p_ent;        // keep candidates: (worker-local index, bits of g_i)
     int32_t* p_cnt;     // [n_chunks]
+    int32_t* k_sub;     // [n_chunks][kSubStride] kept entries of the chunk before each 1024-coordinate slice
     float* c_val;       // |g| of each capped candidate
     int32_t* c_cnt;     // [n_chunks]
     double* s_low;      // [n_chunks] sum of |g| outside C
     int32_t* k_off;     // [n_chunks] kept count of the chunk, then (after k_scan) the offset
                         // of its first kept entry in its worker's output
     uint32_t* e_bits;   // [n_chunks][kChunk / 32] decision bit of every keep candidate
-    int32_t* k_sub;     // [n_chunks][kSubStride] kept entries of the chunk before each 1024-coordinate slice
     int32_t* k_offa;    // [n_chunks] hybrid code only (else NULL): kept entries with p = 1, then their offsets
     int32_t* c_pre;     // [n_chunks + n_seg] prefix scratch for segments with many chunks
     double* b_low;      // [n_chunks] Algorithm 2 only (else NULL): sum of g^2 outside C
@@ -187,7 +191,11 @@ struct PhiloxStream {
         c3k1 = Lo.step ^ rk1[0];
     }
     __device__ __forceinline__ uint4 words(uint32_t q) const {
-        const uint64_t m0 = (uint64_t)0xD2511F53u * (uint64_t)q;
+        return words_after((uint64_t)0xD2511F53u * (uint64_t)q);
+    }
+    // The same words given round 1's product m0 = 0xD2511F53 * q (which a
+    // caller walking consecutive q can carry forward by adding the constant).
+    __device__ __forceinline__ uint4 words_after(uint64_t m0) const {
         uint32_t c0 = x0, c1 = x1, c2 = (uint32_t)(m0 >> 32) ^ c3k1, c3 = (uint32_t)m0;
 #pragma unroll
         for (int r = 1; r < 10; ++r) {

@@ -16,13 +16,18 @@
 //              is in C, so K_j and the uncapped l1 mass are exact.  If the
 //              final lambda exceeds lam_up the segment falls back to an exact
 //              multi-pass solve over g and rebuilds its P lists.
-//   k_count / k_scan / k_write
-//              the Bernoulli draw Z_i = [u_i < p_i] (section 3) on the P
-//              lists, amplification to g_i / p_i, and compaction into
-//              ascending (idx, val) per worker.
+//   k_decide   per (worker, chunk): the Bernoulli draw Z_i = [u_i < p_i]
+//              (section 3) on the P lists as decision bits and kept counts;
+//              the last warp of each worker scans its counts into offsets.
+//   k_emit     per (worker, chunk): amplification to g_i / p_i and
+//              compaction into ascending (idx, val) (k_emit_hybrid: the
+//              hybrid code of section 3.3 instead);
+//   k_sum      per 1024-coordinate slice, for the fused calls: the
+//              worker-order fp32 sum of Algorithm 1 step 6 over the
+//              compacted rows.
 //   k_bucket / k_tiles
-//              the worker-order fp32 sum of the M sparse vectors (Algorithm 1,
-//              step 6).
+//              the worker-order fp32 sum of M arbitrary sparse vectors
+//              (Algorithm 1, step 6; gs_sparse_aggregate).
 #include <cooperative_groups.h>
 #include <cuda_runtime.h>
 
@@ -30,6 +35,7 @@
 #include <cmath>
 #include <algorithm>
 #include <atomic>
+#include <cstddef>
 #include <cstdint>
 
 #include "gs_device.cuh"
@@ -935,21 +941,17 @@ struct Decider {
 };
 
 // ---------------------------------------------------------------------------
-// Compaction in three steps with no waits between chunks:
-//   k_decide  one warp per chunk: draws each candidate's Philox word again,
-//             records its decision as one bit (a warp ballot per 32
-//             candidates) and the chunk's kept count; the last warp to finish
-//             a worker's chunks turns its counts into output offsets
-//             (exclusive prefix) and writes nnz;
-//   k_emit    one warp per chunk: the kept entries in candidate order, with
-//             value g_i / p_i (consecutive lanes write consecutive slots).
+// The hybrid code's compaction, in two steps with no waits between chunks:
+//   k_decide       one warp per chunk: draws each candidate's Philox word
+//                  again, records its decision as one bit (a warp ballot per
+//                  32 candidates) and the chunk's kept counts (all, and
+//                  those with p = 1); the last warp to finish a worker's
+//                  chunks turns its counts into output offsets;
+//   k_emit_hybrid  one warp per chunk: Q_A and Q_B at their offsets.
 // ---------------------------------------------------------------------------
 constexpr int kEmitWarps = 8;
 constexpr int kEmitBatch = 4;                            // candidate rounds whose loads are in flight together
 constexpr int kBitWords = kChunk / 32;                   // decision words per chunk
-constexpr int kSliceLog = 10;                            // sum slices of 1024 coordinates
-constexpr int kSlice = 1 << kSliceLog;
-constexpr int kSlices = kChunk / kSlice;                 // 16 slices per chunk
 constexpr int kScanPer = 8;                              // chunk counts per lane per step of the worker scan
 
 // One warp turns n counts into their exclusive prefix in place (kScanPer
@@ -1006,10 +1008,12 @@ __global__ void __launch_bounds__(kEmitWarps * 32) k_decide(const __grid_constan
     const int2* ent = Ls.p_ent + (int64_t)ch.m * Lo.d + ch.lo;
     const PhiloxStream ph(Lo, Lo.worker0 + (uint32_t)ch.m);
     uint32_t* wb = Ls.e_bits + (size_t)c * kBitWords;
-    int32_t* ks = Ls.k_sub + (size_t)c * kSubStride;
+    const bool hybrid = Ls.k_offa != nullptr;
+    int32_t* ks = Ls.k_sub ? Ls.k_sub + (size_t)c * kSubStride : nullptr;   // only when a sum follows
     const int lo32 = (int)ch.lo;
-    int cnt = 0, last_sub = 0;   // kept so far; slice of the last candidate seen
-    int cnt_a = 0;               // kept with p = 1 (the hybrid code's Q_A)
+    int cnt = 0;        // kept so far
+    int cnt_a = 0;      // kept with p = 1 (the hybrid code's Q_A)
+    int last_sub = 0;   // slice of the last candidate seen
     for (int base = 0; base < n; base += 32 * kEmitBatch) {
         int2 e[kEmitBatch];
 #pragma unroll
@@ -1017,44 +1021,50 @@ __global__ void __launch_bounds__(kEmitWarps * 32) k_decide(const __grid_constan
             const int i = base + r * 32 + lane;
             e[r] = i < n ? ent[i] : make_int2(0, 0);
         }
+        // The batch's decisions first (independent Philox chains), then its ballots.
+        bool keep[kEmitBatch], capped[kEmitBatch];
 #pragma unroll
         for (int r = 0; r < kEmitBatch; ++r) {
             const int i = base + r * 32 + lane;
-            bool keep = false, capped = false;
-            if (i < n) {
-                const float gv = __int_as_float(e[r].y);
-                if (fabsf(gv) >= dd.a_cap) {
-                    keep = true;   // capped: p = 1, kept whatever the draw
-                    capped = true;
-                } else {
-                    const uint32_t x = word_of(ph.words((uint32_t)e[r].x >> 2), e[r].x & 3);
-                    float v;
-                    keep = dd(gv, x, v);
-                }
+            const float gv = __int_as_float(e[r].y);
+            capped[r] = i < n && fabsf(gv) >= dd.a_cap;   // p = 1: kept whatever the draw
+            keep[r] = capped[r];
+            if (i < n && !capped[r]) {
+                const uint32_t x = word_of(ph.words((uint32_t)e[r].x >> 2), e[r].x & 3);
+                float v;
+                keep[r] = dd(gv, x, v);
             }
-            const uint32_t bal = __ballot_sync(0xFFFFFFFFu, keep);
+        }
+#pragma unroll
+        for (int r = 0; r < kEmitBatch; ++r) {
+            const uint32_t bal = __ballot_sync(0xFFFFFFFFu, keep[r]);
             if (base + r * 32 < n) {
                 if (lane == 0) wb[(base >> 5) + r] = bal;
-                // Candidates are in ascending order: a candidate that opens slices
-                // (prev, sub] records the kept count before it for each of them.
-                const int sub = i < n ? (e[r].x - lo32) >> kSliceLog : kSlices;
-                int prev = __shfl_up_sync(0xFFFFFFFFu, sub, 1);
-                if (lane == 0) prev = last_sub;
-                const int before = cnt + __popc(bal & ((1u << lane) - 1u));
-                for (int t = prev + 1; t <= sub && t <= kSlices; ++t) ks[t] = before;
-                last_sub = __shfl_sync(0xFFFFFFFFu, sub, 31);
+                if (ks) {
+                    // Candidates are in ascending order: a candidate that opens slices
+                    // (prev, sub] records the kept count before it for each of them.
+                    const int i = base + r * 32 + lane;
+                    const int sub = i < n ? (e[r].x - lo32) >> kSliceLog : kSlices;
+                    int prev = __shfl_up_sync(0xFFFFFFFFu, sub, 1);
+                    if (lane == 0) prev = last_sub;
+                    const int before = cnt + __popc(bal & ((1u << lane) - 1u));
+                    for (int t = prev + 1; t <= sub && t <= kSlices; ++t) ks[t] = before;
+                    last_sub = __shfl_sync(0xFFFFFFFFu, sub, 31);
+                }
             }
             cnt += __popc(bal);
-            cnt_a += __popc(__ballot_sync(0xFFFFFFFFu, capped));
+            if (hybrid) cnt_a += __popc(__ballot_sync(0xFFFFFFFFu, capped[r]));
         }
     }
-    // Slices after the last candidate (all of them if there is none).
-    if (n == 0) last_sub = 0;
-    if (lane <= kSlices && lane > last_sub) ks[lane] = cnt;
+    if (ks) {
+        // Slices after the last candidate (all of them if there is none).
+        if (n == 0) last_sub = 0;
+        if (lane <= kSlices && lane > last_sub) ks[lane] = cnt;
+        if (lane == 0) ks[0] = 0;
+    }
     if (lane == 0) {
-        ks[0] = 0;
         Ls.k_off[c] = cnt;
-        if (Ls.k_offa) Ls.k_offa[c] = cnt_a;
+        if (hybrid) Ls.k_offa[c] = cnt_a;
     }
 
     // The last warp to finish one of the worker's chunks turns the worker's
@@ -1080,14 +1090,11 @@ __global__ void __launch_bounds__(kEmitWarps * 32) k_decide(const __grid_constan
     }
 }
 
-__global__ void __launch_bounds__(kEmitWarps * 32) k_emit(const __grid_constant__ Layout Lo,
-                                                          const SegParam* __restrict__ sp,
-                                                          const __grid_constant__ Lists Ls, int n_chunks,
-                                                          int32_t* idx, float* val, int64_t cap) {
-    grid_dep_wait();
+// The kept candidates of chunk c at their output positions, value g_i / p_i
+// (one warp; consecutive lanes write consecutive slots).
+__device__ __forceinline__ void emit_chunk(const Layout& Lo, const SegParam* __restrict__ sp, const Lists& Ls, int c,
+                                           int32_t* idx, float* val, int64_t cap) {
     const int lane = threadIdx.x & 31;
-    const int c = blockIdx.x * kEmitWarps + (threadIdx.x >> 5);
-    if (c >= n_chunks) return;
     const Chunk ch = decode_chunk(Lo, c);
     const SegParam& P = sp[ch.seg];
     const float a_cap = P.a_cap, inv_lam32 = P.inv_lam32;
@@ -1120,6 +1127,15 @@ __global__ void __launch_bounds__(kEmitWarps * 32) k_emit(const __grid_constant_
             pos0 += __popc(wd[r]);
         }
     }
+}
+
+__global__ void __launch_bounds__(kEmitWarps * 32) k_emit(const __grid_constant__ Layout Lo,
+                                                          const SegParam* __restrict__ sp,
+                                                          const __grid_constant__ Lists Ls, int n_chunks,
+                                                          int32_t* idx, float* val, int64_t cap) {
+    grid_dep_wait();
+    const int c = blockIdx.x * kEmitWarps + (threadIdx.x >> 5);
+    if (c < n_chunks) emit_chunk(Lo, sp, Ls, c, idx, val, cap);
 }
 
 // The hybrid code of section 3.3 (eqs. 9-10) straight from the decisions: a
@@ -1525,7 +1541,9 @@ cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls
     {
         set_launch_error_site("k_decide launch");
         TraceScope ts(kKDecide, st);
-        e = launch_dep(k_decide, dim3(blocks), dim3(kEmitWarps * 32), 0, st, Lo, const_cast<SegParam*>(sp), Ls,
+        Lists Ld = Ls;
+        if (!sum_out || hybrid) Ld.k_sub = nullptr;   // the slice table serves the sum only
+        e = launch_dep(k_decide, dim3(blocks), dim3(kEmitWarps * 32), 0, st, Lo, const_cast<SegParam*>(sp), Ld,
                        n_chunks, nnz, hybrid ? hybrid->n_a : nullptr, hybrid ? hybrid->n_b : nullptr, cap, status);
     }
     if (e != cudaSuccess) return e;

@@ -40,11 +40,44 @@
 namespace gs {
 namespace {
 
+// Occupancy and ring depth.  The kernel is bound by instruction latency (its
+// integer work per coordinate is mostly Philox), so resident warps matter
+// more than deep rings: GS_TMA_CTAS CTAs of kCW warps per SM, each CTA's
+// rings in GS_TMA_RING_KIB KiB of shared memory.
+#ifndef GS_TMA_CTAS
+#define GS_TMA_CTAS 2
+#endif
+#ifndef GS_TMA_RING_KIB
+#define GS_TMA_RING_KIB 96
+#endif
+// Form of the keep-candidate test (all three compute the same sign bit):
+// 0: shift, three-input add and funnel shift on the integer ALU; 1: the
+// constant minus the float bits by an integer multiply-add first; 2: the
+// shift folded into a multiply-high.
+#ifndef GS_TMA_CAND
+#define GS_TMA_CAND 0
+#endif
+// 1: the Algorithm 3 instantiation also takes two groups (two independent
+// Philox chains) per step, as the sum-of-squares one always does.
+#ifndef GS_TMA_PAIR
+#define GS_TMA_PAIR 0
+#endif
+// 1: round 1's product 0xD2511F53 * q of consecutive groups carried forward
+// by a 64-bit add (integer ALU) instead of a wide multiply each.
+#ifndef GS_TMA_SR
+#define GS_TMA_SR 1
+#endif
+// 1: lam_up |g| formed as |lam_up * g| (a multiply and an add that takes the
+// absolute value of its operand) instead of a fused multiply-add on |g|.
+#ifndef GS_TMA_ABS
+#define GS_TMA_ABS 0
+#endif
 constexpr int kCW = 8;                         // warps per CTA
 constexpr int kTmaThreads = 32 * kCW;
+constexpr int kTmaCtas = GS_TMA_CTAS;
 constexpr int kLaneCoords = 32;                // coordinates per lane per buffer
 constexpr int kBufCoords = 32 * kLaneCoords;   // 1024 coordinates per buffer
-constexpr int kRingBudget = 96 * 1024;         // shared memory for the rings of one CTA (2 CTAs per SM)
+constexpr int kRingBudget = GS_TMA_RING_KIB * 1024;   // shared memory for the rings of one CTA
 constexpr int kRowBytes = 128;
 constexpr long long kWaitLimit = 1ll << 22;    // try_wait polls before giving up
 constexpr int kQueue = 8;                      // per-warp queue of taken chunks (> kRing + 1)
@@ -137,8 +170,23 @@ __device__ __forceinline__ uint32_t shl_in(uint32_t m, float r) {
 // right-hand side is below its 2^-20 slack, so every coordinate kept under a
 // lambda <= lam_up passes (NaN and Inf |g| pass too).
 __device__ __forceinline__ float cand_sign(uint32_t x, float lam_up, float a, float pbias) {
-    const uint32_t pf = __float_as_uint(fmaf(lam_up, a, pbias));
+#if GS_TMA_ABS
+    const uint32_t pf = __float_as_uint(__fadd_rn(fabsf(__fmul_rn(lam_up, a)), pbias));
+#else
+    const uint32_t pf = __float_as_uint(fmaf(lam_up, fabsf(a), pbias));
+#endif
+#if GS_TMA_CAND == 0
     return __uint_as_float((x >> 9) + 0x3F800000u - pf);
+#else
+    uint32_t c, r;
+    asm("mad.lo.u32 %0, %1, 4294967295, 1065353216;" : "=r"(c) : "r"(pf));   // 0x3F800000 - pf
+#if GS_TMA_CAND == 1
+    r = (x >> 9) + c;
+#else
+    asm("mad.hi.u32 %0, %1, 8388608, %2;" : "=r"(r) : "r"(x), "r"(c));      // (x >> 9) + c
+#endif
+    return __uint_as_float(r);
+#endif
 }
 
 // Coordinate k (0..31) of a lane's 32, read back from its row of the buffer
@@ -155,17 +203,24 @@ __device__ __forceinline__ float stage_value(const unsigned char* rp, int first_
     }
 }
 
-// Group j (0..7, four coordinates) of a lane's 32 as |g| values.
+// Group j (0..7, four coordinates) of a lane's 32 as g values (signed; the
+// callers take |g| where they use it, which folds into their float operands).
 template <int kDtype>
 __device__ __forceinline__ float4 stage_group(const unsigned char* rp, int first_chunk, int sw, int j) {
     if (kDtype == 0) {
-        const float4 t = *reinterpret_cast<const float4*>(rp + (((first_chunk + j) ^ sw) << 4));
-        return make_float4(fabsf(t.x), fabsf(t.y), fabsf(t.z), fabsf(t.w));
+        return *reinterpret_cast<const float4*>(rp + (((first_chunk + j) ^ sw) << 4));
     } else {
         const uint2 t = *reinterpret_cast<const uint2*>(rp + (((first_chunk + (j >> 1)) ^ sw) << 4) + ((j & 1) << 3));
-        return make_float4(fabsf(__uint_as_float(t.x << 16)), fabsf(__uint_as_float(t.x & 0xFFFF0000u)),
-                           fabsf(__uint_as_float(t.y << 16)), fabsf(__uint_as_float(t.y & 0xFFFF0000u)));
+        return make_float4(__uint_as_float(t.x << 16), __uint_as_float(t.x & 0xFFFF0000u),
+                           __uint_as_float(t.y << 16), __uint_as_float(t.y & 0xFFFF0000u));
     }
+}
+
+__device__ __forceinline__ float abs_sum4(const float4& a) {
+    return (fabsf(a.x) + fabsf(a.y)) + (fabsf(a.z) + fabsf(a.w));
+}
+__device__ __forceinline__ float abs_sq4(const float4& a) {
+    return (a.x * a.x + a.y * a.y) + (a.z * a.z + a.w * a.w);
 }
 
 // A chunk index with its worker and its chunk within the worker.
@@ -209,7 +264,7 @@ struct ChunkWalk {
 // kDtype 0: fp32 rows of 32; 1: bf16 rows of 64.  kSq: also the sum of g^2
 // outside C (Algorithm 2's solve), the same way as s_low.
 template <int kDtype, bool kSq>
-__global__ void __launch_bounds__(kTmaThreads, 2)
+__global__ void __launch_bounds__(kTmaThreads, kTmaCtas)
     k_stream_tma(const __grid_constant__ CUtensorMap map, const __grid_constant__ StreamArgs A) {
     grid_dep_wait();
     constexpr int kInner = kDtype == 0 ? 32 : 64;          // elements per 128-byte row
@@ -240,20 +295,26 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
     const int first = blockIdx.x * kCW + warp;
 
     // Prefetch cursor: the next buffer's row and its chunk's end row.
+    // (Rows of 128 bytes number fewer than 2^31: the launcher checks.)
     ChunkWalk pc(Lo, first);
-    int64_t prow = 0, prow_end = 0;
-    if (pc.c < A.n_chunks) {
-        int64_t fl, lo, hi;
-        int seg;
-        pc.rows(Lo, kInner, fl, prow, prow_end, seg, lo, hi);
-    }
+    int prow = 0, prow_end = 0;
+    auto cursor = [&]() {
+        if (pc.c < A.n_chunks) {
+            int64_t fl, lo, hi, r0, r1;
+            int seg;
+            pc.rows(Lo, kInner, fl, r0, r1, seg, lo, hi);
+            prow = (int)r0;
+            prow_end = (int)r1;
+        }
+    };
+    cursor();
     int issued = 0;
     auto prefetch = [&]() {
         if (pc.c >= A.n_chunks) return;
         const int b = issued % kRing;
         if (lane == 0) {
             mbar_arrive_tx(&my_full[b], kBufBytes);
-            tma_load_rows(my_buf + b * kBufBytes, &map, (int)prow, &my_full[b]);
+            tma_load_rows(my_buf + b * kBufBytes, &map, prow, &my_full[b]);
         }
         ++issued;
         prow += kBufRows;
@@ -266,11 +327,7 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
             nc = __shfl_sync(0xFFFFFFFFu, nc, 0);
             ++qt;
             pc.jump(Lo, nc);
-            if (pc.c < A.n_chunks) {
-                int64_t fl, lo, hi;
-                int seg;
-                pc.rows(Lo, kInner, fl, prow, prow_end, seg, lo, hi);
-            }
+            cursor();
         }
     };
 #pragma unroll 1
@@ -335,18 +392,23 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
             if (live && rel < len && rel + kLaneCoords > 0) {
                 const uint32_t q0 = (uint32_t)((lo + rel) >> 2);   // worker-local group of coordinate 0
                 if (rel >= 0 && rel + kLaneCoords <= len) {
-                    // All 32 coordinates belong to the chunk: groups of 4 in order.
-                    // Two groups per step (independent Philox chains) pays only in the
-                    // kSq instantiation (303 vs 320 us on 16 x 2^24); the plain one takes
-                    // one group per step (277 vs 287 us).
-                    float s4[8], q4[8];
-                    if constexpr (!kSq) {
+                    // All 32 coordinates belong to the chunk: groups of 4 in order,
+                    // the l1 (and square) sums accumulated group by group.
+                    if constexpr (!kSq && !GS_TMA_PAIR) {
+#if GS_TMA_SR
+                        uint64_t m0 = (uint64_t)0xD2511F53u * (uint64_t)q0;   // round 1's product, carried
+#endif
 #pragma unroll
                         for (int j = 0; j < 8; ++j) {
                             const float4 a = stage_group<kDtype>(rp, first_chunk, sw, j);
-                            s4[j] = (a.x + a.y) + (a.z + a.w);
+                            s32 += abs_sum4(a);
                             if (build_p) {
+#if GS_TMA_SR
+                                const uint4 w = ph.words_after(m0);
+                                m0 += 0xD2511F53u;
+#else
                                 const uint4 w = ph.words(q0 + j);
+#endif
                                 pm = shl_in(pm, cand_sign(w.x, lup, a.x, pbias));
                                 pm = shl_in(pm, cand_sign(w.y, lup, a.y, pbias));
                                 pm = shl_in(pm, cand_sign(w.z, lup, a.z, pbias));
@@ -354,36 +416,34 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
                             }
                         }
                     } else {
+                        // Two groups per step (independent Philox chains) pays in the
+                        // instantiation that also sums squares.
 #pragma unroll
-                    for (int j = 0; j < 8; j += 2) {
-                        const float4 a = stage_group<kDtype>(rp, first_chunk, sw, j);
-                        const float4 b = stage_group<kDtype>(rp, first_chunk, sw, j + 1);
-                        s4[j] = (a.x + a.y) + (a.z + a.w);
-                        s4[j + 1] = (b.x + b.y) + (b.z + b.w);
-                        if (kSq) {
-                            q4[j] = (a.x * a.x + a.y * a.y) + (a.z * a.z + a.w * a.w);
-                            q4[j + 1] = (b.x * b.x + b.y * b.y) + (b.z * b.z + b.w * b.w);
+                        for (int j = 0; j < 8; j += 2) {
+                            const float4 a = stage_group<kDtype>(rp, first_chunk, sw, j);
+                            const float4 b = stage_group<kDtype>(rp, first_chunk, sw, j + 1);
+                            s32 += abs_sum4(a) + abs_sum4(b);
+                            if (kSq) q32 += abs_sq4(a) + abs_sq4(b);
+                            if (build_p) {
+                                const uint4 w = ph.words(q0 + j);
+                                const uint4 v = ph.words(q0 + j + 1);
+                                pm = shl_in(pm, cand_sign(w.x, lup, a.x, pbias));
+                                pm = shl_in(pm, cand_sign(w.y, lup, a.y, pbias));
+                                pm = shl_in(pm, cand_sign(w.z, lup, a.z, pbias));
+                                pm = shl_in(pm, cand_sign(w.w, lup, a.w, pbias));
+                                pm = shl_in(pm, cand_sign(v.x, lup, b.x, pbias));
+                                pm = shl_in(pm, cand_sign(v.y, lup, b.y, pbias));
+                                pm = shl_in(pm, cand_sign(v.z, lup, b.z, pbias));
+                                pm = shl_in(pm, cand_sign(v.w, lup, b.w, pbias));
+                            }
                         }
-                        if (build_p) {
-                            const uint4 w = ph.words(q0 + j);
-                            const uint4 v = ph.words(q0 + j + 1);
-                            pm = shl_in(pm, cand_sign(w.x, lup, a.x, pbias));
-                            pm = shl_in(pm, cand_sign(w.y, lup, a.y, pbias));
-                            pm = shl_in(pm, cand_sign(w.z, lup, a.z, pbias));
-                            pm = shl_in(pm, cand_sign(w.w, lup, a.w, pbias));
-                            pm = shl_in(pm, cand_sign(v.x, lup, b.x, pbias));
-                            pm = shl_in(pm, cand_sign(v.y, lup, b.y, pbias));
-                            pm = shl_in(pm, cand_sign(v.z, lup, b.z, pbias));
-                            pm = shl_in(pm, cand_sign(v.w, lup, b.w, pbias));
-                        }
-                    }
                     }
                     pm = __brev(pm);   // coordinate k at bit k
-                    s32 = ((s4[0] + s4[1]) + (s4[2] + s4[3])) + ((s4[4] + s4[5]) + (s4[6] + s4[7]));
-                    if constexpr (kSq)
-                        q32 = ((q4[0] + q4[1]) + (q4[2] + q4[3])) + ((q4[4] + q4[5]) + (q4[6] + q4[7]));
                     if (!(s32 < t_c)) {
                         // Some |g| may reach t_c (or be non-finite): split exactly.
+                        // (A sum of non-negative floats is at least its largest term.)
+                        s32 = 0.0f;
+                        q32 = 0.0f;
 #pragma unroll
                         for (int j = 0; j < 8; ++j) {
                             float m4[4];
@@ -394,12 +454,9 @@ __global__ void __launch_bounds__(kTmaThreads, 2)
                                 cm |= in_c ? (1u << (4 * j + k)) : 0u;
                                 m4[k] = in_c ? 0.0f : a;
                             }
-                            s4[j] = (m4[0] + m4[1]) + (m4[2] + m4[3]);
-                            if (kSq) q4[j] = (m4[0] * m4[0] + m4[1] * m4[1]) + (m4[2] * m4[2] + m4[3] * m4[3]);
+                            s32 += (m4[0] + m4[1]) + (m4[2] + m4[3]);
+                            if (kSq) q32 += (m4[0] * m4[0] + m4[1] * m4[1]) + (m4[2] * m4[2] + m4[3] * m4[3]);
                         }
-                        s32 = ((s4[0] + s4[1]) + (s4[2] + s4[3])) + ((s4[4] + s4[5]) + (s4[6] + s4[7]));
-                        if (kSq)
-                            q32 = ((q4[0] + q4[1]) + (q4[2] + q4[3])) + ((q4[4] + q4[5]) + (q4[6] + q4[7]));
                     }
                 } else {
                     // The lane straddles an edge of the chunk: test each coordinate.
@@ -589,8 +646,8 @@ cudaError_t launch_stream_tma(const Layout& Lo, const SegParam* sp, const Lists&
     // that wrote the bounds, which this launch waits for).
     A.next_chunk = reinterpret_cast<int*>(reinterpret_cast<char*>(const_cast<SegParam*>(sp)) +
                                           offsetof(SegParam, next_chunk));
-    // One chunk per warp at a time; two CTAs per SM at most.
-    const int grid = std::min((n_chunks + kCW - 1) / kCW, 2 * sm_count_tma());
+    // One chunk per warp at a time; kTmaCtas CTAs per SM at most.
+    const int grid = std::min((n_chunks + kCW - 1) / kCW, kTmaCtas * sm_count_tma());
     cudaError_t e;
     TraceScope ts(kKStreamTma, st);
     void (*kern)(const CUtensorMap, const StreamArgs);
