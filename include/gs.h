@@ -172,6 +172,49 @@ gs_status gs_batched_sparsify_hybrid(const void* g, int dtype, int M, int64_t d,
                                      gs_info* info, void* stream);
 
 /*
+ * The dense code of section 3.3 (last paragraph): per worker, the vector
+ * q~ in {0, +1, -1, 2}^d -- 0 where a coordinate is dropped, sign(g_i) where
+ * it is kept with p_i < 1, 2 where p_i = 1 -- entropy coded under the static
+ * model P(s) = d_s / d (d_s coordinates hold symbol s), whose ideal length
+ * sum_s d_s log2(d / d_s) is at most 2d bits.  Together with Q_A's values
+ * and 1 / lambda it carries Q(g) exactly.  Each non-zero symbol is coded as
+ * the run of zeros before it (geometric in p0 = d_0 / d: its bit length, then
+ * its bits below the leading one) and its value (P(t) = d_t / (d - d_0)),
+ * which costs exactly what the model charges the symbols; the coder is rANS
+ * with 15-bit frequencies and 16-bit words, in independent chunks of
+ * K = 2^log2_k non-zero symbols so that both directions run in parallel.
+ * A worker's code, in 16-bit words (two-word integers low word first):
+ *   header     d, d_{+1}, d_{-1}, d_2 (two words each), log2_k (one word)
+ *   directory  per chunk: index of its first non-zero (two words), stream
+ *              length in words (one word)
+ *   streams    per chunk: the rANS final state (high word first), then the
+ *              renormalisation words in the order the decoder reads them.
+ * Overhead over the model's length: 144 bits per worker, 96 bits at most per
+ * chunk (directory and final state; the run of each chunk's first non-zero
+ * and the zeros after the last are not coded), plus the rounding of the
+ * frequencies.
+ *
+ * gs_dense_encode
+ *   qa_idx, qb_code, n_a, n_b  the hybrid lists of gs_batched_sparsify_hybrid
+ *              (device; rows of `cap` entries; lengths n_a, n_b <= cap)
+ *   log2_k     4 .. 10
+ *   words      device, M x word_cap uint16: row m receives worker m's code
+ *   n_words    device, M int64: each code's length in words.  A code longer
+ *              than word_cap is not written past its header; its length is
+ *              still reported and GS_ERR_CAPACITY recorded.
+ * gs_dense_decode
+ *   words, n_words, word_cap   codes as gs_dense_encode writes them
+ *   qt         device, M x d int8: q~ of each worker (written)
+ *   A malformed code (header, directory, or a stream that does not end in the
+ *   encoder's initial state) records GS_ERR_INVALID_ARG.
+ */
+gs_status gs_dense_encode(const int32_t* qa_idx, const uint32_t* qb_code, const int32_t* n_a, const int32_t* n_b,
+                          int M, int64_t d, int64_t cap, int log2_k, uint16_t* words, int64_t word_cap,
+                          int64_t* n_words, void* stream);
+gs_status gs_dense_decode(const uint16_t* words, const int64_t* n_words, int M, int64_t d, int64_t word_cap,
+                          int8_t* qt, void* stream);
+
+/*
  * Algorithm 2 (section 3.2): the closed-form solution of problem (4) for a
  * variance budget eps >= 0 instead of a density budget.  lambda is the one
  * for which sum_i g_i^2 / p_i = (1 + eps) sum_i g_i^2 with

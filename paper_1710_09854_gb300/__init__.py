@@ -26,7 +26,7 @@ GS_OPT_FORCE_EXACT_SOLVE, GS_OPT_SAMPLE_SIZE, GS_OPT_KERNEL_TIMING, GS_OPT_STREA
 EXPORTS = ("gs_status_string", "gs_last_error", "gs_version", "gs_sync_status", "gs_probabilities", "gs_probabilities_ex",
            "gs_sparsify", "gs_batched_sparsify", "gs_batched_sparsify_hybrid", "gs_probabilities_eps", "gs_batched_sparsify_eps", "gs_segmented_sparsify", "gs_segmented_sparsify_aggregate", "gs_sparse_aggregate",
            "gs_sparsify_aggregate", "gs_sparsify_average_sparsify", "gs_sparsify_noalloc", "gs_pipeline_host", "gs_logreg_grad", "gs_logreg_margins", "gs_row_sq_norms", "gs_sum_rows", "gs_sgd_step",
-           "gs_random_words", "gs_selftest_timeout", "gs_set_option", "gs_kernel_count", "gs_kernel_name",
+           "gs_dense_encode", "gs_dense_decode", "gs_random_words", "gs_selftest_timeout", "gs_set_option", "gs_kernel_count", "gs_kernel_name",
            "gs_kernel_times")
 
 
@@ -64,6 +64,8 @@ def lib():
             "gs_probabilities_ex": ([vp, i64, dbl, i32, vp, vp, vp], i32),
             "gs_sparsify": ([vp, i64, dbl, i32, u64, u32, u32, vp, vp, vp, vp], i32),
             "gs_batched_sparsify": ([vp, i32, i32, i64, dbl, i32, u64, u32, u32, vp, vp, vp, i64, vp, vp], i32),
+            "gs_dense_encode": ([vp, vp, vp, vp, i32, i64, i64, i32, vp, i64, vp, vp], i32),
+            "gs_dense_decode": ([vp, vp, i32, i64, i64, vp, vp], i32),
             "gs_batched_sparsify_hybrid": ([vp, i32, i32, i64, dbl, i32, u64, u32, u32, vp, vp, vp, vp, vp, vp, i64,
                                             vp, vp], i32),
             "gs_probabilities_eps": ([vp, i64, dbl, vp, vp, vp], i32),
@@ -324,6 +326,33 @@ def gs_batched_sparsify_hybrid(g, kappa, iters, seed, step, worker0, qa_idx, qa_
                                             _ptr(n_a, "n_a", (torch.int32,)), _ptr(n_b, "n_b", (torch.int32,)),
                                             _ptr(inv_lam, "inv_lam", (torch.float32,)), cap, _ptr(info, "info"),
                                             _stream(stream)), "gs_batched_sparsify_hybrid")
+
+
+def gs_dense_encode(qa_idx, qb_code, n_a, n_b, d, log2_k, words, n_words, stream=None):
+    """The dense code of section 3.3 from the hybrid lists (M, cap) of
+    gs_batched_sparsify_hybrid: words (M, word_cap) int16 (16-bit words) and
+    n_words (M,) int64 receive each worker's code and its length."""
+    import torch
+    M, cap = qa_idx.shape
+    if tuple(qb_code.shape) != (M, cap) or n_a.numel() != M or n_b.numel() != M or words.shape[0] != M:
+        raise ValueError("qa_idx, qb_code (M, cap); n_a, n_b (M,); words (M, word_cap)")
+    codes = (torch.int32, torch.uint32) if hasattr(torch, "uint32") else (torch.int32,)
+    w16 = (torch.int16, torch.uint16) if hasattr(torch, "uint16") else (torch.int16,)
+    _check(lib().gs_dense_encode(_ptr(qa_idx, "qa_idx", (torch.int32,)), _ptr(qb_code, "qb_code", codes),
+                                 _ptr(n_a, "n_a", (torch.int32,)), _ptr(n_b, "n_b", (torch.int32,)), M, int(d), cap,
+                                 int(log2_k), _ptr(words, "words", w16), words.shape[1],
+                                 _ptr(n_words, "n_words", (torch.int64,)), _stream(stream)), "gs_dense_encode")
+
+
+def gs_dense_decode(words, n_words, d, qt, stream=None):
+    """Decode codes written by gs_dense_encode into qt (M, d) int8 (q~ rows)."""
+    import torch
+    M, word_cap = words.shape
+    if n_words.numel() != M or tuple(qt.shape) != (M, int(d)):
+        raise ValueError("words (M, word_cap), n_words (M,), qt (M, d)")
+    w16 = (torch.int16, torch.uint16) if hasattr(torch, "uint16") else (torch.int16,)
+    _check(lib().gs_dense_decode(_ptr(words, "words", w16), _ptr(n_words, "n_words", (torch.int64,)), M, int(d),
+                                 word_cap, _ptr(qt, "qt", (torch.int8,)), _stream(stream)), "gs_dense_decode")
 
 
 def gs_probabilities_eps(g, eps, p, info=None, stream=None):

@@ -585,6 +585,49 @@ gs_status gs_sparsify_noalloc(const float* g, int64_t d, double kappa, int iters
                        static_cast<cudaStream_t>(stream));
 }
 
+gs_status gs_dense_encode(const int32_t* qa_idx, const uint32_t* qb_code, const int32_t* n_a, const int32_t* n_b,
+                          int M, int64_t d, int64_t cap, int log2_k, uint16_t* words, int64_t word_cap,
+                          int64_t* n_words, void* stream) {
+    if (!qa_idx || !qb_code || !n_a || !n_b || !words || !n_words || M < 1 || d < 1 || d >= kMaxD || cap < 1 ||
+        log2_k < 4 || log2_k > 10 || word_cap < 1)
+        return GS_ERR_INVALID_ARG;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    DevState* s = nullptr;
+    gs_status rc = device_state(&s);
+    if (rc != GS_OK) return rc;
+    // Chunks: at most ceil(min(d, 2 cap) / K) per worker (the lists hold at most 2 cap entries).
+    const int64_t per = (std::min<int64_t>(d, 2 * cap) + (1 << log2_k) - 1) >> log2_k;
+    const int64_t max_chunks = (int64_t)M * per;
+    void* mem = nullptr;
+    GS_TRY(cudaMallocFromPoolAsync(&mem, dense_workspace_bytes(M, max_chunks, true), s->pool, st));
+    const cudaError_t e = launch_dense_encode(qa_idx, qb_code, n_a, n_b, M, d, cap, log2_k, words, word_cap, n_words,
+                                              mem, max_chunks, s->status, st);
+    const cudaError_t ef = cudaFreeAsync(mem, st);
+    if (e != cudaSuccess) return cuda_fail(launch_error_site(), e);
+    if (ef != cudaSuccess) return cuda_fail("cudaFreeAsync", ef);
+    return GS_OK;
+}
+
+gs_status gs_dense_decode(const uint16_t* words, const int64_t* n_words, int M, int64_t d, int64_t word_cap,
+                          int8_t* qt, void* stream) {
+    if (!words || !n_words || !qt || M < 1 || d < 1 || d >= kMaxD || word_cap < 9) return GS_ERR_INVALID_ARG;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    DevState* s = nullptr;
+    gs_status rc = device_state(&s);
+    if (rc != GS_OK) return rc;
+    // Chunks: at most (word_cap - 9) / 3 directory entries per worker, and at
+    // most ceil(d / 16) (K >= 16, one non-zero symbol per coordinate at most).
+    const int64_t per = std::min<int64_t>((d + 15) / 16, (word_cap - 9) / 3);
+    const int64_t max_chunks = std::max<int64_t>(1, (int64_t)M * per);
+    void* mem = nullptr;
+    GS_TRY(cudaMallocFromPoolAsync(&mem, dense_workspace_bytes(M, max_chunks, false), s->pool, st));
+    const cudaError_t e = launch_dense_decode(words, n_words, M, d, word_cap, qt, mem, max_chunks, s->status, st);
+    const cudaError_t ef = cudaFreeAsync(mem, st);
+    if (e != cudaSuccess) return cuda_fail(launch_error_site(), e);
+    if (ef != cudaSuccess) return cuda_fail("cudaFreeAsync", ef);
+    return GS_OK;
+}
+
 gs_status gs_logreg_grad(const float* X, const float* y, int N, int d, const float* w, const int32_t* batch, int M,
                          int B, float lam2, float* G, float* gsq, void* stream) {
     if (!X || !y || !w || !batch || !G || !gsq || N < 1 || d < 1 || M < 1 || B < 1 || B > kMaxLrBatch)

@@ -1,0 +1,665 @@
+// gs_dense.cu -- the dense code of Q(g) (section 3.3, last paragraph): the
+// vector q~ in {0, +1, -1, 2}^d (0: dropped; sign(g_i): kept with p_i < 1;
+// 2: kept with p_i = 1) entropy coded under the static model the paper
+// prices it with, P(s) = d_s / d, whose ideal length is
+// sum_s d_s log2(d / d_s) <= 2d bits.
+//
+// The model is coded one non-zero symbol at a time: the run g of zeros
+// before it under the model's geometric law P(g) = (1 - p0) p0^g
+// (p0 = d_0 / d), then its value t under P(t) = d_t / (d - d_0).  The run is
+// sent as v = g + 1: its bit length l = floor(log2 v) with
+// P(l) = p0^(2^l - 1) (1 - p0^(2^l)), then its l bits below the leading one
+// (most significant first), bit k being 1 with probability
+// p0^(2^k) / (1 + p0^(2^k)); given l these bits are independent and their
+// probabilities multiply back to P(g), so the events cost exactly what the
+// symbols would one by one.
+//
+// Format of one vector (16-bit words; two-word integers low word first):
+//   header     d, d_{+1}, d_{-1}, d_2 (two words each), log2 K (one word)
+//   directory  per chunk of K consecutive non-zero symbols: the index of its
+//              first non-zero (two words) and its stream length (one word)
+//   streams    one rANS stream per chunk, in chunk order; the chunk's first
+//              non-zero is placed by the directory (its run is not coded).
+// rANS: integer frequencies over 2^15 (model below), state x in
+// [2^15, 2^31), 16-bit renormalisation words.  A chunk's coding steps, in
+// decode order, are (run bit length, run bits) for every non-zero but the
+// first, then the value; the encoder visits them last to first starting from
+// x = 2^15, emitting x's low word (x >>= 16) while x >= f 2^16 and setting
+// x = floor(x / f) 2^15 + (x mod f) + c; the stream is the final state (high
+// word first) followed by the emitted words last to first.
+//
+// Frequencies from the counts, in exactly rounded fp64 in this order:
+// p0 = d_0 / d; s_0 = p0, s_{k+1} = s_k s_k; bit k: r = s_k / (1 + s_k),
+// f_1 = (floor(r 2^16) + 1) >> 1 clamped to [1, 2^15 - 1]; length l:
+// P = pi_l (1 - s_l), pi_0 = 1, pi_{l+1} = pi_l s_l; value t: n_t / nz; in a
+// multi-symbol model every symbol that can occur gets max(1, floor(P 2^15))
+// and the largest (first on ties) absorbs the difference to 2^15.
+//
+// Work is per non-zero symbol (about 2 + log2 of its run coding steps), not
+// per coordinate: one thread per chunk, which finds its stretch of the
+// ascending merge of the two hybrid lists (Q_A: p = 1; Q_B: the rest) by a
+// merge-path search and walks it backwards.  The encoder runs twice, first
+// counting each chunk's words, then (after a per-worker scan of the counts)
+// writing them.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstdint>
+
+#include "gs_device.cuh"
+#include "gs_launch.h"
+#include "gs_trace.h"
+
+namespace gs {
+namespace {
+
+constexpr int kScale = 15;
+constexpr uint32_t kM = 1u << kScale;          // total frequency
+constexpr uint32_t kLow = 1u << 15;            // lower end of the state interval
+constexpr int kLens = 31;                      // run bit lengths 0 .. 30
+constexpr int kBitModels = 30;
+constexpr int kHeaderWords = 9;
+constexpr int kDirWords = 3;
+
+// One symbol of a model: frequency, cumulative start, and the exact
+// reciprocal pair for floor(x / f) = (x * rcp) >> sh on x < 2^31.
+struct Sym {
+    uint32_t f, c, rcp, sh;
+};
+
+struct DenseModel {
+    Sym len[kLens];
+    Sym bit0[kBitModels], bit1[kBitModels];
+    Sym val[3];                 // +1, -1, 2
+    uint32_t len_c[kLens + 1];  // cumulative starts for the decoder's search
+    int64_t n_pos, n_neg, n_cap, nz;
+    int64_t n_chunks, chunk0;   // chunks of this worker, and the chunks of all workers before it
+    int64_t words;              // total words of the worker's code (after the scan)
+    int log2_k;                 // non-zero symbols per chunk (log2)
+    int status;                 // unused
+};
+
+// floor(x / f) = (x * rcp) >> sh for every x < 2^31, with s = ceil(log2 f),
+// rcp = ceil(2^(31+s) / f), sh = 31 + s: rcp = 2^(31+s)/f + e (0 <= e < 1), so
+// the product overshoots x / f by x e / 2^(31+s) < 2^-s <= 1 / f, less than the
+// gap between x / f and the next integer.
+__device__ __forceinline__ Sym make_sym(uint32_t f, uint32_t c) {
+    Sym y;
+    y.f = f;
+    y.c = c;
+    int s = 0;
+    while ((1u << s) < f) ++s;
+    y.sh = 31 + s;
+    y.rcp = f ? (uint32_t)((((unsigned long long)1 << y.sh) + f - 1) / f) : 0u;
+    return y;
+}
+
+// max(1, floor(P 2^15)) for the symbols that can occur; the largest absorbs the rest.
+__device__ void quantise(const double* P, const bool* can, int n, uint32_t* f) {
+    long long sum = 0;
+    int best = 0;
+    for (int s = 0; s < n; ++s) {
+        uint32_t q = 0;
+        if (can[s]) {
+            const double t = floor(__dmul_rn(P[s], (double)kM));
+            q = t < 1.0 ? 1u : (uint32_t)t;
+        }
+        f[s] = q;
+        sum += q;
+        if (q > f[best]) best = s;
+    }
+    f[best] = (uint32_t)((long long)f[best] + (long long)kM - sum);
+}
+
+__device__ void build_model(int64_t d, int64_t n_pos, int64_t n_neg, int64_t n_cap, DenseModel& m) {
+    const int64_t nz = n_pos + n_neg + n_cap;
+    m.n_pos = n_pos;
+    m.n_neg = n_neg;
+    m.n_cap = n_cap;
+    m.nz = nz;
+    double sq[kLens], P[kLens];
+    bool can[kLens];
+    uint32_t f[kLens];
+    sq[0] = __ddiv_rn((double)(d - nz), (double)d);
+    for (int k = 1; k < kLens; ++k) sq[k] = __dmul_rn(sq[k - 1], sq[k - 1]);
+    for (int k = 0; k < kBitModels; ++k) {
+        const double r = __ddiv_rn(sq[k], __dadd_rn(1.0, sq[k]));
+        uint32_t f1 = ((uint32_t)floor(__dmul_rn(r, 65536.0)) + 1u) >> 1;
+        f1 = min(max(f1, 1u), kM - 1u);
+        m.bit0[k] = make_sym(kM - f1, 0u);
+        m.bit1[k] = make_sym(f1, kM - f1);
+    }
+    double pi = 1.0;
+    for (int l = 0; l < kLens; ++l) {
+        P[l] = __dmul_rn(pi, __dsub_rn(1.0, sq[l]));
+        pi = __dmul_rn(pi, sq[l]);
+        can[l] = true;
+    }
+    quantise(P, can, kLens, f);
+    uint32_t c = 0;
+    for (int l = 0; l < kLens; ++l) {
+        m.len[l] = make_sym(f[l], c);
+        m.len_c[l] = c;
+        c += f[l];
+    }
+    m.len_c[kLens] = c;
+    double Pv[3];
+    bool cv[3];
+    const int64_t nt[3] = {n_pos, n_neg, n_cap};
+    for (int t = 0; t < 3; ++t) {
+        Pv[t] = nz > 0 ? __ddiv_rn((double)nt[t], (double)nz) : 0.0;
+        cv[t] = nt[t] > 0;
+    }
+    if (nz == 0) cv[0] = true;   // an unused model still sums to 2^15
+    uint32_t fv[3];
+    quantise(Pv, cv, 3, fv);
+    c = 0;
+    for (int t = 0; t < 3; ++t) {
+        m.val[t] = make_sym(fv[t], c);
+        c += fv[t];
+    }
+}
+
+// The two hybrid lists of one worker, ascending: Q_A indices (value 2) and
+// Q_B codes 2 i + [g_i < 0] (value -1 or +1).
+struct Lists2 {
+    const int32_t* a;
+    const uint32_t* b;
+    int na, nb;
+    __device__ __forceinline__ int bi(int j) const { return (int)(b[j] >> 1); }
+};
+
+// Number of Q_A entries among the r smallest indices of the merge.
+__device__ __forceinline__ int merge_split(const Lists2& L, int r) {
+    int lo = max(0, r - L.nb), hi = min(r, L.na);
+    while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (L.a[mid] < L.bi(r - mid - 1)) lo = mid + 1; else hi = mid;
+    }
+    return lo;
+}
+
+// One rANS coding step on the encoder's state; `w` (NULL while counting)
+// receives emitted word number n at w[-n] (the stream is stored last-first).
+__device__ __forceinline__ void put(uint32_t& x, const Sym& s, uint16_t* w, int& n) {
+    if (x >= (s.f << 16)) {
+        if (w) w[-n] = (uint16_t)(x & 0xFFFFu);
+        ++n;
+        x >>= 16;
+    }
+    const uint32_t q = (uint32_t)(((unsigned long long)x * s.rcp) >> s.sh);
+    x += s.c + q * (kM - s.f);
+}
+
+// Encodes the non-zero symbols of merge ranks [r0, r1) of one worker (one
+// chunk).  With out == NULL it only counts the emitted words (n_out) and
+// finds the chunk's first index; otherwise it writes the stream at out,
+// given the count n_emitted from the counting pass.
+__device__ void encode_chunk(const DenseModel& md, const Lists2& L, int64_t r0, int64_t r1, uint16_t* out,
+                             int n_emitted, int& n_out, int32_t& first) {
+    int ia = merge_split(L, (int)r1);
+    int ib = (int)r1 - ia;
+    // pop the largest remaining merge element: its index and value symbol (0: +1, 1: -1, 2: 2)
+    auto pop = [&](int& idx, int& t) {
+        const bool take_a = ib == 0 || (ia > 0 && L.a[ia - 1] > L.bi(ib - 1));
+        if (take_a) {
+            --ia;
+            idx = L.a[ia];
+            t = 2;
+        } else {
+            --ib;
+            const uint32_t code = L.b[ib];
+            idx = (int)(code >> 1);
+            t = (int)(code & 1u);
+        }
+    };
+    uint32_t x = kLow;
+    int n = 0;
+    // The emitted words go last-first right after the two state words; the
+    // writing pass knows their number from the counting pass.
+    uint16_t* w = out ? out + 2 + (n_emitted - 1) : nullptr;
+    int idx, t;
+    pop(idx, t);
+    for (int64_t j = r1 - 1; j >= r0; --j) {
+        put(x, md.val[t], w, n);
+        if (j == r0) break;
+        int pidx, pt;
+        pop(pidx, pt);
+        const uint32_t v = (uint32_t)(idx - pidx);   // run of zeros + 1
+        const int l = 31 - __clz(v);
+        for (int k = 0; k < l; ++k) put(x, ((v >> k) & 1u) ? md.bit1[k] : md.bit0[k], w, n);
+        put(x, md.len[l], w, n);
+        idx = pidx;
+        t = pt;
+    }
+    first = idx;
+    if (out) {
+        out[0] = (uint16_t)(x >> 16);
+        out[1] = (uint16_t)(x & 0xFFFFu);
+    }
+    n_out = n;
+}
+
+__device__ __forceinline__ void put32(uint16_t* w, uint32_t v) {
+    w[0] = (uint16_t)(v & 0xFFFFu);
+    w[1] = (uint16_t)(v >> 16);
+}
+__device__ __forceinline__ uint32_t get32(const uint16_t* w) { return (uint32_t)w[0] | ((uint32_t)w[1] << 16); }
+
+// Per-worker count of the -1 symbols among the Q_B codes (grid: x over the
+// list, y over workers).
+__global__ void k_dense_count(const uint32_t* __restrict__ qb, const int32_t* __restrict__ n_b, int64_t cap,
+                              unsigned long long* neg) {
+    grid_dep_wait();
+    const int m = blockIdx.y;
+    const int64_t n = min((int64_t)n_b[m], cap);
+    const uint32_t* b = qb + (int64_t)m * cap;
+    int cnt = 0;
+    for (int64_t j = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; j < n; j += (int64_t)gridDim.x * blockDim.x)
+        cnt += (int)(b[j] & 1u);
+    cnt = warp_sum(cnt);
+    if ((threadIdx.x & 31) == 0 && cnt) atomicAdd(neg + m, (unsigned long long)cnt);
+}
+
+// One block: every worker's model and chunk count, the header words, and
+// the chunks of all workers before each (serial over the workers).
+__global__ void k_dense_setup(const int32_t* __restrict__ n_a, const int32_t* __restrict__ n_b,
+                              const unsigned long long* __restrict__ neg, int M, int64_t d, int64_t cap, int log2_k,
+                              DenseModel* md, uint16_t* words, int64_t word_cap, int64_t* total_chunks, int* status) {
+    grid_dep_wait();
+    for (int m = threadIdx.x; m < M; m += blockDim.x) {
+        const int64_t na = n_a[m], nb = n_b[m];
+        DenseModel& mm = md[m];
+        if (na > cap || nb > cap || na < 0 || nb < 0 || na + nb > d) {
+            atomicOr(status, kStInvalid);   // lists that overflowed their capacity cannot be coded
+            build_model(d, 0, 0, 0, mm);
+            mm.n_chunks = 0;
+        } else {
+            const int64_t nn = (int64_t)neg[m];
+            build_model(d, nb - nn, nn, na, mm);
+            mm.n_chunks = (mm.nz + ((int64_t)1 << log2_k) - 1) >> log2_k;
+        }
+        mm.log2_k = log2_k;
+        mm.status = 0;
+        if (word_cap >= kHeaderWords) {
+            uint16_t* w = words + (int64_t)m * word_cap;
+            put32(w, (uint32_t)d);
+            put32(w + 2, (uint32_t)mm.n_pos);
+            put32(w + 4, (uint32_t)mm.n_neg);
+            put32(w + 6, (uint32_t)mm.n_cap);
+            w[8] = (uint16_t)log2_k;
+        }
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int64_t acc = 0;
+        for (int m = 0; m < M; ++m) {
+            md[m].chunk0 = acc;
+            acc += md[m].n_chunks;
+        }
+        *total_chunks = acc;
+    }
+}
+
+// The worker of global chunk g (chunk0 ascending).
+__device__ __forceinline__ int chunk_worker(const DenseModel* md, int M, int64_t g) {
+    int a = 0, b = M - 1;
+    while (a < b) {
+        const int mid = (a + b + 1) >> 1;
+        if (md[mid].chunk0 <= g) a = mid; else b = mid - 1;
+    }
+    return a;
+}
+
+// Counting pass (kWrite false): each chunk's stream length and first index.
+// Writing pass: each chunk's stream at its offset (codes that fit only).
+template <bool kWrite>
+__global__ void k_dense_encode(const int32_t* __restrict__ qa, const uint32_t* __restrict__ qb,
+                               const DenseModel* __restrict__ md, int M, int64_t cap, int log2_k,
+                               const int64_t* __restrict__ total_chunks, int32_t* ch_len, int32_t* ch_first,
+                               const int64_t* __restrict__ ch_off, uint16_t* words, int64_t word_cap) {
+    grid_dep_wait();
+    const int64_t total = *total_chunks;
+    for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < total; g += (int64_t)gridDim.x * blockDim.x) {
+        const int m = chunk_worker(md, M, g);
+        const DenseModel& mm = md[m];
+        if (kWrite && mm.words > word_cap) continue;
+        const int64_t i = g - mm.chunk0;
+        const int64_t r0 = i << log2_k, r1 = min(r0 + ((int64_t)1 << log2_k), mm.nz);
+        Lists2 L;
+        L.a = qa + (int64_t)m * cap;
+        L.b = qb + (int64_t)m * cap;
+        L.na = (int)mm.n_cap;
+        L.nb = (int)(mm.n_pos + mm.n_neg);
+        int n = 0;
+        int32_t first = 0;
+        if (!kWrite) {
+            encode_chunk(mm, L, r0, r1, nullptr, 0, n, first);
+            ch_len[g] = n + 2;
+            ch_first[g] = first;
+        } else {
+            uint16_t* out = words + (int64_t)m * word_cap + kHeaderWords + kDirWords * mm.n_chunks + ch_off[g];
+            encode_chunk(mm, L, r0, r1, out, ch_len[g] - 2, n, first);
+        }
+    }
+}
+
+// One block per worker: stream offsets of its chunks (exclusive scan of the
+// lengths), the directory, the worker's total words and the capacity check.
+__global__ void k_dense_scan(DenseModel* md, const int32_t* __restrict__ ch_len, const int32_t* __restrict__ ch_first,
+                             int64_t* ch_off, uint16_t* words, int64_t word_cap, int64_t* n_words, int* status) {
+    grid_dep_wait();
+    __shared__ int64_t s_tot[33];
+    const int m = blockIdx.x;
+    DenseModel& mm = md[m];
+    const int64_t n = mm.n_chunks, c0 = mm.chunk0;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    int64_t run = 0;
+    for (int64_t b0 = 0; b0 < n; b0 += blockDim.x) {
+        const int64_t i = b0 + threadIdx.x;
+        const int64_t v = i < n ? ch_len[c0 + i] : 0;
+        int64_t inc = v;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int64_t t = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+            if (lane >= o) inc += t;
+        }
+        if (lane == 31) s_tot[warp] = inc;
+        __syncthreads();
+        int64_t before = 0, all = 0;
+        for (int w = 0; w < nw; ++w) {
+            before += w < warp ? s_tot[w] : 0;
+            all += s_tot[w];
+        }
+        if (i < n) ch_off[c0 + i] = run + before + inc - v;
+        run += all;
+        __syncthreads();
+    }
+    const int64_t total = kHeaderWords + kDirWords * n + run;
+    if (threadIdx.x == 0) {
+        mm.words = total;
+        n_words[m] = total;
+        if (total > word_cap) atomicOr(status, kStCapacity);
+    }
+    if (total <= word_cap) {
+        uint16_t* dir = words + (int64_t)m * word_cap + kHeaderWords;
+        for (int64_t i = threadIdx.x; i < n; i += blockDim.x) {
+            put32(dir + kDirWords * i, (uint32_t)ch_first[c0 + i]);
+            dir[kDirWords * i + 2] = (uint16_t)ch_len[c0 + i];
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Decoder
+// ---------------------------------------------------------------------------
+// One block: every worker's header read back, its model rebuilt, and the
+// chunks of all workers before each.  A malformed header records kStInvalid
+// and leaves that worker with no chunk.
+__global__ void k_dense_dsetup(const uint16_t* __restrict__ words, const int64_t* __restrict__ n_words, int M,
+                               int64_t d, int64_t word_cap, DenseModel* md, int64_t* total_chunks, int* status) {
+    grid_dep_wait();
+    for (int m = threadIdx.x; m < M; m += blockDim.x) {
+        const uint16_t* w = words + (int64_t)m * word_cap;
+        const int64_t nw = n_words[m];
+        DenseModel& mm = md[m];
+        bool ok = nw >= kHeaderWords && nw <= word_cap;
+        int64_t np = 0, nn = 0, nc = 0;
+        int lk = 4;
+        if (ok) {
+            np = get32(w + 2);
+            nn = get32(w + 4);
+            nc = get32(w + 6);
+            lk = w[8];
+            ok = (int64_t)get32(w) == d && lk >= 4 && lk <= 10 && np + nn + nc <= d;
+        }
+        build_model(d, ok ? np : 0, ok ? nn : 0, ok ? nc : 0, mm);
+        mm.log2_k = lk;
+        mm.n_chunks = ok ? (mm.nz + ((int64_t)1 << lk) - 1) >> lk : 0;
+        if (ok && nw < kHeaderWords + kDirWords * mm.n_chunks) {
+            ok = false;
+            mm.n_chunks = 0;
+        }
+        if (!ok) atomicOr(status, kStInvalid);
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int64_t acc = 0;
+        for (int m = 0; m < M; ++m) {
+            md[m].chunk0 = acc;
+            acc += md[m].n_chunks;
+        }
+        *total_chunks = acc;
+    }
+}
+
+// One block per worker: offsets of the chunk streams from the directory's
+// lengths; the streams must fill the code exactly.
+__global__ void k_dense_dscan(DenseModel* md, const uint16_t* __restrict__ words, const int64_t* __restrict__ n_words,
+                              int64_t word_cap, int64_t* ch_off, int* status) {
+    grid_dep_wait();
+    __shared__ int64_t s_tot[33];
+    const int m = blockIdx.x;
+    DenseModel& mm = md[m];
+    const int64_t n = mm.n_chunks, c0 = mm.chunk0;
+    const uint16_t* dir = words + (int64_t)m * word_cap + kHeaderWords;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    int64_t run = 0;
+    for (int64_t b0 = 0; b0 < n; b0 += blockDim.x) {
+        const int64_t i = b0 + threadIdx.x;
+        const int64_t v = i < n ? dir[kDirWords * i + 2] : 0;
+        int64_t inc = v;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int64_t t = __shfl_up_sync(0xFFFFFFFFu, inc, o);
+            if (lane >= o) inc += t;
+        }
+        if (lane == 31) s_tot[warp] = inc;
+        __syncthreads();
+        int64_t before = 0, all = 0;
+        for (int w = 0; w < nw; ++w) {
+            before += w < warp ? s_tot[w] : 0;
+            all += s_tot[w];
+        }
+        if (i < n) ch_off[c0 + i] = run + before + inc - v;
+        run += all;
+        __syncthreads();
+    }
+    if (threadIdx.x == 0 && n > 0 && kHeaderWords + kDirWords * n + run != n_words[m]) {
+        atomicOr(status, kStInvalid);
+        mm.n_chunks = 0;   // (no chunk of this worker is decoded)
+    }
+}
+
+// One rANS decoding step: the symbol whose [c, c + f) holds x's low 15 bits.
+struct Dec {
+    const uint16_t* w;
+    int pos, len;
+    uint32_t x;
+    bool bad;
+    __device__ __forceinline__ void step(uint32_t f, uint32_t c, uint32_t slot) {
+        x = f * (x >> kScale) + slot - c;
+        if (x < kLow) {
+            if (pos < len) x = (x << 16) | w[pos++];
+            else bad = true;
+        }
+    }
+};
+
+// Decodes every chunk into the dense q~ rows (int8, zeroed beforehand).
+__global__ void k_dense_decode(const uint16_t* __restrict__ words, const DenseModel* __restrict__ md, int M,
+                               int64_t d, int64_t word_cap, const int64_t* __restrict__ total_chunks,
+                               const int64_t* __restrict__ ch_off, int8_t* qt, int* status) {
+    grid_dep_wait();
+    const int64_t total = *total_chunks;
+    for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < total; g += (int64_t)gridDim.x * blockDim.x) {
+        const int m = chunk_worker(md, M, g);
+        const DenseModel& mm = md[m];
+        const int64_t i = g - mm.chunk0;
+        if (i >= mm.n_chunks) continue;   // a worker whose directory did not add up
+        const uint16_t* base = words + (int64_t)m * word_cap;
+        const uint16_t* dir = base + kHeaderWords + kDirWords * i;
+        const int64_t K = (int64_t)1 << mm.log2_k;
+        const int64_t cnt = min(K, mm.nz - i * K);
+        Dec r;
+        r.w = base + kHeaderWords + kDirWords * mm.n_chunks + ch_off[g];
+        r.len = dir[2];
+        r.pos = 2;
+        r.bad = r.len < 2;
+        r.x = r.bad ? kLow : (((uint32_t)r.w[0] << 16) | r.w[1]);
+        int64_t idx = get32(dir);
+        int8_t* row = qt + (int64_t)m * d;
+        for (int64_t j = 0; j < cnt && !r.bad; ++j) {
+            if (j > 0) {
+                // run bit length: the last l with len_c[l] <= slot
+                const uint32_t slot = r.x & (kM - 1u);
+                int a = 0, b = kLens - 1;
+                while (a < b) {
+                    const int mid = (a + b + 1) >> 1;
+                    if (mm.len_c[mid] <= slot) a = mid; else b = mid - 1;
+                }
+                r.step(mm.len[a].f, mm.len[a].c, slot);
+                uint32_t v = 1;
+                for (int k = a - 1; k >= 0; --k) {
+                    const uint32_t sl = r.x & (kM - 1u);
+                    const uint32_t f0 = mm.bit0[k].f;
+                    const uint32_t bit = sl >= f0 ? 1u : 0u;
+                    if (bit) r.step(mm.bit1[k].f, mm.bit1[k].c, sl); else r.step(f0, 0u, sl);
+                    v = 2u * v + bit;
+                }
+                idx += v;
+            }
+            const uint32_t sl = r.x & (kM - 1u);
+            const int t = sl < mm.val[1].c ? 0 : (sl < mm.val[2].c ? 1 : 2);
+            r.step(mm.val[t].f, mm.val[t].c, sl);
+            if (idx < 0 || idx >= d) {
+                r.bad = true;
+                break;
+            }
+            row[idx] = t == 0 ? (int8_t)1 : (t == 1 ? (int8_t)-1 : (int8_t)2);
+        }
+        if (r.bad || r.x != kLow || r.pos != r.len) atomicOr(status, kStInvalid);
+    }
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// Host launchers.  The workspace holds, in order: the per-worker -1 counts,
+// the per-worker models, the chunk total, and per chunk its stream length,
+// first index and stream offset.
+// ---------------------------------------------------------------------------
+namespace {
+struct DenseWs {
+    unsigned long long* neg;
+    DenseModel* md;
+    int64_t* total;
+    int32_t* len;
+    int32_t* first;
+    int64_t* off;
+};
+
+size_t up256(size_t b) { return (b + 255) & ~(size_t)255; }
+
+DenseWs carve_dense(void* base, int M, int64_t max_chunks, bool encode, size_t* bytes) {
+    DenseWs w;
+    char* p = static_cast<char*>(base);
+    size_t o = 0;
+    auto take = [&](size_t n) {
+        char* r = p ? p + o : nullptr;
+        o += up256(n);
+        return r;
+    };
+    w.neg = reinterpret_cast<unsigned long long*>(take(sizeof(unsigned long long) * M));
+    w.md = reinterpret_cast<DenseModel*>(take(sizeof(DenseModel) * M));
+    w.total = reinterpret_cast<int64_t*>(take(sizeof(int64_t)));
+    w.len = reinterpret_cast<int32_t*>(take(encode ? sizeof(int32_t) * max_chunks : 0));
+    w.first = reinterpret_cast<int32_t*>(take(encode ? sizeof(int32_t) * max_chunks : 0));
+    w.off = reinterpret_cast<int64_t*>(take(sizeof(int64_t) * max_chunks));
+    if (bytes) *bytes = o;
+    return w;
+}
+
+int grid_for(int64_t items, int threads, int per_sm) {
+    const int64_t b = (items + threads - 1) / threads;
+    return (int)std::max<int64_t>(1, std::min<int64_t>(b, (int64_t)device_sm_count() * per_sm));
+}
+}  // namespace
+
+size_t dense_workspace_bytes(int M, int64_t max_chunks, bool encode) {
+    size_t b = 0;
+    carve_dense(nullptr, M, max_chunks, encode, &b);
+    return b;
+}
+
+cudaError_t launch_dense_encode(const int32_t* qa, const uint32_t* qb, const int32_t* n_a, const int32_t* n_b, int M,
+                                int64_t d, int64_t cap, int log2_k, uint16_t* words, int64_t word_cap,
+                                int64_t* n_words, void* ws, int64_t max_chunks, int* status, cudaStream_t st) {
+    const DenseWs w = carve_dense(ws, M, max_chunks, true, nullptr);
+    cudaError_t e;
+    set_launch_error_site("dense code: count reset");
+    e = cudaMemsetAsync(w.neg, 0, sizeof(unsigned long long) * M, st);
+    if (e != cudaSuccess) return e;
+    {
+        set_launch_error_site("k_dense_count launch");
+        TraceScope ts(kKDenseCount, st);
+        const int bx = std::max(1, std::min(grid_for(cap, 1024, 1), std::max(1, device_sm_count() * 4 / M)));
+        e = launch_dep(k_dense_count, dim3(bx, M), dim3(1024), 0, st, qb, n_b, cap, w.neg);
+        if (e != cudaSuccess) return e;
+    }
+    {
+        set_launch_error_site("k_dense_setup launch");
+        TraceScope ts(kKDenseSetup, st);
+        e = launch_dep(k_dense_setup, dim3(1), dim3(256), 0, st, n_a, n_b, (const unsigned long long*)w.neg, M, d, cap,
+                       log2_k, w.md, words, word_cap, w.total, status);
+        if (e != cudaSuccess) return e;
+    }
+    const int gb = grid_for(max_chunks, 128, 16);
+    {
+        set_launch_error_site("k_dense_encode (count) launch");
+        TraceScope ts(kKDenseEncode, st);
+        e = launch_dep(k_dense_encode<false>, dim3(gb), dim3(128), 0, st, qa, qb, (const DenseModel*)w.md, M, cap,
+                       log2_k, (const int64_t*)w.total, w.len, w.first, (const int64_t*)w.off, words, word_cap);
+        if (e != cudaSuccess) return e;
+    }
+    {
+        set_launch_error_site("k_dense_scan launch");
+        TraceScope ts(kKDenseScan, st);
+        e = launch_dep(k_dense_scan, dim3(M), dim3(512), 0, st, w.md, (const int32_t*)w.len,
+                       (const int32_t*)w.first, w.off, words, word_cap, n_words, status);
+        if (e != cudaSuccess) return e;
+    }
+    set_launch_error_site("k_dense_encode (write) launch");
+    TraceScope ts(kKDenseEncode, st);
+    return launch_dep(k_dense_encode<true>, dim3(gb), dim3(128), 0, st, qa, qb, (const DenseModel*)w.md, M, cap,
+                      log2_k, (const int64_t*)w.total, w.len, w.first, (const int64_t*)w.off, words, word_cap);
+}
+
+cudaError_t launch_dense_decode(const uint16_t* words, const int64_t* n_words, int M, int64_t d, int64_t word_cap,
+                                int8_t* qt, void* ws, int64_t max_chunks, int* status, cudaStream_t st) {
+    const DenseWs w = carve_dense(ws, M, max_chunks, false, nullptr);
+    cudaError_t e;
+    set_launch_error_site("dense decode: output reset");
+    e = cudaMemsetAsync(qt, 0, (size_t)M * (size_t)d, st);
+    if (e != cudaSuccess) return e;
+    {
+        set_launch_error_site("k_dense_dsetup launch");
+        TraceScope ts(kKDenseSetup, st);
+        e = launch_dep(k_dense_dsetup, dim3(1), dim3(256), 0, st, words, n_words, M, d, word_cap, w.md, w.total,
+                       status);
+        if (e != cudaSuccess) return e;
+    }
+    {
+        set_launch_error_site("k_dense_dscan launch");
+        TraceScope ts(kKDenseScan, st);
+        e = launch_dep(k_dense_dscan, dim3(M), dim3(512), 0, st, w.md, words, n_words, word_cap, w.off, status);
+        if (e != cudaSuccess) return e;
+    }
+    set_launch_error_site("k_dense_decode launch");
+    TraceScope ts(kKDenseDecode, st);
+    return launch_dep(k_dense_decode, dim3(grid_for(max_chunks, 128, 16)), dim3(128), 0, st, words,
+                      (const DenseModel*)w.md, M, d, word_cap, (const int64_t*)w.total, (const int64_t*)w.off, qt,
+                      status);
+}
+
+}  // namespace gs

@@ -121,6 +121,15 @@ cudaError_t launch_row_sq(const float* val, const int32_t* nnz, int M, int64_t c
 cudaError_t launch_sum_rows(const float* G, int M, int64_t d, float* v, cudaStream_t st);
 cudaError_t launch_sgd_step(float* w, const float* v, int64_t d, float scale, float eta0, float T0, int t,
                             const float* qsq, const float* gsq, int M, float* log, cudaStream_t st);
+// The dense code of section 3.3 (gs_dense.cu): workspace bytes for M workers
+// and at most max_chunks chunks in all, the encoder of the hybrid lists and
+// the decoder into dense int8 rows.
+size_t dense_workspace_bytes(int M, int64_t max_chunks, bool encode);
+cudaError_t launch_dense_encode(const int32_t* qa, const uint32_t* qb, const int32_t* n_a, const int32_t* n_b, int M,
+                                int64_t d, int64_t cap, int log2_k, uint16_t* words, int64_t word_cap,
+                                int64_t* n_words, void* ws, int64_t max_chunks, int* status, cudaStream_t st);
+cudaError_t launch_dense_decode(const uint16_t* words, const int64_t* n_words, int M, int64_t d, int64_t word_cap,
+                                int8_t* qt, void* ws, int64_t max_chunks, int* status, cudaStream_t st);
 // The launchers record which step failed; the C ABI reports it.
 void set_launch_error_site(const char* where);
 const char* launch_error_site();

@@ -26,6 +26,11 @@ enum KernelId : int {
     kKRowSq,
     kKSumRows,
     kKSgdStep,
+    kKDenseCount,
+    kKDenseSetup,
+    kKDenseEncode,
+    kKDenseScan,
+    kKDenseDecode,
     kNumKernels
 };
 

@@ -78,13 +78,14 @@ def compare_sum(out_gpu, idx_list, val_list, d):
     return ref
 
 
-def oracle_rows(fn, rows, *args, threads=None, **kw):
-    """fn(rows[m], *args, worker=m, **kw) for every worker row, run on host
-    threads (the oracle is plain C called through ctypes, which releases the
-    interpreter lock, and keeps no state between calls).  Returns the results
-    in worker order."""
+def oracle_rows(fn, rows, *args, threads=None, workers=None, **kw):
+    """fn(rows[j], *args, worker=workers[j], **kw) for every row (workers
+    defaults to 0, 1, ...), run on host threads (the oracle is plain C called
+    through ctypes, which releases the interpreter lock, and keeps no state
+    between calls).  Returns the results in row order."""
     n = len(rows)
+    workers = list(range(n)) if workers is None else list(workers)
     threads = threads or min(n, os.cpu_count() or 1)
     with cf.ThreadPoolExecutor(max_workers=max(1, threads)) as ex:
-        futs = [ex.submit(fn, rows[m], *args, worker=m, **kw) for m in range(n)]
+        futs = [ex.submit(fn, rows[j], *args, worker=workers[j], **kw) for j in range(n)]
         return [f.result() for f in futs]
