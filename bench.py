@@ -494,9 +494,12 @@ def run_e2e(gs, g, kappa, w, args, dev, stream, ws):
     rc = gs.gs_sync_status(stream)
     if rc != gs.GS_OK:
         raise RuntimeError(f"device status after e2e: {gs.status_string(rc)}")
+    h2d = M * d * g.element_size()
     return {"value": job_throughput(M * d, ms, ws), "unit": UNIT, "ms_per_step": ms,
-            "h2d_bytes_per_step": M * d * g.element_size(), "d2h_bytes_per_step": d * 4 + M * 4,
-            "api": "gs_pipeline_host", "host_memory": "pinned"}
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d * 4 + M * 4,
+            "h2d_gbs_over_step": round(h2d / (ms / 1e3) / 1e9, 1),
+            "api": "gs_pipeline_host (worker groups copied on two streams while earlier groups compute)",
+            "host_memory": "pinned"}
 
 
 KERNEL_SOURCES = {"k_stream_tma": ("gs_stream_tma.cu", "gs_device.cuh")}
@@ -607,11 +610,58 @@ def run_hybrid(gs, g, kappa, w, args, dev, stream, n_steps, hbm):
     esz = g.element_size()
     algo = M * d * esz + 8 * int(a.sum()) + 4 * int(b_.sum()) + 4 * M
     gbs = algo / (ms / 1e3) / 1e9
-    return {"api": "gs_batched_sparsify_hybrid", "steps": n_steps, "ms_per_step": round(ms, 4),
+    dense = run_dense_code(gs, qa_i, qb, na, nb, d, bits["dense_entropy"], dev, stream, n_steps, hbm)
+    return {"api": "gs_batched_sparsify_hybrid", "dense_coded": dense, "steps": n_steps, "ms_per_step": round(ms, 4),
             "algorithmic_bytes": algo, "achieved": round(gbs, 1), "peak": hbm, "frac": round(gbs / hbm, 4),
             "unit": "GB/s", "n_a": int(a.sum()), "n_b": int(b_.sum()),
             "bits_per_step": {k: round(v) for k, v in bits.items()},
             "bits_per_coordinate": {k: round(v / (M * d), 4) for k, v in bits.items()}}
+
+
+DENSE_LOG2_K = 9   # non-zero symbols per chunk of the dense code
+
+
+def run_dense_code(gs, qa_i, qb, na, nb, d, entropy_bits, dev, stream, n_steps, hbm):
+    """The dense code of section 3.3 (gs_dense_encode / gs_dense_decode) of one
+    step's hybrid lists: its length in bits per coordinate against the model's
+    entropy length sum_s d_s log2(d / d_s), and the time of each direction.
+    Algorithmic bytes: the lists read (4 bytes per entry) and the code written
+    (encoder); the code read and the dense int8 rows written (decoder)."""
+    import torch
+    M = qa_i.shape[0]
+    word_cap = d // 4 + 4096
+    words = torch.empty((M, word_cap), dtype=torch.int16, device=dev)
+    n_words = torch.zeros(M, dtype=torch.int64, device=dev)
+    qt = torch.empty((M, d), dtype=torch.int8, device=dev)
+
+    def timed(fn):
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(n_steps):
+            fn()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / n_steps
+
+    enc = timed(lambda: gs.gs_dense_encode(qa_i, qb, na, nb, d, DENSE_LOG2_K, words, n_words, stream=stream))
+    dec = timed(lambda: gs.gs_dense_decode(words, n_words, d, qt, stream=stream))
+    rc = gs.gs_sync_status(stream)
+    if rc != gs.GS_OK:
+        return {"error": gs.status_string(rc)}
+    total_words = int(n_words.sum().item())
+    entries = int(na.sum().item()) + int(nb.sum().item())
+    b_enc = 4 * entries + 2 * total_words
+    b_dec = 2 * total_words + M * d
+    return {"api": "gs_dense_encode / gs_dense_decode", "log2_k": DENSE_LOG2_K, "words": total_words,
+            "bits_per_coordinate": round(16.0 * total_words / (M * d), 5),
+            "entropy_bits_per_coordinate": round(entropy_bits / (M * d), 5),
+            "over_entropy": round(16.0 * total_words / entropy_bits, 4) if entropy_bits else None,
+            "encode_ms": round(enc, 4), "encode_gbs": round(b_enc / (enc / 1e3) / 1e9, 1),
+            "decode_ms": round(dec, 4), "decode_gbs": round(b_dec / (dec / 1e3) / 1e9, 1),
+            "coords_per_s_encode": M * d / (enc / 1e3), "peak": hbm}
 
 
 def run_resparsify(gs, g, kappa, w, args, dev, stream, n_steps, hbm, ms_fused):

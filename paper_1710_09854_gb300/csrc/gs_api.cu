@@ -29,11 +29,19 @@ struct SegMeta {
     int cpw = 0;
 };
 
+constexpr int kPipeGroups = 8;   // worker groups of gs_pipeline_host (copies overlapped with compute)
+
 struct DevState {
     bool ready = false;
     cudaMemPool_t pool = nullptr;
     int* status = nullptr;  // device word, OR of kSt* bits
     std::map<std::vector<int64_t>, SegMeta> segs;
+    // gs_pipeline_host: two copy streams and the events that order them
+    bool pipe_ready = false;
+    cudaStream_t copy[2] = {nullptr, nullptr};
+    cudaEvent_t ev_start = nullptr;
+    cudaEvent_t ev_group[kPipeGroups] = {};
+    std::mutex pipe_mu;     // one pipeline call at a time per device (they share the events)
 };
 
 std::mutex g_mu;
@@ -162,7 +170,7 @@ void carve(Arena& a, Workspace& w, int n_seg, int n_chunks, int64_t n, bool buil
 gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off, int L, double kappa, int iters,
               uint64_t seed, uint32_t step, uint32_t worker0, int32_t* idx, float* val, int32_t* nnz, int64_t cap,
               gs_info* info, float* p, cudaStream_t st, float* agg_out = nullptr, const HybridOut* hy = nullptr,
-              double eps = -1.0, bool average = false) {
+              double eps = -1.0, bool average = false, bool accumulate = false) {
     const bool prob = p != nullptr;
     const bool alg2 = eps >= 0.0;
     if (!g || M < 1 || d < 1 || d >= kMaxD) return GS_ERR_INVALID_ARG;
@@ -259,7 +267,7 @@ gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off
     if (e == cudaSuccess) {
         if (prob) e = launch_prob(Lo, w.sp, p, st);
         else e = launch_compact(Lo, w.sp, w.ls, n_chunks, idx, val, hy ? w.nnz : nnz, cap, s->status, st, agg_out,
-                                hy, average);
+                                hy, average, accumulate);
     }
     cudaError_t ef = cudaFreeAsync(mem, st);
     if (e != cudaSuccess) return cuda_fail(launch_error_site(), e);
@@ -599,7 +607,7 @@ gs_status gs_dense_encode(const int32_t* qa_idx, const uint32_t* qb_code, const 
     const int64_t per = (std::min<int64_t>(d, 2 * cap) + (1 << log2_k) - 1) >> log2_k;
     const int64_t max_chunks = (int64_t)M * per;
     void* mem = nullptr;
-    GS_TRY(cudaMallocFromPoolAsync(&mem, dense_workspace_bytes(M, max_chunks, true), s->pool, st));
+    GS_TRY(cudaMallocFromPoolAsync(&mem, dense_workspace_bytes(M, max_chunks, std::min<int64_t>(d, 2 * cap), true), s->pool, st));
     const cudaError_t e = launch_dense_encode(qa_idx, qb_code, n_a, n_b, M, d, cap, log2_k, words, word_cap, n_words,
                                               mem, max_chunks, s->status, st);
     const cudaError_t ef = cudaFreeAsync(mem, st);
@@ -620,7 +628,7 @@ gs_status gs_dense_decode(const uint16_t* words, const int64_t* n_words, int M, 
     const int64_t per = std::min<int64_t>((d + 15) / 16, (word_cap - 9) / 3);
     const int64_t max_chunks = std::max<int64_t>(1, (int64_t)M * per);
     void* mem = nullptr;
-    GS_TRY(cudaMallocFromPoolAsync(&mem, dense_workspace_bytes(M, max_chunks, false), s->pool, st));
+    GS_TRY(cudaMallocFromPoolAsync(&mem, dense_workspace_bytes(M, max_chunks, 0, false), s->pool, st));
     const cudaError_t e = launch_dense_decode(words, n_words, M, d, word_cap, qt, mem, max_chunks, s->status, st);
     const cudaError_t ef = cudaFreeAsync(mem, st);
     if (e != cudaSuccess) return cuda_fail(launch_error_site(), e);
@@ -675,11 +683,45 @@ gs_status gs_pipeline_host(const void* g_host, int dtype, int M, int64_t d, doub
     if (M < 1 || M > kMaxAggM || d < 1 || d >= kMaxD || cap < 1) return GS_ERR_INVALID_ARG;
     if (dtype != GS_DTYPE_F32 && dtype != GS_DTYPE_BF16) return GS_ERR_INVALID_ARG;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
-    const size_t esz = dtype == GS_DTYPE_F32 ? 4 : 2;
-    GS_TRY(cudaMemcpyAsync(g_dev, g_host, esz * (size_t)M * (size_t)d, cudaMemcpyHostToDevice, st));
-    const gs_status rc = run(g_dev, dtype, M, d, nullptr, 1, kappa, iters, seed, step, worker0, idx, val, nnz, cap,
-                             nullptr, nullptr, st, out);
+    DevState* s = nullptr;
+    gs_status rc = device_state(&s);
     if (rc != GS_OK) return rc;
+    std::lock_guard<std::mutex> lk(s->pipe_mu);
+    if (!s->pipe_ready) {
+        for (int i = 0; i < 2; ++i) GS_TRY(cudaStreamCreateWithFlags(&s->copy[i], cudaStreamNonBlocking));
+        GS_TRY(cudaEventCreateWithFlags(&s->ev_start, cudaEventDisableTiming));
+        for (int k = 0; k < kPipeGroups; ++k) GS_TRY(cudaEventCreateWithFlags(&s->ev_group[k], cudaEventDisableTiming));
+        s->pipe_ready = true;
+    }
+    const size_t esz = dtype == GS_DTYPE_F32 ? 4 : 2;
+    // Worker groups: group k's copy (alternating between the two copy
+    // streams, which run side by side) is ordered after everything already on
+    // `stream` (an earlier call may still read g_dev) and before group k's
+    // sparsify + sum on `stream`; the sum continues across groups in worker
+    // order, so out is what one call over all M workers would give.
+    const int G = std::min(M, kPipeGroups);
+    GS_TRY(cudaEventRecord(s->ev_start, st));
+    for (int i = 0; i < 2; ++i) GS_TRY(cudaStreamWaitEvent(s->copy[i], s->ev_start, 0));
+    int m0 = 0;
+    for (int k = 0; k < G; ++k) {
+        const int m1 = (int)((int64_t)M * (k + 1) / G);
+        const size_t off = esz * (size_t)m0 * (size_t)d, bytes = esz * (size_t)(m1 - m0) * (size_t)d;
+        cudaStream_t cs = s->copy[k & 1];
+        GS_TRY(cudaMemcpyAsync(static_cast<char*>(g_dev) + off, static_cast<const char*>(g_host) + off, bytes,
+                               cudaMemcpyHostToDevice, cs));
+        GS_TRY(cudaEventRecord(s->ev_group[k], cs));
+        m0 = m1;
+    }
+    m0 = 0;
+    for (int k = 0; k < G; ++k) {
+        const int m1 = (int)((int64_t)M * (k + 1) / G);
+        GS_TRY(cudaStreamWaitEvent(st, s->ev_group[k], 0));
+        rc = run(static_cast<const char*>(g_dev) + esz * (size_t)m0 * (size_t)d, dtype, m1 - m0, d, nullptr, 1,
+                 kappa, iters, seed, step, worker0 + (uint32_t)m0, idx + (int64_t)m0 * cap, val + (int64_t)m0 * cap,
+                 nnz + m0, cap, nullptr, nullptr, st, out, nullptr, -1.0, false, k > 0);
+        if (rc != GS_OK) return rc;
+        m0 = m1;
+    }
     GS_TRY(cudaMemcpyAsync(out_host, out, sizeof(float) * (size_t)d, cudaMemcpyDeviceToHost, st));
     GS_TRY(cudaMemcpyAsync(nnz_host, nnz, sizeof(int32_t) * (size_t)M, cudaMemcpyDeviceToHost, st));
     return GS_OK;

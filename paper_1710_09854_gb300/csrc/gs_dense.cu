@@ -36,11 +36,12 @@
 // and the largest (first on ties) absorbs the difference to 2^15.
 //
 // Work is per non-zero symbol (about 2 + log2 of its run coding steps), not
-// per coordinate: one thread per chunk, which finds its stretch of the
-// ascending merge of the two hybrid lists (Q_A: p = 1; Q_B: the rest) by a
-// merge-path search and walks it backwards.  The encoder runs twice, first
-// counting each chunk's words, then (after a per-worker scan of the counts)
-// writing them.
+// per coordinate.  The two hybrid lists (Q_A: p = 1; Q_B: the rest) are
+// first merged into one ascending sequence of (index, value) per worker (a
+// warp per chunk, merge-path placement in shared memory); then one thread
+// per chunk runs the chunk's rANS chain from the end of its stretch, once to
+// count its words and, after a per-worker scan of the counts, once to write
+// them.  The decoder runs one thread per chunk too.
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -191,53 +192,69 @@ __device__ __forceinline__ void put(uint32_t& x, const Sym& s, uint16_t* w, int&
     x += s.c + q * (kM - s.f);
 }
 
-// Encodes the non-zero symbols of merge ranks [r0, r1) of one worker (one
-// chunk).  With out == NULL it only counts the emitted words (n_out) and
-// finds the chunk's first index; otherwise it writes the stream at out,
-// given the count n_emitted from the counting pass.
-__device__ void encode_chunk(const DenseModel& md, const Lists2& L, int64_t r0, int64_t r1, uint16_t* out,
-                             int n_emitted, int& n_out, int32_t& first) {
-    int ia = merge_split(L, (int)r1);
-    int ib = (int)r1 - ia;
-    // pop the largest remaining merge element: its index and value symbol (0: +1, 1: -1, 2: 2)
-    auto pop = [&](int& idx, int& t) {
-        const bool take_a = ib == 0 || (ia > 0 && L.a[ia - 1] > L.bi(ib - 1));
-        if (take_a) {
-            --ia;
-            idx = L.a[ia];
-            t = 2;
-        } else {
-            --ib;
-            const uint32_t code = L.b[ib];
-            idx = (int)(code >> 1);
-            t = (int)(code & 1u);
+// Shared memory of one warp's chunk: the worker's model, the chunk's
+// stretches of the two lists, and their merge (indices and value symbols).
+constexpr int kDenseWarps = 4;   // chunks (warps) per block
+
+__host__ __device__ constexpr size_t model_bytes() { return (sizeof(DenseModel) + 15) & ~(size_t)15; }
+__host__ __device__ constexpr size_t warp_bytes(int K) {
+    return model_bytes() + (size_t)K * (sizeof(int32_t) + sizeof(uint32_t) + sizeof(int32_t) + 1) + 16;
+}
+
+struct Staged {
+    DenseModel* md;
+    int32_t* sa;     // the chunk's Q_A stretch
+    uint32_t* sb;    // its Q_B stretch
+    int32_t* idx;    // merged indices
+    uint8_t* typ;    // merged value symbols (0: +1, 1: -1, 2: 2)
+};
+
+__device__ __forceinline__ Staged staged_at(unsigned char* base, int K) {
+    Staged t;
+    t.md = reinterpret_cast<DenseModel*>(base);
+    t.sa = reinterpret_cast<int32_t*>(base + model_bytes());
+    t.sb = reinterpret_cast<uint32_t*>(t.sa + K);
+    t.idx = reinterpret_cast<int32_t*>(t.sb + K);
+    t.typ = reinterpret_cast<uint8_t*>(t.idx + K);
+    return t;
+}
+
+__device__ __forceinline__ void copy_model(DenseModel* dst, const DenseModel* src, int lane) {
+    const uint32_t* s = reinterpret_cast<const uint32_t*>(src);
+    uint32_t* d = reinterpret_cast<uint32_t*>(dst);
+    for (int i = lane; i < (int)(sizeof(DenseModel) / 4); i += 32) d[i] = s[i];
+}
+
+// The warp stages the merge ranks [r0, r1) of worker lists L: both lists'
+// stretches are loaded, then each lane places its output positions by a
+// merge-path search in shared memory.
+__device__ void stage_merge(const Lists2& L, int r0, int r1, const Staged& t, int lane) {
+    int ia0 = 0, ia1 = 0;
+    if (lane == 0) ia0 = merge_split(L, r0);
+    if (lane == 1) ia1 = merge_split(L, r1);
+    ia0 = __shfl_sync(0xFFFFFFFFu, ia0, 0);
+    ia1 = __shfl_sync(0xFFFFFFFFu, ia1, 1);
+    const int ib0 = r0 - ia0, na = ia1 - ia0, nb = (r1 - ia1) - ib0;
+    for (int i = lane; i < na; i += 32) t.sa[i] = L.a[ia0 + i];
+    for (int i = lane; i < nb; i += 32) t.sb[i] = L.b[ib0 + i];
+    __syncwarp();
+    for (int p = lane; p < r1 - r0; p += 32) {
+        int lo = max(0, p - nb), hi = min(p, na);   // A entries among the p smallest
+        while (lo < hi) {
+            const int mid = (lo + hi) >> 1;
+            if (t.sa[mid] < (int)(t.sb[p - mid - 1] >> 1)) lo = mid + 1; else hi = mid;
         }
-    };
-    uint32_t x = kLow;
-    int n = 0;
-    // The emitted words go last-first right after the two state words; the
-    // writing pass knows their number from the counting pass.
-    uint16_t* w = out ? out + 2 + (n_emitted - 1) : nullptr;
-    int idx, t;
-    pop(idx, t);
-    for (int64_t j = r1 - 1; j >= r0; --j) {
-        put(x, md.val[t], w, n);
-        if (j == r0) break;
-        int pidx, pt;
-        pop(pidx, pt);
-        const uint32_t v = (uint32_t)(idx - pidx);   // run of zeros + 1
-        const int l = 31 - __clz(v);
-        for (int k = 0; k < l; ++k) put(x, ((v >> k) & 1u) ? md.bit1[k] : md.bit0[k], w, n);
-        put(x, md.len[l], w, n);
-        idx = pidx;
-        t = pt;
+        const bool from_a = lo < na && (p - lo >= nb || t.sa[lo] < (int)(t.sb[p - lo] >> 1));
+        if (from_a) {
+            t.idx[p] = t.sa[lo];
+            t.typ[p] = 2;
+        } else {
+            const uint32_t code = t.sb[p - lo];
+            t.idx[p] = (int32_t)(code >> 1);
+            t.typ[p] = (uint8_t)(code & 1u);
+        }
     }
-    first = idx;
-    if (out) {
-        out[0] = (uint16_t)(x >> 16);
-        out[1] = (uint16_t)(x & 0xFFFFu);
-    }
-    n_out = n;
+    __syncwarp();
 }
 
 __device__ __forceinline__ void put32(uint16_t* w, uint32_t v) {
@@ -311,13 +328,75 @@ __device__ __forceinline__ int chunk_worker(const DenseModel* md, int M, int64_t
     return a;
 }
 
+// The merge of every worker's two lists into one ascending sequence of
+// (index, value symbol), one warp per chunk: the warp stages the chunk's
+// stretches in shared memory, merges them there, and writes the chunk's
+// stretch of the merged sequence (worker m's at m * stride).
+__global__ void __launch_bounds__(kDenseWarps * 32)
+    k_dense_merge(const int32_t* __restrict__ qa, const uint32_t* __restrict__ qb, const DenseModel* __restrict__ md,
+                  int M, int64_t cap, int log2_k, const int64_t* __restrict__ total_chunks, int32_t* m_idx,
+                  uint8_t* m_typ, int64_t stride) {
+    grid_dep_wait();
+    extern __shared__ __align__(16) unsigned char dsm[];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int K = 1 << log2_k;
+    const Staged t = staged_at(dsm + warp * warp_bytes(K), K);
+    const int64_t total = *total_chunks;
+    for (int64_t g = (int64_t)blockIdx.x * kDenseWarps + warp; g < total; g += (int64_t)gridDim.x * kDenseWarps) {
+        const int m = chunk_worker(md, M, g);
+        const int64_t i = g - md[m].chunk0;
+        const int r0 = (int)(i << log2_k), r1 = (int)min((int64_t)r0 + K, md[m].nz);
+        Lists2 L;
+        L.a = qa + (int64_t)m * cap;
+        L.b = qb + (int64_t)m * cap;
+        L.na = (int)md[m].n_cap;
+        L.nb = (int)(md[m].n_pos + md[m].n_neg);
+        stage_merge(L, r0, r1, t, lane);
+        int32_t* oi = m_idx + (int64_t)m * stride + r0;
+        uint8_t* ot = m_typ + (int64_t)m * stride + r0;
+        for (int p = lane; p < r1 - r0; p += 32) {
+            oi[p] = t.idx[p];
+            ot[p] = t.typ[p];
+        }
+        __syncwarp();
+    }
+}
+
+// rANS encoding of merge ranks [r0, r1) of one worker from its merged
+// sequence (one thread): returns the number of emitted words; with out,
+// writes the stream there (n_emitted from the counting pass).
+__device__ int encode_seq(const DenseModel& md, const int32_t* idx, const uint8_t* typ, int r0, int r1,
+                          uint16_t* out, int n_emitted) {
+    uint32_t x = kLow;
+    int n = 0;
+    uint16_t* w = out ? out + 2 + (n_emitted - 1) : nullptr;
+    int cur = idx[r1 - 1];
+    for (int j = r1 - 1; j >= r0; --j) {
+        put(x, md.val[typ[j]], w, n);
+        if (j == r0) break;
+        const int prev = idx[j - 1];
+        const uint32_t v = (uint32_t)(cur - prev);   // run of zeros + 1
+        const int l = 31 - __clz(v);
+        for (int k = 0; k < l; ++k) put(x, ((v >> k) & 1u) ? md.bit1[k] : md.bit0[k], w, n);
+        put(x, md.len[l], w, n);
+        cur = prev;
+    }
+    if (out) {
+        out[0] = (uint16_t)(x >> 16);
+        out[1] = (uint16_t)(x & 0xFFFFu);
+    }
+    return n;
+}
+
 // Counting pass (kWrite false): each chunk's stream length and first index.
 // Writing pass: each chunk's stream at its offset (codes that fit only).
+// One thread per chunk, reading the merged sequence.
 template <bool kWrite>
-__global__ void k_dense_encode(const int32_t* __restrict__ qa, const uint32_t* __restrict__ qb,
-                               const DenseModel* __restrict__ md, int M, int64_t cap, int log2_k,
-                               const int64_t* __restrict__ total_chunks, int32_t* ch_len, int32_t* ch_first,
-                               const int64_t* __restrict__ ch_off, uint16_t* words, int64_t word_cap) {
+__global__ void __launch_bounds__(128)
+    k_dense_encode(const int32_t* __restrict__ m_idx, const uint8_t* __restrict__ m_typ, int64_t stride,
+                   const DenseModel* __restrict__ md, int M, int log2_k, const int64_t* __restrict__ total_chunks,
+                   int32_t* ch_len, int32_t* ch_first, const int64_t* __restrict__ ch_off, uint16_t* words,
+                   int64_t word_cap) {
     grid_dep_wait();
     const int64_t total = *total_chunks;
     for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < total; g += (int64_t)gridDim.x * blockDim.x) {
@@ -325,21 +404,15 @@ __global__ void k_dense_encode(const int32_t* __restrict__ qa, const uint32_t* _
         const DenseModel& mm = md[m];
         if (kWrite && mm.words > word_cap) continue;
         const int64_t i = g - mm.chunk0;
-        const int64_t r0 = i << log2_k, r1 = min(r0 + ((int64_t)1 << log2_k), mm.nz);
-        Lists2 L;
-        L.a = qa + (int64_t)m * cap;
-        L.b = qb + (int64_t)m * cap;
-        L.na = (int)mm.n_cap;
-        L.nb = (int)(mm.n_pos + mm.n_neg);
-        int n = 0;
-        int32_t first = 0;
+        const int r0 = (int)(i << log2_k), r1 = (int)min((int64_t)r0 + ((int64_t)1 << log2_k), mm.nz);
+        const int32_t* idx = m_idx + (int64_t)m * stride;
+        const uint8_t* typ = m_typ + (int64_t)m * stride;
         if (!kWrite) {
-            encode_chunk(mm, L, r0, r1, nullptr, 0, n, first);
-            ch_len[g] = n + 2;
-            ch_first[g] = first;
+            ch_len[g] = encode_seq(mm, idx, typ, r0, r1, nullptr, 0) + 2;
+            ch_first[g] = idx[r0];
         } else {
             uint16_t* out = words + (int64_t)m * word_cap + kHeaderWords + kDirWords * mm.n_chunks + ch_off[g];
-            encode_chunk(mm, L, r0, r1, out, ch_len[g] - 2, n, first);
+            encode_seq(mm, idx, typ, r0, r1, out, ch_len[g] - 2);
         }
     }
 }
@@ -486,10 +559,12 @@ struct Dec {
     }
 };
 
-// Decodes every chunk into the dense q~ rows (int8, zeroed beforehand).
-__global__ void k_dense_decode(const uint16_t* __restrict__ words, const DenseModel* __restrict__ md, int M,
-                               int64_t d, int64_t word_cap, const int64_t* __restrict__ total_chunks,
-                               const int64_t* __restrict__ ch_off, int8_t* qt, int* status) {
+// Decodes every chunk into the dense q~ rows (int8, zeroed beforehand), one
+// thread per chunk.
+__global__ void __launch_bounds__(128)
+    k_dense_decode(const uint16_t* __restrict__ words, const DenseModel* __restrict__ md, int M, int64_t d,
+                   int64_t word_cap, const int64_t* __restrict__ total_chunks, const int64_t* __restrict__ ch_off,
+                   int8_t* qt, int* status) {
     grid_dep_wait();
     const int64_t total = *total_chunks;
     for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < total; g += (int64_t)gridDim.x * blockDim.x) {
@@ -557,11 +632,13 @@ struct DenseWs {
     int32_t* len;
     int32_t* first;
     int64_t* off;
+    int32_t* m_idx;    // encoder: each worker's merged sequence (row stride `stride`)
+    uint8_t* m_typ;
 };
 
 size_t up256(size_t b) { return (b + 255) & ~(size_t)255; }
 
-DenseWs carve_dense(void* base, int M, int64_t max_chunks, bool encode, size_t* bytes) {
+DenseWs carve_dense(void* base, int M, int64_t max_chunks, int64_t stride, bool encode, size_t* bytes) {
     DenseWs w;
     char* p = static_cast<char*>(base);
     size_t o = 0;
@@ -576,6 +653,8 @@ DenseWs carve_dense(void* base, int M, int64_t max_chunks, bool encode, size_t* 
     w.len = reinterpret_cast<int32_t*>(take(encode ? sizeof(int32_t) * max_chunks : 0));
     w.first = reinterpret_cast<int32_t*>(take(encode ? sizeof(int32_t) * max_chunks : 0));
     w.off = reinterpret_cast<int64_t*>(take(sizeof(int64_t) * max_chunks));
+    w.m_idx = reinterpret_cast<int32_t*>(take(encode ? sizeof(int32_t) * (size_t)M * stride : 0));
+    w.m_typ = reinterpret_cast<uint8_t*>(take(encode ? (size_t)M * stride : 0));
     if (bytes) *bytes = o;
     return w;
 }
@@ -586,16 +665,17 @@ int grid_for(int64_t items, int threads, int per_sm) {
 }
 }  // namespace
 
-size_t dense_workspace_bytes(int M, int64_t max_chunks, bool encode) {
+size_t dense_workspace_bytes(int M, int64_t max_chunks, int64_t stride, bool encode) {
     size_t b = 0;
-    carve_dense(nullptr, M, max_chunks, encode, &b);
+    carve_dense(nullptr, M, max_chunks, stride, encode, &b);
     return b;
 }
 
 cudaError_t launch_dense_encode(const int32_t* qa, const uint32_t* qb, const int32_t* n_a, const int32_t* n_b, int M,
                                 int64_t d, int64_t cap, int log2_k, uint16_t* words, int64_t word_cap,
                                 int64_t* n_words, void* ws, int64_t max_chunks, int* status, cudaStream_t st) {
-    const DenseWs w = carve_dense(ws, M, max_chunks, true, nullptr);
+    const int64_t stride = std::min<int64_t>(d, 2 * cap);   // at most this many non-zero symbols per worker
+    const DenseWs w = carve_dense(ws, M, max_chunks, stride, true, nullptr);
     cudaError_t e;
     set_launch_error_site("dense code: count reset");
     e = cudaMemsetAsync(w.neg, 0, sizeof(unsigned long long) * M, st);
@@ -614,12 +694,25 @@ cudaError_t launch_dense_encode(const int32_t* qa, const uint32_t* qb, const int
                        log2_k, w.md, words, word_cap, w.total, status);
         if (e != cudaSuccess) return e;
     }
+    const size_t smem = kDenseWarps * warp_bytes(1 << log2_k);
+    set_launch_error_site("k_dense_merge shared-memory attribute");
+    e = cudaFuncSetAttribute(k_dense_merge, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    {
+        set_launch_error_site("k_dense_merge launch");
+        TraceScope ts(kKDenseMerge, st);
+        e = launch_dep(k_dense_merge, dim3(grid_for(max_chunks, kDenseWarps, 16)), dim3(kDenseWarps * 32), smem, st,
+                       qa, qb, (const DenseModel*)w.md, M, cap, log2_k, (const int64_t*)w.total, w.m_idx, w.m_typ,
+                       stride);
+        if (e != cudaSuccess) return e;
+    }
     const int gb = grid_for(max_chunks, 128, 16);
     {
         set_launch_error_site("k_dense_encode (count) launch");
         TraceScope ts(kKDenseEncode, st);
-        e = launch_dep(k_dense_encode<false>, dim3(gb), dim3(128), 0, st, qa, qb, (const DenseModel*)w.md, M, cap,
-                       log2_k, (const int64_t*)w.total, w.len, w.first, (const int64_t*)w.off, words, word_cap);
+        e = launch_dep(k_dense_encode<false>, dim3(gb), dim3(128), 0, st, (const int32_t*)w.m_idx,
+                       (const uint8_t*)w.m_typ, stride, (const DenseModel*)w.md, M, log2_k, (const int64_t*)w.total,
+                       w.len, w.first, (const int64_t*)w.off, words, word_cap);
         if (e != cudaSuccess) return e;
     }
     {
@@ -631,13 +724,14 @@ cudaError_t launch_dense_encode(const int32_t* qa, const uint32_t* qb, const int
     }
     set_launch_error_site("k_dense_encode (write) launch");
     TraceScope ts(kKDenseEncode, st);
-    return launch_dep(k_dense_encode<true>, dim3(gb), dim3(128), 0, st, qa, qb, (const DenseModel*)w.md, M, cap,
-                      log2_k, (const int64_t*)w.total, w.len, w.first, (const int64_t*)w.off, words, word_cap);
+    return launch_dep(k_dense_encode<true>, dim3(gb), dim3(128), 0, st, (const int32_t*)w.m_idx,
+                      (const uint8_t*)w.m_typ, stride, (const DenseModel*)w.md, M, log2_k, (const int64_t*)w.total,
+                      w.len, w.first, (const int64_t*)w.off, words, word_cap);
 }
 
 cudaError_t launch_dense_decode(const uint16_t* words, const int64_t* n_words, int M, int64_t d, int64_t word_cap,
                                 int8_t* qt, void* ws, int64_t max_chunks, int* status, cudaStream_t st) {
-    const DenseWs w = carve_dense(ws, M, max_chunks, false, nullptr);
+    const DenseWs w = carve_dense(ws, M, max_chunks, 0, false, nullptr);
     cudaError_t e;
     set_launch_error_site("dense decode: output reset");
     e = cudaMemsetAsync(qt, 0, (size_t)M * (size_t)d, st);

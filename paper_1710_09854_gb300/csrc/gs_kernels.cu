@@ -1208,7 +1208,7 @@ __global__ void __launch_bounds__(kSumWarps * 32) k_sum(const __grid_constant__ 
                                                         const __grid_constant__ Lists Ls,
                                                         const int32_t* __restrict__ idx,
                                                         const float* __restrict__ val, int64_t cap,
-                                                        int n_slices, float div, float* out) {
+                                                        int n_slices, float div, int accumulate, float* out) {
     grid_dep_wait();
     __shared__ __align__(16) float tile[kSumWarps][kSlice];
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
@@ -1222,9 +1222,14 @@ __global__ void __launch_bounds__(kSumWarps * 32) k_sum(const __grid_constant__ 
     if (t0 >= ch.hi) return;
     const int tlen = (int)min((int64_t)kSlice, ch.hi - t0);
     float* acc = tile[w];
+    if (accumulate) {
+        // Continue a worker-order sum already in out (the earlier workers' part).
+        for (int i = lane; i < kSlice; i += 32) acc[i] = i < tlen ? out[t0 + i] : 0.0f;
+    } else {
 #pragma unroll
-    for (int i = 0; i < kSlice / 128; ++i)
-        reinterpret_cast<float4*>(acc)[i * 32 + lane] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+        for (int i = 0; i < kSlice / 128; ++i)
+            reinterpret_cast<float4*>(acc)[i * 32 + lane] = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+    }
     __syncwarp();
     for (int mb = 0; mb < Lo.M; mb += 32) {
         // Lane q describes worker mb + q: where its run starts and how long it is.
@@ -1535,7 +1540,7 @@ cudaError_t launch_solve(const Layout& Lo, SegParam* sp, const Lists& Ls, int n_
 
 cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, int32_t* idx,
                            float* val, int32_t* nnz, int64_t cap, int* status, cudaStream_t st, float* sum_out,
-                           const HybridOut* hybrid, bool average) {
+                           const HybridOut* hybrid, bool average, bool accumulate) {
     const int blocks = (n_chunks + kEmitWarps - 1) / kEmitWarps;
     cudaError_t e;
     {
@@ -1565,7 +1570,7 @@ cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls
     TraceScope ts(kKSum, st);
     return launch_dep(k_sum, dim3((n_slices + kSumWarps - 1) / kSumWarps), dim3(kSumWarps * 32), 0, st, Lo, Ls,
                       static_cast<const int32_t*>(idx), static_cast<const float*>(val), cap, n_slices,
-                      average ? (float)Lo.M : 0.0f, sum_out);
+                      average ? (float)Lo.M : 0.0f, accumulate ? 1 : 0, sum_out);
 }
 
 cudaError_t launch_prob(const Layout& Lo, const SegParam* sp, float* p, cudaStream_t st) {

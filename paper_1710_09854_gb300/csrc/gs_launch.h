@@ -86,11 +86,13 @@ struct HybridOut {
 
 // Decide, scan and compact; with sum_out also the sparse sum of the M
 // compacted rows into sum_out (d fp32), fused with the compaction (with
-// average, the sum divided by M); with hybrid (L == 1 only) the hybrid code
+// average, the sum divided by M; with accumulate, added in worker order to
+// the sum already in sum_out); with hybrid (L == 1 only) the hybrid code
 // instead of the plain lists.
 cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, int32_t* idx,
                            float* val, int32_t* nnz, int64_t cap, int* status, cudaStream_t st,
-                           float* sum_out = nullptr, const HybridOut* hybrid = nullptr, bool average = false);
+                           float* sum_out = nullptr, const HybridOut* hybrid = nullptr, bool average = false,
+                           bool accumulate = false);
 cudaError_t launch_prob(const Layout& Lo, const SegParam* sp, float* p, cudaStream_t st);
 cudaError_t launch_aggregate(const AggArgs& A, int32_t* off, float* out, int* status, cudaStream_t st);
 cudaError_t launch_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t i0, int64_t n, uint32_t* out,
@@ -124,7 +126,7 @@ cudaError_t launch_sgd_step(float* w, const float* v, int64_t d, float scale, fl
 // The dense code of section 3.3 (gs_dense.cu): workspace bytes for M workers
 // and at most max_chunks chunks in all, the encoder of the hybrid lists and
 // the decoder into dense int8 rows.
-size_t dense_workspace_bytes(int M, int64_t max_chunks, bool encode);
+size_t dense_workspace_bytes(int M, int64_t max_chunks, int64_t stride, bool encode);
 cudaError_t launch_dense_encode(const int32_t* qa, const uint32_t* qb, const int32_t* n_a, const int32_t* n_b, int M,
                                 int64_t d, int64_t cap, int log2_k, uint16_t* words, int64_t word_cap,
                                 int64_t* n_words, void* ws, int64_t max_chunks, int* status, cudaStream_t st);

@@ -27,6 +27,7 @@ enum KernelId : int {
     kKSumRows,
     kKSgdStep,
     kKDenseCount,
+    kKDenseMerge,
     kKDenseSetup,
     kKDenseEncode,
     kKDenseScan,

@@ -312,6 +312,41 @@ def test_pipeline_host_matches_device_path(gs):
     compare_sum(out_h.numpy(), il, vl, d)
 
 
+def test_pipeline_host_equals_the_fused_call(gs):
+    """gs_pipeline_host copies worker groups while earlier groups compute and
+    continues the sum across groups: its outputs equal one gs_sparsify_aggregate
+    call's bit for bit (bf16 input, more workers than groups, a ragged d)."""
+    import torch
+    M, d, kappa, iters, seed, step = 19, 70_001, 0.03, 3, 4, 2
+    g_host = np.stack([_vector(k, d, 300 + m) for m, k in enumerate(["t3", "lognormal", "normal"] * 6 + ["ties"])])
+    g_host = workloads.bf16_bits_to_f32(workloads.f32_to_bf16_bits(g_host)).reshape(M, d)
+    bits = workloads.f32_to_bf16_bits(g_host).reshape(M, d)
+    g = _dev(bits).view(torch.bfloat16)
+    outs = []
+    for pipe in (False, True):
+        idx = torch.full((M, d), -1, dtype=torch.int32, device="cuda")
+        val = torch.zeros((M, d), dtype=torch.float32, device="cuda")
+        nnz = torch.zeros(M, dtype=torch.int32, device="cuda")
+        out = torch.full((d,), float("nan"), dtype=torch.float32, device="cuda")
+        if pipe:
+            gh = torch.from_numpy(bits).view(torch.bfloat16).pin_memory()
+            g_dev = torch.empty_like(g)
+            out_h = torch.empty(d, dtype=torch.float32).pin_memory()
+            nnz_h = torch.empty(M, dtype=torch.int32).pin_memory()
+            gs.gs_pipeline_host(gh, kappa, iters, seed, step, 0, g_dev, idx, val, nnz, out, out_h, nnz_h)
+            torch.cuda.synchronize()
+            assert torch.equal(out_h, out.cpu()) and torch.equal(nnz_h, nnz.cpu())
+        else:
+            gs.gs_sparsify_aggregate(g, kappa, iters, seed, step, 0, idx, val, nnz, out)
+        assert gs.gs_sync_status() == gs.GS_OK
+        outs.append((idx, val, nnz, out))
+    (i0, v0, n0, o0), (i1, v1, n1, o1) = outs
+    assert torch.equal(n0, n1) and torch.equal(o0, o1)
+    for m in range(M):
+        k = int(n0[m].item())
+        assert torch.equal(i0[m, :k], i1[m, :k]) and torch.equal(v0[m, :k], v1[m, :k])
+
+
 # ---------------------------------------------------------------------------
 # Full-size workloads in the launch configuration bench.py times.
 # ---------------------------------------------------------------------------
