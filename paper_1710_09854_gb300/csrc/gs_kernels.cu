@@ -600,6 +600,26 @@ __device__ __forceinline__ double warp0_sum_double(double v, double* sh) {
 // solve's single busy warp has to fetch.
 __device__ __noinline__ float cap_threshold_call(double lam) { return cap_threshold(lam); }
 
+// cap_threshold by a whole warp (all 32 lanes, same lam; every lane gets the
+// result): the 32 floats around the fp32 reciprocal of lam are tested side by
+// side, one fp64 product each.  fl64(lam a) >= 1 is monotone in a, so the
+// ballot is one run of ones from some lane up; when that lane is not lane 0
+// the smallest qualifying float lies in the window (the reciprocal is within
+// a few ulps of it), else the serial search decides.
+__device__ __forceinline__ float warp_cap_threshold(double lam) {
+    const int lane = threadIdx.x & 31;
+    const float f = (float)lam;
+    if (lam > 0.0 && f > 0.0f && f < 3.0e38f) {
+        const uint32_t b0 = __float_as_uint(__frcp_rn(f));
+        if (b0 > 16u && b0 < 0x7F7FFFFFu - 16u) {
+            const uint32_t b = b0 - 16u + (uint32_t)lane;
+            const uint32_t bal = __ballot_sync(0xFFFFFFFFu, lam * (double)__uint_as_float(b) >= 1.0);
+            if (bal != 0u && (bal & 1u) == 0u) return __uint_as_float(b0 - 16u + (uint32_t)(__ffs(bal) - 1));
+        }
+    }
+    return cap_threshold_call(lam);
+}
+
 // Exact fallback of k_solve for one segment, by the whole CTA: every sum of
 // Algorithm 3 straight from g, then the segment's P lists rebuilt for the
 // final lambda (sparsify calls only).  Out of line: it almost never runs, and
@@ -839,9 +859,10 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
         double lv = 0.0;
         int jj = 0;
         bool ex = force_exact != 0;
+        float acap = __int_as_float(0x7F800000);
         if (isfinite(S0) && !ex && S0 > 0.0) {
             lv = budget / S0;
-            float acap = cap_threshold_call(lv);
+            acap = warp_cap_threshold(lv);
             bool fresh = false;   // (rh, rl, rk) are the stats at acap
             while (jj < iters) {
                 warp_c_stats(C, acap, rh, rl, rk);
@@ -852,7 +873,7 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
                 if (!(cc > 1.0)) break;
                 lv = cc * lv;
                 ++jj;
-                acap = cap_threshold_call(lv);
+                acap = warp_cap_threshold(lv);
                 fresh = false;
             }
             if (!fresh) warp_c_stats(C, acap, rh, rl, rk);
@@ -862,6 +883,7 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
         if (tid == 0) {
             s_S = S0;
             s_lam = lv;
+            s_acap = acap;   // the threshold of lv (reused for the segment's parameters)
             s_j = jj;
             s_go = ex ? 1 : 0;
             s_K = (double)rk;
@@ -882,12 +904,19 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
         flags |= kSegExact;
         solve_exact(Lo, Ls, m, lo, hi, c0, c1, budget, iters, shd, S, lam, K, Su, j);
     }
+    // The solve's own threshold holds for its final lambda, except after the
+    // exact fallback (or a non-finite sum, where lambda is 0).
+    float a_cap = s_acap;
+    if ((flags & kSegExact) || !isfinite(S) || !(lam > 0.0)) {
+        if (tid < 32) a_cap = warp_cap_threshold(lam);
+        else a_cap = 0.0f;   // unused
+    }
 
     if (tid == 0) {
         SegParam& P = sp[s];
         P.lam = lam;
         P.lam32 = (float)lam;
-        P.a_cap = cap_threshold_call(lam);
+        P.a_cap = a_cap;
         P.inv_lam32 = lam > 0.0 ? (float)(1.0 / lam) : 0.0f;
         P.l1 = S;
         P.capped = (long long)K;
