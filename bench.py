@@ -279,6 +279,10 @@ def run_gpu(args):
     kernel_bytes = {
         "k_stream": M * d * esz,                 # one read of g
         "k_stream_tma": M * d * esz,             # one read of g
+        # the cluster path: one read of g, the codes written (and, for one
+        # worker, the dense sum it writes itself)
+        "k_small": M * d * esz + nnz_total * 8 + (d * 4 if M == 1 else 0),
+        "k_small_sum": M * d // 8 + nnz_total * esz + d * 4,   # decision bits, kept g, dense sum
         "k_emit": nnz_total * 8,                 # the (idx, val) codes written
         "k_sum": nnz_total * 8 + d * 4,          # codes read, dense sum written
         "k_tiles": nnz_total * 8 + d * 4,        # codes read, dense sum written
@@ -430,11 +434,13 @@ def run_configs(gs, args, dev, stream, hbm, rank):
             gs.gs_set_option(gs.GS_OPT_KERNEL_TIMING, 0)
             if gs.gs_sync_status(stream) != gs.GS_OK:
                 raise RuntimeError("device status after timing")
-            sk = "k_stream_tma" if kt.get("k_stream_tma", (0, 0))[1] else "k_stream"
+            # The streaming pass, or the cluster-resident kernel on short rows.
+            sk = next((k for k in ("k_stream_tma", "k_stream", "k_small") if kt.get(k, (0, 0))[1]), "k_stream")
             s_ms = kt[sk][0] / max(kt[sk][1], 1)
             b_sp, b_ag = algorithmic_bytes(M, d, esz, kept)
             step_gbs = (b_sp + b_ag) / (ms / 1e3) / 1e9
-            s_gbs = M * d * esz / (s_ms / 1e3) / 1e9
+            s_bytes = M * d * esz + (kept * 8 + (d * 4 if M == 1 else 0) if sk == "k_small" else 0)
+            s_gbs = s_bytes / (s_ms / 1e3) / 1e9
             rows.append({"workload": w.name, "M": M, "d": d, "kappa": kappa, "dtype": dtype, "iters": w.iters,
                          "api": "gs_segmented_sparsify_aggregate" if off is not None else "gs_sparsify_aggregate",
                          "steps": n, "ms_per_step": round(ms, 5), "coords_per_s": M * d / (ms / 1e3),

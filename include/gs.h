@@ -391,7 +391,8 @@ gs_status gs_random_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t
  *                              on lambda (default 16384; a multiple of 8 in
  *                              256 .. 32768).
  *   GS_OPT_KERNEL_TIMING      1: time every kernel launch (gs_kernel_times);
- *                              2: time the streaming pass only.  The events
+ *                              2: time the streaming pass only (k_small on
+ *                              the cluster path).  The events
  *                              sit between launches, so a timed kernel does
  *                              not overlap its neighbours' launch (mode 2
  *                              leaves the rest of the chain overlapped).
@@ -399,13 +400,25 @@ gs_status gs_random_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t
  *                              kernel whenever the layout allows it), 1 the
  *                              generic-load kernel, 2 the TMA kernel where
  *                              eligible.
+ *   GS_OPT_SMALL_PATH         rows of d <= 2^21 coordinates: 0 automatic
+ *                              (one thread-block cluster per worker when
+ *                              also M d <= 2^24, else the chunked kernels),
+ *                              1 always the chunked kernels, 2 always the
+ *                              cluster path.  Calls with a forced exact
+ *                              solve, probabilities, the hybrid code,
+ *                              Algorithm 2 or layer-wise segments always
+ *                              take the chunked kernels.  Each path is
+ *                              deterministic; the two agree with the oracle
+ *                              to the stated tolerances, not bit for bit
+ *                              (their sums of |g| round in different orders).
  * Options are process-wide; returns GS_ERR_INVALID_ARG for an unknown
  * option or value. */
 typedef enum {
     GS_OPT_FORCE_EXACT_SOLVE = 1,
     GS_OPT_SAMPLE_SIZE = 2,
     GS_OPT_KERNEL_TIMING = 3,
-    GS_OPT_STREAM_PATH = 4
+    GS_OPT_STREAM_PATH = 4,
+    GS_OPT_SMALL_PATH = 5
 } gs_option;
 gs_status gs_set_option(int option, int64_t value);
 

@@ -20,7 +20,7 @@ LIB_PATH = os.path.join(_HERE, "libgs.so")
 (GS_OK, GS_ERR_INVALID_ARG, GS_ERR_CUDA, GS_ERR_CAPACITY, GS_ERR_NONFINITE, GS_ERR_TIMEOUT, GS_ERR_INTERNAL,
  GS_ERR_ABORTED) = range(8)
 GS_DTYPE_F32, GS_DTYPE_BF16 = 0, 1
-GS_OPT_FORCE_EXACT_SOLVE, GS_OPT_SAMPLE_SIZE, GS_OPT_KERNEL_TIMING, GS_OPT_STREAM_PATH = 1, 2, 3, 4
+GS_OPT_FORCE_EXACT_SOLVE, GS_OPT_SAMPLE_SIZE, GS_OPT_KERNEL_TIMING, GS_OPT_STREAM_PATH, GS_OPT_SMALL_PATH = 1, 2, 3, 4, 5
 
 # Symbols include/gs.h declares (checked by the tests).
 EXPORTS = ("gs_status_string", "gs_last_error", "gs_version", "gs_sync_status", "gs_probabilities", "gs_probabilities_ex",

@@ -17,7 +17,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(ROOT, "_build")
 LIB = os.path.join(PKG, "libgs.so")
-SOURCES = ["gs_kernels.cu", "gs_stream_tma.cu", "gs_eps.cu", "gs_lr.cu", "gs_dense.cu", "gs_api.cu", "gs_trace.cu"]
+SOURCES = ["gs_kernels.cu", "gs_stream_tma.cu", "gs_eps.cu", "gs_lr.cu", "gs_dense.cu", "gs_small.cu", "gs_api.cu", "gs_trace.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

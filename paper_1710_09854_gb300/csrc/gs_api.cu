@@ -62,6 +62,22 @@ gs_status cuda_fail(const char* where, cudaError_t e) {
 int g_force_exact = 0;
 int g_sample = 16384;
 int g_stream_path = 0;  // 0 auto, 1 generic loads, 2 TMA (when eligible)
+int g_small_path = 0;   // 0 auto, 1 never, 2 whenever the row is short enough
+
+// Rows of at most kSmallMaxD coordinates take the cluster-resident path
+// (gs_small.cu) when the whole call is small too (M d <= 2^24): there one
+// cluster per worker beats the chunked path's six launches over a few
+// busy warps.  Larger calls fill the GPU through the chunked path, whose
+// single read of g wins once the cluster path's extra passes do not fit in L2.
+bool choose_small(int M, int64_t d) {
+    int opt;
+    {
+        std::lock_guard<std::mutex> lk(g_mu);
+        opt = g_small_path;
+    }
+    if (opt == 1 || !small_path_eligible(d)) return false;
+    return opt == 2 || (int64_t)M * d <= ((int64_t)1 << 24);
+}
 
 gs_status device_state(DevState** out) {
     int dev = 0;
@@ -170,7 +186,7 @@ void carve(Arena& a, Workspace& w, int n_seg, int n_chunks, int64_t n, bool buil
 gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off, int L, double kappa, int iters,
               uint64_t seed, uint32_t step, uint32_t worker0, int32_t* idx, float* val, int32_t* nnz, int64_t cap,
               gs_info* info, float* p, cudaStream_t st, float* agg_out = nullptr, const HybridOut* hy = nullptr,
-              double eps = -1.0, bool average = false, bool accumulate = false) {
+              double eps = -1.0, bool average = false, bool accumulate = false, int path_hint = -1) {
     const bool prob = p != nullptr;
     const bool alg2 = eps >= 0.0;
     if (!g || M < 1 || d < 1 || d >= kMaxD) return GS_ERR_INVALID_ARG;
@@ -209,6 +225,28 @@ gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off
     for (int r = 0; r < 10; ++r) {
         Lo.rk0[r] = (uint32_t)(seed & 0xFFFFFFFFu) + (uint32_t)r * 0x9E3779B9u;
         Lo.rk1[r] = (uint32_t)(seed >> 32) + (uint32_t)r * 0xBB67AE85u;
+    }
+    int force_opt;
+    {
+        std::lock_guard<std::mutex> lk(g_mu);
+        force_opt = g_force_exact;
+    }
+    // Short rows: the cluster-resident path (always exact, so a forced exact
+    // solve, which exercises the chunked path's fallback, keeps the chunked path).
+    const bool small_ok = !prob && !hy && !alg2 && L == 1 && force_opt == 0 && small_path_eligible(d);
+    if (small_ok && (path_hint == 1 || (path_hint < 0 && choose_small(M, d)))) {
+        const bool sum_kernel = agg_out != nullptr && M > 1;
+        void* mem = nullptr;
+        if (sum_kernel) {
+            const cudaError_t ea = cudaMallocFromPoolAsync(&mem, small_scratch_bytes(M, d), s->pool, st);
+            if (ea != cudaSuccess) return cuda_fail("cudaMallocFromPoolAsync", ea);
+        }
+        const cudaError_t e = launch_small(Lo, kappa, iters, idx, val, nnz, cap, s->status, info, agg_out, average,
+                                           accumulate, mem, st);
+        const cudaError_t ef = mem ? cudaFreeAsync(mem, st) : cudaSuccess;
+        if (e != cudaSuccess) return cuda_fail(launch_error_site(), e);
+        if (ef != cudaSuccess) return cuda_fail("cudaFreeAsync", ef);
+        return GS_OK;
     }
     if (L == 1) {
         const int64_t cpw = (d + chunk_size() - 1) / chunk_size();
@@ -425,15 +463,21 @@ gs_status run_noalloc(const float* g, int64_t d, double kappa, int iters, uint64
     // Every scratch word a kernel reads was written earlier in the same call;
     // the status word is the one thing left from the previous call.
     GS_TRY(cudaMemsetAsync(s->status, 0, sizeof(int), st));
-    const bool tma_ok = path != 1 && stream_tma_eligible(Lo);
-    cudaError_t e = launch_bound(Lo, w.sp, 1, kappa, ns, force, st);
-    if (e == cudaSuccess) {
-        bool used = false;
-        if (tma_ok) e = launch_stream_tma(Lo, w.sp, w.ls, n_chunks, s->status, st, &used);
-        if (e == cudaSuccess && !used) e = launch_stream(Lo, w.sp, w.ls, n_chunks, true, st);
+    cudaError_t e = cudaSuccess;
+    if (force == 0 && small_path_eligible(d) && choose_small(1, d)) {
+        // The path gs_sparsify takes for this d (it needs no scratch at all).
+        e = launch_small(Lo, kappa, iters, idx, val, nnz, d, s->status, info, nullptr, false, false, nullptr, st);
+    } else {
+        const bool tma_ok = path != 1 && stream_tma_eligible(Lo);
+        e = launch_bound(Lo, w.sp, 1, kappa, ns, force, st);
+        if (e == cudaSuccess) {
+            bool used = false;
+            if (tma_ok) e = launch_stream_tma(Lo, w.sp, w.ls, n_chunks, s->status, st, &used);
+            if (e == cudaSuccess && !used) e = launch_stream(Lo, w.sp, w.ls, n_chunks, true, st);
+        }
+        if (e == cudaSuccess) e = launch_solve(Lo, w.sp, w.ls, 1, kappa, iters, force, s->status, info, st, d);
+        if (e == cudaSuccess) e = launch_compact(Lo, w.sp, w.ls, n_chunks, idx, val, nnz, d, s->status, st);
     }
-    if (e == cudaSuccess) e = launch_solve(Lo, w.sp, w.ls, 1, kappa, iters, force, s->status, info, st, d);
-    if (e == cudaSuccess) e = launch_compact(Lo, w.sp, w.ls, n_chunks, idx, val, nnz, d, s->status, st);
     if (e == cudaSuccess) {
         k_noalloc_status<<<1, 1, 0, st>>>(s->status, status);
         e = cudaGetLastError();
@@ -700,6 +744,8 @@ gs_status gs_pipeline_host(const void* g_host, int dtype, int M, int64_t d, doub
     // sparsify + sum on `stream`; the sum continues across groups in worker
     // order, so out is what one call over all M workers would give.
     const int G = std::min(M, kPipeGroups);
+    // One path for every group, the one a single call over all M workers takes.
+    const int hint = choose_small(M, d) ? 1 : 0;
     GS_TRY(cudaEventRecord(s->ev_start, st));
     for (int i = 0; i < 2; ++i) GS_TRY(cudaStreamWaitEvent(s->copy[i], s->ev_start, 0));
     int m0 = 0;
@@ -718,7 +764,7 @@ gs_status gs_pipeline_host(const void* g_host, int dtype, int M, int64_t d, doub
         GS_TRY(cudaStreamWaitEvent(st, s->ev_group[k], 0));
         rc = run(static_cast<const char*>(g_dev) + esz * (size_t)m0 * (size_t)d, dtype, m1 - m0, d, nullptr, 1,
                  kappa, iters, seed, step, worker0 + (uint32_t)m0, idx + (int64_t)m0 * cap, val + (int64_t)m0 * cap,
-                 nnz + m0, cap, nullptr, nullptr, st, out, nullptr, -1.0, false, k > 0);
+                 nnz + m0, cap, nullptr, nullptr, st, out, nullptr, -1.0, false, k > 0, hint);
         if (rc != GS_OK) return rc;
         m0 = m1;
     }
@@ -758,6 +804,10 @@ gs_status gs_set_option(int option, int64_t value) {
         case GS_OPT_STREAM_PATH:
             if (value < 0 || value > 2) return GS_ERR_INVALID_ARG;
             g_stream_path = (int)value;
+            return GS_OK;
+        case GS_OPT_SMALL_PATH:
+            if (value < 0 || value > 2) return GS_ERR_INVALID_ARG;
+            g_small_path = (int)value;
             return GS_OK;
         case GS_OPT_KERNEL_TIMING:
             if (value < 0 || value > 2) return GS_ERR_INVALID_ARG;

@@ -132,6 +132,17 @@ cudaError_t launch_dense_encode(const int32_t* qa, const uint32_t* qb, const int
                                 int64_t* n_words, void* ws, int64_t max_chunks, int* status, cudaStream_t st);
 cudaError_t launch_dense_decode(const uint16_t* words, const int64_t* n_words, int M, int64_t d, int64_t word_cap,
                                 int8_t* qt, void* ws, int64_t max_chunks, int* status, cudaStream_t st);
+// The cluster-resident path for rows of d <= kSmallMaxD coordinates
+// (gs_small.cu): Algorithm 3, the draw and the compaction of each worker in
+// one cluster launch, plus a worker-order sum kernel when out is given and
+// M > 1 (scratch: small_scratch_bytes(M, d) bytes of device memory, else
+// unused).  With M == 1 the cluster writes out itself.
+constexpr int64_t kSmallMaxD = (int64_t)1 << 21;
+bool small_path_eligible(int64_t d);
+size_t small_scratch_bytes(int M, int64_t d);
+cudaError_t launch_small(const Layout& Lo, double kappa, int iters, int32_t* idx, float* val, int32_t* nnz,
+                         int64_t cap, int* status, gs_info_dev* info, float* out, bool average, bool accumulate,
+                         void* scratch, cudaStream_t st);
 // The launchers record which step failed; the C ABI reports it.
 void set_launch_error_site(const char* where);
 const char* launch_error_site();

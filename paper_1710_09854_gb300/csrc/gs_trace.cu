@@ -18,7 +18,7 @@ const char* kNames[kNumKernels] = {"k_bound", "k_stream", "k_solve", "k_emit",
                                    "k_eps_hist", "k_eps_bracket", "k_solve_eps",
                                    "k_lr_grad", "k_lr_margins", "k_row_sq", "k_sum_rows", "k_sgd_step",
                                    "k_dense_count", "k_dense_merge", "k_dense_setup", "k_dense_encode", "k_dense_scan",
-                                   "k_dense_decode"};
+                                   "k_dense_decode", "k_small", "k_small_sum"};
 
 struct Pending {
     int k;
@@ -55,8 +55,9 @@ const char* launch_error_site() { return g_site; }
 
 TraceScope::TraceScope(int k, cudaStream_t st) : k_(k), st_(st), a_(nullptr) {
     launches[k].fetch_add(1);
-    const int mode = timing_on.load();   // 1: every kernel; 2: the streaming pass only
-    if (mode == 1 || (mode == 2 && (k == kKStream || k == kKStreamTma))) {
+    // 1: every kernel; 2: the streaming pass only (on the cluster path, its one kernel)
+    const int mode = timing_on.load();
+    if (mode == 1 || (mode == 2 && (k == kKStream || k == kKStreamTma || k == kKSmall))) {
         std::lock_guard<std::mutex> lk(mu);
         a_ = take_event();
         if (a_) cudaEventRecord(a_, st_);

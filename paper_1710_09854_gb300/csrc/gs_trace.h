@@ -32,6 +32,8 @@ enum KernelId : int {
     kKDenseEncode,
     kKDenseScan,
     kKDenseDecode,
+    kKSmall,
+    kKSmallSum,
     kNumKernels
 };
 

@@ -26,6 +26,24 @@ def gs():
     return gs
 
 
+@pytest.fixture(autouse=True)
+def _path(gs, request):
+    """Short rows take the chunked kernels here unless a test asks for the
+    cluster-resident path (its `small` parameter); the full-size workloads
+    take the path the library picks, as bench.py times them."""
+    gs.gs_set_option(gs.GS_OPT_SMALL_PATH, 0 if request.node.name.startswith("test_full") else 1)
+    yield
+    gs.gs_set_option(gs.GS_OPT_SMALL_PATH, 0)
+
+
+# 1: the chunked kernels; 2: one thread-block cluster per worker (rows of d <= 2^21).
+BOTH_PATHS = pytest.mark.parametrize("small", [1, 2], ids=["chunked", "cluster"])
+
+
+def _use(gs, small):
+    gs.gs_set_option(gs.GS_OPT_SMALL_PATH, small)
+
+
 def _dev(x):
     import torch
     return torch.from_numpy(np.ascontiguousarray(x)).cuda()
@@ -92,7 +110,9 @@ def test_probabilities_sizes(gs, d):
 
 
 @pytest.mark.parametrize("d", SIZES)
-def test_sparsify_sizes(gs, d):
+@BOTH_PATHS
+def test_sparsify_sizes(gs, d, small):
+    _use(gs, small)
     import torch
     for kind, kappa, iters, seed, step, worker in [("t3", 0.01, 3, 1, 0, 0), ("lognormal", 0.1, 2, 99, 5, 3),
                                                    ("normal", 0.3, 1, 2**35 + 1, 2**31, 2**32 - 2),
@@ -109,7 +129,9 @@ def test_sparsify_sizes(gs, d):
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
-def test_batched_parity(gs, dtype):
+@BOTH_PATHS
+def test_batched_parity(gs, dtype, small):
+    _use(gs, small)
     M, d, kappa, iters, seed, step, w0 = 5, 100_003, 0.02, 3, 11, 7, 3
     g_host = np.stack([_vector(k, d, 50 + m) for m, k in enumerate(["t3", "lognormal", "normal", "t3", "ties"])])
     if dtype == "bf16":
@@ -128,7 +150,9 @@ def test_batched_parity(gs, dtype):
     assert flips <= 1
 
 
-def test_single_equals_batched_row(gs):
+@BOTH_PATHS
+def test_single_equals_batched_row(gs, small):
+    _use(gs, small)
     import torch
     M, d = 3, 70_001
     g_host = np.stack([_vector("lognormal", d, 900 + m) for m in range(M)])
@@ -143,7 +167,9 @@ def test_single_equals_batched_row(gs):
         assert torch.equal(i1[:k], idx[m, :k]) and torch.equal(v1[:k], val[m, :k])
 
 
-def test_deterministic(gs):
+@BOTH_PATHS
+def test_deterministic(gs, small):
+    _use(gs, small)
     import torch
     M, d = 4, 300_001
     g_host = np.stack([_vector("t3", d, 77 + m) for m in range(M)])
@@ -246,7 +272,9 @@ def test_aggregate_parity_and_validation(gs):
         assert gs.gs_sync_status() == gs.GS_ERR_INVALID_ARG
 
 
-def test_edge_cases(gs):
+@BOTH_PATHS
+def test_edge_cases(gs, small):
+    _use(gs, small)
     import torch
     d = 40_000
     # all zero: nothing kept
@@ -288,7 +316,9 @@ def test_edge_cases(gs):
     np.testing.assert_array_equal(idx[0].cpu().numpy(), ri[:100])
 
 
-def test_pipeline_host_matches_device_path(gs):
+@BOTH_PATHS
+def test_pipeline_host_matches_device_path(gs, small):
+    _use(gs, small)
     import torch
     M, d, kappa, iters, seed, step = 4, 65_537, 0.05, 2, 3, 1
     g_host = np.stack([_vector("t3", d, 10 + m) for m in range(M)])
@@ -312,10 +342,12 @@ def test_pipeline_host_matches_device_path(gs):
     compare_sum(out_h.numpy(), il, vl, d)
 
 
-def test_pipeline_host_equals_the_fused_call(gs):
+@BOTH_PATHS
+def test_pipeline_host_equals_the_fused_call(gs, small):
     """gs_pipeline_host copies worker groups while earlier groups compute and
     continues the sum across groups: its outputs equal one gs_sparsify_aggregate
     call's bit for bit (bf16 input, more workers than groups, a ragged d)."""
+    _use(gs, small)
     import torch
     M, d, kappa, iters, seed, step = 19, 70_001, 0.03, 3, 4, 2
     g_host = np.stack([_vector(k, d, 300 + m) for m, k in enumerate(["t3", "lognormal", "normal"] * 6 + ["ties"])])
@@ -511,9 +543,11 @@ def test_stream_paths(gs, path, dtype):
 
 
 @pytest.mark.parametrize("dtype", ["f32", "bf16"])
-def test_sparsify_aggregate_fused(gs, dtype):
+@BOTH_PATHS
+def test_sparsify_aggregate_fused(gs, dtype, small):
     """gs_sparsify_aggregate equals gs_batched_sparsify + gs_sparse_aggregate
     bit for bit, and the oracle's worker-order sum."""
+    _use(gs, small)
     import torch
     M, d, kappa, iters, seed, step = 6, 3 * 16384 + 1000, 0.03, 3, 21, 2
     g_host = np.stack([_vector(k, d, 400 + m) for m, k in enumerate(["t3", "lognormal", "normal"] * 2)])
@@ -551,9 +585,11 @@ def test_sparsify_aggregate_fused(gs, dtype):
             np.testing.assert_array_equal(out.cpu().numpy(), oracle.aggregate(il, vl, d))
 
 
-def test_sparsify_aggregate_fused_long_runs_many_workers(gs):
+@BOTH_PATHS
+def test_sparsify_aggregate_fused_long_runs_many_workers(gs, small):
     """The fused sum with more than 32 workers (several worker batches per
     slice) and kappa large enough that runs exceed 32 entries per slice."""
+    _use(gs, small)
     import torch
     M, d, kappa, iters, seed, step = 40, 2 * 16384 + 777, 0.2, 2, 5, 9
     kinds = ["t3", "lognormal", "normal", "ties"]
@@ -648,10 +684,12 @@ def test_hybrid_code(gs, dtype, kind, kappa, d):
         compare_sparse(di, dv, g_host[m], kappa, iters, seed, step, m)
 
 
-def test_outputs_stay_inside_their_buffers(gs):
+@BOTH_PATHS
+def test_outputs_stay_inside_their_buffers(gs, small):
     """Guard bands: every output sits inside a larger sentinel-filled buffer;
     after each call the band past the buffer and, within each row, the slots
     past the written count still hold the sentinel."""
+    _use(gs, small)
     import torch
     G = 4096
     SI, SV = -123456789, -7.5e33
