@@ -46,7 +46,8 @@ constexpr int kTile = 128;               // coordinates per warp step (4 consecu
 constexpr int kBatch = 4;                // tiles whose loads a warp has in flight together
 constexpr int kMaxCtas = 16;             // cluster size limit (non-portable above 8)
 // Cluster size the automatic shape stops at: eight 12-CTA clusters of 1024
-// threads are resident together on a GB300, while only seven of 16 are.
+// threads are resident together on a GB300, while only seven of 13, 14 or
+// 16 are (a ninth worker's cluster would wait for a second wave).
 constexpr int kAutoCtas = 12;
 constexpr int kMaxThreads = 1024;
 constexpr int kCacheFloats = 40960;      // shares up to 160 KiB stay in shared memory
@@ -606,23 +607,30 @@ __global__ void __launch_bounds__(kSumThreads) k_small_sum(const __grid_constant
         for (int s = 0; s < 4; ++s) acc[s] = accumulate && i0 + s < d ? out[i0 + s] : 0.0f;
         const int sh = (int)(i0 & 31);
         for (int m0 = 0; m0 < Lo.M; m0 += kSumGroup) {
-            // The group's decision words first (independent loads), then the
-            // kept values in worker order.
-            uint32_t nib[kSumGroup];
-#pragma unroll
-            for (int u = 0; u < kSumGroup; ++u)
-                nib[u] = m0 + u < Lo.M ? (__ldg(bits + (size_t)(m0 + u) * wpr + (i0 >> 5)) >> sh) & 0xFu : 0u;
+            // The group's words of all three planes first (independent
+            // loads), then the kept values in worker order.
+            uint32_t kw[kSumGroup], sw[kSumGroup], cw[kSumGroup];
 #pragma unroll
             for (int u = 0; u < kSumGroup; ++u) {
-                if (nib[u] == 0u) continue;
+                kw[u] = sw[u] = cw[u] = 0u;
+                if (m0 + u < Lo.M) {
+                    const size_t wi = (size_t)(m0 + u) * wpr + (i0 >> 5);
+                    kw[u] = __ldg(bits + wi);
+                    sw[u] = __ldg(bits + (size_t)Lo.M * wpr + wi);
+                    cw[u] = __ldg(bits + (size_t)2 * Lo.M * wpr + wi);
+                }
+            }
+#pragma unroll
+            for (int u = 0; u < kSumGroup; ++u) {
+                const uint32_t nib = (kw[u] >> sh) & 0xFu;
+                if (nib == 0u) continue;
                 const int m = m0 + u;
-                const uint32_t sn = (__ldg(bits + ((size_t)Lo.M + m) * wpr + (i0 >> 5)) >> sh) & 0xFu;
-                const uint32_t cn = (__ldg(bits + ((size_t)2 * Lo.M + m) * wpr + (i0 >> 5)) >> sh) & 0xFu;
                 const float inv = m < kSumStage ? s_inv[m] : sp[m].inv_lam32;
 #pragma unroll
                 for (int s = 0; s < 4; ++s) {
-                    if ((nib[u] >> s) & 1u)
-                        acc[s] += (cn >> s) & 1u ? load_one(Lo, m, i0 + s) : ((sn >> s) & 1u ? -inv : inv);
+                    if ((nib >> s) & 1u)
+                        acc[s] += (cw[u] >> (sh + s)) & 1u ? load_one(Lo, m, i0 + s)
+                                                          : ((sw[u] >> (sh + s)) & 1u ? -inv : inv);
                 }
             }
         }
