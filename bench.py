@@ -501,9 +501,39 @@ def run_e2e(gs, g, kappa, w, args, dev, stream, ws):
     if rc != gs.GS_OK:
         raise RuntimeError(f"device status after e2e: {gs.status_string(rc)}")
     h2d = M * d * g.element_size()
+    # The same host-to-device copies alone (worker groups alternating between
+    # two streams, as the pipelined call issues them): the floor the
+    # pipelined step is measured against.
+    cs = (torch.cuda.Stream(device=dev), torch.cuda.Stream(device=dev))
+    G = min(M, 8)
+
+    def copies():
+        ev = torch.cuda.Event()
+        ev.record(stream)
+        m0 = 0
+        for k in range(G):
+            m1 = M * (k + 1) // G
+            c = cs[k & 1]
+            c.wait_event(ev)
+            with torch.cuda.stream(c):
+                g_dev[m0:m1].copy_(gh[m0:m1], non_blocking=True)
+            m0 = m1
+        stream.wait_stream(cs[0])
+        stream.wait_stream(cs[1])
+
+    copies()
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for t in range(n):
+        copies()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    copy_ms = max_over_ranks(e0.elapsed_time(e1) / n, dev)
     return {"value": job_throughput(M * d, ms, ws), "unit": UNIT, "ms_per_step": ms,
             "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d * 4 + M * 4,
             "h2d_gbs_over_step": round(h2d / (ms / 1e3) / 1e9, 1),
+            "copy_only_ms": round(copy_ms, 4), "copy_only_h2d_gbs": round(h2d / (copy_ms / 1e3) / 1e9, 1),
+            "step_over_copy": round(ms / copy_ms, 3),
             "api": "gs_pipeline_host (worker groups copied on two streams while earlier groups compute)",
             "host_memory": "pinned"}
 

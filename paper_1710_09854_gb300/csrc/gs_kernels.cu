@@ -922,6 +922,9 @@ constexpr int kEmitWarps = 8;
 constexpr int kEmitBatch = 4;                            // candidate rounds whose loads are in flight together
 constexpr int kBitWords = kChunk / 32;                   // decision words per chunk
 constexpr int kScanPer = 8;                              // chunk counts per lane per step of the worker scan
+// Resident CTAs per SM k_decide is compiled for (<= 42 registers a thread):
+// its warps mostly wait on candidate loads, so more of them hide more.
+constexpr int kDecideBlocks = 6;
 
 // One warp turns n counts into their exclusive prefix in place (kScanPer
 // counts per lane per step, read past L1) and returns the total.
@@ -963,7 +966,7 @@ __device__ __forceinline__ Decider chunk_decider(const SegParam& P) {
     return dd;
 }
 
-__global__ void __launch_bounds__(kEmitWarps * 32) k_decide(const __grid_constant__ Layout Lo, SegParam* sp,
+__global__ void __launch_bounds__(kEmitWarps * 32, kDecideBlocks) k_decide(const __grid_constant__ Layout Lo, SegParam* sp,
                                                             const __grid_constant__ Lists Ls, int n_chunks,
                                                             int32_t* nnz, int32_t* n_a, int32_t* n_b, int64_t cap,
                                                             int* status) {
