@@ -364,8 +364,9 @@ gs_status gs_sparsify_noalloc(const float* g, int64_t d, double kappa, int iters
  * library-owned copy streams, each group sparsified on `stream` as soon as it
  * has landed while the next ones copy; the sum continues across the groups in
  * worker order, so every output equals gs_sparsify_aggregate's bit for bit.
- * Calls on one device are serialised on the host (they share the ordering
- * events).  g_dev / idx / val / nnz / out are caller-owned device
+ * The read-back is split in two halves, one per copy stream, and `stream`
+ * waits for both.  Calls on one device are serialised on the host (they
+ * share the ordering events).  g_dev / idx / val / nnz / out are caller-owned device
  * buffers of the sizes gs_batched_sparsify / gs_sparse_aggregate require
  * (idx, val: M x cap).  Host buffers should be pinned for full copy speed.
  * Returns after enqueueing; the host buffers are valid once `stream` has

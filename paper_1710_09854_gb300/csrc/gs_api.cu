@@ -40,6 +40,8 @@ struct DevState {
     bool pipe_ready = false;
     cudaStream_t copy[2] = {nullptr, nullptr};
     cudaEvent_t ev_start = nullptr;
+    cudaEvent_t ev_done = nullptr;       // the last group's sum is written
+    cudaEvent_t ev_back[2] = {};         // each half of the read-back has landed
     cudaEvent_t ev_group[kPipeGroups] = {};
     std::mutex pipe_mu;     // one pipeline call at a time per device (they share the events)
 };
@@ -734,6 +736,8 @@ gs_status gs_pipeline_host(const void* g_host, int dtype, int M, int64_t d, doub
     if (!s->pipe_ready) {
         for (int i = 0; i < 2; ++i) GS_TRY(cudaStreamCreateWithFlags(&s->copy[i], cudaStreamNonBlocking));
         GS_TRY(cudaEventCreateWithFlags(&s->ev_start, cudaEventDisableTiming));
+        GS_TRY(cudaEventCreateWithFlags(&s->ev_done, cudaEventDisableTiming));
+        for (int i = 0; i < 2; ++i) GS_TRY(cudaEventCreateWithFlags(&s->ev_back[i], cudaEventDisableTiming));
         for (int k = 0; k < kPipeGroups; ++k) GS_TRY(cudaEventCreateWithFlags(&s->ev_group[k], cudaEventDisableTiming));
         s->pipe_ready = true;
     }
@@ -768,8 +772,22 @@ gs_status gs_pipeline_host(const void* g_host, int dtype, int M, int64_t d, doub
         if (rc != GS_OK) return rc;
         m0 = m1;
     }
-    GS_TRY(cudaMemcpyAsync(out_host, out, sizeof(float) * (size_t)d, cudaMemcpyDeviceToHost, st));
-    GS_TRY(cudaMemcpyAsync(nnz_host, nnz, sizeof(int32_t) * (size_t)M, cudaMemcpyDeviceToHost, st));
+    // The sum and counts back to the host in two halves, one per copy stream
+    // (one stream reaches about half of the link); `stream` waits for both,
+    // so its completion still means out_host and nnz_host are written.
+    GS_TRY(cudaEventRecord(s->ev_done, st));
+    const size_t half = (size_t)d / 2;
+    for (int i = 0; i < 2; ++i) {
+        cudaStream_t cs = s->copy[i];
+        GS_TRY(cudaStreamWaitEvent(cs, s->ev_done, 0));
+        const size_t b = i == 0 ? 0 : half, e = i == 0 ? half : (size_t)d;
+        if (e > b)
+            GS_TRY(cudaMemcpyAsync(out_host + b, out + b, sizeof(float) * (e - b), cudaMemcpyDeviceToHost, cs));
+        if (i == 1)
+            GS_TRY(cudaMemcpyAsync(nnz_host, nnz, sizeof(int32_t) * (size_t)M, cudaMemcpyDeviceToHost, cs));
+        GS_TRY(cudaEventRecord(s->ev_back[i], cs));
+        GS_TRY(cudaStreamWaitEvent(st, s->ev_back[i], 0));
+    }
     return GS_OK;
 }
 
