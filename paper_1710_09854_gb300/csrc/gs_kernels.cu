@@ -64,9 +64,9 @@ __device__ __forceinline__ uint32_t mix32(uint32_t h) {
 // the offset of each sub-step's first entry of this thread relative to
 // `run`, and advances `run` by the block's total.  Order: sub-step, thread.
 // ---------------------------------------------------------------------------
-__device__ __forceinline__ void ordered_offsets(uint32_t packed, uint32_t (*sh)[kWarps], int& buf, int& run,
+__device__ __forceinline__ void ordered_offsets(uint32_t packed, uint32_t (*sh)[32], int& buf, int& run,
                                                 int off[kGroupsPerThread]) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
     uint32_t inc = packed;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -80,8 +80,7 @@ __device__ __forceinline__ void ordered_offsets(uint32_t packed, uint32_t (*sh)[
 #pragma unroll
     for (int j = 0; j < kGroupsPerThread; ++j) {
         int before = 0, cta = 0;
-#pragma unroll
-        for (int w = 0; w < kWarps; ++w) {
+        for (int w = 0; w < nw; ++w) {
             const int b = (int)((sh[buf][w] >> (8 * j)) & 0xFFu);
             cta += b;
             before += (w < warp) ? b : 0;
@@ -94,7 +93,7 @@ __device__ __forceinline__ void ordered_offsets(uint32_t packed, uint32_t (*sh)[
 }
 
 // ---------------------------------------------------------------------------
-// Candidate lists of one chunk, built by the whole CTA (kThreads threads).
+// Candidate lists of one chunk, built by the whole CTA (any multiple of 32 threads).
 //   P: 1 + (x >> 9) 2^-23 < fl32(lam_up32 |g| + 1 + 2^-20).  Since
 //      (x >> 9) 2^-23 <= u = x 2^-32, every coordinate kept under a lambda
 //      <= lam_up (u < min(lambda |g|, 1)) passes; the 2^-20 slack covers the
@@ -107,8 +106,8 @@ __device__ __forceinline__ void ordered_offsets(uint32_t packed, uint32_t (*sh)[
 template <bool kWithC>
 __device__ void chunk_candidates(const Layout& Lo, int c, const Chunk& ch, float lam_up32, float t_c, const Lists& Ls,
                                  bool build_p) {
-    __shared__ uint32_t shP[2][kWarps];
-    __shared__ uint32_t shC[2][kWarps];
+    __shared__ uint32_t shP[2][32];
+    __shared__ uint32_t shC[2][32];
     __shared__ double shd[33];
     const int tid = threadIdx.x;
     const int64_t q0 = ch.lo >> 2, q1 = (ch.hi + 3) >> 2;
@@ -119,14 +118,15 @@ __device__ void chunk_candidates(const Layout& Lo, int c, const Chunk& ch, float
     const bool sq = kWithC && Ls.b_low != nullptr;
     int runP = 0, runC = 0, bufP = 0, bufC = 0;
 
-    for (int64_t qb = q0; qb < q1; qb += (int64_t)kThreads * kGroupsPerThread) {
+    const int nthr = blockDim.x;
+    for (int64_t qb = q0; qb < q1; qb += (int64_t)nthr * kGroupsPerThread) {
         float v[kGroupsPerThread][4];
         uint4 w[kGroupsPerThread];
         uint32_t pm = 0, cm = 0;
         float s4[kGroupsPerThread], q4[kGroupsPerThread];
 #pragma unroll
         for (int j = 0; j < kGroupsPerThread; ++j) {
-            const int64_t q = qb + (int64_t)j * kThreads + tid;
+            const int64_t q = qb + (int64_t)j * nthr + tid;
             int valid = 0;
             if (q < q1) {
                 valid = load_group(Lo, ch.m, q, ch.lo, ch.hi, v[j]);
@@ -170,7 +170,7 @@ __device__ void chunk_candidates(const Layout& Lo, int c, const Chunk& ch, float
             for (int j = 0; j < kGroupsPerThread; ++j) {
                 uint32_t bits = (pm >> (4 * j)) & 0xFu;
                 int k = 0;
-                const int64_t q = qb + (int64_t)j * kThreads + tid;
+                const int64_t q = qb + (int64_t)j * nthr + tid;
                 while (bits) {
                     const int s = __ffs(bits) - 1;
                     bits &= bits - 1;
@@ -217,12 +217,13 @@ __device__ void segment_stats(const Layout& Lo, int m, int64_t lo, int64_t hi, f
                               double* shd) {
     const int64_t q0 = lo >> 2, q1 = (hi + 3) >> 2;
     double acc = 0.0, cnt = 0.0;
-    for (int64_t qb = q0; qb < q1; qb += (int64_t)kThreads * kGroupsPerThread) {
+    const int nthr = blockDim.x;
+    for (int64_t qb = q0; qb < q1; qb += (int64_t)nthr * kGroupsPerThread) {
         float s4[kGroupsPerThread];
         int k = 0;
 #pragma unroll
         for (int j = 0; j < kGroupsPerThread; ++j) {
-            const int64_t q = qb + (int64_t)j * kThreads + threadIdx.x;
+            const int64_t q = qb + (int64_t)j * nthr + threadIdx.x;
             float v[4] = {0.f, 0.f, 0.f, 0.f};
             int valid = 0;
             if (q < q1) valid = load_group(Lo, m, q, lo, hi, v);
@@ -521,7 +522,13 @@ __global__ void __launch_bounds__(kThreads) k_stream(Layout Lo, const SegParam* 
 constexpr int kSolveSmemChunks = 8192;   // chunk-prefix entries kept in shared memory
 constexpr int kSolveSmemC = 12288;       // candidate values kept in shared memory
 constexpr int kSolvePer = 4;             // chunks per thread of the one-round start (segments <= 1024 chunks)
-constexpr int kSolveCTAs = 16;           // cluster size of k_solve for long segments (non-portable size)
+// Long segments (budgets above 2^20) are solved by a cluster of kSolveCTAs
+// CTAs of kSolveClusterThreads threads: their walks over a C of millions of
+// values wait on L2, and 32 warps per SM hide that where 8 did not; twelve
+// 1024-thread CTAs is the largest cluster of which eight are resident at once.
+constexpr int kSolveCTAs = 12;
+constexpr int kSolveClusterThreads = 1024;
+constexpr int kSolveMaxThreads = 1024;   // k_solve runs on kThreads threads alone, or kSolveClusterThreads in a cluster
 
 // Exclusive prefix of v over the block (any blockDim <= 1024) and the total.
 __device__ __forceinline__ int block_scan_total(int v, int* sh, int& total) {
@@ -638,7 +645,7 @@ __device__ __noinline__ void solve_exact(const Layout& Lo, const Lists& Ls, int 
 // size = segment).  Small C: the cluster's rank 0 solves alone.  Large C: every
 // CTA of the cluster walks a share of the segment's chunks in each pass and the
 // CTA partials are combined through distributed shared memory in rank order.
-__global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lists Ls, double kappa, int iters,
+__global__ void __launch_bounds__(kSolveMaxThreads) k_solve(Layout Lo, SegParam* sp, Lists Ls, double kappa, int iters,
                                                     int force_exact, int* status, gs_info_dev* info,
                                                     int cap_chunks, int cap_c) {
     grid_dep_wait();
@@ -653,7 +660,7 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
     __shared__ double shd[33];
     __shared__ int shi[33];
     __shared__ float s_acap;
-    __shared__ double shdd[kThreads + 1];
+    __shared__ double shdd[kSolveMaxThreads + 1];
     __shared__ double s_S, s_lam, s_K, s_Su;
     __shared__ int s_go, s_j, s_fresh;
     __shared__ float4 sh4[33];
@@ -677,7 +684,8 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
     C.gbase = Ls.c_val + (int64_t)m * Lo.d + lo;
     C.smem = nullptr;
     double sl = 0.0;
-    if (nch <= kSolvePer * kThreads) {
+    const int nthr = blockDim.x, nwarp = nthr >> 5;
+    if (nch <= kSolvePer * nthr) {
         // Every chunk count and l1 partial in one round of loads (kSolvePer
         // consecutive chunks per thread), one block scan, and each thread
         // copies its own chunks' values of C.
@@ -705,7 +713,7 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
             // copies its own, their loads being independent.  Otherwise (few or
             // dense chunks; a short segment takes every coordinate): a warp per
             // chunk, or the whole CTA per chunk when there are few.
-            if (nch >= 2 * kThreads && total <= 32 * nch) {
+            if (nch >= 2 * nthr && total <= 32 * nch) {
                 int at = run - tot;
 #pragma unroll
                 for (int j = 0; j < kSolvePer; ++j) {
@@ -715,13 +723,13 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
                 }
             } else {
                 __syncthreads();   // pre[] complete
-                if (nch <= kWarps) {
+                if (nch <= nwarp) {
                     for (int q = 0; q < nch; ++q) {
                         const int b = pre[q], n = pre[q + 1] - b;
                         for (int v = tid; v < n; v += blockDim.x) sc[b + v] = C.gbase[(int64_t)q * kChunk + v];
                     }
                 } else {
-                    for (int q = warp; q < nch; q += kWarps) {
+                    for (int q = warp; q < nch; q += nwarp) {
                         const int b = pre[q], n = pre[q + 1] - b;
                         for (int v = lane; v < n; v += 32) sc[b + v] = C.gbase[(int64_t)q * kChunk + v];
                     }
@@ -750,7 +758,7 @@ __global__ void __launch_bounds__(kThreads) k_solve(Layout Lo, SegParam* sp, Lis
         auto stats = [&](float acap, float& rh, float& rl, int& rk) {
             float hi_ = 0.0f, lo_ = 0.0f;
             int k_ = 0;
-            for (int q = rank * (kThreads / 32) + warp; q < nch; q += ncta * (kThreads / 32)) {
+            for (int q = rank * nwarp + warp; q < nch; q += ncta * nwarp) {
                 const int n = pre[q + 1] - pre[q];
                 const float* src = C.gbase + (int64_t)q * kChunk;
                 for (int e = lane; e < n; e += 32) {
@@ -1506,7 +1514,7 @@ cudaError_t launch_solve(const Layout& Lo, SegParam* sp, const Lists& Ls, int n_
     if (ncta == 1)
         return launch_dep(k_solve, dim3(n_seg), dim3(kThreads), smem, st, Lo, sp, Ls, kappa, iters, force_exact,
                           status, info, cap_chunks, cap_c);
-    return launch_dep_cluster(k_solve, dim3(n_seg * ncta), dim3(kThreads), smem, ncta, st, Lo, sp, Ls, kappa, iters,
+    return launch_dep_cluster(k_solve, dim3(n_seg * ncta), dim3(kSolveClusterThreads), smem, ncta, st, Lo, sp, Ls, kappa, iters,
                               force_exact, status, info, cap_chunks, cap_c);
 }
 
