@@ -647,6 +647,14 @@ def run_hybrid(gs, g, kappa, w, args, dev, stream, n_steps, hbm):
     algo = M * d * esz + 8 * int(a.sum()) + 4 * int(b_.sum()) + 4 * M
     gbs = algo / (ms / 1e3) / 1e9
     dense = run_dense_code(gs, qa_i, qb, na, nb, d, bits["dense_entropy"], dev, stream, n_steps, hbm)
+    # The chunk size trades bits (each chunk adds a directory entry and a
+    # flushed state) for parallelism (chunks are coded independently).
+    if "error" not in dense:
+        dense["by_chunk_size"] = []
+        for lk in DENSE_LOG2_K_SWEEP:
+            r = run_dense_code(gs, qa_i, qb, na, nb, d, bits["dense_entropy"], dev, stream, n_steps, hbm, log2_k=lk)
+            dense["by_chunk_size"].append({k: r.get(k) for k in ("log2_k", "bits_per_coordinate", "over_entropy",
+                                                                 "encode_ms", "decode_ms", "error") if k in r})
     return {"api": "gs_batched_sparsify_hybrid", "dense_coded": dense, "steps": n_steps, "ms_per_step": round(ms, 4),
             "algorithmic_bytes": algo, "achieved": round(gbs, 1), "peak": hbm, "frac": round(gbs / hbm, 4),
             "unit": "GB/s", "n_a": int(a.sum()), "n_b": int(b_.sum()),
@@ -654,16 +662,18 @@ def run_hybrid(gs, g, kappa, w, args, dev, stream, n_steps, hbm):
             "bits_per_coordinate": {k: round(v / (M * d), 4) for k, v in bits.items()}}
 
 
-DENSE_LOG2_K = 9   # non-zero symbols per chunk of the dense code
+DENSE_LOG2_K = 9   # log2 of the non-zero symbols per chunk of the dense code
+DENSE_LOG2_K_SWEEP = (5, 6, 7, 8, 10)   # the other chunk sizes the bench line reports
 
 
-def run_dense_code(gs, qa_i, qb, na, nb, d, entropy_bits, dev, stream, n_steps, hbm):
+def run_dense_code(gs, qa_i, qb, na, nb, d, entropy_bits, dev, stream, n_steps, hbm, log2_k=None):
     """The dense code of section 3.3 (gs_dense_encode / gs_dense_decode) of one
     step's hybrid lists: its length in bits per coordinate against the model's
     entropy length sum_s d_s log2(d / d_s), and the time of each direction.
     Algorithmic bytes: the lists read (4 bytes per entry) and the code written
     (encoder); the code read and the dense int8 rows written (decoder)."""
     import torch
+    log2_k = DENSE_LOG2_K if log2_k is None else log2_k
     M = qa_i.shape[0]
     word_cap = d // 4 + 4096
     words = torch.empty((M, word_cap), dtype=torch.int16, device=dev)
@@ -682,7 +692,7 @@ def run_dense_code(gs, qa_i, qb, na, nb, d, entropy_bits, dev, stream, n_steps, 
         torch.cuda.synchronize()
         return e0.elapsed_time(e1) / n_steps
 
-    enc = timed(lambda: gs.gs_dense_encode(qa_i, qb, na, nb, d, DENSE_LOG2_K, words, n_words, stream=stream))
+    enc = timed(lambda: gs.gs_dense_encode(qa_i, qb, na, nb, d, log2_k, words, n_words, stream=stream))
     dec = timed(lambda: gs.gs_dense_decode(words, n_words, d, qt, stream=stream))
     rc = gs.gs_sync_status(stream)
     if rc != gs.GS_OK:
@@ -691,7 +701,7 @@ def run_dense_code(gs, qa_i, qb, na, nb, d, entropy_bits, dev, stream, n_steps, 
     entries = int(na.sum().item()) + int(nb.sum().item())
     b_enc = 4 * entries + 2 * total_words
     b_dec = 2 * total_words + M * d
-    return {"api": "gs_dense_encode / gs_dense_decode", "log2_k": DENSE_LOG2_K, "words": total_words,
+    return {"api": "gs_dense_encode / gs_dense_decode", "log2_k": log2_k, "words": total_words,
             "bits_per_coordinate": round(16.0 * total_words / (M * d), 5),
             "entropy_bits_per_coordinate": round(entropy_bits / (M * d), 5),
             "over_entropy": round(16.0 * total_words / entropy_bits, 4) if entropy_bits else None,

@@ -73,6 +73,7 @@ struct DenseModel {
     Sym bit0[kBitModels], bit1[kBitModels];
     Sym val[3];                 // +1, -1, 2
     uint32_t len_c[kLens + 1];  // cumulative starts for the decoder's search
+    uint8_t len_lut[256];       // the length whose range holds slot 128 b: where the decoder's search starts
     int64_t n_pos, n_neg, n_cap, nz;
     int64_t n_chunks, chunk0;   // chunks of this worker, and the chunks of all workers before it
     int64_t words;              // total words of the worker's code (after the scan)
@@ -112,53 +113,90 @@ __device__ void quantise(const double* P, const bool* can, int n, uint32_t* f) {
     f[best] = (uint32_t)((long long)f[best] + (long long)kM - sum);
 }
 
-__device__ void build_model(int64_t d, int64_t n_pos, int64_t n_neg, int64_t n_cap, DenseModel& m) {
+// A worker's model, built by a whole block (any blockDim >= 32) from its
+// symbol counts: p0 = d_0 / d; the bit-length model P(l) = p0^(2^l - 1)
+// (1 - p0^(2^l)) and the bit models P(bit k = 1) = s_k / (1 + s_k) with
+// s_k = p0^(2^k), each quantised as the oracle does; the value model d_t / nz.  The two serial
+// chains (the repeated squaring of p0 and the running product before each
+// length) stay on thread 0; the frequencies' divisions run side by side.
+__device__ void build_model_block(int64_t d, int64_t n_pos, int64_t n_neg, int64_t n_cap, DenseModel& m) {
+    __shared__ double s_sq[kLens], s_P[kLens];
+    __shared__ uint32_t s_f[kLens], s_c[kLens + 1], s_fv[3], s_cv[3];
+    const int tid = threadIdx.x;
     const int64_t nz = n_pos + n_neg + n_cap;
-    m.n_pos = n_pos;
-    m.n_neg = n_neg;
-    m.n_cap = n_cap;
-    m.nz = nz;
-    double sq[kLens], P[kLens];
-    bool can[kLens];
-    uint32_t f[kLens];
-    sq[0] = __ddiv_rn((double)(d - nz), (double)d);
-    for (int k = 1; k < kLens; ++k) sq[k] = __dmul_rn(sq[k - 1], sq[k - 1]);
-    for (int k = 0; k < kBitModels; ++k) {
-        const double r = __ddiv_rn(sq[k], __dadd_rn(1.0, sq[k]));
+    if (tid == 0) {
+        m.n_pos = n_pos;
+        m.n_neg = n_neg;
+        m.n_cap = n_cap;
+        m.nz = nz;
+        double sq = __ddiv_rn((double)(d - nz), (double)d);
+        double pi = 1.0;
+        for (int l = 0; l < kLens; ++l) {
+            s_sq[l] = sq;
+            s_P[l] = __dmul_rn(pi, __dsub_rn(1.0, sq));
+            pi = __dmul_rn(pi, sq);
+            sq = __dmul_rn(sq, sq);
+        }
+    }
+    __syncthreads();
+    for (int k = tid; k < kBitModels; k += blockDim.x) {
+        const double r = __ddiv_rn(s_sq[k], __dadd_rn(1.0, s_sq[k]));
         uint32_t f1 = ((uint32_t)floor(__dmul_rn(r, 65536.0)) + 1u) >> 1;
         f1 = min(max(f1, 1u), kM - 1u);
         m.bit0[k] = make_sym(kM - f1, 0u);
         m.bit1[k] = make_sym(f1, kM - f1);
     }
-    double pi = 1.0;
-    for (int l = 0; l < kLens; ++l) {
-        P[l] = __dmul_rn(pi, __dsub_rn(1.0, sq[l]));
-        pi = __dmul_rn(pi, sq[l]);
-        can[l] = true;
+    for (int l = tid; l < kLens; l += blockDim.x) {
+        const double t = floor(__dmul_rn(s_P[l], (double)kM));
+        s_f[l] = t < 1.0 ? 1u : (uint32_t)t;
     }
-    quantise(P, can, kLens, f);
-    uint32_t c = 0;
-    for (int l = 0; l < kLens; ++l) {
-        m.len[l] = make_sym(f[l], c);
-        m.len_c[l] = c;
-        c += f[l];
+    __syncthreads();
+    if (tid == 0) {
+        // quantise's remainder to the first most probable length, then the starts
+        long long sum = 0;
+        int best = 0;
+        for (int l = 0; l < kLens; ++l) {
+            sum += s_f[l];
+            if (s_f[l] > s_f[best]) best = l;
+        }
+        s_f[best] = (uint32_t)((long long)s_f[best] + (long long)kM - sum);
+        uint32_t c = 0;
+        for (int l = 0; l < kLens; ++l) {
+            s_c[l] = c;
+            c += s_f[l];
+        }
+        s_c[kLens] = c;
+        // the value model (three symbols)
+        const int64_t nt[3] = {n_pos, n_neg, n_cap};
+        double Pv[3];
+        bool cv[3];
+        for (int t = 0; t < 3; ++t) {
+            Pv[t] = nz > 0 ? __ddiv_rn((double)nt[t], (double)nz) : 0.0;
+            cv[t] = nt[t] > 0;
+        }
+        if (nz == 0) cv[0] = true;   // an unused model still sums to 2^15
+        uint32_t fv[3];
+        quantise(Pv, cv, 3, fv);
+        uint32_t cc = 0;
+        for (int t = 0; t < 3; ++t) {
+            s_fv[t] = fv[t];
+            s_cv[t] = cc;
+            cc += fv[t];
+        }
     }
-    m.len_c[kLens] = c;
-    double Pv[3];
-    bool cv[3];
-    const int64_t nt[3] = {n_pos, n_neg, n_cap};
-    for (int t = 0; t < 3; ++t) {
-        Pv[t] = nz > 0 ? __ddiv_rn((double)nt[t], (double)nz) : 0.0;
-        cv[t] = nt[t] > 0;
+    __syncthreads();
+    for (int l = tid; l <= kLens; l += blockDim.x) {
+        m.len_c[l] = s_c[l];
+        if (l < kLens) m.len[l] = make_sym(s_f[l], s_c[l]);
     }
-    if (nz == 0) cv[0] = true;   // an unused model still sums to 2^15
-    uint32_t fv[3];
-    quantise(Pv, cv, 3, fv);
-    c = 0;
-    for (int t = 0; t < 3; ++t) {
-        m.val[t] = make_sym(fv[t], c);
-        c += fv[t];
+    for (int b = tid; b < 256; b += blockDim.x) {
+        const uint32_t slot = (uint32_t)b << 7;
+        int l = 0;
+        while (l + 1 < kLens && s_c[l + 1] <= slot) ++l;
+        m.len_lut[b] = (uint8_t)l;
     }
+    for (int t = tid; t < 3; t += blockDim.x) m.val[t] = make_sym(s_fv[t], s_cv[t]);
+    __syncthreads();
 }
 
 // The two hybrid lists of one worker, ascending: Q_A indices (value 2) and
@@ -219,11 +257,6 @@ __device__ __forceinline__ Staged staged_at(unsigned char* base, int K) {
     return t;
 }
 
-__device__ __forceinline__ void copy_model(DenseModel* dst, const DenseModel* src, int lane) {
-    const uint32_t* s = reinterpret_cast<const uint32_t*>(src);
-    uint32_t* d = reinterpret_cast<uint32_t*>(dst);
-    for (int i = lane; i < (int)(sizeof(DenseModel) / 4); i += 32) d[i] = s[i];
-}
 
 // The warp stages the merge ranks [r0, r1) of worker lists L: both lists'
 // stretches are loaded, then each lane places its output positions by a
@@ -278,26 +311,41 @@ __global__ void k_dense_count(const uint32_t* __restrict__ qb, const int32_t* __
     if ((threadIdx.x & 31) == 0 && cnt) atomicAdd(neg + m, (unsigned long long)cnt);
 }
 
-// One block: every worker's model and chunk count, the header words, and
-// the chunks of all workers before each (serial over the workers).
+// One block per worker: its model and chunk count, the header words, and
+// the chunks of all workers before it (from the list lengths, which every
+// block reads; the last block writes the total).
+__device__ __forceinline__ bool lists_ok(int64_t na, int64_t nb, int64_t cap, int64_t d) {
+    return !(na > cap || nb > cap || na < 0 || nb < 0 || na + nb > d);
+}
+
 __global__ void k_dense_setup(const int32_t* __restrict__ n_a, const int32_t* __restrict__ n_b,
                               const unsigned long long* __restrict__ neg, int M, int64_t d, int64_t cap, int log2_k,
                               DenseModel* md, uint16_t* words, int64_t word_cap, int64_t* total_chunks, int* status) {
     grid_dep_wait();
-    for (int m = threadIdx.x; m < M; m += blockDim.x) {
-        const int64_t na = n_a[m], nb = n_b[m];
-        DenseModel& mm = md[m];
-        if (na > cap || nb > cap || na < 0 || nb < 0 || na + nb > d) {
-            atomicOr(status, kStInvalid);   // lists that overflowed their capacity cannot be coded
-            build_model(d, 0, 0, 0, mm);
-            mm.n_chunks = 0;
-        } else {
-            const int64_t nn = (int64_t)neg[m];
-            build_model(d, nb - nn, nn, na, mm);
-            mm.n_chunks = (mm.nz + ((int64_t)1 << log2_k) - 1) >> log2_k;
-        }
+    __shared__ long long s_red[32];
+    const int m = blockIdx.x, tid = threadIdx.x;
+    const int64_t na = n_a[m], nb = n_b[m];
+    const bool ok = lists_ok(na, nb, cap, d);
+    DenseModel& mm = md[m];
+    if (ok) build_model_block(d, nb - (int64_t)neg[m], (int64_t)neg[m], na, mm);
+    else build_model_block(d, 0, 0, 0, mm);
+    // chunks of the workers before this one
+    long long before = 0;
+    for (int j = tid; j < m; j += blockDim.x) {
+        const int64_t a = n_a[j], bb = n_b[j];
+        if (lists_ok(a, bb, cap, d)) before += (a + bb + ((int64_t)1 << log2_k) - 1) >> log2_k;
+    }
+    before = warp_sum(before);
+    if ((tid & 31) == 0) s_red[tid >> 5] = before;
+    __syncthreads();
+    if (tid == 0) {
+        long long c0 = 0;
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) c0 += s_red[w];
+        mm.n_chunks = ok ? (mm.nz + ((int64_t)1 << log2_k) - 1) >> log2_k : 0;
+        mm.chunk0 = c0;
         mm.log2_k = log2_k;
         mm.status = 0;
+        if (!ok) atomicOr(status, kStInvalid);   // lists that overflowed their capacity cannot be coded
         if (word_cap >= kHeaderWords) {
             uint16_t* w = words + (int64_t)m * word_cap;
             put32(w, (uint32_t)d);
@@ -306,15 +354,7 @@ __global__ void k_dense_setup(const int32_t* __restrict__ n_a, const int32_t* __
             put32(w + 6, (uint32_t)mm.n_cap);
             w[8] = (uint16_t)log2_k;
         }
-    }
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        int64_t acc = 0;
-        for (int m = 0; m < M; ++m) {
-            md[m].chunk0 = acc;
-            acc += md[m].n_chunks;
-        }
-        *total_chunks = acc;
+        if (m == M - 1) *total_chunks = c0 + mm.n_chunks;
     }
 }
 
@@ -364,28 +404,69 @@ __global__ void __launch_bounds__(kDenseWarps * 32)
 
 // rANS encoding of merge ranks [r0, r1) of one worker from its merged
 // sequence (one thread): returns the number of emitted words; with out,
-// writes the stream there (n_emitted from the counting pass).
-__device__ int encode_seq(const DenseModel& md, const int32_t* idx, const uint8_t* typ, int r0, int r1,
-                          uint16_t* out, int n_emitted) {
+// writes the stream there (n_emitted from the counting pass).  Symbols are
+// coded last to first; the value symbols and preceding indices of the next
+// four are loaded while the current four are coded.
+struct Batch {
+    uint32_t typ4;   // value symbols of ranks j, j-1, j-2, j-3 (a byte each)
+    int prev[4];     // index of rank j-u-1 (the end of rank j-u's run)
+};
+
+__device__ __forceinline__ Batch load_batch(const int32_t* idx, const uint8_t* typ, int j, int r0) {
+    Batch b;
+    b.typ4 = 0;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        const int jj = j - u;
+        if (jj >= r0) b.typ4 |= (uint32_t)typ[jj] << (8 * u);
+        b.prev[u] = jj - 1 >= r0 ? idx[jj - 1] : 0;
+    }
+    return b;
+}
+
+__device__ __forceinline__ int encode_seq(const DenseModel& md, const int32_t* idx, const uint8_t* typ, int r0,
+                                          int r1, uint16_t* out, int n_emitted) {
     uint32_t x = kLow;
     int n = 0;
     uint16_t* w = out ? out + 2 + (n_emitted - 1) : nullptr;
     int cur = idx[r1 - 1];
-    for (int j = r1 - 1; j >= r0; --j) {
-        put(x, md.val[typ[j]], w, n);
-        if (j == r0) break;
-        const int prev = idx[j - 1];
-        const uint32_t v = (uint32_t)(cur - prev);   // run of zeros + 1
-        const int l = 31 - __clz(v);
-        for (int k = 0; k < l; ++k) put(x, ((v >> k) & 1u) ? md.bit1[k] : md.bit0[k], w, n);
-        put(x, md.len[l], w, n);
-        cur = prev;
+    Batch b = load_batch(idx, typ, r1 - 1, r0);
+    for (int j = r1 - 1; j >= r0; j -= 4) {
+        const Batch nb = j - 4 >= r0 ? load_batch(idx, typ, j - 4, r0) : b;
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int jj = j - u;
+            if (jj < r0) break;
+            put(x, md.val[(b.typ4 >> (8 * u)) & 0xFFu], w, n);
+            if (jj == r0) break;
+            const int prev = b.prev[u];
+            const uint32_t v = (uint32_t)(cur - prev);   // run of zeros + 1
+            const int l = 31 - __clz(v);
+            for (int k = 0; k < l; ++k) put(x, ((v >> k) & 1u) ? md.bit1[k] : md.bit0[k], w, n);
+            put(x, md.len[l], w, n);
+            cur = prev;
+        }
+        b = nb;
     }
     if (out) {
         out[0] = (uint16_t)(x >> 16);
         out[1] = (uint16_t)(x & 0xFFFFu);
     }
     return n;
+}
+
+// The models of the workers whose chunks one block handles, staged in
+// shared memory: the coding steps read them there, where the global stores
+// of the coded words cannot alias them (a generic pointer could, which
+// would make every step reload its symbol).  kStageModels workers cover a
+// block's 128 consecutive chunks unless workers have fewer chunks than that.
+constexpr int kStageModels = 4;
+
+__device__ __forceinline__ void stage_models(DenseModel* dst, const DenseModel* __restrict__ src, int n) {
+    const int words = n * (int)(sizeof(DenseModel) / 4);
+    const uint32_t* s = reinterpret_cast<const uint32_t*>(src);
+    uint32_t* d = reinterpret_cast<uint32_t*>(dst);
+    for (int i = threadIdx.x; i < words; i += blockDim.x) d[i] = s[i];
 }
 
 // Counting pass (kWrite false): each chunk's stream length and first index.
@@ -398,21 +479,32 @@ __global__ void __launch_bounds__(128)
                    int32_t* ch_len, int32_t* ch_first, const int64_t* __restrict__ ch_off, uint16_t* words,
                    int64_t word_cap) {
     grid_dep_wait();
+    __shared__ DenseModel s_md[kStageModels];
     const int64_t total = *total_chunks;
-    for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < total; g += (int64_t)gridDim.x * blockDim.x) {
+    for (int64_t g0 = (int64_t)blockIdx.x * blockDim.x; g0 < total; g0 += (int64_t)gridDim.x * blockDim.x) {
+        const int m_lo = chunk_worker(md, M, g0);
+        const int m_hi = chunk_worker(md, M, min(g0 + (int64_t)blockDim.x, total) - 1);
+        __syncthreads();   // the previous round's readers are done
+        stage_models(s_md, md + m_lo, min(m_hi - m_lo + 1, kStageModels));
+        __syncthreads();
+        const int64_t g = g0 + threadIdx.x;
+        if (g >= total) continue;
         const int m = chunk_worker(md, M, g);
-        const DenseModel& mm = md[m];
-        if (kWrite && mm.words > word_cap) continue;
-        const int64_t i = g - mm.chunk0;
-        const int r0 = (int)(i << log2_k), r1 = (int)min((int64_t)r0 + ((int64_t)1 << log2_k), mm.nz);
+        const DenseModel& gm = md[m];
+        if (kWrite && gm.words > word_cap) continue;
+        const int64_t i = g - gm.chunk0;
+        const int r0 = (int)(i << log2_k), r1 = (int)min((int64_t)r0 + ((int64_t)1 << log2_k), gm.nz);
         const int32_t* idx = m_idx + (int64_t)m * stride;
         const uint8_t* typ = m_typ + (int64_t)m * stride;
+        uint16_t* out = kWrite ? words + (int64_t)m * word_cap + kHeaderWords + kDirWords * gm.n_chunks + ch_off[g]
+                               : nullptr;
+        const int n_em = kWrite ? ch_len[g] - 2 : 0;
+        int n;
+        if (m - m_lo < kStageModels) n = encode_seq(s_md[m - m_lo], idx, typ, r0, r1, out, n_em);
+        else n = encode_seq(gm, idx, typ, r0, r1, out, n_em);
         if (!kWrite) {
-            ch_len[g] = encode_seq(mm, idx, typ, r0, r1, nullptr, 0) + 2;
+            ch_len[g] = n + 2;
             ch_first[g] = idx[r0];
-        } else {
-            uint16_t* out = words + (int64_t)m * word_cap + kHeaderWords + kDirWords * mm.n_chunks + ch_off[g];
-            encode_seq(mm, idx, typ, r0, r1, out, ch_len[g] - 2);
         }
     }
 }
@@ -466,43 +558,63 @@ __global__ void k_dense_scan(DenseModel* md, const int32_t* __restrict__ ch_len,
 // ---------------------------------------------------------------------------
 // Decoder
 // ---------------------------------------------------------------------------
-// One block: every worker's header read back, its model rebuilt, and the
-// chunks of all workers before each.  A malformed header records kStInvalid
-// and leaves that worker with no chunk.
+// Worker m's header read back: its counts and chunk size, and its chunk
+// count (0 for a malformed header or a code too short for its directory).
+struct Header {
+    int64_t np, nn, nc, n_chunks;
+    int lk;
+    bool ok;
+};
+
+__device__ Header read_header(const uint16_t* __restrict__ words, const int64_t* __restrict__ n_words, int m,
+                              int64_t d, int64_t word_cap) {
+    Header h = {0, 0, 0, 0, 4, false};
+    const uint16_t* w = words + (int64_t)m * word_cap;
+    const int64_t nw = n_words[m];
+    bool ok = nw >= kHeaderWords && nw <= word_cap;
+    if (ok) {
+        h.np = get32(w + 2);
+        h.nn = get32(w + 4);
+        h.nc = get32(w + 6);
+        h.lk = w[8];
+        ok = (int64_t)get32(w) == d && h.lk >= 4 && h.lk <= 10 && h.np + h.nn + h.nc <= d;
+    }
+    if (ok) {
+        h.n_chunks = (h.np + h.nn + h.nc + ((int64_t)1 << h.lk) - 1) >> h.lk;
+        if (nw < kHeaderWords + kDirWords * h.n_chunks) ok = false;
+    }
+    if (!ok) {
+        h.np = h.nn = h.nc = h.n_chunks = 0;
+    }
+    h.ok = ok;
+    return h;
+}
+
+// One block per worker: its header read back and its model rebuilt, and the
+// chunks of all workers before it (from their headers; the last block writes
+// the total).  A malformed header records kStInvalid and leaves that worker
+// with no chunk.
 __global__ void k_dense_dsetup(const uint16_t* __restrict__ words, const int64_t* __restrict__ n_words, int M,
                                int64_t d, int64_t word_cap, DenseModel* md, int64_t* total_chunks, int* status) {
     grid_dep_wait();
-    for (int m = threadIdx.x; m < M; m += blockDim.x) {
-        const uint16_t* w = words + (int64_t)m * word_cap;
-        const int64_t nw = n_words[m];
-        DenseModel& mm = md[m];
-        bool ok = nw >= kHeaderWords && nw <= word_cap;
-        int64_t np = 0, nn = 0, nc = 0;
-        int lk = 4;
-        if (ok) {
-            np = get32(w + 2);
-            nn = get32(w + 4);
-            nc = get32(w + 6);
-            lk = w[8];
-            ok = (int64_t)get32(w) == d && lk >= 4 && lk <= 10 && np + nn + nc <= d;
-        }
-        build_model(d, ok ? np : 0, ok ? nn : 0, ok ? nc : 0, mm);
-        mm.log2_k = lk;
-        mm.n_chunks = ok ? (mm.nz + ((int64_t)1 << lk) - 1) >> lk : 0;
-        if (ok && nw < kHeaderWords + kDirWords * mm.n_chunks) {
-            ok = false;
-            mm.n_chunks = 0;
-        }
-        if (!ok) atomicOr(status, kStInvalid);
-    }
+    __shared__ long long s_red[32];
+    const int m = blockIdx.x, tid = threadIdx.x;
+    const Header h = read_header(words, n_words, m, d, word_cap);
+    DenseModel& mm = md[m];
+    build_model_block(d, h.np, h.nn, h.nc, mm);
+    long long before = 0;
+    for (int j = tid; j < m; j += blockDim.x) before += read_header(words, n_words, j, d, word_cap).n_chunks;
+    before = warp_sum(before);
+    if ((tid & 31) == 0) s_red[tid >> 5] = before;
     __syncthreads();
-    if (threadIdx.x == 0) {
-        int64_t acc = 0;
-        for (int m = 0; m < M; ++m) {
-            md[m].chunk0 = acc;
-            acc += md[m].n_chunks;
-        }
-        *total_chunks = acc;
+    if (tid == 0) {
+        long long c0 = 0;
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) c0 += s_red[w];
+        mm.log2_k = h.lk;
+        mm.n_chunks = h.n_chunks;
+        mm.chunk0 = c0;
+        if (!h.ok) atomicOr(status, kStInvalid);
+        if (m == M - 1) *total_chunks = c0 + h.n_chunks;
     }
 }
 
@@ -545,75 +657,123 @@ __global__ void k_dense_dscan(DenseModel* md, const uint16_t* __restrict__ words
 }
 
 // One rANS decoding step: the symbol whose [c, c + f) holds x's low 15 bits.
+// The stream's next words wait in a register window (four words, refilled
+// four at a time from loads issued one window ahead), so a renormalisation
+// rarely waits on memory.
 struct Dec {
     const uint16_t* w;
-    int pos, len;
+    int pos, len;       // next word to load into the window, stream length
+    uint64_t win, nxt;  // current and next window, low word first
+    int nwin, nnxt;     // words left in each
     uint32_t x;
     bool bad;
+    __device__ __forceinline__ void fetch(uint64_t& v, int& n) {
+        v = 0;
+        n = 0;
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            if (pos + k < len) {
+                v |= (uint64_t)w[pos + k] << (16 * k);
+                ++n;
+            }
+        }
+        pos += n;
+    }
+    __device__ __forceinline__ void start() {
+        fetch(win, nwin);
+        fetch(nxt, nnxt);
+    }
     __device__ __forceinline__ void step(uint32_t f, uint32_t c, uint32_t slot) {
         x = f * (x >> kScale) + slot - c;
         if (x < kLow) {
-            if (pos < len) x = (x << 16) | w[pos++];
-            else bad = true;
+            if (nwin == 0 && nnxt > 0) {
+                win = nxt;
+                nwin = nnxt;
+                fetch(nxt, nnxt);
+            }
+            if (nwin > 0) {
+                x = (x << 16) | (uint32_t)(win & 0xFFFFu);
+                win >>= 16;
+                --nwin;
+            } else {
+                bad = true;
+            }
         }
     }
+    __device__ __forceinline__ bool done() const { return nwin == 0 && nnxt == 0 && pos == len; }
 };
 
+// Decodes chunk i of worker m into its dense q~ row; false when the
+// stream is malformed.
+__device__ __forceinline__ bool decode_chunk(const DenseModel& mm, const uint16_t* base, int64_t i, int64_t off,
+                                             int64_t d, int8_t* row) {
+    const uint16_t* dir = base + kHeaderWords + kDirWords * i;
+    const int64_t K = (int64_t)1 << mm.log2_k;
+    const int64_t cnt = min(K, mm.nz - i * K);
+    Dec r;
+    r.w = base + kHeaderWords + kDirWords * mm.n_chunks + off;
+    r.len = dir[2];
+    r.bad = r.len < 2;
+    r.x = r.bad ? kLow : (((uint32_t)r.w[0] << 16) | r.w[1]);
+    r.pos = r.bad ? r.len : 2;
+    r.start();
+    int64_t idx = get32(dir);
+    for (int64_t j = 0; j < cnt && !r.bad; ++j) {
+        if (j > 0) {
+            // run bit length: the last l with len_c[l] <= slot, searched
+            // forward from the table's start for the slot's top 8 bits
+            const uint32_t slot = r.x & (kM - 1u);
+            int a = mm.len_lut[slot >> 7];
+            while (a + 1 < kLens && mm.len_c[a + 1] <= slot) ++a;
+            r.step(mm.len[a].f, mm.len[a].c, slot);
+            uint32_t v = 1;
+            for (int k = a - 1; k >= 0; --k) {
+                const uint32_t sl = r.x & (kM - 1u);
+                const uint32_t f0 = mm.bit0[k].f;
+                const uint32_t bit = sl >= f0 ? 1u : 0u;
+                if (bit) r.step(mm.bit1[k].f, mm.bit1[k].c, sl); else r.step(f0, 0u, sl);
+                v = 2u * v + bit;
+            }
+            idx += v;
+        }
+        const uint32_t sl = r.x & (kM - 1u);
+        const int t = sl < mm.val[1].c ? 0 : (sl < mm.val[2].c ? 1 : 2);
+        r.step(mm.val[t].f, mm.val[t].c, sl);
+        if (idx < 0 || idx >= d) {
+            r.bad = true;
+            break;
+        }
+        row[idx] = t == 0 ? (int8_t)1 : (t == 1 ? (int8_t)-1 : (int8_t)2);
+    }
+    return !(r.bad || r.x != kLow || !r.done());
+}
+
 // Decodes every chunk into the dense q~ rows (int8, zeroed beforehand), one
-// thread per chunk.
+// thread per chunk, with the block's models staged in shared memory.
 __global__ void __launch_bounds__(128)
     k_dense_decode(const uint16_t* __restrict__ words, const DenseModel* __restrict__ md, int M, int64_t d,
                    int64_t word_cap, const int64_t* __restrict__ total_chunks, const int64_t* __restrict__ ch_off,
                    int8_t* qt, int* status) {
     grid_dep_wait();
+    __shared__ DenseModel s_md[kStageModels];
     const int64_t total = *total_chunks;
-    for (int64_t g = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; g < total; g += (int64_t)gridDim.x * blockDim.x) {
+    for (int64_t g0 = (int64_t)blockIdx.x * blockDim.x; g0 < total; g0 += (int64_t)gridDim.x * blockDim.x) {
+        const int m_lo = chunk_worker(md, M, g0);
+        const int m_hi = chunk_worker(md, M, min(g0 + (int64_t)blockDim.x, total) - 1);
+        __syncthreads();   // the previous round's readers are done
+        stage_models(s_md, md + m_lo, min(m_hi - m_lo + 1, kStageModels));
+        __syncthreads();
+        const int64_t g = g0 + threadIdx.x;
+        if (g >= total) continue;
         const int m = chunk_worker(md, M, g);
-        const DenseModel& mm = md[m];
-        const int64_t i = g - mm.chunk0;
-        if (i >= mm.n_chunks) continue;   // a worker whose directory did not add up
+        const DenseModel& gm = md[m];
+        const int64_t i = g - gm.chunk0;
+        if (i >= gm.n_chunks) continue;   // a worker whose directory did not add up
         const uint16_t* base = words + (int64_t)m * word_cap;
-        const uint16_t* dir = base + kHeaderWords + kDirWords * i;
-        const int64_t K = (int64_t)1 << mm.log2_k;
-        const int64_t cnt = min(K, mm.nz - i * K);
-        Dec r;
-        r.w = base + kHeaderWords + kDirWords * mm.n_chunks + ch_off[g];
-        r.len = dir[2];
-        r.pos = 2;
-        r.bad = r.len < 2;
-        r.x = r.bad ? kLow : (((uint32_t)r.w[0] << 16) | r.w[1]);
-        int64_t idx = get32(dir);
         int8_t* row = qt + (int64_t)m * d;
-        for (int64_t j = 0; j < cnt && !r.bad; ++j) {
-            if (j > 0) {
-                // run bit length: the last l with len_c[l] <= slot
-                const uint32_t slot = r.x & (kM - 1u);
-                int a = 0, b = kLens - 1;
-                while (a < b) {
-                    const int mid = (a + b + 1) >> 1;
-                    if (mm.len_c[mid] <= slot) a = mid; else b = mid - 1;
-                }
-                r.step(mm.len[a].f, mm.len[a].c, slot);
-                uint32_t v = 1;
-                for (int k = a - 1; k >= 0; --k) {
-                    const uint32_t sl = r.x & (kM - 1u);
-                    const uint32_t f0 = mm.bit0[k].f;
-                    const uint32_t bit = sl >= f0 ? 1u : 0u;
-                    if (bit) r.step(mm.bit1[k].f, mm.bit1[k].c, sl); else r.step(f0, 0u, sl);
-                    v = 2u * v + bit;
-                }
-                idx += v;
-            }
-            const uint32_t sl = r.x & (kM - 1u);
-            const int t = sl < mm.val[1].c ? 0 : (sl < mm.val[2].c ? 1 : 2);
-            r.step(mm.val[t].f, mm.val[t].c, sl);
-            if (idx < 0 || idx >= d) {
-                r.bad = true;
-                break;
-            }
-            row[idx] = t == 0 ? (int8_t)1 : (t == 1 ? (int8_t)-1 : (int8_t)2);
-        }
-        if (r.bad || r.x != kLow || r.pos != r.len) atomicOr(status, kStInvalid);
+        const bool ok = m - m_lo < kStageModels ? decode_chunk(s_md[m - m_lo], base, i, ch_off[g], d, row)
+                                                : decode_chunk(gm, base, i, ch_off[g], d, row);
+        if (!ok) atomicOr(status, kStInvalid);
     }
 }
 
@@ -690,7 +850,7 @@ cudaError_t launch_dense_encode(const int32_t* qa, const uint32_t* qb, const int
     {
         set_launch_error_site("k_dense_setup launch");
         TraceScope ts(kKDenseSetup, st);
-        e = launch_dep(k_dense_setup, dim3(1), dim3(256), 0, st, n_a, n_b, (const unsigned long long*)w.neg, M, d, cap,
+        e = launch_dep(k_dense_setup, dim3(M), dim3(128), 0, st, n_a, n_b, (const unsigned long long*)w.neg, M, d, cap,
                        log2_k, w.md, words, word_cap, w.total, status);
         if (e != cudaSuccess) return e;
     }
@@ -739,7 +899,7 @@ cudaError_t launch_dense_decode(const uint16_t* words, const int64_t* n_words, i
     {
         set_launch_error_site("k_dense_dsetup launch");
         TraceScope ts(kKDenseSetup, st);
-        e = launch_dep(k_dense_dsetup, dim3(1), dim3(256), 0, st, words, n_words, M, d, word_cap, w.md, w.total,
+        e = launch_dep(k_dense_dsetup, dim3(M), dim3(128), 0, st, words, n_words, M, d, word_cap, w.md, w.total,
                        status);
         if (e != cudaSuccess) return e;
     }
