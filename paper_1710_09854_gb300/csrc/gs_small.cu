@@ -4,7 +4,7 @@
 // The chunked path (gs_kernels.cu, gs_stream_tma.cu) gives every
 // 16384-coordinate chunk to one warp and runs six kernels; a gradient of
 // 65536 coordinates is then four warps' work behind six launches, and one of
-// 2^20 coordinates sixty-four.  Here one thread-block cluster of up to 16
+// 2^20 coordinates sixty-four.  Here one thread-block cluster of up to 12
 // CTAs owns one worker: each CTA holds a contiguous share of the worker's
 // coordinates (in shared memory when the share fits, else re-read from L2),
 // and the passes of Algorithm 3 are plain walks over those shares, combined
@@ -15,17 +15,18 @@
 //                 mass, then lam_{j+1} = c lam_j (steps 4-10; `iters`
 //                 rescalings at most, stopping at c <= 1);
 //   decide        one Philox4x32-10 call per 4 coordinates, Z_i = [u_i < p_i]
-//                 (section 3) as one bit per coordinate, the kept counts per
-//                 128-coordinate tile and the statistics at the final lambda;
+//                 (section 3) as a kept bit per coordinate (with its sign and
+//                 capped bits), the kept counts per 128-coordinate tile and
+//                 the statistics at the final lambda;
 //   emit          kept coordinates at their output offsets (tile scan plus
 //                 the cluster's exclusive prefix in rank order), value g_i / p_i
 //                 (g_i when capped, sign(g_i) / lambda otherwise, section 5.3);
 //                 for one worker the dense sum (Algorithm 1 step 6) as well.
 //
 // k_small_sum adds M > 1 workers' kept values in worker order from their
-// decision bits (Algorithm 1 step 6).  Every sum is in a fixed order: the
-// result is a function of (g, kappa, iters, seed, step, worker) and of d,
-// not of M or of the other workers in the call.
+// kept, sign and capped bits (Algorithm 1 step 6).  Every sum is in a fixed
+// order: on this path a worker's result is a function of (g, kappa, iters,
+// seed, step, worker) and of d, not of M or of the other workers in the call.
 #include <cooperative_groups.h>
 #include <cuda_runtime.h>
 
@@ -68,8 +69,8 @@ struct SmallArgs {
     int* status;
     gs_info_dev* info;    // [M] or NULL
     SegParam* sp;         // [M] parameters for k_small_sum, or NULL
-    uint32_t* bits;       // [M][wpr] decision bits for k_small_sum, or NULL
-    int64_t wpr;          // words per worker row of `bits`
+    uint32_t* bits;       // [3][M][wpr] kept / sign / capped bits for k_small_sum, or NULL
+    int64_t wpr;          // words per worker row of each plane of `bits`
     float* out;           // M == 1: the dense sum, written here; else NULL
     float div;            // > 0: out is divided by div (the average of Algorithm 1 step 6)
     int accumulate;       // 1: out continues a worker-order sum already in out
