@@ -32,7 +32,6 @@
 
 #include <algorithm>
 #include <cstdint>
-#include <cstdlib>
 
 #include "gs_decide.cuh"
 #include "gs_device.cuh"
@@ -45,7 +44,6 @@ namespace {
 
 constexpr int kTile = 128;               // coordinates per warp step (4 consecutive per lane)
 constexpr int kBatch = 4;                // tiles whose loads a warp has in flight together
-constexpr int kMaxCtas = 16;             // cluster size limit (non-portable above 8)
 // Cluster size the automatic shape stops at: eight 12-CTA clusters of 1024
 // threads are resident together on a GB300, while only seven of 13, 14 or
 // 16 are (a ninth worker's cluster would wait for a second wave).
@@ -651,16 +649,13 @@ __global__ void __launch_bounds__(kSumThreads) k_small_sum(const __grid_constant
 }
 
 // Cluster size and share per CTA for a row of d coordinates: shares of about
-// 4096 coordinates, up to kMaxCtas CTAs (GS_SMALL_CTAS overrides the count),
-// and never above kMaxShare (whose three bitmaps and tile counts take 208 KiB).
+// 4096 coordinates, up to kAutoCtas CTAs, and never above kMaxShare (whose
+// three bitmaps and tile counts take 208 KiB).  A function of d alone: the
+// shape fixes the order of every sum, so a row's result depends on nothing
+// else.
 constexpr int64_t kMaxShare = (int64_t)1 << 19;
 void small_shape(int64_t d, int& ncta, int& n_per) {
-    static const int forced = [] {
-        const char* e = std::getenv("GS_SMALL_CTAS");
-        const int v = e ? std::atoi(e) : 0;
-        return v >= 1 && v <= kMaxCtas ? v : 0;
-    }();
-    ncta = forced ? forced : (int)std::min<int64_t>(kAutoCtas, std::max<int64_t>(1, (d + 4095) / 4096));
+    ncta = (int)std::min<int64_t>(kAutoCtas, std::max<int64_t>(1, (d + 4095) / 4096));
     ncta = (int)std::max<int64_t>(ncta, (d + kMaxShare - 1) / kMaxShare);
     const int64_t per = (d + ncta - 1) / ncta;
     n_per = (int)((per + kTile - 1) / kTile * kTile);
