@@ -307,6 +307,7 @@ def run_gpu(args):
     bd = gs.gs_kernel_times()
     gs.gs_set_option(gs.GS_OPT_KERNEL_TIMING, 0)
     kernels = {k: {"ms_per_step": round(v[0] / n_bd, 4), "launches": v[1]} for k, v in bd.items() if v[1]}
+    step_stats = per_step_stats(lambda t: step(args.warmup + args.steps + n_bd + t), n_bd, stream)
 
     # Sparsify alone (steps 1-5, no sum) against B_sparsify, on the same inputs.
     sp_only = None
@@ -365,7 +366,7 @@ def run_gpu(args):
         "variance_budget": vbudget,
         "average_resparsify": resp,
         "lr_sgd": lr,
-        "kernels": kernels, "kernels_steps": n_bd,
+        "kernels": kernels, "kernels_steps": n_bd, "step_ms_stats": step_stats,
         "nnz_per_step": nnz_total,
         "gpu_launches": launches,
         "clocks": clk,
@@ -383,6 +384,22 @@ def run_gpu(args):
 CONFIG_SWEEP = (("c1", None, None), ("c2", None, None), ("c3", None, None), ("c4", None, None),
                 ("c5", 0.001, "f32"), ("c5", 0.01, "f32"), ("c5", 0.1, "f32"),
                 ("c5", 0.001, "bf16"), ("c5", 0.01, "bf16"), ("c5", 0.1, "bf16"))
+
+
+def per_step_stats(step, n, stream):
+    """Median, p10 and p90 of n steps timed one by one (a pair of CUDA events
+    around each step, which keeps a step's first launch from overlapping the
+    previous step's last, so the median sits a little above ms_per_step)."""
+    import torch
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+    for t, (a, b) in enumerate(evs):
+        a.record(stream)
+        step(t)
+        b.record(stream)
+    torch.cuda.synchronize()
+    xs = sorted(a.elapsed_time(b) for a, b in evs)
+    q = lambda f: xs[min(len(xs) - 1, int(f * len(xs)))]
+    return {"steps": n, "median_ms": round(q(0.5), 5), "p10_ms": round(q(0.1), 5), "p90_ms": round(q(0.9), 5)}
 
 
 def run_configs(gs, args, dev, stream, hbm, rank):
@@ -435,6 +452,7 @@ def run_configs(gs, args, dev, stream, hbm, rank):
             if gs.gs_sync_status(stream) != gs.GS_OK:
                 raise RuntimeError("device status after timing")
             # The streaming pass, or the cluster-resident kernel on short rows.
+            stats = per_step_stats(lambda t: step(5 + 2 * n + t), min(n, 50), stream)
             sk = next((k for k in ("k_stream_tma", "k_stream", "k_small") if kt.get(k, (0, 0))[1]), "k_stream")
             s_ms = kt[sk][0] / max(kt[sk][1], 1)
             b_sp, b_ag = algorithmic_bytes(M, d, esz, kept)
@@ -447,7 +465,7 @@ def run_configs(gs, args, dev, stream, hbm, rank):
                          "nnz_per_step": kept, "algorithmic_bytes": b_sp + b_ag,
                          "step_gbs": round(step_gbs, 1), "step_frac": round(step_gbs / hbm, 4),
                          "stream_kernel": sk, "stream_ms": round(s_ms, 5), "stream_gbs": round(s_gbs, 1),
-                         "stream_frac": round(s_gbs / hbm, 4), "peak": hbm,
+                         "stream_frac": round(s_gbs / hbm, 4), "peak": hbm, "step_ms_stats": stats,
                          "l2": ("fits in L2" if M * d * esz < L2_BYTES else "exceeds L2")})
             del g, idx, val, nnz, out
         except Exception as e:  # one failed row never costs the bench line
@@ -903,25 +921,35 @@ def oracle_step(g_rows, off, kappa, iters, seed, step):
 
 
 def cpu_baseline_sample(g, off, kappa, w, budget_s=15.0):
-    """The oracle as it stands, single-threaded, on whole workers of the same
-    workload until about `budget_s` seconds of CPU work have run."""
+    """The oracle as it stands, single-threaded: whole workers of the same
+    workload sparsified until about `budget_s` seconds of CPU work have run,
+    then the sparse sum of their lists, each timed on its own (the rows'
+    copies to the host are outside the timed work)."""
     import oracle
     oracle.lib()
     M, d = g.shape
-    rows = []
-    t0 = time.perf_counter()
-    done = 0
+    il, vl = [], []
+    t_sp = 0.0
     for m in range(M):
         row = g[m].float().cpu().numpy()
-        rows.append(row)
-        s = time.perf_counter()
-        oracle_step([row], off, kappa, w.iters, w.seed, 0)
-        done += d
-        if time.perf_counter() - t0 > budget_s:
+        t = time.perf_counter()
+        if off is None:
+            i, v, _ = oracle.sparsify(row, kappa, w.iters, w.seed, 0, m)
+        else:
+            i, v, _ = oracle.segmented_sparsify(row, off, kappa, w.iters, w.seed, 0, m)
+        t_sp += time.perf_counter() - t
+        il.append(i)
+        vl.append(v)
+        if t_sp > budget_s:
             break
-    el = time.perf_counter() - t0
-    return {"value": done / el, "unit": UNIT, "cores": 1, "kind": "oracle", "host": host_cpu(),
-            "sample": f"{done // d} of {M} workers at full d={d} (sparsify + sparse sum), {el:.1f} s"}
+    t = time.perf_counter()
+    oracle.aggregate(il, vl, d)
+    t_ag = time.perf_counter() - t
+    done = len(il) * d
+    return {"value": done / (t_sp + t_ag), "unit": UNIT, "cores": 1, "kind": "oracle", "host": host_cpu(),
+            "sparsify_coords_per_s": done / t_sp, "sparsify_s": round(t_sp, 2), "aggregate_s": round(t_ag, 3),
+            "sample": f"{len(il)} of {M} workers at full d={d}: sparsify {t_sp:.1f} s, then the sparse sum of "
+                      f"their lists {t_ag:.2f} s"}
 
 
 def run_reference(args):
