@@ -219,9 +219,15 @@ __device__ __forceinline__ uint32_t word_of(const uint4& w, int s) {
 // Programmatic dependent launch: a kernel launched with programmatic stream
 // serialization may start while its predecessor in the stream still runs;
 // this waits until the predecessor grid has completed and its writes are
-// visible.  Every kernel of the library calls it first, unconditionally (a
-// plain launch returns at once), so completion stays transitive down the stream.
+// visible.  Every kernel of the library calls it, unconditionally, before it
+// reads anything a predecessor may have written (all but the streaming pass
+// call it first; a plain launch returns at once), so completion stays
+// transitive down the stream.
 __device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// Lets the next kernel in the stream launch before this grid completes (it
+// still waits for this grid in its own grid_dep_wait before it reads
+// anything this grid writes).
+__device__ __forceinline__ void grid_dep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
 // 1 + (x >> 9) * 2^-23: a float in [1, 2) that never exceeds 1 + x * 2^-32.
 // hi(x * 2^23) = x >> 9, so one multiply-add forms it on the integer-multiply pipe.

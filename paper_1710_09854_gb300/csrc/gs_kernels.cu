@@ -369,6 +369,9 @@ template <int kCTAs>
 __global__ void __cluster_dims__(kCTAs, 1, 1) __launch_bounds__(kBoundCtaThreads)
     k_bound(Layout Lo, SegParam* sp, double kappa, int ns, int force_exact) {
     grid_dep_wait();
+    // The streaming pass may launch now: it only loads g (an input of the
+    // call) until its own wait for this grid.
+    grid_dep_launch();
     namespace cg = cooperative_groups;
     cg::cluster_group cluster = cg::this_cluster();
     extern __shared__ float sa[];               // rank 0: all ns samples
@@ -1286,7 +1289,21 @@ __global__ void __launch_bounds__(kSumWarps * 32) k_sum(const __grid_constant__ 
     // div > 0: the average of Algorithm 1 step 6 (one correctly rounded
     // division of the worker-order sum), else the sum itself.
     float* dst = out + t0;
-    if (tlen == kSlice && (reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
+    const bool whole = tlen == kSlice && (reinterpret_cast<uintptr_t>(dst) & 15u) == 0;
+    if (whole && !(div > 0.0f)) {
+        // The sum leaves shared memory in one bulk copy (the asynchronous
+        // proxy reads the tile once every lane's writes are fenced).
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        __syncwarp();
+        if (lane == 0) {
+            asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst),
+                         "r"((uint32_t)__cvta_generic_to_shared(acc)), "r"((int)(kSlice * sizeof(float)))
+                         : "memory");
+            asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+            asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");   // the tile may be released
+        }
+        __syncwarp();
+    } else if (whole) {
 #pragma unroll
         for (int i = 0; i < kSlice / 128; ++i) {
             float4 t = reinterpret_cast<const float4*>(acc)[i * 32 + lane];

@@ -205,10 +205,14 @@ __device__ __forceinline__ float stage_value(const unsigned char* rp, int first_
 
 // Group j (0..7, four coordinates) of a lane's 32 as g values (signed; the
 // callers take |g| where they use it, which folds into their float operands).
+// fp32: from a 32-bit shared address, bsa = the lane's row in the buffer with
+// the 128-byte swizzle folded in (row | sw << 4): chunk j sits at j ^ sw, so
+// one XOR finds it.  bf16 (half a row per lane): from the generic row
+// pointer rp, the lane's first chunk and the swizzle (measured faster there).
 template <int kDtype>
-__device__ __forceinline__ float4 stage_group(const unsigned char* rp, int first_chunk, int sw, int j) {
+__device__ __forceinline__ float4 group_at(uint32_t bsa, const unsigned char* rp, int first_chunk, int sw, int j) {
     if (kDtype == 0) {
-        return *reinterpret_cast<const float4*>(rp + (((first_chunk + j) ^ sw) << 4));
+        return *reinterpret_cast<const float4*>(__cvta_shared_to_generic(bsa ^ (uint32_t)(j << 4)));
     } else {
         const uint2 t = *reinterpret_cast<const uint2*>(rp + (((first_chunk + (j >> 1)) ^ sw) << 4) + ((j & 1) << 3));
         return make_float4(__uint_as_float(t.x << 16), __uint_as_float(t.x & 0xFFFF0000u),
@@ -266,7 +270,6 @@ struct ChunkWalk {
 template <int kDtype, bool kSq>
 __global__ void __launch_bounds__(kTmaThreads, kTmaCtas)
     k_stream_tma(const __grid_constant__ CUtensorMap map, const __grid_constant__ StreamArgs A) {
-    grid_dep_wait();
     constexpr int kInner = kDtype == 0 ? 32 : 64;          // elements per 128-byte row
     constexpr int kBufRows = kBufCoords / kInner;          // 32 or 16
     constexpr int kBufBytes = kBufRows * kRowBytes;        // 4 KiB or 2 KiB
@@ -308,10 +311,11 @@ __global__ void __launch_bounds__(kTmaThreads, kTmaCtas)
         }
     };
     cursor();
-    int issued = 0;
+    int issued = 0, pslot = 0;
     auto prefetch = [&]() {
         if (pc.c >= A.n_chunks) return;
-        const int b = issued % kRing;
+        const int b = pslot;
+        pslot = pslot == kRing - 1 ? 0 : pslot + 1;
         if (lane == 0) {
             mbar_arrive_tx(&my_full[b], kBufBytes);
             tma_load_rows(my_buf + b * kBufBytes, &map, prow, &my_full[b]);
@@ -330,8 +334,21 @@ __global__ void __launch_bounds__(kTmaThreads, kTmaCtas)
             cursor();
         }
     };
+    // Until the predecessor grid has completed, only loads of g (an input of
+    // the call) are issued: the buffers of the warp's first chunk that need
+    // no chunk from the counter (the predecessor zeroes it).  Segment
+    // layouts read their tables from device memory, so they wait first.
+    int pre = 0;
+    if (Lo.L == 1) {
 #pragma unroll 1
-    for (int i = 0; i < kRing; ++i) prefetch();
+        while (pre < kRing && pc.c < A.n_chunks && prow + kBufRows < prow_end) {
+            prefetch();
+            ++pre;
+        }
+    }
+    grid_dep_wait();
+#pragma unroll 1
+    for (; pre < kRing; ++pre) prefetch();
 
     // candidate iff 1 + (x >> 9) 2^-23 < fl32(lam_up |g| + 1 + 2^-20) (cand_sign)
     const float pbias = 1.0f + 0x1p-20f;
@@ -344,6 +361,10 @@ __global__ void __launch_bounds__(kTmaThreads, kTmaCtas)
     const int sw = brow & 7;
     int slot = 0, consumed = 0;
     uint32_t full_parity = 0;
+    // This lane's row in buffer 0 as a 32-bit shared address, its first
+    // chunk and the 128-byte swizzle folded in (group_at, fp32).
+    const uint32_t lane_sa =
+        smem_addr(my_buf) + (uint32_t)(brow * kRowBytes) + ((uint32_t)(first_chunk ^ sw) << 4);
     bool live = true;
     // The consumer's next chunk: the one the prefetcher took after the
     // current one; once the prefetcher has stopped (a timeout) the consumer
@@ -373,9 +394,17 @@ __global__ void __launch_bounds__(kTmaThreads, kTmaCtas)
         float acc_hi = 0.0f, acc_lo = 0.0f;
         float sq_hi = 0.0f, sq_lo = 0.0f;
         int runP = 0, runC = 0;
-        for (int buf_off = 0; buf_off < span; buf_off += kBufCoords) {
-            // live stays warp-uniform: the refill below is a warp-wide step.
-            live = __all_sync(0xFFFFFFFFu, live && !*abort_flag);
+        // live stays warp-uniform: the refill below is a warp-wide step.  Another
+        // warp's abort is seen at the next chunk (a warp whose own wait runs
+        // out stops at once).
+        live = __all_sync(0xFFFFFFFFu, live && !*abort_flag);
+        // A whole chunk: every lane's 32 coordinates lie inside it in every
+        // buffer, i.e. its first row starts at the chunk and its length is a
+        // whole number of buffers (then lo is a multiple of 4 and the lane's
+        // first group is lo / 4 + buf_off / 4 + 8 lane).
+        const bool whole = lead == 0 && span == len && len % kBufCoords == 0;
+        uint32_t qw = (uint32_t)(lo >> 2) + (uint32_t)(lane_off >> 2);
+        for (int buf_off = 0; buf_off < span; buf_off += kBufCoords, qw += kBufCoords / 4) {
             if (live) {
                 live = __all_sync(0xFFFFFFFFu, mbar_wait(&my_full[slot], full_parity));
                 if (live) {
@@ -389,18 +418,19 @@ __global__ void __launch_bounds__(kTmaThreads, kTmaCtas)
             const int rel = buf_off + lane_off - lead;      // chunk-relative index of coordinate 0
             uint32_t pm = 0, cm = 0;
             float s32 = 0.0f, q32 = 0.0f;
-            if (live && rel < len && rel + kLaneCoords > 0) {
-                const uint32_t q0 = (uint32_t)((lo + rel) >> 2);   // worker-local group of coordinate 0
-                if (rel >= 0 && rel + kLaneCoords <= len) {
+            if (live && (whole || (rel < len && rel + kLaneCoords > 0))) {
+                const uint32_t q0 = whole ? qw : (uint32_t)((lo + rel) >> 2);   // worker-local group of coordinate 0
+                if (whole || (rel >= 0 && rel + kLaneCoords <= len)) {
                     // All 32 coordinates belong to the chunk: groups of 4 in order,
                     // the l1 (and square) sums accumulated group by group.
                     if constexpr (!kSq && !GS_TMA_PAIR) {
 #if GS_TMA_SR
                         uint64_t m0 = (uint64_t)0xD2511F53u * (uint64_t)q0;   // round 1's product, carried
 #endif
+                        const uint32_t bsa = lane_sa + (uint32_t)(slot * kBufBytes);   // this buffer's row, swizzle folded in
 #pragma unroll
                         for (int j = 0; j < 8; ++j) {
-                            const float4 a = stage_group<kDtype>(rp, first_chunk, sw, j);
+                            const float4 a = group_at<kDtype>(bsa, rp, first_chunk, sw, j);
                             s32 += abs_sum4(a);
                             if (build_p) {
 #if GS_TMA_SR
@@ -418,10 +448,11 @@ __global__ void __launch_bounds__(kTmaThreads, kTmaCtas)
                     } else {
                         // Two groups per step (independent Philox chains) pays in the
                         // instantiation that also sums squares.
+                        const uint32_t bsa = lane_sa + (uint32_t)(slot * kBufBytes);
 #pragma unroll
                         for (int j = 0; j < 8; j += 2) {
-                            const float4 a = stage_group<kDtype>(rp, first_chunk, sw, j);
-                            const float4 b = stage_group<kDtype>(rp, first_chunk, sw, j + 1);
+                            const float4 a = group_at<kDtype>(bsa, rp, first_chunk, sw, j);
+                            const float4 b = group_at<kDtype>(bsa, rp, first_chunk, sw, j + 1);
                             s32 += abs_sum4(a) + abs_sum4(b);
                             if (kSq) q32 += abs_sq4(a) + abs_sq4(b);
                             if (build_p) {
