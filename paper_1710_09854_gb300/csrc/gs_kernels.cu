@@ -360,13 +360,14 @@ __device__ __forceinline__ float4 block_sum3f(float a, float b, float c, float4*
 constexpr int kBoundCTAs = 8;
 constexpr int kBoundCtaThreads = 1024;
 constexpr int kBoundRun = 8;             // consecutive coordinates read per stratum
+constexpr int kBoundWarpMax = 1024;      // samples up to which warp 0 alone runs the fixed point
 
 // One thread-block cluster of kCTAs CTAs per segment (kBoundCTAs, or one for
 // layer-wise calls): the CTAs share the sample's random loads and store the
 // |g| values straight into rank 0's shared memory (DSMEM); rank 0 then runs
 // Algorithm 3 to its fixed point on the sample alone, with block-wide sums.
 template <int kCTAs>
-__global__ void __cluster_dims__(kCTAs, 1, 1) __launch_bounds__(kBoundCtaThreads)
+__global__ void __cluster_dims__(kCTAs, 1, 1) __launch_bounds__(kBoundCtaThreads, 2)
     k_bound(Layout Lo, SegParam* sp, double kappa, int ns, int force_exact) {
     grid_dep_wait();
     // The streaming pass may launch now: it only loads g (an input of the
@@ -374,7 +375,7 @@ __global__ void __cluster_dims__(kCTAs, 1, 1) __launch_bounds__(kBoundCtaThreads
     grid_dep_launch();
     namespace cg = cooperative_groups;
     cg::cluster_group cluster = cg::this_cluster();
-    extern __shared__ float sa[];               // rank 0: all ns samples
+    extern __shared__ __align__(16) float sa[];   // rank 0: all ns samples
     __shared__ float2 sh2[33];
     __shared__ float4 sh4[33];
     const int rank = (int)cluster.block_rank();
@@ -418,26 +419,61 @@ __global__ void __cluster_dims__(kCTAs, 1, 1) __launch_bounds__(kBoundCtaThreads
     const int64_t q = whole ? 1 : len / nst;                        // stratum width (the last one takes the rest)
     const int64_t q_last = whole ? 1 : len - (int64_t)(nst - 1) * q;
     const uint32_t hs = mix32((uint32_t)s + 0x68E31DA4u);
-    for (int e = tid; e < per * kBoundRun; e += kBoundCtaThreads) {
-        const int k = rank * per + e / kBoundRun;                   // stratum
-        const int r = e % kBoundRun;
+    // One thread per stratum: its run's start is found once, and a run that
+    // lies inside the segment on a 16-byte grid is read with vector loads
+    // (its flat start is a multiple of kBoundRun = 8 elements).
+    const bool vec = (reinterpret_cast<uintptr_t>(Lo.g) & 15u) == 0;
+    for (int kk = tid; kk < per; kk += kBoundCtaThreads) {
+        const int k = rank * per + kk;                              // stratum
         const uint32_t h = mix32((uint32_t)k * 0x9E3779B9u ^ hs);
         const int64_t width = k == nst - 1 ? q_last : q;            // >= kBoundRun since len > ns
         const int64_t runs = width / kBoundRun;
         int64_t start = lo + (int64_t)k * q + (int64_t)(h % (uint32_t)runs) * kBoundRun;
         start -= (start + (int64_t)m * Lo.d) % kBoundRun;           // align the run to the flat index
         if (start < lo + (int64_t)k * q) start += kBoundRun;
-        const int64_t pos = min(start + r, hi - 1);
-        float x = fabsf(load_one(Lo, m, pos));
-        if (!(x < kInf)) x = 0.0f;  // non-finite values are reported by the solve
-        dst[k * kBoundRun + r] = x;
+        float x[kBoundRun];
+        if (vec && start + kBoundRun <= hi) {
+            const int64_t flat = (int64_t)m * Lo.d + start;
+            if (Lo.dtype == 0) {
+                const float4* p4 = reinterpret_cast<const float4*>(static_cast<const float*>(Lo.g) + flat);
+                const float4 a = p4[0], b = p4[1];
+                x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w;
+                x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
+            } else {
+                const uint4 t = *reinterpret_cast<const uint4*>(static_cast<const uint16_t*>(Lo.g) + flat);
+                const uint32_t w4[4] = {t.x, t.y, t.z, t.w};
+#pragma unroll
+                for (int r = 0; r < 4; ++r) {
+                    x[2 * r] = bf16_bits_to_float(w4[r] & 0xFFFFu);
+                    x[2 * r + 1] = bf16_bits_to_float(w4[r] >> 16);
+                }
+            }
+        } else {
+#pragma unroll
+            for (int r = 0; r < kBoundRun; ++r) x[r] = load_one(Lo, m, min(start + r, hi - 1));
+        }
+#pragma unroll
+        for (int r = 0; r < kBoundRun; ++r) {
+            float a = fabsf(x[r]);
+            if (!(a < kInf)) a = 0.0f;  // non-finite values are reported by the solve
+            x[r] = a;
+        }
+        float4* d4 = reinterpret_cast<float4*>(dst + (size_t)k * kBoundRun);
+        d4[0] = make_float4(x[0], x[1], x[2], x[3]);
+        d4[1] = make_float4(x[4], x[5], x[6], x[7]);
     }
     cluster.sync();   // the sample is complete in rank 0; nobody touches another CTA's memory after this
     if (rank != 0) return;
 
+    // A sample of at most 1024 values (a short segment taken whole) is
+    // iterated by warp 0 alone with shuffle sums: no block barrier per
+    // iteration.  The other warps leave; nothing below waits for them.
+    const bool one_warp = ns <= kBoundWarpMax;
+    if (one_warp && tid >= 32) return;
+    const int nthr = one_warp ? 32 : kBoundCtaThreads;
     float ls = 0.0f;
-    for (int k = tid; k < ns; k += kBoundCtaThreads) ls += sa[k];
-    const float S = block_sum2f(ls, 0.0f, sh2).x;
+    for (int k = tid; k < ns; k += nthr) ls += sa[k];
+    const float S = one_warp ? warp_sum(ls) : block_sum2f(ls, 0.0f, sh2).x;
     const float budget = (float)(kappa * (double)ns);
     float lam = S > 0.0f ? budget / S : 0.0f;
     float K = 0.0f, Su = S;
@@ -446,11 +482,12 @@ __global__ void __cluster_dims__(kCTAs, 1, 1) __launch_bounds__(kBoundCtaThreads
     for (int it = 0; it < 32 && !take_all; ++it) {
         const float acap = 1.0f / lam;
         float su = 0.0f, kc = 0.0f, sq = 0.0f;
-        for (int k = tid; k < ns; k += kBoundCtaThreads) {
+        for (int k = tid; k < ns; k += nthr) {
             const float x = sa[k];
             if (x >= acap) kc += 1.0f; else { su += x; sq += x * x; }
         }
-        const float4 r = block_sum3f(kc, su, sq, sh4);
+        const float4 r = one_warp ? make_float4(warp_sum(kc), warp_sum(su), warp_sum(sq), 0.0f)
+                                  : block_sum3f(kc, su, sq, sh4);
         K = r.x;
         Su = r.y;
         Sq = r.z;
