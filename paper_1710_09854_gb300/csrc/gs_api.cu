@@ -26,6 +26,8 @@ constexpr int64_t kMaxD = (int64_t)1 << 31;
 struct SegMeta {
     int64_t* off = nullptr;     // device [L+1]
     int32_t* chunk0 = nullptr;  // device [L+1]
+    int32_t* bnd = nullptr;     // device [L]: long segments (> bound_short_max()), then short ones
+    int bnd_long = 0;
     int cpw = 0;
 };
 
@@ -122,12 +124,23 @@ gs_status segment_meta(DevState* s, const int64_t* off, int L, SegMeta* out) {
     }
     c0[L] = (int32_t)acc;
     if (acc > INT32_MAX) return GS_ERR_INVALID_ARG;
+    // The bound pass's order: one CTA for each long segment, then warps for
+    // the short ones (each in index order).
+    std::vector<int32_t> bnd;
+    for (int l = 0; l < L; ++l)
+        if (off[l + 1] - off[l] > bound_short_max()) bnd.push_back(l);
+    const int n_long = (int)bnd.size();
+    for (int l = 0; l < L; ++l)
+        if (off[l + 1] - off[l] <= bound_short_max()) bnd.push_back(l);
     SegMeta m;
     m.cpw = (int)acc;
+    m.bnd_long = n_long;
     GS_TRY(cudaMalloc(&m.off, sizeof(int64_t) * (L + 1)));
     GS_TRY(cudaMalloc(&m.chunk0, sizeof(int32_t) * (L + 1)));
+    GS_TRY(cudaMalloc(&m.bnd, sizeof(int32_t) * L));
     GS_TRY(cudaMemcpy(m.off, off, sizeof(int64_t) * (L + 1), cudaMemcpyHostToDevice));
     GS_TRY(cudaMemcpy(m.chunk0, c0.data(), sizeof(int32_t) * (L + 1), cudaMemcpyHostToDevice));
+    GS_TRY(cudaMemcpy(m.bnd, bnd.data(), sizeof(int32_t) * L, cudaMemcpyHostToDevice));
     if (s->segs.size() >= 32) s->segs.clear();  // bounded cache (device tables are tiny; kept until exit)
     s->segs[key] = m;
     *out = m;
@@ -259,6 +272,8 @@ gs_status run(const void* g, int dtype, int M, int64_t d, const int64_t* seg_off
         if (rc != GS_OK) return rc;
         Lo.seg_off = meta.off;
         Lo.seg_chunk0 = meta.chunk0;
+        Lo.bnd_seg = meta.bnd;
+        Lo.bnd_long = meta.bnd_long;
         Lo.cpw = meta.cpw;
     }
     int64_t max_seg_len = d;   // the longest segment (sizes the solve's shared memory)

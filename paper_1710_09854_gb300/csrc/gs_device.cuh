@@ -52,6 +52,9 @@ struct Layout {
     int64_t d;
     const int64_t* seg_off;   // [L+1] local offsets; NULL when L == 1
     const int32_t* seg_chunk0;// [L+1] first chunk (within a worker) of each segment; NULL when L == 1
+    const int32_t* bnd_seg;   // [L] the bound's segment order: those longer than kBoundWarpMax values
+                              // first, then the short ones; NULL when L == 1
+    int bnd_long;             // how many of bnd_seg are long
     uint64_t seed;
     uint32_t step;
     uint32_t worker0;

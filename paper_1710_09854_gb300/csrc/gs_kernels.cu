@@ -362,13 +362,91 @@ constexpr int kBoundCtaThreads = 1024;
 constexpr int kBoundRun = 8;             // consecutive coordinates read per stratum
 constexpr int kBoundWarpMax = 1024;      // samples up to which warp 0 alone runs the fixed point
 
+// Algorithm 3 run to its fixed point (in fp32) on a sample of |g| in shared
+// memory, and the upper bound on lambda it gives, written to the segment's
+// parameters by thread t == 0.  kWarp: one warp alone (t = lane, shuffle
+// sums); else the whole CTA (t = tid, block sums).  whole: the sample is the
+// whole segment (the fixed point is then Algorithm 3 itself, whose iterates
+// never pass it, so a 1% margin covers the fp32 rounding).
+template <bool kWarp>
+__device__ __forceinline__ void bound_from_sample(SegParam& P, const float* sa, int ns, double kappa, bool whole,
+                                                  int t, float2* sh2, float4* sh4) {
+    const int nthr = kWarp ? 32 : (int)blockDim.x;
+    float ls = 0.0f;
+    for (int k = t; k < ns; k += nthr) ls += sa[k];
+    const float S = kWarp ? warp_sum(ls) : block_sum2f(ls, 0.0f, sh2).x;
+    const float budget = (float)(kappa * (double)ns);
+    float lam = S > 0.0f ? budget / S : 0.0f;
+    float K = 0.0f, Su = S;
+    bool take_all = !(S > 0.0f) || !(lam < kInf);
+    float Sq = 0.0f;   // sum of squares of the uncapped sample values (for the margin)
+    for (int it = 0; it < 32 && !take_all; ++it) {
+        const float acap = 1.0f / lam;
+        float su = 0.0f, kc = 0.0f, sq = 0.0f;
+        for (int k = t; k < ns; k += nthr) {
+            const float x = sa[k];
+            if (x >= acap) kc += 1.0f; else { su += x; sq += x * x; }
+        }
+        const float4 r = kWarp ? make_float4(warp_sum(kc), warp_sum(su), warp_sum(sq), 0.0f)
+                               : block_sum3f(kc, su, sq, sh4);
+        K = r.x;
+        Su = r.y;
+        Sq = r.z;
+        if (!(Su > 0.0f)) { take_all = true; break; }
+        const float c = (budget - K) / (lam * Su);
+        if (!(c > 1.0f + 1e-5f)) break;
+        lam *= c;
+    }
+    if (t == 0) {
+        P.done = 0;
+        P.w_done = 0;
+        P.next_chunk = 0;
+        const float e = take_all ? 0.0f : lam * Su / budget;  // uncapped share of the budget
+        if (take_all || K >= budget || !(lam > 0.0f)) {
+            P.lam_up = (double)kInf;
+            P.lam_up32 = kInf;
+            P.t_c = 0.0f;
+            P.flags = kSegTakeAll;
+        } else {
+            // A count-based bound on the sample's error, tightened by the sample's
+            // own spread: lambda = (kappa d - K) / S_u at the fixed point, so its
+            // relative error is about that of S_u (std of a sum of the
+            // uncapped values) and of kappa d - K (binomial K).  A sample that
+            // caught large values also has a large spread, which keeps the bound
+            // safe for heavy tails; a violated bound only costs the exact fallback.
+            // (fp32 throughout: a heuristic, and fp64 is slow on this part)
+            const float kns = (float)kappa * (float)ns;
+            float margin = 1.0f + (float)kBoundZ * rsqrtf(kns) / fmaxf(e, 1.0f / 16.0f);
+            const float nu = (float)ns - K;
+            if (nu > 1.0f && Su > 0.0f && isfinite(Sq)) {
+                const float mean = Su / nu;
+                const float var = fmaxf(Sq / nu - mean * mean, 0.0f);
+                const float rel_s = sqrtf(var * nu) / Su;
+                const float room = kns - K;
+                const float rel_k = room > 0.0f ? sqrtf(K) / room : 1.0f;
+                margin = fminf(margin, 1.0f + fmaxf((float)kBoundFloor,
+                                                    (float)kBoundZs * sqrtf(rel_s * rel_s + rel_k * rel_k)));
+            }
+            margin = fminf(margin, 64.0f);
+            if (whole) margin = 1.01f;
+            // lam_up32 rounded up and t_c rounded down keep both lists supersets;
+            // the fp64 bound is lam_up32 itself.
+            const float up32 = __fmul_ru(lam, margin);
+            P.lam_up32 = up32;
+            P.lam_up = (double)up32;
+            P.t_c = __fmul_rd(__frcp_rd(up32), 1.0f - 0x1p-20f);
+            P.flags = 0;
+        }
+    }
+}
+
 // One thread-block cluster of kCTAs CTAs per segment (kBoundCTAs, or one for
 // layer-wise calls): the CTAs share the sample's random loads and store the
 // |g| values straight into rank 0's shared memory (DSMEM); rank 0 then runs
 // Algorithm 3 to its fixed point on the sample alone, with block-wide sums.
 template <int kCTAs>
 __global__ void __cluster_dims__(kCTAs, 1, 1) __launch_bounds__(kBoundCtaThreads, 2)
-    k_bound(Layout Lo, SegParam* sp, double kappa, int ns, int force_exact) {
+    k_bound(Layout Lo, SegParam* sp, double kappa, int ns, int force_exact, int short_per_cta) {
     grid_dep_wait();
     // The streaming pass may launch now: it only loads g (an input of the
     // call) until its own wait for this grid.
@@ -379,7 +457,47 @@ __global__ void __cluster_dims__(kCTAs, 1, 1) __launch_bounds__(kBoundCtaThreads
     __shared__ float2 sh2[33];
     __shared__ float4 sh4[33];
     const int rank = (int)cluster.block_rank();
-    const int s = blockIdx.x / kCTAs, tid = threadIdx.x;
+    const int tid = threadIdx.x;
+    int s = blockIdx.x / kCTAs;
+    if (kCTAs == 1 && short_per_cta > 0) {
+        // Layer-wise calls: a CTA for each worker's copy of each long segment
+        // (bnd_seg's first bnd_long), then short_per_cta short segments (at
+        // most kBoundWarpMax values) to a CTA, one per warp, each taken whole
+        // into the warp's own slice of shared memory.
+        const int n_long = Lo.M * Lo.bnd_long;
+        if (s < n_long) {
+            s = (s % Lo.M) * Lo.L + Lo.bnd_seg[s / Lo.M];
+        } else {
+            const int w = tid >> 5, lane = tid & 31;
+            const int t = (s - n_long) * short_per_cta + w;
+            if (w >= short_per_cta || t >= Lo.M * (Lo.L - Lo.bnd_long)) return;
+            const int ss = (t % Lo.M) * Lo.L + Lo.bnd_seg[Lo.bnd_long + t / Lo.M];
+            int m, l, c0, c1;
+            int64_t lo, hi;
+            seg_range(Lo, ss, m, l, lo, hi, c0, c1);
+            const int len = (int)(hi - lo);
+            SegParam& Q = sp[ss];
+            float* ws = sa + w * kBoundWarpMax;
+            if (!force_exact) {
+                for (int e = lane; e < len; e += 32) {
+                    float x = fabsf(load_one(Lo, m, lo + e));
+                    if (!(x < kInf)) x = 0.0f;  // non-finite values are reported by the solve
+                    ws[e] = x;
+                }
+                __syncwarp();
+                bound_from_sample<true>(Q, ws, len, kappa, true, lane, sh2, sh4);
+            } else if (lane == 0) {
+                Q.done = 0;
+                Q.w_done = 0;
+                Q.next_chunk = 0;
+                Q.lam_up = (double)kInf;
+                Q.lam_up32 = kInf;
+                Q.t_c = 0.0f;
+                Q.flags = kSegTakeAll;
+            }
+            return;
+        }
+    }
     int m, l, c0, c1;
     int64_t lo, hi;
     seg_range(Lo, s, m, l, lo, hi, c0, c1);
@@ -465,78 +583,14 @@ __global__ void __cluster_dims__(kCTAs, 1, 1) __launch_bounds__(kBoundCtaThreads
     cluster.sync();   // the sample is complete in rank 0; nobody touches another CTA's memory after this
     if (rank != 0) return;
 
-    // A sample of at most 1024 values (a short segment taken whole) is
-    // iterated by warp 0 alone with shuffle sums: no block barrier per
+    // A sample of at most kBoundWarpMax values (a short segment taken whole)
+    // is iterated by warp 0 alone with shuffle sums: no block barrier per
     // iteration.  The other warps leave; nothing below waits for them.
-    const bool one_warp = ns <= kBoundWarpMax;
-    if (one_warp && tid >= 32) return;
-    const int nthr = one_warp ? 32 : kBoundCtaThreads;
-    float ls = 0.0f;
-    for (int k = tid; k < ns; k += nthr) ls += sa[k];
-    const float S = one_warp ? warp_sum(ls) : block_sum2f(ls, 0.0f, sh2).x;
-    const float budget = (float)(kappa * (double)ns);
-    float lam = S > 0.0f ? budget / S : 0.0f;
-    float K = 0.0f, Su = S;
-    bool take_all = !(S > 0.0f) || !(lam < kInf);
-    float Sq = 0.0f;   // sum of squares of the uncapped sample values (for the margin)
-    for (int it = 0; it < 32 && !take_all; ++it) {
-        const float acap = 1.0f / lam;
-        float su = 0.0f, kc = 0.0f, sq = 0.0f;
-        for (int k = tid; k < ns; k += nthr) {
-            const float x = sa[k];
-            if (x >= acap) kc += 1.0f; else { su += x; sq += x * x; }
-        }
-        const float4 r = one_warp ? make_float4(warp_sum(kc), warp_sum(su), warp_sum(sq), 0.0f)
-                                  : block_sum3f(kc, su, sq, sh4);
-        K = r.x;
-        Su = r.y;
-        Sq = r.z;
-        if (!(Su > 0.0f)) { take_all = true; break; }
-        const float c = (budget - K) / (lam * Su);
-        if (!(c > 1.0f + 1e-5f)) break;
-        lam *= c;
+    if (ns <= kBoundWarpMax) {
+        if (tid < 32) bound_from_sample<true>(P, sa, ns, kappa, whole, tid, sh2, sh4);
+        return;
     }
-    if (tid == 0) {
-        P.done = 0;
-        P.w_done = 0;
-        P.next_chunk = 0;
-        const float e = take_all ? 0.0f : lam * Su / budget;  // uncapped share of the budget
-        if (take_all || K >= budget || !(lam > 0.0f)) {
-            P.lam_up = (double)kInf;
-            P.lam_up32 = kInf;
-            P.t_c = 0.0f;
-            P.flags = kSegTakeAll;
-        } else {
-            // A count-based bound on the sample's error, tightened by the sample's
-            // own spread: lambda = (kappa d - K) / S_u at the fixed point, so its
-            // relative error is about that of S_u (std of a sum of the
-            // uncapped values) and of kappa d - K (binomial K).  A sample that
-            // caught large values also has a large spread, which keeps the bound
-            // safe for heavy tails; a violated bound only costs the exact fallback.
-            // (fp32 throughout: a heuristic, and fp64 is slow on this part)
-            const float kns = (float)kappa * (float)ns;
-            float margin = 1.0f + (float)kBoundZ * rsqrtf(kns) / fmaxf(e, 1.0f / 16.0f);
-            const float nu = (float)ns - K;
-            if (nu > 1.0f && Su > 0.0f && isfinite(Sq)) {
-                const float mean = Su / nu;
-                const float var = fmaxf(Sq / nu - mean * mean, 0.0f);
-                const float rel_s = sqrtf(var * nu) / Su;
-                const float room = kns - K;
-                const float rel_k = room > 0.0f ? sqrtf(K) / room : 1.0f;
-                margin = fminf(margin, 1.0f + fmaxf((float)kBoundFloor,
-                                                    (float)kBoundZs * sqrtf(rel_s * rel_s + rel_k * rel_k)));
-            }
-            margin = fminf(margin, 64.0f);
-            if (whole) margin = 1.01f;
-            // lam_up32 rounded up and t_c rounded down keep both lists supersets;
-            // the fp64 bound is lam_up32 itself.
-            const float up32 = __fmul_ru(lam, margin);
-            P.lam_up32 = up32;
-            P.lam_up = (double)up32;
-            P.t_c = __fmul_rd(__frcp_rd(up32), 1.0f - 0x1p-20f);
-            P.flags = 0;
-        }
-    }
+    bound_from_sample<false>(P, sa, ns, kappa, whole, tid, sh2, sh4);
 }
 
 // ---------------------------------------------------------------------------
@@ -1533,9 +1587,16 @@ cudaError_t launch_bound(const Layout& Lo, SegParam* sp, int n_seg, double kappa
         cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess) return e;
     }
+    // Short segments of a layer-wise call share CTAs, a warp each, when the
+    // sample buffer holds at least one short segment per warp slice.
+    int grid = n_seg * (one ? 1 : kBoundCTAs), per = 0;
+    if (one && Lo.bnd_seg != nullptr && n_seg == Lo.M * Lo.L && ns >= kBoundWarpMax) {
+        per = std::min(kBoundCtaThreads / 32, ns / kBoundWarpMax);
+        const int n_short = Lo.M * (Lo.L - Lo.bnd_long);
+        grid = Lo.M * Lo.bnd_long + (n_short + per - 1) / per;
+    }
     TraceScope ts(kKBound, st);
-    return launch_dep(kern, dim3(n_seg * (one ? 1 : kBoundCTAs)), dim3(kBoundCtaThreads), smem, st, Lo, sp, kappa,
-                      ns, force_exact);
+    return launch_dep(kern, dim3(grid), dim3(kBoundCtaThreads), smem, st, Lo, sp, kappa, ns, force_exact, per);
 }
 
 cudaError_t launch_stream(const Layout& Lo, const SegParam* sp, const Lists& Ls, int n_chunks, bool build_p,
@@ -1644,5 +1705,6 @@ cudaError_t launch_aggregate(const AggArgs& A, int32_t* off, float* out, int* st
 
 int agg_tiles(int64_t d) { return (int)((d + kAggTile - 1) / kAggTile); }
 int chunk_size() { return kChunk; }
+int bound_short_max() { return kBoundWarpMax; }
 
 }  // namespace gs

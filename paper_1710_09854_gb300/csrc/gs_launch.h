@@ -148,6 +148,9 @@ void set_launch_error_site(const char* where);
 const char* launch_error_site();
 int agg_tiles(int64_t d);
 int chunk_size();
+// Segments of at most this many values get a warp of the layer-wise bound
+// pass instead of a CTA.
+int bound_short_max();
 // Multiprocessor count of the current device (looked up once per device ordinal).
 int device_sm_count();
 
