@@ -389,8 +389,10 @@ gs_status gs_random_words(uint64_t seed, uint32_t step, uint32_t worker, int64_t
  *   GS_OPT_FORCE_EXACT_SOLVE  1: skip the sampled bound and use the exact
  *                              fallback solve for every worker (slow).
  *   GS_OPT_SAMPLE_SIZE        sampled coordinates per segment for the bound
- *                              on lambda (default 16384; a multiple of 8 in
- *                              256 .. 32768).
+ *                              on lambda: a multiple of 8 in 256 .. 32768,
+ *                              or 0 (the default): 8192 when the call's
+ *                              longest segment has at most 2^25
+ *                              coordinates, 16384 when it is longer.
  *   GS_OPT_KERNEL_TIMING      1: time every kernel launch (gs_kernel_times);
  *                              2: time the streaming pass only (k_small on
  *                              the cluster path).  The events

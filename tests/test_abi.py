@@ -74,6 +74,7 @@ def test_host_argument_checks(gs):
     assert L.gs_set_option(gs.GS_OPT_SAMPLE_SIZE, 100) == inv
     assert L.gs_set_option(gs.GS_OPT_FORCE_EXACT_SOLVE, 2) == inv
     assert L.gs_set_option(gs.GS_OPT_SAMPLE_SIZE, 16384) == 0
+    assert L.gs_set_option(gs.GS_OPT_SAMPLE_SIZE, 0) == 0   # back to the automatic size
 
 
 def test_eps_entry_points_reject_bad_budgets():

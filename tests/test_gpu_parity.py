@@ -21,7 +21,7 @@ def gs():
     __graft_entry__.build()
     import paper_1710_09854_gb300 as gs
     gs.gs_set_option(gs.GS_OPT_FORCE_EXACT_SOLVE, 0)
-    gs.gs_set_option(gs.GS_OPT_SAMPLE_SIZE, 16384)
+    gs.gs_set_option(gs.GS_OPT_SAMPLE_SIZE, 0)
     assert gs.gs_sync_status() == gs.GS_OK
     return gs
 
@@ -191,7 +191,7 @@ def test_forced_exact_and_small_sample(gs):
             assert gs.gs_sync_status() == gs.GS_OK
         finally:
             gs.gs_set_option(gs.GS_OPT_FORCE_EXACT_SOLVE, 0)
-            gs.gs_set_option(gs.GS_OPT_SAMPLE_SIZE, 16384)
+            gs.gs_set_option(gs.GS_OPT_SAMPLE_SIZE, 0)
         n = nnz.cpu().numpy()
         for m in range(M):
             compare_sparse(idx[m, :n[m]].cpu().numpy(), v[m, :n[m]].cpu().numpy(), g_host[m], kappa, iters, 3, 2, m)
