@@ -50,28 +50,6 @@ namespace {
 #ifndef GS_TMA_RING_KIB
 #define GS_TMA_RING_KIB 96
 #endif
-// Form of the keep-candidate test (all three compute the same sign bit):
-// 0: shift, three-input add and funnel shift on the integer ALU; 1: the
-// constant minus the float bits by an integer multiply-add first; 2: the
-// shift folded into a multiply-high.
-#ifndef GS_TMA_CAND
-#define GS_TMA_CAND 0
-#endif
-// 1: the Algorithm 3 instantiation also takes two groups (two independent
-// Philox chains) per step, as the sum-of-squares one always does.
-#ifndef GS_TMA_PAIR
-#define GS_TMA_PAIR 0
-#endif
-// 1: round 1's product 0xD2511F53 * q of consecutive groups carried forward
-// by a 64-bit add (integer ALU) instead of a wide multiply each.
-#ifndef GS_TMA_SR
-#define GS_TMA_SR 1
-#endif
-// 1: lam_up |g| formed as |lam_up * g| (a multiply and an add that takes the
-// absolute value of its operand) instead of a fused multiply-add on |g|.
-#ifndef GS_TMA_ABS
-#define GS_TMA_ABS 0
-#endif
 constexpr int kCW = 8;                         // warps per CTA
 constexpr int kTmaThreads = 32 * kCW;
 constexpr int kTmaCtas = GS_TMA_CTAS;
@@ -169,24 +147,12 @@ __device__ __forceinline__ uint32_t shl_in(uint32_t m, float r) {
 // the difference).  (x >> 9) 2^-23 <= u = x 2^-32 and the rounding of the
 // right-hand side is below its 2^-20 slack, so every coordinate kept under a
 // lambda <= lam_up passes (NaN and Inf |g| pass too).
+// (A shift, a three-input add and, at the caller, a funnel shift on the
+// integer ALU: measured faster than forming the difference by integer
+// multiply-adds, which share the pipe with Philox's wide multiplies.)
 __device__ __forceinline__ float cand_sign(uint32_t x, float lam_up, float a, float pbias) {
-#if GS_TMA_ABS
-    const uint32_t pf = __float_as_uint(__fadd_rn(fabsf(__fmul_rn(lam_up, a)), pbias));
-#else
     const uint32_t pf = __float_as_uint(fmaf(lam_up, fabsf(a), pbias));
-#endif
-#if GS_TMA_CAND == 0
     return __uint_as_float((x >> 9) + 0x3F800000u - pf);
-#else
-    uint32_t c, r;
-    asm("mad.lo.u32 %0, %1, 4294967295, 1065353216;" : "=r"(c) : "r"(pf));   // 0x3F800000 - pf
-#if GS_TMA_CAND == 1
-    r = (x >> 9) + c;
-#else
-    asm("mad.hi.u32 %0, %1, 8388608, %2;" : "=r"(r) : "r"(x), "r"(c));      // (x >> 9) + c
-#endif
-    return __uint_as_float(r);
-#endif
 }
 
 // Coordinate k (0..31) of a lane's 32, read back from its row of the buffer
@@ -423,22 +389,19 @@ __global__ void __launch_bounds__(kTmaThreads, kTmaCtas)
                 if (whole || (rel >= 0 && rel + kLaneCoords <= len)) {
                     // All 32 coordinates belong to the chunk: groups of 4 in order,
                     // the l1 (and square) sums accumulated group by group.
-                    if constexpr (!kSq && !GS_TMA_PAIR) {
-#if GS_TMA_SR
-                        uint64_t m0 = (uint64_t)0xD2511F53u * (uint64_t)q0;   // round 1's product, carried
-#endif
+                    if constexpr (!kSq) {
+                        // Round 1's product 0xD2511F53 q of consecutive groups is
+                        // carried by a 64-bit add (integer ALU) instead of a wide
+                        // multiply per group.
+                        uint64_t m0 = (uint64_t)0xD2511F53u * (uint64_t)q0;
                         const uint32_t bsa = lane_sa + (uint32_t)(slot * kBufBytes);   // this buffer's row, swizzle folded in
 #pragma unroll
                         for (int j = 0; j < 8; ++j) {
                             const float4 a = group_at<kDtype>(bsa, rp, first_chunk, sw, j);
                             s32 += abs_sum4(a);
                             if (build_p) {
-#if GS_TMA_SR
                                 const uint4 w = ph.words_after(m0);
                                 m0 += 0xD2511F53u;
-#else
-                                const uint4 w = ph.words(q0 + j);
-#endif
                                 pm = shl_in(pm, cand_sign(w.x, lup, a.x, pbias));
                                 pm = shl_in(pm, cand_sign(w.y, lup, a.y, pbias));
                                 pm = shl_in(pm, cand_sign(w.z, lup, a.z, pbias));
@@ -447,7 +410,7 @@ __global__ void __launch_bounds__(kTmaThreads, kTmaCtas)
                         }
                     } else {
                         // Two groups per step (independent Philox chains) pays in the
-                        // instantiation that also sums squares.
+                        // instantiation that also sums squares (not in the one above).
                         const uint32_t bsa = lane_sa + (uint32_t)(slot * kBufBytes);
 #pragma unroll
                         for (int j = 0; j < 8; j += 2) {
