@@ -284,7 +284,7 @@ def run_gpu(args):
         "k_small": M * d * esz + nnz_total * 8 + (d * 4 if M == 1 else 0),
         "k_small_sum": M * d // 8 + nnz_total * esz + d * 4,   # decision bits, kept g, dense sum
         "k_emit": nnz_total * 8,                 # the (idx, val) codes written
-        "k_sum": nnz_total * 8 + d * 4,          # codes read, dense sum written
+        "k_emit_sum": 2 * nnz_total * 8 + d * 4,  # codes written, codes read, dense sum written
         "k_tiles": nnz_total * 8 + d * 4,        # codes read, dense sum written
     }
     kb = kernel_bytes.get(dom_name, 0)

@@ -197,8 +197,8 @@ void carve(Arena& a, Workspace& w, int n_seg, int n_chunks, int64_t n, bool buil
         w.ls.p_cnt = a.take<int32_t>(n_chunks);
         w.ls.k_sub = a.take<int32_t>((size_t)n_chunks * kSubStride);
         w.ls.k_off = a.take<int32_t>(n_chunks);
-        w.ls.e_bits = a.take<uint32_t>((size_t)n_chunks * (kChunk / 32));
         if (hybrid) {
+            w.ls.e_bits = a.take<uint32_t>((size_t)n_chunks * (kChunk / 32));   // the hybrid emit's decision bits
             w.ls.k_offa = a.take<int32_t>(n_chunks);
             w.nnz = a.take<int32_t>(M);
         }

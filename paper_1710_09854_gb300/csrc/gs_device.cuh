@@ -94,7 +94,7 @@ struct Lists {
     double* s_low;      // [n_chunks] sum of |g| outside C
     int32_t* k_off;     // [n_chunks] kept count of the chunk, then (after k_scan) the offset
                         // of its first kept entry in its worker's output
-    uint32_t* e_bits;   // [n_chunks][kChunk / 32] decision bit of every keep candidate
+    uint32_t* e_bits;   // [n_chunks][kChunk / 32] decision bit of every keep candidate (hybrid code only)
     int32_t* k_offa;    // [n_chunks] hybrid code only (else NULL): kept entries with p = 1, then their offsets
     int32_t* c_pre;     // [n_chunks + n_seg] prefix scratch for segments with many chunks
     double* b_low;      // [n_chunks] Algorithm 2 only (else NULL): sum of g^2 outside C

@@ -17,14 +17,16 @@
 //              final lambda exceeds lam_up the segment falls back to an exact
 //              multi-pass solve over g and rebuilds its P lists.
 //   k_decide   per (worker, chunk): the Bernoulli draw Z_i = [u_i < p_i]
-//              (section 3) on the P lists as decision bits and kept counts;
+//              (section 3) on the P lists; the kept entries, amplified to
+//              g_i / p_i, compacted in place over the chunk's P list (for
+//              the hybrid code: decision bits instead), and the kept counts;
 //              the last warp of each worker scans its counts into offsets.
-//   k_emit     per (worker, chunk): amplification to g_i / p_i and
-//              compaction into ascending (idx, val) (k_emit_hybrid: the
-//              hybrid code of section 3.3 instead);
-//   k_sum      per 1024-coordinate slice, for the fused calls: the
-//              worker-order fp32 sum of Algorithm 1 step 6 over the
-//              compacted rows.
+//   k_emit     per (worker, chunk): each chunk's compacted run copied to
+//              its place in the worker's ascending (idx, val) list
+//              (k_emit_hybrid: the hybrid code of section 3.3 instead);
+//   k_emit_sum for the fused calls, k_emit's work and, in the same launch,
+//              per 1024-coordinate slice the worker-order fp32 sum of
+//              Algorithm 1 step 6 over the compacted runs.
 //   k_bucket / k_tiles
 //              the worker-order fp32 sum of M arbitrary sparse vectors
 //              (Algorithm 1, step 6; gs_sparse_aggregate).
@@ -1079,10 +1081,13 @@ __global__ void __launch_bounds__(kEmitWarps * 32, kDecideBlocks) k_decide(const
     const Chunk ch = decode_chunk(Lo, c);
     const Decider dd = chunk_decider(sp[ch.seg]);
     const int n = Ls.p_cnt[c];
-    const int2* ent = Ls.p_ent + (int64_t)ch.m * Lo.d + ch.lo;
+    // The chunk's candidates; the plain lists' kept entries are compacted in
+    // place over them as (index, g_i / p_i) (a batch's candidates are all in
+    // registers before its writes, which land below the next batch).
+    int2* ent = Ls.p_ent + (int64_t)ch.m * Lo.d + ch.lo;
     const PhiloxStream ph(Lo, Lo.worker0 + (uint32_t)ch.m);
-    uint32_t* wb = Ls.e_bits + (size_t)c * kBitWords;
-    const bool hybrid = Ls.k_offa != nullptr;
+    const bool hybrid = Ls.k_offa != nullptr;   // the hybrid code's emit reads the decision bits instead
+    uint32_t* wb = hybrid ? Ls.e_bits + (size_t)c * kBitWords : nullptr;
     int32_t* ks = Ls.k_sub ? Ls.k_sub + (size_t)c * kSubStride : nullptr;   // only when a sum follows
     const int lo32 = (int)ch.lo;
     int cnt = 0;        // kept so far
@@ -1097,23 +1102,30 @@ __global__ void __launch_bounds__(kEmitWarps * 32, kDecideBlocks) k_decide(const
         }
         // The batch's decisions first (independent Philox chains), then its ballots.
         bool keep[kEmitBatch], capped[kEmitBatch];
+        float kv[kEmitBatch];   // the kept value g_i / p_i
 #pragma unroll
         for (int r = 0; r < kEmitBatch; ++r) {
             const int i = base + r * 32 + lane;
             const float gv = __int_as_float(e[r].y);
             capped[r] = i < n && fabsf(gv) >= dd.a_cap;   // p = 1: kept whatever the draw
             keep[r] = capped[r];
+            kv[r] = gv;
             if (i < n && !capped[r]) {
                 const uint32_t x = word_of(ph.words((uint32_t)e[r].x >> 2), e[r].x & 3);
                 float v;
                 keep[r] = dd(gv, x, v);
+                kv[r] = v;
             }
         }
 #pragma unroll
         for (int r = 0; r < kEmitBatch; ++r) {
             const uint32_t bal = __ballot_sync(0xFFFFFFFFu, keep[r]);
             if (base + r * 32 < n) {
-                if (lane == 0) wb[(base >> 5) + r] = bal;
+                if (hybrid) {
+                    if (lane == 0) wb[(base >> 5) + r] = bal;
+                } else if (keep[r]) {
+                    ent[cnt + __popc(bal & ((1u << lane) - 1u))] = make_int2(e[r].x, __float_as_int(kv[r]));
+                }
                 if (ks) {
                     // Candidates are in ascending order: a candidate that opens slices
                     // (prev, sub] records the kept count before it for each of them.
@@ -1164,52 +1176,45 @@ __global__ void __launch_bounds__(kEmitWarps * 32, kDecideBlocks) k_decide(const
     }
 }
 
-// The kept candidates of chunk c at their output positions, value g_i / p_i
-// (one warp; consecutive lanes write consecutive slots).
-__device__ __forceinline__ void emit_chunk(const Layout& Lo, const SegParam* __restrict__ sp, const Lists& Ls, int c,
+// The kept entries of chunk c, compacted in place by k_decide as (index,
+// g_i / p_i), copied to their output positions (one warp; consecutive lanes
+// write consecutive slots).  The chunk's count is the next chunk's offset
+// minus its own (the worker's total after its last chunk).
+__device__ __forceinline__ void emit_chunk(const Layout& Lo, const Lists& Ls, int c, const int32_t* nnz,
                                            int32_t* idx, float* val, int64_t cap) {
     const int lane = threadIdx.x & 31;
     const Chunk ch = decode_chunk(Lo, c);
-    const SegParam& P = sp[ch.seg];
-    const float a_cap = P.a_cap, inv_lam32 = P.inv_lam32;
-    const int n = Ls.p_cnt[c];
     const int2* ent = Ls.p_ent + (int64_t)ch.m * Lo.d + ch.lo;
-    const uint32_t* wb = Ls.e_bits + (size_t)c * kBitWords;
+    const long long pos0 = Ls.k_off[c];
+    const bool last = c - ch.m * Lo.cpw == Lo.cpw - 1;
+    const int n = (int)((last ? (long long)nnz[ch.m] : (long long)Ls.k_off[c + 1]) - pos0);
     const int64_t out0 = (int64_t)ch.m * cap;
-    long long pos0 = Ls.k_off[c];
     for (int base = 0; base < n; base += 32 * kEmitBatch) {
-        // All loads of kEmitBatch rounds first (candidates are ~all kept).
-        uint32_t wd[kEmitBatch];
         int2 en[kEmitBatch];
 #pragma unroll
         for (int r = 0; r < kEmitBatch; ++r) {
             const int i = base + r * 32 + lane;
-            wd[r] = base + r * 32 < n ? wb[(base >> 5) + r] : 0u;
             en[r] = i < n ? ent[i] : make_int2(0, 0);
         }
 #pragma unroll
         for (int r = 0; r < kEmitBatch; ++r) {
-            if ((wd[r] >> lane) & 1u) {
-                const float gv = __int_as_float(en[r].y);
-                const float v = fabsf(gv) >= a_cap ? gv : copysignf(inv_lam32, gv);
-                const long long pos = pos0 + __popc(wd[r] & ((1u << lane) - 1u));
-                if (pos < cap) {
-                    idx[out0 + pos] = en[r].x;
-                    val[out0 + pos] = v;
-                }
+            const int i = base + r * 32 + lane;
+            const long long pos = pos0 + i;
+            if (i < n && pos < cap) {
+                idx[out0 + pos] = en[r].x;
+                val[out0 + pos] = __int_as_float(en[r].y);
             }
-            pos0 += __popc(wd[r]);
         }
     }
 }
 
 __global__ void __launch_bounds__(kEmitWarps * 32) k_emit(const __grid_constant__ Layout Lo,
-                                                          const SegParam* __restrict__ sp,
                                                           const __grid_constant__ Lists Ls, int n_chunks,
-                                                          int32_t* idx, float* val, int64_t cap) {
+                                                          const int32_t* nnz, int32_t* idx, float* val,
+                                                          int64_t cap) {
     grid_dep_wait();
     const int c = blockIdx.x * kEmitWarps + (threadIdx.x >> 5);
-    if (c < n_chunks) emit_chunk(Lo, sp, Ls, c, idx, val, cap);
+    if (c < n_chunks) emit_chunk(Lo, Ls, c, nnz, idx, val, cap);
 }
 
 // The hybrid code of section 3.3 (eqs. 9-10) straight from the decisions: a
@@ -1267,27 +1272,21 @@ __global__ void __launch_bounds__(kEmitWarps * 32) k_emit_hybrid(const __grid_co
 }
 
 // ---------------------------------------------------------------------------
-// k_sum: the sparse sum of Algorithm 1, step 6 over the compacted rows (L == 1),
-// one warp per 1024-coordinate slice.  The slice's entries of worker m are one
-// contiguous run of m's list (k_decide recorded where each slice starts), so
-// a warp gathers the runs of all workers (lane i takes entry i of a run),
-// adds them into a private shared-memory tile worker by worker (a worker's
-// entries have distinct indices; __syncwarp separates workers) and writes
-// the slice once.
+// The sparse sum of Algorithm 1, step 6 over the kept entries, one warp per
+// 1024-coordinate slice.  The slice's entries of worker m are one contiguous
+// run of m's chunk, compacted in place by k_decide (which recorded where each
+// slice starts), so a warp gathers the runs of all workers (lane i takes
+// entry i of a run), adds them into a private shared-memory tile worker by
+// worker (a worker's entries have distinct indices; __syncwarp separates
+// workers) and writes the slice once.  Entries past a worker's output
+// capacity (which k_emit leaves out) are left out of the sum too.
 // ---------------------------------------------------------------------------
 constexpr int kSumWarps = 8;
 constexpr int kSumGroup = 8;                  // workers whose entries are loaded together
 
-__global__ void __launch_bounds__(kSumWarps * 32) k_sum(const __grid_constant__ Layout Lo,
-                                                        const __grid_constant__ Lists Ls,
-                                                        const int32_t* __restrict__ idx,
-                                                        const float* __restrict__ val, int64_t cap,
-                                                        int n_slices, float div, int accumulate, float* out) {
-    grid_dep_wait();
-    __shared__ __align__(16) float tile[kSumWarps][kSlice];
-    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    const int gs = blockIdx.x * kSumWarps + w;
-    if (gs >= n_slices) return;
+__device__ __forceinline__ void sum_slice(const Layout& Lo, const Lists& Ls, int64_t cap, int gs, float div,
+                                          int accumulate, float* out, float* acc) {
+    const int lane = threadIdx.x & 31;
     const int k = gs / kSlices, sl = gs - k * kSlices;
     // Chunk k covers the same coordinates in every worker row (also for
     // layer-wise layouts, whose chunks start at segment starts).
@@ -1295,7 +1294,6 @@ __global__ void __launch_bounds__(kSumWarps * 32) k_sum(const __grid_constant__ 
     const int64_t t0 = ch.lo + (int64_t)sl * kSlice;
     if (t0 >= ch.hi) return;
     const int tlen = (int)min((int64_t)kSlice, ch.hi - t0);
-    float* acc = tile[w];
     if (accumulate) {
         // Continue a worker-order sum already in out (the earlier workers' part).
         for (int i = lane; i < kSlice; i += 32) acc[i] = i < tlen ? out[t0 + i] : 0.0f;
@@ -1313,11 +1311,11 @@ __global__ void __launch_bounds__(kSumWarps * 32) k_sum(const __grid_constant__ 
         if (lane < nq) {
             const int c = (mb + lane) * Lo.cpw + k;
             const int32_t* ks = Ls.k_sub + (size_t)c * kSubStride;
-            const long long o = Ls.k_off[c];
-            long long lo_ = o + ks[sl], hi_ = o + ks[sl + 1];
-            lo_ = lo_ > cap ? cap : lo_;
-            hi_ = hi_ > cap ? cap : hi_;
-            a = (long long)(mb + lane) * cap + lo_;
+            const long long room = cap - (long long)Ls.k_off[c];   // entries of the chunk that were emitted
+            long long lo_ = ks[sl], hi_ = ks[sl + 1];
+            lo_ = lo_ > room ? room : lo_;
+            hi_ = hi_ > room ? room : hi_;
+            a = (long long)(mb + lane) * Lo.d + ch.lo + lo_;
             cnt = hi_ > lo_ ? (int)(hi_ - lo_) : 0;
         }
         int maxc = cnt;
@@ -1338,8 +1336,9 @@ __global__ void __launch_bounds__(kSumWarps * 32) k_sum(const __grid_constant__ 
                     jj[u] = -1;
                     vv[u] = 0.0f;
                     if (q < nq && lane < cq) {
-                        const int j = (int)((int64_t)idx[aq + lane] - t0);
-                        vv[u] = val[aq + lane];
+                        const int2 en = Ls.p_ent[aq + lane];
+                        const int j = (int)((int64_t)en.x - t0);
+                        vv[u] = __int_as_float(en.y);
                         if ((unsigned)j < (unsigned)tlen) jj[u] = j;   // always, for well-formed lists
                     }
                 }
@@ -1364,8 +1363,9 @@ __global__ void __launch_bounds__(kSumWarps * 32) k_sum(const __grid_constant__ 
                         jj[u] = -1;
                         vv[u] = 0.0f;
                         if (e < cq) {
-                            const int j = (int)((int64_t)idx[aq + e] - t0);
-                            vv[u] = val[aq + e];
+                            const int2 en = Ls.p_ent[aq + e];
+                            const int j = (int)((int64_t)en.x - t0);
+                            vv[u] = __int_as_float(en.y);
                             if ((unsigned)j < (unsigned)tlen) jj[u] = j;
                         }
                     }
@@ -1408,6 +1408,37 @@ __global__ void __launch_bounds__(kSumWarps * 32) k_sum(const __grid_constant__ 
         }
     } else {
         for (int i = lane; i < tlen; i += 32) dst[i] = div > 0.0f ? __fdiv_rn(acc[i], div) : acc[i];
+    }
+}
+
+// Emit and sum in one launch: both read what k_decide wrote and neither reads
+// the other's output, so their CTAs run side by side (alternating, the
+// longer role's surplus last).
+__global__ void __launch_bounds__(kEmitWarps * 32) k_emit_sum(const __grid_constant__ Layout Lo,
+                                                              const __grid_constant__ Lists Ls, int n_chunks,
+                                                              const int32_t* nnz, int32_t* idx, float* val,
+                                                              int64_t cap, int n_slices, float div, int accumulate,
+                                                              float* out, int n_emit_blocks, int n_sum_blocks) {
+    grid_dep_wait();
+    static_assert(kEmitWarps == kSumWarps, "one block shape for both roles");
+    __shared__ __align__(16) float tile[kSumWarps][kSlice];
+    const int w = threadIdx.x >> 5;
+    const int b = blockIdx.x, pairs = min(n_emit_blocks, n_sum_blocks);
+    bool emit;
+    int rb;
+    if (b < 2 * pairs) {
+        emit = (b & 1) == 0;
+        rb = b >> 1;
+    } else {
+        emit = n_emit_blocks > n_sum_blocks;
+        rb = pairs + (b - 2 * pairs);
+    }
+    if (emit) {
+        const int c = rb * kEmitWarps + w;
+        if (c < n_chunks) emit_chunk(Lo, Ls, c, nnz, idx, val, cap);
+    } else {
+        const int gs = rb * kSumWarps + w;
+        if (gs < n_slices) sum_slice(Lo, Ls, cap, gs, div, accumulate, out, tile[w]);
     }
 }
 
@@ -1653,19 +1684,21 @@ cudaError_t launch_compact(const Layout& Lo, const SegParam* sp, const Lists& Ls
         return launch_dep(k_emit_hybrid, dim3(blocks), dim3(kEmitWarps * 32), 0, st, Lo, sp, Ls, n_chunks, *hybrid,
                           cap);
     }
-    {
+    if (!sum_out) {
         set_launch_error_site("k_emit launch");
         TraceScope ts(kKEmit, st);
-        e = launch_dep(k_emit, dim3(blocks), dim3(kEmitWarps * 32), 0, st, Lo, sp, Ls, n_chunks, idx, val, cap);
+        return launch_dep(k_emit, dim3(blocks), dim3(kEmitWarps * 32), 0, st, Lo, Ls, n_chunks,
+                          static_cast<const int32_t*>(nnz), idx, val, cap);
     }
-    if (e != cudaSuccess || !sum_out) return e;
-    // The sparse sum of the M compacted rows, one warp per slice.
+    // The output lists and the sparse sum of the M rows (one warp per slice),
+    // side by side in one launch.
     const int n_slices = Lo.cpw * kSlices;
-    set_launch_error_site("k_sum launch");
-    TraceScope ts(kKSum, st);
-    return launch_dep(k_sum, dim3((n_slices + kSumWarps - 1) / kSumWarps), dim3(kSumWarps * 32), 0, st, Lo, Ls,
-                      static_cast<const int32_t*>(idx), static_cast<const float*>(val), cap, n_slices,
-                      average ? (float)Lo.M : 0.0f, accumulate ? 1 : 0, sum_out);
+    const int sblocks = (n_slices + kSumWarps - 1) / kSumWarps;
+    set_launch_error_site("k_emit_sum launch");
+    TraceScope ts(kKEmitSum, st);
+    return launch_dep(k_emit_sum, dim3(blocks + sblocks), dim3(kEmitWarps * 32), 0, st, Lo, Ls, n_chunks,
+                      static_cast<const int32_t*>(nnz), idx, val, cap, n_slices, average ? (float)Lo.M : 0.0f,
+                      accumulate ? 1 : 0, sum_out, blocks, sblocks);
 }
 
 cudaError_t launch_prob(const Layout& Lo, const SegParam* sp, float* p, cudaStream_t st) {

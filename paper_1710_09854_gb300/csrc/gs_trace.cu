@@ -18,7 +18,7 @@ const char* kNames[kNumKernels] = {"k_bound", "k_stream", "k_solve", "k_emit",
                                    "k_eps_hist", "k_eps_bracket", "k_solve_eps",
                                    "k_lr_grad", "k_lr_margins", "k_row_sq", "k_sum_rows", "k_sgd_step",
                                    "k_dense_count", "k_dense_merge", "k_dense_setup", "k_dense_encode", "k_dense_scan",
-                                   "k_dense_decode", "k_small", "k_small_sum"};
+                                   "k_dense_decode", "k_small", "k_small_sum", "k_emit_sum"};
 
 struct Pending {
     int k;

@@ -34,6 +34,7 @@ enum KernelId : int {
     kKDenseDecode,
     kKSmall,
     kKSmallSum,
+    kKEmitSum,
     kNumKernels
 };
 
