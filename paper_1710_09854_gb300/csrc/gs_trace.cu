@@ -14,7 +14,7 @@ namespace {
 
 const char* kNames[kNumKernels] = {"k_bound", "k_stream", "k_solve", "k_emit",
                                    "k_prob",  "k_words",  "k_bucket", "k_tiles",
-                                   "k_stream_tma", "k_decide", "k_scan", "k_sum",
+                                   "k_stream_tma", "k_decide",
                                    "k_eps_hist", "k_eps_bracket", "k_solve_eps",
                                    "k_lr_grad", "k_lr_margins", "k_row_sq", "k_sum_rows", "k_sgd_step",
                                    "k_dense_count", "k_dense_merge", "k_dense_setup", "k_dense_encode", "k_dense_scan",

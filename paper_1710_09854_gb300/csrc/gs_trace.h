@@ -16,8 +16,6 @@ enum KernelId : int {
     kKTiles,
     kKStreamTma,
     kKDecide,
-    kKScan,
-    kKSum,
     kKEpsHist,
     kKEpsBracket,
     kKSolveEps,
