@@ -1061,6 +1061,30 @@ __device__ __forceinline__ long long warp_scan_counts(int32_t* ko, int n, int la
     return carry;
 }
 
+// Word j (0..3) of group q alone: rounds 1-9 of PhiloxStream::words_after,
+// and of the last round only the product that word comes from (words 0 and 1
+// are the high and low halves of 0xCD9E8D57 c2, words 2 and 3 those of
+// 0xD2511F53 c0).
+__device__ __forceinline__ uint32_t philox_word(const PhiloxStream& ph, uint32_t q, int j) {
+    const uint64_t m0 = (uint64_t)0xD2511F53u * (uint64_t)q;
+    uint32_t c0 = ph.x0, c1 = ph.x1, c2 = (uint32_t)(m0 >> 32) ^ ph.c3k1, c3 = (uint32_t)m0;
+#pragma unroll
+    for (int r = 1; r < 9; ++r) {
+        const uint64_t p0 = (uint64_t)0xD2511F53u * (uint64_t)c0;
+        const uint64_t p1 = (uint64_t)0xCD9E8D57u * (uint64_t)c2;
+        const uint32_t n0 = (uint32_t)(p1 >> 32) ^ c1 ^ ph.rk0[r];
+        const uint32_t n2 = (uint32_t)(p0 >> 32) ^ c3 ^ ph.rk1[r];
+        c1 = (uint32_t)p1;
+        c3 = (uint32_t)p0;
+        c0 = n0;
+        c2 = n2;
+    }
+    const bool from_c0 = (j & 2) != 0;
+    const uint64_t p = (uint64_t)(from_c0 ? 0xD2511F53u : 0xCD9E8D57u) * (uint64_t)(from_c0 ? c0 : c2);
+    if (j & 1) return (uint32_t)p;
+    return (uint32_t)(p >> 32) ^ (from_c0 ? (c3 ^ ph.rk1[9]) : (c1 ^ ph.rk0[9]));
+}
+
 __device__ __forceinline__ Decider chunk_decider(const SegParam& P) {
     Decider dd;
     dd.lam = P.lam;
@@ -1111,7 +1135,7 @@ __global__ void __launch_bounds__(kEmitWarps * 32, kDecideBlocks) k_decide(const
             keep[r] = capped[r];
             kv[r] = gv;
             if (i < n && !capped[r]) {
-                const uint32_t x = word_of(ph.words((uint32_t)e[r].x >> 2), e[r].x & 3);
+                const uint32_t x = philox_word(ph, (uint32_t)e[r].x >> 2, e[r].x & 3);
                 float v;
                 keep[r] = dd(gv, x, v);
                 kv[r] = v;
