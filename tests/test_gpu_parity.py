@@ -199,10 +199,23 @@ def test_forced_exact_and_small_sample(gs):
             assert all(r["flags"] & 1 for r in gs.decode_info(inf))
 
 
-def test_segmented_parity(gs):
+@pytest.mark.parametrize("sample", [0, 1024, 256])
+def test_segmented_parity(gs, sample):
+    """Layer-wise calls against the oracle, layer by layer.  The bound's
+    sample size decides how its short segments (at most 1024 values) are
+    taken: the default packs them a warp each, several to a CTA; a sample of
+    1024 leaves one per CTA; 256 sends every segment through one CTA each."""
+    gs.gs_set_option(gs.GS_OPT_SAMPLE_SIZE, sample)
+    try:
+        _segmented_parity(gs)
+    finally:
+        gs.gs_set_option(gs.GS_OPT_SAMPLE_SIZE, 0)
+
+
+def _segmented_parity(gs):
     import torch
     rng = np.random.default_rng(4)
-    lens = [64, 3, 1, 17000, 5, 40000, 64, 16384, 2]
+    lens = [64, 3, 1, 17000, 5, 40000, 64, 16384, 2, 1024, 1025, 700, 9]
     off = np.concatenate([[0], np.cumsum(lens)]).astype(np.int64)
     M, d = 3, int(off[-1])
     g_host = np.stack([(rng.standard_normal(d) * rng.choice([1e-3, 1, 50], d)).astype(np.float32) for _ in range(M)])
