@@ -42,20 +42,18 @@ namespace {
 
 // Occupancy and ring depth.  The kernel is bound by instruction latency (its
 // integer work per coordinate is mostly Philox), so resident warps matter
-// more than deep rings: GS_TMA_CTAS CTAs of kCW warps per SM, each CTA's
-// rings in GS_TMA_RING_KIB KiB of shared memory.
-#ifndef GS_TMA_CTAS
-#define GS_TMA_CTAS 2
-#endif
-#ifndef GS_TMA_RING_KIB
-#define GS_TMA_RING_KIB 96
-#endif
+// more than deep rings: kCtas CTAs of kCW warps per SM, each CTA's rings in
+// 64 KiB (three CTAs, at most 85 registers a thread: two fp32 buffers a
+// warp) or 96 KiB (two CTAs) of shared memory.  Three are faster for whole
+// fp32 rows under Algorithm 3; bf16 rows, layer-wise rows (whose segment
+// edges take the per-lane path) and the instantiation that also sums
+// squares run faster with two.
+template <int kCtas>
+__host__ __device__ constexpr int ring_budget() { return (kCtas == 3 ? 64 : 96) * 1024; }
 constexpr int kCW = 8;                         // warps per CTA
 constexpr int kTmaThreads = 32 * kCW;
-constexpr int kTmaCtas = GS_TMA_CTAS;
 constexpr int kLaneCoords = 32;                // coordinates per lane per buffer
 constexpr int kBufCoords = 32 * kLaneCoords;   // 1024 coordinates per buffer
-constexpr int kRingBudget = GS_TMA_RING_KIB * 1024;   // shared memory for the rings of one CTA
 constexpr int kRowBytes = 128;
 constexpr long long kWaitLimit = 1ll << 22;    // try_wait polls before giving up
 constexpr int kQueue = 8;                      // per-warp queue of taken chunks (> kRing + 1)
@@ -233,13 +231,13 @@ struct ChunkWalk {
 
 // kDtype 0: fp32 rows of 32; 1: bf16 rows of 64.  kSq: also the sum of g^2
 // outside C (Algorithm 2's solve), the same way as s_low.
-template <int kDtype, bool kSq>
-__global__ void __launch_bounds__(kTmaThreads, kTmaCtas)
+template <int kDtype, bool kSq, int kCtas>
+__global__ void __launch_bounds__(kTmaThreads, kCtas)
     k_stream_tma(const __grid_constant__ CUtensorMap map, const __grid_constant__ StreamArgs A) {
     constexpr int kInner = kDtype == 0 ? 32 : 64;          // elements per 128-byte row
     constexpr int kBufRows = kBufCoords / kInner;          // 32 or 16
     constexpr int kBufBytes = kBufRows * kRowBytes;        // 4 KiB or 2 KiB
-    constexpr int kRing = kRingBudget / (kCW * kBufBytes); // buffers per warp: 3 or 6
+    constexpr int kRing = ring_budget<kCtas>() / (kCW * kBufBytes);   // buffers per warp
     extern __shared__ unsigned char dsm_raw[];
     unsigned char* base = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(dsm_raw) + 1023) & ~uintptr_t(1023));
     uint64_t* full = reinterpret_cast<uint64_t*>(base + kCW * kRing * kBufBytes);   // [kCW][kRing]
@@ -588,11 +586,11 @@ bool make_map(CUtensorMap* map, const void* g, int dtype, int64_t rows, int box_
     return r == CUDA_SUCCESS;
 }
 
-template <int kDtype>
+template <int kDtype, int kCtas>
 size_t tma_smem_bytes() {
     constexpr int kInner = kDtype == 0 ? 32 : 64;
     constexpr int kBufBytes = (kBufCoords / kInner) * kRowBytes;
-    constexpr int kRing = kRingBudget / (kCW * kBufBytes);
+    constexpr int kRing = ring_budget<kCtas>() / (kCW * kBufBytes);
     static_assert(kQueue > kRing + 1, "the chunk queue must hold every chunk the prefetcher can be ahead");
     // alignment slack + buffers + full barriers + abort flag + chunk queues
     return 1024 + (size_t)kCW * kRing * kBufBytes + (size_t)kCW * kRing * 8 + 16 + (size_t)kCW * kQueue * 4;
@@ -640,18 +638,20 @@ cudaError_t launch_stream_tma(const Layout& Lo, const SegParam* sp, const Lists&
     // that wrote the bounds, which this launch waits for).
     A.next_chunk = reinterpret_cast<int*>(reinterpret_cast<char*>(const_cast<SegParam*>(sp)) +
                                           offsetof(SegParam, next_chunk));
-    // One chunk per warp at a time; kTmaCtas CTAs per SM at most.
-    const int grid = std::min((n_chunks + kCW - 1) / kCW, kTmaCtas * sm_count_tma());
+    // One chunk per warp at a time; as many CTAs as fit on the SMs at once.
+    const bool sq = Ls.b_low != nullptr;
+    const int ctas = (Lo.dtype == 0 && !sq && Lo.L == 1) ? 3 : 2;
+    const int grid = std::min((n_chunks + kCW - 1) / kCW, ctas * sm_count_tma());
     cudaError_t e;
     TraceScope ts(kKStreamTma, st);
     void (*kern)(const CUtensorMap, const StreamArgs);
     size_t smem;
     if (Lo.dtype == 0) {
-        kern = Ls.b_low ? k_stream_tma<0, true> : k_stream_tma<0, false>;
-        smem = tma_smem_bytes<0>();
+        kern = sq ? k_stream_tma<0, true, 2> : (ctas == 3 ? k_stream_tma<0, false, 3> : k_stream_tma<0, false, 2>);
+        smem = ctas == 3 ? tma_smem_bytes<0, 3>() : tma_smem_bytes<0, 2>();
     } else {
-        kern = Ls.b_low ? k_stream_tma<1, true> : k_stream_tma<1, false>;
-        smem = tma_smem_bytes<1>();
+        kern = sq ? k_stream_tma<1, true, 2> : k_stream_tma<1, false, 2>;
+        smem = tma_smem_bytes<1, 2>();
     }
     set_launch_error_site("k_stream_tma shared-memory attribute");
     e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
